@@ -1,0 +1,159 @@
+"""Float64 CPU oracle for the FLARE++ routing chain -- TEST INFRASTRUCTURE ONLY.
+
+Only ``tests/``, ``__graft_entry__.smoke()`` and the CPU-baseline leg of ``bench.py`` may
+import this package. It shares no code with the CUDA library and never calls it; the
+CUDA library never calls it either.
+
+What it computes (FLARE++ paper):
+  * ``sdpa``           -- SDPA(Q, K, V) = softmax(s Q K^T) V over the keys (Sec. 2, eq. sdpa_definition)
+  * ``route``          -- Q = SDPA(Qseed, Kt, Vt); Z = SDPA(Q, K, V); Y = SDPA(K, Q, Z)
+                          (Sec. 3.2, eqs. flarepp_dynamic_query and flarepp_mixer)
+  * ``encode_sharded`` -- the encoder evaluated shard by shard, then merged by the stable
+                          log-sum-exp reduction (App. A.2, A.3)
+
+All arithmetic is float64 in ``flarepp_oracle.c``; this module only marshals numpy arrays.
+"""
+import ctypes
+
+import numpy as np
+
+from . import build as _build
+
+_c_i64 = ctypes.c_int64
+_c_dp = ctypes.POINTER(ctypes.c_double)
+
+
+class Oracle:
+    """One loaded build of the oracle library (``plant`` != 0 only in pin-strength tests)."""
+
+    def __init__(self, plant: int = 0, build_dir: str = _build.BUILD_DIR):
+        path = _build.build(plant, build_dir)
+        self.lib = ctypes.CDLL(path)
+        self.plant = plant
+        lib = self.lib
+        lib.oracle_sdpa_f64.restype = ctypes.c_int
+        lib.oracle_sdpa_f64.argtypes = [_c_i64, _c_i64, _c_i64, _c_i64, _c_dp, ctypes.c_int,
+                                        _c_dp, _c_dp, ctypes.c_double, _c_dp, _c_dp]
+        lib.oracle_route_f64.restype = ctypes.c_int
+        lib.oracle_route_f64.argtypes = [_c_i64] * 5 + [_c_dp] * 5 + [ctypes.c_double] + [_c_dp] * 3
+        lib.oracle_encode_sharded_f64.restype = ctypes.c_int
+        lib.oracle_encode_sharded_f64.argtypes = [_c_i64] * 4 + [_c_dp] * 3 + [
+            ctypes.c_double, _c_i64, _c_i64, _c_dp, _c_dp]
+        lib.oracle_max_threads.restype = ctypes.c_int
+        lib.oracle_set_threads.argtypes = [ctypes.c_int]
+        assert lib.oracle_plant() == plant
+
+    # ------------------------------------------------------------------ helpers
+    @staticmethod
+    def _f64(a):
+        return np.ascontiguousarray(np.asarray(a, dtype=np.float64))
+
+    @staticmethod
+    def _p(a):
+        return a.ctypes.data_as(_c_dp)
+
+    def max_threads(self) -> int:
+        return int(self.lib.oracle_max_threads())
+
+    def set_threads(self, n: int) -> None:
+        self.lib.oracle_set_threads(int(n))
+
+    # ------------------------------------------------------------------ API
+    def sdpa(self, q, k, v, scale):
+        """SDPA over the last two axes. q [..., nq, D]; k, v [..., nk, D] (same leading shape).
+
+        Returns (out [..., nq, D], lse [..., nq]); a row with no keys gives out 0, lse -inf.
+        """
+        q, k, v = self._f64(q), self._f64(k), self._f64(v)
+        lead = q.shape[:-2]
+        assert k.shape[:-2] == lead and v.shape == k.shape and q.shape[-1] == k.shape[-1]
+        G = int(np.prod(lead)) if lead else 1
+        nq, D = q.shape[-2], q.shape[-1]
+        nk = k.shape[-2]
+        out = np.zeros(lead + (nq, D))
+        lse = np.zeros(lead + (nq,))
+        rc = self.lib.oracle_sdpa_f64(G, nq, nk, D, self._p(q), 0, self._p(k), self._p(v),
+                                      float(scale), self._p(out), self._p(lse))
+        if rc:
+            raise MemoryError("oracle scratch allocation failed")
+        return out, lse
+
+    def route(self, seeds, Kt, Vt, K, V, scale):
+        """The routing chain. seeds [H, M, D]; Kt, Vt, K, V [B, H, N, D].
+
+        Returns (Q [B, H, M, D], Z [B, H, M, D], Y [B, H, N, D]).
+        """
+        seeds, Kt, Vt, K, V = (self._f64(a) for a in (seeds, Kt, Vt, K, V))
+        B, H, N, D = K.shape
+        M = seeds.shape[1]
+        assert seeds.shape == (H, M, D)
+        for a in (Kt, Vt, V):
+            assert a.shape == (B, H, N, D)
+        Q = np.zeros((B, H, M, D))
+        Z = np.zeros((B, H, M, D))
+        Y = np.zeros((B, H, N, D))
+        rc = self.lib.oracle_route_f64(B, H, N, M, D, self._p(seeds), self._p(Kt), self._p(Vt),
+                                       self._p(K), self._p(V), float(scale), self._p(Q),
+                                       self._p(Z), self._p(Y))
+        if rc:
+            raise MemoryError("oracle scratch allocation failed")
+        return Q, Z, Y
+
+    def encode_sharded(self, q, k, v, scale, chunk, n_empty=0):
+        """Encoder over shards of ``chunk`` keys merged by the stable LSE reduction (App. A.3).
+
+        q [..., nq, D]; k, v [..., nk, D]. ``n_empty`` extra empty shards are merged in.
+        Returns (out [..., nq, D], lse [..., nq]).
+        """
+        q, k, v = self._f64(q), self._f64(k), self._f64(v)
+        lead = q.shape[:-2]
+        G = int(np.prod(lead)) if lead else 1
+        nq, D = q.shape[-2], q.shape[-1]
+        nk = k.shape[-2]
+        out = np.zeros(lead + (nq, D))
+        lse = np.zeros(lead + (nq,))
+        rc = self.lib.oracle_encode_sharded_f64(G, nq, nk, D, self._p(q), self._p(k), self._p(v),
+                                                float(scale), int(chunk), int(n_empty),
+                                                self._p(out), self._p(lse))
+        if rc:
+            raise ValueError("oracle_encode_sharded_f64 failed (chunk <= 0 or allocation)")
+        return out, lse
+
+
+_default = None
+
+
+def default() -> Oracle:
+    global _default
+    if _default is None:
+        _default = Oracle(0)
+    return _default
+
+
+def sdpa(q, k, v, scale):
+    return default().sdpa(q, k, v, scale)
+
+
+def route(seeds, Kt, Vt, K, V, scale):
+    return default().route(seeds, Kt, Vt, K, V, scale)
+
+
+def encode_sharded(q, k, v, scale, chunk, n_empty=0):
+    return default().encode_sharded(q, k, v, scale, chunk, n_empty)
+
+
+def max_threads() -> int:
+    return default().max_threads()
+
+
+def set_threads(n: int) -> None:
+    default().set_threads(n)
+
+
+def build() -> str:
+    """Compile the oracle library (called by the package build step)."""
+    return _build.build()
+
+
+__all__ = ["Oracle", "default", "sdpa", "route", "encode_sharded", "max_threads",
+           "set_threads", "build"]
