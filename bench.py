@@ -1,0 +1,391 @@
+"""Benchmark of the FLARE++ routing chain on GB300: one JSON line on stdout.
+
+A step is one flarepp_route_fwd over the whole workload (encode call 1, combine, encode
+call 2, combine, decode call 3; Sec. 3.2). The default workload is the 3D-mesh shape
+B=1, H=8, N=1,048,576, M=512, D=32, bf16, with clustered keys; its five B*H*N*D tensors
+(2.7 GB) are far larger than the 129 MB L2, so no flush is needed between steps.
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--workload NAME] [--impl ours|reference]
+
+Under torchrun every rank runs an independent replica on its own GPU (the chain has no
+cross-GPU exchange on one box); rank 0 prints the aggregate.
+"""
+import argparse
+import hashlib
+import json
+import math
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+import torch
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+from paper_2608_11519_gb300 import inputs  # noqa: E402
+
+METRIC = "routed tokens·heads/sec for the 3-call FLARE++ chain; % of roofline"
+UNIT = "token·heads/s"
+KERNEL_SOURCES = ("paper_2608_11519_gb300/csrc",)
+FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0,
+                  "source": "fallback"}
+
+
+# ------------------------------------------------------------------ helpers
+
+def load_peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        with open(p) as f:
+            d = json.load(f)
+        d["source"] = "measured"
+        return d
+    return dict(FALLBACK_PEAKS)
+
+
+def kernel_source_hash():
+    h = hashlib.sha256()
+    for d in KERNEL_SOURCES:
+        full = os.path.join(ROOT, d)
+        for name in sorted(os.listdir(full)):
+            with open(os.path.join(full, name), "rb") as f:
+                h.update(name.encode() + f.read())
+    return h.hexdigest()[:16]
+
+
+def recorded_traffic(workload, stage):
+    """DRAM bytes per launch from the committed ncu summary, if it was taken on the current
+    kernel sources (else None)."""
+    p = os.path.join(ROOT, "profiles", "traffic.json")
+    if not os.path.exists(p):
+        return None
+    with open(p) as f:
+        d = json.load(f)
+    e = d.get(workload, {}).get(stage)
+    if not e or e.get("source_hash") != kernel_source_hash():
+        return None
+    return e.get("dram_bytes_per_launch")
+
+
+def stage_work(w, stage):
+    """Algorithmic flops and bytes of one launch of a stage.
+
+    encode (calls 1, 2): S = s Q K^T and O = P V over all tokens: 4*B*H*N*M*D flops; reads
+      the call's K and V: 2*B*H*N*D elements.
+    decode (call 3): S^T = s K Q^T and Y = P Z: 4*B*H*N*M*D flops; reads K, writes Y:
+      2*B*H*N*D elements.
+    combine: reads the chunk partials, writes Q or Z (latent-sized; no algorithmic tokens).
+    """
+    tok = w.B * w.H * w.N
+    flops = 4.0 * tok * w.M * w.D
+    byts = 2.0 * tok * w.D * w.elt_bytes
+    if stage.startswith("combine"):
+        return 0.0, 2.0 * w.B * w.H * w.M * w.D * 4
+    return flops, byts
+
+
+class ClockSampler:
+    """nvidia-smi sampling of SM clocks and throttle reasons during the timed region."""
+
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self):
+        self.proc = None
+        self.path = None
+
+    def start(self):
+        try:
+            fd, self.path = tempfile.mkstemp(suffix=".csv")
+            os.close(fd)
+            self.out = open(self.path, "w")
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits",
+                 "-lms", "200"], stdout=self.out, stderr=subprocess.DEVNULL)
+        except (OSError, FileNotFoundError):
+            self.proc = None
+
+    def stop(self, gpu_index):
+        if self.proc is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+        self.out.close()
+        sm, smax, reasons, power = [], [], set(), []
+        names = ("hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap")
+        with open(self.path) as f:
+            for line in f:
+                parts = [p.strip() for p in line.split(",")]
+                if len(parts) < 9:
+                    continue
+                try:
+                    if int(parts[0]) != gpu_index:
+                        continue
+                    sm.append(float(parts[1]))
+                    smax.append(float(parts[2]))
+                    power.append(float(parts[3]))
+                except ValueError:
+                    continue
+                for n, v in zip(names, parts[5:9]):
+                    if v.lower() == "active":
+                        reasons.add(n)
+        os.unlink(self.path)
+        if not sm:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["no samples"]}
+        loaded = [s for s in sm if s > 0.5 * max(sm)] or sm
+        return {"sm_mhz": statistics.median(loaded), "sm_max_mhz": max(smax),
+                "power_w_max": max(power) if power else None, "samples": len(sm),
+                "reasons": sorted(reasons)}
+
+
+def dist_setup(n_gpus):
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    if world > 1:
+        import torch.distributed as dist
+        os.environ.setdefault("MASTER_ADDR", "127.0.0.1")
+        torch.cuda.set_device(local)
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+    elif torch.cuda.is_available():
+        torch.cuda.set_device(0)
+    return world, rank, local
+
+
+def barrier(world):
+    if world > 1:
+        import torch.distributed as dist
+        dist.barrier()
+
+
+def max_over_ranks(x, world):
+    if world == 1:
+        return x
+    import torch.distributed as dist
+    t = torch.tensor([x], dtype=torch.float64, device="cuda")
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+# ------------------------------------------------------------------ CPU baseline (oracle)
+
+def cpu_oracle_sample(w, target_s, seed=0):
+    """Time the float64 oracle on one (b, h) slice with a token prefix of the workload,
+    sized from a short probe to take about ``target_s`` seconds. Returns a cpu_baseline dict."""
+    import oracle
+    x = inputs.make_inputs(w.with_(B=1, H=1, N=min(w.N, 4096)), seed)
+    f = inputs.to_f64_numpy(x)
+    t0 = time.perf_counter()
+    oracle.route(f["seeds"], f["Kt"], f["Vt"], f["K"], f["V"], w.scale)
+    probe = time.perf_counter() - t0
+    n = int(min(w.N, max(1024, f["K"].shape[2] * target_s / max(probe, 1e-3))))
+    x = inputs.make_inputs(w.with_(B=1, H=1, N=n), seed)
+    f = inputs.to_f64_numpy(x)
+    t0 = time.perf_counter()
+    oracle.route(f["seeds"], f["Kt"], f["Vt"], f["K"], f["V"], w.scale)
+    dt = time.perf_counter() - t0
+    return {"value": n / dt, "unit": UNIT, "cores": oracle.max_threads(), "kind": "oracle",
+            "sample": f"one head, N={n} tokens of the {w.name} shape (M={w.M}, D={w.D}), "
+                      f"float64, {dt:.2f} s"}
+
+
+# ------------------------------------------------------------------ reference arm
+
+def run_reference(args, w):
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    if rank != 0:
+        return 0
+    import oracle
+    n = int(min(w.N, args.ref_tokens))
+    x = inputs.make_inputs(w.with_(B=1, H=1, N=n), args.seed)
+    f = inputs.to_f64_numpy(x)
+    for _ in range(args.warmup):
+        oracle.route(f["seeds"], f["Kt"], f["Vt"], f["K"], f["V"], w.scale)
+    t0 = time.perf_counter()
+    for _ in range(args.steps):
+        oracle.route(f["seeds"], f["Kt"], f["Vt"], f["K"], f["V"], w.scale)
+    dt = (time.perf_counter() - t0) / args.steps
+    value = n / dt
+    sample = (f"one head, N={n} tokens of the {w.name} shape (M={w.M}, D={w.D}), float64 oracle "
+              f"on the host cores, per step")
+    line = {"impl": "reference", "metric": METRIC, "value": value, "unit": UNIT,
+            "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
+            "ms_per_step": dt * 1e3, "higher_is_better": True, "scaling": "weak",
+            "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+            "config": {"workload": w.name, "B": w.B, "H": w.H, "N": w.N, "M": w.M, "D": w.D,
+                       "input_dtype": w.dtype, "sample_tokens": n},
+            "cpu_baseline": {"value": value, "unit": UNIT, "cores": oracle.max_threads(),
+                             "kind": "oracle", "sample": sample},
+            "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0,
+                    "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+    return 0
+
+
+# ------------------------------------------------------------------ our arm
+
+def run_ours(args, w):
+    from paper_2608_11519_gb300 import flarepp
+
+    world, rank, local = dist_setup(args.gpus)
+    dev = torch.device("cuda", local if world > 1 else 0)
+    flarepp.load()
+    peaks = load_peaks()
+
+    x = inputs.make_inputs(w, args.seed + rank, device=dev)
+    Y = torch.empty_like(x["K"])
+    ws = flarepp.Workspace()
+    stream = torch.cuda.current_stream(dev)
+    args_ = (x["seeds"], x["Kt"], x["Vt"], x["K"], x["V"])
+
+    ev_sets = [flarepp.StageEvents(stream) for _ in range(args.steps)]
+    warm_ev = flarepp.StageEvents(stream)
+    for _ in range(args.warmup):
+        flarepp.route_fwd_profiled(*args_, warm_ev, scale=w.scale, Y=Y, workspace=ws)
+    torch.cuda.synchronize(dev)
+
+    clocks = ClockSampler()
+    if rank == 0:
+        clocks.start()
+        time.sleep(0.3)
+    t_start = torch.cuda.Event(enable_timing=True)
+    t_end = torch.cuda.Event(enable_timing=True)
+    barrier(world)
+    torch.cuda.synchronize(dev)
+    t_start.record(stream)
+    for i in range(args.steps):
+        flarepp.route_fwd_profiled(*args_, ev_sets[i], scale=w.scale, Y=Y, workspace=ws)
+    t_end.record(stream)
+    torch.cuda.synchronize(dev)
+    barrier(world)
+    clk = clocks.stop(dev.index) if rank == 0 else None
+    total_ms = t_start.elapsed_time(t_end)
+    total_ms = max_over_ranks(total_ms, world)
+    ms_per_step = total_ms / args.steps
+
+    # per-stage durations over the timed region
+    stage_ms = {s: 0.0 for s in flarepp.STAGES}
+    for e in ev_sets:
+        for s, v in e.stage_ms().items():
+            stage_ms[s] += v / args.steps
+    dominant = max(stage_ms, key=stage_ms.get)
+    flops, byts = stage_work(w, dominant)
+    t_dom = stage_ms[dominant] * 1e-3
+    tc_peak = peaks["bf16_tflops_sustained"] if w.dtype == "bf16" else None
+    bw_peak = peaks["hbm_gbs"]
+    t_tc = flops / (tc_peak * 1e12) if tc_peak else 0.0
+    t_mem = byts / (bw_peak * 1e9)
+    if t_tc >= t_mem and tc_peak:
+        roof = {"bound": "tensor", "achieved": flops / t_dom / 1e12, "peak": tc_peak,
+                "unit": "TFLOP/s", "peak_kind": "bf16_tflops_sustained (" + peaks["source"] + ")"}
+    else:
+        roof = {"bound": "hbm", "achieved": byts / t_dom / 1e9, "peak": bw_peak, "unit": "GB/s",
+                "peak_kind": "hbm_gbs (" + peaks["source"] + ")"}
+    roof["frac"] = roof["achieved"] / roof["peak"]
+    roof["kernel"] = dominant
+    roof["ms_per_launch"] = stage_ms[dominant]
+    roof["algorithmic_flops_per_launch"] = flops
+    roof["algorithmic_bytes_per_launch"] = byts
+    roof["traffic"] = recorded_traffic(w.name, dominant)
+
+    # whole-chain roofline: max(12 BNMHD / tensor peak, 5 BHND elt / HBM)
+    tok = w.B * w.H * w.N
+    t_chain_tc = 12.0 * tok * w.M * w.D / ((tc_peak or peaks["bf16_tflops"]) * 1e12)
+    t_chain_mem = 5.0 * tok * w.D * w.elt_bytes / (bw_peak * 1e9)
+    t_chain = max(t_chain_tc, t_chain_mem)
+    t_chain_burst = max(12.0 * tok * w.M * w.D / (peaks["bf16_tflops"] * 1e12), t_chain_mem)
+    chain = {"roofline_us": t_chain * 1e6, "bound": "tensor" if t_chain_tc >= t_chain_mem else "hbm",
+             "frac": t_chain / (ms_per_step * 1e-3),
+             "frac_vs_burst_peak": t_chain_burst / (ms_per_step * 1e-3),
+             "peaks": {"bf16_tflops_sustained": peaks.get("bf16_tflops_sustained"),
+                       "bf16_tflops": peaks.get("bf16_tflops"), "hbm_gbs": bw_peak,
+                       "source": peaks["source"]}}
+
+    value = tok * world / (ms_per_step * 1e-3)
+
+    # end to end through the public API with host buffers
+    e2e = None
+    if not args.no_e2e:
+        xh = {k: v.to("cpu").pin_memory() for k, v in x.items()}
+        Yh = torch.empty(Y.shape, dtype=Y.dtype, pin_memory=True)
+        bufs = {}
+        ha = (xh["seeds"], xh["Kt"], xh["Vt"], xh["K"], xh["V"])
+        for _ in range(2):
+            flarepp.route_fwd_host(*ha, w.scale, Y_host=Yh, device=dev, workspace=ws, dev_bufs=bufs)
+        n_e2e = max(1, min(args.steps, args.e2e_steps))
+        barrier(world)
+        torch.cuda.synchronize(dev)
+        e0 = torch.cuda.Event(enable_timing=True)
+        e1 = torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        for _ in range(n_e2e):
+            flarepp.route_fwd_host(*ha, w.scale, Y_host=Yh, device=dev, workspace=ws, dev_bufs=bufs)
+        e1.record(stream)
+        torch.cuda.synchronize(dev)
+        e2e_ms = max_over_ranks(e0.elapsed_time(e1) / n_e2e, world)
+        h2d = sum(t.numel() * t.element_size() for t in ha)
+        d2h = Yh.numel() * Yh.element_size()
+        e2e = {"value": tok * world / (e2e_ms * 1e-3), "unit": UNIT, "ms_per_step": e2e_ms,
+               "steps": n_e2e, "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h}
+        del xh, Yh, bufs
+
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        cpu = cpu_oracle_sample(w, args.cpu_seconds, args.seed)
+
+    if rank == 0:
+        line = {
+            "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms_per_step,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+            "dtype": "bf16" if w.dtype == "bf16" else "f32", "data": "synthetic",
+            "config": {"workload": w.name, "B": w.B, "H": w.H, "N": w.N, "M": w.M, "D": w.D,
+                       "keys": f"clustered, {w.n_centres} centres" if w.n_centres else "iid",
+                       "l2": "inputs larger than L2 (no flush)"
+                       if 5 * tok * w.D * w.elt_bytes > 2 * 129e6 else "inputs near L2 size",
+                       "parallelism": f"replicas x{world}"},
+            "roofline": roof, "chain_roofline": chain, "stage_ms": stage_ms,
+            "cpu_baseline": cpu, "e2e": e2e, "clocks": clk,
+            "gpu_launches": 5 * args.steps,
+        }
+        print(json.dumps(line), flush=True)
+    if world > 1:
+        import torch.distributed as dist
+        dist.destroy_process_group()
+    return 0
+
+
+def main():
+    ap = argparse.ArgumentParser(description=__doc__)
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=20)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", choices=("ours", "reference"), default="ours")
+    ap.add_argument("--workload", default="mesh3d", choices=sorted(inputs.WORKLOADS))
+    ap.add_argument("--seed", type=int, default=0)
+    ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--e2e-steps", type=int, default=5)
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--cpu-seconds", type=float, default=12.0)
+    ap.add_argument("--ref-tokens", type=int, default=16384,
+                    help="token sample per reference step (one head)")
+    args = ap.parse_args()
+    w = inputs.get(args.workload)
+    if args.warmup < 3 and args.impl == "ours":
+        print("warning: fewer than 3 warm-up steps", file=sys.stderr)
+    if args.impl == "reference":
+        return run_reference(args, w)
+    return run_ours(args, w)
+
+
+if __name__ == "__main__":
+    sys.exit(main())

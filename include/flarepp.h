@@ -1,0 +1,134 @@
+/*
+ * libflarepp -- the FLARE++ routing chain on one GB300 (sm_103a).
+ *
+ * For every batch element b and head h the library computes three scaled-dot-product
+ * attention calls (FLARE++ paper, Sec. 3.2, eqs. flarepp_dynamic_query and flarepp_mixer;
+ * SDPA as in Sec. 2, eq. sdpa_definition):
+ *
+ *   call 1  Q = SDPA(seeds_h, Kt, Vt)   softmax over the N tokens   -> Q [M, D]
+ *   call 2  Z = SDPA(Q, K, V)           softmax over the N tokens   -> Z [M, D]
+ *   call 3  Y = SDPA(K, Q, Z)           softmax over the M routes   -> Y [N, D]
+ *
+ * with SDPA(A, B, C) = softmax(scale * A B^T) C. Calls 1 and 2 run as a split-N encode
+ * (each CTA reduces a chunk of tokens to online-softmax partials) followed by the stable
+ * log-sum-exp merge of App. A.3, the single-GPU form of the token-sharded encoder of
+ * Sec. 3.3 / eq. distributed_flare_encoder. Call 3 runs as an N-tiled decode.
+ *
+ * Conventions shared by every entry point
+ *   - Layout: dense row-major, D innermost. seeds [H, M, D]; Kt, Vt, K, V, Y [B, H, N, D].
+ *     Inputs and Y share one element type, chosen by flarepp_shape.dtype.
+ *   - Pointers: device pointers (or managed memory), each 16-byte aligned. The caller owns
+ *     every buffer; the library keeps no pointer after a call returns and allocates no
+ *     device memory. Y must not overlap any input or the workspace.
+ *   - Stream: all work is enqueued on `stream` (a cudaStream_t; NULL = legacy default
+ *     stream) and the call returns without synchronising. The workspace must stay untouched
+ *     until that work has finished.
+ *   - Errors: arguments are checked before anything is launched; on a non-OK status nothing
+ *     has been enqueued, except FLAREPP_ERR_CUDA, which reports a failed launch. No C++
+ *     exception crosses this interface and nothing is printed.
+ *   - Supported: D in {16, 32, 64}; 0 <= M <= 2048; B, H, N >= 0; finite scale.
+ *     N = 0 or B*H = 0 is a no-op. M = 0 writes Y = 0: every decode row then has no keys,
+ *     and an attention row with no keys outputs 0 (App. A.3).
+ *   - Threads: entry points may be called from several host threads at once (on distinct
+ *     workspaces and outputs).
+ */
+#ifndef FLAREPP_H
+#define FLAREPP_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+#if defined(__GNUC__)
+#define FLAREPP_API __attribute__((visibility("default")))
+#else
+#define FLAREPP_API
+#endif
+
+typedef enum {
+    FLAREPP_F32 = 0,  /* inputs and Y are float32; the path computes in float32 */
+    FLAREPP_BF16 = 1  /* inputs and Y are bfloat16; tensor-core products, float32 accumulate */
+} flarepp_dtype;
+
+typedef enum {
+    FLAREPP_OK = 0,
+    FLAREPP_ERR_INVALID_ARGUMENT = 1, /* null/misaligned pointer, negative size, NaN/inf scale,
+                                         overlapping Y, bad dtype */
+    FLAREPP_ERR_UNSUPPORTED = 2,      /* a valid shape outside the supported set (D, M limits) */
+    FLAREPP_ERR_WORKSPACE = 3,        /* workspace missing, misaligned or too small */
+    FLAREPP_ERR_CUDA = 4,             /* a CUDA call or kernel launch failed */
+    FLAREPP_ERR_TIMEOUT = 5           /* reserved: a bounded device wait gave up */
+} flarepp_status;
+
+typedef struct {
+    int64_t B; /* batch elements */
+    int64_t H; /* heads */
+    int64_t N; /* tokens */
+    int64_t M; /* routes (latent slots) */
+    int64_t D; /* head width */
+    int32_t dtype; /* flarepp_dtype */
+} flarepp_shape;
+
+/*
+ * Bytes of device workspace that flarepp_route_fwd needs for `shape` (a function of the
+ * shape alone). Returns 0 when the shape is invalid or needs none. The workspace holds the
+ * split-N partials (running max, sum and weighted value sum per chunk and route) and the
+ * routing queries Q and latents Z of calls 1 and 2.
+ */
+FLAREPP_API size_t flarepp_route_workspace_bytes(const flarepp_shape* shape);
+
+/*
+ * The routing chain (Sec. 3.2, eqs. flarepp_dynamic_query and flarepp_mixer).
+ *   seeds      [H, M, D]     learned route seeds, shared by all b (App. A.1)
+ *   Kt, Vt     [B, H, N, D]  keys and values of the query-synthesis call
+ *   K, V       [B, H, N, D]  keys and values of the gather/scatter pair
+ *   scale      softmax temperature of all three calls; 1/sqrt(D) in the paper
+ *   Y          [B, H, N, D]  output, written in full
+ *   workspace  >= flarepp_route_workspace_bytes(shape) bytes, 256-byte aligned
+ *   stream     cudaStream_t to enqueue on
+ */
+FLAREPP_API flarepp_status flarepp_route_fwd(const flarepp_shape* shape, const void* seeds, const void* Kt,
+                                 const void* Vt, const void* K, const void* V, float scale,
+                                 void* Y, void* workspace, size_t workspace_bytes, void* stream);
+
+/*
+ * flarepp_route_fwd that also copies the intermediates out, so each call of the chain can be
+ * checked on its own: Q_out and Z_out are float32 [B, H, M, D] device buffers (each may be
+ * NULL). Same rules and errors as flarepp_route_fwd.
+ */
+FLAREPP_API flarepp_status flarepp_route_fwd_debug(const flarepp_shape* shape, const void* seeds,
+                                       const void* Kt, const void* Vt, const void* K,
+                                       const void* V, float scale, void* Y, void* workspace,
+                                       size_t workspace_bytes, void* stream, float* Q_out,
+                                       float* Z_out);
+
+/*
+ * flarepp_route_fwd that also records six caller-created CUDA events (cudaEvent_t) on
+ * `stream` around its stages, so a caller can time each kernel of the chain on the stream
+ * it runs on: events[0] before the call-1 encode, [1] after it, [2] after the call-1
+ * combine, [3] after the call-2 encode, [4] after the call-2 combine, [5] after the
+ * call-3 decode. n_events must be >= 6 and no event may be NULL (else
+ * FLAREPP_ERR_INVALID_ARGUMENT). On degenerate shapes (N, M or B*H zero) no event is
+ * recorded. Otherwise identical to flarepp_route_fwd.
+ */
+FLAREPP_API flarepp_status flarepp_route_fwd_profiled(const flarepp_shape* shape,
+                                                      const void* seeds, const void* Kt,
+                                                      const void* Vt, const void* K,
+                                                      const void* V, float scale, void* Y,
+                                                      void* workspace, size_t workspace_bytes,
+                                                      void* stream, void* const* events,
+                                                      int n_events);
+
+/* Static description of a status code (never NULL). */
+FLAREPP_API const char* flarepp_status_string(flarepp_status status);
+
+/* Library version string, e.g. "0.1.0". */
+FLAREPP_API const char* flarepp_version(void);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* FLAREPP_H */

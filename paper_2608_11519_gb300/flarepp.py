@@ -1,0 +1,247 @@
+"""Python binding of libflarepp (ctypes): argument marshalling only.
+
+Every step of the routing chain runs in the library's CUDA kernels. PyTorch provides the
+device memory and the stream. There is no fallback: if the library is not built, every
+call raises.
+
+    from paper_2608_11519_gb300 import flarepp
+    Y = flarepp.route_fwd(seeds, Kt, Vt, K, V)              # device tensors
+    Y, Q, Z = flarepp.route_fwd_debug(seeds, Kt, Vt, K, V)  # plus the intermediates
+    Y = flarepp.route_fwd_host(seeds, Kt, Vt, K, V)         # host tensors in, host Y out
+"""
+import ctypes
+import math
+import os
+
+import torch
+
+from . import build as _build
+
+F32, BF16 = 0, 1
+OK, ERR_INVALID_ARGUMENT, ERR_UNSUPPORTED, ERR_WORKSPACE, ERR_CUDA, ERR_TIMEOUT = range(6)
+_DTYPES = {torch.float32: F32, torch.bfloat16: BF16}
+
+EXPORTED = ("flarepp_route_workspace_bytes", "flarepp_route_fwd", "flarepp_route_fwd_debug",
+            "flarepp_route_fwd_profiled", "flarepp_status_string", "flarepp_version")
+N_STAGE_EVENTS = 6
+STAGES = ("encode1", "combine1", "encode2", "combine2", "decode")
+
+
+class Shape(ctypes.Structure):
+    """Mirror of ``flarepp_shape`` in include/flarepp.h."""
+    _fields_ = [("B", ctypes.c_int64), ("H", ctypes.c_int64), ("N", ctypes.c_int64),
+                ("M", ctypes.c_int64), ("D", ctypes.c_int64), ("dtype", ctypes.c_int32)]
+
+
+class FlareppError(RuntimeError):
+    def __init__(self, status: int, what: str):
+        super().__init__(f"{what}: status {status} ({status_string(status)})")
+        self.status = status
+
+
+_LIB = None
+
+
+def lib_path() -> str:
+    return _build.lib_path()
+
+
+def load(path: str = None):
+    """Load libflarepp.so (built by ``build.build()``); raises if it is missing."""
+    global _LIB
+    if _LIB is not None and path is None:
+        return _LIB
+    path = path or lib_path()
+    if not os.path.exists(path):
+        raise RuntimeError(f"libflarepp is not built ({path} missing); run "
+                           "`python -c 'import __graft_entry__ as g; g.build()'` first")
+    lib = ctypes.CDLL(path)
+    vp, sz = ctypes.c_void_p, ctypes.c_size_t
+    sp = ctypes.POINTER(Shape)
+    lib.flarepp_route_workspace_bytes.restype = sz
+    lib.flarepp_route_workspace_bytes.argtypes = [sp]
+    lib.flarepp_route_fwd.restype = ctypes.c_int
+    lib.flarepp_route_fwd.argtypes = [sp, vp, vp, vp, vp, vp, ctypes.c_float, vp, vp, sz, vp]
+    lib.flarepp_route_fwd_debug.restype = ctypes.c_int
+    lib.flarepp_route_fwd_debug.argtypes = [sp, vp, vp, vp, vp, vp, ctypes.c_float, vp, vp, sz,
+                                            vp, vp, vp]
+    lib.flarepp_route_fwd_profiled.restype = ctypes.c_int
+    lib.flarepp_route_fwd_profiled.argtypes = [sp, vp, vp, vp, vp, vp, ctypes.c_float, vp, vp, sz,
+                                               vp, ctypes.POINTER(ctypes.c_void_p), ctypes.c_int]
+    lib.flarepp_status_string.restype = ctypes.c_char_p
+    lib.flarepp_status_string.argtypes = [ctypes.c_int]
+    lib.flarepp_version.restype = ctypes.c_char_p
+    if path == lib_path():
+        _LIB = lib
+    return lib
+
+
+def status_string(status: int) -> str:
+    return load().flarepp_status_string(int(status)).decode()
+
+
+def version() -> str:
+    return load().flarepp_version().decode()
+
+
+def make_shape(B, H, N, M, D, dtype) -> Shape:
+    if isinstance(dtype, torch.dtype):
+        dtype = _DTYPES[dtype]
+    return Shape(int(B), int(H), int(N), int(M), int(D), int(dtype))
+
+
+def workspace_bytes(B, H, N, M, D, dtype) -> int:
+    return int(load().flarepp_route_workspace_bytes(ctypes.byref(make_shape(B, H, N, M, D, dtype))))
+
+
+def _ptr(t):
+    return None if t is None else ctypes.c_void_p(t.data_ptr())
+
+
+def _shape_of(seeds, Kt, Vt, K, V) -> Shape:
+    for t in (seeds, Kt, Vt, K, V):
+        if not isinstance(t, torch.Tensor):
+            raise TypeError("inputs must be torch tensors")
+        if not t.is_contiguous():
+            raise ValueError("inputs must be contiguous (D innermost)")
+        if t.dtype != K.dtype:
+            raise TypeError("all inputs must share one dtype")
+    if K.dtype not in _DTYPES:
+        raise TypeError(f"unsupported dtype {K.dtype}; use float32 or bfloat16")
+    if K.dim() != 4 or seeds.dim() != 3:
+        raise ValueError("expected seeds [H,M,D] and Kt, Vt, K, V [B,H,N,D]")
+    B, H, N, D = K.shape
+    M = seeds.shape[1]
+    if tuple(seeds.shape) != (H, M, D):
+        raise ValueError(f"seeds shape {tuple(seeds.shape)} != {(H, M, D)}")
+    for t in (Kt, Vt, V):
+        if tuple(t.shape) != (B, H, N, D):
+            raise ValueError(f"input shape {tuple(t.shape)} != {(B, H, N, D)}")
+    return make_shape(B, H, N, M, D, K.dtype)
+
+
+class Workspace:
+    """A reusable device workspace, grown on demand (one per stream at a time)."""
+
+    def __init__(self, device=None):
+        self.device = device
+        self.buf = None
+
+    def get(self, nbytes: int, device):
+        if nbytes == 0:
+            return None
+        if self.buf is None or self.buf.numel() < nbytes or self.buf.device != device:
+            self.buf = torch.empty(nbytes + 256, dtype=torch.uint8, device=device)
+        # the library wants 256-byte alignment; torch allocations are at least that aligned
+        assert self.buf.data_ptr() % 256 == 0
+        return self.buf
+
+
+def _call(debug, seeds, Kt, Vt, K, V, scale, Y, workspace, stream, Q_out, Z_out, events=None):
+    lib = load()
+    shape = _shape_of(seeds, Kt, Vt, K, V)
+    if K.device.type != "cuda":
+        raise ValueError("route_fwd takes device tensors; use route_fwd_host for host tensors")
+    if scale is None:
+        scale = 1.0 / math.sqrt(shape.D)
+    if Y is None:
+        Y = torch.empty_like(K)
+    nbytes = int(lib.flarepp_route_workspace_bytes(ctypes.byref(shape)))
+    if isinstance(workspace, Workspace):
+        ws = workspace.get(nbytes, K.device)
+    elif workspace is None:
+        ws = torch.empty(nbytes, dtype=torch.uint8, device=K.device) if nbytes else None
+    else:
+        ws = workspace
+    ws_bytes = 0 if ws is None else ws.numel() * ws.element_size()
+    if stream is None:
+        stream = torch.cuda.current_stream(K.device)
+    st = ctypes.c_void_p(stream.cuda_stream if hasattr(stream, "cuda_stream") else int(stream))
+    if events is not None:
+        arr = (ctypes.c_void_p * len(events))(*[ctypes.c_void_p(e) for e in events])
+        rc = lib.flarepp_route_fwd_profiled(ctypes.byref(shape), _ptr(seeds), _ptr(Kt), _ptr(Vt),
+                                            _ptr(K), _ptr(V), float(scale), _ptr(Y), _ptr(ws),
+                                            ws_bytes, st, arr, len(events))
+        if rc != OK:
+            raise FlareppError(rc, "flarepp_route_fwd_profiled")
+        return Y
+    if debug:
+        rc = lib.flarepp_route_fwd_debug(ctypes.byref(shape), _ptr(seeds), _ptr(Kt), _ptr(Vt),
+                                         _ptr(K), _ptr(V), float(scale), _ptr(Y), _ptr(ws),
+                                         ws_bytes, st, _ptr(Q_out), _ptr(Z_out))
+    else:
+        rc = lib.flarepp_route_fwd(ctypes.byref(shape), _ptr(seeds), _ptr(Kt), _ptr(Vt), _ptr(K),
+                                   _ptr(V), float(scale), _ptr(Y), _ptr(ws), ws_bytes, st)
+    if rc != OK:
+        raise FlareppError(rc, "flarepp_route_fwd" + ("_debug" if debug else ""))
+    return Y
+
+
+def route_fwd(seeds, Kt, Vt, K, V, scale=None, Y=None, workspace=None, stream=None):
+    """Y = routing chain (Sec. 3.2) on device tensors; returns Y [B,H,N,D] (enqueued on
+    ``stream``, default torch's current stream)."""
+    return _call(False, seeds, Kt, Vt, K, V, scale, Y, workspace, stream, None, None)
+
+
+class StageEvents:
+    """Six timing events the library records around its stages (flarepp_route_fwd_profiled)."""
+
+    def __init__(self, stream=None):
+        stream = stream or torch.cuda.current_stream()
+        self.events = [torch.cuda.Event(enable_timing=True) for _ in range(N_STAGE_EVENTS)]
+        for e in self.events:  # create the underlying cudaEvent_t
+            e.record(stream)
+        self.handles = [int(e.cuda_event) for e in self.events]
+
+    def stage_ms(self):
+        """Milliseconds of each stage of the last recorded call (synchronises on the events)."""
+        self.events[-1].synchronize()
+        return {name: self.events[i].elapsed_time(self.events[i + 1])
+                for i, name in enumerate(STAGES)}
+
+
+def route_fwd_profiled(seeds, Kt, Vt, K, V, events: StageEvents, scale=None, Y=None,
+                       workspace=None, stream=None):
+    """``route_fwd`` that records ``events`` around each stage on the launching stream."""
+    return _call(False, seeds, Kt, Vt, K, V, scale, Y, workspace, stream, None, None,
+                 events.handles)
+
+
+def route_fwd_debug(seeds, Kt, Vt, K, V, scale=None, Y=None, workspace=None, stream=None):
+    """Like ``route_fwd``, also returning the float32 intermediates Q and Z [B,H,M,D]."""
+    B, H, N, D = K.shape
+    M = seeds.shape[1]
+    Q = torch.empty(B, H, M, D, dtype=torch.float32, device=K.device)
+    Z = torch.empty_like(Q)
+    Y = _call(True, seeds, Kt, Vt, K, V, scale, Y, workspace, stream, Q, Z)
+    return Y, Q, Z
+
+
+def route_fwd_host(seeds, Kt, Vt, K, V, scale=None, Y_host=None, device="cuda", workspace=None,
+                   stream=None, dev_bufs=None):
+    """End-to-end call on host tensors: copies the inputs to the device, runs the chain and
+    copies Y back into ``Y_host`` (pinned if allocated here). Returns Y_host after the copy
+    has completed. ``dev_bufs`` (a dict) keeps device buffers between calls."""
+    dev = torch.device(device)
+    bufs = dev_bufs if dev_bufs is not None else {}
+    names = ("seeds", "Kt", "Vt", "K", "V")
+    hs = dict(zip(names, (seeds, Kt, Vt, K, V)))
+    ds = {}
+    for n in names:
+        h = hs[n]
+        d = bufs.get(n)
+        if d is None or d.shape != h.shape or d.dtype != h.dtype:
+            d = torch.empty(h.shape, dtype=h.dtype, device=dev)
+            bufs[n] = d
+        d.copy_(h, non_blocking=True)
+        ds[n] = d
+    Yd = bufs.get("Y")
+    if Yd is None or Yd.shape != K.shape or Yd.dtype != K.dtype:
+        Yd = torch.empty(K.shape, dtype=K.dtype, device=dev)
+        bufs["Y"] = Yd
+    route_fwd(ds["seeds"], ds["Kt"], ds["Vt"], ds["K"], ds["V"], scale, Yd, workspace, stream)
+    if Y_host is None:
+        Y_host = torch.empty(K.shape, dtype=K.dtype, pin_memory=True)
+    Y_host.copy_(Yd, non_blocking=True)
+    torch.cuda.current_stream(dev).synchronize()
+    return Y_host

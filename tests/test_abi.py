@@ -1,0 +1,139 @@
+"""The C ABI on the host: the library loads, exports every declared symbol, sizes its
+workspace from the shape, and rejects bad arguments before touching the GPU.
+
+Nothing here launches a kernel: every call below fails validation (or is a no-op shape),
+so these tests run on a machine without a GPU.
+"""
+import ctypes
+import os
+import re
+
+import pytest
+
+from paper_2608_11519_gb300 import build as lib_build
+from paper_2608_11519_gb300 import flarepp
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+@pytest.fixture(scope="module")
+def lib():
+    lib_build.build()
+    return flarepp.load()
+
+
+def declared_symbols():
+    syms = []
+    for name in os.listdir(os.path.join(ROOT, "include")):
+        if name.endswith(".h"):
+            text = open(os.path.join(ROOT, "include", name)).read()
+            syms += re.findall(r"FLAREPP_API\s+[\w\s\*]+?\b(flarepp_\w+)\s*\(", text)
+    return sorted(set(syms))
+
+
+def test_every_declared_symbol_is_exported(lib):
+    syms = declared_symbols()
+    assert len(syms) >= 6
+    for s in syms:
+        assert hasattr(lib, s), s
+    assert set(flarepp.EXPORTED) <= set(syms)
+
+
+def test_status_strings(lib):
+    for code in range(6):
+        assert flarepp.status_string(code)
+    assert flarepp.status_string(99) == "unknown status"
+    assert flarepp.version().count(".") == 2
+
+
+def S(B=1, H=2, N=1000, M=32, D=32, dtype=flarepp.BF16):
+    return flarepp.Shape(B, H, N, M, D, dtype)
+
+
+def test_workspace_bytes(lib):
+    ws = lambda s: lib.flarepp_route_workspace_bytes(ctypes.byref(s))
+    assert ws(S()) > 0
+    assert ws(S()) % 256 == 0
+    # invalid or unsupported shapes need none
+    assert ws(S(D=24)) == 0
+    assert ws(S(M=4096)) == 0
+    assert ws(S(B=-1)) == 0
+    assert ws(S(dtype=7)) == 0
+    assert lib.flarepp_route_workspace_bytes(None) == 0
+    # degenerate shapes need none
+    assert ws(S(N=0)) == 0 and ws(S(B=0)) == 0 and ws(S(M=0)) == 0
+    # grows with the problem; holds at least Q and Z in float32
+    small, big = ws(S(N=1000)), ws(S(N=1000, M=1024))
+    assert big > small >= 2 * 1 * 2 * 32 * 32 * 4
+    # a function of the shape alone
+    assert ws(S(B=4, H=8, N=16384, M=128)) == ws(S(B=4, H=8, N=16384, M=128))
+
+
+FAKE = 0x7F0000000000  # an aligned address that is never dereferenced
+
+
+def call(lib, shape, ptrs=None, scale=0.25, ws=None, ws_bytes=None, Y=None):
+    p = ptrs or {}
+    base = FAKE
+    vals = {}
+    for i, n in enumerate(("seeds", "Kt", "Vt", "K", "V")):
+        vals[n] = p.get(n, base + (i + 1) * (1 << 36))
+    Yp = Y if Y is not None else base + 6 * (1 << 36)
+    wsp = ws if ws is not None else base + 7 * (1 << 36)
+    need = lib.flarepp_route_workspace_bytes(ctypes.byref(shape)) if shape is not None else 0
+    wsb = need if ws_bytes is None else ws_bytes
+    v = lambda x: None if x is None else ctypes.c_void_p(x)
+    return lib.flarepp_route_fwd(None if shape is None else ctypes.byref(shape), v(vals["seeds"]),
+                                 v(vals["Kt"]), v(vals["Vt"]), v(vals["K"]), v(vals["V"]),
+                                 ctypes.c_float(scale), v(Yp), v(wsp), wsb, None)
+
+
+def test_invalid_arguments_rejected_before_launch(lib):
+    E = flarepp
+    assert call(lib, None) == E.ERR_INVALID_ARGUMENT
+    assert call(lib, S(dtype=3)) == E.ERR_INVALID_ARGUMENT
+    assert call(lib, S(N=-5)) == E.ERR_INVALID_ARGUMENT
+    assert call(lib, S(D=48)) == E.ERR_UNSUPPORTED
+    assert call(lib, S(D=128)) == E.ERR_UNSUPPORTED
+    assert call(lib, S(M=2049)) == E.ERR_UNSUPPORTED
+    assert call(lib, S(B=1 << 20, H=1 << 20, N=1 << 20)) == E.ERR_UNSUPPORTED
+    assert call(lib, S(), scale=float("nan")) == E.ERR_INVALID_ARGUMENT
+    assert call(lib, S(), scale=float("inf")) == E.ERR_INVALID_ARGUMENT
+    assert call(lib, S(), ptrs={"K": None}) == E.ERR_INVALID_ARGUMENT
+    assert call(lib, S(), ptrs={"seeds": None}) == E.ERR_INVALID_ARGUMENT
+    assert call(lib, S(), ptrs={"V": FAKE + 8}) == E.ERR_INVALID_ARGUMENT  # misaligned
+    assert call(lib, S(), Y=FAKE + (1 << 36) + 64) == E.ERR_INVALID_ARGUMENT  # Y overlaps Kt...
+    assert call(lib, S(), Y=FAKE + 1 * (1 << 36)) == E.ERR_INVALID_ARGUMENT
+    assert call(lib, S(), ws_bytes=16) == E.ERR_WORKSPACE
+    assert call(lib, S(), ws=FAKE + 7 * (1 << 36) + 128) == E.ERR_WORKSPACE  # not 256-aligned
+    assert call(lib, S(), ws=0) == E.ERR_WORKSPACE
+    # profiled entry: events required
+    assert lib.flarepp_route_fwd_profiled(ctypes.byref(S()), None, None, None, None, None,
+                                          ctypes.c_float(0.25), None, None, 0, None, None,
+                                          6) == E.ERR_INVALID_ARGUMENT
+
+
+def test_degenerate_shapes_are_noops(lib):
+    # B*H = 0 and N = 0 enqueue nothing, so they succeed even without a GPU
+    assert call(lib, S(B=0)) == flarepp.OK
+    assert call(lib, S(H=0)) == flarepp.OK
+    assert call(lib, S(N=0), ptrs={k: None for k in ("Kt", "Vt", "K", "V")}) == flarepp.OK
+
+
+def test_python_binding_rejects_bad_tensors(lib):
+    import torch
+    x = torch.zeros(1, 2, 8, 32, dtype=torch.bfloat16)
+    s = torch.zeros(2, 4, 32, dtype=torch.bfloat16)
+    with pytest.raises(ValueError):
+        flarepp.route_fwd(s, x, x, x, x)  # host tensors
+    with pytest.raises(TypeError):
+        flarepp.route_fwd(s, x, x, x.float(), x)
+    with pytest.raises(ValueError):
+        flarepp.route_fwd(s[:1], x, x, x, x)
+    with pytest.raises(ValueError):
+        flarepp.route_fwd(s, x.transpose(2, 3), x, x, x)
+
+
+def test_missing_library_fails_loudly(tmp_path):
+    with pytest.raises(RuntimeError):
+        flarepp.load(str(tmp_path / "libflarepp.so"))

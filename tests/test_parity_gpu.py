@@ -1,0 +1,230 @@
+"""GPU parity of the routing chain against the float64 oracle, through the C ABI.
+
+Tolerances (max abs error, after upcasting Y to float64):
+  * float32 inputs: 1e-5 on Q, Z and Y
+  * bf16 inputs, float32 accumulation: 2e-2 on Q, Z and Y
+Inputs come from paper_2608_11519_gb300.inputs (seeded); the oracle sees the exact input
+values the GPU sees. Full-size workloads are checked on whole (b, h) slices (slices are
+independent, Sec. 3.2) or, for the largest, on sampled tokens of one slice, plus the
+convex-hull property on every output.
+"""
+import math
+
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from paper_2608_11519_gb300 import flarepp, inputs
+
+pytestmark = pytest.mark.gpu
+
+TOL = {"f32": 1e-5, "bf16": 2e-2}
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _lib():
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    flarepp.load()
+    torch.cuda.set_device(0)
+
+
+def _np(t):
+    return t.detach().to("cpu", torch.float64).numpy()
+
+
+def _run(x, scale, stream=None):
+    xd = {k: v.cuda() for k, v in x.items()}
+    Y, Q, Z = flarepp.route_fwd_debug(xd["seeds"], xd["Kt"], xd["Vt"], xd["K"], xd["V"], scale,
+                                      stream=stream)
+    torch.cuda.synchronize()
+    return _np(Y), _np(Q), _np(Z)
+
+
+def _check(name, got, want, tol):
+    err = float(np.abs(got - want).max()) if got.size else 0.0
+    assert err <= tol and not math.isnan(err), f"{name}: max|err| {err} > {tol}"
+    return err
+
+
+def _full_check(w, seed=0, scale=None, x=None):
+    x = x if x is not None else inputs.make_inputs(w, seed)
+    s = w.scale if scale is None else scale
+    Y, Q, Z = _run(x, s)
+    f = inputs.to_f64_numpy(x)
+    Qo, Zo, Yo = oracle.route(f["seeds"], f["Kt"], f["Vt"], f["K"], f["V"], s)
+    tol = TOL[w.dtype]
+    return {n: _check(n, g, o, tol) for n, g, o in (("Q", Q, Qo), ("Z", Z, Zo), ("Y", Y, Yo))}
+
+
+def _hull_check(Y, V, slack):
+    lo = V.min(axis=2, keepdims=True)
+    hi = V.max(axis=2, keepdims=True)
+    assert np.all(Y >= lo - slack) and np.all(Y <= hi + slack)
+
+
+def _slice_check(w, slices, seed=0, sample_tokens=None):
+    """Full-size run; oracle on the listed (b, h) slices (all tokens, or a token sample)."""
+    x = inputs.make_inputs(w, seed, device="cuda")
+    Y, Q, Z = _run(x, w.scale)
+    tol = TOL[w.dtype]
+    V = x["V"]
+    for (b, h) in slices:
+        f = {k: _np(v[h:h + 1] if k == "seeds" else v[b:b + 1, h:h + 1]) for k, v in x.items()}
+        if sample_tokens is None:
+            Qo, Zo, Yo = oracle.route(f["seeds"], f["Kt"], f["Vt"], f["K"], f["V"], w.scale)
+            _check(f"Y[{b},{h}]", Y[b:b + 1, h:h + 1], Yo, tol)
+        else:
+            seeds_b = f["seeds"][None]
+            Qo, _ = oracle.sdpa(seeds_b, f["Kt"], f["Vt"], w.scale)
+            Zo, _ = oracle.sdpa(Qo, f["K"], f["V"], w.scale)
+            rng = np.random.default_rng(b * 131 + h)
+            rows = np.unique(np.concatenate([rng.integers(0, w.N, sample_tokens), [0, w.N - 1]]))
+            Yo, _ = oracle.sdpa(f["K"][:, :, rows], Qo, Zo, w.scale)
+            _check(f"Y[{b},{h}] sampled", Y[b:b + 1, h:h + 1][:, :, rows], Yo, tol)
+        _check(f"Q[{b},{h}]", Q[b:b + 1, h:h + 1], Qo, tol)
+        _check(f"Z[{b},{h}]", Z[b:b + 1, h:h + 1], Zo, tol)
+    _hull_check(Y, _np(V), 1e-2 if w.dtype == "bf16" else 1e-6)
+
+
+# ------------------------------------------------------------------ the stated workloads
+
+def test_tiny_f32_full():
+    _full_check(inputs.get("tiny"), seed=0)
+
+
+def test_golden_fixture_f32():
+    import json
+    import os
+    with open(os.path.join(os.path.dirname(__file__), "golden", "route_small.json")) as fh:
+        doc = json.load(fh)
+    x = {k: torch.tensor(v, dtype=torch.float32) for k, v in doc["inputs"].items()}
+    Y, Q, Z = _run(x, doc["scale"])
+    for name, got in (("Q", Q), ("Z", Z), ("Y", Y)):
+        _check(name, got, np.array(doc["expected"][name]), 1e-5)
+
+
+def test_pde2d_full_size():
+    _slice_check(inputs.get("pde2d"), [(0, 0), (1, 3), (2, 6), (3, 7)])
+
+
+def test_longseq_full_size():
+    _slice_check(inputs.get("longseq"), [(0, 0), (17, 4), (31, 7)])
+
+
+def test_mesh3d_full_size_sampled():
+    _slice_check(inputs.get("mesh3d"), [(0, 5)], sample_tokens=2048)
+
+
+@pytest.mark.parametrize("M,D", [(16, 16), (64, 32), (128, 64), (256, 16)])
+def test_sweep_full_size(M, D):
+    _slice_check(inputs.get(f"sweep_M{M}_D{D}"), [(0, 3)])
+
+
+@pytest.mark.parametrize("M,D", [(512, 32), (1024, 64), (2048, 16), (2048, 64)])
+def test_sweep_large_M_reduced_N(M, D):
+    w = inputs.get(f"sweep_M{M}_D{D}").with_(H=2, N=8192)
+    _full_check(w)
+
+
+# ------------------------------------------------------------------ edge cases
+
+@pytest.mark.parametrize("dtype", ["f32", "bf16"])
+@pytest.mark.parametrize("N,M,D", [(1, 1, 16), (2, 3, 32), (31, 5, 64), (127, 32, 16),
+                                   (129, 100, 32), (1000, 130, 64), (4097, 300, 32),
+                                   (257, 1, 32), (5000, 17, 16)])
+def test_ragged_shapes(dtype, N, M, D):
+    w = inputs.Workload("ragged", 2, 3, N, M, D, dtype)
+    _full_check(w, seed=N + M + D)
+
+
+@pytest.mark.parametrize("dtype", ["f32", "bf16"])
+def test_clustered_peaked_small(dtype):
+    w = inputs.Workload("peaked", 1, 2, 3000, 64, 32, dtype, n_centres=16)
+    _full_check(w, seed=3)
+
+
+def test_scale_zero_and_large():
+    w = inputs.Workload("s", 1, 2, 700, 24, 32, "f32")
+    _full_check(w, scale=0.0)
+    _full_check(w, scale=2.0)  # logits of order 10: tests the running max
+
+
+def test_m_zero_writes_zero():
+    w = inputs.Workload("m0", 1, 2, 100, 0, 32, "bf16")
+    x = {k: v.cuda() for k, v in inputs.make_inputs(w).items()}
+    Y = torch.full_like(x["K"], 7.0)
+    flarepp.route_fwd(x["seeds"], x["Kt"], x["Vt"], x["K"], x["V"], Y=Y)
+    torch.cuda.synchronize()
+    assert torch.all(Y == 0)
+
+
+def test_n_zero_and_b_zero_are_noops():
+    for (B, N) in [(2, 0), (0, 50)]:
+        w = inputs.Workload("e", B, 2, N, 8, 16, "f32")
+        x = {k: v.cuda() for k, v in inputs.make_inputs(w).items()}
+        Y, Q, Z = flarepp.route_fwd_debug(x["seeds"], x["Kt"], x["Vt"], x["K"], x["V"])
+        torch.cuda.synchronize()
+        assert Y.numel() == 0 or B == 0
+        assert torch.all(Q == 0) and torch.all(Z == 0)
+
+
+def test_constant_values_give_constant_output():
+    w = inputs.get("pde2d").with_(B=1, N=20000)
+    x = inputs.make_inputs(w, seed=1, device="cuda")
+    c = torch.randn(1, w.H, 1, w.D, device="cuda").to(torch.bfloat16)
+    x["V"] = c.expand_as(x["V"]).contiguous()
+    Y = flarepp.route_fwd(x["seeds"], x["Kt"], x["Vt"], x["K"], x["V"])
+    torch.cuda.synchronize()
+    assert float((Y.float() - x["V"].float()).abs().max()) <= 2e-2
+
+
+def test_deterministic_bitwise():
+    w = inputs.get("pde2d").with_(B=2, N=9000)
+    x = inputs.make_inputs(w, seed=4, device="cuda")
+    a = flarepp.route_fwd(x["seeds"], x["Kt"], x["Vt"], x["K"], x["V"])
+    b = flarepp.route_fwd(x["seeds"], x["Kt"], x["Vt"], x["K"], x["V"])
+    torch.cuda.synchronize()
+    assert torch.equal(a, b)
+
+
+def test_guard_bands_untouched():
+    """Canaries right after Y and after the workspace must survive a call."""
+    w = inputs.get("pde2d").with_(B=1, N=5000)
+    x = inputs.make_inputs(w, seed=5, device="cuda")
+    nY = x["K"].numel()
+    ybuf = torch.full((nY + 4096,), 1234.0, dtype=torch.bfloat16, device="cuda")
+    Y = ybuf[:nY].view_as(x["K"])
+    nws = flarepp.workspace_bytes(w.B, w.H, w.N, w.M, w.D, flarepp.BF16)
+    wsbuf = torch.full((nws + 65536,), 0xA5, dtype=torch.uint8, device="cuda")
+    flarepp.route_fwd(x["seeds"], x["Kt"], x["Vt"], x["K"], x["V"], Y=Y, workspace=wsbuf)
+    torch.cuda.synchronize()
+    assert torch.all(ybuf[nY:] == 1234.0)
+    assert torch.all(wsbuf[nws:] == 0xA5)
+
+
+def test_side_stream_and_host_entry():
+    w = inputs.get("tiny")
+    x = inputs.make_inputs(w, seed=9)
+    f = inputs.to_f64_numpy(x)
+    _, _, Yo = oracle.route(f["seeds"], f["Kt"], f["Vt"], f["K"], f["V"], w.scale)
+    s = torch.cuda.Stream()
+    with torch.cuda.stream(s):
+        Y, _, _ = _run(x, w.scale, stream=s)
+    _check("Y side stream", Y, Yo, 1e-5)
+    xh = {k: v.pin_memory() for k, v in x.items()}
+    Yh = flarepp.route_fwd_host(xh["seeds"], xh["Kt"], xh["Vt"], xh["K"], xh["V"], w.scale)
+    _check("Y host entry", _np(Yh), Yo, 1e-5)
+
+
+def test_profiled_entry_records_stages():
+    w = inputs.get("pde2d").with_(B=1, N=8192)
+    x = inputs.make_inputs(w, seed=2, device="cuda")
+    ev = flarepp.StageEvents()
+    Y = flarepp.route_fwd_profiled(x["seeds"], x["Kt"], x["Vt"], x["K"], x["V"], ev)
+    ms = ev.stage_ms()
+    assert set(ms) == set(flarepp.STAGES) and all(v >= 0 for v in ms.values())
+    Y2 = flarepp.route_fwd(x["seeds"], x["Kt"], x["Vt"], x["K"], x["V"])
+    torch.cuda.synchronize()
+    assert torch.equal(Y, Y2)
