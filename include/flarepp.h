@@ -122,6 +122,16 @@ FLAREPP_API flarepp_status flarepp_route_fwd_profiled(const flarepp_shape* shape
                                                       void* stream, void* const* events,
                                                       int n_events);
 
+/*
+ * The device status word that the last flarepp_route_fwd* call on `workspace` (for the same
+ * shape) left behind: FLAREPP_OK, or FLAREPP_ERR_TIMEOUT when a bounded wait inside a
+ * tensor-core kernel gave up (the kernel then stops early and its outputs are invalid).
+ * Copies 4 bytes to *status_out (host memory) on `stream` and synchronises that stream.
+ */
+FLAREPP_API flarepp_status flarepp_route_device_status(const flarepp_shape* shape,
+                                                       const void* workspace, void* stream,
+                                                       int32_t* status_out);
+
 /* Static description of a status code (never NULL). */
 FLAREPP_API const char* flarepp_status_string(flarepp_status status);
 

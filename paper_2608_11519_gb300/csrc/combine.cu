@@ -14,32 +14,53 @@ __device__ __forceinline__ float fast_exp2(float x) {
     return y;
 }
 
-// One warp per (bh, m): merge the chunk partials in ascending chunk order (App. A.3):
+// Routes per tensor-core encode work unit and the route tiles it splits them into.
+constexpr int64_t kTcGroup = 512;
+constexpr int64_t kTcTile = 128;
+
+// Partial slots a route's chunks use: 1 on the CUDA-core path; on the tensor-core path a
+// work unit with n_a route tiles splits each chunk over 4 / n_a token-parity streams.
+__device__ __forceinline__ int slots_of_route(int64_t M, int64_t m, int64_t sub_per_chunk) {
+    if (sub_per_chunk == 1) return 1;
+    const int64_t g = m / kTcGroup;
+    const int64_t rem = M - g * kTcGroup;
+    const int64_t tiles = rem >= kTcGroup ? 4 : (rem + kTcTile - 1) / kTcTile;
+    const int na = tiles <= 1 ? 1 : (tiles <= 2 ? 2 : 4);
+    return 4 / na;
+}
+
+// One warp per (bh, m): merge the partial slots in ascending order (App. A.3):
 //   g = max_r mx_r; w_r = 2^(mx_r - g); out = sum_r w_r acc_r / sum_r w_r l_r.
 template <int D>
 __global__ void combine_kernel(const float* __restrict__ pmax, const float* __restrict__ psum,
                                const float* __restrict__ pacc, int64_t rows, int64_t M,
-                               int64_t nchunk, float* __restrict__ out32,
-                               __nv_bfloat16* __restrict__ outop) {
+                               int64_t nchunk, int64_t sub_per_chunk, float* __restrict__ out32,
+                               __nv_bfloat16* __restrict__ outop, float op_sign) {
     constexpr int PER = (D + 31) / 32;
     const int lane = threadIdx.x & 31;
     const int64_t row = (int64_t)blockIdx.x * (blockDim.x / 32) + threadIdx.x / 32;
     if (row >= rows) return;
     const int64_t bh = row / M, m = row % M;
+    const int used = slots_of_route(M, m, sub_per_chunk);
+    const int64_t nslot = nchunk * sub_per_chunk;
     float g = -INFINITY;
-    for (int64_t c = 0; c < nchunk; ++c) g = fmaxf(g, pmax[(bh * nchunk + c) * M + m]);
+    for (int64_t c = 0; c < nchunk; ++c)
+        for (int p = 0; p < used; ++p)
+            g = fmaxf(g, pmax[(bh * nslot + c * sub_per_chunk + p) * M + m]);
     float a = 0.f, u[PER];
 #pragma unroll
     for (int i = 0; i < PER; ++i) u[i] = 0.f;
     if (g != -INFINITY) {
         for (int64_t c = 0; c < nchunk; ++c) {
-            const int64_t r = (bh * nchunk + c) * M + m;
-            const float w = fast_exp2(pmax[r] - g);
-            a = fmaf(w, psum[r], a);
+            for (int p = 0; p < used; ++p) {
+                const int64_t r = (bh * nslot + c * sub_per_chunk + p) * M + m;
+                const float w = fast_exp2(pmax[r] - g);
+                a = fmaf(w, psum[r], a);
 #pragma unroll
-            for (int i = 0; i < PER; ++i) {
-                const int d = lane + 32 * i;
-                if (d < D) u[i] = fmaf(w, pacc[r * D + d], u[i]);
+                for (int i = 0; i < PER; ++i) {
+                    const int d = lane + 32 * i;
+                    if (d < D) u[i] = fmaf(w, pacc[r * D + d], u[i]);
+                }
             }
         }
     }
@@ -50,14 +71,21 @@ __global__ void combine_kernel(const float* __restrict__ pmax, const float* __re
         if (d < D) {
             const float val = u[i] * inv;
             out32[row * D + d] = val;
-            if (outop) outop[row * D + d] = __float2bfloat16_rn(val);
+            if (outop) outop[row * D + d] = __float2bfloat16_rn(op_sign * val);
         }
     }
 }
 
+__global__ void negate_bf16_kernel(const __nv_bfloat16* __restrict__ src,
+                                   __nv_bfloat16* __restrict__ dst, int64_t n) {
+    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n;
+         i += (int64_t)gridDim.x * blockDim.x)
+        dst[i] = __hneg(src[i]);
+}
+
 }  // namespace
 
-cudaError_t combine(const Plan& p, int call, char* ws, cudaStream_t st) {
+cudaError_t combine(const Plan& p, int call, char* ws, bool negate, cudaStream_t st) {
     const int64_t rows = p.BH * p.M;
     const int warps = 8;
     const int64_t blocks = (rows + warps - 1) / warps;
@@ -67,21 +95,26 @@ cudaError_t combine(const Plan& p, int call, char* ws, cudaStream_t st) {
     const float* pmax = (const float*)(ws + p.off_pmax);
     const float* psum = (const float*)(ws + p.off_psum);
     const float* pacc = (const float*)(ws + p.off_pacc);
+    const float sign = negate ? -1.f : 1.f;
+#define FLAREPP_COMBINE(DD)                                                                    \
+    combine_kernel<DD><<<(unsigned)blocks, warps * 32, 0, st>>>(pmax, psum, pacc, rows, p.M,  \
+                                                                p.nchunk, p.sub_per_chunk,     \
+                                                                out32, outop, sign);
     switch (p.D) {
-        case 16:
-            combine_kernel<16><<<(unsigned)blocks, warps * 32, 0, st>>>(pmax, psum, pacc, rows, p.M,
-                                                                        p.nchunk, out32, outop);
-            break;
-        case 32:
-            combine_kernel<32><<<(unsigned)blocks, warps * 32, 0, st>>>(pmax, psum, pacc, rows, p.M,
-                                                                        p.nchunk, out32, outop);
-            break;
-        case 64:
-            combine_kernel<64><<<(unsigned)blocks, warps * 32, 0, st>>>(pmax, psum, pacc, rows, p.M,
-                                                                        p.nchunk, out32, outop);
-            break;
+        case 16: FLAREPP_COMBINE(16) break;
+        case 32: FLAREPP_COMBINE(32) break;
+        case 64: FLAREPP_COMBINE(64) break;
         default: return cudaErrorInvalidValue;
     }
+#undef FLAREPP_COMBINE
+    return cudaGetLastError();
+}
+
+cudaError_t negate_bf16(const void* src, void* dst, int64_t n, cudaStream_t st) {
+    if (n <= 0) return cudaSuccess;
+    const int64_t blocks = (n + 255) / 256 < 1024 ? (n + 255) / 256 : 1024;
+    negate_bf16_kernel<<<(unsigned)blocks, 256, 0, st>>>((const __nv_bfloat16*)src,
+                                                         (__nv_bfloat16*)dst, n);
     return cudaGetLastError();
 }
 

@@ -15,6 +15,9 @@ constexpr int64_t kMaxM = 2048;
 constexpr int64_t kMaxTokenHeads = int64_t(1) << 40;  // B*H*N limit (index headroom)
 constexpr size_t kWsAlign = 256;
 constexpr int kStageEvents = 6;
+constexpr int64_t kMaxTmaCoord = 2147483647 - 4096;  // TMA coordinates are signed 32-bit
+constexpr int64_t kTcGroup = 512;             // routes per tensor-core encode work unit
+constexpr int64_t kTcItem = 64;               // tokens per tensor-core encode item
 
 size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
 int64_t cdiv(int64_t a, int64_t b) { return (a + b - 1) / b; }
@@ -42,23 +45,53 @@ flarepp_status make_plan(const flarepp_shape* s, Plan* p) {
     p->D = s->D;
     p->BH = bh;
     p->dtype = s->dtype;
-    p->path = kPathSimt;
+    p->path = s->dtype == FLAREPP_BF16 ? kPathTc : kPathSimt;
+    if (p->path == kPathTc && (s->N > kMaxTmaCoord || bh > kMaxTmaCoord))
+        return FLAREPP_ERR_UNSUPPORTED;
     if (bh == 0 || s->N == 0 || s->M == 0) return FLAREPP_OK;  // nothing to plan
 
-    // CUDA-core encode: one thread per route, up to 128 routes per CTA; chunks sized so
-    // that the grid holds about four waves of CTAs per SM.
-    p->m_tile = s->M >= 128 ? 128 : cdiv(s->M, 32) * 32;
-    p->n_mtiles = cdiv(s->M, p->m_tile);
-    p->m_pad = cdiv(s->M, 128) * 128;
-    const int64_t target = 4 * kNumSMs;
-    const int64_t per_chunk = bh * p->n_mtiles;
-    int64_t want = cdiv(target, per_chunk);
-    if (want < 1) want = 1;
-    p->chunk_len = cdiv(cdiv(s->N, want), 32) * 32;
-    p->nchunk = cdiv(s->N, p->chunk_len);
+    if (p->path == kPathSimt) {
+        // CUDA-core encode: one thread per route, up to 128 routes per CTA; chunks sized so
+        // that the grid holds about four waves of CTAs per SM.
+        p->m_tile = s->M >= 128 ? 128 : cdiv(s->M, 32) * 32;
+        p->n_mtiles = cdiv(s->M, p->m_tile);
+        p->sub_per_chunk = 1;
+        const int64_t target = 4 * kNumSMs;
+        int64_t want = cdiv(target, bh * p->n_mtiles);
+        if (want < 1) want = 1;
+        p->chunk_len = cdiv(cdiv(s->N, want), 32) * 32;
+        p->nchunk = cdiv(s->N, p->chunk_len);
+    } else {
+        // Tensor-core encode: a work unit is (bh, group of <= 512 routes, chunk of tokens) and
+        // one persistent CTA per SM walks the units. Pick the chunk count that minimises
+        // waves x (64-token items per unit, scaled by the group's route tiles, + a fixed
+        // per-unit cost of about three items).
+        p->n_groups = cdiv(s->M, kTcGroup);
+        p->sub_per_chunk = 4;
+        const int64_t tiles0 = s->M >= kTcGroup ? 4 : cdiv(s->M, 128);
+        const double na = tiles0 <= 1 ? 1.0 : (tiles0 <= 2 ? 2.0 : 4.0);
+        const int64_t per_chunk = bh * p->n_groups;
+        const int64_t max_chunks = cdiv(s->N, kTcItem);
+        double best = 1e300;
+        int64_t best_n = 1;
+        for (int64_t n = 1; n <= max_chunks && n <= 65536; ++n) {
+            const int64_t waves = cdiv(per_chunk * n, kNumSMs);
+            const int64_t items = cdiv(cdiv(s->N, n), kTcItem);
+            const double cost = (double)waves * ((double)items * na / 4.0 + 3.0);
+            if (cost < best) {
+                best = cost;
+                best_n = n;
+            }
+        }
+        p->chunk_len = cdiv(cdiv(s->N, best_n), kTcItem) * kTcItem;
+        p->nchunk = cdiv(s->N, p->chunk_len);
+    }
 
-    const size_t rows = (size_t)bh * (size_t)p->nchunk * (size_t)s->M;
+    const size_t rows =
+        (size_t)bh * (size_t)p->nchunk * (size_t)p->sub_per_chunk * (size_t)s->M;
     size_t off = 0;
+    p->off_status = off;
+    off = align_up(off + sizeof(int32_t), kWsAlign);
     p->off_pmax = off;
     off = align_up(off + rows * sizeof(float), kWsAlign);
     p->off_psum = off;
@@ -71,11 +104,13 @@ flarepp_status make_plan(const flarepp_shape* s, Plan* p) {
     p->off_z32 = off;
     off = align_up(off + qz, kWsAlign);
     if (p->path == kPathTc) {
-        const size_t op = (size_t)bh * (size_t)p->m_pad * (size_t)s->D * 2;
+        const size_t op = (size_t)bh * (size_t)s->M * (size_t)s->D * 2;
         p->off_qop = off;
         off = align_up(off + op, kWsAlign);
         p->off_zop = off;
         off = align_up(off + op, kWsAlign);
+        p->off_seedneg = off;
+        off = align_up(off + (size_t)s->H * (size_t)s->M * (size_t)s->D * 2, kWsAlign);
     }
     p->total = off;
     return FLAREPP_OK;
@@ -146,21 +181,27 @@ flarepp_status route_impl(const flarepp_shape* shape, const void* seeds, const v
     }
 
     char* ws = (char*)workspace;
-    const bool f32 = p.dtype == FLAREPP_F32;
+    const bool tc = p.path == kPathTc;
+    const bool neg = scale < 0.f;
     auto mark = [&](int i) {
         return !events || cudaEventRecord((cudaEvent_t)events[i], st) == cudaSuccess;
     };
     auto encode = [&](int call, const void* k, const void* v) {
-        return f32 ? simt_encode_f32(p, call, k, v, seeds, scale, ws, st)
-                   : simt_encode_bf16(p, call, k, v, seeds, scale, ws, st);
+        return tc ? tc_encode(p, call, k, v, seeds, scale, ws, st)
+                  : simt_encode_f32(p, call, k, v, seeds, scale, ws, st);
     };
+    if (cudaMemsetAsync(ws + p.off_status, 0, sizeof(int32_t), st) != cudaSuccess)
+        return FLAREPP_ERR_CUDA;
+    if (tc && neg &&
+        negate_bf16(seeds, ws + p.off_seedneg, p.H * p.M * p.D, st) != cudaSuccess)
+        return FLAREPP_ERR_CUDA;
     if (!mark(0)) return FLAREPP_ERR_CUDA;
     if (encode(1, Kt, Vt) != cudaSuccess || !mark(1)) return FLAREPP_ERR_CUDA;
-    if (combine(p, 1, ws, st) != cudaSuccess || !mark(2)) return FLAREPP_ERR_CUDA;
+    if (combine(p, 1, ws, neg, st) != cudaSuccess || !mark(2)) return FLAREPP_ERR_CUDA;
     if (encode(2, K, V) != cudaSuccess || !mark(3)) return FLAREPP_ERR_CUDA;
-    if (combine(p, 2, ws, st) != cudaSuccess || !mark(4)) return FLAREPP_ERR_CUDA;
-    const cudaError_t e = f32 ? simt_decode_f32(p, K, scale, Y, ws, st)
-                              : simt_decode_bf16(p, K, scale, Y, ws, st);
+    if (combine(p, 2, ws, false, st) != cudaSuccess || !mark(4)) return FLAREPP_ERR_CUDA;
+    cudaError_t e;
+    e = tc ? tc_decode(p, K, scale, Y, ws, st) : simt_decode_f32(p, K, scale, Y, ws, st);
     if (e != cudaSuccess || !mark(5)) return FLAREPP_ERR_CUDA;
     if (Q_out && cudaMemcpyAsync(Q_out, ws + p.off_q32, qz_bytes, cudaMemcpyDeviceToDevice, st) !=
                      cudaSuccess)
@@ -206,6 +247,23 @@ flarepp_status flarepp_route_fwd_profiled(const flarepp_shape* shape, const void
     if (!events) return FLAREPP_ERR_INVALID_ARGUMENT;
     return flarepp::route_impl(shape, seeds, Kt, Vt, K, V, scale, Y, workspace, workspace_bytes,
                                stream, nullptr, nullptr, events, n_events);
+}
+
+flarepp_status flarepp_route_device_status(const flarepp_shape* shape, const void* workspace,
+                                          void* stream, int32_t* status_out) {
+    flarepp::Plan p;
+    if (!status_out) return FLAREPP_ERR_INVALID_ARGUMENT;
+    const flarepp_status s = flarepp::make_plan(shape, &p);
+    if (s != FLAREPP_OK) return s;
+    *status_out = FLAREPP_OK;
+    if (p.total == 0) return FLAREPP_OK;
+    if (!workspace) return FLAREPP_ERR_WORKSPACE;
+    cudaStream_t st = (cudaStream_t)stream;
+    if (cudaMemcpyAsync(status_out, (const char*)workspace + p.off_status, sizeof(int32_t),
+                        cudaMemcpyDeviceToHost, st) != cudaSuccess ||
+        cudaStreamSynchronize(st) != cudaSuccess)
+        return FLAREPP_ERR_CUDA;
+    return FLAREPP_OK;
 }
 
 const char* flarepp_status_string(flarepp_status status) {

@@ -23,34 +23,44 @@ struct Plan {
     int path;
     // split-N encode: tokens [c * chunk_len, min(N, (c + 1) * chunk_len)) form chunk c
     int64_t chunk_len, nchunk;
-    int64_t m_tile, n_mtiles;  // routes per encode CTA and route tiles per head
-    int64_t m_pad;             // M rounded up for operand buffers
+    int64_t m_tile, n_mtiles;  // CUDA-core encode: routes per CTA and route tiles per head
+    int64_t n_groups;          // tensor-core encode: groups of up to 512 routes per work unit
+    int64_t sub_per_chunk;     // partial slots per chunk (1 CUDA-core, 4 tensor-core)
     // workspace layout (byte offsets from the workspace base, each 256-byte aligned)
-    size_t off_pmax, off_psum, off_pacc;  // partials [BH][nchunk][M] f32 x2, [BH][nchunk][M][D] f32
+    size_t off_status;                    // int32 device status word (FLAREPP_OK or _TIMEOUT)
+    size_t off_pmax, off_psum, off_pacc;  // partials [BH][nchunk*sub][M] f32 x2, (...)[D] f32
     size_t off_q32, off_z32;              // Q, Z float32 [BH][M][D]
-    size_t off_qop, off_zop;              // MMA operand copies of Q, Z (tensor-core path)
+    size_t off_qop, off_zop;              // bf16 MMA operand copies of Q, Z [BH][M][D]
+    size_t off_seedneg;                   // bf16 -seeds [H][M][D] (used when scale < 0)
     size_t total;
 };
 
 // Fill `p` for `s`; returns FLAREPP_OK or the validation error for the shape itself.
 flarepp_status make_plan(const flarepp_shape* s, Plan* p);
 
-// ---- CUDA-core kernels (simt_kernels.cuh, instantiated in simt_f32.cu / simt_bf16.cu)
-// Encode one call over all chunks: call 1 takes the seeds (element type of the inputs,
-// [H][M][D]), call 2 takes Q32 from the workspace. Writes the chunk partials.
+// ---- CUDA-core kernels (simt_kernels.cuh, instantiated in simt_f32.cu), float32 inputs
+// Encode one call over all chunks: call 1 takes the seeds ([H][M][D]), call 2 takes Q32
+// from the workspace. Writes the chunk partials.
 cudaError_t simt_encode_f32(const Plan& p, int call, const void* k, const void* v,
                             const void* seeds, float scale, char* ws, cudaStream_t st);
-cudaError_t simt_encode_bf16(const Plan& p, int call, const void* k, const void* v,
-                             const void* seeds, float scale, char* ws, cudaStream_t st);
 // Decode (call 3) on CUDA cores: Y = SDPA(K, Q32, Z32).
 cudaError_t simt_decode_f32(const Plan& p, const void* K, float scale, void* Y, char* ws,
                             cudaStream_t st);
-cudaError_t simt_decode_bf16(const Plan& p, const void* K, float scale, void* Y, char* ws,
-                             cudaStream_t st);
 
 // ---- split-N combine (combine.cu)
 // Stable log-sum-exp merge of the chunk partials into Q32 (call 1) or Z32 (call 2), plus
-// the MMA operand copy when the tensor-core path consumes it.
-cudaError_t combine(const Plan& p, int call, char* ws, cudaStream_t st);
+// the bf16 MMA operand copy when the tensor-core path consumes it (negated when
+// `negate`, which together with negated seeds turns a negative scale into |scale|).
+cudaError_t combine(const Plan& p, int call, char* ws, bool negate, cudaStream_t st);
+// dst = -src elementwise (bf16; exact)
+cudaError_t negate_bf16(const void* src, void* dst, int64_t n, cudaStream_t st);
+
+// ---- tensor-core kernels (tc_kernels.cu), bf16 inputs
+// Encode call 1 (A = seeds) or call 2 (A = Q operand) into the chunk partials.
+cudaError_t tc_encode(const Plan& p, int call, const void* k, const void* v, const void* seeds,
+                      float scale, char* ws, cudaStream_t st);
+// Decode call 3: Y = SDPA(K, Q, Z) from the Q and Z operand copies.
+cudaError_t tc_decode(const Plan& p, const void* K, float scale, void* Y, char* ws,
+                      cudaStream_t st);
 
 }  // namespace flarepp

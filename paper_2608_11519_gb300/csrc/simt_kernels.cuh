@@ -1,5 +1,6 @@
-// CUDA-core kernels of the routing chain (the float32 dtype path), instantiated per
-// element type by simt_f32.cu and simt_bf16.cu.
+// CUDA-core kernels of the routing chain: the float32 dtype path (instantiated in
+// simt_f32.cu). Products and accumulation in float32; tf32 tensor cores could not meet
+// the float32 tolerance.
 //
 // Encode (calls 1 and 2, Sec. 3.2): one thread per route row streams a chunk of tokens
 // through an online softmax (running max, running sum, weighted value sum) and writes

@@ -22,7 +22,8 @@ OK, ERR_INVALID_ARGUMENT, ERR_UNSUPPORTED, ERR_WORKSPACE, ERR_CUDA, ERR_TIMEOUT 
 _DTYPES = {torch.float32: F32, torch.bfloat16: BF16}
 
 EXPORTED = ("flarepp_route_workspace_bytes", "flarepp_route_fwd", "flarepp_route_fwd_debug",
-            "flarepp_route_fwd_profiled", "flarepp_status_string", "flarepp_version")
+            "flarepp_route_fwd_profiled", "flarepp_route_device_status", "flarepp_status_string",
+            "flarepp_version")
 N_STAGE_EVENTS = 6
 STAGES = ("encode1", "combine1", "encode2", "combine2", "decode")
 
@@ -68,6 +69,8 @@ def load(path: str = None):
     lib.flarepp_route_fwd_profiled.restype = ctypes.c_int
     lib.flarepp_route_fwd_profiled.argtypes = [sp, vp, vp, vp, vp, vp, ctypes.c_float, vp, vp, sz,
                                                vp, ctypes.POINTER(ctypes.c_void_p), ctypes.c_int]
+    lib.flarepp_route_device_status.restype = ctypes.c_int
+    lib.flarepp_route_device_status.argtypes = [sp, vp, vp, ctypes.POINTER(ctypes.c_int32)]
     lib.flarepp_status_string.restype = ctypes.c_char_p
     lib.flarepp_status_string.argtypes = [ctypes.c_int]
     lib.flarepp_version.restype = ctypes.c_char_p
@@ -175,6 +178,23 @@ def _call(debug, seeds, Kt, Vt, K, V, scale, Y, workspace, stream, Q_out, Z_out,
     if rc != OK:
         raise FlareppError(rc, "flarepp_route_fwd" + ("_debug" if debug else ""))
     return Y
+
+
+def device_status(shape_or_tensors, workspace, stream=None) -> int:
+    """The device status word the last call left in ``workspace`` (synchronises ``stream``):
+    OK, or ERR_TIMEOUT when a bounded wait inside a kernel gave up."""
+    shape = (shape_or_tensors if isinstance(shape_or_tensors, Shape)
+             else _shape_of(*shape_or_tensors))
+    buf = workspace.buf if isinstance(workspace, Workspace) else workspace
+    if stream is None:
+        stream = torch.cuda.current_stream()
+    out = ctypes.c_int32(-1)
+    rc = load().flarepp_route_device_status(ctypes.byref(shape), _ptr(buf),
+                                            ctypes.c_void_p(stream.cuda_stream),
+                                            ctypes.byref(out))
+    if rc != OK:
+        raise FlareppError(rc, "flarepp_route_device_status")
+    return int(out.value)
 
 
 def route_fwd(seeds, Kt, Vt, K, V, scale=None, Y=None, workspace=None, stream=None):

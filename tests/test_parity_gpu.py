@@ -48,13 +48,13 @@ def _check(name, got, want, tol):
     return err
 
 
-def _full_check(w, seed=0, scale=None, x=None):
+def _full_check(w, seed=0, scale=None, x=None, tol=None):
     x = x if x is not None else inputs.make_inputs(w, seed)
     s = w.scale if scale is None else scale
     Y, Q, Z = _run(x, s)
     f = inputs.to_f64_numpy(x)
     Qo, Zo, Yo = oracle.route(f["seeds"], f["Kt"], f["Vt"], f["K"], f["V"], s)
-    tol = TOL[w.dtype]
+    tol = TOL[w.dtype] if tol is None else tol
     return {n: _check(n, g, o, tol) for n, g, o in (("Q", Q, Qo), ("Z", Z, Zo), ("Y", Y, Yo))}
 
 
@@ -148,7 +148,11 @@ def test_clustered_peaked_small(dtype):
 def test_scale_zero_and_large():
     w = inputs.Workload("s", 1, 2, 700, 24, 32, "f32")
     _full_check(w, scale=0.0)
-    _full_check(w, scale=2.0)  # logits of order 10: tests the running max
+    # scale 2 gives logits of order +-30, which exercises the running max. The chain then
+    # amplifies float32 rounding: an error dQ in a routing query moves call-2 logits by
+    # s*|k|*dQ (s|k| ~ 2*8) and Z by that times the spread of V (~6), so the float32 bound
+    # here is ~1e-6 * 16 * 6 ~ 1e-4 rather than the 1e-5 of the paper's scale 1/sqrt(D).
+    _full_check(w, scale=2.0, tol=2e-4)
 
 
 def test_m_zero_writes_zero():
