@@ -123,6 +123,32 @@ FLAREPP_API flarepp_status flarepp_route_fwd_profiled(const flarepp_shape* shape
                                                       int n_events);
 
 /*
+ * flarepp_route_fwd without a caller-provided workspace. The paper has no counterpart: this
+ * entry point exists for callers that cannot allocate device memory when they call the
+ * chain. Examples are a plugin whose host application owns all device memory, and a
+ * latency-critical loop where cudaMalloc or cudaFree would synchronise the device.
+ * Inputs and Y are the caller's, exactly as in flarepp_route_fwd.
+ *   - Scratch: a fixed 64 MiB device array inside the library, held by every GPU that
+ *     loads it until the process exits. A shape whose flarepp_route_workspace_bytes
+ *     exceeds 64 MiB returns FLAREPP_ERR_WORKSPACE and enqueues nothing.
+ *   - No allocation: no cudaMalloc, cudaFree or other allocating call is made.
+ *   - First call per device: it looks up the array's device address (cudaGetSymbolAddress
+ *     with that device current) and caches it. Make that first call before any stream
+ *     capture.
+ *   - Sharing: every call on a device shares the one array, and the array keeps the last
+ *     call's contents. Each call clears the status word and writes all the scratch it
+ *     reads. Calls whose work overlaps on the GPU (other streams, other host threads) race
+ *     on the array and corrupt each other's results. Serialise them.
+ *   - The device status word of these calls lives in the array, so
+ *     flarepp_route_device_status, which reads a caller's workspace, cannot report it.
+ */
+FLAREPP_API flarepp_status flarepp_route_fwd_noalloc(const flarepp_shape* shape,
+                                                     const void* seeds, const void* Kt,
+                                                     const void* Vt, const void* K,
+                                                     const void* V, float scale, void* Y,
+                                                     void* stream);
+
+/*
  * The device status word that the last flarepp_route_fwd* call on `workspace` (for the same
  * shape) left behind: FLAREPP_OK, or FLAREPP_ERR_TIMEOUT when a bounded wait inside a
  * tensor-core kernel gave up (the kernel then stops early and its outputs are invalid).

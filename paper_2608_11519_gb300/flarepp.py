@@ -22,8 +22,8 @@ OK, ERR_INVALID_ARGUMENT, ERR_UNSUPPORTED, ERR_WORKSPACE, ERR_CUDA, ERR_TIMEOUT 
 _DTYPES = {torch.float32: F32, torch.bfloat16: BF16}
 
 EXPORTED = ("flarepp_route_workspace_bytes", "flarepp_route_fwd", "flarepp_route_fwd_debug",
-            "flarepp_route_fwd_profiled", "flarepp_route_device_status", "flarepp_status_string",
-            "flarepp_version")
+            "flarepp_route_fwd_profiled", "flarepp_route_fwd_noalloc",
+            "flarepp_route_device_status", "flarepp_status_string", "flarepp_version")
 N_STAGE_EVENTS = 6
 STAGES = ("encode1", "combine1", "encode2", "combine2", "decode")
 
@@ -69,6 +69,8 @@ def load(path: str = None):
     lib.flarepp_route_fwd_profiled.restype = ctypes.c_int
     lib.flarepp_route_fwd_profiled.argtypes = [sp, vp, vp, vp, vp, vp, ctypes.c_float, vp, vp, sz,
                                                vp, ctypes.POINTER(ctypes.c_void_p), ctypes.c_int]
+    lib.flarepp_route_fwd_noalloc.restype = ctypes.c_int
+    lib.flarepp_route_fwd_noalloc.argtypes = [sp, vp, vp, vp, vp, vp, ctypes.c_float, vp, vp]
     lib.flarepp_route_device_status.restype = ctypes.c_int
     lib.flarepp_route_device_status.argtypes = [sp, vp, vp, ctypes.POINTER(ctypes.c_int32)]
     lib.flarepp_status_string.restype = ctypes.c_char_p
@@ -225,6 +227,30 @@ def route_fwd_profiled(seeds, Kt, Vt, K, V, events: StageEvents, scale=None, Y=N
     """``route_fwd`` that records ``events`` around each stage on the launching stream."""
     return _call(False, seeds, Kt, Vt, K, V, scale, Y, workspace, stream, None, None,
                  events.handles)
+
+
+def route_fwd_noalloc(seeds, Kt, Vt, K, V, scale=None, Y=None, stream=None):
+    """``route_fwd`` through flarepp_route_fwd_noalloc: for callers that cannot allocate
+    device memory at call time, the library uses its own fixed 64 MiB scratch array instead
+    of a workspace (larger shapes raise ERR_WORKSPACE). Calls that overlap on the GPU share
+    that array and race; the first call on a device should come before any stream capture.
+    Y is allocated here only when not given."""
+    lib = load()
+    shape = _shape_of(seeds, Kt, Vt, K, V)
+    if K.device.type != "cuda":
+        raise ValueError("route_fwd_noalloc takes device tensors")
+    if scale is None:
+        scale = 1.0 / math.sqrt(shape.D)
+    if Y is None:
+        Y = torch.empty_like(K)
+    if stream is None:
+        stream = torch.cuda.current_stream(K.device)
+    rc = lib.flarepp_route_fwd_noalloc(ctypes.byref(shape), _ptr(seeds), _ptr(Kt), _ptr(Vt),
+                                       _ptr(K), _ptr(V), float(scale), _ptr(Y),
+                                       ctypes.c_void_p(stream.cuda_stream))
+    if rc != OK:
+        raise FlareppError(rc, "flarepp_route_fwd_noalloc")
+    return Y
 
 
 def route_fwd_debug(seeds, Kt, Vt, K, V, scale=None, Y=None, workspace=None, stream=None):
