@@ -14,19 +14,18 @@ __device__ __forceinline__ float fast_exp2(float x) {
     return y;
 }
 
-// Routes per tensor-core encode work unit and the route tiles it splits them into.
-constexpr int64_t kTcGroup = 512;
-constexpr int64_t kTcTile = 128;
-
-// Partial slots a route's chunks use: 1 on the CUDA-core path; on the tensor-core path a
-// work unit with n_a route tiles splits each chunk over 4 / n_a token-parity streams.
-__device__ __forceinline__ int slots_of_route(int64_t M, int64_t m, int64_t sub_per_chunk) {
+// Partial slots a route's chunks use: 1 on the CUDA-core path. On the tensor-core path a
+// work unit covers a group of `group` routes in tiles of 128; a unit with n_a route tiles
+// (rounded to 1, 2 or 4) splits each chunk over (group / 128) / n_a token-parity streams.
+__device__ __forceinline__ int slots_of_route(int64_t M, int64_t m, int64_t sub_per_chunk,
+                                              int64_t group) {
     if (sub_per_chunk == 1) return 1;
-    const int64_t g = m / kTcGroup;
-    const int64_t rem = M - g * kTcGroup;
-    const int64_t tiles = rem >= kTcGroup ? 4 : (rem + kTcTile - 1) / kTcTile;
-    const int na = tiles <= 1 ? 1 : (tiles <= 2 ? 2 : 4);
-    return 4 / na;
+    const int64_t ns = group / 128;
+    const int64_t g = m / group;
+    const int64_t rem = M - g * group;
+    const int64_t tiles = rem >= group ? ns : (rem + 127) / 128;
+    const int64_t na = tiles <= 1 ? 1 : (tiles <= 2 ? 2 : 4);
+    return (int)(ns / na);
 }
 
 // One warp per (bh, m): merge the partial slots in ascending order (App. A.3):
@@ -34,14 +33,15 @@ __device__ __forceinline__ int slots_of_route(int64_t M, int64_t m, int64_t sub_
 template <int D>
 __global__ void combine_kernel(const float* __restrict__ pmax, const float* __restrict__ psum,
                                const float* __restrict__ pacc, int64_t rows, int64_t M,
-                               int64_t nchunk, int64_t sub_per_chunk, float* __restrict__ out32,
+                               int64_t nchunk, int64_t sub_per_chunk, int64_t group,
+                               float* __restrict__ out32,
                                __nv_bfloat16* __restrict__ outop, float op_sign) {
     constexpr int PER = (D + 31) / 32;
     const int lane = threadIdx.x & 31;
     const int64_t row = (int64_t)blockIdx.x * (blockDim.x / 32) + threadIdx.x / 32;
     if (row >= rows) return;
     const int64_t bh = row / M, m = row % M;
-    const int used = slots_of_route(M, m, sub_per_chunk);
+    const int used = slots_of_route(M, m, sub_per_chunk, group);
     const int64_t nslot = nchunk * sub_per_chunk;
     float g = -INFINITY;
     for (int64_t c = 0; c < nchunk; ++c)
@@ -99,6 +99,7 @@ cudaError_t combine(const Plan& p, int call, char* ws, bool negate, cudaStream_t
 #define FLAREPP_COMBINE(DD)                                                                    \
     combine_kernel<DD><<<(unsigned)blocks, warps * 32, 0, st>>>(pmax, psum, pacc, rows, p.M,  \
                                                                 p.nchunk, p.sub_per_chunk,     \
+                                                                p.tc_group,                    \
                                                                 out32, outop, sign);
     switch (p.D) {
         case 16: FLAREPP_COMBINE(16) break;

@@ -16,7 +16,6 @@ constexpr int64_t kMaxTokenHeads = int64_t(1) << 40;  // B*H*N limit (index head
 constexpr size_t kWsAlign = 256;
 constexpr int kStageEvents = 6;
 constexpr int64_t kMaxTmaCoord = 2147483647 - 4096;  // TMA coordinates are signed 32-bit
-constexpr int64_t kTcGroup = 512;             // routes per tensor-core encode work unit
 constexpr int64_t kTcItem = 64;               // tokens per tensor-core encode item
 
 size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
@@ -66,9 +65,11 @@ flarepp_status make_plan(const flarepp_shape* s, Plan* p) {
         // one persistent CTA per SM walks the units. Pick the chunk count that minimises
         // waves x (64-token items per unit, scaled by the group's route tiles, + a fixed
         // per-unit cost of about three items).
-        p->n_groups = cdiv(s->M, kTcGroup);
+        p->tc_group = tc_group_rows(s->D);
+        p->n_groups = cdiv(s->M, p->tc_group);
         p->sub_per_chunk = 4;
-        const int64_t tiles0 = s->M >= kTcGroup ? 4 : cdiv(s->M, 128);
+        const int64_t ns = p->tc_group / 128;
+        const int64_t tiles0 = s->M >= p->tc_group ? ns : cdiv(s->M, 128);
         const double na = tiles0 <= 1 ? 1.0 : (tiles0 <= 2 ? 2.0 : 4.0);
         const int64_t per_chunk = bh * p->n_groups;
         const int64_t max_chunks = cdiv(s->N, kTcItem);
@@ -77,7 +78,7 @@ flarepp_status make_plan(const flarepp_shape* s, Plan* p) {
         for (int64_t n = 1; n <= max_chunks && n <= 65536; ++n) {
             const int64_t waves = cdiv(per_chunk * n, kNumSMs);
             const int64_t items = cdiv(cdiv(s->N, n), kTcItem);
-            const double cost = (double)waves * ((double)items * na / 4.0 + 3.0);
+            const double cost = (double)waves * ((double)items * na / (double)ns + 3.0);
             if (cost < best) {
                 best = cost;
                 best_n = n;

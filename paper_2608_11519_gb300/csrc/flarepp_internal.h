@@ -4,7 +4,7 @@
 #include <stddef.h>
 #include <stdint.h>
 
-#include "../../include/flarepp.h"
+#include "flarepp.h"
 
 namespace flarepp {
 
@@ -24,7 +24,8 @@ struct Plan {
     // split-N encode: tokens [c * chunk_len, min(N, (c + 1) * chunk_len)) form chunk c
     int64_t chunk_len, nchunk;
     int64_t m_tile, n_mtiles;  // CUDA-core encode: routes per CTA and route tiles per head
-    int64_t n_groups;          // tensor-core encode: groups of up to 512 routes per work unit
+    int64_t n_groups;          // tensor-core encode: route groups per head
+    int64_t tc_group;          // tensor-core encode: routes per group (4 or 2 tiles of 128)
     int64_t sub_per_chunk;     // partial slots per chunk (1 CUDA-core, 4 tensor-core)
     // workspace layout (byte offsets from the workspace base, each 256-byte aligned)
     size_t off_status;                    // int32 device status word (FLAREPP_OK or _TIMEOUT)
@@ -59,6 +60,8 @@ cudaError_t negate_bf16(const void* src, void* dst, int64_t n, cudaStream_t st);
 // Encode call 1 (A = seeds) or call 2 (A = Q operand) into the chunk partials.
 cudaError_t tc_encode(const Plan& p, int call, const void* k, const void* v, const void* seeds,
                       float scale, char* ws, cudaStream_t st);
+// Rows per tensor-core work unit (route group of the encode, token group of the decode).
+int64_t tc_group_rows(int64_t D);
 // Decode call 3: Y = SDPA(K, Q, Z) from the Q and Z operand copies.
 cudaError_t tc_decode(const Plan& p, const void* K, float scale, void* Y, char* ws,
                       cudaStream_t st);

@@ -3,28 +3,30 @@
 // One warp-specialised kernel template serves both directions of the routing chain
 // (Sec. 3.2, eqs. flarepp_dynamic_query and flarepp_mixer):
 //
-//   encode (calls 1, 2): TMEM lanes are routes. A resident group of up to 4 route tiles
-//     (128 routes each, the A operand: seeds or Q) meets a stream of 64-token items
-//     (K and V tiles) from a chunk of the sequence; each route row keeps an online
-//     softmax over tokens and the CTA writes per-chunk partials (running max, sum and
-//     unnormalised value sum) for the log-sum-exp merge of App. A.3.
-//   decode (call 3): TMEM lanes are tokens. A resident group of 4 token tiles (K, 128
-//     tokens each) meets a stream of 64-route items (Q and Z tiles); each token row keeps
-//     an online softmax over routes and writes its normalised output row of Y.
+//   encode (calls 1, 2): TMEM lanes are routes. A group of NS route tiles (128 routes
+//     each; the A operand: seeds or Q) meets a stream of 64-token items (K and V tiles)
+//     from one chunk of the sequence. Each route row keeps an online softmax over tokens,
+//     and the CTA writes per-chunk partials (reference max, sum, unnormalised value sum)
+//     for the log-sum-exp merge of App. A.3.
+//   decode (call 3): TMEM lanes are tokens. A group of NS token tiles (K, 128 tokens each)
+//     meets a stream of 64-route items (Q and Z tiles). Each token row keeps an online
+//     softmax over routes and writes its normalised row of Y.
 //
-// Roles (10 warps): warp 0 issues TMA loads, warp 1 issues tcgen05.mma (one thread) and
-// owns the TMEM allocation, warps 2-9 form two softmax warpgroups. The four TMEM
-// "streams" s = 0..3 each hold a 128 x 64 fp32 score tile S (reused in place for the
-// bf16 probabilities P, the A operand of the PV product) and a 128 x D fp32 accumulator
-// O; warpgroup w serves streams w and w + 2. Per stream and item:
-//   MMA warp: S = A_tile * B_item^T (K-major, smem x smem) -> commit s_ready
-//   softmax:  row max, lazily raised running max (rescaling O in TMEM only when the max
-//             grows by more than 2^8), P = 2^(c S - m) in bf16 back into TMEM, row sum
-//             -> arrive p_ready
-//   MMA warp: O += P * C_item (P from TMEM, C MN-major in smem); the next S of the stream
-//             is issued after it, so a completed s_ready also means the previous PV is done.
+// Work is cut into NS TMEM "streams" (NS = 4 for D <= 32, 2 for D = 64). Stream s owns a
+// 128 x 64 fp32 score tile S (rewritten in place as bf16 P, the A operand of the PV
+// product) and a 128 x D fp32 accumulator O, and reads one resident A tile kept in TMEM,
+// so that S = A * B^T is a TMEM x SMEM product. Roles (13 warps):
+//   warp 0        TMA producer: A tiles (unswizzled) and the item ring (swizzled K/V or Q/Z)
+//   warps 1..4    one MMA warp per stream: the PV of its previous item, the S of its next
+//                 item, one commit per item (a commit stalls only the warp that issues it)
+//   warps 5..12   two softmax warpgroups; warpgroup w serves streams w and w + 2 (NS = 4)
+//                 or stream w (NS = 2) and copies its A tiles from smem into TMEM
+// The softmax keeps a reference max that is recomputed exactly only on a stream's first
+// item or when an item's probabilities sum past 2^48 (values stay far inside the fp32 and
+// bf16 ranges); otherwise P = 2^(c S - m) with the old reference.
 // Every wait is bounded (2 s of %globaltimer): on expiry the kernel records
-// FLAREPP_ERR_TIMEOUT in the status word, all roles leave their loops, and TMEM is freed.
+// FLAREPP_ERR_TIMEOUT in the status word, every role leaves its loops, the producer waits
+// for its copies in flight, and TMEM is freed.
 #include <cuda.h>
 #include <cudaTypedefs.h>
 #include <cuda_bf16.h>
@@ -39,32 +41,44 @@ namespace {
 
 using namespace tc;
 
-constexpr int kThreads = 320;
-constexpr int kTileRows = 128;
-constexpr int kItem = 64;          // streamed rows per item
-constexpr int kGroup = 512;        // resident rows per work unit (4 tiles of 128)
-constexpr float kLazyTau = 8.0f;   // log2 headroom of the lazy running max
+constexpr int kWarps = 13;
+constexpr int kThreads = kWarps * 32;
+constexpr int kFirstMmaWarp = 1;
+constexpr int kFirstSoftmaxWarp = 5;
+constexpr int kTileRows = 128;  // TMEM lanes, MMA M
+constexpr int kItem = 64;       // streamed rows per item
 constexpr uint64_t kWaitLimitNs = 2000000000ull;
 constexpr uint32_t kTmemCols = 512;
 constexpr float kLog2e = 1.4426950408889634f;
+// Sum of one item's probabilities above which the reference max is recomputed exactly.
+constexpr float kFastLimit = 281474976710656.0f;  // 2^48
 
 template <int D>
 struct Cfg {
-    static constexpr int kStages = D == 64 ? 5 : 8;
-    static constexpr int kATile = kTileRows * D * 2;
-    static constexpr int kABytes = 4 * kATile;
+    static constexpr int NS = D == 64 ? 2 : 4;        // streams
+    static constexpr int kGroup = NS * kTileRows;     // resident rows per work unit
+    static constexpr int kStages = 8;                 // a multiple of 4
+    static constexpr int kATile = kTileRows * D * 2;  // one 128-row operand tile
+    static constexpr int kABytes = NS * kATile;
     static constexpr int kItemTile = kItem * D * 2;
     static constexpr int kStage = 2 * kItemTile;
     static constexpr uint32_t kSwz = D == 16 ? kSw32 : (D == 32 ? kSw64 : kSw128);
-    static constexpr uint32_t kSBO = 8 * D * 2;
-    static constexpr int kNumBars = 2 * kStages + 12;
+    static constexpr uint32_t kSBO = 8 * D * 2;  // bytes between 8-row groups
+    // barriers: full[S], empty[S], asmem_full[2], asmem_empty[2], a_ready[2], a_free[2],
+    //           s_ready[NS], p_ready[NS]
+    static constexpr int kNumBars = 2 * kStages + 8 + 2 * NS;
     static constexpr int kData = 2 * kABytes + kStages * kStage;
     static constexpr int kNeed = 1024 + kData + kNumBars * 8 + 16;
     // at least 120 KB so that one CTA owns an SM and its 512 TMEM columns
     static constexpr int kSmem = kNeed > 122880 ? kNeed : 122880;
     static constexpr uint32_t kIdescS = idesc_bf16_f32(128, kItem, false, false);
     static constexpr uint32_t kIdescPV = idesc_bf16_f32(128, D, false, true);
-    static constexpr uint32_t kOCol = 4 * kItem;  // O accumulators follow the 4 score tiles
+    // TMEM columns
+    static constexpr uint32_t kColS = 0;               // NS x 64
+    static constexpr uint32_t kColO = NS * kItem;      // NS x D
+    static constexpr uint32_t kColA = kColO + NS * D;  // 2 buffers x NS tiles x D/2
+    static_assert(kColA + 2 * NS * (D / 2) <= kTmemCols, "TMEM budget");
+    static_assert(kSmem <= 232448, "shared memory budget");
 };
 
 struct TcParams {
@@ -81,9 +95,11 @@ struct TcParams {
     int* status;
 };
 
+// route tiles of encode group g, rounded up to 1, 2 or 4 (a divisor of the stream count)
+template <int NS>
 __device__ __forceinline__ int na_of_group(int64_t M, int64_t g) {
-    const int64_t rem = M - g * kGroup;
-    const int64_t tiles = rem >= kGroup ? 4 : (rem + kTileRows - 1) / kTileRows;
+    const int64_t rem = M - g * NS * kTileRows;
+    const int64_t tiles = rem >= NS * kTileRows ? NS : (rem + kTileRows - 1) / kTileRows;
     return tiles <= 1 ? 1 : (tiles <= 2 ? 2 : 4);
 }
 
@@ -94,8 +110,9 @@ struct Unit {
     int64_t item0, item_end;
 };
 
-template <bool DEC>
+template <int D, bool DEC>
 __device__ __forceinline__ Unit get_unit(const TcParams& p, int64_t u) {
+    using C = Cfg<D>;
     Unit U;
     if (DEC) {
         U.tg = u % p.n_tok_groups;
@@ -103,8 +120,8 @@ __device__ __forceinline__ Unit get_unit(const TcParams& p, int64_t u) {
         U.chunk = 0;
         U.g = 0;
         U.zA = (int)U.bh;
-        U.rowA0 = (int)(U.tg * kGroup);
-        U.n_a = 4;
+        U.rowA0 = (int)(U.tg * C::kGroup);
+        U.n_a = C::NS;
         U.n_par = 1;
         U.item0 = 0;
         U.item_end = p.M;
@@ -115,9 +132,9 @@ __device__ __forceinline__ Unit get_unit(const TcParams& p, int64_t u) {
         U.bh = t / p.n_groups;
         U.tg = 0;
         U.zA = (int)(p.a_per_head ? U.bh % p.H : U.bh);
-        U.rowA0 = (int)(U.g * kGroup);
-        U.n_a = na_of_group(p.M, U.g);
-        U.n_par = 4 / U.n_a;
+        U.rowA0 = (int)(U.g * C::kGroup);
+        U.n_a = na_of_group<C::NS>(p.M, U.g);
+        U.n_par = C::NS / U.n_a;
         U.item0 = U.chunk * p.chunk_len;
         U.item_end = min(p.N, U.item0 + p.chunk_len);
     }
@@ -154,44 +171,286 @@ __device__ __forceinline__ bool wait_bar(uint32_t bar, uint32_t parity, volatile
         }
     }
 }
+// The same wait taken by a whole warp: true only if every lane saw the phase complete.
+__device__ __forceinline__ bool warp_wait(uint32_t bar, uint32_t parity, volatile int* abort_flag,
+                                          int* status) {
+    const bool got = wait_bar(bar, parity, abort_flag, status);
+    return __all_sync(0xffffffffu, got);
+}
+
+// ------------------------------------------------------------------ softmax helpers
+
+// Online-softmax state of one TMEM stream, held by every thread of its warpgroup for its row.
+struct SoftmaxStream {
+    int s;          // stream index
+    int cnt, j;     // items of the stream in this unit, items done
+    float m, l;     // reference max (base 2, scaled) and running sum
+    uint32_t scnt;  // s_ready phases consumed so far (across units)
+    int prev_st;    // ring stage of the previous item (-1: none)
+    __device__ __forceinline__ void begin(const Unit& U) {
+        const int par = s / U.n_a;
+        cnt = U.n_items > par ? (U.n_items - par + U.n_par - 1) / U.n_par : 0;
+        j = 0;
+        m = -INFINITY;
+        l = 0.f;
+        prev_st = -1;
+    }
+};
+
+// Max over the valid columns [0, nv) of one 32-column half (columns base .. base + 31).
+__device__ __forceinline__ float half_max(const uint32_t* sr, int base, int nv) {
+    float a0 = -INFINITY, a1 = -INFINITY, a2 = -INFINITY, a3 = -INFINITY;
+    if (base + 32 <= nv) {
+#pragma unroll
+        for (int k = 0; k < 32; k += 8) {
+            a0 = max3f(a0, __uint_as_float(sr[k]), __uint_as_float(sr[k + 1]));
+            a1 = max3f(a1, __uint_as_float(sr[k + 2]), __uint_as_float(sr[k + 3]));
+            a2 = max3f(a2, __uint_as_float(sr[k + 4]), __uint_as_float(sr[k + 5]));
+            a3 = max3f(a3, __uint_as_float(sr[k + 6]), __uint_as_float(sr[k + 7]));
+        }
+    } else {
+#pragma unroll
+        for (int k = 0; k < 32; ++k)
+            if (base + k < nv) a0 = fmaxf(a0, __uint_as_float(sr[k]));
+    }
+    return max3f(a0, a1, fmaxf(a2, a3));
+}
+
+// P = 2^(c S - m) for one 32-column half, packed bf16 pairs into pr[0..15]; returns the
+// half's row sum. Columns at or beyond nv are not part of the softmax: probability 0.
+__device__ __forceinline__ float exp_half(const uint32_t* sr, uint32_t* pr, int base, int nv,
+                                          float c, uint64_t c2, float m) {
+    if (base + 32 <= nv) {
+        const uint64_t nm2 = pack_f32x2(-m, -m);
+        uint64_t acc0 = 0, acc1 = 0;  // two packed (lo, hi) partial sums
+#pragma unroll
+        for (int k = 0; k < 16; k += 2) {
+            pr[k] = exp2_pair(__uint_as_float(sr[2 * k]), __uint_as_float(sr[2 * k + 1]), c2,
+                              nm2, acc0);
+            pr[k + 1] = exp2_pair(__uint_as_float(sr[2 * k + 2]), __uint_as_float(sr[2 * k + 3]),
+                                  c2, nm2, acc1);
+        }
+        float a, b, x, y;
+        unpack_f32x2(acc0, a, b);
+        unpack_f32x2(acc1, x, y);
+        return (a + b) + (x + y);
+    }
+    float t0 = 0.f, t1 = 0.f;
+#pragma unroll
+    for (int k = 0; k < 16; ++k) {
+        const float p0 =
+            base + 2 * k < nv ? ex2(fmaf(__uint_as_float(sr[2 * k]), c, -m)) : 0.f;
+        const float p1 =
+            base + 2 * k + 1 < nv ? ex2(fmaf(__uint_as_float(sr[2 * k + 1]), c, -m)) : 0.f;
+        t0 += p0;
+        t1 += p1;
+        pr[k] = pack_bf16(p0, p1);
+    }
+    return t0 + t1;
+}
+
+// P for the whole 64-column tile at TMEM column scol (S is read half by half).
+__device__ __forceinline__ float exp_tile(uint32_t scol, uint32_t* pr, int nv, float c,
+                                          uint64_t c2, float m) {
+    float sum = 0.f;
+#pragma unroll
+    for (int h = 0; h < 2; ++h) {
+        uint32_t sr[32];
+        tmem_ld32(scol + 32 * h, sr);
+        tmem_wait_ld32(sr);
+        sum += exp_half(sr, pr + 16 * h, 32 * h, nv, c, c2, m);
+    }
+    return sum;
+}
+
+// One item of one stream for this thread's row: read S, update the online softmax, write P
+// back over S, signal the stream's MMA warp. Once S is ready the stream's previous PV has
+// completed, so the warpgroup leader also frees the ring stage of the previous item.
+// Returns false when the kernel is aborting.
+template <int D>
+__device__ __forceinline__ bool softmax_step(SoftmaxStream& S, const Unit& U, uint32_t tmem,
+                                             uint32_t lane_off, float c, uint64_t c2,
+                                             uint32_t sready, uint32_t pready, uint32_t empty0,
+                                             bool wg_leader, int stage, volatile int* abort_flag,
+                                             int* status) {
+    using C = Cfg<D>;
+    if (!warp_wait(sready, S.scnt & 1, abort_flag, status)) return false;
+    ++S.scnt;
+    tc_fence_after();
+    if (wg_leader && S.prev_st >= 0) mbar_arrive(empty0 + 8u * S.prev_st);
+    S.prev_st = stage;
+    const int item = S.s / U.n_a + S.j * U.n_par;
+    const int64_t start = U.item0 + (int64_t)item * kItem;
+    const int nv = (int)min((int64_t)kItem, U.item_end - start);
+    const uint32_t scol = tmem + lane_off + C::kColS + S.s * kItem;
+    uint32_t pr[kItem / 2];
+    float sum = 0.f;
+    bool slow = S.j == 0;
+    if (!slow) {
+        sum = exp_tile(scol, pr, nv, c, c2, S.m);
+        slow = __any_sync(0xffffffffu, !(sum <= kFastLimit));
+    }
+    if (slow) {
+        // exact max of this item (S is still intact in TMEM: P has not been written yet)
+        float mx = -INFINITY;
+#pragma unroll
+        for (int h = 0; h < 2; ++h) {
+            uint32_t sr[32];
+            tmem_ld32(scol + 32 * h, sr);
+            tmem_wait_ld32(sr);
+            mx = fmaxf(mx, half_max(sr, 32 * h, nv));
+        }
+        const float cand = mx * c;
+        bool need = false;
+        float alpha = 1.f;
+        if (cand > S.m) {
+            alpha = ex2(S.m - cand);  // 0 when S.m is -inf
+            need = S.j > 0;
+            S.l *= alpha;
+            S.m = cand;
+        }
+        if (__any_sync(0xffffffffu, need)) {
+            const uint32_t ocol = tmem + lane_off + C::kColO + S.s * D;
+            const float f = need ? alpha : 1.f;
+#pragma unroll
+            for (int k = 0; k < D / 16; ++k) {
+                uint32_t o[16];
+                tmem_ld16(ocol + 16 * k, o);
+                tmem_wait_ld16(o);
+#pragma unroll
+                for (int e = 0; e < 16; ++e) o[e] = __float_as_uint(__uint_as_float(o[e]) * f);
+                tmem_st16(ocol + 16 * k, o);
+            }
+        }
+        sum = exp_tile(scol, pr, nv, c, c2, S.m);
+    }
+    S.l += sum;
+    tmem_st32(scol, pr);
+    tmem_wait_st();
+    tc_fence_before();
+    mbar_arrive(pready);
+    ++S.j;
+    return true;
+}
+
+// After a stream's last item: read O and write the unit's result for this row (the chunk
+// partial in the encode, the normalised output row of Y in the decode).
+template <int D, bool DEC>
+__device__ __forceinline__ bool finish_stream(SoftmaxStream& S, const Unit& U,
+                                              const TcParams& prm, uint32_t tmem,
+                                              uint32_t lane_off, int r, uint32_t sready,
+                                              uint32_t empty0, bool wg_leader,
+                                              volatile int* abort_flag) {
+    using C = Cfg<D>;
+    const int a = S.s % U.n_a;
+    const int par = S.s / U.n_a;
+    float o[D];
+    if (S.cnt > 0) {
+        if (!warp_wait(sready, S.scnt & 1, abort_flag, prm.status)) return false;
+        ++S.scnt;
+        tc_fence_after();
+        if (wg_leader) mbar_arrive(empty0 + 8u * S.prev_st);
+        const uint32_t ocol = tmem + lane_off + C::kColO + S.s * D;
+#pragma unroll
+        for (int k = 0; k < D / 16; ++k) {
+            uint32_t t[16];
+            tmem_ld16(ocol + 16 * k, t);
+            tmem_wait_ld16(t);
+#pragma unroll
+            for (int e = 0; e < 16; ++e) o[16 * k + e] = __uint_as_float(t[e]);
+        }
+    } else {
+#pragma unroll
+        for (int d = 0; d < D; ++d) o[d] = 0.f;
+    }
+    if (DEC) {
+        const int64_t tok = U.tg * C::kGroup + a * kTileRows + r;
+        if (tok < prm.N) {
+            const float inv = 1.f / S.l;
+            uint4* dst = reinterpret_cast<uint4*>(prm.Y + (U.bh * prm.N + tok) * D);
+#pragma unroll
+            for (int k = 0; k < D / 8; ++k) {
+                uint4 v;
+                v.x = pack_bf16(o[8 * k + 0] * inv, o[8 * k + 1] * inv);
+                v.y = pack_bf16(o[8 * k + 2] * inv, o[8 * k + 3] * inv);
+                v.z = pack_bf16(o[8 * k + 4] * inv, o[8 * k + 5] * inv);
+                v.w = pack_bf16(o[8 * k + 6] * inv, o[8 * k + 7] * inv);
+                dst[k] = v;
+            }
+        }
+    } else {
+        const int64_t route = U.g * C::kGroup + a * kTileRows + r;
+        if (route < prm.M) {
+            const int64_t idx = (U.bh * (prm.nchunk * 4) + U.chunk * 4 + par) * prm.M + route;
+            prm.pmax[idx] = S.cnt > 0 ? S.m : -INFINITY;
+            prm.psum[idx] = S.l;
+            float4* dst = reinterpret_cast<float4*>(prm.pacc + idx * D);
+#pragma unroll
+            for (int k = 0; k < D / 4; ++k)
+                dst[k] = make_float4(o[4 * k], o[4 * k + 1], o[4 * k + 2], o[4 * k + 3]);
+        }
+    }
+    return true;
+}
+
+// PV of stream s: O_s (+)= P_s * C-tile of ring stage `st` (one elected lane issues).
+template <int D>
+__device__ __forceinline__ void issue_pv(uint32_t tmem, uint8_t* ring, int s, int st, int npv) {
+    using C = Cfg<D>;
+    const uint32_t cb = smem_u32(ring + st * C::kStage + C::kItemTile);
+#pragma unroll
+    for (int k = 0; k < kItem / 16; ++k) {
+        const uint64_t bd = smem_desc(cb + k * 16 * D * 2, C::kItemTile, C::kSBO, C::kSwz);
+        if (elect_one())
+            mma_ts(tmem + C::kColO + s * D, tmem + C::kColS + s * kItem + 8 * k, bd, C::kIdescPV,
+                   (npv > 0 || k > 0) ? 1u : 0u);
+        __syncwarp();
+    }
+}
+
+// ------------------------------------------------------------------ the kernel
 
 template <int D, bool DEC>
 __global__ void __launch_bounds__(kThreads, 1)
     tc_chain_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
                     const __grid_constant__ CUtensorMap tmC, const TcParams prm) {
     using C = Cfg<D>;
+    constexpr int NS = C::NS;
     extern __shared__ uint8_t smem_raw[];
     uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                                ~static_cast<uintptr_t>(1023));
-    uint8_t* abuf = smem;
-    uint8_t* ring = smem + 2 * C::kABytes;
+    uint8_t* abuf = smem;                   // 2 x NS unswizzled A tiles
+    uint8_t* ring = smem + 2 * C::kABytes;  // kStages x (B tile, C tile), swizzled
     uint64_t* bars = reinterpret_cast<uint64_t*>(ring + C::kStages * C::kStage);
     uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + C::kNumBars);
     volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
 
-    const uint32_t bar0 = smem_u32(bars);
-    auto full_bar = [&](int st) { return bar0 + 8u * st; };
-    auto empty_bar = [&](int st) { return bar0 + 8u * (C::kStages + st); };
-    auto afull_bar = [&](int b) { return bar0 + 8u * (2 * C::kStages + b); };
-    auto aempty_bar = [&](int b) { return bar0 + 8u * (2 * C::kStages + 2 + b); };
-    auto sready_bar = [&](int s) { return bar0 + 8u * (2 * C::kStages + 4 + s); };
-    auto pready_bar = [&](int s) { return bar0 + 8u * (2 * C::kStages + 8 + s); };
+    const uint32_t full0 = smem_u32(bars);
+    const uint32_t empty0 = full0 + 8u * C::kStages;
+    const uint32_t asfull0 = full0 + 8u * (2 * C::kStages);
+    const uint32_t asempty0 = asfull0 + 16u;
+    const uint32_t aready0 = asfull0 + 32u;
+    const uint32_t afree0 = asfull0 + 48u;
+    const uint32_t sready0 = asfull0 + 64u;
+    const uint32_t pready0 = sready0 + 8u * NS;
 
     const int warp = threadIdx.x >> 5;
     const int lane = threadIdx.x & 31;
 
     if (threadIdx.x == 0) {
         for (int st = 0; st < C::kStages; ++st) {
-            mbar_init(full_bar(st), 1);
-            mbar_init(empty_bar(st), 1);
+            mbar_init(full0 + 8u * st, 1);
+            mbar_init(empty0 + 8u * st, NS);
         }
         for (int b = 0; b < 2; ++b) {
-            mbar_init(afull_bar(b), 1);
-            mbar_init(aempty_bar(b), 1);
+            mbar_init(asfull0 + 8u * b, 1);
+            mbar_init(asempty0 + 8u * b, 256);
+            mbar_init(aready0 + 8u * b, 256);
+            mbar_init(afree0 + 8u * b, NS);
         }
-        for (int s = 0; s < 4; ++s) {
-            mbar_init(sready_bar(s), 1);
-            mbar_init(pready_bar(s), 128);
+        for (int s = 0; s < NS; ++s) {
+            mbar_init(sready0 + 8u * s, 1);
+            mbar_init(pready0 + 8u * s, 128);
         }
         *abort_flag = 0;
         fence_mbar_init();
@@ -213,27 +472,30 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (lane == 0) {
             uint32_t it = 0, ua = 0;
             for (int64_t u = blockIdx.x; u < prm.n_units; u += gridDim.x) {
-                const Unit U = get_unit<DEC>(prm, u);
+                const Unit U = get_unit<D, DEC>(prm, u);
                 const int ab = ua & 1;
-                if (!wait_bar(aempty_bar(ab), ((ua >> 1) & 1) ^ 1, abort_flag, prm.status)) break;
-                mbar_expect_tx(afull_bar(ab), U.n_a * C::kATile);
+                if (!wait_bar(asempty0 + 8u * ab, ((ua >> 1) & 1) ^ 1, abort_flag, prm.status))
+                    break;
+                mbar_expect_tx(asfull0 + 8u * ab, U.n_a * C::kATile);
                 for (int a = 0; a < U.n_a; ++a)
                     tma_load_3d(smem_u32(abuf + ab * C::kABytes + a * C::kATile), &tmA, 0,
-                                U.rowA0 + a * kTileRows, U.zA, afull_bar(ab));
+                                U.rowA0 + a * kTileRows, U.zA, asfull0 + 8u * ab);
                 ++ua;
                 bool ok = true;
                 for (int i = 0; i < U.n_items; ++i) {
                     const int st = it % C::kStages;
-                    if (!wait_bar(empty_bar(st), ((it / C::kStages) & 1) ^ 1, abort_flag,
+                    if (!wait_bar(empty0 + 8u * st, ((it / C::kStages) & 1) ^ 1, abort_flag,
                                   prm.status)) {
                         ok = false;
                         break;
                     }
-                    mbar_expect_tx(full_bar(st), C::kStage);
+                    mbar_expect_tx(full0 + 8u * st, C::kStage);
                     const int row = (int)(U.item0 + (int64_t)i * kItem);
                     const uint32_t dst = smem_u32(ring + st * C::kStage);
-                    tma_load_3d(dst, &tmB, 0, row, U.zB, full_bar(st));
-                    tma_load_3d(dst + C::kItemTile, &tmC, 0, row, U.zB, full_bar(st));
+                    tma_load_3d(dst, &tmB, 0, row, U.zB, full0 + 8u * st);
+                    tma_load_3d(dst + C::kItemTile, &tmC, 0, row, U.zB, full0 + 8u * st);
+                    // streams that do not consume this item count as having released it
+                    for (int x = U.n_a; x < NS; ++x) mbar_arrive(empty0 + 8u * st);
                     ++it;
                 }
                 if (!ok) break;
@@ -245,278 +507,160 @@ __global__ void __launch_bounds__(kThreads, 1)
                 for (int st = 0; st < C::kStages; ++st) {
                     if ((uint32_t)st >= it) break;
                     const uint32_t x = it - 1 - ((it - 1 - st) % C::kStages);
-                    while (!mbar_try_wait(full_bar(st), (x / C::kStages) & 1) &&
+                    while (!mbar_try_wait(full0 + 8u * st, (x / C::kStages) & 1) &&
                            globaltimer_ns() - t0 < kWaitLimitNs) {
                     }
                 }
                 for (int b = 0; b < 2; ++b) {
                     if ((uint32_t)b >= ua) break;
                     const uint32_t y = ua - 1 - ((ua - 1 - b) % 2);
-                    while (!mbar_try_wait(afull_bar(b), (y >> 1) & 1) &&
+                    while (!mbar_try_wait(asfull0 + 8u * b, (y >> 1) & 1) &&
                            globaltimer_ns() - t0 < kWaitLimitNs) {
                     }
                 }
             }
         }
-    } else if (warp == 1) {
-        // ------------------------------------------------------------ MMA issuer
-        if (lane == 0) {
-            uint32_t it = 0, ua = 0;
-            uint32_t pcnt[4] = {0, 0, 0, 0};
+    } else if (warp < kFirstSoftmaxWarp) {
+        // ------------------------------------------------------------ MMA warps
+        // Warp 1 + s drives stream s. For each of its items: the PV of its previous item
+        // (P from TMEM, V or Z from the ring), the S of this item (A from TMEM, K or Q from
+        // the ring) and one commit, which the softmax waits on. It observes the full
+        // barrier of every ring item in order, so each parity test names one phase.
+        const int s = warp - kFirstMmaWarp;
+        if (s < NS) {
+            uint32_t it = 0, ua = 0, pcnt = 0;
             bool ok = true;
             for (int64_t u = blockIdx.x; u < prm.n_units && ok; u += gridDim.x, ++ua) {
-                const Unit U = get_unit<DEC>(prm, u);
+                const Unit U = get_unit<D, DEC>(prm, u);
                 const int ab = ua & 1;
-                if (!wait_bar(afull_bar(ab), (ua >> 1) & 1, abort_flag, prm.status)) break;
+                if (!warp_wait(aready0 + 8u * ab, (ua >> 1) & 1, abort_flag, prm.status)) break;
                 tc_fence_after();
-                const uint32_t a_base = smem_u32(abuf + ab * C::kABytes);
-                int prev_st[4] = {-1, -1, -1, -1};
-                int npv[4] = {0, 0, 0, 0};
-                int done[C::kStages];
-#pragma unroll
-                for (int st = 0; st < C::kStages; ++st) done[st] = 0;
-
-                auto issue_pv = [&](int s) {
-                    const uint32_t cb = smem_u32(ring + prev_st[s] * C::kStage + C::kItemTile);
-#pragma unroll
-                    for (int k = 0; k < kItem / 16; ++k) {
-                        const uint64_t bd = smem_desc(cb + k * 16 * D * 2, C::kItemTile, C::kSBO,
-                                                      C::kSwz);
-                        mma_ts(tmem + C::kOCol + s * D, tmem + s * kItem + 8 * k, bd,
-                               C::kIdescPV, (npv[s] > 0 || k > 0) ? 1u : 0u);
-                    }
-                    ++npv[s];
-                    if (++done[prev_st[s]] == U.n_a) {
-                        done[prev_st[s]] = 0;
-                        mma_commit(empty_bar(prev_st[s]));
-                    }
-                };
-
-                for (int i = 0; i < U.n_items && ok; ++i, ++it) {
+                const int a = s % U.n_a;
+                const int par = s / U.n_a;
+                const uint32_t a_tmem = tmem + C::kColA + (ab * NS + a) * (D / 2);
+                int prev = -1, npv = 0;
+                for (int i = 0; i < U.n_items; ++i, ++it) {
                     const int st = it % C::kStages;
-                    const uint32_t bb = smem_u32(ring + st * C::kStage);
-                    bool have_item = false;
-                    for (int a = 0; a < U.n_a; ++a) {
-                        const int s = a + U.n_a * (i % U.n_par);
-                        // the stream's previous PV first: it may free the stage item i needs
-                        if (prev_st[s] >= 0) {
-                            if (!wait_bar(pready_bar(s), pcnt[s] & 1, abort_flag, prm.status)) {
-                                ok = false;
-                                break;
-                            }
-                            ++pcnt[s];
-                            tc_fence_after();
-                            issue_pv(s);
+                    const bool mine = (i % U.n_par) == par;
+                    if (mine && prev >= 0) {
+                        if (!warp_wait(pready0 + 8u * s, pcnt & 1, abort_flag, prm.status)) {
+                            ok = false;
+                            break;
                         }
-                        if (!have_item) {
-                            if (!wait_bar(full_bar(st), (it / C::kStages) & 1, abort_flag,
-                                          prm.status)) {
-                                ok = false;
-                                break;
-                            }
-                            tc_fence_after();
-                            have_item = true;
-                        }
-                        const uint32_t ab_tile = a_base + a * C::kATile;
-#pragma unroll
-                        for (int k = 0; k < D / 16; ++k) {
-                            const uint64_t ad = smem_desc(ab_tile + 32 * k, 16, C::kSBO, C::kSwz);
-                            const uint64_t bd = smem_desc(bb + 32 * k, 16, C::kSBO, C::kSwz);
-                            mma_ss(tmem + s * kItem, ad, bd, C::kIdescS, k > 0 ? 1u : 0u);
-                        }
-                        mma_commit(sready_bar(s));
-                        prev_st[s] = st;
+                        ++pcnt;
+                        tc_fence_after();
+                        issue_pv<D>(tmem, ring, s, prev, npv);
+                        ++npv;
                     }
-                }
-                // drain: the last PV of every stream, then the final s_ready (O complete)
-                for (int s = 0; s < 4 && ok; ++s) {
-                    if (prev_st[s] < 0) continue;
-                    if (!wait_bar(pready_bar(s), pcnt[s] & 1, abort_flag, prm.status)) {
+                    if (!warp_wait(full0 + 8u * st, (it / C::kStages) & 1, abort_flag,
+                                   prm.status)) {
                         ok = false;
                         break;
                     }
-                    ++pcnt[s];
+                    if (!mine) continue;
                     tc_fence_after();
-                    issue_pv(s);
-                    mma_commit(sready_bar(s));
+                    const uint32_t bb = smem_u32(ring + st * C::kStage);
+#pragma unroll
+                    for (int k = 0; k < D / 16; ++k) {
+                        const uint64_t bd = smem_desc(bb + 32 * k, 16, C::kSBO, C::kSwz);
+                        if (elect_one())
+                            mma_ts(tmem + C::kColS + s * kItem, a_tmem + 8 * k, bd, C::kIdescS,
+                                   k > 0 ? 1u : 0u);
+                        __syncwarp();
+                    }
+                    if (elect_one()) mma_commit(sready0 + 8u * s);
+                    __syncwarp();
+                    prev = st;
                 }
-                mma_commit(aempty_bar(ab));
+                if (!ok) break;
+                if (prev >= 0) {  // the last PV of the stream, then the final s_ready
+                    if (!warp_wait(pready0 + 8u * s, pcnt & 1, abort_flag, prm.status)) break;
+                    ++pcnt;
+                    tc_fence_after();
+                    issue_pv<D>(tmem, ring, s, prev, npv);
+                    if (elect_one()) mma_commit(sready0 + 8u * s);
+                    __syncwarp();
+                }
+                // this stream's MMAs no longer read the unit's A buffer
+                if (elect_one()) mma_commit(afree0 + 8u * ab);
+                __syncwarp();
             }
         }
     } else {
         // ------------------------------------------------------------ softmax warpgroups
-        const int wg = (warp - 2) >> 2;
+        const int wg = (warp - kFirstSoftmaxWarp) >> 2;
         const int q = warp & 3;
         const int r = q * 32 + lane;
         const uint32_t lane_off = static_cast<uint32_t>(q * 32) << 16;
+        const bool wg_leader = ((warp - kFirstSoftmaxWarp) & 3) == 0 && lane == 0;
         const float c = prm.c;
-        uint32_t scnt[2] = {0, 0};
+        const uint64_t c2 = pack_f32x2(c, c);
+        SoftmaxStream st0, st1;
+        st0.s = wg;
+        st1.s = wg + 2;  // used when NS == 4
+        st0.scnt = st1.scnt = 0;
         bool alive = true;
-        for (int64_t u = blockIdx.x; u < prm.n_units && alive; u += gridDim.x) {
-            const Unit U = get_unit<DEC>(prm, u);
-            int cnt[2], sid[2];
-            float m[2], l[2];
-            int j[2] = {0, 0};
+        uint32_t ua = 0, it0 = 0;
+        for (int64_t u = blockIdx.x; u < prm.n_units && alive; u += gridDim.x, ++ua) {
+            const Unit U = get_unit<D, DEC>(prm, u);
+            const int ab = ua & 1;
+            // copy this warpgroup's A tiles (one row per thread) from smem into TMEM, once
+            // the MMAs of the unit that last used this TMEM buffer are complete
+            if (!warp_wait(asfull0 + 8u * ab, (ua >> 1) & 1, abort_flag, prm.status)) break;
+            if (!warp_wait(afree0 + 8u * ab, ((ua >> 1) & 1) ^ 1, abort_flag, prm.status)) break;
+            tc_fence_after();
+            for (int a = 0; a < U.n_a; ++a) {
+                const int writer = U.n_a == 1 ? 0 : (a & 1);
+                if (writer != wg) continue;
+                const uint4* src = reinterpret_cast<const uint4*>(abuf + ab * C::kABytes +
+                                                                  a * C::kATile + r * D * 2);
+                uint32_t v[D / 2];
 #pragma unroll
-            for (int sl = 0; sl < 2; ++sl) {
-                sid[sl] = wg + 2 * sl;
-                const int par = sid[sl] / U.n_a;
-                cnt[sl] = U.n_items > par ? (U.n_items - par + U.n_par - 1) / U.n_par : 0;
-                m[sl] = -INFINITY;
-                l[sl] = 0.f;
-            }
-            while (alive && (j[0] < cnt[0] || j[1] < cnt[1])) {
-#pragma unroll
-                for (int sl = 0; sl < 2; ++sl) {
-                    if (j[sl] >= cnt[sl] || !alive) continue;
-                    const int s = sid[sl];
-                    const bool got = wait_bar(sready_bar(s), scnt[sl] & 1, abort_flag, prm.status);
-                    ++scnt[sl];
-                    if (!__all_sync(0xffffffffu, got)) {
-                        alive = false;
-                        continue;
-                    }
-                    tc_fence_after();
-                    const int item = (s / U.n_a) + j[sl] * U.n_par;
-                    const int64_t start = U.item0 + (int64_t)item * kItem;
-                    const int nv = (int)min((int64_t)kItem, U.item_end - start);
-                    const uint32_t scol = tmem + lane_off + s * kItem;
-                    uint32_t sr[kItem];
-#pragma unroll
-                    for (int k = 0; k < kItem / 16; ++k) tmem_ld16(scol + 16 * k, sr + 16 * k);
-                    tmem_wait_ld();
-                    float mx;
-                    if (nv == kItem) {
-                        float a0 = __uint_as_float(sr[0]), a1 = __uint_as_float(sr[1]);
-                        float a2 = __uint_as_float(sr[2]), a3 = __uint_as_float(sr[3]);
-#pragma unroll
-                        for (int k = 4; k < kItem; k += 4) {
-                            a0 = fmaxf(a0, __uint_as_float(sr[k]));
-                            a1 = fmaxf(a1, __uint_as_float(sr[k + 1]));
-                            a2 = fmaxf(a2, __uint_as_float(sr[k + 2]));
-                            a3 = fmaxf(a3, __uint_as_float(sr[k + 3]));
-                        }
-                        mx = fmaxf(fmaxf(a0, a1), fmaxf(a2, a3));
-                    } else {
-                        mx = -INFINITY;
-#pragma unroll
-                        for (int k = 0; k < kItem; ++k)
-                            if (k < nv) mx = fmaxf(mx, __uint_as_float(sr[k]));
-                    }
-                    const float cand = mx * c;
-                    bool need = false;
-                    float alpha = 1.f;
-                    if (cand > m[sl] + kLazyTau) {
-                        alpha = ex2(m[sl] - cand);  // 0 on the first item
-                        need = j[sl] > 0;
-                        l[sl] *= alpha;
-                        m[sl] = cand;
-                    }
-                    if (__any_sync(0xffffffffu, need)) {
-                        const uint32_t ocol = tmem + lane_off + C::kOCol + s * D;
-                        const float f = need ? alpha : 1.f;
-#pragma unroll
-                        for (int k = 0; k < D / 16; ++k) {
-                            uint32_t o[16];
-                            tmem_ld16(ocol + 16 * k, o);
-                            tmem_wait_ld();
-#pragma unroll
-                            for (int e = 0; e < 16; ++e)
-                                o[e] = __float_as_uint(__uint_as_float(o[e]) * f);
-                            tmem_st16(ocol + 16 * k, o);
-                        }
-                    }
-                    const float nm = -m[sl];
-                    float sum0 = 0.f, sum1 = 0.f;
-                    uint32_t pr[kItem / 2];
-                    if (nv == kItem) {
-#pragma unroll
-                        for (int k = 0; k < kItem / 2; ++k) {
-                            const float p0 = ex2(fmaf(__uint_as_float(sr[2 * k]), c, nm));
-                            const float p1 = ex2(fmaf(__uint_as_float(sr[2 * k + 1]), c, nm));
-                            sum0 += p0;
-                            sum1 += p1;
-                            pr[k] = pack_bf16(p0, p1);
-                        }
-                    } else {
-#pragma unroll
-                        for (int k = 0; k < kItem / 2; ++k) {
-                            float p0 = ex2(fmaf(__uint_as_float(sr[2 * k]), c, nm));
-                            float p1 = ex2(fmaf(__uint_as_float(sr[2 * k + 1]), c, nm));
-                            p0 = (2 * k < nv) ? p0 : 0.f;
-                            p1 = (2 * k + 1 < nv) ? p1 : 0.f;
-                            sum0 += p0;
-                            sum1 += p1;
-                            pr[k] = pack_bf16(p0, p1);
-                        }
-                    }
-                    l[sl] += sum0 + sum1;
-                    tmem_st16(scol, pr);
-                    tmem_st16(scol + 16, pr + 16);
-                    tmem_wait_st();
-                    tc_fence_before();
-                    mbar_arrive(pready_bar(s));
-                    ++j[sl];
+                for (int k = 0; k < D / 8; ++k) {
+                    const uint4 x = src[k];
+                    v[4 * k] = x.x;
+                    v[4 * k + 1] = x.y;
+                    v[4 * k + 2] = x.z;
+                    v[4 * k + 3] = x.w;
                 }
-            }
-            // results of the unit
-#pragma unroll
-            for (int sl = 0; sl < 2; ++sl) {
-                if (!alive) break;
-                const int s = sid[sl];
-                const int a = s % U.n_a;
-                const int par = s / U.n_a;
-                float o[D];
-                if (cnt[sl] > 0) {
-                    const bool got = wait_bar(sready_bar(s), scnt[sl] & 1, abort_flag, prm.status);
-                    ++scnt[sl];
-                    if (!__all_sync(0xffffffffu, got)) {
-                        alive = false;
-                        break;
-                    }
-                    tc_fence_after();
-                    const uint32_t ocol = tmem + lane_off + C::kOCol + s * D;
-#pragma unroll
-                    for (int k = 0; k < D / 16; ++k) {
-                        uint32_t t[16];
-                        tmem_ld16(ocol + 16 * k, t);
-                        tmem_wait_ld();
-#pragma unroll
-                        for (int e = 0; e < 16; ++e) o[16 * k + e] = __uint_as_float(t[e]);
-                    }
+                const uint32_t acol = tmem + lane_off + C::kColA + (ab * NS + a) * (D / 2);
+                if (D == 16) {
+                    tmem_st8(acol, v);
                 } else {
 #pragma unroll
-                    for (int d = 0; d < D; ++d) o[d] = 0.f;
-                }
-                if (DEC) {
-                    const int64_t tok = U.tg * kGroup + a * kTileRows + r;
-                    if (tok < prm.N) {
-                        const float inv = 1.f / l[sl];
-                        uint4* dst = reinterpret_cast<uint4*>(prm.Y + (U.bh * prm.N + tok) * D);
-#pragma unroll
-                        for (int k = 0; k < D / 8; ++k) {
-                            uint4 v;
-                            v.x = pack_bf16(o[8 * k + 0] * inv, o[8 * k + 1] * inv);
-                            v.y = pack_bf16(o[8 * k + 2] * inv, o[8 * k + 3] * inv);
-                            v.z = pack_bf16(o[8 * k + 4] * inv, o[8 * k + 5] * inv);
-                            v.w = pack_bf16(o[8 * k + 6] * inv, o[8 * k + 7] * inv);
-                            dst[k] = v;
-                        }
-                    }
-                } else {
-                    const int64_t route = U.g * kGroup + a * kTileRows + r;
-                    if (route < prm.M) {
-                        const int64_t idx =
-                            (U.bh * (prm.nchunk * 4) + U.chunk * 4 + par) * prm.M + route;
-                        prm.pmax[idx] = cnt[sl] > 0 ? m[sl] : -INFINITY;
-                        prm.psum[idx] = l[sl];
-                        float4* dst = reinterpret_cast<float4*>(prm.pacc + idx * D);
-#pragma unroll
-                        for (int k = 0; k < D / 4; ++k)
-                            dst[k] = make_float4(o[4 * k], o[4 * k + 1], o[4 * k + 2], o[4 * k + 3]);
-                    }
+                    for (int k = 0; k < D / 32; ++k) tmem_st16(acol + 16 * k, v + 16 * k);
                 }
             }
+            tmem_wait_st();
+            tc_fence_before();
+            mbar_arrive(aready0 + 8u * ab);
+            mbar_arrive(asempty0 + 8u * ab);
+
+            st0.begin(U);
+            if (NS == 4) st1.begin(U);
+            while (alive && (st0.j < st0.cnt || (NS == 4 && st1.j < st1.cnt))) {
+                if (st0.j < st0.cnt) {
+                    const int item = st0.s / U.n_a + st0.j * U.n_par;
+                    alive = softmax_step<D>(st0, U, tmem, lane_off, c, c2, sready0 + 8u * st0.s,
+                                            pready0 + 8u * st0.s, empty0, wg_leader,
+                                            (int)((it0 + item) % C::kStages), abort_flag,
+                                            prm.status);
+                }
+                if (NS == 4 && alive && st1.j < st1.cnt) {
+                    const int item = st1.s / U.n_a + st1.j * U.n_par;
+                    alive = softmax_step<D>(st1, U, tmem, lane_off, c, c2, sready0 + 8u * st1.s,
+                                            pready0 + 8u * st1.s, empty0, wg_leader,
+                                            (int)((it0 + item) % C::kStages), abort_flag,
+                                            prm.status);
+                }
+            }
+            if (alive)
+                alive = finish_stream<D, DEC>(st0, U, prm, tmem, lane_off, r, sready0 + 8u * st0.s,
+                                              empty0, wg_leader, abort_flag);
+            if (NS == 4 && alive)
+                alive = finish_stream<D, DEC>(st1, U, prm, tmem, lane_off, r, sready0 + 8u * st1.s,
+                                              empty0, wg_leader, abort_flag);
+            it0 += U.n_items;
         }
     }
 
@@ -545,19 +689,21 @@ PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
     return fn;
 }
 
-// 3D bf16 map over [z, rows, D] (D innermost) with a box of box_rows x D and the swizzle
-// that matches one D-wide row.
+// 3D bf16 map over [z, rows, D] (D innermost) with a box of box_rows x D. `swizzled` picks
+// the swizzle matching one D-wide row (MMA operand tiles); otherwise rows are stored plain
+// (A tiles, which the softmax threads copy into TMEM row by row).
 bool make_map(CUtensorMap* m, const void* base, int64_t D, int64_t rows, int64_t z,
-              uint32_t box_rows) {
+              uint32_t box_rows, bool swizzled) {
     auto fn = encode_fn();
     if (!fn) return false;
     cuuint64_t dims[3] = {(cuuint64_t)D, (cuuint64_t)rows, (cuuint64_t)z};
     cuuint64_t strides[2] = {(cuuint64_t)(D * 2), (cuuint64_t)(rows * D * 2)};
     cuuint32_t box[3] = {(cuuint32_t)D, box_rows, 1};
     cuuint32_t estr[3] = {1, 1, 1};
-    const CUtensorMapSwizzle sw = D == 16 ? CU_TENSOR_MAP_SWIZZLE_32B
-                                  : D == 32 ? CU_TENSOR_MAP_SWIZZLE_64B
-                                            : CU_TENSOR_MAP_SWIZZLE_128B;
+    CUtensorMapSwizzle sw = CU_TENSOR_MAP_SWIZZLE_NONE;
+    if (swizzled)
+        sw = D == 16 ? CU_TENSOR_MAP_SWIZZLE_32B
+                     : (D == 32 ? CU_TENSOR_MAP_SWIZZLE_64B : CU_TENSOR_MAP_SWIZZLE_128B);
     return fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(base), dims, strides, box,
               estr, CU_TENSOR_MAP_INTERLEAVE_NONE, sw, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
               CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
@@ -591,6 +737,8 @@ cudaError_t launch_d(int64_t D, const CUtensorMap& a, const CUtensorMap& b, cons
 
 }  // namespace
 
+int64_t tc_group_rows(int64_t D) { return (D == 64 ? 2 : 4) * kTileRows; }
+
 cudaError_t tc_encode(const Plan& p, int call, const void* k, const void* v, const void* seeds,
                       float scale, char* ws, cudaStream_t st) {
     CUtensorMap ma, mb, mc;
@@ -604,8 +752,9 @@ cudaError_t tc_encode(const Plan& p, int call, const void* k, const void* v, con
         a_src = ws + p.off_qop;
         a_z = p.BH;
     }
-    if (!make_map(&ma, a_src, p.D, p.M, a_z, kTileRows) || !make_map(&mb, k, p.D, p.N, p.BH, kItem) ||
-        !make_map(&mc, v, p.D, p.N, p.BH, kItem))
+    if (!make_map(&ma, a_src, p.D, p.M, a_z, kTileRows, false) ||
+        !make_map(&mb, k, p.D, p.N, p.BH, kItem, true) ||
+        !make_map(&mc, v, p.D, p.N, p.BH, kItem, true))
         return cudaErrorInvalidValue;
     TcParams prm{};
     prm.BH = p.BH;
@@ -628,9 +777,9 @@ cudaError_t tc_encode(const Plan& p, int call, const void* k, const void* v, con
 cudaError_t tc_decode(const Plan& p, const void* K, float scale, void* Y, char* ws,
                       cudaStream_t st) {
     CUtensorMap ma, mb, mc;
-    if (!make_map(&ma, K, p.D, p.N, p.BH, kTileRows) ||
-        !make_map(&mb, ws + p.off_qop, p.D, p.M, p.BH, kItem) ||
-        !make_map(&mc, ws + p.off_zop, p.D, p.M, p.BH, kItem))
+    if (!make_map(&ma, K, p.D, p.N, p.BH, kTileRows, false) ||
+        !make_map(&mb, ws + p.off_qop, p.D, p.M, p.BH, kItem, true) ||
+        !make_map(&mc, ws + p.off_zop, p.D, p.M, p.BH, kItem, true))
         return cudaErrorInvalidValue;
     TcParams prm{};
     prm.BH = p.BH;
@@ -638,7 +787,8 @@ cudaError_t tc_decode(const Plan& p, const void* K, float scale, void* Y, char* 
     prm.N = p.N;
     prm.M = p.M;
     prm.c = fabsf(scale) * kLog2e;
-    prm.n_tok_groups = (p.N + kGroup - 1) / kGroup;
+    const int64_t grp = tc_group_rows(p.D);
+    prm.n_tok_groups = (p.N + grp - 1) / grp;
     prm.Y = (__nv_bfloat16*)Y;
     prm.n_units = p.BH * prm.n_tok_groups;
     prm.status = (int*)(ws + p.off_status);
