@@ -12,20 +12,24 @@
 //     meets a stream of 64-route items (Q and Z tiles). Each token row keeps an online
 //     softmax over routes and writes its normalised row of Y.
 //
-// Work is cut into NS TMEM "streams" (NS = 4 for D <= 32, 2 for D = 64). Stream s owns a
-// 128 x 64 fp32 score tile S (rewritten in place as bf16 P, the A operand of the PV
-// product) and a 128 x D fp32 accumulator O, and reads one resident A tile kept in TMEM,
-// so that S = A * B^T is a TMEM x SMEM product. Roles (13 warps):
-//   warp 0        TMA producer: A tiles (unswizzled) and the item ring (swizzled K/V or Q/Z)
-//   warps 1..4    one MMA warp per stream: the PV of its previous item, the S of its next
-//                 item, one commit per item (a commit stalls only the warp that issues it)
-//   warps 5..12   two softmax warpgroups; warpgroup w serves streams w and w + 2 (NS = 4)
-//                 or stream w (NS = 2) and copies its A tiles from smem into TMEM
+// Work is cut into four TMEM "streams". Stream s owns B score buffers of 128 x kItem fp32
+// (kItem = 64 tokens or routes, 32 for D = 64; S is rewritten in place as bf16 P, the A
+// operand of the PV product) and a 128 x D fp32 accumulator O, and reads one resident A
+// tile kept in TMEM, so that S = A * B^T is a TMEM x SMEM product. The protocol supports
+// B = 2 (the MMA warp computes the S of item j+1 while the softmax works on item j); the
+// TMEM budget of four streams allows it only for 32-wide items, which measured slower
+// than single-buffered 64-wide items, so B = 1. Roles (20 warps):
+//   warps 0..3    one MMA warp per stream: for item j, the PV of item j-B and the S of
+//                 item j, then one commit (a commit stalls only the warp that issues it);
+//                 warp 0 also issues the TMA loads (A tiles, unswizzled; the item ring,
+//                 swizzled K/V or Q/Z) from a non-blocking poll between its own waits
+//   warps 4..19   four softmax warpgroups; warpgroup s serves stream s and copies its A tile
+//                 from smem into TMEM (four warps per SMSP hide each other's latencies)
 // The softmax keeps a reference max that is recomputed exactly only on a stream's first
 // item or when an item's probabilities sum past 2^48 (values stay far inside the fp32 and
 // bf16 ranges); otherwise P = 2^(c S - m) with the old reference.
 // Every wait is bounded (2 s of %globaltimer): on expiry the kernel records
-// FLAREPP_ERR_TIMEOUT in the status word, every role leaves its loops, the producer waits
+// FLAREPP_ERR_TIMEOUT in the status word, every role leaves its loops, the TMA issuer waits
 // for its copies in flight, and TMEM is freed.
 #include <cuda.h>
 #include <cudaTypedefs.h>
@@ -41,12 +45,11 @@ namespace {
 
 using namespace tc;
 
-constexpr int kWarps = 13;
+constexpr int kWarps = 20;
 constexpr int kThreads = kWarps * 32;
-constexpr int kFirstMmaWarp = 1;
-constexpr int kFirstSoftmaxWarp = 5;
+constexpr int kFirstSoftmaxWarp = 4;
+constexpr int NS = 4;           // TMEM streams
 constexpr int kTileRows = 128;  // TMEM lanes, MMA M
-constexpr int kItem = 64;       // streamed rows per item
 constexpr uint64_t kWaitLimitNs = 2000000000ull;
 constexpr uint32_t kTmemCols = 512;
 constexpr float kLog2e = 1.4426950408889634f;
@@ -55,9 +58,11 @@ constexpr float kFastLimit = 281474976710656.0f;  // 2^48
 
 template <int D>
 struct Cfg {
-    static constexpr int NS = D == 64 ? 2 : 4;        // streams
+    static constexpr int kItem = D == 64 ? 32 : 64;   // streamed rows per item
+    static constexpr int B = 1;                       // score buffers per stream (1 or 2)
+    static constexpr int kABuf = D == 64 ? 1 : 2;     // TMEM copies of the A tiles
     static constexpr int kGroup = NS * kTileRows;     // resident rows per work unit
-    static constexpr int kStages = 8;                 // a multiple of 4
+    static constexpr int kStages = D == 64 ? 8 : (kItem == 32 ? 16 : 8);  // multiple of 4
     static constexpr int kATile = kTileRows * D * 2;  // one 128-row operand tile
     static constexpr int kABytes = NS * kATile;
     static constexpr int kItemTile = kItem * D * 2;
@@ -65,8 +70,9 @@ struct Cfg {
     static constexpr uint32_t kSwz = D == 16 ? kSw32 : (D == 32 ? kSw64 : kSw128);
     static constexpr uint32_t kSBO = 8 * D * 2;  // bytes between 8-row groups
     // barriers: full[S], empty[S], asmem_full[2], asmem_empty[2], a_ready[2], a_free[2],
-    //           s_ready[NS], p_ready[NS]
-    static constexpr int kNumBars = 2 * kStages + 8 + 2 * NS;
+    //           s_ready[NS][2], p_ready[NS][2] (per score buffer: the four warps of a
+    //           softmax warpgroup can be one item apart, never two)
+    static constexpr int kNumBars = 2 * kStages + 8 + 4 * NS;
     static constexpr int kData = 2 * kABytes + kStages * kStage;
     static constexpr int kNeed = 1024 + kData + kNumBars * 8 + 16;
     // at least 120 KB so that one CTA owns an SM and its 512 TMEM columns
@@ -74,11 +80,16 @@ struct Cfg {
     static constexpr uint32_t kIdescS = idesc_bf16_f32(128, kItem, false, false);
     static constexpr uint32_t kIdescPV = idesc_bf16_f32(128, D, false, true);
     // TMEM columns
-    static constexpr uint32_t kColS = 0;               // NS x 64
-    static constexpr uint32_t kColO = NS * kItem;      // NS x D
-    static constexpr uint32_t kColA = kColO + NS * D;  // 2 buffers x NS tiles x D/2
-    static_assert(kColA + 2 * NS * (D / 2) <= kTmemCols, "TMEM budget");
+    static constexpr uint32_t kColS = 0;                  // NS x B x kItem
+    static constexpr uint32_t kColO = NS * B * kItem;     // NS x D
+    static constexpr uint32_t kColA = kColO + NS * D;     // kABuf x NS tiles x D/2
+    static_assert(kColA + kABuf * NS * (D / 2) <= kTmemCols, "TMEM budget");
     static_assert(kSmem <= 232448, "shared memory budget");
+    // s_ready phases buffer b receives in a unit where the stream has cnt items: one per
+    // k in [0, cnt + B - 1] with k % B == b (k >= cnt are the closing commits)
+    __device__ static __forceinline__ uint32_t phases(int cnt, int b) {
+        return cnt > 0 ? (uint32_t)((cnt + B - 1 - b) / B + 1) : 0u;
+    }
 };
 
 struct TcParams {
@@ -96,7 +107,6 @@ struct TcParams {
 };
 
 // route tiles of encode group g, rounded up to 1, 2 or 4 (a divisor of the stream count)
-template <int NS>
 __device__ __forceinline__ int na_of_group(int64_t M, int64_t g) {
     const int64_t rem = M - g * NS * kTileRows;
     const int64_t tiles = rem >= NS * kTileRows ? NS : (rem + kTileRows - 1) / kTileRows;
@@ -121,7 +131,7 @@ __device__ __forceinline__ Unit get_unit(const TcParams& p, int64_t u) {
         U.g = 0;
         U.zA = (int)U.bh;
         U.rowA0 = (int)(U.tg * C::kGroup);
-        U.n_a = C::NS;
+        U.n_a = NS;
         U.n_par = 1;
         U.item0 = 0;
         U.item_end = p.M;
@@ -133,13 +143,13 @@ __device__ __forceinline__ Unit get_unit(const TcParams& p, int64_t u) {
         U.tg = 0;
         U.zA = (int)(p.a_per_head ? U.bh % p.H : U.bh);
         U.rowA0 = (int)(U.g * C::kGroup);
-        U.n_a = na_of_group<C::NS>(p.M, U.g);
-        U.n_par = C::NS / U.n_a;
+        U.n_a = na_of_group(p.M, U.g);
+        U.n_par = NS / U.n_a;
         U.item0 = U.chunk * p.chunk_len;
         U.item_end = min(p.N, U.item0 + p.chunk_len);
     }
     U.zB = (int)U.bh;
-    U.n_items = (int)((U.item_end - U.item0 + kItem - 1) / kItem);
+    U.n_items = (int)((U.item_end - U.item0 + C::kItem - 1) / C::kItem);
     return U;
 }
 
@@ -185,15 +195,13 @@ struct SoftmaxStream {
     int s;          // stream index
     int cnt, j;     // items of the stream in this unit, items done
     float m, l;     // reference max (base 2, scaled) and running sum
-    uint32_t scnt;  // s_ready phases consumed so far (across units)
-    int prev_st;    // ring stage of the previous item (-1: none)
+    uint32_t ph0, ph1;  // s_ready phases of buffers 0 and 1 completed in earlier units
     __device__ __forceinline__ void begin(const Unit& U) {
         const int par = s / U.n_a;
         cnt = U.n_items > par ? (U.n_items - par + U.n_par - 1) / U.n_par : 0;
         j = 0;
         m = -INFINITY;
         l = 0.f;
-        prev_st = -1;
     }
 };
 
@@ -249,12 +257,14 @@ __device__ __forceinline__ float exp_half(const uint32_t* sr, uint32_t* pr, int 
     return t0 + t1;
 }
 
-// P for the whole 64-column tile at TMEM column scol (S is read half by half).
+// P for a whole item tile of ITEM columns at TMEM column scol (S is read 32 columns at a
+// time); packed bf16 pairs go to pr[0 .. ITEM/2). Returns the row sum.
+template <int ITEM>
 __device__ __forceinline__ float exp_tile(uint32_t scol, uint32_t* pr, int nv, float c,
                                           uint64_t c2, float m) {
     float sum = 0.f;
 #pragma unroll
-    for (int h = 0; h < 2; ++h) {
+    for (int h = 0; h < ITEM / 32; ++h) {
         uint32_t sr[32];
         tmem_ld32(scol + 32 * h, sr);
         tmem_wait_ld32(sr);
@@ -263,38 +273,43 @@ __device__ __forceinline__ float exp_tile(uint32_t scol, uint32_t* pr, int nv, f
     return sum;
 }
 
-// One item of one stream for this thread's row: read S, update the online softmax, write P
-// back over S, signal the stream's MMA warp. Once S is ready the stream's previous PV has
-// completed, so the warpgroup leader also frees the ring stage of the previous item.
-// Returns false when the kernel is aborting.
+// One item of this warpgroup's stream for this thread's row: read S, update the online
+// softmax, write P back over S, signal the stream's MMA warp. S of item j being ready
+// means the PV of item j - B has completed, so the warpgroup leader frees that item's ring
+// stage. Returns false when the kernel is aborting.
 template <int D>
 __device__ __forceinline__ bool softmax_step(SoftmaxStream& S, const Unit& U, uint32_t tmem,
                                              uint32_t lane_off, float c, uint64_t c2,
-                                             uint32_t sready, uint32_t pready, uint32_t empty0,
-                                             bool wg_leader, int stage, volatile int* abort_flag,
-                                             int* status) {
+                                             uint32_t sready_s, uint32_t pready_s, uint32_t empty0,
+                                             bool wg_leader, uint32_t it0,
+                                             volatile int* abort_flag, int* status) {
     using C = Cfg<D>;
-    if (!warp_wait(sready, S.scnt & 1, abort_flag, status)) return false;
-    ++S.scnt;
+    const int j = S.j;
+    const int b = j % C::B;
+    const uint32_t par_j = ((b == 0 ? S.ph0 : S.ph1) + (uint32_t)(j / C::B)) & 1u;
+    if (!warp_wait(sready_s + 8u * b, par_j, abort_flag, status)) return false;
     tc_fence_after();
-    if (wg_leader && S.prev_st >= 0) mbar_arrive(empty0 + 8u * S.prev_st);
-    S.prev_st = stage;
-    const int item = S.s / U.n_a + S.j * U.n_par;
-    const int64_t start = U.item0 + (int64_t)item * kItem;
-    const int nv = (int)min((int64_t)kItem, U.item_end - start);
-    const uint32_t scol = tmem + lane_off + C::kColS + S.s * kItem;
-    uint32_t pr[kItem / 2];
+    const int par = S.s / U.n_a;
+    if (wg_leader && j >= C::B) {
+        const int i_old = par + (j - C::B) * U.n_par;
+        mbar_arrive(empty0 + 8u * ((it0 + i_old) % C::kStages));
+    }
+    const int item = par + j * U.n_par;
+    const int64_t start = U.item0 + (int64_t)item * C::kItem;
+    const int nv = (int)min((int64_t)C::kItem, U.item_end - start);
+    const uint32_t scol = tmem + lane_off + C::kColS + (S.s * C::B + b) * C::kItem;
+    uint32_t pr[C::kItem / 2];
     float sum = 0.f;
-    bool slow = S.j == 0;
+    bool slow = j == 0;
     if (!slow) {
-        sum = exp_tile(scol, pr, nv, c, c2, S.m);
+        sum = exp_tile<C::kItem>(scol, pr, nv, c, c2, S.m);
         slow = __any_sync(0xffffffffu, !(sum <= kFastLimit));
     }
     if (slow) {
         // exact max of this item (S is still intact in TMEM: P has not been written yet)
         float mx = -INFINITY;
 #pragma unroll
-        for (int h = 0; h < 2; ++h) {
+        for (int h = 0; h < C::kItem / 32; ++h) {
             uint32_t sr[32];
             tmem_ld32(scol + 32 * h, sr);
             tmem_wait_ld32(sr);
@@ -305,11 +320,19 @@ __device__ __forceinline__ bool softmax_step(SoftmaxStream& S, const Unit& U, ui
         float alpha = 1.f;
         if (cand > S.m) {
             alpha = ex2(S.m - cand);  // 0 when S.m is -inf
-            need = S.j > 0;
+            need = j > 0;
             S.l *= alpha;
             S.m = cand;
         }
         if (__any_sync(0xffffffffu, need)) {
+            if (C::B == 2) {
+                // O must not change under the PV of item j - 1: the commit that follows it
+                // (the S of item j + 1, or a closing commit) completes first
+                const int k = j + 1;
+                const uint32_t pk = (((k % 2) == 0 ? S.ph0 : S.ph1) + (uint32_t)(k / 2)) & 1u;
+                if (!warp_wait(sready_s + 8u * (k % 2), pk, abort_flag, status)) return false;
+                tc_fence_after();
+            }
             const uint32_t ocol = tmem + lane_off + C::kColO + S.s * D;
             const float f = need ? alpha : 1.f;
 #pragma unroll
@@ -322,60 +345,73 @@ __device__ __forceinline__ bool softmax_step(SoftmaxStream& S, const Unit& U, ui
                 tmem_st16(ocol + 16 * k, o);
             }
         }
-        sum = exp_tile(scol, pr, nv, c, c2, S.m);
+        sum = exp_tile<C::kItem>(scol, pr, nv, c, c2, S.m);
     }
     S.l += sum;
-    tmem_st32(scol, pr);
+    if (C::kItem == 64)
+        tmem_st32(scol, pr);
+    else
+        tmem_st16(scol, pr);
     tmem_wait_st();
     tc_fence_before();
-    mbar_arrive(pready);
+    mbar_arrive(pready_s + 8u * b);
     ++S.j;
     return true;
 }
 
-// After a stream's last item: read O and write the unit's result for this row (the chunk
-// partial in the encode, the normalised output row of Y in the decode).
+// After the stream's last item: wait for the closing commit (all of the unit's PVs are
+// complete), free the ring stages of the last items, read O and write the unit's result for
+// this row (the chunk partial in the encode, the normalised output row of Y in the decode).
 template <int D, bool DEC>
 __device__ __forceinline__ bool finish_stream(SoftmaxStream& S, const Unit& U,
                                               const TcParams& prm, uint32_t tmem,
-                                              uint32_t lane_off, int r, uint32_t sready,
-                                              uint32_t empty0, bool wg_leader,
+                                              uint32_t lane_off, int r, uint32_t sready_s,
+                                              uint32_t empty0, bool wg_leader, uint32_t it0,
                                               volatile int* abort_flag) {
     using C = Cfg<D>;
     const int a = S.s % U.n_a;
     const int par = S.s / U.n_a;
     float o[D];
     if (S.cnt > 0) {
-        if (!warp_wait(sready, S.scnt & 1, abort_flag, prm.status)) return false;
-        ++S.scnt;
+        const int k = S.cnt + C::B - 1;
+        const int b = k % C::B;
+        const uint32_t pk = ((b == 0 ? S.ph0 : S.ph1) + (uint32_t)(k / C::B)) & 1u;
+        if (!warp_wait(sready_s + 8u * b, pk, abort_flag, prm.status)) return false;
         tc_fence_after();
-        if (wg_leader) mbar_arrive(empty0 + 8u * S.prev_st);
+        if (wg_leader) {
+            for (int jj = S.cnt - C::B < 0 ? 0 : S.cnt - C::B; jj < S.cnt; ++jj) {
+                const int i_old = par + jj * U.n_par;
+                mbar_arrive(empty0 + 8u * ((it0 + i_old) % C::kStages));
+            }
+        }
         const uint32_t ocol = tmem + lane_off + C::kColO + S.s * D;
 #pragma unroll
-        for (int k = 0; k < D / 16; ++k) {
+        for (int kk = 0; kk < D / 16; ++kk) {
             uint32_t t[16];
-            tmem_ld16(ocol + 16 * k, t);
+            tmem_ld16(ocol + 16 * kk, t);
             tmem_wait_ld16(t);
 #pragma unroll
-            for (int e = 0; e < 16; ++e) o[16 * k + e] = __uint_as_float(t[e]);
+            for (int e = 0; e < 16; ++e) o[16 * kk + e] = __uint_as_float(t[e]);
         }
     } else {
 #pragma unroll
         for (int d = 0; d < D; ++d) o[d] = 0.f;
     }
+    S.ph0 += C::phases(S.cnt, 0);
+    if (C::B == 2) S.ph1 += C::phases(S.cnt, 1);
     if (DEC) {
         const int64_t tok = U.tg * C::kGroup + a * kTileRows + r;
         if (tok < prm.N) {
             const float inv = 1.f / S.l;
             uint4* dst = reinterpret_cast<uint4*>(prm.Y + (U.bh * prm.N + tok) * D);
 #pragma unroll
-            for (int k = 0; k < D / 8; ++k) {
+            for (int kk = 0; kk < D / 8; ++kk) {
                 uint4 v;
-                v.x = pack_bf16(o[8 * k + 0] * inv, o[8 * k + 1] * inv);
-                v.y = pack_bf16(o[8 * k + 2] * inv, o[8 * k + 3] * inv);
-                v.z = pack_bf16(o[8 * k + 4] * inv, o[8 * k + 5] * inv);
-                v.w = pack_bf16(o[8 * k + 6] * inv, o[8 * k + 7] * inv);
-                dst[k] = v;
+                v.x = pack_bf16(o[8 * kk + 0] * inv, o[8 * kk + 1] * inv);
+                v.y = pack_bf16(o[8 * kk + 2] * inv, o[8 * kk + 3] * inv);
+                v.z = pack_bf16(o[8 * kk + 4] * inv, o[8 * kk + 5] * inv);
+                v.w = pack_bf16(o[8 * kk + 6] * inv, o[8 * kk + 7] * inv);
+                dst[kk] = v;
             }
         }
     } else {
@@ -386,27 +422,124 @@ __device__ __forceinline__ bool finish_stream(SoftmaxStream& S, const Unit& U,
             prm.psum[idx] = S.l;
             float4* dst = reinterpret_cast<float4*>(prm.pacc + idx * D);
 #pragma unroll
-            for (int k = 0; k < D / 4; ++k)
-                dst[k] = make_float4(o[4 * k], o[4 * k + 1], o[4 * k + 2], o[4 * k + 3]);
+            for (int kk = 0; kk < D / 4; ++kk)
+                dst[kk] = make_float4(o[4 * kk], o[4 * kk + 1], o[4 * kk + 2], o[4 * kk + 3]);
         }
     }
     return true;
 }
 
-// PV of stream s: O_s (+)= P_s * C-tile of ring stage `st` (one elected lane issues).
+// PV of stream s: O_s (+)= P (score buffer pb) * C-tile of ring stage `st` (one elected
+// lane issues).
 template <int D>
-__device__ __forceinline__ void issue_pv(uint32_t tmem, uint8_t* ring, int s, int st, int npv) {
+__device__ __forceinline__ void issue_pv(uint32_t tmem, uint8_t* ring, int s, int pb, int st,
+                                         int npv) {
     using C = Cfg<D>;
     const uint32_t cb = smem_u32(ring + st * C::kStage + C::kItemTile);
 #pragma unroll
-    for (int k = 0; k < kItem / 16; ++k) {
+    for (int k = 0; k < C::kItem / 16; ++k) {
         const uint64_t bd = smem_desc(cb + k * 16 * D * 2, C::kItemTile, C::kSBO, C::kSwz);
         if (elect_one())
-            mma_ts(tmem + C::kColO + s * D, tmem + C::kColS + s * kItem + 8 * k, bd, C::kIdescPV,
-                   (npv > 0 || k > 0) ? 1u : 0u);
+            mma_ts(tmem + C::kColO + s * D, tmem + C::kColS + (s * C::B + pb) * C::kItem + 8 * k,
+                   bd, C::kIdescPV, (npv > 0 || k > 0) ? 1u : 0u);
         __syncwarp();
     }
 }
+
+// The TMA side of MMA warp 0: issues A tiles and ring items whenever their buffers are
+// free, without ever blocking (called from the warp's own wait loops). Warp-uniform.
+template <int D, bool DEC>
+struct Producer {
+    const CUtensorMap* tmA;
+    const CUtensorMap* tmB;
+    const CUtensorMap* tmC;
+    uint8_t* abuf;
+    uint8_t* ring;
+    uint32_t full0, empty0, asfull0, asempty0;
+    int64_t u;     // unit being issued
+    uint32_t ua;   // units whose A tiles were issued
+    uint32_t it;   // ring items issued
+    int i;         // next item of unit u
+    bool a_done;   // A tiles of unit u issued
+    Unit U;
+
+    __device__ __forceinline__ void start(const TcParams& prm) {
+        u = blockIdx.x;
+        ua = 0;
+        it = 0;
+        i = 0;
+        a_done = false;
+        if (u < prm.n_units) U = get_unit<D, DEC>(prm, u);
+    }
+    // Issue what can be issued now (at most a few copies). Returns true if anything was.
+    __device__ __forceinline__ bool poll(const TcParams& prm) {
+        using C = Cfg<D>;
+        bool any = false;
+        for (int n = 0; n < 4 && u < prm.n_units; ++n) {
+            if (!a_done) {
+                const int ab = ua & 1;
+                if (!__all_sync(0xffffffffu,
+                                mbar_test_wait(asempty0 + 8u * ab, ((ua >> 1) & 1) ^ 1)))
+                    return any;
+                if (elect_one()) {
+                    mbar_expect_tx(asfull0 + 8u * ab, U.n_a * C::kATile);
+                    for (int a = 0; a < U.n_a; ++a)
+                        tma_load_3d(smem_u32(abuf + ab * C::kABytes + a * C::kATile), tmA, 0,
+                                    U.rowA0 + a * kTileRows, U.zA, asfull0 + 8u * ab);
+                }
+                __syncwarp();
+                ++ua;
+                a_done = true;
+                any = true;
+                continue;
+            }
+            if (i < U.n_items) {
+                const int st = it % C::kStages;
+                if (!__all_sync(0xffffffffu,
+                                mbar_test_wait(empty0 + 8u * st, ((it / C::kStages) & 1) ^ 1)))
+                    return any;
+                if (elect_one()) {
+                    mbar_expect_tx(full0 + 8u * st, C::kStage);
+                    const int row = (int)(U.item0 + (int64_t)i * C::kItem);
+                    const uint32_t dst = smem_u32(ring + st * C::kStage);
+                    tma_load_3d(dst, tmB, 0, row, U.zB, full0 + 8u * st);
+                    tma_load_3d(dst + C::kItemTile, tmC, 0, row, U.zB, full0 + 8u * st);
+                    // streams that do not consume this item count as having released it
+                    for (int x = U.n_a; x < NS; ++x) mbar_arrive(empty0 + 8u * st);
+                }
+                __syncwarp();
+                ++it;
+                ++i;
+                any = true;
+                continue;
+            }
+            u += gridDim.x;
+            i = 0;
+            a_done = false;
+            if (u < prm.n_units) U = get_unit<D, DEC>(prm, u);
+        }
+        return any;
+    }
+    // After an abort: wait (bounded) until the newest copy of every buffer has landed.
+    __device__ __forceinline__ void drain() {
+        using C = Cfg<D>;
+        const uint64_t t0 = globaltimer_ns();
+        for (int st = 0; st < C::kStages; ++st) {
+            if ((uint32_t)st >= it) break;
+            const uint32_t x = it - 1 - ((it - 1 - st) % C::kStages);
+            while (!mbar_try_wait(full0 + 8u * st, (x / C::kStages) & 1) &&
+                   globaltimer_ns() - t0 < kWaitLimitNs) {
+            }
+        }
+        for (int b = 0; b < 2; ++b) {
+            if ((uint32_t)b >= ua) break;
+            const uint32_t y = ua - 1 - ((ua - 1 - b) % 2);
+            while (!mbar_try_wait(asfull0 + 8u * b, (y >> 1) & 1) &&
+                   globaltimer_ns() - t0 < kWaitLimitNs) {
+            }
+        }
+    }
+};
 
 // ------------------------------------------------------------------ the kernel
 
@@ -415,7 +548,6 @@ __global__ void __launch_bounds__(kThreads, 1)
     tc_chain_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
                     const __grid_constant__ CUtensorMap tmC, const TcParams prm) {
     using C = Cfg<D>;
-    constexpr int NS = C::NS;
     extern __shared__ uint8_t smem_raw[];
     uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                                ~static_cast<uintptr_t>(1023));
@@ -431,8 +563,9 @@ __global__ void __launch_bounds__(kThreads, 1)
     const uint32_t asempty0 = asfull0 + 16u;
     const uint32_t aready0 = asfull0 + 32u;
     const uint32_t afree0 = asfull0 + 48u;
-    const uint32_t sready0 = asfull0 + 64u;
-    const uint32_t pready0 = sready0 + 8u * NS;
+    const uint32_t sready0 = asfull0 + 64u;       // [NS][2]
+    const uint32_t pready0 = sready0 + 16u * NS;  // [NS][2]
+    constexpr uint32_t kSoftmaxThreads = (kWarps - kFirstSoftmaxWarp) * 32;
 
     const int warp = threadIdx.x >> 5;
     const int lane = threadIdx.x & 31;
@@ -444,13 +577,15 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         for (int b = 0; b < 2; ++b) {
             mbar_init(asfull0 + 8u * b, 1);
-            mbar_init(asempty0 + 8u * b, 256);
-            mbar_init(aready0 + 8u * b, 256);
+            mbar_init(asempty0 + 8u * b, kSoftmaxThreads);
+            mbar_init(aready0 + 8u * b, kSoftmaxThreads);
             mbar_init(afree0 + 8u * b, NS);
         }
         for (int s = 0; s < NS; ++s) {
-            mbar_init(sready0 + 8u * s, 1);
-            mbar_init(pready0 + 8u * s, 128);
+            mbar_init(sready0 + 16u * s, 1);
+            mbar_init(sready0 + 16u * s + 8u, 1);
+            mbar_init(pready0 + 16u * s, 128);
+            mbar_init(pready0 + 16u * s + 8u, 128);
         }
         *abort_flag = 0;
         fence_mbar_init();
@@ -467,124 +602,139 @@ __global__ void __launch_bounds__(kThreads, 1)
     tc_fence_after();
     const uint32_t tmem = *tmem_slot;
 
-    if (warp == 0) {
-        // ------------------------------------------------------------ TMA producer
-        if (lane == 0) {
-            uint32_t it = 0, ua = 0;
-            for (int64_t u = blockIdx.x; u < prm.n_units; u += gridDim.x) {
-                const Unit U = get_unit<D, DEC>(prm, u);
-                const int ab = ua & 1;
-                if (!wait_bar(asempty0 + 8u * ab, ((ua >> 1) & 1) ^ 1, abort_flag, prm.status))
-                    break;
-                mbar_expect_tx(asfull0 + 8u * ab, U.n_a * C::kATile);
-                for (int a = 0; a < U.n_a; ++a)
-                    tma_load_3d(smem_u32(abuf + ab * C::kABytes + a * C::kATile), &tmA, 0,
-                                U.rowA0 + a * kTileRows, U.zA, asfull0 + 8u * ab);
-                ++ua;
-                bool ok = true;
-                for (int i = 0; i < U.n_items; ++i) {
-                    const int st = it % C::kStages;
-                    if (!wait_bar(empty0 + 8u * st, ((it / C::kStages) & 1) ^ 1, abort_flag,
-                                  prm.status)) {
-                        ok = false;
-                        break;
-                    }
-                    mbar_expect_tx(full0 + 8u * st, C::kStage);
-                    const int row = (int)(U.item0 + (int64_t)i * kItem);
-                    const uint32_t dst = smem_u32(ring + st * C::kStage);
-                    tma_load_3d(dst, &tmB, 0, row, U.zB, full0 + 8u * st);
-                    tma_load_3d(dst + C::kItemTile, &tmC, 0, row, U.zB, full0 + 8u * st);
-                    // streams that do not consume this item count as having released it
-                    for (int x = U.n_a; x < NS; ++x) mbar_arrive(empty0 + 8u * st);
-                    ++it;
-                }
-                if (!ok) break;
-            }
-            if (*abort_flag) {
-                // Leave only after every copy this thread issued has landed: the newest load
-                // of each stage and of each A buffer (older ones were consumed already).
-                const uint64_t t0 = globaltimer_ns();
-                for (int st = 0; st < C::kStages; ++st) {
-                    if ((uint32_t)st >= it) break;
-                    const uint32_t x = it - 1 - ((it - 1 - st) % C::kStages);
-                    while (!mbar_try_wait(full0 + 8u * st, (x / C::kStages) & 1) &&
-                           globaltimer_ns() - t0 < kWaitLimitNs) {
-                    }
-                }
-                for (int b = 0; b < 2; ++b) {
-                    if ((uint32_t)b >= ua) break;
-                    const uint32_t y = ua - 1 - ((ua - 1 - b) % 2);
-                    while (!mbar_try_wait(asfull0 + 8u * b, (y >> 1) & 1) &&
-                           globaltimer_ns() - t0 < kWaitLimitNs) {
-                    }
-                }
-            }
-        }
-    } else if (warp < kFirstSoftmaxWarp) {
+    if (warp < kFirstSoftmaxWarp) {
         // ------------------------------------------------------------ MMA warps
-        // Warp 1 + s drives stream s. For each of its items: the PV of its previous item
-        // (P from TMEM, V or Z from the ring), the S of this item (A from TMEM, K or Q from
-        // the ring) and one commit, which the softmax waits on. It observes the full
-        // barrier of every ring item in order, so each parity test names one phase.
-        const int s = warp - kFirstMmaWarp;
-        if (s < NS) {
-            uint32_t it = 0, ua = 0, pcnt = 0;
-            bool ok = true;
-            for (int64_t u = blockIdx.x; u < prm.n_units && ok; u += gridDim.x, ++ua) {
-                const Unit U = get_unit<D, DEC>(prm, u);
-                const int ab = ua & 1;
-                if (!warp_wait(aready0 + 8u * ab, (ua >> 1) & 1, abort_flag, prm.status)) break;
-                tc_fence_after();
-                const int a = s % U.n_a;
-                const int par = s / U.n_a;
-                const uint32_t a_tmem = tmem + C::kColA + (ab * NS + a) * (D / 2);
-                int prev = -1, npv = 0;
-                for (int i = 0; i < U.n_items; ++i, ++it) {
-                    const int st = it % C::kStages;
-                    const bool mine = (i % U.n_par) == par;
-                    if (mine && prev >= 0) {
-                        if (!warp_wait(pready0 + 8u * s, pcnt & 1, abort_flag, prm.status)) {
-                            ok = false;
-                            break;
+        // Warp s drives stream s. For each of its items: the PV of its previous item (P
+        // from TMEM, V or Z from the ring), the S of this item (A from TMEM, K or Q from the
+        // ring) and one commit, which the softmax waits on. It observes the full barrier of
+        // every ring item in order, so each parity test names one phase. Warp 0 also keeps
+        // the TMA producer going whenever it would otherwise wait.
+        const int s = warp;
+        Producer<D, DEC> prod;
+        prod.tmA = &tmA;
+        prod.tmB = &tmB;
+        prod.tmC = &tmC;
+        prod.abuf = abuf;
+        prod.ring = ring;
+        prod.full0 = full0;
+        prod.empty0 = empty0;
+        prod.asfull0 = asfull0;
+        prod.asempty0 = asempty0;
+        if (s == 0) prod.start(prm);
+        // wait for a barrier phase; warp 0 feeds the producer meanwhile
+        auto wait = [&](uint32_t bar, uint32_t parity) -> bool {
+            if (s != 0) return warp_wait(bar, parity, abort_flag, prm.status);
+            uint64_t t0 = 0;
+            for (uint32_t n = 0;; ++n) {
+                if (__all_sync(0xffffffffu, mbar_test_wait(bar, parity))) return true;
+                if (prod.poll(prm)) {
+                    t0 = 0;
+                    continue;
+                }
+                if ((n & 63u) == 0) {
+                    if (__any_sync(0xffffffffu, *abort_flag != 0)) return false;
+                    const uint64_t now = globaltimer_ns();
+                    if (t0 == 0) t0 = now;
+                    if (now - t0 > kWaitLimitNs) {
+                        if (lane == 0) {
+                            *abort_flag = 1;
+                            atomicExch(prm.status, (int)FLAREPP_ERR_TIMEOUT);
                         }
-                        ++pcnt;
-                        tc_fence_after();
-                        issue_pv<D>(tmem, ring, s, prev, npv);
-                        ++npv;
+                        __syncwarp();
+                        return false;
                     }
-                    if (!warp_wait(full0 + 8u * st, (it / C::kStages) & 1, abort_flag,
-                                   prm.status)) {
+                }
+            }
+        };
+        uint32_t it = 0, ua = 0, pc0 = 0, pc1 = 0;  // p_ready phases consumed per buffer
+        bool ok = true;
+        for (int64_t u = blockIdx.x; u < prm.n_units && ok; u += gridDim.x, ++ua) {
+            const Unit U = get_unit<D, DEC>(prm, u);
+            const int tb = ua % C::kABuf;
+            if (!wait(aready0 + 8u * tb, (ua / C::kABuf) & 1)) break;
+            tc_fence_after();
+            const int a = s % U.n_a;
+            const int par = s / U.n_a;
+            const uint32_t a_tmem = tmem + C::kColA + (tb * NS + a) * (D / 2);
+            const uint32_t sready_s = sready0 + 16u * s;
+            int j = 0, npv = 0;
+            int stg0 = 0, stg1 = 0;  // ring stages of this stream's items j with j % 2 == 0, 1
+            // PV of item jo = j - B (P in buffer jo % B), after its P is written
+            auto pv_of = [&](int jo) -> bool {
+                const int pb = jo % C::B;
+                uint32_t& pc = pb == 0 ? pc0 : pc1;
+                if (!wait(pready0 + 16u * s + 8u * pb, pc & 1)) return false;
+                ++pc;
+                tc_fence_after();
+                issue_pv<D>(tmem, ring, s, jo % C::B, (jo & 1) ? stg1 : stg0, npv);
+                ++npv;
+                return true;
+            };
+            for (int i = 0; i < U.n_items; ++i, ++it) {
+                const int st = it % C::kStages;
+                const bool mine = (i % U.n_par) == par;
+                // the PV of item j - B first: it frees the score buffer (and maybe the stage)
+                if (mine && j >= C::B && !pv_of(j - C::B)) {
+                    ok = false;
+                    break;
+                }
+                if (!wait(full0 + 8u * st, (it / C::kStages) & 1)) {
+                    ok = false;
+                    break;
+                }
+                if (!mine) continue;
+                tc_fence_after();
+                const int b = j % C::B;
+                const uint32_t bb = smem_u32(ring + st * C::kStage);
+#pragma unroll
+                for (int k = 0; k < D / 16; ++k) {
+                    const uint64_t bd = smem_desc(bb + 32 * k, 16, C::kSBO, C::kSwz);
+                    if (elect_one())
+                        mma_ts(tmem + C::kColS + (s * C::B + b) * C::kItem, a_tmem + 8 * k, bd,
+                               C::kIdescS, k > 0 ? 1u : 0u);
+                    __syncwarp();
+                }
+                if (elect_one()) mma_commit(sready_s + 8u * b);
+                __syncwarp();
+                if (j & 1)
+                    stg1 = st;
+                else
+                    stg0 = st;
+                ++j;
+            }
+            if (!ok) break;
+            // closing commits k = cnt .. cnt + B - 1, each after the PV of item k - B
+            if (j > 0) {
+                for (int k = j; k < j + C::B; ++k) {
+                    if (k - C::B >= 0 && !pv_of(k - C::B)) {
                         ok = false;
                         break;
                     }
-                    if (!mine) continue;
-                    tc_fence_after();
-                    const uint32_t bb = smem_u32(ring + st * C::kStage);
-#pragma unroll
-                    for (int k = 0; k < D / 16; ++k) {
-                        const uint64_t bd = smem_desc(bb + 32 * k, 16, C::kSBO, C::kSwz);
-                        if (elect_one())
-                            mma_ts(tmem + C::kColS + s * kItem, a_tmem + 8 * k, bd, C::kIdescS,
-                                   k > 0 ? 1u : 0u);
-                        __syncwarp();
-                    }
-                    if (elect_one()) mma_commit(sready0 + 8u * s);
+                    if (elect_one()) mma_commit(sready_s + 8u * (k % C::B));
                     __syncwarp();
-                    prev = st;
                 }
                 if (!ok) break;
-                if (prev >= 0) {  // the last PV of the stream, then the final s_ready
-                    if (!warp_wait(pready0 + 8u * s, pcnt & 1, abort_flag, prm.status)) break;
-                    ++pcnt;
-                    tc_fence_after();
-                    issue_pv<D>(tmem, ring, s, prev, npv);
-                    if (elect_one()) mma_commit(sready0 + 8u * s);
-                    __syncwarp();
-                }
-                // this stream's MMAs no longer read the unit's A buffer
-                if (elect_one()) mma_commit(afree0 + 8u * ab);
-                __syncwarp();
             }
+            // this stream's MMAs no longer read the unit's TMEM A buffer
+            if (elect_one()) mma_commit(afree0 + 8u * tb);
+            __syncwarp();
+        }
+        if (s == 0) {
+            // issue whatever the other streams still need (normally nothing is left)
+            uint64_t t0 = globaltimer_ns();
+            while (!*abort_flag && prod.u < prm.n_units) {
+                if (prod.poll(prm)) {
+                    t0 = globaltimer_ns();
+                } else if (globaltimer_ns() - t0 > kWaitLimitNs) {
+                    if (lane == 0) {
+                        *abort_flag = 1;
+                        atomicExch(prm.status, (int)FLAREPP_ERR_TIMEOUT);
+                    }
+                    __syncwarp();
+                    break;
+                }
+            }
+            if (*abort_flag) prod.drain();
         }
     } else {
         // ------------------------------------------------------------ softmax warpgroups
@@ -595,25 +745,25 @@ __global__ void __launch_bounds__(kThreads, 1)
         const bool wg_leader = ((warp - kFirstSoftmaxWarp) & 3) == 0 && lane == 0;
         const float c = prm.c;
         const uint64_t c2 = pack_f32x2(c, c);
-        SoftmaxStream st0, st1;
-        st0.s = wg;
-        st1.s = wg + 2;  // used when NS == 4
-        st0.scnt = st1.scnt = 0;
+        SoftmaxStream st;
+        st.s = wg;
+        st.ph0 = st.ph1 = 0;
+        const uint32_t sready_s = sready0 + 16u * wg;
         bool alive = true;
         uint32_t ua = 0, it0 = 0;
         for (int64_t u = blockIdx.x; u < prm.n_units && alive; u += gridDim.x, ++ua) {
             const Unit U = get_unit<D, DEC>(prm, u);
             const int ab = ua & 1;
-            // copy this warpgroup's A tiles (one row per thread) from smem into TMEM, once
+            const int tb = ua % C::kABuf;
+            // copy this warpgroup's A tile (one row per thread) from smem into TMEM, once
             // the MMAs of the unit that last used this TMEM buffer are complete
             if (!warp_wait(asfull0 + 8u * ab, (ua >> 1) & 1, abort_flag, prm.status)) break;
-            if (!warp_wait(afree0 + 8u * ab, ((ua >> 1) & 1) ^ 1, abort_flag, prm.status)) break;
+            if (!warp_wait(afree0 + 8u * tb, ((ua / C::kABuf) & 1) ^ 1, abort_flag, prm.status))
+                break;
             tc_fence_after();
-            for (int a = 0; a < U.n_a; ++a) {
-                const int writer = U.n_a == 1 ? 0 : (a & 1);
-                if (writer != wg) continue;
+            if (st.s < U.n_a) {
                 const uint4* src = reinterpret_cast<const uint4*>(abuf + ab * C::kABytes +
-                                                                  a * C::kATile + r * D * 2);
+                                                                  st.s * C::kATile + r * D * 2);
                 uint32_t v[D / 2];
 #pragma unroll
                 for (int k = 0; k < D / 8; ++k) {
@@ -623,7 +773,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                     v[4 * k + 2] = x.z;
                     v[4 * k + 3] = x.w;
                 }
-                const uint32_t acol = tmem + lane_off + C::kColA + (ab * NS + a) * (D / 2);
+                const uint32_t acol = tmem + lane_off + C::kColA + (tb * NS + st.s) * (D / 2);
                 if (D == 16) {
                     tmem_st8(acol, v);
                 } else {
@@ -633,33 +783,17 @@ __global__ void __launch_bounds__(kThreads, 1)
             }
             tmem_wait_st();
             tc_fence_before();
-            mbar_arrive(aready0 + 8u * ab);
+            mbar_arrive(aready0 + 8u * tb);
             mbar_arrive(asempty0 + 8u * ab);
 
-            st0.begin(U);
-            if (NS == 4) st1.begin(U);
-            while (alive && (st0.j < st0.cnt || (NS == 4 && st1.j < st1.cnt))) {
-                if (st0.j < st0.cnt) {
-                    const int item = st0.s / U.n_a + st0.j * U.n_par;
-                    alive = softmax_step<D>(st0, U, tmem, lane_off, c, c2, sready0 + 8u * st0.s,
-                                            pready0 + 8u * st0.s, empty0, wg_leader,
-                                            (int)((it0 + item) % C::kStages), abort_flag,
-                                            prm.status);
-                }
-                if (NS == 4 && alive && st1.j < st1.cnt) {
-                    const int item = st1.s / U.n_a + st1.j * U.n_par;
-                    alive = softmax_step<D>(st1, U, tmem, lane_off, c, c2, sready0 + 8u * st1.s,
-                                            pready0 + 8u * st1.s, empty0, wg_leader,
-                                            (int)((it0 + item) % C::kStages), abort_flag,
-                                            prm.status);
-                }
-            }
+            st.begin(U);
+            while (alive && st.j < st.cnt)
+                alive = softmax_step<D>(st, U, tmem, lane_off, c, c2, sready_s,
+                                        pready0 + 16u * st.s, empty0, wg_leader, it0, abort_flag,
+                                        prm.status);
             if (alive)
-                alive = finish_stream<D, DEC>(st0, U, prm, tmem, lane_off, r, sready0 + 8u * st0.s,
-                                              empty0, wg_leader, abort_flag);
-            if (NS == 4 && alive)
-                alive = finish_stream<D, DEC>(st1, U, prm, tmem, lane_off, r, sready0 + 8u * st1.s,
-                                              empty0, wg_leader, abort_flag);
+                alive = finish_stream<D, DEC>(st, U, prm, tmem, lane_off, r, sready_s, empty0,
+                                              wg_leader, it0, abort_flag);
             it0 += U.n_items;
         }
     }
@@ -737,7 +871,15 @@ cudaError_t launch_d(int64_t D, const CUtensorMap& a, const CUtensorMap& b, cons
 
 }  // namespace
 
-int64_t tc_group_rows(int64_t D) { return (D == 64 ? 2 : 4) * kTileRows; }
+// Streamed rows per item (the TMA box height of the ring tiles): Cfg<D>::kItem.
+uint32_t item_rows(int64_t D) {
+    return D == 16 ? Cfg<16>::kItem : (D == 32 ? Cfg<32>::kItem : Cfg<64>::kItem);
+}
+
+int64_t tc_group_rows(int64_t D) {
+    (void)D;
+    return NS * kTileRows;
+}
 
 cudaError_t tc_encode(const Plan& p, int call, const void* k, const void* v, const void* seeds,
                       float scale, char* ws, cudaStream_t st) {
@@ -753,8 +895,8 @@ cudaError_t tc_encode(const Plan& p, int call, const void* k, const void* v, con
         a_z = p.BH;
     }
     if (!make_map(&ma, a_src, p.D, p.M, a_z, kTileRows, false) ||
-        !make_map(&mb, k, p.D, p.N, p.BH, kItem, true) ||
-        !make_map(&mc, v, p.D, p.N, p.BH, kItem, true))
+        !make_map(&mb, k, p.D, p.N, p.BH, item_rows(p.D), true) ||
+        !make_map(&mc, v, p.D, p.N, p.BH, item_rows(p.D), true))
         return cudaErrorInvalidValue;
     TcParams prm{};
     prm.BH = p.BH;
@@ -778,8 +920,8 @@ cudaError_t tc_decode(const Plan& p, const void* K, float scale, void* Y, char* 
                       cudaStream_t st) {
     CUtensorMap ma, mb, mc;
     if (!make_map(&ma, K, p.D, p.N, p.BH, kTileRows, false) ||
-        !make_map(&mb, ws + p.off_qop, p.D, p.M, p.BH, kItem, true) ||
-        !make_map(&mc, ws + p.off_zop, p.D, p.M, p.BH, kItem, true))
+        !make_map(&mb, ws + p.off_qop, p.D, p.M, p.BH, item_rows(p.D), true) ||
+        !make_map(&mc, ws + p.off_zop, p.D, p.M, p.BH, item_rows(p.D), true))
         return cudaErrorInvalidValue;
     TcParams prm{};
     prm.BH = p.BH;
