@@ -85,6 +85,7 @@ struct Cfg {
     static constexpr uint32_t kColA = kColO + NS * D;     // kABuf x NS tiles x D/2
     static_assert(kColA + kABuf * NS * (D / 2) <= kTmemCols, "TMEM budget");
     static_assert(kSmem <= 232448, "shared memory budget");
+    static_assert(kStages >= 2 * B * NS, "ring depth: the full wait precedes the PV");
     // s_ready phases buffer b receives in a unit where the stream has cnt items: one per
     // k in [0, cnt + B - 1] with k % B == b (k >= cnt are the closing commits)
     __device__ static __forceinline__ uint32_t phases(int cnt, int b) {
@@ -673,16 +674,20 @@ __global__ void __launch_bounds__(kThreads, 1)
             for (int i = 0; i < U.n_items; ++i, ++it) {
                 const int st = it % C::kStages;
                 const bool mine = (i % U.n_par) == par;
-                // the PV of item j - B first: it frees the score buffer (and maybe the stage)
-                if (mine && j >= C::B && !pv_of(j - C::B)) {
-                    ok = false;
-                    break;
-                }
+                // the item's full barrier first (the softmax is still busy with item j - B, so
+                // this wait is off the P -> PV -> S round trip), then the PV of item j - B,
+                // which frees the score buffer for S(j). Item i lands once item i - kStages
+                // is released; with kStages >= 2 B NS that item's PV was issued in an
+                // earlier iteration, so this wait cannot close a cycle.
                 if (!wait(full0 + 8u * st, (it / C::kStages) & 1)) {
                     ok = false;
                     break;
                 }
                 if (!mine) continue;
+                if (j >= C::B && !pv_of(j - C::B)) {
+                    ok = false;
+                    break;
+                }
                 tc_fence_after();
                 const int b = j % C::B;
                 const uint32_t bb = smem_u32(ring + st * C::kStage);
