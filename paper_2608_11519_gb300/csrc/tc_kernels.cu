@@ -12,13 +12,12 @@
 //     meets a stream of 64-route items (Q and Z tiles). Each token row keeps an online
 //     softmax over routes and writes its normalised row of Y.
 //
-// Work is cut into four TMEM "streams". Stream s owns B score buffers of 128 x kItem fp32
+// Work is cut into four TMEM "streams". Stream s owns one score buffer of 128 x kItem fp32
 // (kItem = 64 tokens or routes, 32 for D = 64; S is rewritten in place as bf16 P, the A
 // operand of the PV product) and a 128 x D fp32 accumulator O, and reads one resident A
-// tile kept in TMEM, so that S = A * B^T is a TMEM x SMEM product. The protocol supports
-// B = 2 (the MMA warp computes the S of item j+1 while the softmax works on item j); the
-// TMEM budget of four streams allows it only for 32-wide items, which measured slower
-// than single-buffered 64-wide items, so B = 1. Roles (20 warps):
+// tile kept in TMEM, so that S = A * B^T is a TMEM x SMEM product. With two TMEM copies of
+// the A tiles (D <= 32) the softmax copies the next unit's tiles while it works on the
+// current unit, so a unit boundary does not drain the pipeline. Roles (20 warps):
 //   warps 0..3    one MMA warp per stream: for item j, the PV of item j-B and the S of
 //                 item j, then one commit (a commit stalls only the warp that issues it);
 //                 warp 0 also issues the TMA loads (A tiles, unswizzled; the item ring,
@@ -59,7 +58,7 @@ constexpr float kFastLimit = 281474976710656.0f;  // 2^48
 template <int D>
 struct Cfg {
     static constexpr int kItem = D == 64 ? 32 : 64;   // streamed rows per item
-    static constexpr int B = 1;                       // score buffers per stream (1 or 2)
+    static constexpr int B = 1;                       // score buffers per stream
     static constexpr int kABuf = D == 64 ? 1 : 2;     // TMEM copies of the A tiles
     static constexpr int kGroup = NS * kTileRows;     // resident rows per work unit
     static constexpr int kStages = D == 64 ? 8 : (kItem == 32 ? 16 : 8);  // multiple of 4
@@ -70,8 +69,11 @@ struct Cfg {
     static constexpr uint32_t kSwz = D == 16 ? kSw32 : (D == 32 ? kSw64 : kSw128);
     static constexpr uint32_t kSBO = 8 * D * 2;  // bytes between 8-row groups
     // barriers: full[S], empty[S], asmem_full[2], asmem_empty[2], a_ready[2], a_free[2],
-    //           s_ready[NS][2], p_ready[NS][2] (per score buffer: the four warps of a
-    //           softmax warpgroup can be one item apart, never two)
+    //           sync[NS][2] = {s_ready, o_done} per stream (S of an item complete; every PV
+    //           of the stream's unit complete), p_ready[NS][2] (slot 0 used). A barrier that
+    //           a warp waits on by parity never runs two phases ahead of that warp: s_ready
+    //           of the next item needs this item's P (p_ready counts every warp of the
+    //           warpgroup), o_done of the next unit needs that unit's P.
     static constexpr int kNumBars = 2 * kStages + 8 + 4 * NS;
     static constexpr int kData = 2 * kABytes + kStages * kStage;
     static constexpr int kNeed = 1024 + kData + kNumBars * 8 + 16;
@@ -86,11 +88,7 @@ struct Cfg {
     static_assert(kColA + kABuf * NS * (D / 2) <= kTmemCols, "TMEM budget");
     static_assert(kSmem <= 232448, "shared memory budget");
     static_assert(kStages >= 2 * B * NS, "ring depth: the full wait precedes the PV");
-    // s_ready phases buffer b receives in a unit where the stream has cnt items: one per
-    // k in [0, cnt + B - 1] with k % B == b (k >= cnt are the closing commits)
-    __device__ static __forceinline__ uint32_t phases(int cnt, int b) {
-        return cnt > 0 ? (uint32_t)((cnt + B - 1 - b) / B + 1) : 0u;
-    }
+    static_assert(B == 1, "the s_ready / o_done protocol has one score buffer per stream");
 };
 
 struct TcParams {
@@ -196,7 +194,8 @@ struct SoftmaxStream {
     int s;          // stream index
     int cnt, j;     // items of the stream in this unit, items done
     float m, l;     // reference max (base 2, scaled) and running sum
-    uint32_t ph0, ph1;  // s_ready phases of buffers 0 and 1 completed in earlier units
+    uint32_t ph0;   // s_ready phases completed in earlier units (one per item)
+    uint32_t od;    // o_done phases completed in earlier units (one per unit with items)
     __device__ __forceinline__ void begin(const Unit& U) {
         const int par = s / U.n_a;
         cnt = U.n_items > par ? (U.n_items - par + U.n_par - 1) / U.n_par : 0;
@@ -287,7 +286,7 @@ __device__ __forceinline__ bool softmax_step(SoftmaxStream& S, const Unit& U, ui
     using C = Cfg<D>;
     const int j = S.j;
     const int b = j % C::B;
-    const uint32_t par_j = ((b == 0 ? S.ph0 : S.ph1) + (uint32_t)(j / C::B)) & 1u;
+    const uint32_t par_j = (S.ph0 + (uint32_t)j) & 1u;
     if (!warp_wait(sready_s + 8u * b, par_j, abort_flag, status)) return false;
     tc_fence_after();
     const int par = S.s / U.n_a;
@@ -326,14 +325,7 @@ __device__ __forceinline__ bool softmax_step(SoftmaxStream& S, const Unit& U, ui
             S.m = cand;
         }
         if (__any_sync(0xffffffffu, need)) {
-            if (C::B == 2) {
-                // O must not change under the PV of item j - 1: the commit that follows it
-                // (the S of item j + 1, or a closing commit) completes first
-                const int k = j + 1;
-                const uint32_t pk = (((k % 2) == 0 ? S.ph0 : S.ph1) + (uint32_t)(k / 2)) & 1u;
-                if (!warp_wait(sready_s + 8u * (k % 2), pk, abort_flag, status)) return false;
-                tc_fence_after();
-            }
+            // (the PV of item j - 1 is complete: S of item j followed it in the tensor pipe)
             const uint32_t ocol = tmem + lane_off + C::kColO + S.s * D;
             const float f = need ? alpha : 1.f;
 #pragma unroll
@@ -360,8 +352,8 @@ __device__ __forceinline__ bool softmax_step(SoftmaxStream& S, const Unit& U, ui
     return true;
 }
 
-// After the stream's last item: wait for the closing commit (all of the unit's PVs are
-// complete), free the ring stages of the last items, read O and write the unit's result for
+// After the stream's last item: wait for o_done (all of the unit's PVs are complete), free
+// the ring stage of the last item, read O and write the unit's result for
 // this row (the chunk partial in the encode, the normalised output row of Y in the decode).
 template <int D, bool DEC>
 __device__ __forceinline__ bool finish_stream(SoftmaxStream& S, const Unit& U,
@@ -374,10 +366,8 @@ __device__ __forceinline__ bool finish_stream(SoftmaxStream& S, const Unit& U,
     const int par = S.s / U.n_a;
     float o[D];
     if (S.cnt > 0) {
-        const int k = S.cnt + C::B - 1;
-        const int b = k % C::B;
-        const uint32_t pk = ((b == 0 ? S.ph0 : S.ph1) + (uint32_t)(k / C::B)) & 1u;
-        if (!warp_wait(sready_s + 8u * b, pk, abort_flag, prm.status)) return false;
+        if (!warp_wait(sready_s + 8u, S.od & 1u, abort_flag, prm.status)) return false;
+        ++S.od;
         tc_fence_after();
         if (wg_leader) {
             for (int jj = S.cnt - C::B < 0 ? 0 : S.cnt - C::B; jj < S.cnt; ++jj) {
@@ -398,8 +388,7 @@ __device__ __forceinline__ bool finish_stream(SoftmaxStream& S, const Unit& U,
 #pragma unroll
         for (int d = 0; d < D; ++d) o[d] = 0.f;
     }
-    S.ph0 += C::phases(S.cnt, 0);
-    if (C::B == 2) S.ph1 += C::phases(S.cnt, 1);
+    S.ph0 += (uint32_t)S.cnt;
     if (DEC) {
         const int64_t tok = U.tg * C::kGroup + a * kTileRows + r;
         if (tok < prm.N) {
@@ -448,7 +437,9 @@ __device__ __forceinline__ void issue_pv(uint32_t tmem, uint8_t* ring, int s, in
 }
 
 // The TMA side of MMA warp 0: issues A tiles and ring items whenever their buffers are
-// free, without ever blocking (called from the warp's own wait loops). Warp-uniform.
+// free, without ever blocking (called from the warp's own wait loops). Warp-uniform. With
+// two TMEM copies of the A tiles the A tiles run one unit ahead of the ring items, so that
+// the softmax can copy the next unit's A tiles into TMEM while it works on the current one.
 template <int D, bool DEC>
 struct Producer {
     const CUtensorMap* tmA;
@@ -457,43 +448,51 @@ struct Producer {
     uint8_t* abuf;
     uint8_t* ring;
     uint32_t full0, empty0, asfull0, asempty0;
-    int64_t u;     // unit being issued
-    uint32_t ua;   // units whose A tiles were issued
-    uint32_t it;   // ring items issued
-    int i;         // next item of unit u
-    bool a_done;   // A tiles of unit u issued
+    int64_t u;      // unit whose ring items are being issued
+    uint32_t ui;    // its ordinal among this CTA's units
+    int i;          // its next item
+    uint32_t it;    // ring items issued
+    int64_t u_a;    // next unit whose A tiles are to be issued
+    uint32_t ua;    // units whose A tiles were issued
     Unit U;
 
     __device__ __forceinline__ void start(const TcParams& prm) {
         u = blockIdx.x;
-        ua = 0;
-        it = 0;
+        ui = 0;
         i = 0;
-        a_done = false;
+        it = 0;
+        u_a = blockIdx.x;
+        ua = 0;
         if (u < prm.n_units) U = get_unit<D, DEC>(prm, u);
+    }
+    __device__ __forceinline__ bool done(const TcParams& prm) const {
+        return u >= prm.n_units && u_a >= prm.n_units;
     }
     // Issue what can be issued now (at most a few copies). Returns true if anything was.
     __device__ __forceinline__ bool poll(const TcParams& prm) {
         using C = Cfg<D>;
+        constexpr uint32_t kAhead = C::kABuf == 2 ? 1u : 0u;
         bool any = false;
-        for (int n = 0; n < 4 && u < prm.n_units; ++n) {
-            if (!a_done) {
+        for (int n = 0; n < 4; ++n) {
+            if (u_a < prm.n_units && ua <= ui + kAhead) {
                 const int ab = ua & 1;
-                if (!__all_sync(0xffffffffu,
-                                mbar_test_wait(asempty0 + 8u * ab, ((ua >> 1) & 1) ^ 1)))
-                    return any;
-                if (elect_one()) {
-                    mbar_expect_tx(asfull0 + 8u * ab, U.n_a * C::kATile);
-                    for (int a = 0; a < U.n_a; ++a)
-                        tma_load_3d(smem_u32(abuf + ab * C::kABytes + a * C::kATile), tmA, 0,
-                                    U.rowA0 + a * kTileRows, U.zA, asfull0 + 8u * ab);
+                if (__all_sync(0xffffffffu,
+                               mbar_test_wait(asempty0 + 8u * ab, ((ua >> 1) & 1) ^ 1))) {
+                    const Unit UA = get_unit<D, DEC>(prm, u_a);
+                    if (elect_one()) {
+                        mbar_expect_tx(asfull0 + 8u * ab, UA.n_a * C::kATile);
+                        for (int a = 0; a < UA.n_a; ++a)
+                            tma_load_3d(smem_u32(abuf + ab * C::kABytes + a * C::kATile), tmA, 0,
+                                        UA.rowA0 + a * kTileRows, UA.zA, asfull0 + 8u * ab);
+                    }
+                    __syncwarp();
+                    ++ua;
+                    u_a += gridDim.x;
+                    any = true;
+                    continue;
                 }
-                __syncwarp();
-                ++ua;
-                a_done = true;
-                any = true;
-                continue;
             }
+            if (u >= prm.n_units) return any;
             if (i < U.n_items) {
                 const int st = it % C::kStages;
                 if (!__all_sync(0xffffffffu,
@@ -515,8 +514,8 @@ struct Producer {
                 continue;
             }
             u += gridDim.x;
+            ++ui;
             i = 0;
-            a_done = false;
             if (u < prm.n_units) U = get_unit<D, DEC>(prm, u);
         }
         return any;
@@ -708,17 +707,11 @@ __global__ void __launch_bounds__(kThreads, 1)
                 ++j;
             }
             if (!ok) break;
-            // closing commits k = cnt .. cnt + B - 1, each after the PV of item k - B
+            // the PV of the unit's last item, then o_done: O is final for the softmax
             if (j > 0) {
-                for (int k = j; k < j + C::B; ++k) {
-                    if (k - C::B >= 0 && !pv_of(k - C::B)) {
-                        ok = false;
-                        break;
-                    }
-                    if (elect_one()) mma_commit(sready_s + 8u * (k % C::B));
-                    __syncwarp();
-                }
-                if (!ok) break;
+                if (!pv_of(j - C::B)) break;
+                if (elect_one()) mma_commit(sready_s + 8u);
+                __syncwarp();
             }
             // this stream's MMAs no longer read the unit's TMEM A buffer
             if (elect_one()) mma_commit(afree0 + 8u * tb);
@@ -727,7 +720,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (s == 0) {
             // issue whatever the other streams still need (normally nothing is left)
             uint64_t t0 = globaltimer_ns();
-            while (!*abort_flag && prod.u < prm.n_units) {
+            while (!*abort_flag && !prod.done(prm)) {
                 if (prod.poll(prm)) {
                     t0 = globaltimer_ns();
                 } else if (globaltimer_ns() - t0 > kWaitLimitNs) {
@@ -752,21 +745,24 @@ __global__ void __launch_bounds__(kThreads, 1)
         const uint64_t c2 = pack_f32x2(c, c);
         SoftmaxStream st;
         st.s = wg;
-        st.ph0 = st.ph1 = 0;
+        st.ph0 = 0;
+        st.od = 0;
         const uint32_t sready_s = sready0 + 16u * wg;
         bool alive = true;
         uint32_t ua = 0, it0 = 0;
-        for (int64_t u = blockIdx.x; u < prm.n_units && alive; u += gridDim.x, ++ua) {
-            const Unit U = get_unit<D, DEC>(prm, u);
-            const int ab = ua & 1;
-            const int tb = ua % C::kABuf;
-            // copy this warpgroup's A tile (one row per thread) from smem into TMEM, once
-            // the MMAs of the unit that last used this TMEM buffer are complete
-            if (!warp_wait(asfull0 + 8u * ab, (ua >> 1) & 1, abort_flag, prm.status)) break;
-            if (!warp_wait(afree0 + 8u * tb, ((ua / C::kABuf) & 1) ^ 1, abort_flag, prm.status))
-                break;
+        constexpr bool kAhead = C::kABuf == 2;
+        // Copy this warpgroup's A tile of unit ua (one row per thread) from smem into TMEM
+        // copy ua % kABuf, once the MMAs of the unit that last used that copy are complete.
+        auto copy_a = [&](uint32_t ua_c, int64_t u_c) -> bool {
+            const int n_a = get_unit<D, DEC>(prm, u_c).n_a;
+            const int ab = ua_c & 1;
+            const int tb = ua_c % C::kABuf;
+            if (!warp_wait(asfull0 + 8u * ab, (ua_c >> 1) & 1, abort_flag, prm.status))
+                return false;
+            if (!warp_wait(afree0 + 8u * tb, ((ua_c / C::kABuf) & 1) ^ 1, abort_flag, prm.status))
+                return false;
             tc_fence_after();
-            if (st.s < U.n_a) {
+            if (st.s < n_a) {
                 const uint4* src = reinterpret_cast<const uint4*>(abuf + ab * C::kABytes +
                                                                   st.s * C::kATile + r * D * 2);
                 uint32_t v[D / 2];
@@ -790,7 +786,17 @@ __global__ void __launch_bounds__(kThreads, 1)
             tc_fence_before();
             mbar_arrive(aready0 + 8u * tb);
             mbar_arrive(asempty0 + 8u * ab);
-
+            return true;
+        };
+        for (int64_t u = blockIdx.x; u < prm.n_units && alive; u += gridDim.x, ++ua) {
+            const Unit U = get_unit<D, DEC>(prm, u);
+            // this unit's A tiles (copied one unit ahead when TMEM holds two copies)
+            if (kAhead) {
+                if (ua == 0 && !copy_a(0, u)) break;
+                if (u + gridDim.x < prm.n_units && !copy_a(ua + 1, u + gridDim.x)) break;
+            } else if (!copy_a(ua, u)) {
+                break;
+            }
             st.begin(U);
             while (alive && st.j < st.cnt)
                 alive = softmax_step<D>(st, U, tmem, lane_off, c, c2, sready_s,
