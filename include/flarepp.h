@@ -123,6 +123,38 @@ FLAREPP_API flarepp_status flarepp_route_fwd_profiled(const flarepp_shape* shape
                                                       int n_events);
 
 /*
+ * Bytes of device memory that flarepp_route_fwd_host needs for `shape` (its workspace plus
+ * device copies of the inputs and of Y), or 0 for an invalid shape or an empty Y.
+ */
+FLAREPP_API size_t flarepp_route_host_buffer_bytes(const flarepp_shape* shape);
+
+/*
+ * The routing chain of flarepp_route_fwd (Sec. 3.2, eqs. flarepp_dynamic_query and
+ * flarepp_mixer) on HOST buffers: copies the inputs to the device, runs the chain and copies
+ * Y back, with the copies overlapped with the computation. The (b, h) slices of the chain are
+ * independent, so the heads are processed in up to four groups: while the chain of one group
+ * runs on `stream`, the next group's inputs are copied in on a second stream and the previous
+ * group's Y is copied out on a third.
+ *   seeds, Kt, Vt, K, V, Y: host pointers, same layouts and dtypes as flarepp_route_fwd. The
+ *     copies overlap the kernels only when the host memory is page-locked (pinned).
+ *   device_buffer: caller-owned device memory of at least flarepp_route_host_buffer_bytes
+ *     bytes, 256-byte aligned (else FLAREPP_ERR_WORKSPACE). It starts with the workspace, so
+ *     flarepp_route_device_status(shape, device_buffer, ...) reports a timeout in any group.
+ *   Streams: the second and third streams and the events that order them are created by the
+ *     call and released at its end; CUDA frees them once their work has finished.
+ *   Asynchronous: everything is ordered after the work already on `stream`, and later work
+ *     on `stream` is ordered after the last copy into Y. The host buffers must stay valid
+ *     (and Y unread) until then.
+ *   Errors: as flarepp_route_fwd, plus FLAREPP_ERR_CUDA if a stream or event cannot be
+ *     created. An empty Y (N or B*H zero) returns FLAREPP_OK without any work.
+ */
+FLAREPP_API flarepp_status flarepp_route_fwd_host(const flarepp_shape* shape, const void* seeds,
+                                                  const void* Kt, const void* Vt, const void* K,
+                                                  const void* V, float scale, void* Y,
+                                                  void* device_buffer,
+                                                  size_t device_buffer_bytes, void* stream);
+
+/*
  * flarepp_route_fwd without a caller-provided workspace. The paper has no counterpart: this
  * entry point exists for callers that cannot allocate device memory when they call the
  * chain. Examples are a plugin whose host application owns all device memory, and a

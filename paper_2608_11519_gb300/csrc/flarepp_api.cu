@@ -130,7 +130,8 @@ bool overlaps(const void* a, size_t na, const void* b, size_t nb) {
 flarepp_status route_impl(const flarepp_shape* shape, const void* seeds, const void* Kt,
                           const void* Vt, const void* K, const void* V, float scale, void* Y,
                           void* workspace, size_t workspace_bytes, void* stream, float* Q_out,
-                          float* Z_out, void* const* events, int n_events) {
+                          float* Z_out, void* const* events, int n_events,
+                          bool reset_status = true) {
     Plan p;
     flarepp_status stt = make_plan(shape, &p);
     if (stt != FLAREPP_OK) return stt;
@@ -191,7 +192,7 @@ flarepp_status route_impl(const flarepp_shape* shape, const void* seeds, const v
         return tc ? tc_encode(p, call, k, v, seeds, scale, ws, st)
                   : simt_encode_f32(p, call, k, v, seeds, scale, ws, st);
     };
-    if (cudaMemsetAsync(ws + p.off_status, 0, sizeof(int32_t), st) != cudaSuccess)
+    if (reset_status && cudaMemsetAsync(ws + p.off_status, 0, sizeof(int32_t), st) != cudaSuccess)
         return FLAREPP_ERR_CUDA;
     if (tc && neg &&
         negate_bf16(seeds, ws + p.off_seedneg, p.H * p.M * p.D, st) != cudaSuccess)
@@ -211,6 +212,187 @@ flarepp_status route_impl(const flarepp_shape* shape, const void* seeds, const v
                      cudaSuccess)
         return FLAREPP_ERR_CUDA;
     return FLAREPP_OK;
+}
+
+// ---------------------------------------------------------------- the chain on host buffers
+
+// Heads of one pipeline group: a run of consecutive (b, h) slices, either a block of heads
+// of one batch element or whole batch elements (so that every group is a valid shape).
+struct HostGroups {
+    int64_t len;  // (b, h) slices per group
+    int64_t n;    // groups
+};
+
+HostGroups host_groups(const Plan& p) {
+    constexpr int64_t kTarget = 4;  // enough to overlap copies with compute
+    const int64_t bh = p.BH;
+    int64_t want = (bh + kTarget - 1) / kTarget;
+    if (want < 1) want = 1;
+    int64_t len;
+    if (want >= p.H) {
+        len = (want + p.H - 1) / p.H * p.H;  // whole batch elements
+    } else {
+        len = p.H;  // the smallest divisor of H that is at least `want`
+        for (int64_t d = want; d <= p.H; ++d)
+            if (p.H % d == 0) {
+                len = d;
+                break;
+            }
+    }
+    if (len > bh) len = bh;
+    HostGroups g;
+    g.len = len;
+    g.n = (bh + len - 1) / len;
+    return g;
+}
+
+// Layout of the device buffer of flarepp_route_fwd_host: the workspace of one group first
+// (so that its status word sits at offset 0), then the device copies of the inputs and Y.
+struct HostLayout {
+    flarepp_shape group;  // shape of a full group
+    size_t ws_bytes;
+    size_t off_seeds, off_kt, off_vt, off_k, off_v, off_y, total;
+};
+
+bool host_layout(const flarepp_shape* s, const Plan& p, const HostGroups& g, HostLayout* L) {
+    const size_t elt = p.dtype == FLAREPP_F32 ? 4 : 2;
+    const size_t tok = (size_t)p.BH * (size_t)p.N * (size_t)p.D * elt;
+    const size_t seed = (size_t)p.H * (size_t)p.M * (size_t)p.D * elt;
+    L->group = *s;
+    if (g.len >= p.H) {
+        L->group.B = g.len / p.H;
+    } else {
+        L->group.B = 1;
+        L->group.H = g.len;
+    }
+    Plan gp;
+    if (make_plan(&L->group, &gp) != FLAREPP_OK) return false;
+    L->ws_bytes = gp.total;
+    const int64_t last = p.BH - (g.n - 1) * g.len;  // a shorter last group of batch elements
+    if (last != g.len) {
+        flarepp_shape ls = L->group;
+        ls.B = last / p.H;
+        if (make_plan(&ls, &gp) != FLAREPP_OK) return false;
+        if (gp.total > L->ws_bytes) L->ws_bytes = gp.total;
+    }
+    size_t off = align_up(L->ws_bytes, kWsAlign);
+    L->off_seeds = off;
+    off = align_up(off + seed, kWsAlign);
+    L->off_kt = off;
+    off = align_up(off + tok, kWsAlign);
+    L->off_vt = off;
+    off = align_up(off + tok, kWsAlign);
+    L->off_k = off;
+    off = align_up(off + tok, kWsAlign);
+    L->off_v = off;
+    off = align_up(off + tok, kWsAlign);
+    L->off_y = off;
+    off = align_up(off + tok, kWsAlign);
+    L->total = off;
+    return true;
+}
+
+flarepp_status route_host_impl(const flarepp_shape* shape, const void* seeds_h, const void* Kt_h,
+                               const void* Vt_h, const void* K_h, const void* V_h, float scale,
+                               void* Y_h, void* dbuf, size_t dbuf_bytes, void* stream) {
+    Plan p;
+    flarepp_status stt = make_plan(shape, &p);
+    if (stt != FLAREPP_OK) return stt;
+    if (!isfinite(scale)) return FLAREPP_ERR_INVALID_ARGUMENT;
+    if (p.BH == 0 || p.N == 0) return FLAREPP_OK;  // Y is empty
+    const size_t elt = p.dtype == FLAREPP_F32 ? 4 : 2;
+    const size_t tok = (size_t)p.BH * (size_t)p.N * (size_t)p.D * elt;
+    const size_t seed = (size_t)p.H * (size_t)p.M * (size_t)p.D * elt;
+    {
+        const void* ptrs[5] = {Kt_h, Vt_h, K_h, V_h, Y_h};
+        for (const void* q : ptrs)
+            if (!q) return FLAREPP_ERR_INVALID_ARGUMENT;
+        const void* ins[4] = {Kt_h, Vt_h, K_h, V_h};
+        for (const void* q : ins)
+            if (overlaps(Y_h, tok, q, tok)) return FLAREPP_ERR_INVALID_ARGUMENT;
+        if (seed && (!seeds_h || overlaps(Y_h, tok, seeds_h, seed)))
+            return FLAREPP_ERR_INVALID_ARGUMENT;
+    }
+    const HostGroups g = host_groups(p);
+    HostLayout L;
+    if (!host_layout(shape, p, g, &L)) return FLAREPP_ERR_UNSUPPORTED;
+    if (!dbuf || ((uintptr_t)dbuf % kWsAlign) != 0 || dbuf_bytes < L.total)
+        return FLAREPP_ERR_WORKSPACE;
+    char* db = (char*)dbuf;
+    cudaStream_t st = (cudaStream_t)stream;
+
+    // two streams of the library's own (inputs in, Y out) and the events that order them
+    // against `stream`; each is released when its work is done
+    constexpr int kMaxEvents = 2 * 64 + 2;
+    cudaStream_t cin = nullptr, cout = nullptr;
+    cudaEvent_t ev[kMaxEvents] = {};
+    int n_ev = 0;
+    if (g.n > 64) return FLAREPP_ERR_UNSUPPORTED;  // not reached: host_groups targets 4
+    flarepp_status rc = FLAREPP_OK;
+    auto cleanup = [&]() {
+        for (int i = 0; i < n_ev; ++i) cudaEventDestroy(ev[i]);
+        if (cin) cudaStreamDestroy(cin);
+        if (cout) cudaStreamDestroy(cout);
+    };
+    auto new_event = [&](cudaEvent_t* e) {
+        if (cudaEventCreateWithFlags(e, cudaEventDisableTiming) != cudaSuccess) return false;
+        ev[n_ev++] = *e;
+        return true;
+    };
+    cudaEvent_t e_start, e_end;
+    if (cudaStreamCreateWithFlags(&cin, cudaStreamNonBlocking) != cudaSuccess ||
+        cudaStreamCreateWithFlags(&cout, cudaStreamNonBlocking) != cudaSuccess ||
+        !new_event(&e_start) || !new_event(&e_end)) {
+        cleanup();
+        return FLAREPP_ERR_CUDA;
+    }
+    const size_t gtok = (size_t)g.len * (size_t)p.N * (size_t)p.D * elt;  // bytes of a group
+    bool ok = cudaEventRecord(e_start, st) == cudaSuccess &&
+              cudaStreamWaitEvent(cin, e_start, 0) == cudaSuccess &&
+              cudaStreamWaitEvent(cout, e_start, 0) == cudaSuccess;
+    if (ok && seed)
+        ok = cudaMemcpyAsync(db + L.off_seeds, seeds_h, seed, cudaMemcpyHostToDevice, cin) ==
+             cudaSuccess;
+    // inputs of every group, in order, on the input stream
+    cudaEvent_t e_in[64], e_done[64];
+    for (int64_t k = 0; ok && k < g.n; ++k) {
+        const size_t o = (size_t)k * gtok;
+        const size_t n = o + gtok <= tok ? gtok : tok - o;
+        const void* src[4] = {Kt_h, Vt_h, K_h, V_h};
+        const size_t dst[4] = {L.off_kt, L.off_vt, L.off_k, L.off_v};
+        for (int t = 0; ok && t < 4; ++t)
+            ok = cudaMemcpyAsync(db + dst[t] + o, (const char*)src[t] + o, n,
+                                 cudaMemcpyHostToDevice, cin) == cudaSuccess;
+        ok = ok && new_event(&e_in[k]) && new_event(&e_done[k]) &&
+             cudaEventRecord(e_in[k], cin) == cudaSuccess;
+    }
+    // the chain of each group on `stream`, and its Y back on the output stream
+    for (int64_t k = 0; ok && k < g.n; ++k) {
+        const int64_t bh0 = k * g.len;
+        const int64_t len = bh0 + g.len <= p.BH ? g.len : p.BH - bh0;
+        flarepp_shape gs = L.group;
+        if (len >= p.H) gs.B = len / p.H;  // a shorter last group of whole batch elements
+        const size_t o = (size_t)bh0 * (size_t)p.N * (size_t)p.D * elt;
+        const size_t n = (size_t)len * (size_t)p.N * (size_t)p.D * elt;
+        const size_t so = (size_t)(bh0 % p.H) * (size_t)p.M * (size_t)p.D * elt;
+        ok = cudaStreamWaitEvent(st, e_in[k], 0) == cudaSuccess;
+        if (!ok) break;
+        rc = route_impl(&gs, db + L.off_seeds + so, db + L.off_kt + o, db + L.off_vt + o,
+                        db + L.off_k + o, db + L.off_v + o, scale, db + L.off_y + o, db,
+                        L.ws_bytes, st, nullptr, nullptr, nullptr, 0, k == 0);
+        if (rc != FLAREPP_OK) break;
+        ok = cudaEventRecord(e_done[k], st) == cudaSuccess &&
+             cudaStreamWaitEvent(cout, e_done[k], 0) == cudaSuccess &&
+             cudaMemcpyAsync((char*)Y_h + o, db + L.off_y + o, n, cudaMemcpyDeviceToHost, cout) ==
+                 cudaSuccess;
+    }
+    // later work on `stream` follows the last copy of Y
+    if (ok && rc == FLAREPP_OK)
+        ok = cudaEventRecord(e_end, cout) == cudaSuccess &&
+             cudaStreamWaitEvent(st, e_end, 0) == cudaSuccess;
+    cleanup();
+    if (rc != FLAREPP_OK) return rc;
+    return ok ? FLAREPP_OK : FLAREPP_ERR_CUDA;
 }
 
 }  // namespace
@@ -265,6 +447,24 @@ flarepp_status flarepp_route_device_status(const flarepp_shape* shape, const voi
         cudaStreamSynchronize(st) != cudaSuccess)
         return FLAREPP_ERR_CUDA;
     return FLAREPP_OK;
+}
+
+size_t flarepp_route_host_buffer_bytes(const flarepp_shape* shape) {
+    flarepp::Plan p;
+    if (flarepp::make_plan(shape, &p) != FLAREPP_OK) return 0;
+    if (p.BH == 0 || p.N == 0) return 0;
+    const flarepp::HostGroups g = flarepp::host_groups(p);
+    flarepp::HostLayout L;
+    if (!flarepp::host_layout(shape, p, g, &L)) return 0;
+    return L.total;
+}
+
+flarepp_status flarepp_route_fwd_host(const flarepp_shape* shape, const void* seeds,
+                                      const void* Kt, const void* Vt, const void* K,
+                                      const void* V, float scale, void* Y, void* device_buffer,
+                                      size_t device_buffer_bytes, void* stream) {
+    return flarepp::route_host_impl(shape, seeds, Kt, Vt, K, V, scale, Y, device_buffer,
+                                    device_buffer_bytes, stream);
 }
 
 const char* flarepp_status_string(flarepp_status status) {

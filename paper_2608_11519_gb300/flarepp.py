@@ -23,6 +23,7 @@ _DTYPES = {torch.float32: F32, torch.bfloat16: BF16}
 
 EXPORTED = ("flarepp_route_workspace_bytes", "flarepp_route_fwd", "flarepp_route_fwd_debug",
             "flarepp_route_fwd_profiled", "flarepp_route_fwd_noalloc",
+            "flarepp_route_host_buffer_bytes", "flarepp_route_fwd_host",
             "flarepp_route_device_status", "flarepp_status_string", "flarepp_version")
 N_STAGE_EVENTS = 6
 STAGES = ("encode1", "combine1", "encode2", "combine2", "decode")
@@ -71,6 +72,10 @@ def load(path: str = None):
                                                vp, ctypes.POINTER(ctypes.c_void_p), ctypes.c_int]
     lib.flarepp_route_fwd_noalloc.restype = ctypes.c_int
     lib.flarepp_route_fwd_noalloc.argtypes = [sp, vp, vp, vp, vp, vp, ctypes.c_float, vp, vp]
+    lib.flarepp_route_host_buffer_bytes.restype = sz
+    lib.flarepp_route_host_buffer_bytes.argtypes = [sp]
+    lib.flarepp_route_fwd_host.restype = ctypes.c_int
+    lib.flarepp_route_fwd_host.argtypes = [sp, vp, vp, vp, vp, vp, ctypes.c_float, vp, vp, sz, vp]
     lib.flarepp_route_device_status.restype = ctypes.c_int
     lib.flarepp_route_device_status.argtypes = [sp, vp, vp, ctypes.POINTER(ctypes.c_int32)]
     lib.flarepp_status_string.restype = ctypes.c_char_p
@@ -265,29 +270,36 @@ def route_fwd_debug(seeds, Kt, Vt, K, V, scale=None, Y=None, workspace=None, str
 
 def route_fwd_host(seeds, Kt, Vt, K, V, scale=None, Y_host=None, device="cuda", workspace=None,
                    stream=None, dev_bufs=None):
-    """End-to-end call on host tensors: copies the inputs to the device, runs the chain and
-    copies Y back into ``Y_host`` (pinned if allocated here). Returns Y_host after the copy
-    has completed. ``dev_bufs`` (a dict) keeps device buffers between calls."""
-    dev = torch.device(device)
-    bufs = dev_bufs if dev_bufs is not None else {}
-    names = ("seeds", "Kt", "Vt", "K", "V")
-    hs = dict(zip(names, (seeds, Kt, Vt, K, V)))
-    ds = {}
-    for n in names:
-        h = hs[n]
-        d = bufs.get(n)
-        if d is None or d.shape != h.shape or d.dtype != h.dtype:
-            d = torch.empty(h.shape, dtype=h.dtype, device=dev)
-            bufs[n] = d
-        d.copy_(h, non_blocking=True)
-        ds[n] = d
-    Yd = bufs.get("Y")
-    if Yd is None or Yd.shape != K.shape or Yd.dtype != K.dtype:
-        Yd = torch.empty(K.shape, dtype=K.dtype, device=dev)
-        bufs["Y"] = Yd
-    route_fwd(ds["seeds"], ds["Kt"], ds["Vt"], ds["K"], ds["V"], scale, Yd, workspace, stream)
+    """End-to-end call on host tensors through ``flarepp_route_fwd_host``: the library copies
+    the inputs to the device, runs the chain and copies Y back into ``Y_host`` (allocated
+    pinned here if not given), overlapping the copies with the computation by head groups.
+    Pass pinned host tensors for the copies to overlap. Returns Y_host once the copy has
+    completed. ``workspace`` (a :class:`Workspace`) holds the device buffer between calls;
+    ``dev_bufs`` is accepted for compatibility and unused."""
+    del dev_bufs
+    lib = load()
+    shape = _shape_of(seeds, Kt, Vt, K, V)
+    for t in (seeds, Kt, Vt, K, V):
+        if t.is_cuda:
+            raise ValueError("route_fwd_host takes host tensors")
+    if scale is None:
+        scale = 1.0 / math.sqrt(shape.D)
     if Y_host is None:
         Y_host = torch.empty(K.shape, dtype=K.dtype, pin_memory=True)
-    Y_host.copy_(Yd, non_blocking=True)
-    torch.cuda.current_stream(dev).synchronize()
+    elif tuple(Y_host.shape) != tuple(K.shape) or Y_host.dtype != K.dtype or Y_host.is_cuda:
+        raise ValueError("Y_host must be a host tensor of K's shape and dtype")
+    dev = torch.device(device)
+    if dev.index is None:
+        dev = torch.device("cuda", torch.cuda.current_device())
+    nbytes = int(lib.flarepp_route_host_buffer_bytes(ctypes.byref(shape)))
+    ws = workspace if workspace is not None else Workspace()
+    buf = ws.get(nbytes, dev) if nbytes else None
+    st = stream if stream is not None else torch.cuda.current_stream(dev)
+    rc = lib.flarepp_route_fwd_host(ctypes.byref(shape), _ptr(seeds), _ptr(Kt), _ptr(Vt), _ptr(K),
+                                    _ptr(V), float(scale), _ptr(Y_host),
+                                    None if buf is None else ctypes.c_void_p(buf.data_ptr()),
+                                    nbytes, ctypes.c_void_p(st.cuda_stream))
+    if rc != 0:
+        raise FlareppError(rc, "flarepp_route_fwd_host")
+    st.synchronize()
     return Y_host

@@ -137,3 +137,30 @@ def test_python_binding_rejects_bad_tensors(lib):
 def test_missing_library_fails_loudly(tmp_path):
     with pytest.raises(RuntimeError):
         flarepp.load(str(tmp_path / "libflarepp.so"))
+
+
+def test_host_entry_sizes_and_rejects_before_any_cuda_call(lib):
+    E = flarepp
+    hb = lambda s: lib.flarepp_route_host_buffer_bytes(ctypes.byref(s))
+    # the device buffer holds a group's workspace plus device copies of the inputs and Y
+    s = S(B=1, H=8, N=5000, M=128, D=32)
+    tok = 1 * 8 * 5000 * 32 * 2
+    assert hb(s) >= 5 * tok and hb(s) % 256 == 0
+    assert hb(S(D=48)) == 0 and hb(S(N=0)) == 0 and hb(S(B=0)) == 0
+
+    def host_call(shape, Y=FAKE + 6 * (1 << 36), buf=FAKE + 7 * (1 << 36), nbytes=None,
+                  scale=0.25):
+        ptrs = [ctypes.c_void_p(FAKE + (i + 1) * (1 << 36)) for i in range(5)]
+        nb = hb(shape) if nbytes is None else nbytes
+        return lib.flarepp_route_fwd_host(ctypes.byref(shape), *ptrs, ctypes.c_float(scale),
+                                          ctypes.c_void_p(Y) if Y else None,
+                                          ctypes.c_void_p(buf) if buf else None, nb, None)
+
+    assert host_call(S(D=48)) == E.ERR_UNSUPPORTED
+    assert host_call(S(), scale=float("nan")) == E.ERR_INVALID_ARGUMENT
+    assert host_call(S(), Y=0) == E.ERR_INVALID_ARGUMENT
+    assert host_call(S(), Y=FAKE + (1 << 36) + 64) == E.ERR_INVALID_ARGUMENT  # Y overlaps Kt
+    assert host_call(S(), buf=0) == E.ERR_WORKSPACE
+    assert host_call(S(), nbytes=1024) == E.ERR_WORKSPACE
+    assert host_call(S(), buf=FAKE + 7 * (1 << 36) + 128) == E.ERR_WORKSPACE  # not aligned
+    assert host_call(S(N=0)) == E.OK  # empty Y: nothing to do

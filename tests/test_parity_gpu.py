@@ -222,6 +222,29 @@ def test_side_stream_and_host_entry():
     _check("Y host entry", _np(Yh), Yo, 1e-5)
 
 
+@pytest.mark.parametrize("B,H,N,M,D,dtype", [
+    (1, 8, 5000, 128, 32, "bf16"),   # four groups of two heads
+    (5, 2, 3000, 100, 16, "bf16"),   # groups of two batch elements, a shorter last group
+    (3, 3, 2000, 64, 64, "bf16"),    # one batch element per group
+    (1, 4, 700, 20, 16, "f32"),      # one head per group, CUDA-core path
+])
+def test_host_entry_pipelined_groups(B, H, N, M, D, dtype):
+    """flarepp_route_fwd_host splits the heads into groups and overlaps copies with compute;
+    every group shape must give the oracle's Y."""
+    w = inputs.Workload("host", B, H, N, M, D, dtype)
+    x = inputs.make_inputs(w, seed=4)
+    f = inputs.to_f64_numpy(x)
+    _, _, Yo = oracle.route(f["seeds"], f["Kt"], f["Vt"], f["K"], f["V"], w.scale)
+    xh = {k: v.pin_memory() for k, v in x.items()}
+    ws = flarepp.Workspace()
+    for _ in range(2):  # the second call reuses the device buffer
+        Yh = flarepp.route_fwd_host(xh["seeds"], xh["Kt"], xh["Vt"], xh["K"], xh["V"], w.scale,
+                                    workspace=ws)
+        _check("Y host pipelined", _np(Yh), Yo, TOL[dtype])
+    st = flarepp.device_status((x["seeds"], x["Kt"], x["Vt"], x["K"], x["V"]), ws)
+    assert st == 0
+
+
 def test_profiled_entry_records_stages():
     w = inputs.get("pde2d").with_(B=1, N=8192)
     x = inputs.make_inputs(w, seed=2, device="cuda")
