@@ -132,7 +132,7 @@ FLAREPP_API size_t flarepp_route_host_buffer_bytes(const flarepp_shape* shape);
  * The routing chain of flarepp_route_fwd (Sec. 3.2, eqs. flarepp_dynamic_query and
  * flarepp_mixer) on HOST buffers: copies the inputs to the device, runs the chain and copies
  * Y back, with the copies overlapped with the computation. The (b, h) slices of the chain are
- * independent, so the heads are processed in up to four groups: while the chain of one group
+ * independent, so the heads are processed in up to eight groups: while the chain of one group
  * runs on `stream`, the next group's inputs are copied in on a second stream and the previous
  * group's Y is copied out on a third.
  *   seeds, Kt, Vt, K, V, Y: host pointers, same layouts and dtypes as flarepp_route_fwd. The

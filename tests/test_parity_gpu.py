@@ -223,8 +223,9 @@ def test_side_stream_and_host_entry():
 
 
 @pytest.mark.parametrize("B,H,N,M,D,dtype", [
-    (1, 8, 5000, 128, 32, "bf16"),   # four groups of two heads
-    (5, 2, 3000, 100, 16, "bf16"),   # groups of two batch elements, a shorter last group
+    (1, 8, 5000, 128, 32, "bf16"),   # eight groups of one head
+    (1, 16, 2000, 64, 32, "bf16"),   # eight groups of two heads
+    (9, 2, 3000, 100, 16, "bf16"),   # groups of two batch elements, a shorter last group
     (3, 3, 2000, 64, 64, "bf16"),    # one batch element per group
     (1, 4, 700, 20, 16, "f32"),      # one head per group, CUDA-core path
 ])
