@@ -123,6 +123,23 @@ FLAREPP_API flarepp_status flarepp_route_fwd_profiled(const flarepp_shape* shape
                                                       int n_events);
 
 /*
+ * FLARE, the fixed-query form of the routing (Sec. 3, eq. prelim_flare_sdpa): per (b, h),
+ *   Z = SDPA(Q_h, K, V)   (softmax over the N tokens, one row per route)
+ *   Y = SDPA(K, Q_h, Z)   (softmax over the M routes, one row per token)
+ * with learned queries Q_h shared by the batch: the routing chain without its first call.
+ *   shape: as for flarepp_route_fwd (M routes per head); workspace: at least
+ *     flarepp_route_workspace_bytes(shape) bytes, 256-byte aligned.
+ *   Q: [H, M, D] in the input dtype. K, V, Y: [B, H, N, D]. Same alignment, aliasing and
+ *     scale rules as flarepp_route_fwd (Y must not overlap K, V, Q or the workspace).
+ *   Z_out: NULL, or float32 [B, H, M, D] device memory that receives Z.
+ * Errors and the device status word: as flarepp_route_fwd.
+ */
+FLAREPP_API flarepp_status flarepp_flare_fwd(const flarepp_shape* shape, const void* Q,
+                                             const void* K, const void* V, float scale, void* Y,
+                                             void* workspace, size_t workspace_bytes,
+                                             void* stream, float* Z_out);
+
+/*
  * Bytes of device memory that flarepp_route_fwd_host needs for `shape` (its workspace plus
  * device copies of the inputs and of Y), or 0 for an invalid shape or an empty Y.
  */
@@ -136,7 +153,8 @@ FLAREPP_API size_t flarepp_route_host_buffer_bytes(const flarepp_shape* shape);
  * runs on `stream`, the next group's inputs are copied in on a second stream and the previous
  * group's Y is copied out on a third.
  *   seeds, Kt, Vt, K, V, Y: host pointers, same layouts and dtypes as flarepp_route_fwd. The
- *     copies overlap the kernels only when the host memory is page-locked (pinned).
+ *     copies overlap the kernels only when the host memory is page-locked (pinned). Passing
+ *     Kt == K and Vt == V (the shared-projection variant, App. cost_model) copies them once.
  *   device_buffer: caller-owned device memory of at least flarepp_route_host_buffer_bytes
  *     bytes, 256-byte aligned (else FLAREPP_ERR_WORKSPACE). It starts with the workspace, so
  *     flarepp_route_device_status(shape, device_buffer, ...) reports a timeout in any group.

@@ -8,6 +8,8 @@ What it computes (FLARE++ paper):
   * ``sdpa``           -- SDPA(Q, K, V) = softmax(s Q K^T) V over the keys (Sec. 2, eq. sdpa_definition)
   * ``route``          -- Q = SDPA(Qseed, Kt, Vt); Z = SDPA(Q, K, V); Y = SDPA(K, Q, Z)
                           (Sec. 3.2, eqs. flarepp_dynamic_query and flarepp_mixer)
+  * ``flare``          -- Z = SDPA(Q_h, K, V); Y = SDPA(K, Q_h, Z) with learned queries Q_h
+                          shared by the batch (Sec. 3, eq. prelim_flare_sdpa)
   * ``encode_sharded`` -- the encoder evaluated shard by shard, then merged by the stable
                           log-sum-exp reduction (App. A.2, A.3)
 
@@ -99,6 +101,21 @@ class Oracle:
             raise MemoryError("oracle scratch allocation failed")
         return Q, Z, Y
 
+    def flare(self, Q, K, V, scale):
+        """FLARE with learned queries (Sec. 3, eq. prelim_flare_sdpa): per (b, h), the encoder
+        Z = SDPA(Q_h, K, V) and the decoder Y = SDPA(K, Q_h, Z), both this oracle's SDPA.
+        Q [H, M, D] is shared by the batch; K, V [B, H, N, D].
+
+        Returns (Z [B, H, M, D], Y [B, H, N, D]).
+        """
+        Q, K, V = self._f64(Q), self._f64(K), self._f64(V)
+        B, H, N, D = K.shape
+        assert Q.shape[0] == H and Q.shape[2] == D and V.shape == K.shape
+        Qb = np.ascontiguousarray(np.broadcast_to(Q, (B,) + Q.shape))
+        Z, _ = self.sdpa(Qb, K, V, scale)
+        Y, _ = self.sdpa(K, Qb, Z, scale)
+        return Z, Y
+
     def encode_sharded(self, q, k, v, scale, chunk, n_empty=0):
         """Encoder over shards of ``chunk`` keys merged by the stable LSE reduction (App. A.3).
 
@@ -138,6 +155,10 @@ def route(seeds, Kt, Vt, K, V, scale):
     return default().route(seeds, Kt, Vt, K, V, scale)
 
 
+def flare(Q, K, V, scale):
+    return default().flare(Q, K, V, scale)
+
+
 def encode_sharded(q, k, v, scale, chunk, n_empty=0):
     return default().encode_sharded(q, k, v, scale, chunk, n_empty)
 
@@ -155,5 +176,5 @@ def build() -> str:
     return _build.build()
 
 
-__all__ = ["Oracle", "default", "sdpa", "route", "encode_sharded", "max_threads",
+__all__ = ["Oracle", "default", "sdpa", "route", "flare", "encode_sharded", "max_threads",
            "set_threads", "build"]

@@ -214,6 +214,75 @@ flarepp_status route_impl(const flarepp_shape* shape, const void* seeds, const v
     return FLAREPP_OK;
 }
 
+// ---------------------------------------------------------------- FLARE (fixed queries)
+
+// FLARE (Sec. 3, eq. prelim_flare_sdpa): Z = SDPA(Q_h, K, V), Y = SDPA(K, Q_h, Z) with learned
+// queries Q [H, M, D] shared by the batch. The routing chain without its first call: the
+// encode runs as call 1 does (A = the per-head queries), its merge writes Z, and the decode
+// reads a per-(b, h) copy of Q as its keys.
+flarepp_status flare_impl(const flarepp_shape* shape, const void* Qh, const void* K, const void* V,
+                          float scale, void* Y, void* workspace, size_t workspace_bytes,
+                          void* stream, float* Z_out) {
+    Plan p;
+    flarepp_status stt = make_plan(shape, &p);
+    if (stt != FLAREPP_OK) return stt;
+    if (!isfinite(scale)) return FLAREPP_ERR_INVALID_ARGUMENT;
+    cudaStream_t st = (cudaStream_t)stream;
+    const size_t elt = p.dtype == FLAREPP_F32 ? 4 : 2;
+    const size_t tok_bytes = (size_t)p.BH * (size_t)p.N * (size_t)p.D * elt;
+    const size_t q_bytes = (size_t)p.H * (size_t)p.M * (size_t)p.D * elt;
+    const size_t z_bytes = (size_t)p.BH * (size_t)p.M * (size_t)p.D * sizeof(float);
+    if (tok_bytes) {
+        const void* ptrs[3] = {K, V, Y};
+        for (const void* q : ptrs)
+            if (!q || !aligned16(q)) return FLAREPP_ERR_INVALID_ARGUMENT;
+        if (overlaps(Y, tok_bytes, K, tok_bytes) || overlaps(Y, tok_bytes, V, tok_bytes) ||
+            overlaps(Y, tok_bytes, Qh, q_bytes))
+            return FLAREPP_ERR_INVALID_ARGUMENT;
+    }
+    if (q_bytes && tok_bytes && (!Qh || !aligned16(Qh))) return FLAREPP_ERR_INVALID_ARGUMENT;
+    if (z_bytes && Z_out && !aligned16(Z_out)) return FLAREPP_ERR_INVALID_ARGUMENT;
+    if (p.total) {
+        if (!workspace || ((uintptr_t)workspace % kWsAlign) != 0) return FLAREPP_ERR_WORKSPACE;
+        if (workspace_bytes < p.total) return FLAREPP_ERR_WORKSPACE;
+        if (overlaps(Y, tok_bytes, workspace, p.total)) return FLAREPP_ERR_INVALID_ARGUMENT;
+    }
+    if (p.BH == 0) return FLAREPP_OK;
+    if (p.N == 0) {  // every route has no keys: Z = 0 (App. A.3); Y is empty
+        if (Z_out && z_bytes && cudaMemsetAsync(Z_out, 0, z_bytes, st) != cudaSuccess)
+            return FLAREPP_ERR_CUDA;
+        return FLAREPP_OK;
+    }
+    if (p.M == 0)
+        return cudaMemsetAsync(Y, 0, tok_bytes, st) == cudaSuccess ? FLAREPP_OK : FLAREPP_ERR_CUDA;
+
+    char* ws = (char*)workspace;
+    const bool tc = p.path == kPathTc;
+    const bool neg = scale < 0.f;
+    if (cudaMemsetAsync(ws + p.off_status, 0, sizeof(int32_t), st) != cudaSuccess)
+        return FLAREPP_ERR_CUDA;
+    // the encode of call 1 with the learned queries, merged into Z
+    if (tc && neg && negate_bf16(Qh, ws + p.off_seedneg, p.H * p.M * p.D, st) != cudaSuccess)
+        return FLAREPP_ERR_CUDA;
+    cudaError_t e = tc ? tc_encode(p, 1, K, V, Qh, scale, ws, st)
+                       : simt_encode_f32(p, 1, K, V, Qh, scale, ws, st);
+    if (e != cudaSuccess || combine(p, 2, ws, false, st) != cudaSuccess) return FLAREPP_ERR_CUDA;
+    // the decode's keys: Q for every batch element (on the tensor-core path the bf16 operand,
+    // negated for a negative scale as the chain's call-1 merge does)
+    const void* qsrc = tc && neg ? (const void*)(ws + p.off_seedneg) : Qh;
+    char* qdst = ws + (tc ? p.off_qop : p.off_q32);
+    for (int64_t b = 0; b < p.B; ++b)
+        if (cudaMemcpyAsync(qdst + (size_t)b * q_bytes, qsrc, q_bytes, cudaMemcpyDeviceToDevice,
+                            st) != cudaSuccess)
+            return FLAREPP_ERR_CUDA;
+    e = tc ? tc_decode(p, K, scale, Y, ws, st) : simt_decode_f32(p, K, scale, Y, ws, st);
+    if (e != cudaSuccess) return FLAREPP_ERR_CUDA;
+    if (Z_out && cudaMemcpyAsync(Z_out, ws + p.off_z32, z_bytes, cudaMemcpyDeviceToDevice, st) !=
+                     cudaSuccess)
+        return FLAREPP_ERR_CUDA;
+    return FLAREPP_OK;
+}
+
 // ---------------------------------------------------------------- the chain on host buffers
 
 // Heads of one pipeline group: a run of consecutive (b, h) slices, either a block of heads
@@ -353,14 +422,18 @@ flarepp_status route_host_impl(const flarepp_shape* shape, const void* seeds_h, 
     if (ok && seed)
         ok = cudaMemcpyAsync(db + L.off_seeds, seeds_h, seed, cudaMemcpyHostToDevice, cin) ==
              cudaSuccess;
-    // inputs of every group, in order, on the input stream
+    // inputs of every group, in order, on the input stream. With the shared projection
+    // (Kt = K and Vt = V on the host, App. cost_model) K and V are copied once and serve as
+    // both pairs.
+    const bool shared = Kt_h == K_h && Vt_h == V_h;
+    const size_t off_kt = shared ? L.off_k : L.off_kt, off_vt = shared ? L.off_v : L.off_vt;
     cudaEvent_t e_in[64], e_done[64];
     for (int64_t k = 0; ok && k < g.n; ++k) {
         const size_t o = (size_t)k * gtok;
         const size_t n = o + gtok <= tok ? gtok : tok - o;
-        const void* src[4] = {Kt_h, Vt_h, K_h, V_h};
-        const size_t dst[4] = {L.off_kt, L.off_vt, L.off_k, L.off_v};
-        for (int t = 0; ok && t < 4; ++t)
+        const void* src[4] = {K_h, V_h, Kt_h, Vt_h};
+        const size_t dst[4] = {L.off_k, L.off_v, L.off_kt, L.off_vt};
+        for (int t = 0; ok && t < (shared ? 2 : 4); ++t)
             ok = cudaMemcpyAsync(db + dst[t] + o, (const char*)src[t] + o, n,
                                  cudaMemcpyHostToDevice, cin) == cudaSuccess;
         ok = ok && new_event(&e_in[k]) && new_event(&e_done[k]) &&
@@ -377,7 +450,7 @@ flarepp_status route_host_impl(const flarepp_shape* shape, const void* seeds_h, 
         const size_t so = (size_t)(bh0 % p.H) * (size_t)p.M * (size_t)p.D * elt;
         ok = cudaStreamWaitEvent(st, e_in[k], 0) == cudaSuccess;
         if (!ok) break;
-        rc = route_impl(&gs, db + L.off_seeds + so, db + L.off_kt + o, db + L.off_vt + o,
+        rc = route_impl(&gs, db + L.off_seeds + so, db + off_kt + o, db + off_vt + o,
                         db + L.off_k + o, db + L.off_v + o, scale, db + L.off_y + o, db,
                         L.ws_bytes, st, nullptr, nullptr, nullptr, 0, k == 0);
         if (rc != FLAREPP_OK) break;
@@ -447,6 +520,13 @@ flarepp_status flarepp_route_device_status(const flarepp_shape* shape, const voi
         cudaStreamSynchronize(st) != cudaSuccess)
         return FLAREPP_ERR_CUDA;
     return FLAREPP_OK;
+}
+
+flarepp_status flarepp_flare_fwd(const flarepp_shape* shape, const void* Q, const void* K,
+                                 const void* V, float scale, void* Y, void* workspace,
+                                 size_t workspace_bytes, void* stream, float* Z_out) {
+    return flarepp::flare_impl(shape, Q, K, V, scale, Y, workspace, workspace_bytes, stream,
+                               Z_out);
 }
 
 size_t flarepp_route_host_buffer_bytes(const flarepp_shape* shape) {

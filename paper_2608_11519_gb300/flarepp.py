@@ -23,7 +23,7 @@ _DTYPES = {torch.float32: F32, torch.bfloat16: BF16}
 
 EXPORTED = ("flarepp_route_workspace_bytes", "flarepp_route_fwd", "flarepp_route_fwd_debug",
             "flarepp_route_fwd_profiled", "flarepp_route_fwd_noalloc",
-            "flarepp_route_host_buffer_bytes", "flarepp_route_fwd_host",
+            "flarepp_flare_fwd", "flarepp_route_host_buffer_bytes", "flarepp_route_fwd_host",
             "flarepp_route_device_status", "flarepp_status_string", "flarepp_version")
 N_STAGE_EVENTS = 6
 STAGES = ("encode1", "combine1", "encode2", "combine2", "decode")
@@ -72,6 +72,8 @@ def load(path: str = None):
                                                vp, ctypes.POINTER(ctypes.c_void_p), ctypes.c_int]
     lib.flarepp_route_fwd_noalloc.restype = ctypes.c_int
     lib.flarepp_route_fwd_noalloc.argtypes = [sp, vp, vp, vp, vp, vp, ctypes.c_float, vp, vp]
+    lib.flarepp_flare_fwd.restype = ctypes.c_int
+    lib.flarepp_flare_fwd.argtypes = [sp, vp, vp, vp, ctypes.c_float, vp, vp, sz, vp, vp]
     lib.flarepp_route_host_buffer_bytes.restype = sz
     lib.flarepp_route_host_buffer_bytes.argtypes = [sp]
     lib.flarepp_route_fwd_host.restype = ctypes.c_int
@@ -266,6 +268,32 @@ def route_fwd_debug(seeds, Kt, Vt, K, V, scale=None, Y=None, workspace=None, str
     Z = torch.empty_like(Q)
     Y = _call(True, seeds, Kt, Vt, K, V, scale, Y, workspace, stream, Q, Z)
     return Y, Q, Z
+
+
+def flare_fwd(Q, K, V, scale=None, Y=None, workspace=None, stream=None, Z_out=None):
+    """FLARE with learned queries (Sec. 3, eq. prelim_flare_sdpa) on device tensors:
+    Z = SDPA(Q_h, K, V), Y = SDPA(K, Q_h, Z). Q [H, M, D] is shared by the batch; K, V
+    [B, H, N, D]. Returns Y; ``Z_out`` (float32 [B, H, M, D], device) receives Z if given."""
+    lib = load()
+    shape = _shape_of(Q, K, V, K, V)
+    if K.device.type != "cuda":
+        raise ValueError("flare_fwd takes device tensors")
+    if scale is None:
+        scale = 1.0 / math.sqrt(shape.D)
+    if Y is None:
+        Y = torch.empty_like(K)
+    if Z_out is not None and (Z_out.dtype != torch.float32 or not Z_out.is_contiguous() or
+                              tuple(Z_out.shape) != (shape.B, shape.H, shape.M, shape.D)):
+        raise ValueError("Z_out must be a contiguous float32 [B, H, M, D] tensor")
+    nbytes = int(lib.flarepp_route_workspace_bytes(ctypes.byref(shape)))
+    ws = (workspace if isinstance(workspace, Workspace) else Workspace()).get(nbytes, K.device)
+    st = stream if stream is not None else torch.cuda.current_stream(K.device)
+    rc = lib.flarepp_flare_fwd(ctypes.byref(shape), _ptr(Q), _ptr(K), _ptr(V), float(scale),
+                               _ptr(Y), None if ws is None else ctypes.c_void_p(ws.data_ptr()),
+                               nbytes, ctypes.c_void_p(st.cuda_stream), _ptr(Z_out))
+    if rc != OK:
+        raise FlareppError(rc, "flarepp_flare_fwd")
+    return Y
 
 
 def route_fwd_host(seeds, Kt, Vt, K, V, scale=None, Y_host=None, device="cuda", workspace=None,

@@ -264,9 +264,62 @@ def pin_large_logits(o):
     np.testing.assert_allclose(Z, Zr, rtol=0, atol=1e-10)
 
 
+def pin_flare_brute_force(o):
+    """FLARE (Sec. 3, eqs. prelim_flare_sdpa and prelim_flare_operator): explicit
+    W_enc = softmax(s Q K^T) (M x N, over tokens) and W_dec = softmax(s K Q^T) (N x M, over
+    routes) give Z = W_enc V and Y = W_dec W_enc V, with rank(W_dec W_enc) <= M; also two
+    torch float64 SDPA calls in the paper's order."""
+    rng = np.random.default_rng(21)
+    for (N, M, D, s) in [(64, 6, 4, 0.7), (150, 16, 8, 0.35), (29, 40, 2, 1.1)]:
+        Q, K, V = _rand(1, M, D, rng=rng), _rand(1, 1, N, D, rng=rng), _rand(1, 1, N, D, rng=rng)
+        Z, Y = o.flare(Q, K, V, s)
+        Wenc = _softmax_rows(s * Q[0] @ K[0, 0].T)
+        Wdec = _softmax_rows(s * K[0, 0] @ Q[0].T)
+        np.testing.assert_allclose(Z[0, 0], Wenc @ V[0, 0], rtol=0, atol=1e-13)
+        np.testing.assert_allclose(Y[0, 0], Wdec @ Wenc @ V[0, 0], rtol=0, atol=1e-13)
+        sv = np.linalg.svd(Wdec @ Wenc, compute_uv=False)
+        if M < N:
+            assert sv[M] / sv[0] < 1e-12
+        Zr = _torch_sdpa(Q[None], K, V, s)
+        np.testing.assert_allclose(Y, _torch_sdpa(K, Q[None], Zr, s), rtol=0, atol=1e-12)
+
+
+def pin_flare_is_the_chain_without_call_one(o):
+    """FLARE++ is FLARE whose queries come from call 1 (Sec. 3.2): the chain's Z and Y equal
+    FLARE's on the chain's own Q; for B > 1 the learned Q is shared by the batch."""
+    rng = np.random.default_rng(22)
+    for (N, M, D) in [(70, 8, 4), (33, 3, 8)]:
+        s = 1.0 / math.sqrt(D)
+        seeds, Kt, Vt, K, V = _chain_inputs(1, 2, N, M, D, rng)
+        Q, Z, Y = o.route(seeds, Kt, Vt, K, V, s)
+        Zf, Yf = o.flare(Q[0], K, V, s)
+        np.testing.assert_allclose(Zf, Z, rtol=0, atol=1e-14)
+        np.testing.assert_allclose(Yf, Y, rtol=0, atol=1e-14)
+    Qh = _rand(2, 5, 4, rng=rng)
+    K, V = _rand(3, 2, 20, 4, rng=rng), _rand(3, 2, 20, 4, rng=rng)
+    Z, Y = o.flare(Qh, K, V, 0.5)
+    for b in range(3):
+        Zb, Yb = o.flare(Qh, K[b:b + 1], V[b:b + 1], 0.5)
+        np.testing.assert_allclose(Z[b:b + 1], Zb, rtol=0, atol=0)
+        np.testing.assert_allclose(Y[b:b + 1], Yb, rtol=0, atol=0)
+
+
+def pin_flare_closed_forms(o):
+    """scale 0: every route and token averages V uniformly; one route: every token gets Z."""
+    rng = np.random.default_rng(23)
+    Q, K, V = _rand(2, 6, 4, rng=rng), _rand(1, 2, 25, 4, rng=rng), _rand(1, 2, 25, 4, rng=rng)
+    Z, Y = o.flare(Q, K, V, 0.0)
+    mean = V.mean(axis=2, keepdims=True)
+    np.testing.assert_allclose(Z, np.broadcast_to(mean, Z.shape), rtol=0, atol=1e-14)
+    np.testing.assert_allclose(Y, np.broadcast_to(mean, Y.shape), rtol=0, atol=1e-14)
+    Z, Y = o.flare(Q[:, :1], K, V, 0.8)
+    np.testing.assert_allclose(Y, np.broadcast_to(Z, Y.shape), rtol=0, atol=1e-14)
+
+
 PINS = [pin_sdpa_vs_torch, pin_route_vs_torch_three_calls, pin_brute_force_matrices,
         pin_rank_and_stochastic, pin_convex_hull, pin_constant_values, pin_closed_forms,
-        pin_two_token_hand_example, pin_symmetries, pin_sharded_merge, pin_large_logits]
+        pin_two_token_hand_example, pin_symmetries, pin_sharded_merge, pin_large_logits,
+        pin_flare_brute_force, pin_flare_is_the_chain_without_call_one, pin_flare_closed_forms]
 
 
 @pytest.mark.parametrize("pin", PINS, ids=[p.__name__ for p in PINS])

@@ -246,6 +246,45 @@ def test_host_entry_pipelined_groups(B, H, N, M, D, dtype):
     assert st == 0
 
 
+@pytest.mark.parametrize("B,H,N,M,D,dtype,scale", [
+    (1, 2, 3000, 128, 32, "bf16", None),
+    (2, 3, 2000, 100, 16, "bf16", -0.3),    # negative scale: negated query operands
+    (1, 2, 5000, 700, 64, "bf16", None),    # two route groups, 32-route items
+    (1, 1, 64, 512, 32, "bf16", None),      # one token item
+    (2, 2, 700, 20, 16, "f32", None),       # CUDA-core path
+])
+def test_flare_fixed_queries(B, H, N, M, D, dtype, scale):
+    """FLARE (Sec. 3, eq. prelim_flare_sdpa): Z = SDPA(Q_h, K, V), Y = SDPA(K, Q_h, Z)."""
+    w = inputs.Workload("flare", B, H, N, M, D, dtype)
+    s = w.scale if scale is None else scale
+    x = inputs.make_inputs(w, seed=5)
+    f = inputs.to_f64_numpy(x)
+    Zo, Yo = oracle.flare(f["seeds"], f["K"], f["V"], s)
+    xd = {k: v.cuda() for k, v in x.items()}
+    Z = torch.empty((B, H, M, D), dtype=torch.float32, device="cuda")
+    Y = flarepp.flare_fwd(xd["seeds"], xd["K"], xd["V"], s, Z_out=Z)
+    torch.cuda.synchronize()
+    _check("Z", _np(Z), Zo, TOL[dtype])
+    _check("Y", _np(Y), Yo, TOL[dtype])
+
+
+def test_shared_projection():
+    """The shared-projection variant ties Kt, Vt to K, V (App. cost_model): the chain on
+    aliased inputs, on device buffers and through the host entry (which copies K, V once)."""
+    w = inputs.get("pde2d").with_(B=1, H=2, N=6000)
+    x = inputs.make_inputs(w, seed=6)
+    f = inputs.to_f64_numpy(x)
+    Qo, Zo, Yo = oracle.route(f["seeds"], f["K"], f["V"], f["K"], f["V"], w.scale)
+    xd = {k: v.cuda() for k, v in x.items()}
+    Y, Q, Z = flarepp.route_fwd_debug(xd["seeds"], xd["K"], xd["V"], xd["K"], xd["V"], w.scale)
+    torch.cuda.synchronize()
+    for n, g, o in (("Q", Q, Qo), ("Z", Z, Zo), ("Y", Y, Yo)):
+        _check(n, _np(g), o, TOL["bf16"])
+    xh = {k: v.pin_memory() for k, v in x.items()}
+    Yh = flarepp.route_fwd_host(xh["seeds"], xh["K"], xh["V"], xh["K"], xh["V"], w.scale)
+    _check("Y host shared", _np(Yh), Yo, TOL["bf16"])
+
+
 def test_profiled_entry_records_stages():
     w = inputs.get("pde2d").with_(B=1, N=8192)
     x = inputs.make_inputs(w, seed=2, device="cuda")
