@@ -30,7 +30,11 @@ from paper_2608_11519_gb300 import inputs  # noqa: E402
 
 METRIC = "routed tokens·heads/sec for the 3-call FLARE++ chain; % of roofline"
 UNIT = "token·heads/s"
-KERNEL_SOURCES = ("paper_2608_11519_gb300/csrc",)
+# the files that fix what a kernel launch reads and writes: the kernels and the plan that
+# sets their launch configuration (the C ABI's argument handling is not among them)
+KERNEL_SOURCES = tuple("paper_2608_11519_gb300/csrc/" + f for f in (
+    "combine.cu", "flarepp_internal.h", "plan.cu", "simt_f32.cu", "simt_kernels.cuh",
+    "tc_kernels.cu", "tc_ptx.cuh"))
 FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0,
                   "source": "fallback"}
 
@@ -49,11 +53,9 @@ def load_peaks():
 
 def kernel_source_hash():
     h = hashlib.sha256()
-    for d in KERNEL_SOURCES:
-        full = os.path.join(ROOT, d)
-        for name in sorted(os.listdir(full)):
-            with open(os.path.join(full, name), "rb") as f:
-                h.update(name.encode() + f.read())
+    for rel in KERNEL_SOURCES:
+        with open(os.path.join(ROOT, rel), "rb") as f:
+            h.update(os.path.basename(rel).encode() + f.read())
     return h.hexdigest()[:16]
 
 
@@ -177,20 +179,30 @@ def max_over_ranks(x, world):
 
 # ------------------------------------------------------------------ CPU baseline (oracle)
 
-def cpu_oracle_sample(w, target_s, seed=0):
+def oracle_call(f, w, variant):
+    """The float64 oracle of the benchmarked variant on numpy inputs."""
+    import oracle
+    if variant == "flare":
+        return oracle.flare(f["seeds"], f["K"], f["V"], w.scale)
+    if variant == "shared":
+        return oracle.route(f["seeds"], f["K"], f["V"], f["K"], f["V"], w.scale)
+    return oracle.route(f["seeds"], f["Kt"], f["Vt"], f["K"], f["V"], w.scale)
+
+
+def cpu_oracle_sample(w, target_s, seed=0, variant="flarepp"):
     """Time the float64 oracle on one (b, h) slice with a token prefix of the workload,
     sized from a short probe to take about ``target_s`` seconds. Returns a cpu_baseline dict."""
     import oracle
     x = inputs.make_inputs(w.with_(B=1, H=1, N=min(w.N, 4096)), seed)
     f = inputs.to_f64_numpy(x)
     t0 = time.perf_counter()
-    oracle.route(f["seeds"], f["Kt"], f["Vt"], f["K"], f["V"], w.scale)
+    oracle_call(f, w, variant)
     probe = time.perf_counter() - t0
     n = int(min(w.N, max(1024, f["K"].shape[2] * target_s / max(probe, 1e-3))))
     x = inputs.make_inputs(w.with_(B=1, H=1, N=n), seed)
     f = inputs.to_f64_numpy(x)
     t0 = time.perf_counter()
-    oracle.route(f["seeds"], f["Kt"], f["Vt"], f["K"], f["V"], w.scale)
+    oracle_call(f, w, variant)
     dt = time.perf_counter() - t0
     return {"value": n / dt, "unit": UNIT, "cores": oracle.max_threads(), "kind": "oracle",
             "sample": f"one head, N={n} tokens of the {w.name} shape (M={w.M}, D={w.D}), "
@@ -209,19 +221,21 @@ def run_reference(args, w):
     x = inputs.make_inputs(w.with_(B=1, H=1, N=n), args.seed)
     f = inputs.to_f64_numpy(x)
     for _ in range(args.warmup):
-        oracle.route(f["seeds"], f["Kt"], f["Vt"], f["K"], f["V"], w.scale)
+        oracle_call(f, w, args.variant)
     t0 = time.perf_counter()
     for _ in range(args.steps):
-        oracle.route(f["seeds"], f["Kt"], f["Vt"], f["K"], f["V"], w.scale)
+        oracle_call(f, w, args.variant)
     dt = (time.perf_counter() - t0) / args.steps
     value = n / dt
     sample = (f"one head, N={n} tokens of the {w.name} shape (M={w.M}, D={w.D}), float64 oracle "
               f"on the host cores, per step")
-    line = {"impl": "reference", "metric": METRIC, "value": value, "unit": UNIT,
+    metric = FLARE_METRIC if args.variant == "flare" else METRIC
+    line = {"impl": "reference", "metric": metric, "value": value, "unit": UNIT,
             "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
             "ms_per_step": dt * 1e3, "higher_is_better": True, "scaling": "weak",
             "vs_baseline": None, "dtype": "f64", "data": "synthetic",
-            "config": {"workload": w.name, "B": w.B, "H": w.H, "N": w.N, "M": w.M, "D": w.D,
+            "config": {"workload": w.name, "variant": args.variant,
+                       "B": w.B, "H": w.H, "N": w.N, "M": w.M, "D": w.D,
                        "input_dtype": w.dtype, "sample_tokens": n},
             "cpu_baseline": {"value": value, "unit": UNIT, "cores": oracle.max_threads(),
                              "kind": "oracle", "sample": sample},
@@ -232,6 +246,118 @@ def run_reference(args, w):
 
 
 # ------------------------------------------------------------------ our arm
+
+FLARE_METRIC = "routed tokens·heads/sec for the 2-call FLARE layer (fixed queries); % of roofline"
+
+
+def flare_launches(w):
+    """Kernels of one FLARE call: encode, merge and decode, plus the negation of the
+    bf16 queries when the scale is negative."""
+    return 3 + (1 if w.dtype == "bf16" and w.scale < 0 else 0)
+
+
+def run_flare(args, w, flarepp, world, rank, dev, peaks, x, Y, ws, stream):
+    """FLARE (Sec. 3, eq. prelim_flare_sdpa) with the seeds as the learned queries: whole
+    calls timed with CUDA events (a call is one encode, one merge and one decode)."""
+    Q, K, V = x["seeds"], x["K"], x["V"]
+    for _ in range(args.warmup):
+        flarepp.flare_fwd(Q, K, V, w.scale, Y=Y, workspace=ws, stream=stream)
+    torch.cuda.synchronize(dev)
+    clocks = ClockSampler()
+    if rank == 0:
+        clocks.start()
+        time.sleep(0.3)
+    t0 = torch.cuda.Event(enable_timing=True)
+    t1 = torch.cuda.Event(enable_timing=True)
+    barrier(world)
+    torch.cuda.synchronize(dev)
+    t0.record(stream)
+    for _ in range(args.steps):
+        flarepp.flare_fwd(Q, K, V, w.scale, Y=Y, workspace=ws, stream=stream)
+    t1.record(stream)
+    torch.cuda.synchronize(dev)
+    barrier(world)
+    clk = clocks.stop(dev.index) if rank == 0 else None
+    ms = max_over_ranks(t0.elapsed_time(t1), world) / args.steps
+    tok = w.B * w.H * w.N
+    value = tok * world / (ms * 1e-3)
+    # algorithmic work of a call: 8 BNMHD flops (two token-latent SDPA calls); K, V read
+    # and Y written, 3 BHND elements
+    flops = 8.0 * tok * w.M * w.D
+    byts = 3.0 * tok * w.D * w.elt_bytes
+    tc_peak = peaks["bf16_tflops_sustained"] if w.dtype == "bf16" else None
+    bw = peaks["hbm_gbs"]
+    t_tc = flops / (tc_peak * 1e12) if tc_peak else 0.0
+    t_mem = byts / (bw * 1e9)
+    if t_tc >= t_mem and tc_peak:
+        roof = {"bound": "tensor", "achieved": flops / (ms * 1e-3) / 1e12, "peak": tc_peak,
+                "unit": "TFLOP/s", "peak_kind": "bf16_tflops_sustained (" + peaks["source"] + ")"}
+    else:
+        roof = {"bound": "hbm", "achieved": byts / (ms * 1e-3) / 1e9, "peak": bw, "unit": "GB/s",
+                "peak_kind": "hbm_gbs (" + peaks["source"] + ")"}
+    roof["frac"] = roof["achieved"] / roof["peak"]
+    roof["kernel"] = "whole call (encode, merge, decode)"
+    roof["ms_per_launch"] = ms
+    roof["algorithmic_flops_per_launch"] = flops
+    roof["algorithmic_bytes_per_launch"] = byts
+    roof["traffic"] = None
+    e2e = None
+    if not args.no_e2e:
+        xh = {k: x[k].to("cpu").pin_memory() for k in ("seeds", "K", "V")}
+        dv = {k: torch.empty_like(x[k]) for k in xh}
+        Yh = torch.empty(Y.shape, dtype=Y.dtype, pin_memory=True)
+
+        def e2e_call():
+            with torch.cuda.stream(stream):
+                for k in xh:
+                    dv[k].copy_(xh[k], non_blocking=True)
+            flarepp.flare_fwd(dv["seeds"], dv["K"], dv["V"], w.scale, Y=Y, workspace=ws,
+                              stream=stream)
+            with torch.cuda.stream(stream):
+                Yh.copy_(Y, non_blocking=True)
+            stream.synchronize()
+
+        for _ in range(2):
+            e2e_call()
+        n_e2e = max(1, min(args.steps, args.e2e_steps))
+        e0 = torch.cuda.Event(enable_timing=True)
+        e1 = torch.cuda.Event(enable_timing=True)
+        barrier(world)
+        torch.cuda.synchronize(dev)
+        e0.record(stream)
+        for _ in range(n_e2e):
+            e2e_call()
+        e1.record(stream)
+        torch.cuda.synchronize(dev)
+        e2e_ms = max_over_ranks(e0.elapsed_time(e1) / n_e2e, world)
+        e2e = {"value": tok * world / (e2e_ms * 1e-3), "unit": UNIT, "ms_per_step": e2e_ms,
+               "steps": n_e2e, "copies": "serial on the call's stream",
+               "h2d_bytes_per_step": sum(t.numel() * t.element_size() for t in xh.values()),
+               "d2h_bytes_per_step": Yh.numel() * Yh.element_size()}
+        del xh, dv, Yh
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        cpu = cpu_oracle_sample(w, args.cpu_seconds, args.seed, "flare")
+    if rank == 0:
+        line = {
+            "metric": FLARE_METRIC, "value": value, "unit": UNIT, "n_gpus": world,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+            "dtype": "bf16" if w.dtype == "bf16" else "f32", "data": "synthetic",
+            "config": {"workload": w.name, "variant": "flare", "B": w.B, "H": w.H, "N": w.N,
+                       "M": w.M, "D": w.D, "queries": "the workload's seeds, as learned queries",
+                       "l2": "inputs larger than L2 (no flush)"
+                       if 3 * tok * w.D * w.elt_bytes > 2 * 129e6 else "inputs near L2 size",
+                       "parallelism": f"replicas x{world}"},
+            "roofline": roof, "cpu_baseline": cpu, "e2e": e2e, "clocks": clk,
+            "gpu_launches": flare_launches(w) * args.steps,
+        }
+        print(json.dumps(line), flush=True)
+    if world > 1:
+        import torch.distributed as dist
+        dist.destroy_process_group()
+    return 0
+
 
 def run_ours(args, w):
     from paper_2608_11519_gb300 import flarepp
@@ -246,6 +372,10 @@ def run_ours(args, w):
     ws = flarepp.Workspace()
     stream = torch.cuda.current_stream(dev)
     args_ = (x["seeds"], x["Kt"], x["Vt"], x["K"], x["V"])
+    if args.variant == "shared":  # Kt, Vt tied to K, V (App. cost_model)
+        args_ = (x["seeds"], x["K"], x["V"], x["K"], x["V"])
+    if args.variant == "flare":
+        return run_flare(args, w, flarepp, world, rank, dev, peaks, x, Y, ws, stream)
 
     ev_sets = [flarepp.StageEvents(stream) for _ in range(args.steps)]
     warm_ev = flarepp.StageEvents(stream)
@@ -297,10 +427,12 @@ def run_ours(args, w):
     roof["algorithmic_bytes_per_launch"] = byts
     roof["traffic"] = recorded_traffic(w.name, dominant)
 
-    # whole-chain roofline: max(12 BNMHD / tensor peak, 5 BHND elt / HBM)
+    # whole-chain roofline: max(12 BNMHD / tensor peak, 5 BHND elt / HBM); the shared
+    # projection streams 3 token tensors (K, V, Y) instead of 5
     tok = w.B * w.H * w.N
+    n_tensors = 3.0 if args.variant == "shared" else 5.0
     t_chain_tc = 12.0 * tok * w.M * w.D / ((tc_peak or peaks["bf16_tflops"]) * 1e12)
-    t_chain_mem = 5.0 * tok * w.D * w.elt_bytes / (bw_peak * 1e9)
+    t_chain_mem = n_tensors * tok * w.D * w.elt_bytes / (bw_peak * 1e9)
     t_chain = max(t_chain_tc, t_chain_mem)
     t_chain_burst = max(12.0 * tok * w.M * w.D / (peaks["bf16_tflops"] * 1e12), t_chain_mem)
     chain = {"roofline_us": t_chain * 1e6, "bound": "tensor" if t_chain_tc >= t_chain_mem else "hbm",
@@ -319,6 +451,8 @@ def run_ours(args, w):
         Yh = torch.empty(Y.shape, dtype=Y.dtype, pin_memory=True)
         bufs = {}
         ha = (xh["seeds"], xh["Kt"], xh["Vt"], xh["K"], xh["V"])
+        if args.variant == "shared":
+            ha = (xh["seeds"], xh["K"], xh["V"], xh["K"], xh["V"])
         for _ in range(2):
             flarepp.route_fwd_host(*ha, w.scale, Y_host=Yh, device=dev, workspace=ws, dev_bufs=bufs)
         n_e2e = max(1, min(args.steps, args.e2e_steps))
@@ -332,7 +466,7 @@ def run_ours(args, w):
         e1.record(stream)
         torch.cuda.synchronize(dev)
         e2e_ms = max_over_ranks(e0.elapsed_time(e1) / n_e2e, world)
-        h2d = sum(t.numel() * t.element_size() for t in ha)
+        h2d = sum(t.numel() * t.element_size() for t in {id(t): t for t in ha}.values())
         d2h = Yh.numel() * Yh.element_size()
         e2e = {"value": tok * world / (e2e_ms * 1e-3), "unit": UNIT, "ms_per_step": e2e_ms,
                "steps": n_e2e, "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h}
@@ -340,7 +474,7 @@ def run_ours(args, w):
 
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
-        cpu = cpu_oracle_sample(w, args.cpu_seconds, args.seed)
+        cpu = cpu_oracle_sample(w, args.cpu_seconds, args.seed, args.variant)
 
     if rank == 0:
         line = {
@@ -348,7 +482,8 @@ def run_ours(args, w):
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms_per_step,
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
             "dtype": "bf16" if w.dtype == "bf16" else "f32", "data": "synthetic",
-            "config": {"workload": w.name, "B": w.B, "H": w.H, "N": w.N, "M": w.M, "D": w.D,
+            "config": {"workload": w.name, "variant": args.variant,
+                       "B": w.B, "H": w.H, "N": w.N, "M": w.M, "D": w.D,
                        "keys": f"clustered, {w.n_centres} centres" if w.n_centres else "iid",
                        "l2": "inputs larger than L2 (no flush)"
                        if 5 * tok * w.D * w.elt_bytes > 2 * 129e6 else "inputs near L2 size",
@@ -372,6 +507,9 @@ def main():
     ap.add_argument("--impl", choices=("ours", "reference"), default="ours")
     ap.add_argument("--workload", default="mesh3d", choices=sorted(inputs.WORKLOADS))
     ap.add_argument("--seed", type=int, default=0)
+    ap.add_argument("--variant", choices=("flarepp", "shared", "flare"), default="flarepp",
+                    help="flarepp: the routing chain (default); shared: the chain with Kt, Vt "
+                         "tied to K, V; flare: FLARE with fixed learned queries")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--e2e-steps", type=int, default=5)
     ap.add_argument("--no-cpu-baseline", action="store_true")

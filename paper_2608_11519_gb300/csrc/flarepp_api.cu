@@ -1,5 +1,5 @@
-// The C ABI of libflarepp: argument checks, the shape-derived plan and workspace layout,
-// and the launch sequence of the routing chain (Sec. 3.2):
+// The C ABI of libflarepp: argument checks and the launch sequence of the routing chain
+// (Sec. 3.2):
 //   encode(call 1) -> combine -> encode(call 2) -> combine -> decode(call 3).
 #include <cuda_runtime.h>
 #include <math.h>
@@ -11,113 +11,7 @@
 namespace flarepp {
 namespace {
 
-constexpr int64_t kMaxM = 2048;
-constexpr int64_t kMaxTokenHeads = int64_t(1) << 40;  // B*H*N limit (index headroom)
-constexpr size_t kWsAlign = 256;
 constexpr int kStageEvents = 6;
-constexpr int64_t kMaxTmaCoord = 2147483647 - 4096;  // TMA coordinates are signed 32-bit
-constexpr int64_t kTcItem = 64;               // tokens per tensor-core encode item
-
-size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
-int64_t cdiv(int64_t a, int64_t b) { return (a + b - 1) / b; }
-
-bool mul_ok(int64_t a, int64_t b, int64_t* out) { return !__builtin_mul_overflow(a, b, out); }
-
-}  // namespace
-
-flarepp_status make_plan(const flarepp_shape* s, Plan* p) {
-    if (!s || !p) return FLAREPP_ERR_INVALID_ARGUMENT;
-    if (s->dtype != FLAREPP_F32 && s->dtype != FLAREPP_BF16) return FLAREPP_ERR_INVALID_ARGUMENT;
-    if (s->B < 0 || s->H < 0 || s->N < 0 || s->M < 0 || s->D < 0)
-        return FLAREPP_ERR_INVALID_ARGUMENT;
-    if (s->D != 16 && s->D != 32 && s->D != 64) return FLAREPP_ERR_UNSUPPORTED;
-    if (s->M > kMaxM) return FLAREPP_ERR_UNSUPPORTED;
-    int64_t bh, bhn;
-    if (!mul_ok(s->B, s->H, &bh) || !mul_ok(bh, s->N, &bhn)) return FLAREPP_ERR_UNSUPPORTED;
-    if (bhn > kMaxTokenHeads) return FLAREPP_ERR_UNSUPPORTED;
-
-    memset(p, 0, sizeof(*p));
-    p->B = s->B;
-    p->H = s->H;
-    p->N = s->N;
-    p->M = s->M;
-    p->D = s->D;
-    p->BH = bh;
-    p->dtype = s->dtype;
-    p->path = s->dtype == FLAREPP_BF16 ? kPathTc : kPathSimt;
-    if (p->path == kPathTc && (s->N > kMaxTmaCoord || bh > kMaxTmaCoord))
-        return FLAREPP_ERR_UNSUPPORTED;
-    if (bh == 0 || s->N == 0 || s->M == 0) return FLAREPP_OK;  // nothing to plan
-
-    if (p->path == kPathSimt) {
-        // CUDA-core encode: one thread per route, up to 128 routes per CTA; chunks sized so
-        // that the grid holds about four waves of CTAs per SM.
-        p->m_tile = s->M >= 128 ? 128 : cdiv(s->M, 32) * 32;
-        p->n_mtiles = cdiv(s->M, p->m_tile);
-        p->sub_per_chunk = 1;
-        const int64_t target = 4 * kNumSMs;
-        int64_t want = cdiv(target, bh * p->n_mtiles);
-        if (want < 1) want = 1;
-        p->chunk_len = cdiv(cdiv(s->N, want), 32) * 32;
-        p->nchunk = cdiv(s->N, p->chunk_len);
-    } else {
-        // Tensor-core encode: a work unit is (bh, group of <= 512 routes, chunk of tokens) and
-        // one persistent CTA per SM walks the units. Pick the chunk count that minimises
-        // waves x (64-token items per unit, scaled by the group's route tiles, + a fixed
-        // per-unit cost of about three items).
-        p->tc_group = tc_group_rows(s->D);
-        p->n_groups = cdiv(s->M, p->tc_group);
-        p->sub_per_chunk = 4;
-        const int64_t ns = p->tc_group / 128;
-        const int64_t tiles0 = s->M >= p->tc_group ? ns : cdiv(s->M, 128);
-        const double na = tiles0 <= 1 ? 1.0 : (tiles0 <= 2 ? 2.0 : 4.0);
-        const int64_t per_chunk = bh * p->n_groups;
-        const int64_t max_chunks = cdiv(s->N, kTcItem);
-        double best = 1e300;
-        int64_t best_n = 1;
-        for (int64_t n = 1; n <= max_chunks && n <= 65536; ++n) {
-            const int64_t waves = cdiv(per_chunk * n, kNumSMs);
-            const int64_t items = cdiv(cdiv(s->N, n), kTcItem);
-            const double cost = (double)waves * ((double)items * na / (double)ns + 3.0);
-            if (cost < best) {
-                best = cost;
-                best_n = n;
-            }
-        }
-        p->chunk_len = cdiv(cdiv(s->N, best_n), kTcItem) * kTcItem;
-        p->nchunk = cdiv(s->N, p->chunk_len);
-    }
-
-    const size_t rows =
-        (size_t)bh * (size_t)p->nchunk * (size_t)p->sub_per_chunk * (size_t)s->M;
-    size_t off = 0;
-    p->off_status = off;
-    off = align_up(off + sizeof(int32_t), kWsAlign);
-    p->off_pmax = off;
-    off = align_up(off + rows * sizeof(float), kWsAlign);
-    p->off_psum = off;
-    off = align_up(off + rows * sizeof(float), kWsAlign);
-    p->off_pacc = off;
-    off = align_up(off + rows * (size_t)s->D * sizeof(float), kWsAlign);
-    const size_t qz = (size_t)bh * (size_t)s->M * (size_t)s->D * sizeof(float);
-    p->off_q32 = off;
-    off = align_up(off + qz, kWsAlign);
-    p->off_z32 = off;
-    off = align_up(off + qz, kWsAlign);
-    if (p->path == kPathTc) {
-        const size_t op = (size_t)bh * (size_t)s->M * (size_t)s->D * 2;
-        p->off_qop = off;
-        off = align_up(off + op, kWsAlign);
-        p->off_zop = off;
-        off = align_up(off + op, kWsAlign);
-        p->off_seedneg = off;
-        off = align_up(off + (size_t)s->H * (size_t)s->M * (size_t)s->D * 2, kWsAlign);
-    }
-    p->total = off;
-    return FLAREPP_OK;
-}
-
-namespace {
 
 bool aligned16(const void* ptr) { return ((uintptr_t)ptr & 15u) == 0; }
 

@@ -9,6 +9,10 @@
 namespace flarepp {
 
 constexpr int kNumSMs = 152;  // GB300: two dies of 76 SMs
+constexpr size_t kWsAlign = 256;  // alignment of every workspace sub-buffer
+
+inline size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
+inline int64_t cdiv(int64_t a, int64_t b) { return (a + b - 1) / b; }
 
 // Which kernels a shape runs on.
 enum Path : int {
@@ -36,7 +40,7 @@ struct Plan {
     size_t total;
 };
 
-// Fill `p` for `s`; returns FLAREPP_OK or the validation error for the shape itself.
+// Fill `p` for `s` (plan.cu); returns FLAREPP_OK or the validation error for the shape itself.
 flarepp_status make_plan(const flarepp_shape* s, Plan* p);
 
 // ---- CUDA-core kernels (simt_kernels.cuh, instantiated in simt_f32.cu), float32 inputs
