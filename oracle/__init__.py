@@ -12,6 +12,12 @@ What it computes (FLARE++ paper):
                           shared by the batch (Sec. 3, eq. prelim_flare_sdpa)
   * ``encode_sharded`` -- the encoder evaluated shard by shard, then merged by the stable
                           log-sum-exp reduction (App. A.2, A.3)
+  * ``sdpa_bwd``       -- the backward of one SDPA from its saved output and log-normaliser
+                          (App. A.5): P = exp(S - L), c = <dO, O>, dV = P^T dO,
+                          dS = P o (dO V^T - c), dK = s dS^T Q, dQ = s dS K
+  * ``route_bwd``      -- the chain's backward: calls 3, 2, 1 in turn, the decoder's query
+                          gradient added to call 2's before call 1, the seeds' gradient
+                          summed over the batch (App. A.5)
 
 All arithmetic is float64 in ``flarepp_oracle.c``; this module only marshals numpy arrays.
 """
@@ -41,6 +47,12 @@ class Oracle:
         lib.oracle_encode_sharded_f64.restype = ctypes.c_int
         lib.oracle_encode_sharded_f64.argtypes = [_c_i64] * 4 + [_c_dp] * 3 + [
             ctypes.c_double, _c_i64, _c_i64, _c_dp, _c_dp]
+        lib.oracle_sdpa_bwd_f64.restype = ctypes.c_int
+        lib.oracle_sdpa_bwd_f64.argtypes = [_c_i64] * 4 + [_c_dp] * 6 + [ctypes.c_double] + [
+            _c_dp] * 3
+        lib.oracle_route_bwd_f64.restype = ctypes.c_int
+        lib.oracle_route_bwd_f64.argtypes = [_c_i64] * 5 + [_c_dp] * 5 + [ctypes.c_double] + [
+            _c_dp] * 6
         lib.oracle_max_threads.restype = ctypes.c_int
         lib.oracle_set_threads.argtypes = [ctypes.c_int]
         assert lib.oracle_plant() == plant
@@ -116,6 +128,48 @@ class Oracle:
         Y, _ = self.sdpa(K, Qb, Z, scale)
         return Z, Y
 
+    def sdpa_bwd(self, q, k, v, out, lse, dout, scale):
+        """Backward of ``sdpa`` (App. A.5) from the forward's ``out`` and ``lse``.
+
+        q, out, dout [..., nq, D]; k, v [..., nk, D]; lse [..., nq].
+        Returns (dq, dk, dv) shaped like q, k, v.
+        """
+        q, k, v, out, lse, dout = (self._f64(a) for a in (q, k, v, out, lse, dout))
+        lead = q.shape[:-2]
+        assert k.shape[:-2] == lead and v.shape == k.shape and out.shape == q.shape
+        assert dout.shape == q.shape and lse.shape == q.shape[:-1]
+        G = int(np.prod(lead)) if lead else 1
+        nq, D = q.shape[-2], q.shape[-1]
+        nk = k.shape[-2]
+        dq, dk, dv = np.zeros(q.shape), np.zeros(k.shape), np.zeros(v.shape)
+        rc = self.lib.oracle_sdpa_bwd_f64(G, nq, nk, D, self._p(q), self._p(k), self._p(v),
+                                          self._p(out), self._p(lse), self._p(dout),
+                                          float(scale), self._p(dq), self._p(dk), self._p(dv))
+        if rc:
+            raise MemoryError("oracle scratch allocation failed")
+        return dq, dk, dv
+
+    def route_bwd(self, seeds, Kt, Vt, K, V, scale, dY):
+        """Gradients of the routing chain for the output gradient dY [B, H, N, D].
+
+        Returns (dseeds [H, M, D], dKt, dVt, dK, dV [B, H, N, D]).
+        """
+        seeds, Kt, Vt, K, V, dY = (self._f64(a) for a in (seeds, Kt, Vt, K, V, dY))
+        B, H, N, D = K.shape
+        M = seeds.shape[1]
+        assert seeds.shape == (H, M, D)
+        for a in (Kt, Vt, V, dY):
+            assert a.shape == (B, H, N, D)
+        dseeds = np.zeros((H, M, D))
+        grads = [np.zeros((B, H, N, D)) for _ in range(4)]
+        rc = self.lib.oracle_route_bwd_f64(B, H, N, M, D, self._p(seeds), self._p(Kt),
+                                           self._p(Vt), self._p(K), self._p(V), float(scale),
+                                           self._p(dY), self._p(dseeds),
+                                           *(self._p(g) for g in grads))
+        if rc:
+            raise MemoryError("oracle scratch allocation failed")
+        return (dseeds, *grads)
+
     def encode_sharded(self, q, k, v, scale, chunk, n_empty=0):
         """Encoder over shards of ``chunk`` keys merged by the stable LSE reduction (App. A.3).
 
@@ -163,6 +217,14 @@ def encode_sharded(q, k, v, scale, chunk, n_empty=0):
     return default().encode_sharded(q, k, v, scale, chunk, n_empty)
 
 
+def sdpa_bwd(q, k, v, out, lse, dout, scale):
+    return default().sdpa_bwd(q, k, v, out, lse, dout, scale)
+
+
+def route_bwd(seeds, Kt, Vt, K, V, scale, dY):
+    return default().route_bwd(seeds, Kt, Vt, K, V, scale, dY)
+
+
 def max_threads() -> int:
     return default().max_threads()
 
@@ -176,5 +238,5 @@ def build() -> str:
     return _build.build()
 
 
-__all__ = ["Oracle", "default", "sdpa", "route", "flare", "encode_sharded", "max_threads",
-           "set_threads", "build"]
+__all__ = ["Oracle", "default", "sdpa", "route", "flare", "encode_sharded", "sdpa_bwd",
+           "route_bwd", "max_threads", "set_threads", "build"]

@@ -16,6 +16,11 @@
  *   merge  L_max = max_r L_r, a_r = exp(L_r - L_max), a = sum_r a_r,
  *          U = sum_r a_r O_r, L = L_max + log a, Z = U / a                         (App. A.3)
  *   an attention row with no keys has L = -inf and output 0, never NaN            (App. A.3)
+ *   backward of one SDPA with the saved output O and log-normaliser L          (App. A.5):
+ *          P = exp(S - L),  c = <dO, O>_D,  dV = P^T dO,  dS = P o (dO V^T - c),
+ *          dK = s dS^T Q,  dQ = s dS K
+ *   chain backward: the decoder's query gradient is added to the encoder's before call 1's
+ *          backward, and each call uses its own saved L                          (App. A.5)
  *
  * Every softmax is two-pass: the exact row maximum first, then exp(x - max) summed in
  * ascending key order. Dot products run in ascending channel order. OpenMP splits only
@@ -251,5 +256,165 @@ int oracle_encode_sharded_f64(int64_t G, int64_t nq, int64_t nk, int64_t D, cons
         free(O);
         free(L);
     }
+    return err ? -1 : 0;
+}
+
+/*
+ * Backward of one SDPA group (App. A.5, one shard), accumulating into dq, dk, dv:
+ *   q [nq, D], k, v [nk, D], the forward output o [nq, D] and log-normaliser lse [nq],
+ *   the output gradient dO [nq, D]. With S = s q k^T:
+ *     P = exp(S - lse)            (the saved L broadcast along the keys)
+ *     c_i = <dO_i, o_i>_D
+ *     dS = P o (dO v^T - c)
+ *     dq += s dS k,  dk += s dS^T q,  dv += P^T dO
+ *   P and dS are held as full [nq, nk] matrices; the query-side sums run over rows in
+ *   parallel, the key-side sums over key rows in parallel, each in ascending order.
+ */
+static int sdpa_bwd_group(int64_t nq, int64_t nk, int64_t D, const double* q, const double* k,
+                          const double* v, const double* o, const double* lse, const double* dO,
+                          double s, double* dq, double* dk, double* dv) {
+    if (nq == 0 || nk == 0) return 0;
+    double* P = (double*)malloc((size_t)nq * (size_t)nk * sizeof(double));
+    double* dS = (double*)malloc((size_t)nq * (size_t)nk * sizeof(double));
+    if (!P || !dS) {
+        free(P);
+        free(dS);
+        return -1;
+    }
+#pragma omp parallel for schedule(static)
+    for (int64_t i = 0; i < nq; ++i) {
+        const double* qi = q + i * D;
+        const double* dOi = dO + i * D;
+        double c = 0.0;
+        for (int64_t d = 0; d < D; ++d) c += dOi[d] * o[i * D + d];
+#if ORACLE_PLANT == 7
+        c = 0.0; /* planted: the <dO, O> correction dropped */
+#endif
+        for (int64_t j = 0; j < nk; ++j) {
+            double dot = 0.0;
+            for (int64_t d = 0; d < D; ++d) dot += qi[d] * k[j * D + d];
+            const double p = exp(s * dot - lse[i]);
+            double dp = 0.0;
+            for (int64_t d = 0; d < D; ++d) dp += dOi[d] * v[j * D + d];
+            P[i * nk + j] = p;
+            dS[i * nk + j] = p * (dp - c);
+        }
+        for (int64_t j = 0; j < nk; ++j)
+            for (int64_t d = 0; d < D; ++d) dq[i * D + d] += s * dS[i * nk + j] * k[j * D + d];
+    }
+#pragma omp parallel for schedule(static)
+    for (int64_t j = 0; j < nk; ++j) {
+        for (int64_t i = 0; i < nq; ++i) {
+            const double ds = dS[i * nk + j], p = P[i * nk + j];
+            for (int64_t d = 0; d < D; ++d) {
+#if ORACLE_PLANT == 8
+                dk[j * D + d] += s * ds * k[j * D + d]; /* planted: key gradient through k */
+#else
+                dk[j * D + d] += s * ds * q[i * D + d];
+#endif
+                dv[j * D + d] += p * dO[i * D + d];
+            }
+        }
+    }
+    free(P);
+    free(dS);
+    return 0;
+}
+
+/*
+ * Batched SDPA backward over G independent groups (App. A.5): the shapes of
+ * oracle_sdpa_f64 with the forward's out and lse, and dO [G, nq, D]. Writes (not
+ * accumulates) dq [G, nq, D], dk, dv [G, nk, D].
+ */
+int oracle_sdpa_bwd_f64(int64_t G, int64_t nq, int64_t nk, int64_t D, const double* q,
+                        const double* k, const double* v, const double* out, const double* lse,
+                        const double* dO, double s, double* dq, double* dk, double* dv) {
+    memset(dq, 0, (size_t)(G * nq * D) * sizeof(double));
+    memset(dk, 0, (size_t)(G * nk * D) * sizeof(double));
+    memset(dv, 0, (size_t)(G * nk * D) * sizeof(double));
+    for (int64_t g = 0; g < G; ++g) {
+        const int64_t qo = g * nq * D, ko = g * nk * D;
+        if (sdpa_bwd_group(nq, nk, D, q + qo, k + ko, v + ko, out + qo, lse + g * nq, dO + qo,
+                           s, dq + qo, dk + ko, dv + ko))
+            return -1;
+    }
+    return 0;
+}
+
+/*
+ * Backward of the routing chain (App. A.5 applied to eqs. flarepp_dynamic_query and
+ * flarepp_mixer), per (b, h), given dY [B, H, N, D]:
+ *   forward again: Q, L1 = SDPA(seeds_h, Kt, Vt); Z, L2 = SDPA(Q, K, V); Y, L3 = SDPA(K, Q, Z)
+ *   call 3 (decode; queries K, keys Q, values Z):  dK  = ..., dQ = ..., dZ = ...
+ *   call 2 (encode; queries Q, keys K, values V):  dQ += ..., dK += ..., dV = ...
+ *   call 1 (encode; queries seeds, keys Kt, values Vt), with the summed dQ as its output
+ *          gradient:  dKt, dVt, and the seeds' gradient summed over the batch.
+ * Outputs dseeds [H, M, D] and dKt, dVt, dK, dV [B, H, N, D] are overwritten.
+ */
+int oracle_route_bwd_f64(int64_t B, int64_t H, int64_t N, int64_t M, int64_t D,
+                         const double* seeds, const double* Kt, const double* Vt, const double* K,
+                         const double* V, double s, const double* dY, double* dseeds, double* dKt,
+                         double* dVt, double* dK, double* dV) {
+    const int64_t G = B * H;
+    const size_t lat = (size_t)(G * M * D), tok = (size_t)(G * N * D);
+    double* Qs = (double*)malloc((lat ? lat : 1) * sizeof(double));
+    double* Q = (double*)malloc((lat ? lat : 1) * sizeof(double));
+    double* Z = (double*)malloc((lat ? lat : 1) * sizeof(double));
+    double* Y = (double*)malloc((tok ? tok : 1) * sizeof(double));
+    double* L1 = (double*)malloc((size_t)(G * M + 1) * sizeof(double));
+    double* L2 = (double*)malloc((size_t)(G * M + 1) * sizeof(double));
+    double* L3 = (double*)malloc((size_t)(G * N + 1) * sizeof(double));
+    double* dQ = (double*)malloc((lat ? lat : 1) * sizeof(double));
+    double* dQ2 = (double*)malloc((lat ? lat : 1) * sizeof(double));
+    double* dZ = (double*)malloc((lat ? lat : 1) * sizeof(double));
+    double* dK2 = (double*)malloc((tok ? tok : 1) * sizeof(double));
+    double* dQs = (double*)malloc((lat ? lat : 1) * sizeof(double));
+    int err = !Qs || !Q || !Z || !Y || !L1 || !L2 || !L3 || !dQ || !dQ2 || !dZ || !dK2 || !dQs;
+    if (!err) {
+        /* the seeds of head h serve every batch element */
+        for (int64_t g = 0; g < G; ++g)
+            memcpy(Qs + g * M * D, seeds + (g % H) * M * D, (size_t)(M * D) * sizeof(double));
+        err = oracle_sdpa_f64(G, M, N, D, Qs, 0, Kt, Vt, s, Q, L1) ||
+              oracle_sdpa_f64(G, M, N, D, Q, 0, K, V, s, Z, L2) ||
+              oracle_sdpa_f64(G, N, M, D, K, 0, Q, Z, s, Y, L3);
+    }
+    /* call 3: Y = SDPA(K, Q, Z) */
+    if (!err) err = oracle_sdpa_bwd_f64(G, N, M, D, K, Q, Z, Y, L3, dY, s, dK, dQ, dZ);
+    /* call 2: Z = SDPA(Q, K, V) with output gradient dZ */
+    if (!err) err = oracle_sdpa_bwd_f64(G, M, N, D, Q, K, V, Z, L2, dZ, s, dQ2, dK2, dV);
+    if (!err) {
+        for (size_t i = 0; i < tok; ++i) dK[i] += dK2[i];
+#if ORACLE_PLANT == 9
+        /* planted: call 1 sees only the decoder's query gradient */
+#else
+        for (size_t i = 0; i < lat; ++i) dQ[i] += dQ2[i];
+#endif
+        /* call 1: Q = SDPA(seeds, Kt, Vt) with output gradient dQ */
+        err = oracle_sdpa_bwd_f64(G, M, N, D, Qs, Kt, Vt, Q, L1, dQ, s, dQs, dKt, dVt);
+    }
+    if (!err) {
+        memset(dseeds, 0, (size_t)(H * M * D) * sizeof(double));
+#if ORACLE_PLANT == 10
+        const int64_t bend = B > 0 ? 1 : 0; /* planted: seeds' gradient from b = 0 only */
+#else
+        const int64_t bend = B;
+#endif
+        for (int64_t b = 0; b < bend; ++b)
+            for (int64_t h = 0; h < H; ++h)
+                for (int64_t i = 0; i < M * D; ++i)
+                    dseeds[h * M * D + i] += dQs[(b * H + h) * M * D + i];
+    }
+    free(Qs);
+    free(Q);
+    free(Z);
+    free(Y);
+    free(L1);
+    free(L2);
+    free(L3);
+    free(dQ);
+    free(dQ2);
+    free(dZ);
+    free(dK2);
+    free(dQs);
     return err ? -1 : 0;
 }
