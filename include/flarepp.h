@@ -199,6 +199,57 @@ FLAREPP_API flarepp_status flarepp_route_fwd_noalloc(const flarepp_shape* shape,
                                                      void* stream);
 
 /*
+ * Bytes of the state a training forward keeps for the backward (App. A.5): float32 Q and Z
+ * [B, H, M, D] and the base-2 log-normalisers of the three calls,
+ * L = log2 sum_j 2^(scale * log2(e) <a, b_j>), for calls 1 and 2 [B, H, M] and call 3
+ * [B, H, N]. 0 for an invalid or unsupported shape and for N, M or B*H zero.
+ */
+FLAREPP_API size_t flarepp_route_saved_bytes(const flarepp_shape* shape);
+
+/*
+ * flarepp_route_fwd that also fills `saved` (device memory, 16-byte aligned, at least
+ * flarepp_route_saved_bytes(shape) bytes, disjoint from the inputs, Y and the workspace;
+ * FLAREPP_ERR_INVALID_ARGUMENT otherwise) with the state flarepp_route_bwd reads. The
+ * layout of `saved` is private to the library; the caller only keeps it until the backward.
+ * On degenerate shapes `saved` is not touched and may be NULL.
+ */
+FLAREPP_API flarepp_status flarepp_route_fwd_train(const flarepp_shape* shape,
+                                                   const void* seeds, const void* Kt,
+                                                   const void* Vt, const void* K, const void* V,
+                                                   float scale, void* Y, void* saved,
+                                                   size_t saved_bytes, void* workspace,
+                                                   size_t workspace_bytes, void* stream);
+
+/* Workspace bytes flarepp_route_bwd needs for `shape` (0: none needed or shape invalid). */
+FLAREPP_API size_t flarepp_route_bwd_workspace_bytes(const flarepp_shape* shape);
+
+/*
+ * Backward of the routing chain (App. A.5): for the output gradient dY, the gradients of
+ * the seeds and of Kt, Vt, K, V. Each SDPA is differentiated from its saved output and
+ * log-normaliser (P = exp(S - L), c = <dO, O>, dV = P^T dO, dS = P o (dO V^T - c),
+ * dK = s dS^T Q, dQ = s dS K); the decoder's gradient of Q is added to the encoder's before
+ * call 1's backward, and the seeds' gradient is summed over the batch.
+ *   seeds, Kt, Vt, K, V, scale: the forward's inputs (device pointers, as flarepp_route_fwd).
+ *   Y: the forward's output [B, H, N, D]; dY: its gradient [B, H, N, D]; both input dtype.
+ *   saved: what flarepp_route_fwd_train wrote for these inputs (saved_bytes as there).
+ *   dseeds [H, M, D], dKt, dVt, dK, dV [B, H, N, D]: outputs in the input dtype, written
+ *     (not accumulated), 16-byte aligned, disjoint from each other and from every input.
+ *   workspace: device memory, 256-byte aligned, flarepp_route_bwd_workspace_bytes(shape)
+ *     bytes; its first 4 bytes are the device status word (flarepp_route_device_status).
+ * Degenerate shapes (N, M or B*H zero) write zeros to every non-empty output. Errors:
+ * FLAREPP_ERR_INVALID_ARGUMENT (a missing, misaligned or overlapping pointer, too small a
+ * saved buffer, non-finite scale), FLAREPP_ERR_UNSUPPORTED (as flarepp_route_fwd),
+ * FLAREPP_ERR_WORKSPACE, FLAREPP_ERR_CUDA. Enqueued on `stream`; no host synchronisation.
+ */
+FLAREPP_API flarepp_status flarepp_route_bwd(const flarepp_shape* shape, const void* seeds,
+                                             const void* Kt, const void* Vt, const void* K,
+                                             const void* V, float scale, const void* Y,
+                                             const void* dY, const void* saved,
+                                             size_t saved_bytes, void* dseeds, void* dKt,
+                                             void* dVt, void* dK, void* dV, void* workspace,
+                                             size_t workspace_bytes, void* stream);
+
+/*
  * The device status word that the last flarepp_route_fwd* call on `workspace` (for the same
  * shape) left behind: FLAREPP_OK, or FLAREPP_ERR_TIMEOUT when a bounded wait inside a
  * tensor-core kernel gave up (the kernel then stops early and its outputs are invalid).

@@ -1,0 +1,389 @@
+// Backward of the routing chain on CUDA cores (App. A.5), for bf16 or f32 inputs.
+//
+// Every SDPA of the chain is differentiated from its saved output O and log-normaliser L:
+//   P = 2^(x - L) with x = scale * log2(e) <a, b> (L kept in base 2 by the forward),
+//   c = <dO, O>_D,  dS = P o (dO C^T - c),  dA = s dS B,  dB = s dS^T A,  dC = P^T dO
+// for SDPA(A, B, C) with output O. The chain runs the three calls backwards:
+//   call 3  Y = SDPA(K, Q, Z):   c3 per token;  dZ = P3^T dY,  dQ += s dS3^T K,  dK += s dS3 Q
+//   call 2  Z = SDPA(Q, K, V):   c2 per route;  dV = P2^T dZ,  dQ += s dS2 K,    dK += s dS2^T Q
+//   call 1  Q = SDPA(Qs, Kt, Vt) with the summed dQ (App. A.5: the decoder's query gradient is
+//           added to the encoder's): c1 per route; dVt = P1^T dQ, dKt = s dS1^T Qs,
+//           dQs = s dS1 Kt, summed over the batch for the shared seeds.
+//
+// Two kernel shapes cover it. A route pass gives one thread per route and streams a chunk
+// of tokens, accumulating the latent-side sums (dZ, dQ, dQs) into per-chunk partials that a
+// reduce kernel adds in chunk order. A token pass gives one thread per token and streams
+// every route, producing that token's dK, dV (calls 2 and 3 together) or dKt, dVt (call 1).
+#include <cuda_bf16.h>
+#include <math.h>
+
+#include "flarepp_internal.h"
+
+namespace flarepp {
+namespace {
+
+constexpr float kLog2e = 1.4426950408889634f;
+constexpr int kTok = 16;    // tokens staged per step of a route pass
+constexpr int kRoute = 16;  // routes staged per step of a token pass
+
+__device__ __forceinline__ float ld_f32(const float* p) { return *p; }
+__device__ __forceinline__ float ld_f32(const __nv_bfloat16* p) { return __bfloat162float(*p); }
+__device__ __forceinline__ void st_out(float* p, float x) { *p = x; }
+__device__ __forceinline__ void st_out(__nv_bfloat16* p, float x) { *p = __float2bfloat16_rn(x); }
+
+// The bf16 forward multiplies bf16 copies of Q and Z (its MMA operands); the backward
+// differentiates that same function, so on the bf16 path it rounds Q and Z alike wherever
+// they enter a product (logits, and Z in call 3's values).
+template <typename T>
+__device__ __forceinline__ float operand(float x) {
+    if constexpr (sizeof(T) == 2) return __bfloat162float(__float2bfloat16_rn(x));
+    return x;
+}
+
+__device__ __forceinline__ float ex2(float x) {
+    float y;
+    asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+    return y;
+}
+
+// c3[n] = <dY_n, Y_n>: one thread per token.
+template <int D, typename T>
+__global__ void __launch_bounds__(256) delta_tokens_kernel(const T* __restrict__ dY,
+                                                           const T* __restrict__ Y, int64_t rows,
+                                                           float* __restrict__ c3) {
+    const int64_t r = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+    if (r >= rows) return;
+    float acc = 0.f;
+#pragma unroll
+    for (int d = 0; d < D; ++d) acc = fmaf(ld_f32(dY + r * D + d), ld_f32(Y + r * D + d), acc);
+    c3[r] = acc;
+}
+
+// Route pass of call MODE (3, 2 or 1) over one chunk of tokens; thread = route m.
+//   MODE 3: a = Q, keys b = K, w = dY, g = Z, column statistics L3[n], c3[n];
+//           pa += P w (dZ), pb += dS k (dQ / s)
+//   MODE 2: a = Q, keys = K, w = V, g = dZ, row statistics L2[m], c2[m]; pb += dS k
+//   MODE 1: a = seeds (per head), keys = Kt, w = Vt, g = dQ, row statistics L1[m], c1[m];
+//           pb += dS kt
+// dS here is P o (dP - c); the factor s is applied by the reduce.
+// grid.x = nchunk * n_mtiles * BH; block = m_tile threads.
+template <int D, typename T, typename AT, int MODE>
+__global__ void __launch_bounds__(128) route_pass_kernel(
+    const AT* __restrict__ a, int a_per_head, const T* __restrict__ kb, const T* __restrict__ wb,
+    const float* __restrict__ g, const float* __restrict__ Lrow, const float* __restrict__ crow,
+    const float* __restrict__ Lcol, const float* __restrict__ ccol, int64_t H, int64_t N,
+    int64_t M, int64_t chunk_len, int64_t nchunk, int64_t n_mtiles, float sl2,
+    float* __restrict__ pa, float* __restrict__ pb) {
+    __shared__ float ks[kTok][D];
+    __shared__ float ws[kTok][D];
+    __shared__ float lc[kTok], cc[kTok];
+
+    int64_t bid = blockIdx.x;
+    const int64_t c = bid % nchunk;
+    bid /= nchunk;
+    const int64_t mt = bid % n_mtiles;
+    const int64_t bh = bid / n_mtiles;
+    const int64_t m = mt * blockDim.x + threadIdx.x;
+    const bool active = m < M;
+    const int64_t mm = active ? m : 0;
+
+    float ar[D], gr[D], accA[MODE == 3 ? D : 1], accB[D];
+    {
+        const AT* ap = a + ((a_per_head ? bh % H : bh) * M + mm) * D;
+        const float* gp = g + (bh * M + mm) * D;
+#pragma unroll
+        for (int d = 0; d < D; ++d) {
+            ar[d] = operand<T>(ld_f32(ap + d)) * sl2;
+            gr[d] = MODE == 3 ? operand<T>(gp[d]) : gp[d];
+            accB[d] = 0.f;
+            if (MODE == 3) accA[d] = 0.f;
+        }
+    }
+    const float Lr = MODE == 3 ? 0.f : Lrow[bh * M + mm];
+    const float cr = MODE == 3 ? 0.f : crow[bh * M + mm];
+
+    const int64_t n_begin = c * chunk_len;
+    const int64_t n_end = min(N, n_begin + chunk_len);
+    const T* kp = kb + bh * N * D;
+    const T* wp = wb + bh * N * D;
+    for (int64_t n0 = n_begin; n0 < n_end; n0 += kTok) {
+        const int cnt = (int)min((int64_t)kTok, n_end - n0);
+        __syncthreads();
+        for (int i = threadIdx.x; i < kTok * D; i += blockDim.x) {
+            const int j = i / D, d = i % D;
+            const bool in = j < cnt;
+            ks[j][d] = in ? ld_f32(kp + (n0 + j) * D + d) : 0.f;
+            ws[j][d] = in ? ld_f32(wp + (n0 + j) * D + d) : 0.f;
+        }
+        if (MODE == 3 && threadIdx.x < kTok) {
+            const int j = threadIdx.x;
+            lc[j] = j < cnt ? Lcol[bh * N + n0 + j] : 0.f;
+            cc[j] = j < cnt ? ccol[bh * N + n0 + j] : 0.f;
+        }
+        __syncthreads();
+        for (int j = 0; j < cnt; ++j) {
+            float x = 0.f, dp = 0.f;
+#pragma unroll
+            for (int d = 0; d < D; ++d) {
+                x = fmaf(ar[d], ks[j][d], x);
+                dp = fmaf(gr[d], ws[j][d], dp);
+            }
+            const float p = ex2(x - (MODE == 3 ? lc[j] : Lr));
+            const float ds = p * (dp - (MODE == 3 ? cc[j] : cr));
+#pragma unroll
+            for (int d = 0; d < D; ++d) {
+                accB[d] = fmaf(ds, ks[j][d], accB[d]);
+                if (MODE == 3) accA[d] = fmaf(p, ws[j][d], accA[d]);
+            }
+        }
+    }
+    if (active) {
+        const int64_t row = (bh * nchunk + c) * M + m;
+#pragma unroll
+        for (int d = 0; d < D; ++d) {
+            pb[row * D + d] = accB[d];
+            if (MODE == 3) pa[row * D + d] = accA[d];
+        }
+    }
+}
+
+// Reduce of the route passes' partials, one warp per latent row, chunks in ascending order.
+//   MODE 3: dZ = sum pa, dQ = s sum pb, c2 = <dZ, Z>
+//   MODE 2: dQ += s sum pb, c1 = <dQ, Q>
+//   MODE 1: dseeds[h, m] = s sum_b sum_chunks pb (rows = H * M)
+template <int D, typename T, int MODE>
+__global__ void bwd_reduce_kernel(const float* __restrict__ pa, const float* __restrict__ pb,
+                                  int64_t rows, int64_t B, int64_t H, int64_t M, int64_t nchunk,
+                                  float scale, const float* __restrict__ O,
+                                  float* __restrict__ dz, float* __restrict__ dq,
+                                  float* __restrict__ cout, T* __restrict__ dseeds) {
+    constexpr int PER = (D + 31) / 32;
+    const int lane = threadIdx.x & 31;
+    const int64_t row = (int64_t)blockIdx.x * (blockDim.x / 32) + threadIdx.x / 32;
+    if (row >= rows) return;
+    float sa[PER], sb[PER];
+#pragma unroll
+    for (int i = 0; i < PER; ++i) sa[i] = sb[i] = 0.f;
+    if (MODE == 1) {
+        const int64_t h = row / M, m = row % M;
+        for (int64_t b = 0; b < B; ++b)
+            for (int64_t c = 0; c < nchunk; ++c) {
+                const int64_t r = ((b * H + h) * nchunk + c) * M + m;
+#pragma unroll
+                for (int i = 0; i < PER; ++i) {
+                    const int d = lane + 32 * i;
+                    if (d < D) sb[i] += pb[r * D + d];
+                }
+            }
+#pragma unroll
+        for (int i = 0; i < PER; ++i) {
+            const int d = lane + 32 * i;
+            if (d < D) st_out(dseeds + row * D + d, scale * sb[i]);
+        }
+        return;
+    }
+    const int64_t bh = row / M, m = row % M;
+    for (int64_t c = 0; c < nchunk; ++c) {
+        const int64_t r = (bh * nchunk + c) * M + m;
+#pragma unroll
+        for (int i = 0; i < PER; ++i) {
+            const int d = lane + 32 * i;
+            if (d < D) {
+                sb[i] += pb[r * D + d];
+                if (MODE == 3) sa[i] += pa[r * D + d];
+            }
+        }
+    }
+    float dot = 0.f;
+#pragma unroll
+    for (int i = 0; i < PER; ++i) {
+        const int d = lane + 32 * i;
+        if (d < D) {
+            if (MODE == 3) {
+                dz[row * D + d] = sa[i];
+                dq[row * D + d] = scale * sb[i];
+                dot = fmaf(sa[i], O[row * D + d], dot);
+            } else {
+                const float v = dq[row * D + d] + scale * sb[i];
+                dq[row * D + d] = v;
+                dot = fmaf(v, O[row * D + d], dot);
+            }
+        }
+    }
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) dot += __shfl_xor_sync(0xffffffffu, dot, off);
+    if (lane == 0) cout[row] = dot;
+}
+
+// Token pass; thread = token n, every route streamed.
+//   MODE 23 (calls 3 and 2 together): keys k = K_n, w = V_n, y = dY_n; routes a = Q, g = dZ,
+//     z = Z with L2, c2 per route and L3, c3 of the token:
+//     x = s' <k, q_m>; P2 = 2^(x - L2_m); P3 = 2^(x - L3_n);
+//     dS = P2 (<w, dz_m> - c2_m) + P3 (<y, z_m> - c3_n)
+//     dK = s sum_m dS q_m;  dV = sum_m P2 dz_m
+//   MODE 1: k = Kt_n, w = Vt_n; routes a = seeds (per head), g = dQ with L1, c1:
+//     P1 = 2^(x - L1_m); dS = P1 (<w, dq_m> - c1_m); dKt = s sum_m dS a_m; dVt = sum_m P1 dq_m
+// grid.x = ceil(N / 128) * BH; block = 128 threads.
+template <int D, typename T, typename AT, int MODE>
+__global__ void __launch_bounds__(128) token_pass_kernel(
+    const T* __restrict__ kb, const T* __restrict__ wb, const T* __restrict__ yb,
+    const AT* __restrict__ a, int a_per_head, const float* __restrict__ g,
+    const float* __restrict__ z, const float* __restrict__ Lrow, const float* __restrict__ crow,
+    const float* __restrict__ Lcol, const float* __restrict__ ccol, int64_t H, int64_t N,
+    int64_t M, float sl2, float scale, T* __restrict__ dk_out, T* __restrict__ dv_out) {
+    __shared__ float as_[kRoute][D];
+    __shared__ float gs[kRoute][D];
+    __shared__ float zs[MODE == 23 ? kRoute : 1][D];
+    __shared__ float ls[kRoute], cs[kRoute];
+    const int64_t ntiles = (N + 127) / 128;
+    const int64_t bh = blockIdx.x / ntiles;
+    const int64_t n = (blockIdx.x % ntiles) * 128 + threadIdx.x;
+    const bool active = n < N;
+    const int64_t nn = active ? n : 0;
+    float kr[D], wr[D], yr[MODE == 23 ? D : 1], dk[D], dv[D];
+#pragma unroll
+    for (int d = 0; d < D; ++d) {
+        kr[d] = ld_f32(kb + (bh * N + nn) * D + d) * sl2;
+        wr[d] = ld_f32(wb + (bh * N + nn) * D + d);
+        if (MODE == 23) yr[d] = ld_f32(yb + (bh * N + nn) * D + d);
+        dk[d] = dv[d] = 0.f;
+    }
+    const float L3 = MODE == 23 ? Lcol[bh * N + nn] : 0.f;
+    const float c3 = MODE == 23 ? ccol[bh * N + nn] : 0.f;
+    const AT* ab = a + (a_per_head ? bh % H : bh) * M * D;
+    const float* gb = g + bh * M * D;
+    const float* zb = MODE == 23 ? z + bh * M * D : nullptr;
+    for (int64_t m0 = 0; m0 < M; m0 += kRoute) {
+        const int cnt = (int)min((int64_t)kRoute, M - m0);
+        __syncthreads();
+        for (int i = threadIdx.x; i < kRoute * D; i += blockDim.x) {
+            const int j = i / D, d = i % D;
+            const bool in = j < cnt;
+            as_[j][d] = in ? operand<T>(ld_f32(ab + (m0 + j) * D + d)) : 0.f;
+            gs[j][d] = in ? gb[(m0 + j) * D + d] : 0.f;
+            if (MODE == 23) zs[j][d] = in ? operand<T>(zb[(m0 + j) * D + d]) : 0.f;
+        }
+        if (threadIdx.x < kRoute) {
+            const int j = threadIdx.x;
+            ls[j] = j < cnt ? Lrow[bh * M + m0 + j] : 0.f;
+            cs[j] = j < cnt ? crow[bh * M + m0 + j] : 0.f;
+        }
+        __syncthreads();
+        for (int j = 0; j < cnt; ++j) {
+            float x = 0.f, dp = 0.f, dp3 = 0.f;
+#pragma unroll
+            for (int d = 0; d < D; ++d) {
+                x = fmaf(kr[d], as_[j][d], x);
+                dp = fmaf(wr[d], gs[j][d], dp);
+                if (MODE == 23) dp3 = fmaf(yr[d], zs[j][d], dp3);
+            }
+            const float p = ex2(x - ls[j]);
+            float ds = p * (dp - cs[j]);
+            if (MODE == 23) ds = fmaf(ex2(x - L3), dp3 - c3, ds);
+#pragma unroll
+            for (int d = 0; d < D; ++d) {
+                dk[d] = fmaf(ds, as_[j][d], dk[d]);
+                dv[d] = fmaf(p, gs[j][d], dv[d]);
+            }
+        }
+    }
+    if (active) {
+#pragma unroll
+        for (int d = 0; d < D; ++d) {
+            st_out(dk_out + (bh * N + n) * D + d, scale * dk[d]);
+            st_out(dv_out + (bh * N + n) * D + d, dv[d]);
+        }
+    }
+}
+
+template <int D, typename T>
+cudaError_t route_bwd_d(const Plan& p, const BwdPlan& bp, const T* seeds, const T* Kt,
+                        const T* Vt, const T* K, const T* V, float scale, const T* Y,
+                        const T* dY, const char* saved, T* dseeds, T* dKt, T* dVt, T* dK,
+                        T* dV, char* ws, cudaStream_t st) {
+    const SavedLayout sl = saved_layout(p);
+    const float* Q32 = (const float*)(saved + sl.off_q);
+    const float* Z32 = (const float*)(saved + sl.off_z);
+    const float* L1 = (const float*)(saved + sl.off_l1);
+    const float* L2 = (const float*)(saved + sl.off_l2);
+    const float* L3 = (const float*)(saved + sl.off_l3);
+    float* pa = (float*)(ws + bp.off_pa);
+    float* pb = (float*)(ws + bp.off_pb);
+    float* dz = (float*)(ws + bp.off_dz);
+    float* dq = (float*)(ws + bp.off_dq);
+    float* c1 = (float*)(ws + bp.off_d1);
+    float* c2 = (float*)(ws + bp.off_d2);
+    float* c3 = (float*)(ws + bp.off_d3);
+    const float sl2 = scale * kLog2e;
+    const int64_t tok_rows = p.BH * p.N;
+    const int64_t lat_rows = p.BH * p.M;
+    const unsigned route_blocks = (unsigned)(bp.nchunk * bp.n_mtiles * p.BH);
+    const int route_threads = (int)bp.m_tile;
+    const unsigned token_blocks = (unsigned)(((p.N + 127) / 128) * p.BH);
+    const unsigned red_blocks = (unsigned)((lat_rows + 7) / 8);
+
+    delta_tokens_kernel<D, T><<<(unsigned)((tok_rows + 255) / 256), 256, 0, st>>>(dY, Y, tok_rows,
+                                                                                  c3);
+    // call 3: dZ and the decoder's dQ
+    route_pass_kernel<D, T, float, 3><<<route_blocks, route_threads, 0, st>>>(
+        Q32, 0, K, dY, Z32, nullptr, nullptr, L3, c3, p.H, p.N, p.M, bp.chunk_len, bp.nchunk,
+        bp.n_mtiles, sl2, pa, pb);
+    bwd_reduce_kernel<D, T, 3><<<red_blocks, 256, 0, st>>>(pa, pb, lat_rows, p.B, p.H, p.M,
+                                                           bp.nchunk, scale, Z32, dz, dq, c2,
+                                                           nullptr);
+    // calls 3 and 2: dK and dV per token
+    token_pass_kernel<D, T, float, 23><<<token_blocks, 128, 0, st>>>(
+        K, V, dY, Q32, 0, dz, Z32, L2, c2, L3, c3, p.H, p.N, p.M, sl2, scale, dK, dV);
+    // call 2: the encoder's dQ, added to the decoder's
+    route_pass_kernel<D, T, float, 2><<<route_blocks, route_threads, 0, st>>>(
+        Q32, 0, K, V, dz, L2, c2, nullptr, nullptr, p.H, p.N, p.M, bp.chunk_len, bp.nchunk,
+        bp.n_mtiles, sl2, nullptr, pb);
+    bwd_reduce_kernel<D, T, 2><<<red_blocks, 256, 0, st>>>(nullptr, pb, lat_rows, p.B, p.H, p.M,
+                                                           bp.nchunk, scale, Q32, nullptr, dq, c1,
+                                                           nullptr);
+    // call 1: dKt, dVt per token, then the seeds' gradient
+    token_pass_kernel<D, T, T, 1><<<token_blocks, 128, 0, st>>>(
+        Kt, Vt, nullptr, seeds, 1, dq, nullptr, L1, c1, nullptr, nullptr, p.H, p.N, p.M, sl2,
+        scale, dKt, dVt);
+    route_pass_kernel<D, T, T, 1><<<route_blocks, route_threads, 0, st>>>(
+        seeds, 1, Kt, Vt, dq, L1, c1, nullptr, nullptr, p.H, p.N, p.M, bp.chunk_len, bp.nchunk,
+        bp.n_mtiles, sl2, nullptr, pb);
+    const int64_t seed_rows = p.H * p.M;
+    bwd_reduce_kernel<D, T, 1><<<(unsigned)((seed_rows + 7) / 8), 256, 0, st>>>(
+        nullptr, pb, seed_rows, p.B, p.H, p.M, bp.nchunk, scale, nullptr, nullptr, nullptr,
+        nullptr, dseeds);
+    return cudaGetLastError();
+}
+
+template <typename T>
+cudaError_t route_bwd_t(const Plan& p, const BwdPlan& bp, const void* seeds, const void* Kt,
+                        const void* Vt, const void* K, const void* V, float scale, const void* Y,
+                        const void* dY, const char* saved, void* dseeds, void* dKt, void* dVt,
+                        void* dK, void* dV, char* ws, cudaStream_t st) {
+#define FLAREPP_BWD(DD)                                                                          \
+    return route_bwd_d<DD, T>(p, bp, (const T*)seeds, (const T*)Kt, (const T*)Vt, (const T*)K,  \
+                              (const T*)V, scale, (const T*)Y, (const T*)dY, saved, (T*)dseeds, \
+                              (T*)dKt, (T*)dVt, (T*)dK, (T*)dV, ws, st);
+    switch (p.D) {
+        case 16: FLAREPP_BWD(16)
+        case 32: FLAREPP_BWD(32)
+        case 64: FLAREPP_BWD(64)
+        default: return cudaErrorInvalidValue;
+    }
+#undef FLAREPP_BWD
+}
+
+}  // namespace
+
+cudaError_t simt_route_bwd(const Plan& p, const BwdPlan& bp, const void* seeds, const void* Kt,
+                           const void* Vt, const void* K, const void* V, float scale,
+                           const void* Y, const void* dY, const char* saved, void* dseeds,
+                           void* dKt, void* dVt, void* dK, void* dV, char* ws, cudaStream_t st) {
+    if (p.dtype == FLAREPP_F32)
+        return route_bwd_t<float>(p, bp, seeds, Kt, Vt, K, V, scale, Y, dY, saved, dseeds, dKt,
+                                  dVt, dK, dV, ws, st);
+    return route_bwd_t<__nv_bfloat16>(p, bp, seeds, Kt, Vt, K, V, scale, Y, dY, saved, dseeds,
+                                      dKt, dVt, dK, dV, ws, st);
+}
+
+}  // namespace flarepp

@@ -29,13 +29,15 @@ __device__ __forceinline__ int slots_of_route(int64_t M, int64_t m, int64_t sub_
 }
 
 // One warp per (bh, m): merge the partial slots in ascending order (App. A.3):
-//   g = max_r mx_r; w_r = 2^(mx_r - g); out = sum_r w_r acc_r / sum_r w_r l_r.
+//   g = max_r mx_r; w_r = 2^(mx_r - g); out = sum_r w_r acc_r / sum_r w_r l_r;
+//   the row's base-2 log-normaliser is g + log2(sum_r w_r l_r).
 template <int D>
 __global__ void combine_kernel(const float* __restrict__ pmax, const float* __restrict__ psum,
                                const float* __restrict__ pacc, int64_t rows, int64_t M,
                                int64_t nchunk, int64_t sub_per_chunk, int64_t group,
                                float* __restrict__ out32,
-                               __nv_bfloat16* __restrict__ outop, float op_sign) {
+                               __nv_bfloat16* __restrict__ outop, float op_sign,
+                               float* __restrict__ lse) {
     constexpr int PER = (D + 31) / 32;
     const int lane = threadIdx.x & 31;
     const int64_t row = (int64_t)blockIdx.x * (blockDim.x / 32) + threadIdx.x / 32;
@@ -65,6 +67,7 @@ __global__ void combine_kernel(const float* __restrict__ pmax, const float* __re
         }
     }
     const float inv = a > 0.f ? 1.f / a : 0.f;
+    if (lse && lane == 0) lse[row] = a > 0.f ? g + log2f(a) : -INFINITY;
 #pragma unroll
     for (int i = 0; i < PER; ++i) {
         const int d = lane + 32 * i;
@@ -85,7 +88,8 @@ __global__ void negate_bf16_kernel(const __nv_bfloat16* __restrict__ src,
 
 }  // namespace
 
-cudaError_t combine(const Plan& p, int call, char* ws, bool negate, cudaStream_t st) {
+cudaError_t combine(const Plan& p, int call, char* ws, bool negate, cudaStream_t st,
+                    float* lse) {
     const int64_t rows = p.BH * p.M;
     const int warps = 8;
     const int64_t blocks = (rows + warps - 1) / warps;
@@ -100,7 +104,7 @@ cudaError_t combine(const Plan& p, int call, char* ws, bool negate, cudaStream_t
     combine_kernel<DD><<<(unsigned)blocks, warps * 32, 0, st>>>(pmax, psum, pacc, rows, p.M,  \
                                                                 p.nchunk, p.sub_per_chunk,     \
                                                                 p.tc_group,                    \
-                                                                out32, outop, sign);
+                                                                out32, outop, sign, lse);
     switch (p.D) {
         case 16: FLAREPP_COMBINE(16) break;
         case 32: FLAREPP_COMBINE(32) break;

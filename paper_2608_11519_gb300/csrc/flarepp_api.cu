@@ -25,7 +25,7 @@ flarepp_status route_impl(const flarepp_shape* shape, const void* seeds, const v
                           const void* Vt, const void* K, const void* V, float scale, void* Y,
                           void* workspace, size_t workspace_bytes, void* stream, float* Q_out,
                           float* Z_out, void* const* events, int n_events,
-                          bool reset_status = true) {
+                          bool reset_status = true, char* saved = nullptr) {
     Plan p;
     flarepp_status stt = make_plan(shape, &p);
     if (stt != FLAREPP_OK) return stt;
@@ -93,12 +93,21 @@ flarepp_status route_impl(const flarepp_shape* shape, const void* seeds, const v
         return FLAREPP_ERR_CUDA;
     if (!mark(0)) return FLAREPP_ERR_CUDA;
     if (encode(1, Kt, Vt) != cudaSuccess || !mark(1)) return FLAREPP_ERR_CUDA;
-    if (combine(p, 1, ws, neg, st) != cudaSuccess || !mark(2)) return FLAREPP_ERR_CUDA;
+    // the training forward keeps each call's log-normaliser for the backward (App. A.5)
+    const SavedLayout sv = saved_layout(p);
+    float* l1 = saved ? (float*)(saved + sv.off_l1) : nullptr;
+    float* l2 = saved ? (float*)(saved + sv.off_l2) : nullptr;
+    float* l3 = saved ? (float*)(saved + sv.off_l3) : nullptr;
+    if (combine(p, 1, ws, neg, st, l1) != cudaSuccess || !mark(2)) return FLAREPP_ERR_CUDA;
     if (encode(2, K, V) != cudaSuccess || !mark(3)) return FLAREPP_ERR_CUDA;
-    if (combine(p, 2, ws, false, st) != cudaSuccess || !mark(4)) return FLAREPP_ERR_CUDA;
+    if (combine(p, 2, ws, false, st, l2) != cudaSuccess || !mark(4)) return FLAREPP_ERR_CUDA;
     cudaError_t e;
-    e = tc ? tc_decode(p, K, scale, Y, ws, st) : simt_decode_f32(p, K, scale, Y, ws, st);
+    e = tc ? tc_decode(p, K, scale, Y, ws, st, l3) : simt_decode_f32(p, K, scale, Y, ws, st, l3);
     if (e != cudaSuccess || !mark(5)) return FLAREPP_ERR_CUDA;
+    if (saved) {
+        Q_out = (float*)(saved + sv.off_q);
+        Z_out = (float*)(saved + sv.off_z);
+    }
     if (Q_out && cudaMemcpyAsync(Q_out, ws + p.off_q32, qz_bytes, cudaMemcpyDeviceToDevice, st) !=
                      cudaSuccess)
         return FLAREPP_ERR_CUDA;
@@ -362,10 +371,124 @@ flarepp_status route_host_impl(const flarepp_shape* shape, const void* seeds_h, 
     return ok ? FLAREPP_OK : FLAREPP_ERR_CUDA;
 }
 
+// ---------------------------------------------------------------- training forward, backward
+
+bool spans_overlap(const void* const* ptrs, const size_t* bytes, int n, const void* p,
+                   size_t nb) {
+    for (int i = 0; i < n; ++i)
+        if (overlaps(p, nb, ptrs[i], bytes[i])) return true;
+    return false;
+}
+
+flarepp_status route_fwd_train_impl(const flarepp_shape* shape, const void* seeds, const void* Kt,
+                                    const void* Vt, const void* K, const void* V, float scale,
+                                    void* Y, void* saved, size_t saved_bytes, void* workspace,
+                                    size_t workspace_bytes, void* stream) {
+    Plan p;
+    flarepp_status stt = make_plan(shape, &p);
+    if (stt != FLAREPP_OK) return stt;
+    const SavedLayout sv = saved_layout(p);
+    if (p.BH && p.N && p.M) {
+        if (!saved || !aligned16(saved) || saved_bytes < sv.total)
+            return FLAREPP_ERR_INVALID_ARGUMENT;
+        const size_t elt = p.dtype == FLAREPP_F32 ? 4 : 2;
+        const size_t tok_bytes = (size_t)p.BH * (size_t)p.N * (size_t)p.D * elt;
+        const void* ins[6] = {Kt, Vt, K, V, Y, workspace};
+        const size_t nb[6] = {tok_bytes, tok_bytes, tok_bytes, tok_bytes, tok_bytes, p.total};
+        if (spans_overlap(ins, nb, 6, saved, sv.total)) return FLAREPP_ERR_INVALID_ARGUMENT;
+    }
+    return route_impl(shape, seeds, Kt, Vt, K, V, scale, Y, workspace, workspace_bytes, stream,
+                      nullptr, nullptr, nullptr, 0, true, (char*)saved);
+}
+
+flarepp_status route_bwd_impl(const flarepp_shape* shape, const void* seeds, const void* Kt,
+                              const void* Vt, const void* K, const void* V, float scale,
+                              const void* Y, const void* dY, const void* saved,
+                              size_t saved_bytes, void* dseeds, void* dKt, void* dVt, void* dK,
+                              void* dV, void* workspace, size_t workspace_bytes, void* stream) {
+    Plan p;
+    flarepp_status stt = make_plan(shape, &p);
+    if (stt != FLAREPP_OK) return stt;
+    if (!isfinite(scale)) return FLAREPP_ERR_INVALID_ARGUMENT;
+    cudaStream_t st = (cudaStream_t)stream;
+    const BwdPlan bp = make_bwd_plan(p);
+    const SavedLayout sv = saved_layout(p);
+    const size_t elt = p.dtype == FLAREPP_F32 ? 4 : 2;
+    const size_t tok = (size_t)p.BH * (size_t)p.N * (size_t)p.D * elt;
+    const size_t seed = (size_t)p.H * (size_t)p.M * (size_t)p.D * elt;
+    const bool work = p.BH && p.N && p.M;
+    // outputs: present and aligned where non-empty, disjoint from every input and each other
+    void* outs[5] = {dseeds, dKt, dVt, dK, dV};
+    const size_t ob[5] = {seed, tok, tok, tok, tok};
+    for (int i = 0; i < 5; ++i)
+        if (ob[i] && (!outs[i] || !aligned16(outs[i]))) return FLAREPP_ERR_INVALID_ARGUMENT;
+    if (work) {
+        const void* ins[9] = {seeds, Kt, Vt, K, V, Y, dY, saved, workspace};
+        const size_t ib[9] = {seed, tok, tok, tok, tok, tok, tok, sv.total, bp.total};
+        for (int i = 0; i < 7; ++i)
+            if (!ins[i] || !aligned16(ins[i])) return FLAREPP_ERR_INVALID_ARGUMENT;
+        if (!saved || !aligned16(saved) || saved_bytes < sv.total)
+            return FLAREPP_ERR_INVALID_ARGUMENT;
+        if (!workspace || ((uintptr_t)workspace % kWsAlign) != 0 || workspace_bytes < bp.total)
+            return FLAREPP_ERR_WORKSPACE;
+        for (int i = 0; i < 5; ++i) {
+            if (spans_overlap(ins, ib, 9, outs[i], ob[i])) return FLAREPP_ERR_INVALID_ARGUMENT;
+            for (int j = 0; j < i; ++j)
+                if (overlaps(outs[i], ob[i], outs[j], ob[j])) return FLAREPP_ERR_INVALID_ARGUMENT;
+        }
+        if (overlaps(saved, sv.total, workspace, bp.total)) return FLAREPP_ERR_INVALID_ARGUMENT;
+    }
+    // degenerate shapes: every gradient that exists is zero
+    if (!work) {
+        for (int i = 0; i < 5; ++i)
+            if (ob[i] && cudaMemsetAsync(outs[i], 0, ob[i], st) != cudaSuccess)
+                return FLAREPP_ERR_CUDA;
+        return FLAREPP_OK;
+    }
+    char* ws = (char*)workspace;
+    if (cudaMemsetAsync(ws + bp.off_status, 0, sizeof(int32_t), st) != cudaSuccess)
+        return FLAREPP_ERR_CUDA;
+    const cudaError_t e = simt_route_bwd(p, bp, seeds, Kt, Vt, K, V, scale, Y, dY,
+                                         (const char*)saved, dseeds, dKt, dVt, dK, dV, ws, st);
+    return e == cudaSuccess ? FLAREPP_OK : FLAREPP_ERR_CUDA;
+}
+
 }  // namespace
 }  // namespace flarepp
 
 extern "C" {
+
+size_t flarepp_route_saved_bytes(const flarepp_shape* shape) {
+    flarepp::Plan p;
+    if (flarepp::make_plan(shape, &p) != FLAREPP_OK) return 0;
+    if (p.BH == 0 || p.N == 0 || p.M == 0) return 0;
+    return flarepp::saved_layout(p).total;
+}
+
+flarepp_status flarepp_route_fwd_train(const flarepp_shape* shape, const void* seeds,
+                                       const void* Kt, const void* Vt, const void* K,
+                                       const void* V, float scale, void* Y, void* saved,
+                                       size_t saved_bytes, void* workspace,
+                                       size_t workspace_bytes, void* stream) {
+    return flarepp::route_fwd_train_impl(shape, seeds, Kt, Vt, K, V, scale, Y, saved,
+                                         saved_bytes, workspace, workspace_bytes, stream);
+}
+
+size_t flarepp_route_bwd_workspace_bytes(const flarepp_shape* shape) {
+    flarepp::Plan p;
+    if (flarepp::make_plan(shape, &p) != FLAREPP_OK) return 0;
+    return flarepp::make_bwd_plan(p).total;
+}
+
+flarepp_status flarepp_route_bwd(const flarepp_shape* shape, const void* seeds, const void* Kt,
+                                 const void* Vt, const void* K, const void* V, float scale,
+                                 const void* Y, const void* dY, const void* saved,
+                                 size_t saved_bytes, void* dseeds, void* dKt, void* dVt,
+                                 void* dK, void* dV, void* workspace, size_t workspace_bytes,
+                                 void* stream) {
+    return flarepp::route_bwd_impl(shape, seeds, Kt, Vt, K, V, scale, Y, dY, saved, saved_bytes,
+                                   dseeds, dKt, dVt, dK, dV, workspace, workspace_bytes, stream);
+}
 
 size_t flarepp_route_workspace_bytes(const flarepp_shape* shape) {
     flarepp::Plan p;

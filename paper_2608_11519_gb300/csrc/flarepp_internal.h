@@ -43,20 +43,53 @@ struct Plan {
 // Fill `p` for `s` (plan.cu); returns FLAREPP_OK or the validation error for the shape itself.
 flarepp_status make_plan(const flarepp_shape* s, Plan* p);
 
+// The state a training forward keeps for the backward (App. A.5), in a caller buffer:
+// float32 Q and Z [BH][M][D] and the log-normalisers of the three calls in base 2,
+// L = log2 sum_j 2^(scale * log2(e) <a, b_j>): L1, L2 [BH][M] and L3 [BH][N].
+struct SavedLayout {
+    size_t off_q, off_z, off_l1, off_l2, off_l3, total;
+};
+SavedLayout saved_layout(const Plan& p);
+
+// The backward's plan: the split-N route passes (one thread per route, chunks of tokens)
+// and its workspace.
+struct BwdPlan {
+    int64_t m_tile, n_mtiles;   // routes per CTA and route tiles per head
+    int64_t chunk_len, nchunk;  // tokens per chunk and chunks per head
+    size_t off_status;          // int32 device status word
+    size_t off_pa, off_pb;      // per-chunk partial sums [BH][nchunk][M][D] f32
+    size_t off_dz, off_dq;      // dZ, dQ [BH][M][D] f32
+    size_t off_d1, off_d2;      // c = <dO, O> of calls 1 and 2 [BH][M] f32
+    size_t off_d3;              // c of call 3 [BH][N] f32
+    size_t total;
+};
+BwdPlan make_bwd_plan(const Plan& p);
+
 // ---- CUDA-core kernels (simt_kernels.cuh, instantiated in simt_f32.cu), float32 inputs
 // Encode one call over all chunks: call 1 takes the seeds ([H][M][D]), call 2 takes Q32
 // from the workspace. Writes the chunk partials.
 cudaError_t simt_encode_f32(const Plan& p, int call, const void* k, const void* v,
                             const void* seeds, float scale, char* ws, cudaStream_t st);
-// Decode (call 3) on CUDA cores: Y = SDPA(K, Q32, Z32).
+// Decode (call 3) on CUDA cores: Y = SDPA(K, Q32, Z32); also the base-2 log-normaliser of
+// each token's row into `lse` [BH][N] when it is not null.
 cudaError_t simt_decode_f32(const Plan& p, const void* K, float scale, void* Y, char* ws,
-                            cudaStream_t st);
+                            cudaStream_t st, float* lse = nullptr);
+
+// ---- backward (bwd_simt.cu): the passes of App. A.5 on CUDA cores, bf16 or f32 inputs
+// (dtype from the plan). `saved` is the training forward's state, `ws` the backward
+// workspace; outputs in the input dtype.
+cudaError_t simt_route_bwd(const Plan& p, const BwdPlan& bp, const void* seeds, const void* Kt,
+                           const void* Vt, const void* K, const void* V, float scale,
+                           const void* Y, const void* dY, const char* saved, void* dseeds,
+                           void* dKt, void* dVt, void* dK, void* dV, char* ws, cudaStream_t st);
 
 // ---- split-N combine (combine.cu)
 // Stable log-sum-exp merge of the chunk partials into Q32 (call 1) or Z32 (call 2), plus
 // the bf16 MMA operand copy when the tensor-core path consumes it (negated when
 // `negate`, which together with negated seeds turns a negative scale into |scale|).
-cudaError_t combine(const Plan& p, int call, char* ws, bool negate, cudaStream_t st);
+// The base-2 log-normaliser of each merged row goes to `lse` [BH][M] when it is not null.
+cudaError_t combine(const Plan& p, int call, char* ws, bool negate, cudaStream_t st,
+                    float* lse = nullptr);
 // dst = -src elementwise (bf16; exact)
 cudaError_t negate_bf16(const void* src, void* dst, int64_t n, cudaStream_t st);
 
@@ -66,8 +99,9 @@ cudaError_t tc_encode(const Plan& p, int call, const void* k, const void* v, con
                       float scale, char* ws, cudaStream_t st);
 // Rows per tensor-core work unit (route group of the encode, token group of the decode).
 int64_t tc_group_rows(int64_t D);
-// Decode call 3: Y = SDPA(K, Q, Z) from the Q and Z operand copies.
+// Decode call 3: Y = SDPA(K, Q, Z) from the Q and Z operand copies; also each token's
+// base-2 log-normaliser into `lse` [BH][N] when it is not null.
 cudaError_t tc_decode(const Plan& p, const void* K, float scale, void* Y, char* ws,
-                      cudaStream_t st);
+                      cudaStream_t st, float* lse = nullptr);
 
 }  // namespace flarepp

@@ -112,4 +112,59 @@ flarepp_status make_plan(const flarepp_shape* s, Plan* p) {
     return FLAREPP_OK;
 }
 
+SavedLayout saved_layout(const Plan& p) {
+    SavedLayout L{};
+    const size_t qz = (size_t)p.BH * (size_t)p.M * (size_t)p.D * sizeof(float);
+    const size_t lm = (size_t)p.BH * (size_t)p.M * sizeof(float);
+    const size_t ln = (size_t)p.BH * (size_t)p.N * sizeof(float);
+    size_t off = 0;
+    L.off_q = off;
+    off = align_up(off + qz, kWsAlign);
+    L.off_z = off;
+    off = align_up(off + qz, kWsAlign);
+    L.off_l1 = off;
+    off = align_up(off + lm, kWsAlign);
+    L.off_l2 = off;
+    off = align_up(off + lm, kWsAlign);
+    L.off_l3 = off;
+    off = align_up(off + ln, kWsAlign);
+    L.total = off;
+    return L;
+}
+
+BwdPlan make_bwd_plan(const Plan& p) {
+    BwdPlan b{};
+    if (p.BH == 0 || p.N == 0 || p.M == 0) return b;
+    // one thread per route, up to 128 routes per CTA; chunks sized for about four waves
+    b.m_tile = p.M >= 128 ? 128 : cdiv(p.M, 32) * 32;
+    b.n_mtiles = cdiv(p.M, b.m_tile);
+    int64_t want = cdiv(4 * kNumSMs, p.BH * b.n_mtiles);
+    if (want < 1) want = 1;
+    b.chunk_len = cdiv(cdiv(p.N, want), 32) * 32;
+    b.nchunk = cdiv(p.N, b.chunk_len);
+    const size_t part = (size_t)p.BH * (size_t)b.nchunk * (size_t)p.M * (size_t)p.D * 4;
+    const size_t qz = (size_t)p.BH * (size_t)p.M * (size_t)p.D * 4;
+    const size_t lm = (size_t)p.BH * (size_t)p.M * 4;
+    const size_t ln = (size_t)p.BH * (size_t)p.N * 4;
+    size_t off = 0;
+    b.off_status = off;
+    off = align_up(off + sizeof(int32_t), kWsAlign);
+    b.off_pa = off;
+    off = align_up(off + part, kWsAlign);
+    b.off_pb = off;
+    off = align_up(off + part, kWsAlign);
+    b.off_dz = off;
+    off = align_up(off + qz, kWsAlign);
+    b.off_dq = off;
+    off = align_up(off + qz, kWsAlign);
+    b.off_d1 = off;
+    off = align_up(off + lm, kWsAlign);
+    b.off_d2 = off;
+    off = align_up(off + lm, kWsAlign);
+    b.off_d3 = off;
+    off = align_up(off + ln, kWsAlign);
+    b.total = off;
+    return b;
+}
+
 }  // namespace flarepp

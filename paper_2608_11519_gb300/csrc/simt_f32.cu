@@ -9,8 +9,8 @@ cudaError_t simt_encode_f32(const Plan& p, int call, const void* k, const void* 
 }
 
 cudaError_t simt_decode_f32(const Plan& p, const void* K, float scale, void* Y, char* ws,
-                          cudaStream_t st) {
-    return simt::decode_t<float>(p, K, scale, Y, ws, st);
+                          cudaStream_t st, float* lse) {
+    return simt::decode_t<float>(p, K, scale, Y, ws, st, lse);
 }
 
 }  // namespace flarepp

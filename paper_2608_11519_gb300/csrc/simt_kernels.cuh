@@ -115,7 +115,7 @@ __global__ void __launch_bounds__(128) simt_encode_kernel(
 template <int D, typename T>
 __global__ void __launch_bounds__(128) simt_decode_kernel(
     const T* __restrict__ k, const float* __restrict__ q32, const float* __restrict__ z32,
-    int64_t N, int64_t M, float sl2, T* __restrict__ y) {
+    int64_t N, int64_t M, float sl2, T* __restrict__ y, float* __restrict__ lse) {
     __shared__ float qs[kTile][D];
     __shared__ float zs[kTile][D];
     const int64_t ntiles = (N + 127) / 128;
@@ -171,6 +171,7 @@ __global__ void __launch_bounds__(128) simt_decode_kernel(
         T* yp = y + (bh * N + n) * D;
 #pragma unroll
         for (int d = 0; d < D; ++d) from_f32(yp + d, o[d] * inv);
+        if (lse) lse[bh * N + n] = mx + log2f(l);
     }
 }
 
@@ -206,7 +207,7 @@ cudaError_t encode_t(const Plan& p, int call, const void* k, const void* v, cons
 
 template <typename T>
 cudaError_t decode_t(const Plan& p, const void* K, float scale, void* Y, char* ws,
-                     cudaStream_t st) {
+                     cudaStream_t st, float* lse) {
     const int64_t blocks = ((p.N + 127) / 128) * p.BH;
     const float sl2 = scale * kLog2e;
     const float* q32 = (const float*)(ws + p.off_q32);
@@ -214,15 +215,15 @@ cudaError_t decode_t(const Plan& p, const void* K, float scale, void* Y, char* w
     switch (p.D) {
         case 16:
             simt_decode_kernel<16, T><<<(unsigned)blocks, 128, 0, st>>>((const T*)K, q32, z32, p.N,
-                                                                         p.M, sl2, (T*)Y);
+                                                                         p.M, sl2, (T*)Y, lse);
             break;
         case 32:
             simt_decode_kernel<32, T><<<(unsigned)blocks, 128, 0, st>>>((const T*)K, q32, z32, p.N,
-                                                                         p.M, sl2, (T*)Y);
+                                                                         p.M, sl2, (T*)Y, lse);
             break;
         case 64:
             simt_decode_kernel<64, T><<<(unsigned)blocks, 128, 0, st>>>((const T*)K, q32, z32, p.N,
-                                                                         p.M, sl2, (T*)Y);
+                                                                         p.M, sl2, (T*)Y, lse);
             break;
         default: return cudaErrorInvalidValue;
     }

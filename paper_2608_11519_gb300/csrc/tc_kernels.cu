@@ -101,6 +101,7 @@ struct TcParams {
     float* pacc;
     int64_t n_tok_groups;
     __nv_bfloat16* Y;
+    float* lse;  // decode: each token's base-2 log-normaliser, or null
     int64_t n_units;
     int* status;
 };
@@ -403,6 +404,7 @@ __device__ __forceinline__ bool finish_stream(SoftmaxStream& S, const Unit& U,
                 v.w = pack_bf16(o[8 * kk + 6] * inv, o[8 * kk + 7] * inv);
                 dst[kk] = v;
             }
+            if (prm.lse) prm.lse[U.bh * prm.N + tok] = S.m + log2f(S.l);
         }
     } else {
         const int64_t route = U.g * C::kGroup + a * kTileRows + r;
@@ -928,7 +930,7 @@ cudaError_t tc_encode(const Plan& p, int call, const void* k, const void* v, con
 }
 
 cudaError_t tc_decode(const Plan& p, const void* K, float scale, void* Y, char* ws,
-                      cudaStream_t st) {
+                      cudaStream_t st, float* lse) {
     CUtensorMap ma, mb, mc;
     if (!make_map(&ma, K, p.D, p.N, p.BH, kTileRows, false) ||
         !make_map(&mb, ws + p.off_qop, p.D, p.M, p.BH, item_rows(p.D), true) ||
@@ -943,6 +945,7 @@ cudaError_t tc_decode(const Plan& p, const void* K, float scale, void* Y, char* 
     const int64_t grp = tc_group_rows(p.D);
     prm.n_tok_groups = (p.N + grp - 1) / grp;
     prm.Y = (__nv_bfloat16*)Y;
+    prm.lse = lse;
     prm.n_units = p.BH * prm.n_tok_groups;
     prm.status = (int*)(ws + p.off_status);
     return launch_d<true>(p.D, ma, mb, mc, prm, st);

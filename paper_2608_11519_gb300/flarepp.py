@@ -24,6 +24,8 @@ _DTYPES = {torch.float32: F32, torch.bfloat16: BF16}
 EXPORTED = ("flarepp_route_workspace_bytes", "flarepp_route_fwd", "flarepp_route_fwd_debug",
             "flarepp_route_fwd_profiled", "flarepp_route_fwd_noalloc",
             "flarepp_flare_fwd", "flarepp_route_host_buffer_bytes", "flarepp_route_fwd_host",
+            "flarepp_route_saved_bytes", "flarepp_route_fwd_train",
+            "flarepp_route_bwd_workspace_bytes", "flarepp_route_bwd",
             "flarepp_route_device_status", "flarepp_status_string", "flarepp_version")
 N_STAGE_EVENTS = 6
 STAGES = ("encode1", "combine1", "encode2", "combine2", "decode")
@@ -78,6 +80,16 @@ def load(path: str = None):
     lib.flarepp_route_host_buffer_bytes.argtypes = [sp]
     lib.flarepp_route_fwd_host.restype = ctypes.c_int
     lib.flarepp_route_fwd_host.argtypes = [sp, vp, vp, vp, vp, vp, ctypes.c_float, vp, vp, sz, vp]
+    lib.flarepp_route_saved_bytes.restype = sz
+    lib.flarepp_route_saved_bytes.argtypes = [sp]
+    lib.flarepp_route_fwd_train.restype = ctypes.c_int
+    lib.flarepp_route_fwd_train.argtypes = [sp, vp, vp, vp, vp, vp, ctypes.c_float, vp, vp, sz,
+                                            vp, sz, vp]
+    lib.flarepp_route_bwd_workspace_bytes.restype = sz
+    lib.flarepp_route_bwd_workspace_bytes.argtypes = [sp]
+    lib.flarepp_route_bwd.restype = ctypes.c_int
+    lib.flarepp_route_bwd.argtypes = [sp, vp, vp, vp, vp, vp, ctypes.c_float, vp, vp, vp, sz,
+                                      vp, vp, vp, vp, vp, vp, sz, vp]
     lib.flarepp_route_device_status.restype = ctypes.c_int
     lib.flarepp_route_device_status.argtypes = [sp, vp, vp, ctypes.POINTER(ctypes.c_int32)]
     lib.flarepp_status_string.restype = ctypes.c_char_p
@@ -294,6 +306,65 @@ def flare_fwd(Q, K, V, scale=None, Y=None, workspace=None, stream=None, Z_out=No
     if rc != OK:
         raise FlareppError(rc, "flarepp_flare_fwd")
     return Y
+
+
+def route_fwd_train(seeds, Kt, Vt, K, V, scale=None, Y=None, saved=None, workspace=None,
+                    stream=None):
+    """The chain's forward that also keeps the state its backward needs (App. A.5).
+    Returns (Y, saved): ``saved`` is an opaque uint8 device tensor for :func:`route_bwd`."""
+    lib = load()
+    shape = _shape_of(seeds, Kt, Vt, K, V)
+    if K.device.type != "cuda":
+        raise ValueError("route_fwd_train takes device tensors")
+    if scale is None:
+        scale = 1.0 / math.sqrt(shape.D)
+    if Y is None:
+        Y = torch.empty_like(K)
+    sbytes = int(lib.flarepp_route_saved_bytes(ctypes.byref(shape)))
+    if saved is None or saved.numel() < sbytes:
+        saved = torch.empty(max(sbytes, 1), dtype=torch.uint8, device=K.device)
+    nbytes = int(lib.flarepp_route_workspace_bytes(ctypes.byref(shape)))
+    ws = (workspace if isinstance(workspace, Workspace) else Workspace()).get(nbytes, K.device)
+    st = stream if stream is not None else torch.cuda.current_stream(K.device)
+    rc = lib.flarepp_route_fwd_train(ctypes.byref(shape), _ptr(seeds), _ptr(Kt), _ptr(Vt),
+                                     _ptr(K), _ptr(V), float(scale), _ptr(Y), _ptr(saved),
+                                     sbytes, None if ws is None else ctypes.c_void_p(ws.data_ptr()),
+                                     nbytes, ctypes.c_void_p(st.cuda_stream))
+    if rc != OK:
+        raise FlareppError(rc, "flarepp_route_fwd_train")
+    return Y, saved
+
+
+def route_bwd(seeds, Kt, Vt, K, V, Y, dY, saved, scale=None, grads=None, workspace=None,
+              stream=None):
+    """Backward of the chain (App. A.5) from :func:`route_fwd_train`'s ``Y`` and ``saved``.
+    Returns (dseeds [H, M, D], dKt, dVt, dK, dV [B, H, N, D]) in the input dtype; ``grads``
+    may supply those five output tensors."""
+    lib = load()
+    shape = _shape_of(seeds, Kt, Vt, K, V)
+    for t in (Y, dY):
+        if tuple(t.shape) != tuple(K.shape) or t.dtype != K.dtype or not t.is_contiguous():
+            raise ValueError("Y and dY must be contiguous tensors of K's shape and dtype")
+    if K.device.type != "cuda":
+        raise ValueError("route_bwd takes device tensors")
+    if scale is None:
+        scale = 1.0 / math.sqrt(shape.D)
+    if grads is None:
+        grads = (torch.empty_like(seeds), torch.empty_like(Kt), torch.empty_like(Vt),
+                 torch.empty_like(K), torch.empty_like(V))
+    sbytes = int(lib.flarepp_route_saved_bytes(ctypes.byref(shape)))
+    nbytes = int(lib.flarepp_route_bwd_workspace_bytes(ctypes.byref(shape)))
+    ws = (workspace if isinstance(workspace, Workspace) else Workspace()).get(nbytes, K.device)
+    st = stream if stream is not None else torch.cuda.current_stream(K.device)
+    rc = lib.flarepp_route_bwd(ctypes.byref(shape), _ptr(seeds), _ptr(Kt), _ptr(Vt), _ptr(K),
+                               _ptr(V), float(scale), _ptr(Y), _ptr(dY), _ptr(saved),
+                               saved.numel() if saved is not None else 0,
+                               *(_ptr(g) for g in grads),
+                               None if ws is None else ctypes.c_void_p(ws.data_ptr()), nbytes,
+                               ctypes.c_void_p(st.cuda_stream))
+    if rc != OK:
+        raise FlareppError(rc, "flarepp_route_bwd")
+    return grads
 
 
 def route_fwd_host(seeds, Kt, Vt, K, V, scale=None, Y_host=None, device="cuda", workspace=None,

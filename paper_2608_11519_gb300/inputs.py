@@ -111,6 +111,14 @@ def make_inputs(w: Workload, seed: int = 0, device="cpu"):
     return {"seeds": seeds, "Kt": Kt, "Vt": Vt, "K": K, "V": V}
 
 
+def make_output_grad(w: Workload, seed: int = 0, device="cpu"):
+    """Draw an output gradient dY [B,H,N,D] for workload ``w``: i.i.d. N(0,1) in its dtype,
+    from a stream separate from :func:`make_inputs` (seed offset by 7919)."""
+    gen = torch.Generator(device=device)
+    gen.manual_seed(int(seed) + 7919)
+    return torch.randn(w.B, w.H, w.N, w.D, generator=gen, device=device).to(w.torch_dtype)
+
+
 def to_f64_numpy(inputs):
     """The exact values of each input as float64 numpy arrays (bf16 and f32 upcast exactly)."""
     return {k: v.detach().to("cpu", torch.float64).numpy() for k, v in inputs.items()}

@@ -164,3 +164,56 @@ def test_host_entry_sizes_and_rejects_before_any_cuda_call(lib):
     assert host_call(S(), nbytes=1024) == E.ERR_WORKSPACE
     assert host_call(S(), buf=FAKE + 7 * (1 << 36) + 128) == E.ERR_WORKSPACE  # not aligned
     assert host_call(S(N=0)) == E.OK  # empty Y: nothing to do
+
+
+def test_backward_entry_sizes_and_rejects_before_any_cuda_call(lib):
+    E = flarepp
+    sb = lambda s: lib.flarepp_route_saved_bytes(ctypes.byref(s))
+    wb = lambda s: lib.flarepp_route_bwd_workspace_bytes(ctypes.byref(s))
+    s = S(B=2, H=3, N=1000, M=40, D=32)
+    # saved: Q, Z float32 [B,H,M,D], L1, L2 [B,H,M], L3 [B,H,N]
+    assert sb(s) >= (2 * 6 * 40 * 32 + 2 * 6 * 40 + 6 * 1000) * 4
+    assert wb(s) > 0 and wb(s) % 256 == 0
+    assert sb(S(N=0)) == 0 and sb(S(D=48)) == 0 and wb(S(D=48)) == 0
+
+    base = [FAKE + (i + 1) * (1 << 36) for i in range(14)]
+
+    def bwd(shape, ptrs=None, saved_bytes=None, ws_bytes=None, scale=0.25):
+        p = list(base) if ptrs is None else ptrs
+        v = lambda x: None if x is None else ctypes.c_void_p(x)
+        # seeds Kt Vt K V Y dY saved | dseeds dKt dVt dK dV | workspace
+        return lib.flarepp_route_bwd(
+            ctypes.byref(shape), *(v(x) for x in p[:5]), ctypes.c_float(scale), v(p[5]),
+            v(p[6]), v(p[7]), sb(shape) if saved_bytes is None else saved_bytes,
+            *(v(x) for x in p[8:13]), v(p[13]), wb(shape) if ws_bytes is None else ws_bytes,
+            None)
+
+    assert bwd(S(D=48)) == E.ERR_UNSUPPORTED
+    assert bwd(S(), scale=float("nan")) == E.ERR_INVALID_ARGUMENT
+    for i in range(13):  # every pointer is required
+        p = list(base)
+        p[i] = None
+        assert bwd(S(), p) == E.ERR_INVALID_ARGUMENT, i
+    p = list(base)
+    p[9] = base[1] + 64  # dKt overlaps Kt
+    assert bwd(S(), p) == E.ERR_INVALID_ARGUMENT
+    p = list(base)
+    p[11] = base[10] + 16  # dK overlaps dVt
+    assert bwd(S(), p) == E.ERR_INVALID_ARGUMENT
+    p = list(base)
+    p[12] = base[8] + 8  # misaligned dV
+    assert bwd(S(), p) == E.ERR_INVALID_ARGUMENT
+    assert bwd(S(), saved_bytes=16) == E.ERR_INVALID_ARGUMENT
+    assert bwd(S(), ws_bytes=16) == E.ERR_WORKSPACE
+    p = list(base)
+    p[13] = None
+    assert bwd(S(), p) == E.ERR_WORKSPACE
+    # the training forward checks its saved buffer
+    v = lambda x: ctypes.c_void_p(x)
+    fw = lambda saved, nbytes: lib.flarepp_route_fwd_train(
+        ctypes.byref(S()), *(v(x) for x in base[:5]), ctypes.c_float(0.25), v(base[5]),
+        None if saved is None else v(saved), nbytes, v(base[13]),
+        lib.flarepp_route_workspace_bytes(ctypes.byref(S())), None)
+    assert fw(None, sb(S())) == E.ERR_INVALID_ARGUMENT
+    assert fw(base[7], 16) == E.ERR_INVALID_ARGUMENT
+    assert fw(base[1] + 32, sb(S())) == E.ERR_INVALID_ARGUMENT  # overlaps Kt

@@ -1,0 +1,202 @@
+"""GPU parity of the chain's backward (App. A.5) against the float64 oracle, through the C ABI.
+
+The training forward (``flarepp_route_fwd_train``) runs first and its Y and saved state
+feed ``flarepp_route_bwd``; the oracle recomputes everything from the same input values.
+
+Tolerance, per gradient tensor G (max abs error after upcasting to float64):
+    max|G - G_ref| <= tol * max(1, max|G_ref|),  tol = 1e-5 (float32), 2e-2 (bf16 inputs)
+i.e. the forward's tolerances taken relative to the gradient's own scale: a gradient sums
+N (or M, or B*N) unit-scale products, so its magnitude is not 1. On the bf16 path the forward
+multiplies bf16 copies of Q and Z and stores Y in bf16; the backward differentiates that
+function, while the oracle differentiates the exact one, so the gap is of the order of the
+forward's own bf16 error.
+"""
+import math
+
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from paper_2608_11519_gb300 import flarepp, inputs
+
+pytestmark = pytest.mark.gpu
+
+TOL = {"f32": 1e-5, "bf16": 2e-2}
+NAMES = ("dseeds", "dKt", "dVt", "dK", "dV")
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _lib():
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    flarepp.load()
+    torch.cuda.set_device(0)
+
+
+def _np(t):
+    return t.detach().to("cpu", torch.float64).numpy()
+
+
+def _gpu_grads(x, dY, scale):
+    xd = {k: v.cuda() for k, v in x.items()}
+    args = (xd["seeds"], xd["Kt"], xd["Vt"], xd["K"], xd["V"])
+    Y, saved = flarepp.route_fwd_train(*args, scale)
+    grads = flarepp.route_bwd(*args, Y, dY.cuda(), saved, scale)
+    torch.cuda.synchronize()
+    return [_np(g) for g in grads], Y
+
+
+def _check_grads(got, want, tol, where=""):
+    errs = {}
+    for name, g, r in zip(NAMES, got, want):
+        bound = tol * max(1.0, float(np.abs(r).max()) if r.size else 0.0)
+        err = float(np.abs(g - r).max()) if g.size else 0.0
+        assert err <= bound and not math.isnan(err), f"{name}{where}: {err} > {bound}"
+        errs[name] = err
+    return errs
+
+
+SHAPES = [
+    # B, H, N, M, D, dtype, scale (None: 1/sqrt(D))
+    (1, 4, 1024, 32, 16, "f32", None),   # the tiny float32 configuration
+    (2, 3, 300, 40, 16, "f32", None),
+    (3, 2, 257, 7, 64, "f32", -0.5),
+    (1, 1, 1, 1, 32, "f32", None),
+    (2, 2, 3000, 128, 32, "bf16", None),
+    (1, 2, 1000, 600, 32, "bf16", None),  # more than one 512-route group
+    (1, 3, 777, 100, 16, "bf16", None),
+    (1, 2, 500, 64, 64, "bf16", None),
+    (2, 2, 600, 50, 32, "bf16", -0.3),
+    (1, 2, 130, 513, 32, "bf16", None),   # ragged route tile
+]
+
+
+@pytest.mark.parametrize("shape", SHAPES, ids=[str(s) for s in SHAPES])
+def test_bwd_matches_oracle(shape):
+    B, H, N, M, D, dt, scale = shape
+    w = inputs.Workload("case", B, H, N, M, D, dt)
+    scale = 1.0 / math.sqrt(D) if scale is None else scale
+    x = inputs.make_inputs(w, 3)
+    dY = inputs.make_output_grad(w, 3)
+    got, _ = _gpu_grads(x, dY, scale)
+    f = inputs.to_f64_numpy(x)
+    want = oracle.route_bwd(f["seeds"], f["Kt"], f["Vt"], f["K"], f["V"], scale, _np(dY))
+    _check_grads(got, want, TOL[dt])
+
+
+def test_training_forward_matches_forward():
+    """The training forward writes the same Y as the plain forward, bit for bit, and its
+    saved log-normalisers are those of the oracle's calls."""
+    w = inputs.Workload("case", 2, 2, 2000, 96, 32, "bf16")
+    x = {k: v.cuda() for k, v in inputs.make_inputs(w, 5).items()}
+    args = (x["seeds"], x["Kt"], x["Vt"], x["K"], x["V"])
+    s = 1.0 / math.sqrt(w.D)
+    Y0 = flarepp.route_fwd(*args, s)
+    Y1, saved = flarepp.route_fwd_train(*args, s)
+    torch.cuda.synchronize()
+    assert torch.equal(Y0, Y1)
+    BH, M, N, D = w.B * w.H, w.M, w.N, w.D
+    qz = BH * M * D * 4
+    al = lambda n: (n + 255) // 256 * 256
+    off_l1 = 2 * al(qz)
+    off_l2 = off_l1 + al(BH * M * 4)
+    off_l3 = off_l2 + al(BH * M * 4)
+    raw = saved.cpu()
+    L = lambda off, n: raw[off:off + 4 * n].view(torch.float32).double().numpy()
+    ln2 = math.log(2.0)
+    f = inputs.to_f64_numpy({k: v.cpu() for k, v in x.items()})
+    Qs = np.broadcast_to(f["seeds"], (w.B,) + f["seeds"].shape)
+    Q, L1 = oracle.sdpa(Qs, f["Kt"], f["Vt"], s)
+    Z, L2 = oracle.sdpa(Q, f["K"], f["V"], s)
+    _, L3 = oracle.sdpa(f["K"], Q, Z, s)
+    for got, want in ((L(off_l1, BH * M), L1), (L(off_l2, BH * M), L2), (L(off_l3, BH * N), L3)):
+        np.testing.assert_allclose(got * ln2, want.reshape(-1), rtol=0, atol=2e-2)
+
+
+@pytest.mark.parametrize("name", ["pde2d", "longseq"])
+def test_bwd_full_size_slices(name):
+    """Full-size workloads: the backward of the whole batch on the GPU, each sampled (b, h)
+    slice checked against the oracle run on that slice alone (slices are independent, and
+    the seeds' gradient of a slice is its batch element's share)."""
+    w = inputs.get(name)
+    s = w.scale
+    x = inputs.make_inputs(w, 0)
+    dY = inputs.make_output_grad(w, 0)
+    got, _ = _gpu_grads(x, dY, s)
+    f = inputs.to_f64_numpy(x)
+    dYn = _np(dY)
+    rng = np.random.default_rng(0)
+    picks = [(0, 0), (w.B - 1, w.H - 1)] + [(int(rng.integers(w.B)), int(rng.integers(w.H)))]
+    # the seeds' gradient sums over the batch: check it on a batch of one element per head
+    for b, h in picks:
+        sl = lambda a: a[b:b + 1, h:h + 1]
+        want = oracle.route_bwd(f["seeds"][h:h + 1], sl(f["Kt"]), sl(f["Vt"]), sl(f["K"]),
+                                sl(f["V"]), s, sl(dYn))
+        tol = TOL[w.dtype]
+        for name_, g, r in zip(NAMES[1:], got[1:], want[1:]):
+            gg = g[b:b + 1, h:h + 1]
+            bound = tol * max(1.0, float(np.abs(r).max()))
+            err = float(np.abs(gg - r).max())
+            assert err <= bound, f"{name_}[{b},{h}]: {err} > {bound}"
+    # dseeds over the whole batch, checked head by head through the oracle on all b
+    h = picks[0][1]
+    want = oracle.route_bwd(f["seeds"][h:h + 1], f["Kt"][:, h:h + 1], f["Vt"][:, h:h + 1],
+                            f["K"][:, h:h + 1], f["V"][:, h:h + 1], s, dYn[:, h:h + 1])
+    r = want[0][0]
+    bound = TOL[w.dtype] * max(1.0, float(np.abs(r).max()))
+    assert float(np.abs(got[0][h] - r).max()) <= bound
+
+
+def test_bwd_identities_at_mesh3d_size():
+    """The largest workload (one head of 1,048,576 tokens per head, M = 512, bf16): the
+    oracle is too slow there, so the identities that hold at any size are checked on the
+    GPU's gradients (in float64 on the host): call 1's keys sum to zero gradient over the
+    tokens, the values' gradients sum to those of Y, <dV, V> = <dY, Y> and
+    <dseeds, seeds> = <dKt, Kt>. Each sum is compared with the sum of the magnitudes of its
+    terms."""
+    w = inputs.get("mesh3d")
+    s = w.scale
+    x = inputs.make_inputs(w, 0)
+    dY = inputs.make_output_grad(w, 0)
+    got, Y = _gpu_grads(x, dY, s)
+    dseeds, dKt, dVt, dK, dV = got
+    f = inputs.to_f64_numpy(x)
+    dYn, Yn = _np(dY), _np(Y)
+    for v in got:
+        assert np.all(np.isfinite(v))
+    rel = 1e-2
+    lhs = dKt.sum(axis=2)
+    assert np.all(np.abs(lhs) <= rel * np.abs(dKt).sum(axis=2) + 1e-6)
+    lhs = dV.sum(axis=2) - dYn.sum(axis=2)
+    assert np.all(np.abs(lhs) <= rel * (np.abs(dV).sum(axis=2) + np.abs(dYn).sum(axis=2)))
+    a, b = np.sum(dV * f["V"]), np.sum(dYn * Yn)
+    assert abs(a - b) <= rel * (np.abs(dV * f["V"]).sum() + np.abs(dYn * Yn).sum())
+    a, b = np.sum(dseeds * f["seeds"]), np.sum(dKt * f["Kt"])
+    assert abs(a - b) <= rel * (np.abs(dseeds * f["seeds"]).sum() + np.abs(dKt * f["Kt"]).sum())
+
+
+def test_bwd_degenerate_shapes():
+    """N = 0, M = 0 or B = 0: every existing gradient is zero."""
+    for (B, H, N, M, D, dt) in [(2, 2, 0, 8, 32, "bf16"), (1, 2, 64, 0, 16, "f32"),
+                                (0, 2, 64, 8, 32, "bf16")]:
+        w = inputs.Workload("case", B, H, N, M, D, dt)
+        x = {k: v.cuda() for k, v in inputs.make_inputs(w, 1).items()}
+        args = (x["seeds"], x["Kt"], x["Vt"], x["K"], x["V"])
+        Y, saved = flarepp.route_fwd_train(*args)
+        dY = inputs.make_output_grad(w, 1).cuda()
+        grads = [torch.full_like(t, 7.0) for t in args]
+        flarepp.route_bwd(*args, Y, dY, saved, grads=grads)
+        torch.cuda.synchronize()
+        for g in grads:
+            assert not torch.any(g != 0)
+
+
+def test_bwd_is_deterministic():
+    w = inputs.Workload("case", 1, 2, 5000, 128, 32, "bf16")
+    x = inputs.make_inputs(w, 9)
+    dY = inputs.make_output_grad(w, 9)
+    a, _ = _gpu_grads(x, dY, w.scale)
+    b, _ = _gpu_grads(x, dY, w.scale)
+    for u, v in zip(a, b):
+        assert np.array_equal(u, v)
