@@ -21,6 +21,7 @@ import sys
 import tempfile
 import time
 
+import numpy as np
 import torch
 
 ROOT = os.path.dirname(os.path.abspath(__file__))
@@ -186,6 +187,9 @@ def oracle_call(f, w, variant):
         return oracle.flare(f["seeds"], f["K"], f["V"], w.scale)
     if variant == "shared":
         return oracle.route(f["seeds"], f["K"], f["V"], f["K"], f["V"], w.scale)
+    if variant == "train":  # the oracle's backward runs the forward itself
+        dY = np.ones_like(f["K"])
+        return oracle.route_bwd(f["seeds"], f["Kt"], f["Vt"], f["K"], f["V"], w.scale, dY)
     return oracle.route(f["seeds"], f["Kt"], f["Vt"], f["K"], f["V"], w.scale)
 
 
@@ -229,7 +233,7 @@ def run_reference(args, w):
     value = n / dt
     sample = (f"one head, N={n} tokens of the {w.name} shape (M={w.M}, D={w.D}), float64 oracle "
               f"on the host cores, per step")
-    metric = FLARE_METRIC if args.variant == "flare" else METRIC
+    metric = {"flare": FLARE_METRIC, "train": TRAIN_METRIC}.get(args.variant, METRIC)
     line = {"impl": "reference", "metric": metric, "value": value, "unit": UNIT,
             "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
             "ms_per_step": dt * 1e3, "higher_is_better": True, "scaling": "weak",
@@ -359,6 +363,105 @@ def run_flare(args, w, flarepp, world, rank, dev, peaks, x, Y, ws, stream):
     return 0
 
 
+TRAIN_METRIC = ("routed tokens·heads/sec for a training step of the 3-call FLARE++ chain "
+                "(forward with saved state + backward); % of roofline")
+
+
+def run_train(args, w, flarepp, world, rank, dev, peaks, x, Y, ws, stream):
+    """A training step of the chain: flarepp_route_fwd_train then flarepp_route_bwd (App. A.5)
+    on device-resident inputs and output gradient, each part bracketed by CUDA events."""
+    args_ = (x["seeds"], x["Kt"], x["Vt"], x["K"], x["V"])
+    dY = inputs.make_output_grad(w, args.seed + rank, device=dev)
+    saved = None
+    ws_b = flarepp.Workspace()
+    grads = tuple(torch.empty_like(t) for t in args_)
+
+    def step(ev=None):
+        nonlocal saved
+        if ev:
+            ev[0].record(stream)
+        _, saved = flarepp.route_fwd_train(*args_, w.scale, Y=Y, saved=saved, workspace=ws,
+                                           stream=stream)
+        if ev:
+            ev[1].record(stream)
+        flarepp.route_bwd(*args_, Y, dY, saved, w.scale, grads=grads, workspace=ws_b,
+                          stream=stream)
+        if ev:
+            ev[2].record(stream)
+
+    for _ in range(args.warmup):
+        step()
+    torch.cuda.synchronize(dev)
+    evs = [[torch.cuda.Event(enable_timing=True) for _ in range(3)] for _ in range(args.steps)]
+    clocks = ClockSampler()
+    if rank == 0:
+        clocks.start()
+        time.sleep(0.3)
+    t0 = torch.cuda.Event(enable_timing=True)
+    t1 = torch.cuda.Event(enable_timing=True)
+    barrier(world)
+    torch.cuda.synchronize(dev)
+    t0.record(stream)
+    for i in range(args.steps):
+        step(evs[i])
+    t1.record(stream)
+    torch.cuda.synchronize(dev)
+    barrier(world)
+    clk = clocks.stop(dev.index) if rank == 0 else None
+    ms = max_over_ranks(t0.elapsed_time(t1), world) / args.steps
+    fwd_ms = sum(e[0].elapsed_time(e[1]) for e in evs) / args.steps
+    bwd_ms = sum(e[1].elapsed_time(e[2]) for e in evs) / args.steps
+    tok = w.B * w.H * w.N
+    value = tok * world / (ms * 1e-3)
+    # backward algorithmic work: per SDPA, S (recomputed), dP, dV, dK and dQ, 2 NMD flops
+    # each: 30 BNMHD over the three calls; reads Kt, Vt, K, V, Y, dY and writes four
+    # gradients: 10 BHND elements
+    flops = 30.0 * tok * w.M * w.D
+    byts = 10.0 * tok * w.D * w.elt_bytes
+    tc_peak = peaks["bf16_tflops_sustained"] if w.dtype == "bf16" else None
+    bw = peaks["hbm_gbs"]
+    t_tc = flops / (tc_peak * 1e12) if tc_peak else 0.0
+    t_mem = byts / (bw * 1e9)
+    if t_tc >= t_mem and tc_peak:
+        roof = {"bound": "tensor", "achieved": flops / (bwd_ms * 1e-3) / 1e12, "peak": tc_peak,
+                "unit": "TFLOP/s", "peak_kind": "bf16_tflops_sustained (" + peaks["source"] + ")"}
+    else:
+        roof = {"bound": "hbm", "achieved": byts / (bwd_ms * 1e-3) / 1e9, "peak": bw,
+                "unit": "GB/s", "peak_kind": "hbm_gbs (" + peaks["source"] + ")"}
+    roof["frac"] = roof["achieved"] / roof["peak"]
+    roof["kernel"] = "backward (all passes)"
+    roof["ms_per_launch"] = bwd_ms
+    roof["algorithmic_flops_per_launch"] = flops
+    roof["algorithmic_bytes_per_launch"] = byts
+    roof["traffic"] = None
+    t_step = max((12.0 + 30.0) * tok * w.M * w.D / ((tc_peak or peaks["bf16_tflops"]) * 1e12),
+                 15.0 * tok * w.D * w.elt_bytes / (bw * 1e9))
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        cpu = cpu_oracle_sample(w, args.cpu_seconds, args.seed, "train")
+    if rank == 0:
+        line = {
+            "metric": TRAIN_METRIC, "value": value, "unit": UNIT, "n_gpus": world,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+            "dtype": "bf16" if w.dtype == "bf16" else "f32", "data": "synthetic",
+            "config": {"workload": w.name, "variant": "train", "B": w.B, "H": w.H, "N": w.N,
+                       "M": w.M, "D": w.D, "l2": "inputs larger than L2 (no flush)",
+                       "parallelism": f"replicas x{world}"},
+            "stage_ms": {"forward_train": fwd_ms, "backward": bwd_ms},
+            "roofline": roof,
+            "step_roofline": {"roofline_us": t_step * 1e6, "frac": t_step / (ms * 1e-3),
+                              "flops": "42 BNMHD", "tensors": 15},
+            "cpu_baseline": cpu, "e2e": None, "clocks": clk,
+            "gpu_launches": None,
+        }
+        print(json.dumps(line), flush=True)
+    if world > 1:
+        import torch.distributed as dist
+        dist.destroy_process_group()
+    return 0
+
+
 def run_ours(args, w):
     from paper_2608_11519_gb300 import flarepp
 
@@ -376,6 +479,8 @@ def run_ours(args, w):
         args_ = (x["seeds"], x["K"], x["V"], x["K"], x["V"])
     if args.variant == "flare":
         return run_flare(args, w, flarepp, world, rank, dev, peaks, x, Y, ws, stream)
+    if args.variant == "train":
+        return run_train(args, w, flarepp, world, rank, dev, peaks, x, Y, ws, stream)
 
     ev_sets = [flarepp.StageEvents(stream) for _ in range(args.steps)]
     warm_ev = flarepp.StageEvents(stream)
@@ -507,9 +612,11 @@ def main():
     ap.add_argument("--impl", choices=("ours", "reference"), default="ours")
     ap.add_argument("--workload", default="mesh3d", choices=sorted(inputs.WORKLOADS))
     ap.add_argument("--seed", type=int, default=0)
-    ap.add_argument("--variant", choices=("flarepp", "shared", "flare"), default="flarepp",
+    ap.add_argument("--variant", choices=("flarepp", "shared", "flare", "train"),
+                    default="flarepp",
                     help="flarepp: the routing chain (default); shared: the chain with Kt, Vt "
-                         "tied to K, V; flare: FLARE with fixed learned queries")
+                         "tied to K, V; flare: FLARE with fixed learned queries; train: the "
+                         "chain's training forward and backward")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--e2e-steps", type=int, default=5)
     ap.add_argument("--no-cpu-baseline", action="store_true")
