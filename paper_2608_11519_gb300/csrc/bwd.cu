@@ -1,4 +1,6 @@
-// Backward of the routing chain on CUDA cores (App. A.5), for bf16 or f32 inputs.
+// Backward of the routing chain (App. A.5): the CUDA-core passes (float32 inputs), the
+// kernels both paths share (c of call 3, the reduces of the route passes' partials) and
+// the launch sequence of both paths; the tensor-core passes are in tc_bwd.cu.
 //
 // Every SDPA of the chain is differentiated from its saved output O and log-normaliser L:
 //   P = 2^(x - L) with x = scale * log2(e) <a, b> (L kept in base 2 by the forward),
@@ -10,10 +12,12 @@
 //           added to the encoder's): c1 per route; dVt = P1^T dQ, dKt = s dS1^T Qs,
 //           dQs = s dS1 Kt, summed over the batch for the shared seeds.
 //
-// Two kernel shapes cover it. A route pass gives one thread per route and streams a chunk
-// of tokens, accumulating the latent-side sums (dZ, dQ, dQs) into per-chunk partials that a
-// reduce kernel adds in chunk order. A token pass gives one thread per token and streams
-// every route, producing that token's dK, dV (calls 2 and 3 together) or dKt, dVt (call 1).
+// Two kernel shapes cover it on CUDA cores. A route pass gives one thread per route and
+// streams a chunk of tokens, accumulating the latent-side sums (dZ, dQ, dQs) into per-chunk
+// partials that a reduce kernel adds in chunk order. A token pass gives one thread per
+// token and streams every route, producing that token's dK, dV (calls 2 and 3 together) or
+// dKt, dVt (call 1). The tensor-core path has the same structure (passes R3, T23, R2, T1,
+// R1) with bf16 copies of Q, Z, dZ and dQ as MMA operands.
 #include <cuda_bf16.h>
 #include <math.h>
 
@@ -57,6 +61,14 @@ __global__ void __launch_bounds__(256) delta_tokens_kernel(const T* __restrict__
 #pragma unroll
     for (int d = 0; d < D; ++d) acc = fmaf(ld_f32(dY + r * D + d), ld_f32(Y + r * D + d), acc);
     c3[r] = acc;
+}
+
+// bf16 copy of a float32 array (the tensor-core passes' Q and Z operands)
+__global__ void to_bf16_kernel(const float* __restrict__ src, __nv_bfloat16* __restrict__ dst,
+                               int64_t n) {
+    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n;
+         i += (int64_t)gridDim.x * blockDim.x)
+        dst[i] = __float2bfloat16_rn(src[i]);
 }
 
 // Route pass of call MODE (3, 2 or 1) over one chunk of tokens; thread = route m.
@@ -151,12 +163,14 @@ __global__ void __launch_bounds__(128) route_pass_kernel(
 //   MODE 3: dZ = sum pa, dQ = s sum pb, c2 = <dZ, Z>
 //   MODE 2: dQ += s sum pb, c1 = <dQ, Q>
 //   MODE 1: dseeds[h, m] = s sum_b sum_chunks pb (rows = H * M)
+// `op`, when not null, receives a bf16 copy of dZ (MODE 3) or dQ (MODE 2).
 template <int D, typename T, int MODE>
 __global__ void bwd_reduce_kernel(const float* __restrict__ pa, const float* __restrict__ pb,
                                   int64_t rows, int64_t B, int64_t H, int64_t M, int64_t nchunk,
                                   float scale, const float* __restrict__ O,
                                   float* __restrict__ dz, float* __restrict__ dq,
-                                  float* __restrict__ cout, T* __restrict__ dseeds) {
+                                  float* __restrict__ cout, T* __restrict__ dseeds,
+                                  __nv_bfloat16* __restrict__ op) {
     constexpr int PER = (D + 31) / 32;
     const int lane = threadIdx.x & 31;
     const int64_t row = (int64_t)blockIdx.x * (blockDim.x / 32) + threadIdx.x / 32;
@@ -203,10 +217,12 @@ __global__ void bwd_reduce_kernel(const float* __restrict__ pa, const float* __r
                 dz[row * D + d] = sa[i];
                 dq[row * D + d] = scale * sb[i];
                 dot = fmaf(sa[i], O[row * D + d], dot);
+                if (op) op[row * D + d] = __float2bfloat16_rn(sa[i]);
             } else {
                 const float v = dq[row * D + d] + scale * sb[i];
                 dq[row * D + d] = v;
                 dot = fmaf(v, O[row * D + d], dot);
+                if (op) op[row * D + d] = __float2bfloat16_rn(v);
             }
         }
     }
@@ -330,7 +346,7 @@ cudaError_t route_bwd_d(const Plan& p, const BwdPlan& bp, const T* seeds, const 
         bp.n_mtiles, sl2, pa, pb);
     bwd_reduce_kernel<D, T, 3><<<red_blocks, 256, 0, st>>>(pa, pb, lat_rows, p.B, p.H, p.M,
                                                            bp.nchunk, scale, Z32, dz, dq, c2,
-                                                           nullptr);
+                                                           nullptr, nullptr);
     // calls 3 and 2: dK and dV per token
     token_pass_kernel<D, T, float, 23><<<token_blocks, 128, 0, st>>>(
         K, V, dY, Q32, 0, dz, Z32, L2, c2, L3, c3, p.H, p.N, p.M, sl2, scale, dK, dV);
@@ -340,7 +356,7 @@ cudaError_t route_bwd_d(const Plan& p, const BwdPlan& bp, const T* seeds, const 
         bp.n_mtiles, sl2, nullptr, pb);
     bwd_reduce_kernel<D, T, 2><<<red_blocks, 256, 0, st>>>(nullptr, pb, lat_rows, p.B, p.H, p.M,
                                                            bp.nchunk, scale, Q32, nullptr, dq, c1,
-                                                           nullptr);
+                                                           nullptr, nullptr);
     // call 1: dKt, dVt per token, then the seeds' gradient
     token_pass_kernel<D, T, T, 1><<<token_blocks, 128, 0, st>>>(
         Kt, Vt, nullptr, seeds, 1, dq, nullptr, L1, c1, nullptr, nullptr, p.H, p.N, p.M, sl2,
@@ -351,7 +367,78 @@ cudaError_t route_bwd_d(const Plan& p, const BwdPlan& bp, const T* seeds, const 
     const int64_t seed_rows = p.H * p.M;
     bwd_reduce_kernel<D, T, 1><<<(unsigned)((seed_rows + 7) / 8), 256, 0, st>>>(
         nullptr, pb, seed_rows, p.B, p.H, p.M, bp.nchunk, scale, nullptr, nullptr, nullptr,
-        nullptr, dseeds);
+        nullptr, dseeds, nullptr);
+    return cudaGetLastError();
+}
+
+// The tensor-core path (bf16 inputs): c3, the bf16 operand copies of Q and Z, then
+// R3 -> reduce (dZ, the decoder's dQ, c2) -> T23 (dK, dV) and R2 -> reduce (dQ, c1) ->
+// T1 (dKt, dVt) and R1 -> reduce (dseeds).
+template <int D>
+cudaError_t route_bwd_tc_d(const Plan& p, const BwdPlan& bp, const void* seeds, const void* Kt,
+                           const void* Vt, const void* K, const void* V, float scale,
+                           const void* Y, const void* dY, const char* saved, void* dseeds,
+                           void* dKt, void* dVt, void* dK, void* dV, char* ws, cudaStream_t st) {
+    using T = __nv_bfloat16;
+    const SavedLayout sl = saved_layout(p);
+    const float* Q32 = (const float*)(saved + sl.off_q);
+    const float* Z32 = (const float*)(saved + sl.off_z);
+    const float* L1 = (const float*)(saved + sl.off_l1);
+    const float* L2 = (const float*)(saved + sl.off_l2);
+    const float* L3 = (const float*)(saved + sl.off_l3);
+    float* pa = (float*)(ws + bp.off_pa);
+    float* pb = (float*)(ws + bp.off_pb);
+    float* dz = (float*)(ws + bp.off_dz);
+    float* dq = (float*)(ws + bp.off_dq);
+    float* c1 = (float*)(ws + bp.off_d1);
+    float* c2 = (float*)(ws + bp.off_d2);
+    float* c3 = (float*)(ws + bp.off_d3);
+    T* qb = (T*)(ws + bp.off_qb);
+    T* zb = (T*)(ws + bp.off_zb);
+    T* dzb = (T*)(ws + bp.off_dzb);
+    T* dqb = (T*)(ws + bp.off_dqb);
+    int* status = (int*)(ws + bp.off_status);
+    const int64_t tok_rows = p.BH * p.N;
+    const int64_t lat_rows = p.BH * p.M;
+    const int64_t lat = lat_rows * p.D;
+    const unsigned red_blocks = (unsigned)((lat_rows + 7) / 8);
+    const unsigned cvt_blocks = (unsigned)min((int64_t)1024, (lat + 255) / 256);
+    cudaError_t e;
+
+    delta_tokens_kernel<D, T><<<(unsigned)((tok_rows + 255) / 256), 256, 0, st>>>(
+        (const T*)dY, (const T*)Y, tok_rows, c3);
+    to_bf16_kernel<<<cvt_blocks, 256, 0, st>>>(Q32, qb, lat);
+    to_bf16_kernel<<<cvt_blocks, 256, 0, st>>>(Z32, zb, lat);
+    TcBwdOperands o{};
+    // R3: route rows; S = Q K^T, dP = Z dY^T; column statistics L3, c3 -> dQ3, dZ partials
+    o = TcBwdOperands{{qb, zb, zb}, {K, dY, dY}, nullptr, nullptr, L3, c3, pa, pb, nullptr,
+                      nullptr};
+    if ((e = tc_bwd_pass(p, bp, 0, o, scale, status, st)) != cudaSuccess) return e;
+    bwd_reduce_kernel<D, T, 3><<<red_blocks, 256, 0, st>>>(pa, pb, lat_rows, p.B, p.H, p.M,
+                                                           bp.nchunk, scale, Z32, dz, dq, c2,
+                                                           nullptr, dzb);
+    // T23: token rows; S = K Q^T, dP2 = V dZ^T, dP3 = dY Z^T -> dK, dV
+    o = TcBwdOperands{{K, V, dY}, {qb, dzb, zb}, L3, c3, L2, c2, nullptr, nullptr, dK, dV};
+    if ((e = tc_bwd_pass(p, bp, 3, o, scale, status, st)) != cudaSuccess) return e;
+    // R2: route rows; S = Q K^T, dP = dZ V^T; row statistics L2, c2 -> dQ2 partials
+    o = TcBwdOperands{{qb, dzb, dzb}, {K, V, V}, L2, c2, nullptr, nullptr, nullptr, pb, nullptr,
+                      nullptr};
+    if ((e = tc_bwd_pass(p, bp, 1, o, scale, status, st)) != cudaSuccess) return e;
+    bwd_reduce_kernel<D, T, 2><<<red_blocks, 256, 0, st>>>(nullptr, pb, lat_rows, p.B, p.H, p.M,
+                                                           bp.nchunk, scale, Q32, nullptr, dq, c1,
+                                                           nullptr, dqb);
+    // T1: token rows; S = Kt Qs^T, dP = Vt dQ^T; column statistics L1, c1 -> dKt, dVt
+    o = TcBwdOperands{{Kt, Vt, Vt}, {seeds, dqb, dqb}, nullptr, nullptr, L1, c1, nullptr,
+                      nullptr, dKt, dVt};
+    if ((e = tc_bwd_pass(p, bp, 4, o, scale, status, st)) != cudaSuccess) return e;
+    // R1: route rows; S = Qs Kt^T, dP = dQ Vt^T; row statistics L1, c1 -> dQs partials
+    o = TcBwdOperands{{seeds, dqb, dqb}, {Kt, Vt, Vt}, L1, c1, nullptr, nullptr, nullptr, pb,
+                      nullptr, nullptr};
+    if ((e = tc_bwd_pass(p, bp, 2, o, scale, status, st)) != cudaSuccess) return e;
+    const int64_t seed_rows = p.H * p.M;
+    bwd_reduce_kernel<D, T, 1><<<(unsigned)((seed_rows + 7) / 8), 256, 0, st>>>(
+        nullptr, pb, seed_rows, p.B, p.H, p.M, bp.nchunk, scale, nullptr, nullptr, nullptr,
+        nullptr, (T*)dseeds, nullptr);
     return cudaGetLastError();
 }
 
@@ -375,15 +462,24 @@ cudaError_t route_bwd_t(const Plan& p, const BwdPlan& bp, const void* seeds, con
 
 }  // namespace
 
-cudaError_t simt_route_bwd(const Plan& p, const BwdPlan& bp, const void* seeds, const void* Kt,
-                           const void* Vt, const void* K, const void* V, float scale,
-                           const void* Y, const void* dY, const char* saved, void* dseeds,
-                           void* dKt, void* dVt, void* dK, void* dV, char* ws, cudaStream_t st) {
-    if (p.dtype == FLAREPP_F32)
-        return route_bwd_t<float>(p, bp, seeds, Kt, Vt, K, V, scale, Y, dY, saved, dseeds, dKt,
-                                  dVt, dK, dV, ws, st);
-    return route_bwd_t<__nv_bfloat16>(p, bp, seeds, Kt, Vt, K, V, scale, Y, dY, saved, dseeds,
-                                      dKt, dVt, dK, dV, ws, st);
+cudaError_t route_bwd(const Plan& p, const BwdPlan& bp, const void* seeds, const void* Kt,
+                      const void* Vt, const void* K, const void* V, float scale, const void* Y,
+                      const void* dY, const char* saved, void* dseeds, void* dKt, void* dVt,
+                      void* dK, void* dV, char* ws, cudaStream_t st) {
+    if (bp.path == kPathTc) {
+#define FLAREPP_TCBWD(DD)                                                                     \
+    return route_bwd_tc_d<DD>(p, bp, seeds, Kt, Vt, K, V, scale, Y, dY, saved, dseeds, dKt, \
+                              dVt, dK, dV, ws, st);
+        switch (p.D) {
+            case 16: FLAREPP_TCBWD(16)
+            case 32: FLAREPP_TCBWD(32)
+            case 64: FLAREPP_TCBWD(64)
+            default: return cudaErrorInvalidValue;
+        }
+#undef FLAREPP_TCBWD
+    }
+    return route_bwd_t<float>(p, bp, seeds, Kt, Vt, K, V, scale, Y, dY, saved, dseeds, dKt, dVt,
+                              dK, dV, ws, st);
 }
 
 }  // namespace flarepp

@@ -448,8 +448,8 @@ flarepp_status route_bwd_impl(const flarepp_shape* shape, const void* seeds, con
     char* ws = (char*)workspace;
     if (cudaMemsetAsync(ws + bp.off_status, 0, sizeof(int32_t), st) != cudaSuccess)
         return FLAREPP_ERR_CUDA;
-    const cudaError_t e = simt_route_bwd(p, bp, seeds, Kt, Vt, K, V, scale, Y, dY,
-                                         (const char*)saved, dseeds, dKt, dVt, dK, dV, ws, st);
+    const cudaError_t e = route_bwd(p, bp, seeds, Kt, Vt, K, V, scale, Y, dY,
+                                    (const char*)saved, dseeds, dKt, dVt, dK, dV, ws, st);
     return e == cudaSuccess ? FLAREPP_OK : FLAREPP_ERR_CUDA;
 }
 

@@ -51,16 +51,21 @@ struct SavedLayout {
 };
 SavedLayout saved_layout(const Plan& p);
 
-// The backward's plan: the split-N route passes (one thread per route, chunks of tokens)
-// and its workspace.
+// The backward's plan: the split-N route passes (chunks of tokens) and its workspace. On
+// the CUDA-core path a route pass gives one thread per route (m_tile routes per CTA); on
+// the tensor-core path a work unit is a group of 256 routes and a chunk of tokens, and
+// chunk_len is a multiple of the 64- (D = 64: 32-) token item.
 struct BwdPlan {
-    int64_t m_tile, n_mtiles;   // routes per CTA and route tiles per head
+    int path;                   // kPathSimt or kPathTc
+    int64_t m_tile, n_mtiles;   // CUDA-core route passes: routes per CTA, route tiles per head
     int64_t chunk_len, nchunk;  // tokens per chunk and chunks per head
     size_t off_status;          // int32 device status word
     size_t off_pa, off_pb;      // per-chunk partial sums [BH][nchunk][M][D] f32
     size_t off_dz, off_dq;      // dZ, dQ [BH][M][D] f32
     size_t off_d1, off_d2;      // c = <dO, O> of calls 1 and 2 [BH][M] f32
-    size_t off_d3;              // c of call 3 [BH][N] f32
+    size_t off_d3;              // c of call 3 [BH][N] f32 (+ 256 bytes of slack)
+    size_t off_qb, off_zb;      // tensor-core path: bf16 MMA operands Q, Z [BH][M][D]
+    size_t off_dzb, off_dqb;    // ... and dZ, dQ
     size_t total;
 };
 BwdPlan make_bwd_plan(const Plan& p);
@@ -75,13 +80,13 @@ cudaError_t simt_encode_f32(const Plan& p, int call, const void* k, const void* 
 cudaError_t simt_decode_f32(const Plan& p, const void* K, float scale, void* Y, char* ws,
                             cudaStream_t st, float* lse = nullptr);
 
-// ---- backward (bwd_simt.cu): the passes of App. A.5 on CUDA cores, bf16 or f32 inputs
-// (dtype from the plan). `saved` is the training forward's state, `ws` the backward
-// workspace; outputs in the input dtype.
-cudaError_t simt_route_bwd(const Plan& p, const BwdPlan& bp, const void* seeds, const void* Kt,
-                           const void* Vt, const void* K, const void* V, float scale,
-                           const void* Y, const void* dY, const char* saved, void* dseeds,
-                           void* dKt, void* dVt, void* dK, void* dV, char* ws, cudaStream_t st);
+// ---- backward (bwd.cu): the passes of App. A.5. f32 inputs run on CUDA cores, bf16 inputs
+// on the tensor-core passes of tc_bwd.cu. `saved` is the training forward's state, `ws`
+// the backward workspace; outputs in the input dtype.
+cudaError_t route_bwd(const Plan& p, const BwdPlan& bp, const void* seeds, const void* Kt,
+                      const void* Vt, const void* K, const void* V, float scale, const void* Y,
+                      const void* dY, const char* saved, void* dseeds, void* dKt, void* dVt,
+                      void* dK, void* dV, char* ws, cudaStream_t st);
 
 // ---- split-N combine (combine.cu)
 // Stable log-sum-exp merge of the chunk partials into Q32 (call 1) or Z32 (call 2), plus
@@ -92,6 +97,28 @@ cudaError_t combine(const Plan& p, int call, char* ws, bool negate, cudaStream_t
                     float* lse = nullptr);
 // dst = -src elementwise (bf16; exact)
 cudaError_t negate_bf16(const void* src, void* dst, int64_t n, cudaStream_t st);
+
+// ---- tensor-core backward passes (tc_bwd.cu), bf16 inputs
+// Operands of one pass: its A tiles and item tiles (bf16 [z][rows][D]; an unused third
+// entry may repeat a used one), the row and column statistics, and its outputs (partial
+// sums of the route-row passes, bf16 gradients of the token-row passes).
+struct TcBwdOperands {
+    const void* a[3];
+    const void* i[3];
+    const float* Lrow;
+    const float* crow;
+    const float* Lcol;
+    const float* ccol;
+    float* pa;
+    float* pb;
+    void* out0;
+    void* out1;
+};
+// pass: 0 = R3, 1 = R2, 2 = R1 (route rows), 3 = T23, 4 = T1 (token rows)
+cudaError_t tc_bwd_pass(const Plan& p, const BwdPlan& bp, int pass, const TcBwdOperands& o,
+                        float scale, int* status, cudaStream_t st);
+// Tokens (route-row passes) or routes (token-row passes) per streamed item.
+int64_t tc_bwd_item(int64_t D);
 
 // ---- tensor-core kernels (tc_kernels.cu), bf16 inputs
 // Encode call 1 (A = seeds) or call 2 (A = Q operand) into the chunk partials.

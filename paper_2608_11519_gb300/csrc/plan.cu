@@ -134,13 +134,23 @@ SavedLayout saved_layout(const Plan& p) {
 
 BwdPlan make_bwd_plan(const Plan& p) {
     BwdPlan b{};
+    b.path = p.path;
     if (p.BH == 0 || p.N == 0 || p.M == 0) return b;
-    // one thread per route, up to 128 routes per CTA; chunks sized for about four waves
     b.m_tile = p.M >= 128 ? 128 : cdiv(p.M, 32) * 32;
     b.n_mtiles = cdiv(p.M, b.m_tile);
-    int64_t want = cdiv(4 * kNumSMs, p.BH * b.n_mtiles);
-    if (want < 1) want = 1;
-    b.chunk_len = cdiv(cdiv(p.N, want), 32) * 32;
+    if (p.path == kPathTc) {
+        // work units (b*h, 256-route group, chunk): about two waves of persistent CTAs
+        const int64_t item = p.D == 64 ? 32 : 64;
+        const int64_t groups = cdiv(p.M, 256);
+        int64_t want = cdiv(2 * kNumSMs, p.BH * groups);
+        if (want < 1) want = 1;
+        b.chunk_len = cdiv(cdiv(p.N, want), item) * item;
+    } else {
+        // one thread per route, up to 128 routes per CTA; chunks for about four waves
+        int64_t want = cdiv(4 * kNumSMs, p.BH * b.n_mtiles);
+        if (want < 1) want = 1;
+        b.chunk_len = cdiv(cdiv(p.N, want), 32) * 32;
+    }
     b.nchunk = cdiv(p.N, b.chunk_len);
     const size_t part = (size_t)p.BH * (size_t)b.nchunk * (size_t)p.M * (size_t)p.D * 4;
     const size_t qz = (size_t)p.BH * (size_t)p.M * (size_t)p.D * 4;
@@ -162,7 +172,18 @@ BwdPlan make_bwd_plan(const Plan& p) {
     b.off_d2 = off;
     off = align_up(off + lm, kWsAlign);
     b.off_d3 = off;
-    off = align_up(off + ln, kWsAlign);
+    off = align_up(off + ln + 256, kWsAlign);
+    if (p.path == kPathTc) {
+        const size_t op = (size_t)p.BH * (size_t)p.M * (size_t)p.D * 2;
+        b.off_qb = off;
+        off = align_up(off + op, kWsAlign);
+        b.off_zb = off;
+        off = align_up(off + op, kWsAlign);
+        b.off_dzb = off;
+        off = align_up(off + op, kWsAlign);
+        b.off_dqb = off;
+        off = align_up(off + op, kWsAlign);
+    }
     b.total = off;
     return b;
 }

@@ -1,0 +1,711 @@
+// Tensor-core (tcgen05 / TMEM / TMA) backward of the routing chain, bf16 inputs (App. A.5).
+//
+// Every SDPA(A, B, C) of the chain is differentiated from its saved log-normaliser L
+// (base 2) and c = <dO, O>:  P = 2^(x - L) with x = scale log2(e) <a, b>,
+// dS = P o (dP - c) with dP = <dO, C>, and the products dA = s dS B, dB = s dS^T A,
+// dC = P^T dO. Five passes cover the three calls. In every pass a score tile of 128 TMEM
+// lanes x kItem columns is produced by the tensor cores, turned into bf16 P and dS in place
+// by a softmax warpgroup, and consumed as the TMEM A operand of one or two accumulating
+// products whose B operand is the same streamed item:
+//
+//   route-row passes (TMEM lanes are routes, items are tokens; per-chunk partial sums):
+//     R3  call 3, column statistics L3, c3 of the tokens:
+//         S = Q K^T, dP = Z dY^T;  acc0 += dS K (-> dQ / s),  acc1 += P dY (-> dZ)
+//     R2  call 2, row statistics L2, c2:   S = Q K^T,  dP = dZ V^T;   acc0 += dS K
+//     R1  call 1, row statistics L1, c1:   S = Qs Kt^T, dP = dQ Vt^T; acc0 += dS Kt
+//   token-row passes (TMEM lanes are tokens, items are routes; final per-token outputs):
+//     T23 calls 3 and 2, token statistics L3, c3 and route statistics L2, c2:
+//         S = K Q^T, dP2 = V dZ^T, dP3 = dY Z^T,
+//         dS = P2 o (dP2 - c2) + P3 o (dP3 - c3) with P2 = 2^(x - L2), P3 = 2^(x - L3);
+//         acc0 += dS Q (-> dK / s),  acc1 += P2 dZ (-> dV)
+//     T1  call 1, route statistics L1, c1:  S = Kt Qs^T, dP = Vt dQ^T;
+//         acc0 += dS Qs (-> dKt / s),  acc1 += P dQ (-> dVt)
+// Score products take both operands from shared memory (TMA, swizzled, K-major); the
+// accumulating products read P or dS from TMEM and the item, MN-major, from shared memory.
+//
+// Roles (12 warps): warp 0 the TMA producer (it also stages each item's column statistics
+// in shared memory), warp 1 the MMA issuer, warps 4..11 two softmax warpgroups, one per
+// TMEM stream of 128 rows. A work unit is (b*h, group of 2 x 128 rows, chunk of items).
+// Every wait is bounded (2 s of %globaltimer): on expiry the kernel records
+// FLAREPP_ERR_TIMEOUT in the status word, every role leaves its loops, the producer waits
+// for its copies in flight, the MMA issuer for its products, and TMEM is freed.
+#include <cuda.h>
+#include <cudaTypedefs.h>
+#include <cuda_bf16.h>
+#include <math.h>
+#include <mutex>
+
+#include "flarepp_internal.h"
+#include "tc_ptx.cuh"
+
+namespace flarepp {
+namespace {
+
+using namespace tc;
+
+constexpr int kWarps = 12;
+constexpr int kThreads = kWarps * 32;
+constexpr int kFirstSoftmaxWarp = 4;
+constexpr int NS = 2;           // TMEM streams (softmax warpgroups)
+constexpr int kRows = 128;      // TMEM lanes per stream, MMA M
+constexpr uint64_t kWaitLimitNs = 2000000000ull;
+constexpr uint32_t kTmemCols = 512;
+
+enum Pass : int { kR3 = 0, kR2 = 1, kR1 = 2, kT23 = 3, kT1 = 4 };
+
+template <int D, int PASS>
+struct BCfg {
+    static constexpr bool kRouteRows = PASS <= kR1;
+    static constexpr int kNA = PASS == kT23 ? 3 : 2;  // score products (A tiles, item tiles)
+    static constexpr int kNAcc = (PASS == kR2 || PASS == kR1) ? 1 : 2;
+    static constexpr bool kColStats = PASS == kR3 || PASS == kT23 || PASS == kT1;
+    static constexpr bool kRowStats = PASS == kR2 || PASS == kR1 || PASS == kT23;
+    static constexpr int kItem = D == 64 ? 32 : 64;
+    static constexpr int kABuf = D == 64 ? 1 : 2;  // shared-memory copies of a unit's A tiles
+    static constexpr int kStages = 6;
+    static constexpr int kATile = kRows * D * 2;
+    static constexpr int kABytes = NS * kNA * kATile;  // one unit's A tiles
+    static constexpr int kItemTile = kItem * D * 2;
+    static constexpr int kStage = kNA * kItemTile;
+    static constexpr uint32_t kSwz = D == 16 ? kSw32 : (D == 32 ? kSw64 : kSw128);
+    static constexpr uint32_t kSBO = 8 * D * 2;
+    // TMEM per stream: kNA score tiles of kItem columns, then kNAcc accumulators of D
+    static constexpr uint32_t kColStream = kNA * kItem + kNAcc * D;
+    static_assert(NS * kColStream <= kTmemCols, "TMEM budget");
+    // barriers: full[S], empty[S], afull[kABuf], afree[kABuf], sready[NS], pready[NS],
+    //           accdone[NS], accfree[NS], fin
+    static constexpr int kNumBars = 2 * kStages + 2 * kABuf + 4 * NS + 1;
+    static constexpr int kStatBytes = kStages * 2 * kItem * 4;
+    static constexpr int kData = kABuf * kABytes + kStages * kStage;
+    static constexpr int kNeed = 1024 + kData + kStatBytes + kNumBars * 8 + 16;
+    // at least 120 KB so that one CTA owns an SM and its 512 TMEM columns
+    static constexpr int kSmem = kNeed > 122880 ? kNeed : 122880;
+    static_assert(kSmem <= 232448, "shared memory budget");
+    static constexpr uint32_t kIdescS = idesc_bf16_f32(128, kItem, false, false);
+    static constexpr uint32_t kIdescAcc = idesc_bf16_f32(128, D, false, true);
+};
+
+struct BwdParams {
+    int64_t BH, H, N, M;
+    float c;      // scale * log2(e), signed
+    float scale;  // s
+    int a0_per_head;     // R1: the first A operand (seeds) is indexed by head
+    int i0_per_head;     // T1: the first item operand (seeds) is indexed by head
+    int64_t chunk_len, nchunk, n_groups;  // route-row passes
+    int64_t n_tok_groups;                 // token-row passes
+    int64_t n_units;
+    const float* Lrow;  // row statistics [BH][rows]: L (base 2) and c
+    const float* crow;
+    const float* Lcol;  // column statistics [BH][items' rows]
+    const float* ccol;
+    float* pa;  // route-row passes: partial sums [BH][nchunk][M][D] (acc1, acc0)
+    float* pb;
+    __nv_bfloat16* out0;  // token-row passes: s * acc0 and acc1, [BH][N][D]
+    __nv_bfloat16* out1;
+    int* status;
+};
+
+struct BUnit {
+    int64_t bh, g, chunk;
+    int64_t row0;          // first TMEM row (route or token) of stream 0
+    int64_t rows;          // route or token count of the rows' dimension (M or N)
+    int64_t item0, item_end;
+    int n_act;             // streams with at least one valid row
+    int n_items;
+};
+
+template <int D, int PASS>
+__device__ __forceinline__ BUnit bwd_unit(const BwdParams& p, int64_t u) {
+    using C = BCfg<D, PASS>;
+    BUnit U;
+    if (C::kRouteRows) {
+        U.chunk = u % p.nchunk;
+        const int64_t t = u / p.nchunk;
+        U.g = t % p.n_groups;
+        U.bh = t / p.n_groups;
+        U.rows = p.M;
+        U.item0 = U.chunk * p.chunk_len;
+        U.item_end = min(p.N, U.item0 + p.chunk_len);
+    } else {
+        U.g = u % p.n_tok_groups;
+        U.bh = u / p.n_tok_groups;
+        U.chunk = 0;
+        U.rows = p.N;
+        U.item0 = 0;
+        U.item_end = p.M;
+    }
+    U.row0 = U.g * (NS * kRows);
+    const int64_t left = U.rows - U.row0;
+    U.n_act = left >= NS * kRows ? NS : (int)((left + kRows - 1) / kRows);
+    U.n_items = (int)((U.item_end - U.item0 + C::kItem - 1) / C::kItem);
+    return U;
+}
+
+__device__ __forceinline__ float ex2(float x) {
+    float y;
+    asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+    return y;
+}
+
+__device__ __forceinline__ uint32_t pack_bf16(float lo, float hi) {
+    __nv_bfloat162 v = __floats2bfloat162_rn(lo, hi);
+    return *reinterpret_cast<uint32_t*>(&v);
+}
+
+// Bounded wait on an mbarrier phase. Returns false when the kernel is aborting.
+__device__ __forceinline__ bool wait_bar(uint32_t bar, uint32_t parity, volatile int* abort_flag,
+                                         int* status) {
+    if (mbar_try_wait(bar, parity)) return true;
+    const uint64_t t0 = globaltimer_ns();
+    for (uint32_t i = 1;; ++i) {
+        if (mbar_try_wait(bar, parity)) return true;
+        if ((i & 63u) == 0) {
+            if (*abort_flag) return false;
+            if (globaltimer_ns() - t0 > kWaitLimitNs) {
+                *abort_flag = 1;
+                atomicExch(status, (int)FLAREPP_ERR_TIMEOUT);
+                return false;
+            }
+        }
+    }
+}
+__device__ __forceinline__ bool warp_wait(uint32_t bar, uint32_t parity, volatile int* abort_flag,
+                                          int* status) {
+    const bool got = wait_bar(bar, parity, abort_flag, status);
+    return __all_sync(0xffffffffu, got);
+}
+
+// One 32-column slice of an item for this thread's row: reads the score tiles, writes bf16
+// dS over score tile 0 and (when a second accumulator reads it) bf16 P over score tile 1.
+// Columns at or beyond nv are outside the item: P = dS = 0.
+template <int D, int PASS>
+__device__ __forceinline__ void bwd_slice(uint32_t t0, int h, int nv, float c, float Lr, float cr,
+                                          const float* Lc, const float* cc) {
+    using C = BCfg<D, PASS>;
+    uint32_t sr[32], d1[32], d2[PASS == kT23 ? 32 : 1];
+    tmem_ld32(t0 + 32 * h, sr);
+    tmem_ld32(t0 + C::kItem + 32 * h, d1);
+    if (PASS == kT23) tmem_ld32(t0 + 2 * C::kItem + 32 * h, d2);
+    tmem_wait_ld32(sr);
+    tmem_wait_ld32(d1);
+    if (PASS == kT23) tmem_wait_ld32(d2);
+    uint32_t ds[16], pp[16];
+#pragma unroll
+    for (int k = 0; k < 16; ++k) {
+        float dsv[2], pv[2];
+#pragma unroll
+        for (int e = 0; e < 2; ++e) {
+            const int col = 32 * h + 2 * k + e;
+            const float x = __uint_as_float(sr[2 * k + e]);
+            const float dp = __uint_as_float(d1[2 * k + e]);
+            float p, d;
+            if (PASS == kR2 || PASS == kR1) {
+                p = ex2(fmaf(c, x, -Lr));
+                d = p * (dp - cr);
+            } else if (PASS == kT23) {
+                p = ex2(fmaf(c, x, -Lc[col]));
+                const float p3 = ex2(fmaf(c, x, -Lr));
+                d = fmaf(p3, __uint_as_float(d2[2 * k + e]) - cr, p * (dp - cc[col]));
+            } else {  // R3, T1: column statistics only
+                p = ex2(fmaf(c, x, -Lc[col]));
+                d = p * (dp - cc[col]);
+            }
+            const bool in = col < nv;
+            dsv[e] = in ? d : 0.f;
+            pv[e] = in ? p : 0.f;
+        }
+        ds[k] = pack_bf16(dsv[0], dsv[1]);
+        pp[k] = pack_bf16(pv[0], pv[1]);
+    }
+    tmem_st16(t0 + 16 * h, ds);
+    if (C::kNAcc == 2) tmem_st16(t0 + C::kItem + 16 * h, pp);
+}
+
+// ------------------------------------------------------------------ the kernel
+
+template <int D, int PASS>
+__global__ void __launch_bounds__(kThreads, 1)
+    tc_bwd_kernel(const __grid_constant__ CUtensorMap tmA0, const __grid_constant__ CUtensorMap tmA1,
+                  const __grid_constant__ CUtensorMap tmA2, const __grid_constant__ CUtensorMap tmI0,
+                  const __grid_constant__ CUtensorMap tmI1, const __grid_constant__ CUtensorMap tmI2,
+                  const BwdParams prm) {
+    using C = BCfg<D, PASS>;
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
+                                               ~static_cast<uintptr_t>(1023));
+    uint8_t* abuf = smem;                         // kABuf x [NS][kNA] A tiles, swizzled
+    uint8_t* ring = smem + C::kABuf * C::kABytes;  // kStages x kNA item tiles, swizzled
+    float* stats = reinterpret_cast<float*>(ring + C::kStages * C::kStage);  // [S][2][kItem]
+    uint64_t* bars = reinterpret_cast<uint64_t*>(stats + C::kStages * 2 * C::kItem);
+    uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + C::kNumBars);
+    volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+
+    const uint32_t full0 = smem_u32(bars);
+    const uint32_t empty0 = full0 + 8u * C::kStages;
+    const uint32_t afull0 = empty0 + 8u * C::kStages;
+    const uint32_t afree0 = afull0 + 8u * C::kABuf;
+    const uint32_t sready0 = afree0 + 8u * C::kABuf;
+    const uint32_t pready0 = sready0 + 8u * NS;
+    const uint32_t accdone0 = pready0 + 8u * NS;
+    const uint32_t accfree0 = accdone0 + 8u * NS;
+    const uint32_t fin = accfree0 + 8u * NS;
+
+    const int warp = threadIdx.x >> 5;
+    const int lane = threadIdx.x & 31;
+
+    if (threadIdx.x == 0) {
+        for (int st = 0; st < C::kStages; ++st) {
+            mbar_init(full0 + 8u * st, C::kColStats ? 33 : 1);
+            mbar_init(empty0 + 8u * st, 1);
+        }
+        for (int b = 0; b < C::kABuf; ++b) {
+            mbar_init(afull0 + 8u * b, 1);
+            mbar_init(afree0 + 8u * b, 1);
+        }
+        for (int s = 0; s < NS; ++s) {
+            mbar_init(sready0 + 8u * s, 1);
+            mbar_init(pready0 + 8u * s, kRows);
+            mbar_init(accdone0 + 8u * s, 1);
+            mbar_init(accfree0 + 8u * s, kRows);
+        }
+        mbar_init(fin, 1);
+        *abort_flag = 0;
+        fence_mbar_init();
+        prefetch_tmap(&tmA0);
+        prefetch_tmap(&tmA1);
+        prefetch_tmap(&tmI0);
+        prefetch_tmap(&tmI1);
+        if (C::kNA == 3) {
+            prefetch_tmap(&tmA2);
+            prefetch_tmap(&tmI2);
+        }
+    }
+    if (warp == 1) {
+        tmem_alloc(smem_u32(tmem_slot), kTmemCols);
+        tmem_relinquish();
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = *tmem_slot;
+
+    if (warp == 0) {
+        // ------------------------------------------------------------ TMA producer
+        uint32_t it = 0, ua = 0, a_issued = 0;
+        bool ok = true;
+        for (int64_t u = blockIdx.x; u < prm.n_units && ok; u += gridDim.x, ++ua) {
+            const BUnit U = bwd_unit<D, PASS>(prm, u);
+            const int ab = ua % C::kABuf;
+            if (ua >= (uint32_t)C::kABuf &&
+                !warp_wait(afree0 + 8u * ab, ((ua / C::kABuf) - 1) & 1, abort_flag, prm.status)) {
+                ok = false;
+                break;
+            }
+            if (elect_one()) {
+                mbar_expect_tx(afull0 + 8u * ab, U.n_act * C::kNA * C::kATile);
+                const int za0 = (int)(prm.a0_per_head ? U.bh % prm.H : U.bh);
+                for (int s = 0; s < U.n_act; ++s) {
+                    const int row = (int)(U.row0 + s * kRows);
+                    uint8_t* dst = abuf + ab * C::kABytes + s * C::kNA * C::kATile;
+                    tma_load_3d(smem_u32(dst), &tmA0, 0, row, za0, afull0 + 8u * ab);
+                    tma_load_3d(smem_u32(dst + C::kATile), &tmA1, 0, row, (int)U.bh,
+                                afull0 + 8u * ab);
+                    if (C::kNA == 3)
+                        tma_load_3d(smem_u32(dst + 2 * C::kATile), &tmA2, 0, row, (int)U.bh,
+                                    afull0 + 8u * ab);
+                }
+            }
+            __syncwarp();
+            ++a_issued;
+            const int zi0 = (int)(prm.i0_per_head ? U.bh % prm.H : U.bh);
+            for (int i = 0; i < U.n_items; ++i, ++it) {
+                const int st = it % C::kStages;
+                if (it >= (uint32_t)C::kStages &&
+                    !warp_wait(empty0 + 8u * st, ((it / C::kStages) - 1) & 1, abort_flag,
+                               prm.status)) {
+                    ok = false;
+                    break;
+                }
+                const int64_t row = U.item0 + (int64_t)i * C::kItem;
+                if (elect_one()) {
+                    mbar_expect_tx(full0 + 8u * st, C::kStage);
+                    const uint32_t dst = smem_u32(ring + st * C::kStage);
+                    tma_load_3d(dst, &tmI0, 0, (int)row, zi0, full0 + 8u * st);
+                    tma_load_3d(dst + C::kItemTile, &tmI1, 0, (int)row, (int)U.bh,
+                                full0 + 8u * st);
+                    if (C::kNA == 3)
+                        tma_load_3d(dst + 2 * C::kItemTile, &tmI2, 0, (int)row, (int)U.bh,
+                                    full0 + 8u * st);
+                }
+                __syncwarp();
+                if (C::kColStats) {
+                    float* sl = stats + st * 2 * C::kItem;
+                    const int64_t nvalid = U.item_end - row;
+                    for (int k = lane; k < C::kItem; k += 32) {
+                        const bool in = k < nvalid;
+                        const int64_t idx = U.bh * (C::kRouteRows ? prm.N : prm.M) + row + k;
+                        sl[k] = in ? prm.Lcol[idx] : 0.f;
+                        sl[C::kItem + k] = in ? prm.ccol[idx] : 0.f;
+                    }
+                    mbar_arrive(full0 + 8u * st);
+                }
+            }
+        }
+        // after an abort: wait (bounded) until the newest copy of every buffer has landed
+        if (!ok) {
+            const uint64_t t0 = globaltimer_ns();
+            for (int st = 0; st < C::kStages && (uint32_t)st < it; ++st) {
+                const uint32_t x = it - 1 - ((it - 1 - st) % C::kStages);
+                while (!mbar_try_wait(full0 + 8u * st, (x / C::kStages) & 1) &&
+                       globaltimer_ns() - t0 < kWaitLimitNs) {
+                }
+            }
+            for (int b = 0; b < C::kABuf && (uint32_t)b < a_issued; ++b) {
+                const uint32_t x = a_issued - 1 - ((a_issued - 1 - b) % C::kABuf);
+                while (!mbar_try_wait(afull0 + 8u * b, (x / C::kABuf) & 1) &&
+                       globaltimer_ns() - t0 < kWaitLimitNs) {
+                }
+            }
+        }
+    } else if (warp == 1) {
+        // ------------------------------------------------------------ MMA issuer
+        uint32_t it = 0, ua = 0;
+        uint32_t pj[NS] = {0, 0};   // p_ready phases consumed per stream
+        uint32_t nu[NS] = {0, 0};   // units completed per stream (acc_free phases)
+        bool ok = true;
+        auto wait = [&](uint32_t bar, uint32_t parity) {
+            return warp_wait(bar, parity, abort_flag, prm.status);
+        };
+        // the accumulating products of item `stg` for stream s (P / dS of that item in TMEM)
+        auto issue_acc = [&](int s, int stg, bool accumulate) {
+            const uint32_t t0 = tmem + s * C::kColStream;
+            const uint32_t acc = t0 + C::kNA * C::kItem;
+            const uint32_t ib = smem_u32(ring + stg * C::kStage);
+#pragma unroll
+            for (int k = 0; k < C::kItem / 16; ++k) {
+                const uint64_t bd = smem_desc(ib + k * 16 * D * 2, C::kItemTile, C::kSBO, C::kSwz);
+                if (elect_one())
+                    mma_ts(acc, t0 + 8 * k, bd, C::kIdescAcc, (accumulate || k > 0) ? 1u : 0u);
+                __syncwarp();
+            }
+            if (C::kNAcc == 2) {
+#pragma unroll
+                for (int k = 0; k < C::kItem / 16; ++k) {
+                    const uint64_t bd = smem_desc(ib + C::kItemTile + k * 16 * D * 2, C::kItemTile,
+                                                  C::kSBO, C::kSwz);
+                    if (elect_one())
+                        mma_ts(acc + D, t0 + C::kItem + 8 * k, bd, C::kIdescAcc,
+                               (accumulate || k > 0) ? 1u : 0u);
+                    __syncwarp();
+                }
+            }
+        };
+        for (int64_t u = blockIdx.x; u < prm.n_units && ok; u += gridDim.x, ++ua) {
+            const BUnit U = bwd_unit<D, PASS>(prm, u);
+            const int ab = ua % C::kABuf;
+            if (!wait(afull0 + 8u * ab, (ua / C::kABuf) & 1)) {
+                ok = false;
+                break;
+            }
+            tc_fence_after();
+            int prev_st = 0;
+            for (int i = 0; i <= U.n_items && ok; ++i) {
+                const int st = it % C::kStages;
+                if (i < U.n_items) {
+                    if (!wait(full0 + 8u * st, (it / C::kStages) & 1)) {
+                        ok = false;
+                        break;
+                    }
+                    tc_fence_after();
+                }
+                for (int s = 0; s < U.n_act; ++s) {
+                    if (i > 0) {
+                        // dS / P of item i - 1 written: its accumulating products
+                        if (!wait(pready0 + 8u * s, pj[s] & 1)) {
+                            ok = false;
+                            break;
+                        }
+                        ++pj[s];
+                        if (i == 1 && nu[s] > 0 && !wait(accfree0 + 8u * s, (nu[s] - 1) & 1)) {
+                            ok = false;
+                            break;
+                        }
+                        tc_fence_after();
+                        issue_acc(s, prev_st, i > 1);
+                    }
+                    if (i < U.n_items) {
+                        const uint32_t t0 = tmem + s * C::kColStream;
+                        const uint32_t a_base =
+                            smem_u32(abuf + ab * C::kABytes + s * C::kNA * C::kATile);
+                        const uint32_t i_base = smem_u32(ring + st * C::kStage);
+#pragma unroll
+                        for (int t = 0; t < C::kNA; ++t) {
+#pragma unroll
+                            for (int k = 0; k < D / 16; ++k) {
+                                const uint64_t ad =
+                                    smem_desc(a_base + t * C::kATile + 32 * k, 16, C::kSBO, C::kSwz);
+                                const uint64_t bd = smem_desc(i_base + t * C::kItemTile + 32 * k, 16,
+                                                              C::kSBO, C::kSwz);
+                                if (elect_one())
+                                    mma_ss(t0 + t * C::kItem, ad, bd, C::kIdescS, k > 0 ? 1u : 0u);
+                                __syncwarp();
+                            }
+                        }
+                        if (elect_one()) mma_commit(sready0 + 8u * s);
+                        __syncwarp();
+                    } else {
+                        if (elect_one()) mma_commit(accdone0 + 8u * s);
+                        __syncwarp();
+                        ++nu[s];
+                    }
+                }
+                if (!ok) break;
+                if (i > 0) {
+                    if (elect_one()) mma_commit(empty0 + 8u * prev_st);  // item i - 1 consumed
+                    __syncwarp();
+                }
+                if (i < U.n_items) {
+                    prev_st = st;
+                    ++it;
+                }
+            }
+            if (!ok) break;
+            if (elect_one()) mma_commit(afree0 + 8u * ab);
+            __syncwarp();
+        }
+        // every product issued has completed before TMEM is released
+        if (elect_one()) mma_commit(fin);
+        __syncwarp();
+        const uint64_t t0 = globaltimer_ns();
+        while (!__all_sync(0xffffffffu, mbar_try_wait(fin, 0)) &&
+               globaltimer_ns() - t0 < kWaitLimitNs) {
+        }
+    } else if (warp >= kFirstSoftmaxWarp) {
+        // ------------------------------------------------------------ softmax warpgroups
+        const int s = (warp - kFirstSoftmaxWarp) / 4;
+        const int q = warp % 4;  // TMEM lane quadrant of this warp
+        const int r = 32 * q + lane;
+        const uint32_t t0 = tmem + ((uint32_t)(32 * q) << 16) + s * C::kColStream;
+        const float c = prm.c;
+        uint32_t it = 0, sj = 0, na = 0;
+        bool ok = true;
+        for (int64_t u = blockIdx.x; u < prm.n_units && ok; u += gridDim.x) {
+            const BUnit U = bwd_unit<D, PASS>(prm, u);
+            if (s >= U.n_act) {
+                it += U.n_items;
+                continue;
+            }
+            const int64_t row = U.row0 + s * kRows + r;
+            const bool valid = row < U.rows;
+            float Lr = 0.f, cr = 0.f;
+            if (C::kRowStats && valid) {
+                Lr = prm.Lrow[U.bh * U.rows + row];
+                cr = prm.crow[U.bh * U.rows + row];
+            }
+            for (int i = 0; i < U.n_items; ++i, ++it) {
+                const int st = it % C::kStages;
+                if (!warp_wait(sready0 + 8u * s, sj & 1, abort_flag, prm.status)) {
+                    ok = false;
+                    break;
+                }
+                ++sj;
+                if (C::kColStats &&
+                    !warp_wait(full0 + 8u * st, (it / C::kStages) & 1, abort_flag, prm.status)) {
+                    ok = false;
+                    break;
+                }
+                tc_fence_after();
+                const int nv = (int)min((int64_t)C::kItem, U.item_end - (U.item0 + (int64_t)i * C::kItem));
+                const float* Lc = stats + st * 2 * C::kItem;
+                const float* cc = Lc + C::kItem;
+#pragma unroll
+                for (int h = 0; h < C::kItem / 32; ++h)
+                    bwd_slice<D, PASS>(t0, h, nv, c, Lr, cr, Lc, cc);
+                tmem_wait_st();
+                tc_fence_before();
+                mbar_arrive(pready0 + 8u * s);
+            }
+            if (!ok) break;
+            // epilogue: the unit's accumulators
+            if (!warp_wait(accdone0 + 8u * s, na & 1, abort_flag, prm.status)) {
+                ok = false;
+                break;
+            }
+            ++na;
+            tc_fence_after();
+            float a0[D], a1[C::kNAcc == 2 ? D : 1];
+            const uint32_t acc = t0 + C::kNA * C::kItem;
+#pragma unroll
+            for (int k = 0; k < D / 16; ++k) {
+                uint32_t t[16];
+                tmem_ld16(acc + 16 * k, t);
+                tmem_wait_ld16(t);
+#pragma unroll
+                for (int e = 0; e < 16; ++e) a0[16 * k + e] = __uint_as_float(t[e]);
+                if (C::kNAcc == 2) {
+                    tmem_ld16(acc + D + 16 * k, t);
+                    tmem_wait_ld16(t);
+#pragma unroll
+                    for (int e = 0; e < 16; ++e) a1[16 * k + e] = __uint_as_float(t[e]);
+                }
+            }
+            tc_fence_before();
+            mbar_arrive(accfree0 + 8u * s);
+            if (valid) {
+                if (C::kRouteRows) {
+                    const int64_t idx = (U.bh * prm.nchunk + U.chunk) * prm.M + row;
+                    float4* d0 = reinterpret_cast<float4*>(prm.pb + idx * D);
+#pragma unroll
+                    for (int k = 0; k < D / 4; ++k)
+                        d0[k] = make_float4(a0[4 * k], a0[4 * k + 1], a0[4 * k + 2], a0[4 * k + 3]);
+                    if (C::kNAcc == 2) {
+                        float4* d1 = reinterpret_cast<float4*>(prm.pa + idx * D);
+#pragma unroll
+                        for (int k = 0; k < D / 4; ++k)
+                            d1[k] =
+                                make_float4(a1[4 * k], a1[4 * k + 1], a1[4 * k + 2], a1[4 * k + 3]);
+                    }
+                } else {
+                    const float sc = prm.scale;
+                    uint4* d0 = reinterpret_cast<uint4*>(prm.out0 + (U.bh * prm.N + row) * D);
+                    uint4* d1 = reinterpret_cast<uint4*>(prm.out1 + (U.bh * prm.N + row) * D);
+#pragma unroll
+                    for (int k = 0; k < D / 8; ++k) {
+                        uint4 v;
+                        v.x = pack_bf16(sc * a0[8 * k + 0], sc * a0[8 * k + 1]);
+                        v.y = pack_bf16(sc * a0[8 * k + 2], sc * a0[8 * k + 3]);
+                        v.z = pack_bf16(sc * a0[8 * k + 4], sc * a0[8 * k + 5]);
+                        v.w = pack_bf16(sc * a0[8 * k + 6], sc * a0[8 * k + 7]);
+                        d0[k] = v;
+                        v.x = pack_bf16(a1[8 * k + 0], a1[8 * k + 1]);
+                        v.y = pack_bf16(a1[8 * k + 2], a1[8 * k + 3]);
+                        v.z = pack_bf16(a1[8 * k + 4], a1[8 * k + 5]);
+                        v.w = pack_bf16(a1[8 * k + 6], a1[8 * k + 7]);
+                        d1[k] = v;
+                    }
+                }
+            }
+        }
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    if (warp == 1) tmem_dealloc(tmem, kTmemCols);
+}
+
+// ------------------------------------------------------------------ host side
+
+PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
+    static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+    static std::once_flag once;
+    std::call_once(once, [] {
+        void* p = nullptr;
+        cudaDriverEntryPointQueryResult q;
+        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000,
+                                             cudaEnableDefault, &q) == cudaSuccess &&
+            q == cudaDriverEntryPointSuccess)
+            fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(p);
+    });
+    return fn;
+}
+
+// A bf16 [z][rows][D] tensor, boxes of box_rows x D, swizzled to the row width.
+bool make_map(CUtensorMap* m, const void* base, int64_t D, int64_t rows, int64_t z,
+              uint32_t box_rows) {
+    auto fn = encode_fn();
+    if (!fn) return false;
+    cuuint64_t dims[3] = {(cuuint64_t)D, (cuuint64_t)rows, (cuuint64_t)z};
+    cuuint64_t strides[2] = {(cuuint64_t)(D * 2), (cuuint64_t)(rows * D * 2)};
+    cuuint32_t box[3] = {(cuuint32_t)D, box_rows, 1};
+    cuuint32_t estr[3] = {1, 1, 1};
+    const CUtensorMapSwizzle sw = D == 16 ? CU_TENSOR_MAP_SWIZZLE_32B
+                                          : (D == 32 ? CU_TENSOR_MAP_SWIZZLE_64B
+                                                     : CU_TENSOR_MAP_SWIZZLE_128B);
+    return fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(base), dims, strides, box,
+              estr, CU_TENSOR_MAP_INTERLEAVE_NONE, sw, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+              CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+template <int D, int PASS>
+cudaError_t launch_pass(const CUtensorMap* maps, const BwdParams& prm, cudaStream_t st) {
+    using Cf = BCfg<D, PASS>;
+    static cudaError_t attr = cudaFuncSetAttribute(
+        tc_bwd_kernel<D, PASS>, cudaFuncAttributeMaxDynamicSharedMemorySize, Cf::kSmem);
+    if (attr != cudaSuccess) return attr;
+    if (prm.n_units == 0) return cudaSuccess;
+    int dev = 0, sms = kNumSMs;
+    cudaGetDevice(&dev);
+    cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+    const int64_t grid = prm.n_units < sms ? prm.n_units : sms;
+    tc_bwd_kernel<D, PASS><<<(unsigned)grid, kThreads, Cf::kSmem, st>>>(
+        maps[0], maps[1], maps[2], maps[3], maps[4], maps[5], prm);
+    return cudaGetLastError();
+}
+
+template <int PASS>
+cudaError_t launch_d(int64_t D, const CUtensorMap* maps, const BwdParams& prm, cudaStream_t st) {
+    switch (D) {
+        case 16: return launch_pass<16, PASS>(maps, prm, st);
+        case 32: return launch_pass<32, PASS>(maps, prm, st);
+        case 64: return launch_pass<64, PASS>(maps, prm, st);
+        default: return cudaErrorInvalidValue;
+    }
+}
+
+}  // namespace
+
+int64_t tc_bwd_item(int64_t D) { return D == 64 ? 32 : 64; }
+
+cudaError_t tc_bwd_pass(const Plan& p, const BwdPlan& bp, int pass, const TcBwdOperands& o,
+                        float scale, int* status, cudaStream_t st) {
+    const int64_t item = tc_bwd_item(p.D);
+    const bool route_rows = pass <= kR1;
+    // A tiles: 128 rows of the pass's row dimension; items: `item` rows of the other one
+    const int64_t arows = route_rows ? p.M : p.N;
+    const int64_t irows = route_rows ? p.N : p.M;
+    CUtensorMap maps[6];
+    const void* srcs[6] = {o.a[0], o.a[1], o.a[2], o.i[0], o.i[1], o.i[2]};
+    const int nmaps = pass == kT23 ? 3 : 2;
+    for (int k = 0; k < 6; ++k) {
+        const bool used = (k % 3) < nmaps;
+        const void* base = used ? srcs[k] : srcs[k % 3 == 2 ? k - 2 : k];
+        const bool a_side = k < 3;
+        const bool per_head = a_side ? (pass == kR1 && k == 0) : (pass == kT1 && k == 3);
+        if (!make_map(&maps[k], base, p.D, a_side ? arows : irows, per_head ? p.H : p.BH,
+                      a_side ? kRows : (uint32_t)item))
+            return cudaErrorInvalidValue;
+    }
+    BwdParams prm{};
+    prm.BH = p.BH;
+    prm.H = p.H;
+    prm.N = p.N;
+    prm.M = p.M;
+    prm.c = scale * 1.4426950408889634f;
+    prm.scale = scale;
+    prm.a0_per_head = pass == kR1 ? 1 : 0;
+    prm.i0_per_head = pass == kT1 ? 1 : 0;
+    prm.chunk_len = bp.chunk_len;
+    prm.nchunk = bp.nchunk;
+    prm.n_groups = (p.M + NS * kRows - 1) / (NS * kRows);
+    prm.n_tok_groups = (p.N + NS * kRows - 1) / (NS * kRows);
+    prm.n_units = route_rows ? p.BH * prm.n_groups * bp.nchunk : p.BH * prm.n_tok_groups;
+    prm.Lrow = o.Lrow;
+    prm.crow = o.crow;
+    prm.Lcol = o.Lcol;
+    prm.ccol = o.ccol;
+    prm.pa = o.pa;
+    prm.pb = o.pb;
+    prm.out0 = (__nv_bfloat16*)o.out0;
+    prm.out1 = (__nv_bfloat16*)o.out1;
+    prm.status = status;
+    switch (pass) {
+        case kR3: return launch_d<kR3>(p.D, maps, prm, st);
+        case kR2: return launch_d<kR2>(p.D, maps, prm, st);
+        case kR1: return launch_d<kR1>(p.D, maps, prm, st);
+        case kT23: return launch_d<kT23>(p.D, maps, prm, st);
+        case kT1: return launch_d<kT1>(p.D, maps, prm, st);
+        default: return cudaErrorInvalidValue;
+    }
+}
+
+}  // namespace flarepp

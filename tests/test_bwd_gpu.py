@@ -69,6 +69,8 @@ SHAPES = [
     (1, 2, 500, 64, 64, "bf16", None),
     (2, 2, 600, 50, 32, "bf16", -0.3),
     (1, 2, 130, 513, 32, "bf16", None),   # ragged route tile
+    (1, 1, 50, 10, 32, "bf16", None),     # one partial tile each way
+    (2, 1, 129, 257, 64, "bf16", 0.2),    # tails of both 256-row groups
 ]
 
 
