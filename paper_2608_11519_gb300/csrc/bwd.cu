@@ -50,17 +50,36 @@ __device__ __forceinline__ float ex2(float x) {
     return y;
 }
 
-// c3[n] = <dY_n, Y_n>: one thread per token.
+// c3[n] = <dY_n, Y_n>: each thread reads one 16-byte vector of a row of dY and of Y (so a
+// warp reads consecutive rows whole), and the D / V threads of a row add their partial dot
+// products with shuffles. rows * D / V threads in all.
 template <int D, typename T>
 __global__ void __launch_bounds__(256) delta_tokens_kernel(const T* __restrict__ dY,
                                                            const T* __restrict__ Y, int64_t rows,
                                                            float* __restrict__ c3) {
-    const int64_t r = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
-    if (r >= rows) return;
+    constexpr int V = 16 / (int)sizeof(T);  // elements per 16-byte vector
+    constexpr int TPR = D / V;              // threads per row (2 .. 16, a power of two)
+    const int64_t t = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+    const int64_t r = t / TPR;
     float acc = 0.f;
+    if (r < rows) {
+        const uint4 a = reinterpret_cast<const uint4*>(dY)[t];
+        const uint4 b = reinterpret_cast<const uint4*>(Y)[t];
+        const T* av = reinterpret_cast<const T*>(&a);
+        const T* bv = reinterpret_cast<const T*>(&b);
 #pragma unroll
-    for (int d = 0; d < D; ++d) acc = fmaf(ld_f32(dY + r * D + d), ld_f32(Y + r * D + d), acc);
-    c3[r] = acc;
+        for (int e = 0; e < V; ++e) acc = fmaf(ld_f32(av + e), ld_f32(bv + e), acc);
+    }
+#pragma unroll
+    for (int off = TPR / 2; off > 0; off >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, off);
+    if (r < rows && (t % TPR) == 0) c3[r] = acc;
+}
+
+template <int D, typename T>
+void launch_delta_tokens(const T* dY, const T* Y, int64_t rows, float* c3, cudaStream_t st) {
+    constexpr int TPR = D / (16 / (int)sizeof(T));
+    const int64_t threads = rows * TPR;
+    delta_tokens_kernel<D, T><<<(unsigned)((threads + 255) / 256), 256, 0, st>>>(dY, Y, rows, c3);
 }
 
 // bf16 copy of a float32 array (the tensor-core passes' Q and Z operands)
@@ -338,8 +357,7 @@ cudaError_t route_bwd_d(const Plan& p, const BwdPlan& bp, const T* seeds, const 
     const unsigned token_blocks = (unsigned)(((p.N + 127) / 128) * p.BH);
     const unsigned red_blocks = (unsigned)((lat_rows + 7) / 8);
 
-    delta_tokens_kernel<D, T><<<(unsigned)((tok_rows + 255) / 256), 256, 0, st>>>(dY, Y, tok_rows,
-                                                                                  c3);
+    launch_delta_tokens<D, T>(dY, Y, tok_rows, c3, st);
     // call 3: dZ and the decoder's dQ
     route_pass_kernel<D, T, float, 3><<<route_blocks, route_threads, 0, st>>>(
         Q32, 0, K, dY, Z32, nullptr, nullptr, L3, c3, p.H, p.N, p.M, bp.chunk_len, bp.nchunk,
@@ -405,8 +423,7 @@ cudaError_t route_bwd_tc_d(const Plan& p, const BwdPlan& bp, const void* seeds, 
     const unsigned cvt_blocks = (unsigned)min((int64_t)1024, (lat + 255) / 256);
     cudaError_t e;
 
-    delta_tokens_kernel<D, T><<<(unsigned)((tok_rows + 255) / 256), 256, 0, st>>>(
-        (const T*)dY, (const T*)Y, tok_rows, c3);
+    launch_delta_tokens<D, T>((const T*)dY, (const T*)Y, tok_rows, c3, st);
     to_bf16_kernel<<<cvt_blocks, 256, 0, st>>>(Q32, qb, lat);
     to_bf16_kernel<<<cvt_blocks, 256, 0, st>>>(Z32, zb, lat);
     TcBwdOperands o{};

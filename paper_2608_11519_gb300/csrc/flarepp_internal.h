@@ -53,8 +53,8 @@ SavedLayout saved_layout(const Plan& p);
 
 // The backward's plan: the split-N route passes (chunks of tokens) and its workspace. On
 // the CUDA-core path a route pass gives one thread per route (m_tile routes per CTA); on
-// the tensor-core path a work unit is a group of 256 routes and a chunk of tokens, and
-// chunk_len is a multiple of the 64- (D = 64: 32-) token item.
+// the tensor-core path a work unit is a group of up to 512 routes and a chunk of tokens,
+// and chunk_len is a multiple of 64 tokens (whole items of either size).
 struct BwdPlan {
     int path;                   // kPathSimt or kPathTc
     int64_t m_tile, n_mtiles;   // CUDA-core route passes: routes per CTA, route tiles per head
@@ -117,8 +117,6 @@ struct TcBwdOperands {
 // pass: 0 = R3, 1 = R2, 2 = R1 (route rows), 3 = T23, 4 = T1 (token rows)
 cudaError_t tc_bwd_pass(const Plan& p, const BwdPlan& bp, int pass, const TcBwdOperands& o,
                         float scale, int* status, cudaStream_t st);
-// Tokens (route-row passes) or routes (token-row passes) per streamed item.
-int64_t tc_bwd_item(int64_t D);
 
 // ---- tensor-core kernels (tc_kernels.cu), bf16 inputs
 // Encode call 1 (A = seeds) or call 2 (A = Q operand) into the chunk partials.

@@ -139,9 +139,10 @@ BwdPlan make_bwd_plan(const Plan& p) {
     b.m_tile = p.M >= 128 ? 128 : cdiv(p.M, 32) * 32;
     b.n_mtiles = cdiv(p.M, b.m_tile);
     if (p.path == kPathTc) {
-        // work units (b*h, 256-route group, chunk): about two waves of persistent CTAs
-        const int64_t item = p.D == 64 ? 32 : 64;
-        const int64_t groups = cdiv(p.M, 256);
+        // work units (b*h, route group of up to 512, chunk): about two waves of persistent
+        // CTAs; chunks are whole items (64 tokens covers both item sizes)
+        const int64_t item = 64;
+        const int64_t groups = cdiv(p.M, 512);
         int64_t want = cdiv(2 * kNumSMs, p.BH * groups);
         if (want < 1) want = 1;
         b.chunk_len = cdiv(cdiv(p.N, want), item) * item;

@@ -23,9 +23,12 @@
 // Score products take both operands from shared memory (TMA, swizzled, K-major); the
 // accumulating products read P or dS from TMEM and the item, MN-major, from shared memory.
 //
-// Roles (12 warps): warp 0 the TMA producer (it also stages each item's column statistics
-// in shared memory), warp 1 the MMA issuer, warps 4..11 two softmax warpgroups, one per
-// TMEM stream of 128 rows. A work unit is (b*h, group of 2 x 128 rows, chunk of items).
+// Roles: one MMA warp per TMEM stream of 128 rows (a commit stalls only the warp that
+// issues it), one softmax warpgroup per stream (warps 4..), and a TMA producer warp that
+// also stages each item's column statistics in shared memory. A pass has as many streams as
+// its TMEM columns allow (at most four) and items of 64 rows when three streams fit with
+// them, else 32; the softmax works on 16-column slices in packed f32x2 arithmetic. A work
+// unit is (b*h, group of NS x 128 rows, chunk of items).
 // Every wait is bounded (2 s of %globaltimer): on expiry the kernel records
 // FLAREPP_ERR_TIMEOUT in the status word, every role leaves its loops, the producer waits
 // for its copies in flight, the MMA issuer for its products, and TMEM is freed.
@@ -43,11 +46,8 @@ namespace {
 
 using namespace tc;
 
-constexpr int kWarps = 12;
-constexpr int kThreads = kWarps * 32;
 constexpr int kFirstSoftmaxWarp = 4;
-constexpr int NS = 2;           // TMEM streams (softmax warpgroups)
-constexpr int kRows = 128;      // TMEM lanes per stream, MMA M
+constexpr int kRows = 128;  // TMEM lanes per stream, MMA M
 constexpr uint64_t kWaitLimitNs = 2000000000ull;
 constexpr uint32_t kTmemCols = 512;
 
@@ -60,21 +60,33 @@ struct BCfg {
     static constexpr int kNAcc = (PASS == kR2 || PASS == kR1) ? 1 : 2;
     static constexpr bool kColStats = PASS == kR3 || PASS == kT23 || PASS == kT1;
     static constexpr bool kRowStats = PASS == kR2 || PASS == kR1 || PASS == kT23;
-    static constexpr int kItem = D == 64 ? 32 : 64;
-    static constexpr int kABuf = D == 64 ? 1 : 2;  // shared-memory copies of a unit's A tiles
-    static constexpr int kStages = 6;
+    // TMEM per stream: kNA score tiles of kItem columns, then kNAcc accumulators of D.
+    // Items of 64 rows when three streams fit with them, else 32; as many streams as fit
+    // in 512 columns, at most four.
+    static constexpr uint32_t col_stream(int item) { return kNA * item + kNAcc * D; }
+    static constexpr int kItem = 3 * col_stream(64) <= kTmemCols ? 64 : 32;
+    static constexpr uint32_t kColStream = col_stream(kItem);
+    static constexpr int kFit = (int)(kTmemCols / kColStream);
+    static constexpr int NS = kFit > 4 ? 4 : kFit;
+    static_assert(NS >= 1, "TMEM budget");
+    // warps 0..NS-1 issue MMAs (one per stream), warps 4.. are the softmax warpgroups, and
+    // the TMA producer is warp 3 (NS < 4) or the warp after the softmax warps (NS = 4)
+    static constexpr int kProdWarp = NS < 4 ? 3 : kFirstSoftmaxWarp + 4 * NS;
+    static constexpr int kWarps = kFirstSoftmaxWarp + 4 * NS + (NS < 4 ? 0 : 1);
+    static constexpr int kThreads = kWarps * 32;
+    static constexpr int kGroup = NS * kRows;  // rows per work unit
+    static constexpr int kStages = kItem == 64 ? 6 : 10;
     static constexpr int kATile = kRows * D * 2;
     static constexpr int kABytes = NS * kNA * kATile;  // one unit's A tiles
     static constexpr int kItemTile = kItem * D * 2;
     static constexpr int kStage = kNA * kItemTile;
+    // two shared-memory copies of a unit's A tiles when they fit beside the ring
+    static constexpr int kABuf = 2 * kABytes + kStages * kStage <= 200 * 1024 ? 2 : 1;
     static constexpr uint32_t kSwz = D == 16 ? kSw32 : (D == 32 ? kSw64 : kSw128);
     static constexpr uint32_t kSBO = 8 * D * 2;
-    // TMEM per stream: kNA score tiles of kItem columns, then kNAcc accumulators of D
-    static constexpr uint32_t kColStream = kNA * kItem + kNAcc * D;
-    static_assert(NS * kColStream <= kTmemCols, "TMEM budget");
-    // barriers: full[S], empty[S], afull[kABuf], afree[kABuf], sready[NS], pready[NS],
-    //           accdone[NS], accfree[NS], fin
-    static constexpr int kNumBars = 2 * kStages + 2 * kABuf + 4 * NS + 1;
+    // barriers: full[S], empty[S], afull[kABuf], afree[kABuf], then per stream sready,
+    //           pready, accdone, accfree, fin
+    static constexpr int kNumBars = 2 * kStages + 2 * kABuf + 5 * NS;
     static constexpr int kStatBytes = kStages * 2 * kItem * 4;
     static constexpr int kData = kABuf * kABytes + kStages * kStage;
     static constexpr int kNeed = 1024 + kData + kStatBytes + kNumBars * 8 + 16;
@@ -89,10 +101,10 @@ struct BwdParams {
     int64_t BH, H, N, M;
     float c;      // scale * log2(e), signed
     float scale;  // s
-    int a0_per_head;     // R1: the first A operand (seeds) is indexed by head
-    int i0_per_head;     // T1: the first item operand (seeds) is indexed by head
-    int64_t chunk_len, nchunk, n_groups;  // route-row passes
-    int64_t n_tok_groups;                 // token-row passes
+    int a0_per_head;            // R1: the first A operand (seeds) is indexed by head
+    int i0_per_head;            // T1: the first item operand (seeds) is indexed by head
+    int64_t chunk_len, nchunk;  // route-row passes
+    int64_t n_groups;           // route groups (route-row passes) or token groups
     int64_t n_units;
     const float* Lrow;  // row statistics [BH][rows]: L (base 2) and c
     const float* crow;
@@ -107,10 +119,10 @@ struct BwdParams {
 
 struct BUnit {
     int64_t bh, g, chunk;
-    int64_t row0;          // first TMEM row (route or token) of stream 0
-    int64_t rows;          // route or token count of the rows' dimension (M or N)
+    int64_t row0;  // first TMEM row (route or token) of stream 0
+    int64_t rows;  // route or token count of the rows' dimension (M or N)
     int64_t item0, item_end;
-    int n_act;             // streams with at least one valid row
+    int n_act;  // streams with at least one valid row
     int n_items;
 };
 
@@ -127,16 +139,16 @@ __device__ __forceinline__ BUnit bwd_unit(const BwdParams& p, int64_t u) {
         U.item0 = U.chunk * p.chunk_len;
         U.item_end = min(p.N, U.item0 + p.chunk_len);
     } else {
-        U.g = u % p.n_tok_groups;
-        U.bh = u / p.n_tok_groups;
+        U.g = u % p.n_groups;
+        U.bh = u / p.n_groups;
         U.chunk = 0;
         U.rows = p.N;
         U.item0 = 0;
         U.item_end = p.M;
     }
-    U.row0 = U.g * (NS * kRows);
+    U.row0 = U.g * C::kGroup;
     const int64_t left = U.rows - U.row0;
-    U.n_act = left >= NS * kRows ? NS : (int)((left + kRows - 1) / kRows);
+    U.n_act = left >= C::kGroup ? C::NS : (int)((left + kRows - 1) / kRows);
     U.n_items = (int)((U.item_end - U.item0 + C::kItem - 1) / C::kItem);
     return U;
 }
@@ -150,6 +162,39 @@ __device__ __forceinline__ float ex2(float x) {
 __device__ __forceinline__ uint32_t pack_bf16(float lo, float hi) {
     __nv_bfloat162 v = __floats2bfloat162_rn(lo, hi);
     return *reinterpret_cast<uint32_t*>(&v);
+}
+
+// packed pairs of f32 (lo, hi) in one 64-bit register
+__device__ __forceinline__ uint64_t fma2(uint64_t a, uint64_t b, uint64_t c) {
+    uint64_t d;
+    asm("fma.rn.f32x2 %0, %1, %2, %3;" : "=l"(d) : "l"(a), "l"(b), "l"(c));
+    return d;
+}
+__device__ __forceinline__ uint64_t add2(uint64_t a, uint64_t b) {
+    uint64_t d;
+    asm("add.rn.f32x2 %0, %1, %2;" : "=l"(d) : "l"(a), "l"(b));
+    return d;
+}
+__device__ __forceinline__ uint64_t mul2(uint64_t a, uint64_t b) {
+    uint64_t d;
+    asm("mul.rn.f32x2 %0, %1, %2;" : "=l"(d) : "l"(a), "l"(b));
+    return d;
+}
+__device__ __forceinline__ uint64_t ex2x2(uint64_t x) {
+    float a, b;
+    unpack_f32x2(x, a, b);
+    return pack_f32x2(ex2(a), ex2(b));
+}
+// bf16 pair (lo in the low half) from a packed f32 pair
+__device__ __forceinline__ uint32_t bf16x2(uint64_t v) {
+    uint32_t r;
+    asm("{\n\t.reg .f32 a, b;\n\tmov.b64 {a, b}, %1;\n\tcvt.rn.bf16x2.f32 %0, b, a;\n\t}"
+        : "=r"(r)
+        : "l"(v));
+    return r;
+}
+__device__ __forceinline__ uint64_t ld_pair(const uint32_t* r, int k) {
+    return pack_f32x2(__uint_as_float(r[2 * k]), __uint_as_float(r[2 * k + 1]));
 }
 
 // Bounded wait on an mbarrier phase. Returns false when the kernel is aborting.
@@ -175,65 +220,70 @@ __device__ __forceinline__ bool warp_wait(uint32_t bar, uint32_t parity, volatil
     return __all_sync(0xffffffffu, got);
 }
 
-// One 32-column slice of an item for this thread's row: reads the score tiles, writes bf16
-// dS over score tile 0 and (when a second accumulator reads it) bf16 P over score tile 1.
-// Columns at or beyond nv are outside the item: P = dS = 0.
-template <int D, int PASS>
-__device__ __forceinline__ void bwd_slice(uint32_t t0, int h, int nv, float c, float Lr, float cr,
-                                          const float* Lc, const float* cc) {
+// One 16-column slice h of an item for this thread's row: reads the score tiles, writes
+// bf16 dS over score tile 0 and (when a second accumulator reads it) bf16 P over score
+// tile 1. Math on packed f32 pairs. The row statistics come as (-L, -L) and (-c, -c) pairs;
+// the column statistics sit negated in shared memory. When the item is short (FULL false),
+// columns at or beyond nv get P = dS = 0.
+template <int D, int PASS, bool FULL>
+__device__ __forceinline__ void bwd_slice(uint32_t t0, int h, int nv, uint64_t c2, uint64_t nLr2,
+                                          uint64_t ncr2, const float* nLc, const float* ncc) {
     using C = BCfg<D, PASS>;
-    uint32_t sr[32], d1[32], d2[PASS == kT23 ? 32 : 1];
-    tmem_ld32(t0 + 32 * h, sr);
-    tmem_ld32(t0 + C::kItem + 32 * h, d1);
-    if (PASS == kT23) tmem_ld32(t0 + 2 * C::kItem + 32 * h, d2);
-    tmem_wait_ld32(sr);
-    tmem_wait_ld32(d1);
-    if (PASS == kT23) tmem_wait_ld32(d2);
-    uint32_t ds[16], pp[16];
+    uint32_t sr[16], d1[16], d2[PASS == kT23 ? 16 : 1];
+    tmem_ld16(t0 + 16 * h, sr);
+    tmem_ld16(t0 + C::kItem + 16 * h, d1);
+    if (PASS == kT23) tmem_ld16(t0 + 2 * C::kItem + 16 * h, d2);
+    tmem_wait_ld16(sr);
+    tmem_wait_ld16(d1);
+    if (PASS == kT23) tmem_wait_ld16(d2);
+    uint32_t ds[8], pp[8];
 #pragma unroll
-    for (int k = 0; k < 16; ++k) {
-        float dsv[2], pv[2];
-#pragma unroll
-        for (int e = 0; e < 2; ++e) {
-            const int col = 32 * h + 2 * k + e;
-            const float x = __uint_as_float(sr[2 * k + e]);
-            const float dp = __uint_as_float(d1[2 * k + e]);
-            float p, d;
-            if (PASS == kR2 || PASS == kR1) {
-                p = ex2(fmaf(c, x, -Lr));
-                d = p * (dp - cr);
-            } else if (PASS == kT23) {
-                p = ex2(fmaf(c, x, -Lc[col]));
-                const float p3 = ex2(fmaf(c, x, -Lr));
-                d = fmaf(p3, __uint_as_float(d2[2 * k + e]) - cr, p * (dp - cc[col]));
-            } else {  // R3, T1: column statistics only
-                p = ex2(fmaf(c, x, -Lc[col]));
-                d = p * (dp - cc[col]);
+    for (int k = 0; k < 8; ++k) {
+        const int col = 16 * h + 2 * k;
+        const uint64_t x = ld_pair(sr, k);
+        const uint64_t dp = ld_pair(d1, k);
+        uint64_t p, d;
+        if (PASS == kR2 || PASS == kR1) {
+            p = ex2x2(fma2(x, c2, nLr2));
+            d = mul2(p, add2(dp, ncr2));
+        } else {
+            const uint64_t nL = *reinterpret_cast<const uint64_t*>(nLc + col);
+            const uint64_t nc = *reinterpret_cast<const uint64_t*>(ncc + col);
+            p = ex2x2(fma2(x, c2, nL));
+            d = mul2(p, add2(dp, nc));
+            if (PASS == kT23) {
+                const uint64_t p3 = ex2x2(fma2(x, c2, nLr2));
+                d = fma2(p3, add2(ld_pair(d2, k), ncr2), d);
             }
-            const bool in = col < nv;
-            dsv[e] = in ? d : 0.f;
-            pv[e] = in ? p : 0.f;
         }
-        ds[k] = pack_bf16(dsv[0], dsv[1]);
-        pp[k] = pack_bf16(pv[0], pv[1]);
+        if (!FULL) {
+            float a, b;
+            unpack_f32x2(d, a, b);
+            d = pack_f32x2(col < nv ? a : 0.f, col + 1 < nv ? b : 0.f);
+            unpack_f32x2(p, a, b);
+            p = pack_f32x2(col < nv ? a : 0.f, col + 1 < nv ? b : 0.f);
+        }
+        ds[k] = bf16x2(d);
+        pp[k] = bf16x2(p);
     }
-    tmem_st16(t0 + 16 * h, ds);
-    if (C::kNAcc == 2) tmem_st16(t0 + C::kItem + 16 * h, pp);
+    tmem_st8(t0 + 8 * h, ds);
+    if (C::kNAcc == 2) tmem_st8(t0 + C::kItem + 8 * h, pp);
 }
 
 // ------------------------------------------------------------------ the kernel
 
 template <int D, int PASS>
-__global__ void __launch_bounds__(kThreads, 1)
+__global__ void __launch_bounds__(BCfg<D, PASS>::kThreads, 1)
     tc_bwd_kernel(const __grid_constant__ CUtensorMap tmA0, const __grid_constant__ CUtensorMap tmA1,
                   const __grid_constant__ CUtensorMap tmA2, const __grid_constant__ CUtensorMap tmI0,
                   const __grid_constant__ CUtensorMap tmI1, const __grid_constant__ CUtensorMap tmI2,
                   const BwdParams prm) {
     using C = BCfg<D, PASS>;
+    constexpr int NS = C::NS;
     extern __shared__ uint8_t smem_raw[];
     uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                                ~static_cast<uintptr_t>(1023));
-    uint8_t* abuf = smem;                         // kABuf x [NS][kNA] A tiles, swizzled
+    uint8_t* abuf = smem;                          // kABuf x [NS][kNA] A tiles, swizzled
     uint8_t* ring = smem + C::kABuf * C::kABytes;  // kStages x kNA item tiles, swizzled
     float* stats = reinterpret_cast<float*>(ring + C::kStages * C::kStage);  // [S][2][kItem]
     uint64_t* bars = reinterpret_cast<uint64_t*>(stats + C::kStages * 2 * C::kItem);
@@ -248,7 +298,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     const uint32_t pready0 = sready0 + 8u * NS;
     const uint32_t accdone0 = pready0 + 8u * NS;
     const uint32_t accfree0 = accdone0 + 8u * NS;
-    const uint32_t fin = accfree0 + 8u * NS;
+    const uint32_t fin0 = accfree0 + 8u * NS;
 
     const int warp = threadIdx.x >> 5;
     const int lane = threadIdx.x & 31;
@@ -256,19 +306,19 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (threadIdx.x == 0) {
         for (int st = 0; st < C::kStages; ++st) {
             mbar_init(full0 + 8u * st, C::kColStats ? 33 : 1);
-            mbar_init(empty0 + 8u * st, 1);
+            mbar_init(empty0 + 8u * st, NS);
         }
         for (int b = 0; b < C::kABuf; ++b) {
             mbar_init(afull0 + 8u * b, 1);
-            mbar_init(afree0 + 8u * b, 1);
+            mbar_init(afree0 + 8u * b, NS);
         }
         for (int s = 0; s < NS; ++s) {
             mbar_init(sready0 + 8u * s, 1);
             mbar_init(pready0 + 8u * s, kRows);
             mbar_init(accdone0 + 8u * s, 1);
             mbar_init(accfree0 + 8u * s, kRows);
+            mbar_init(fin0 + 8u * s, 1);
         }
-        mbar_init(fin, 1);
         *abort_flag = 0;
         fence_mbar_init();
         prefetch_tmap(&tmA0);
@@ -280,7 +330,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             prefetch_tmap(&tmI2);
         }
     }
-    if (warp == 1) {
+    if (warp == 0) {
         tmem_alloc(smem_u32(tmem_slot), kTmemCols);
         tmem_relinquish();
     }
@@ -289,7 +339,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     tc_fence_after();
     const uint32_t tmem = *tmem_slot;
 
-    if (warp == 0) {
+    if (warp == C::kProdWarp) {
         // ------------------------------------------------------------ TMA producer
         uint32_t it = 0, ua = 0, a_issued = 0;
         bool ok = true;
@@ -336,16 +386,19 @@ __global__ void __launch_bounds__(kThreads, 1)
                     if (C::kNA == 3)
                         tma_load_3d(dst + 2 * C::kItemTile, &tmI2, 0, (int)row, (int)U.bh,
                                     full0 + 8u * st);
+                    // streams idle in this unit count as having released the stage
+                    for (int x = U.n_act; x < NS; ++x) mbar_arrive(empty0 + 8u * st);
                 }
                 __syncwarp();
                 if (C::kColStats) {
+                    // the item's column statistics, negated (P = 2^(c x + (-L)))
                     float* sl = stats + st * 2 * C::kItem;
                     const int64_t nvalid = U.item_end - row;
                     for (int k = lane; k < C::kItem; k += 32) {
                         const bool in = k < nvalid;
                         const int64_t idx = U.bh * (C::kRouteRows ? prm.N : prm.M) + row + k;
-                        sl[k] = in ? prm.Lcol[idx] : 0.f;
-                        sl[C::kItem + k] = in ? prm.ccol[idx] : 0.f;
+                        sl[k] = in ? -prm.Lcol[idx] : 0.f;
+                        sl[C::kItem + k] = in ? -prm.ccol[idx] : 0.f;
                     }
                     mbar_arrive(full0 + 8u * st);
                 }
@@ -367,19 +420,21 @@ __global__ void __launch_bounds__(kThreads, 1)
                 }
             }
         }
-    } else if (warp == 1) {
-        // ------------------------------------------------------------ MMA issuer
-        uint32_t it = 0, ua = 0;
-        uint32_t pj[NS] = {0, 0};   // p_ready phases consumed per stream
-        uint32_t nu[NS] = {0, 0};   // units completed per stream (acc_free phases)
+    } else if (warp < NS) {
+        // ------------------------------------------------------------ MMA warp of stream s
+        // For item j: the accumulating products of item j - 1 (after its P / dS is written)
+        // and the score products of item j, then one commit that the softmax waits on. The
+        // softmax frees ring stage j - 1 once S(j) is complete (the tensor pipe runs this
+        // warp's products in order), and the last stage of a unit after acc_done.
+        const int s = warp;
+        uint32_t it = 0, ua = 0, pj = 0, nu = 0;
         bool ok = true;
         auto wait = [&](uint32_t bar, uint32_t parity) {
             return warp_wait(bar, parity, abort_flag, prm.status);
         };
-        // the accumulating products of item `stg` for stream s (P / dS of that item in TMEM)
-        auto issue_acc = [&](int s, int stg, bool accumulate) {
-            const uint32_t t0 = tmem + s * C::kColStream;
-            const uint32_t acc = t0 + C::kNA * C::kItem;
+        const uint32_t t0 = tmem + s * C::kColStream;
+        const uint32_t acc = t0 + C::kNA * C::kItem;
+        auto issue_acc = [&](int stg, bool accumulate) {
             const uint32_t ib = smem_u32(ring + stg * C::kStage);
 #pragma unroll
             for (int k = 0; k < C::kItem / 16; ++k) {
@@ -403,90 +458,87 @@ __global__ void __launch_bounds__(kThreads, 1)
         for (int64_t u = blockIdx.x; u < prm.n_units && ok; u += gridDim.x, ++ua) {
             const BUnit U = bwd_unit<D, PASS>(prm, u);
             const int ab = ua % C::kABuf;
+            // the unit's A tiles (an idle stream waits too, so that its release of the A
+            // buffer counts for this unit's phase)
             if (!wait(afull0 + 8u * ab, (ua / C::kABuf) & 1)) {
                 ok = false;
                 break;
             }
+            if (s >= U.n_act) {
+                if (elect_one()) mbar_arrive(afree0 + 8u * ab);
+                __syncwarp();
+                it += U.n_items;
+                continue;
+            }
             tc_fence_after();
+            const uint32_t a_base = smem_u32(abuf + ab * C::kABytes + s * C::kNA * C::kATile);
             int prev_st = 0;
-            for (int i = 0; i <= U.n_items && ok; ++i) {
+            for (int i = 0; i <= U.n_items; ++i) {
                 const int st = it % C::kStages;
                 if (i < U.n_items) {
                     if (!wait(full0 + 8u * st, (it / C::kStages) & 1)) {
                         ok = false;
                         break;
                     }
-                    tc_fence_after();
                 }
-                for (int s = 0; s < U.n_act; ++s) {
-                    if (i > 0) {
-                        // dS / P of item i - 1 written: its accumulating products
-                        if (!wait(pready0 + 8u * s, pj[s] & 1)) {
-                            ok = false;
-                            break;
-                        }
-                        ++pj[s];
-                        if (i == 1 && nu[s] > 0 && !wait(accfree0 + 8u * s, (nu[s] - 1) & 1)) {
-                            ok = false;
-                            break;
-                        }
-                        tc_fence_after();
-                        issue_acc(s, prev_st, i > 1);
-                    }
-                    if (i < U.n_items) {
-                        const uint32_t t0 = tmem + s * C::kColStream;
-                        const uint32_t a_base =
-                            smem_u32(abuf + ab * C::kABytes + s * C::kNA * C::kATile);
-                        const uint32_t i_base = smem_u32(ring + st * C::kStage);
-#pragma unroll
-                        for (int t = 0; t < C::kNA; ++t) {
-#pragma unroll
-                            for (int k = 0; k < D / 16; ++k) {
-                                const uint64_t ad =
-                                    smem_desc(a_base + t * C::kATile + 32 * k, 16, C::kSBO, C::kSwz);
-                                const uint64_t bd = smem_desc(i_base + t * C::kItemTile + 32 * k, 16,
-                                                              C::kSBO, C::kSwz);
-                                if (elect_one())
-                                    mma_ss(t0 + t * C::kItem, ad, bd, C::kIdescS, k > 0 ? 1u : 0u);
-                                __syncwarp();
-                            }
-                        }
-                        if (elect_one()) mma_commit(sready0 + 8u * s);
-                        __syncwarp();
-                    } else {
-                        if (elect_one()) mma_commit(accdone0 + 8u * s);
-                        __syncwarp();
-                        ++nu[s];
-                    }
-                }
-                if (!ok) break;
                 if (i > 0) {
-                    if (elect_one()) mma_commit(empty0 + 8u * prev_st);  // item i - 1 consumed
-                    __syncwarp();
+                    // dS / P of item i - 1 written: its accumulating products
+                    if (!wait(pready0 + 8u * s, pj & 1)) {
+                        ok = false;
+                        break;
+                    }
+                    ++pj;
+                    if (i == 1 && nu > 0 && !wait(accfree0 + 8u * s, (nu - 1) & 1)) {
+                        ok = false;
+                        break;
+                    }
                 }
+                tc_fence_after();
+                if (i > 0) issue_acc(prev_st, i > 1);
                 if (i < U.n_items) {
+                    const uint32_t i_base = smem_u32(ring + st * C::kStage);
+#pragma unroll
+                    for (int t = 0; t < C::kNA; ++t) {
+#pragma unroll
+                        for (int k = 0; k < D / 16; ++k) {
+                            const uint64_t ad =
+                                smem_desc(a_base + t * C::kATile + 32 * k, 16, C::kSBO, C::kSwz);
+                            const uint64_t bd =
+                                smem_desc(i_base + t * C::kItemTile + 32 * k, 16, C::kSBO, C::kSwz);
+                            if (elect_one())
+                                mma_ss(t0 + t * C::kItem, ad, bd, C::kIdescS, k > 0 ? 1u : 0u);
+                            __syncwarp();
+                        }
+                    }
+                    if (elect_one()) mma_commit(sready0 + 8u * s);
+                    __syncwarp();
                     prev_st = st;
                     ++it;
+                } else {
+                    if (elect_one()) {
+                        mma_commit(accdone0 + 8u * s);
+                        mma_commit(afree0 + 8u * ab);
+                    }
+                    __syncwarp();
+                    ++nu;
                 }
             }
-            if (!ok) break;
-            if (elect_one()) mma_commit(afree0 + 8u * ab);
-            __syncwarp();
         }
         // every product issued has completed before TMEM is released
-        if (elect_one()) mma_commit(fin);
+        if (elect_one()) mma_commit(fin0 + 8u * s);
         __syncwarp();
-        const uint64_t t0 = globaltimer_ns();
-        while (!__all_sync(0xffffffffu, mbar_try_wait(fin, 0)) &&
-               globaltimer_ns() - t0 < kWaitLimitNs) {
+        const uint64_t tw = globaltimer_ns();
+        while (!__all_sync(0xffffffffu, mbar_try_wait(fin0 + 8u * s, 0)) &&
+               globaltimer_ns() - tw < kWaitLimitNs) {
         }
-    } else if (warp >= kFirstSoftmaxWarp) {
+    } else if (warp >= kFirstSoftmaxWarp && warp < kFirstSoftmaxWarp + 4 * NS) {
         // ------------------------------------------------------------ softmax warpgroups
         const int s = (warp - kFirstSoftmaxWarp) / 4;
         const int q = warp % 4;  // TMEM lane quadrant of this warp
         const int r = 32 * q + lane;
+        const bool leader = q == 0 && lane == 0;
         const uint32_t t0 = tmem + ((uint32_t)(32 * q) << 16) + s * C::kColStream;
-        const float c = prm.c;
+        const uint64_t c2 = pack_f32x2(prm.c, prm.c);
         uint32_t it = 0, sj = 0, na = 0;
         bool ok = true;
         for (int64_t u = blockIdx.x; u < prm.n_units && ok; u += gridDim.x) {
@@ -502,6 +554,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                 Lr = prm.Lrow[U.bh * U.rows + row];
                 cr = prm.crow[U.bh * U.rows + row];
             }
+            const uint64_t nLr2 = pack_f32x2(-Lr, -Lr), ncr2 = pack_f32x2(-cr, -cr);
             for (int i = 0; i < U.n_items; ++i, ++it) {
                 const int st = it % C::kStages;
                 if (!warp_wait(sready0 + 8u * s, sj & 1, abort_flag, prm.status)) {
@@ -509,18 +562,27 @@ __global__ void __launch_bounds__(kThreads, 1)
                     break;
                 }
                 ++sj;
+                // S of item i complete: every product of item i - 1 is, so its stage is free
+                if (i > 0 && leader) mbar_arrive(empty0 + 8u * ((it - 1) % C::kStages));
                 if (C::kColStats &&
                     !warp_wait(full0 + 8u * st, (it / C::kStages) & 1, abort_flag, prm.status)) {
                     ok = false;
                     break;
                 }
                 tc_fence_after();
-                const int nv = (int)min((int64_t)C::kItem, U.item_end - (U.item0 + (int64_t)i * C::kItem));
-                const float* Lc = stats + st * 2 * C::kItem;
-                const float* cc = Lc + C::kItem;
+                const int nv =
+                    (int)min((int64_t)C::kItem, U.item_end - (U.item0 + (int64_t)i * C::kItem));
+                const float* nLc = stats + st * 2 * C::kItem;
+                const float* ncc = nLc + C::kItem;
+                if (nv == C::kItem) {
 #pragma unroll
-                for (int h = 0; h < C::kItem / 32; ++h)
-                    bwd_slice<D, PASS>(t0, h, nv, c, Lr, cr, Lc, cc);
+                    for (int h = 0; h < C::kItem / 16; ++h)
+                        bwd_slice<D, PASS, true>(t0, h, nv, c2, nLr2, ncr2, nLc, ncc);
+                } else {
+#pragma unroll
+                    for (int h = 0; h < C::kItem / 16; ++h)
+                        bwd_slice<D, PASS, false>(t0, h, nv, c2, nLr2, ncr2, nLc, ncc);
+                }
                 tmem_wait_st();
                 tc_fence_before();
                 mbar_arrive(pready0 + 8u * s);
@@ -532,6 +594,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                 break;
             }
             ++na;
+            if (leader) mbar_arrive(empty0 + 8u * ((it - 1) % C::kStages));
             tc_fence_after();
             float a0[D], a1[C::kNAcc == 2 ? D : 1];
             const uint32_t acc = t0 + C::kNA * C::kItem;
@@ -590,7 +653,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
-    if (warp == 1) tmem_dealloc(tmem, kTmemCols);
+    if (warp == 0) tmem_dealloc(tmem, kTmemCols);
 }
 
 // ------------------------------------------------------------------ host side
@@ -627,54 +690,58 @@ bool make_map(CUtensorMap* m, const void* base, int64_t D, int64_t rows, int64_t
 }
 
 template <int D, int PASS>
-cudaError_t launch_pass(const CUtensorMap* maps, const BwdParams& prm, cudaStream_t st) {
+cudaError_t launch_pass(const void* const* srcs, const Plan& p, BwdParams prm, cudaStream_t st) {
     using Cf = BCfg<D, PASS>;
     static cudaError_t attr = cudaFuncSetAttribute(
         tc_bwd_kernel<D, PASS>, cudaFuncAttributeMaxDynamicSharedMemorySize, Cf::kSmem);
     if (attr != cudaSuccess) return attr;
+    if (Cf::kRouteRows) {
+        prm.n_groups = (prm.M + Cf::kGroup - 1) / Cf::kGroup;
+        prm.n_units = prm.BH * prm.n_groups * prm.nchunk;
+    } else {
+        prm.n_groups = (prm.N + Cf::kGroup - 1) / Cf::kGroup;
+        prm.n_units = prm.BH * prm.n_groups;
+    }
     if (prm.n_units == 0) return cudaSuccess;
+    if (Cf::kRouteRows && prm.chunk_len % Cf::kItem != 0) return cudaErrorInvalidValue;
+    // A tiles: 128 rows of the pass's row dimension; items: kItem rows of the other one
+    const int64_t arows = Cf::kRouteRows ? p.M : p.N;
+    const int64_t irows = Cf::kRouteRows ? p.N : p.M;
+    CUtensorMap maps[6];
+    for (int k = 0; k < 6; ++k) {
+        const bool used = (k % 3) < Cf::kNA;
+        const void* base = used ? srcs[k] : srcs[k - 2];
+        const bool a_side = k < 3;
+        const bool per_head = a_side ? (prm.a0_per_head && k == 0) : (prm.i0_per_head && k == 3);
+        if (!make_map(&maps[k], base, p.D, a_side ? arows : irows, per_head ? p.H : p.BH,
+                      a_side ? (uint32_t)kRows : (uint32_t)Cf::kItem))
+            return cudaErrorInvalidValue;
+    }
     int dev = 0, sms = kNumSMs;
     cudaGetDevice(&dev);
     cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
     const int64_t grid = prm.n_units < sms ? prm.n_units : sms;
-    tc_bwd_kernel<D, PASS><<<(unsigned)grid, kThreads, Cf::kSmem, st>>>(
+    tc_bwd_kernel<D, PASS><<<(unsigned)grid, Cf::kThreads, Cf::kSmem, st>>>(
         maps[0], maps[1], maps[2], maps[3], maps[4], maps[5], prm);
     return cudaGetLastError();
 }
 
 template <int PASS>
-cudaError_t launch_d(int64_t D, const CUtensorMap* maps, const BwdParams& prm, cudaStream_t st) {
-    switch (D) {
-        case 16: return launch_pass<16, PASS>(maps, prm, st);
-        case 32: return launch_pass<32, PASS>(maps, prm, st);
-        case 64: return launch_pass<64, PASS>(maps, prm, st);
+cudaError_t launch_d(const void* const* srcs, const Plan& p, const BwdParams& prm,
+                     cudaStream_t st) {
+    switch (p.D) {
+        case 16: return launch_pass<16, PASS>(srcs, p, prm, st);
+        case 32: return launch_pass<32, PASS>(srcs, p, prm, st);
+        case 64: return launch_pass<64, PASS>(srcs, p, prm, st);
         default: return cudaErrorInvalidValue;
     }
 }
 
 }  // namespace
 
-int64_t tc_bwd_item(int64_t D) { return D == 64 ? 32 : 64; }
-
 cudaError_t tc_bwd_pass(const Plan& p, const BwdPlan& bp, int pass, const TcBwdOperands& o,
                         float scale, int* status, cudaStream_t st) {
-    const int64_t item = tc_bwd_item(p.D);
-    const bool route_rows = pass <= kR1;
-    // A tiles: 128 rows of the pass's row dimension; items: `item` rows of the other one
-    const int64_t arows = route_rows ? p.M : p.N;
-    const int64_t irows = route_rows ? p.N : p.M;
-    CUtensorMap maps[6];
     const void* srcs[6] = {o.a[0], o.a[1], o.a[2], o.i[0], o.i[1], o.i[2]};
-    const int nmaps = pass == kT23 ? 3 : 2;
-    for (int k = 0; k < 6; ++k) {
-        const bool used = (k % 3) < nmaps;
-        const void* base = used ? srcs[k] : srcs[k % 3 == 2 ? k - 2 : k];
-        const bool a_side = k < 3;
-        const bool per_head = a_side ? (pass == kR1 && k == 0) : (pass == kT1 && k == 3);
-        if (!make_map(&maps[k], base, p.D, a_side ? arows : irows, per_head ? p.H : p.BH,
-                      a_side ? kRows : (uint32_t)item))
-            return cudaErrorInvalidValue;
-    }
     BwdParams prm{};
     prm.BH = p.BH;
     prm.H = p.H;
@@ -686,9 +753,6 @@ cudaError_t tc_bwd_pass(const Plan& p, const BwdPlan& bp, int pass, const TcBwdO
     prm.i0_per_head = pass == kT1 ? 1 : 0;
     prm.chunk_len = bp.chunk_len;
     prm.nchunk = bp.nchunk;
-    prm.n_groups = (p.M + NS * kRows - 1) / (NS * kRows);
-    prm.n_tok_groups = (p.N + NS * kRows - 1) / (NS * kRows);
-    prm.n_units = route_rows ? p.BH * prm.n_groups * bp.nchunk : p.BH * prm.n_tok_groups;
     prm.Lrow = o.Lrow;
     prm.crow = o.crow;
     prm.Lcol = o.Lcol;
@@ -699,11 +763,11 @@ cudaError_t tc_bwd_pass(const Plan& p, const BwdPlan& bp, int pass, const TcBwdO
     prm.out1 = (__nv_bfloat16*)o.out1;
     prm.status = status;
     switch (pass) {
-        case kR3: return launch_d<kR3>(p.D, maps, prm, st);
-        case kR2: return launch_d<kR2>(p.D, maps, prm, st);
-        case kR1: return launch_d<kR1>(p.D, maps, prm, st);
-        case kT23: return launch_d<kT23>(p.D, maps, prm, st);
-        case kT1: return launch_d<kT1>(p.D, maps, prm, st);
+        case kR3: return launch_d<kR3>(srcs, p, prm, st);
+        case kR2: return launch_d<kR2>(srcs, p, prm, st);
+        case kR1: return launch_d<kR1>(srcs, p, prm, st);
+        case kT23: return launch_d<kT23>(srcs, p, prm, st);
+        case kT1: return launch_d<kT1>(srcs, p, prm, st);
         default: return cudaErrorInvalidValue;
     }
 }
