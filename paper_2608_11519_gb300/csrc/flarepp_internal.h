@@ -54,7 +54,7 @@ SavedLayout saved_layout(const Plan& p);
 // The backward's plan: the split-N route passes (chunks of tokens) and its workspace. On
 // the CUDA-core path a route pass gives one thread per route (m_tile routes per CTA); on
 // the tensor-core path a work unit is a group of up to 512 routes and a chunk of tokens,
-// and chunk_len is a multiple of 64 tokens (whole items of either size).
+// and chunk_len is a multiple of 192 tokens (whole items of every size: 32, 48, 64).
 struct BwdPlan {
     int path;                   // kPathSimt or kPathTc
     int64_t m_tile, n_mtiles;   // CUDA-core route passes: routes per CTA, route tiles per head

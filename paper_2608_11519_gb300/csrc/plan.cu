@@ -140,8 +140,8 @@ BwdPlan make_bwd_plan(const Plan& p) {
     b.n_mtiles = cdiv(p.M, b.m_tile);
     if (p.path == kPathTc) {
         // work units (b*h, route group of up to 512, chunk): about two waves of persistent
-        // CTAs; chunks are whole items (64 tokens covers both item sizes)
-        const int64_t item = 64;
+        // CTAs; chunks are whole items (192 tokens is a multiple of every item size)
+        const int64_t item = 192;
         const int64_t groups = cdiv(p.M, 512);
         int64_t want = cdiv(2 * kNumSMs, p.BH * groups);
         if (want < 1) want = 1;

@@ -60,15 +60,20 @@ struct BCfg {
     static constexpr int kNAcc = (PASS == kR2 || PASS == kR1) ? 1 : 2;
     static constexpr bool kColStats = PASS == kR3 || PASS == kT23 || PASS == kT1;
     static constexpr bool kRowStats = PASS == kR2 || PASS == kR1 || PASS == kT23;
-    // TMEM per stream: kNA score tiles of kItem columns, then kNAcc accumulators of D.
-    // Items of 64 rows when three streams fit with them, else 32; as many streams as fit
-    // in 512 columns, at most four.
+    // TMEM per stream: kNA score tiles of kItem columns, then kNAcc accumulators of D. The
+    // most streams (at most four) that fit in 512 columns, with the widest item of 64, 48 or
+    // 32 rows for that count: four streams make a 512-row group, so M = 512 fills every unit.
     static constexpr uint32_t col_stream(int item) { return kNA * item + kNAcc * D; }
-    static constexpr int kItem = 3 * col_stream(64) <= kTmemCols ? 64 : 32;
-    static constexpr uint32_t kColStream = col_stream(kItem);
-    static constexpr int kFit = (int)(kTmemCols / kColStream);
-    static constexpr int NS = kFit > 4 ? 4 : kFit;
+    static constexpr int fits(int ns, int item) { return ns * col_stream(item) <= kTmemCols; }
+    static constexpr int pick_ns() {
+        for (int ns = 4; ns >= 1; --ns)
+            if (fits(ns, 32)) return ns;
+        return 0;
+    }
+    static constexpr int NS = pick_ns();
     static_assert(NS >= 1, "TMEM budget");
+    static constexpr int kItem = fits(NS, 64) ? 64 : (fits(NS, 48) ? 48 : 32);
+    static constexpr uint32_t kColStream = col_stream(kItem);
     // warps 0..NS-1 issue MMAs (one per stream), warps 4.. are the softmax warpgroups, and
     // the TMA producer is warp 3 (NS < 4) or the warp after the softmax warps (NS = 4)
     static constexpr int kProdWarp = NS < 4 ? 3 : kFirstSoftmaxWarp + 4 * NS;
