@@ -66,6 +66,10 @@ struct BCfg {
     static constexpr uint32_t col_stream(int item) { return kNA * item + kNAcc * D; }
     static constexpr int fits(int ns, int item) { return ns * col_stream(item) <= kTmemCols; }
     static constexpr int pick_ns() {
+        // T23 (three score products, 6 ss MMAs per item): two streams of 64-row items
+        // measured faster than three of 32 (3.41 vs 3.60 ms at mesh3d); for R3 and T1 the
+        // most streams win (two of 64 rows: 3.67 vs 2.12 ms; three of 48: 2.38 vs 2.17 ms)
+        if (PASS == kT23 && fits(2, 64)) return 2;
         for (int ns = 4; ns >= 1; --ns)
             if (fits(ns, 32)) return ns;
         return 0;
