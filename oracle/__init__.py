@@ -12,6 +12,9 @@ What it computes (FLARE++ paper):
                           shared by the batch (Sec. 3, eq. prelim_flare_sdpa)
   * ``encode_sharded`` -- the encoder evaluated shard by shard, then merged by the stable
                           log-sum-exp reduction (App. A.2, A.3)
+  * ``mixer``          -- the FLARE++ token-mixing layer (Fig. 1; eqs. flarepp_query_synthesis
+                          and flarepp_mixer): K, V, K~, V~ = X W^T split into heads, the routing
+                          chain, then O = merge(Y) Wo^T; the projections are numpy matmuls
   * ``sdpa_bwd``       -- the backward of one SDPA from its saved output and log-normaliser
                           (App. A.5): P = exp(S - L), c = <dO, O>, dV = P^T dO,
                           dS = P o (dO V^T - c), dK = s dS^T Q, dQ = s dS K
@@ -128,6 +131,28 @@ class Oracle:
         Y, _ = self.sdpa(K, Qb, Z, scale)
         return Z, Y
 
+    def mixer(self, X, W_in, Wo, seeds, scale):
+        """The FLARE++ mixer (Fig. 1): X [B, N, C]; W_in [P*C, C] in the out x in layout, its
+        row blocks the projections of K, V, K~, V~ (P = 4; P = 2 ties K~, V~ to K, V, the
+        shared-projection variant of App. C.2); Wo [C, C] (out x in); seeds [H, M, D] with
+        C = H * D. Returns O [B, N, C]."""
+        X, W_in, Wo, seeds = (self._f64(a) for a in (X, W_in, Wo, seeds))
+        B, N, C = X.shape
+        H, M, D = seeds.shape
+        assert H * D == C and W_in.shape[1] == C and W_in.shape[0] in (2 * C, 4 * C)
+        assert Wo.shape == (C, C)
+        proj = X @ W_in.T  # [B, N, P*C]: the pointwise projections of eq. flarepp_mixer
+
+        def heads(i):  # block i of the projection, split into H heads of width D
+            blk = proj[..., i * C:(i + 1) * C].reshape(B, N, H, D)
+            return np.ascontiguousarray(blk.transpose(0, 2, 1, 3))
+
+        K, V = heads(0), heads(1)
+        Kt, Vt = (heads(2), heads(3)) if W_in.shape[0] == 4 * C else (K, V)
+        _, _, Y = self.route(seeds, Kt, Vt, K, V, scale)
+        merged = Y.transpose(0, 2, 1, 3).reshape(B, N, C)  # merge(Y): heads side by side
+        return merged @ Wo.T
+
     def sdpa_bwd(self, q, k, v, out, lse, dout, scale):
         """Backward of ``sdpa`` (App. A.5) from the forward's ``out`` and ``lse``.
 
@@ -217,6 +242,10 @@ def encode_sharded(q, k, v, scale, chunk, n_empty=0):
     return default().encode_sharded(q, k, v, scale, chunk, n_empty)
 
 
+def mixer(X, W_in, Wo, seeds, scale):
+    return default().mixer(X, W_in, Wo, seeds, scale)
+
+
 def sdpa_bwd(q, k, v, out, lse, dout, scale):
     return default().sdpa_bwd(q, k, v, out, lse, dout, scale)
 
@@ -238,5 +267,5 @@ def build() -> str:
     return _build.build()
 
 
-__all__ = ["Oracle", "default", "sdpa", "route", "flare", "encode_sharded", "sdpa_bwd",
-           "route_bwd", "max_threads", "set_threads", "build"]
+__all__ = ["Oracle", "default", "sdpa", "route", "flare", "encode_sharded", "mixer",
+           "sdpa_bwd", "route_bwd", "max_threads", "set_threads", "build"]
