@@ -199,6 +199,31 @@ FLAREPP_API flarepp_status flarepp_route_fwd_noalloc(const flarepp_shape* shape,
                                                      void* stream);
 
 /*
+ * The FLARE++ token-mixing layer (Fig. 1; eqs. flarepp_query_synthesis, flarepp_mixer): the
+ * pointwise projections K, V, K~, V~ = X W_in^T (split into H heads of width D, C = H * D),
+ * the routing chain, and O = merge(Y) Wo^T, where merge places the heads side by side.
+ *   shape: B, H, N (tokens), M (routes), D and dtype; bf16 only (FLAREPP_ERR_UNSUPPORTED for
+ *     float32).
+ *   n_proj: 4 (K, V, K~, V~) or 2 (K, V; the shared-projection variant of App. C.2, which
+ *     uses K, V as K~, V~).
+ *   X: [B, N, C]; W_in: [n_proj * C, C], out x in (row block 0 is W_K, then W_V, W_K~, W_V~);
+ *     Wo: [C, C], out x in; seeds: [H, M, D]; O: [B, N, C]. Device pointers, 16-byte
+ *     aligned; O must not overlap an input or the workspace. No biases.
+ *   workspace: flarepp_mixer_workspace_bytes(shape, n_proj) bytes, 256-byte aligned; it holds
+ *     the chain's workspace (its status word at offset 0, read by
+ *     flarepp_route_device_status), the projections and Y.
+ * Degenerate shapes: N or B*H zero leave O (empty) alone; M = 0 writes O = 0.
+ * Errors: FLAREPP_ERR_INVALID_ARGUMENT, FLAREPP_ERR_UNSUPPORTED, FLAREPP_ERR_WORKSPACE,
+ * FLAREPP_ERR_CUDA, as for flarepp_route_fwd. Enqueued on `stream`.
+ */
+FLAREPP_API size_t flarepp_mixer_workspace_bytes(const flarepp_shape* shape, int n_proj);
+FLAREPP_API flarepp_status flarepp_mixer_fwd(const flarepp_shape* shape, int n_proj,
+                                             const void* X, const void* W_in, const void* Wo,
+                                             const void* seeds, float scale, void* O,
+                                             void* workspace, size_t workspace_bytes,
+                                             void* stream);
+
+/*
  * Bytes of the state a training forward keeps for the backward (App. A.5): float32 Q and Z
  * [B, H, M, D] and the base-2 log-normalisers of the three calls,
  * L = log2 sum_j 2^(scale * log2(e) <a, b_j>), for calls 1 and 2 [B, H, M] and call 3

@@ -453,10 +453,99 @@ flarepp_status route_bwd_impl(const flarepp_shape* shape, const void* seeds, con
     return e == cudaSuccess ? FLAREPP_OK : FLAREPP_ERR_CUDA;
 }
 
+// ---------------------------------------------------------------- the mixer layer
+
+// Workspace of flarepp_mixer_fwd: the chain's workspace first (its status word at offset 0),
+// then the projections (K, V and, for four projections, K~, V~) and Y, each [B][H][N][D] bf16.
+struct MixerLayout {
+    size_t off_proj[4], off_y, total;
+};
+
+bool mixer_layout(const Plan& p, int n_proj, MixerLayout* L) {
+    const size_t tok = (size_t)p.BH * (size_t)p.N * (size_t)p.D * 2;
+    size_t off = align_up(p.total, kWsAlign);
+    for (int i = 0; i < 4; ++i) {
+        L->off_proj[i] = off;
+        if (i < n_proj) off = align_up(off + tok, kWsAlign);
+    }
+    L->off_y = off;
+    off = align_up(off + tok, kWsAlign);
+    L->total = off;
+    return true;
+}
+
+flarepp_status mixer_impl(const flarepp_shape* shape, int n_proj, const void* X, const void* W_in,
+                          const void* Wo, const void* seeds, float scale, void* O,
+                          void* workspace, size_t workspace_bytes, void* stream) {
+    Plan p;
+    flarepp_status stt = make_plan(shape, &p);
+    if (stt != FLAREPP_OK) return stt;
+    if (n_proj != 2 && n_proj != 4) return FLAREPP_ERR_INVALID_ARGUMENT;
+    if (p.dtype != FLAREPP_BF16) return FLAREPP_ERR_UNSUPPORTED;  // tensor-core GEMMs only
+    if (!isfinite(scale)) return FLAREPP_ERR_INVALID_ARGUMENT;
+    cudaStream_t st = (cudaStream_t)stream;
+    const int64_t C = p.H * p.D;
+    const size_t x_bytes = (size_t)p.B * (size_t)p.N * (size_t)C * 2;
+    const size_t w_bytes = (size_t)n_proj * (size_t)C * (size_t)C * 2;
+    const size_t wo_bytes = (size_t)C * (size_t)C * 2;
+    const size_t seed_bytes = (size_t)p.H * (size_t)p.M * (size_t)p.D * 2;
+    if (x_bytes) {
+        const void* ptrs[4] = {X, W_in, Wo, O};
+        for (const void* q : ptrs)
+            if (!q || !aligned16(q)) return FLAREPP_ERR_INVALID_ARGUMENT;
+        if (overlaps(O, x_bytes, X, x_bytes) || overlaps(O, x_bytes, W_in, w_bytes) ||
+            overlaps(O, x_bytes, Wo, wo_bytes) || overlaps(O, x_bytes, seeds, seed_bytes))
+            return FLAREPP_ERR_INVALID_ARGUMENT;
+        if (seed_bytes && (!seeds || !aligned16(seeds))) return FLAREPP_ERR_INVALID_ARGUMENT;
+    }
+    MixerLayout L;
+    mixer_layout(p, n_proj, &L);
+    if (p.BH == 0 || p.N == 0) return FLAREPP_OK;  // O is empty
+    if (!workspace || ((uintptr_t)workspace % kWsAlign) != 0 || workspace_bytes < L.total)
+        return FLAREPP_ERR_WORKSPACE;
+    if (overlaps(O, x_bytes, workspace, L.total)) return FLAREPP_ERR_INVALID_ARGUMENT;
+    if (p.M == 0)  // every decode row has no keys: Y = 0, so O = 0
+        return cudaMemsetAsync(O, 0, x_bytes, st) == cudaSuccess ? FLAREPP_OK : FLAREPP_ERR_CUDA;
+    char* ws = (char*)workspace;
+    int* status = (int*)(ws + p.off_status);
+    if (cudaMemsetAsync(status, 0, sizeof(int32_t), st) != cudaSuccess) return FLAREPP_ERR_CUDA;
+    void* proj[4];
+    for (int i = 0; i < 4; ++i) proj[i] = ws + L.off_proj[i < n_proj ? i : i - 2];
+    // K, V, K~, V~ = X W_in^T, split into heads (eqs. flarepp_query_synthesis, flarepp_mixer)
+    if (tc_projection(p.B, p.N, p.H, p.D, n_proj, X, W_in, proj, status, st) != cudaSuccess)
+        return FLAREPP_ERR_CUDA;
+    // the routing chain; the shared variant reads K, V as K~, V~ (App. C.2)
+    void* Y = ws + L.off_y;
+    stt = route_impl(shape, seeds, proj[2], proj[3], proj[0], proj[1], scale, Y, workspace,
+                     p.total, stream, nullptr, nullptr, nullptr, 0, false);
+    if (stt != FLAREPP_OK) return stt;
+    // O = merge(Y) Wo^T
+    if (tc_output_projection(p.B, p.N, p.H, p.D, Y, Wo, O, status, st) != cudaSuccess)
+        return FLAREPP_ERR_CUDA;
+    return FLAREPP_OK;
+}
+
 }  // namespace
 }  // namespace flarepp
 
 extern "C" {
+
+size_t flarepp_mixer_workspace_bytes(const flarepp_shape* shape, int n_proj) {
+    flarepp::Plan p;
+    if (flarepp::make_plan(shape, &p) != FLAREPP_OK) return 0;
+    if ((n_proj != 2 && n_proj != 4) || p.dtype != FLAREPP_BF16) return 0;
+    if (p.BH == 0 || p.N == 0) return 0;
+    flarepp::MixerLayout L;
+    flarepp::mixer_layout(p, n_proj, &L);
+    return L.total;
+}
+
+flarepp_status flarepp_mixer_fwd(const flarepp_shape* shape, int n_proj, const void* X,
+                                 const void* W_in, const void* Wo, const void* seeds, float scale,
+                                 void* O, void* workspace, size_t workspace_bytes, void* stream) {
+    return flarepp::mixer_impl(shape, n_proj, X, W_in, Wo, seeds, scale, O, workspace,
+                               workspace_bytes, stream);
+}
 
 size_t flarepp_route_saved_bytes(const flarepp_shape* shape) {
     flarepp::Plan p;

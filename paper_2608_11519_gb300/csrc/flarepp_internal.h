@@ -118,6 +118,15 @@ struct TcBwdOperands {
 cudaError_t tc_bwd_pass(const Plan& p, const BwdPlan& bp, int pass, const TcBwdOperands& o,
                         float scale, int* status, cudaStream_t st);
 
+// ---- the mixer's pointwise projections (tc_gemm.cu), bf16
+// X [B][N][C] times W_in [P*C][C] (out x in) into the P tensors outs[p] [B][H][N][D]
+// (C = H * D; P = 4: K, V, K~, V~; P = 2: K, V).
+cudaError_t tc_projection(int64_t B, int64_t N, int64_t H, int64_t D, int P, const void* X,
+                          const void* W_in, void* const* outs, int* status, cudaStream_t st);
+// merge(Y) times Wo [C][C] (out x in) into O [B][N][C], Y read head by head [B][H][N][D].
+cudaError_t tc_output_projection(int64_t B, int64_t N, int64_t H, int64_t D, const void* Y,
+                                 const void* Wo, void* O, int* status, cudaStream_t st);
+
 // ---- tensor-core kernels (tc_kernels.cu), bf16 inputs
 // Encode call 1 (A = seeds) or call 2 (A = Q operand) into the chunk partials.
 cudaError_t tc_encode(const Plan& p, int call, const void* k, const void* v, const void* seeds,

@@ -24,6 +24,7 @@ _DTYPES = {torch.float32: F32, torch.bfloat16: BF16}
 EXPORTED = ("flarepp_route_workspace_bytes", "flarepp_route_fwd", "flarepp_route_fwd_debug",
             "flarepp_route_fwd_profiled", "flarepp_route_fwd_noalloc",
             "flarepp_flare_fwd", "flarepp_route_host_buffer_bytes", "flarepp_route_fwd_host",
+            "flarepp_mixer_workspace_bytes", "flarepp_mixer_fwd",
             "flarepp_route_saved_bytes", "flarepp_route_fwd_train",
             "flarepp_route_bwd_workspace_bytes", "flarepp_route_bwd",
             "flarepp_route_device_status", "flarepp_status_string", "flarepp_version")
@@ -80,6 +81,11 @@ def load(path: str = None):
     lib.flarepp_route_host_buffer_bytes.argtypes = [sp]
     lib.flarepp_route_fwd_host.restype = ctypes.c_int
     lib.flarepp_route_fwd_host.argtypes = [sp, vp, vp, vp, vp, vp, ctypes.c_float, vp, vp, sz, vp]
+    lib.flarepp_mixer_workspace_bytes.restype = sz
+    lib.flarepp_mixer_workspace_bytes.argtypes = [sp, ctypes.c_int]
+    lib.flarepp_mixer_fwd.restype = ctypes.c_int
+    lib.flarepp_mixer_fwd.argtypes = [sp, ctypes.c_int, vp, vp, vp, vp, ctypes.c_float, vp, vp,
+                                      sz, vp]
     lib.flarepp_route_saved_bytes.restype = sz
     lib.flarepp_route_saved_bytes.argtypes = [sp]
     lib.flarepp_route_fwd_train.restype = ctypes.c_int
@@ -306,6 +312,41 @@ def flare_fwd(Q, K, V, scale=None, Y=None, workspace=None, stream=None, Z_out=No
     if rc != OK:
         raise FlareppError(rc, "flarepp_flare_fwd")
     return Y
+
+
+def mixer_fwd(X, W_in, Wo, seeds, scale=None, O=None, workspace=None, stream=None):
+    """The FLARE++ mixer layer (Fig. 1) on device tensors: X [B, N, C], W_in [P*C, C] (P = 4:
+    K, V, K~, V~; P = 2: shared projection), Wo [C, C] (both out x in), seeds [H, M, D].
+    Returns O [B, N, C]."""
+    lib = load()
+    for t in (X, W_in, Wo, seeds):
+        if not isinstance(t, torch.Tensor) or not t.is_contiguous():
+            raise ValueError("inputs must be contiguous torch tensors")
+        if t.dtype != torch.bfloat16:
+            raise TypeError("the mixer takes bfloat16 tensors")
+    if X.device.type != "cuda":
+        raise ValueError("mixer_fwd takes device tensors")
+    B, N, C = X.shape
+    H, M, D = seeds.shape
+    if H * D != C or tuple(Wo.shape) != (C, C) or W_in.shape[1] != C or \
+            W_in.shape[0] not in (2 * C, 4 * C):
+        raise ValueError("expected X [B,N,C], W_in [P*C,C], Wo [C,C], seeds [H,M,D], C = H*D")
+    P = W_in.shape[0] // C
+    shape = make_shape(B, H, N, M, D, torch.bfloat16)
+    if scale is None:
+        scale = 1.0 / math.sqrt(D)
+    if O is None:
+        O = torch.empty_like(X)
+    nbytes = int(lib.flarepp_mixer_workspace_bytes(ctypes.byref(shape), P))
+    ws = (workspace if isinstance(workspace, Workspace) else Workspace()).get(nbytes, X.device)
+    st = stream if stream is not None else torch.cuda.current_stream(X.device)
+    rc = lib.flarepp_mixer_fwd(ctypes.byref(shape), P, _ptr(X), _ptr(W_in), _ptr(Wo),
+                               _ptr(seeds), float(scale), _ptr(O),
+                               None if ws is None else ctypes.c_void_p(ws.data_ptr()), nbytes,
+                               ctypes.c_void_p(st.cuda_stream))
+    if rc != OK:
+        raise FlareppError(rc, "flarepp_mixer_fwd")
+    return O
 
 
 def route_fwd_train(seeds, Kt, Vt, K, V, scale=None, Y=None, saved=None, workspace=None,

@@ -217,3 +217,35 @@ def test_backward_entry_sizes_and_rejects_before_any_cuda_call(lib):
     assert fw(None, sb(S())) == E.ERR_INVALID_ARGUMENT
     assert fw(base[7], 16) == E.ERR_INVALID_ARGUMENT
     assert fw(base[1] + 32, sb(S())) == E.ERR_INVALID_ARGUMENT  # overlaps Kt
+
+
+def test_mixer_entry_sizes_and_rejects(lib):
+    E = flarepp
+    wb = lambda s, p: lib.flarepp_mixer_workspace_bytes(ctypes.byref(s), p)
+    s = S(B=1, H=8, N=4096, M=64, D=32)
+    tok = 8 * 4096 * 32 * 2
+    assert wb(s, 4) >= 5 * tok and wb(s, 2) >= 3 * tok and wb(s, 4) > wb(s, 2)
+    assert wb(s, 3) == 0 and wb(S(dtype=flarepp.F32), 4) == 0 and wb(S(N=0), 4) == 0
+    v = lambda x: ctypes.c_void_p(x)
+    ptr = [FAKE + (i + 1) * (1 << 36) for i in range(6)]
+
+    def call(shape, n_proj=4, scale=0.25, ptrs=None):
+        p = ptr if ptrs is None else ptrs
+        return lib.flarepp_mixer_fwd(ctypes.byref(shape), n_proj, *(v(x) if x else None
+                                                                    for x in p[:4]),
+                                     ctypes.c_float(scale), v(p[4]) if p[4] else None,
+                                     v(p[5]) if p[5] else None, wb(shape, n_proj), None)
+
+    assert call(S(dtype=flarepp.F32)) == E.ERR_UNSUPPORTED
+    assert call(S(), n_proj=3) == E.ERR_INVALID_ARGUMENT
+    assert call(S(), scale=float("inf")) == E.ERR_INVALID_ARGUMENT
+    for i in range(5):
+        p = list(ptr)
+        p[i] = None
+        assert call(S(), ptrs=p) == E.ERR_INVALID_ARGUMENT, i
+    p = list(ptr)
+    p[4] = ptr[0] + 64  # O overlaps X
+    assert call(S(), ptrs=p) == E.ERR_INVALID_ARGUMENT
+    p = list(ptr)
+    p[5] = None
+    assert call(S(), ptrs=p) == E.ERR_WORKSPACE

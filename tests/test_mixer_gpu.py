@@ -1,0 +1,94 @@
+"""GPU parity of the FLARE++ mixer layer (Fig. 1: projections, chain, head merge, output
+projection) against the float64 oracle, through the C ABI.
+
+Tolerance: max|O - O_ref| <= 2e-2 * max(1, max|O_ref|) (bf16 inputs, float32 accumulation;
+the projections are stored in bf16 before the chain reads them, as the chain's own inputs are).
+With permutation weights every projection output is one input value (a sum with one nonzero
+term), so there the layer must equal the chain on the permuted copies bit for bit.
+"""
+import math
+
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from paper_2608_11519_gb300 import flarepp
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _lib():
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    flarepp.load()
+    torch.cuda.set_device(0)
+
+
+def _np(t):
+    return t.detach().to("cpu", torch.float64).numpy()
+
+
+def _case(B, H, N, M, D, P, seed):
+    g = torch.Generator().manual_seed(seed)
+    C = H * D
+    X = torch.randn(B, N, C, generator=g).to(torch.bfloat16)
+    W_in = (torch.randn(P * C, C, generator=g) / math.sqrt(C)).to(torch.bfloat16)
+    Wo = (torch.randn(C, C, generator=g) / math.sqrt(C)).to(torch.bfloat16)
+    seeds = torch.randn(H, M, D, generator=g).to(torch.bfloat16)
+    return X, W_in, Wo, seeds
+
+
+SHAPES = [
+    # B, H, N, M, D, P
+    (1, 8, 3000, 128, 32, 4),
+    (2, 2, 500, 64, 32, 4),
+    (2, 4, 300, 40, 16, 4),
+    (1, 2, 129, 20, 64, 4),
+    (1, 8, 1000, 96, 32, 2),
+    (3, 3, 200, 30, 16, 2),   # C = 48: 16-channel tiles
+]
+
+
+@pytest.mark.parametrize("shape", SHAPES, ids=[str(s) for s in SHAPES])
+def test_mixer_matches_oracle(shape):
+    B, H, N, M, D, P = shape
+    X, W_in, Wo, seeds = _case(B, H, N, M, D, P, 7)
+    s = 1.0 / math.sqrt(D)
+    O = flarepp.mixer_fwd(X.cuda(), W_in.cuda(), Wo.cuda(), seeds.cuda(), s)
+    torch.cuda.synchronize()
+    want = oracle.mixer(_np(X), _np(W_in), _np(Wo), _np(seeds), s)
+    got = _np(O)
+    bound = 2e-2 * max(1.0, float(np.abs(want).max()))
+    assert float(np.abs(got - want).max()) <= bound
+
+
+def test_mixer_with_permutation_weights_is_the_chain_exactly():
+    B, H, N, M, D = 2, 4, 700, 64, 32
+    C = H * D
+    g = torch.Generator().manual_seed(3)
+    X = torch.randn(B, N, C, generator=g).to(torch.bfloat16)
+    perms = [torch.randperm(C, generator=g) for _ in range(4)]
+    W_in = torch.cat([torch.eye(C)[p] for p in perms]).to(torch.bfloat16)
+    Wo = torch.eye(C).to(torch.bfloat16)
+    seeds = torch.randn(H, M, D, generator=g).to(torch.bfloat16)
+    s = 1.0 / math.sqrt(D)
+    O = flarepp.mixer_fwd(X.cuda(), W_in.cuda(), Wo.cuda(), seeds.cuda(), s)
+    split = lambda T: T.reshape(B, N, H, D).transpose(1, 2).contiguous().cuda()
+    K, V, Kt, Vt = (split(X[..., p]) for p in perms)
+    Y = flarepp.route_fwd(seeds.cuda(), Kt, Vt, K, V, s)
+    torch.cuda.synchronize()
+    merged = Y.transpose(1, 2).reshape(B, N, C)
+    assert torch.equal(O, merged)
+
+
+def test_mixer_degenerate_shapes():
+    X, W_in, Wo, seeds = _case(1, 2, 50, 0, 16, 4, 1)  # M = 0: Y = 0, so O = 0
+    O = torch.full_like(X, 3.0).cuda()
+    flarepp.mixer_fwd(X.cuda(), W_in.cuda(), Wo.cuda(), seeds.cuda(), O=O)
+    torch.cuda.synchronize()
+    assert not torch.any(O != 0)
+    X, W_in, Wo, seeds = _case(2, 2, 0, 8, 16, 4, 1)  # N = 0: nothing to do
+    O = flarepp.mixer_fwd(X.cuda(), W_in.cuda(), Wo.cuda(), seeds.cuda())
+    assert O.numel() == 0
