@@ -222,18 +222,30 @@ def run_reference(args, w):
         return 0
     import oracle
     n = int(min(w.N, args.ref_tokens))
-    x = inputs.make_inputs(w.with_(B=1, H=1, N=n), args.seed)
-    f = inputs.to_f64_numpy(x)
+    if args.variant.startswith("mixer"):
+        # the whole layer on one batch element: all H heads of n tokens
+        m = inputs.to_f64_numpy(inputs.make_mixer_inputs(
+            w.with_(B=1, N=n), args.seed, "cpu", 2 if args.variant == "mixer_shared" else 4))
+        step = lambda: oracle.mixer(m["X"], m["W_in"], m["Wo"], m["seeds"], w.scale)
+        heads = w.H
+        sample = (f"one batch element, N={n} tokens, H={w.H} heads of the {w.name} shape "
+                  f"(M={w.M}, D={w.D}), float64 oracle on the host cores, per step")
+    else:
+        x = inputs.make_inputs(w.with_(B=1, H=1, N=n), args.seed)
+        f = inputs.to_f64_numpy(x)
+        step = lambda: oracle_call(f, w, args.variant)
+        heads = 1
+        sample = (f"one head, N={n} tokens of the {w.name} shape (M={w.M}, D={w.D}), float64 "
+                  f"oracle on the host cores, per step")
     for _ in range(args.warmup):
-        oracle_call(f, w, args.variant)
+        step()
     t0 = time.perf_counter()
     for _ in range(args.steps):
-        oracle_call(f, w, args.variant)
+        step()
     dt = (time.perf_counter() - t0) / args.steps
-    value = n / dt
-    sample = (f"one head, N={n} tokens of the {w.name} shape (M={w.M}, D={w.D}), float64 oracle "
-              f"on the host cores, per step")
-    metric = {"flare": FLARE_METRIC, "train": TRAIN_METRIC}.get(args.variant, METRIC)
+    value = heads * n / dt
+    metric = {"flare": FLARE_METRIC, "train": TRAIN_METRIC, "mixer": MIXER_METRIC,
+              "mixer_shared": MIXER_METRIC}.get(args.variant, METRIC)
     line = {"impl": "reference", "metric": metric, "value": value, "unit": UNIT,
             "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
             "ms_per_step": dt * 1e3, "higher_is_better": True, "scaling": "weak",
@@ -462,6 +474,116 @@ def run_train(args, w, flarepp, world, rank, dev, peaks, x, Y, ws, stream):
     return 0
 
 
+MIXER_METRIC = ("routed tokens·heads/sec for the FLARE++ mixer layer (projections, 3-call chain, "
+                "output projection); % of roofline")
+
+
+def mixer_cpu_sample(w, target_s, seed, n_proj):
+    """The oracle's mixer on one batch element with a token prefix sized from a short probe."""
+    import oracle
+    probe_n = min(w.N, 2048)
+    x = inputs.to_f64_numpy(inputs.make_mixer_inputs(w.with_(B=1, N=probe_n), seed, "cpu", n_proj))
+    t0 = time.perf_counter()
+    oracle.mixer(x["X"], x["W_in"], x["Wo"], x["seeds"], w.scale)
+    probe = time.perf_counter() - t0
+    n = int(min(w.N, max(512, probe_n * target_s / max(probe, 1e-3))))
+    x = inputs.to_f64_numpy(inputs.make_mixer_inputs(w.with_(B=1, N=n), seed, "cpu", n_proj))
+    t0 = time.perf_counter()
+    oracle.mixer(x["X"], x["W_in"], x["Wo"], x["seeds"], w.scale)
+    dt = time.perf_counter() - t0
+    return {"value": w.H * n / dt, "unit": UNIT, "cores": oracle.max_threads(), "kind": "oracle",
+            "sample": f"one batch element, N={n} tokens of the {w.name} shape (H={w.H}, M={w.M}, "
+                      f"D={w.D}), float64, {dt:.2f} s"}
+
+
+def run_mixer(args, w, flarepp, world, rank, dev, peaks, stream):
+    """The FLARE++ mixer layer (Fig. 1) on device-resident inputs, each stage bracketed by the
+    library's own events."""
+    n_proj = 2 if args.variant == "mixer_shared" else 4
+    x = inputs.make_mixer_inputs(w, args.seed + rank, device=dev, n_proj=n_proj)
+    O = torch.empty_like(x["X"])
+    ws = flarepp.Workspace()
+    call = lambda ev=None: flarepp.mixer_fwd(x["X"], x["W_in"], x["Wo"], x["seeds"], w.scale,
+                                             O=O, workspace=ws, stream=stream, events=ev)
+    for _ in range(args.warmup):
+        call()
+    torch.cuda.synchronize(dev)
+    evs = [flarepp.MixerEvents(stream) for _ in range(args.steps)]
+    clocks = ClockSampler()
+    if rank == 0:
+        clocks.start()
+        time.sleep(0.3)
+    t0 = torch.cuda.Event(enable_timing=True)
+    t1 = torch.cuda.Event(enable_timing=True)
+    barrier(world)
+    torch.cuda.synchronize(dev)
+    t0.record(stream)
+    for i in range(args.steps):
+        call(evs[i])
+    t1.record(stream)
+    torch.cuda.synchronize(dev)
+    barrier(world)
+    clk = clocks.stop(dev.index) if rank == 0 else None
+    ms = max_over_ranks(t0.elapsed_time(t1), world) / args.steps
+    stage_ms = {s: 0.0 for s in flarepp.MIXER_STAGES}
+    for e in evs:
+        for s, v in e.stage_ms().items():
+            stage_ms[s] += v / args.steps
+    tok = w.B * w.H * w.N
+    BN, C = w.B * w.N, w.H * w.D
+    e = w.elt_bytes
+    # algorithmic work of each stage (the stages as built, each reading and writing HBM)
+    work = {
+        "projection": (2.0 * BN * C * n_proj * C, (1 + n_proj) * BN * C * e),
+        "chain": (12.0 * tok * w.M * w.D, (3 if n_proj == 2 else 5) * tok * w.D * e),
+        "output": (2.0 * BN * C * C, 2 * BN * C * e),
+    }
+    tc_peak = peaks["bf16_tflops_sustained"]
+    bw = peaks["hbm_gbs"]
+    roof_t = {s: max(f / (tc_peak * 1e12), b / (bw * 1e9)) for s, (f, b) in work.items()}
+    dominant = max(stage_ms, key=stage_ms.get)
+    f, b = work[dominant]
+    t_dom = stage_ms[dominant] * 1e-3
+    if f / (tc_peak * 1e12) >= b / (bw * 1e9):
+        roof = {"bound": "tensor", "achieved": f / t_dom / 1e12, "peak": tc_peak,
+                "unit": "TFLOP/s", "peak_kind": "bf16_tflops_sustained (" + peaks["source"] + ")"}
+    else:
+        roof = {"bound": "hbm", "achieved": b / t_dom / 1e9, "peak": bw, "unit": "GB/s",
+                "peak_kind": "hbm_gbs (" + peaks["source"] + ")"}
+    roof["frac"] = roof["achieved"] / roof["peak"]
+    roof["kernel"] = dominant
+    roof["ms_per_launch"] = stage_ms[dominant]
+    roof["algorithmic_flops_per_launch"] = f
+    roof["algorithmic_bytes_per_launch"] = b
+    roof["traffic"] = None
+    stage_frac = {s: roof_t[s] / (stage_ms[s] * 1e-3) for s in stage_ms}
+    layer = {"roofline_us": sum(roof_t.values()) * 1e6,
+             "frac": sum(roof_t.values()) / (ms * 1e-3),
+             "stage_frac": stage_frac,
+             "note": "sum of the stages' own rooflines (each stage streams its tensors through HBM)"}
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        cpu = mixer_cpu_sample(w, args.cpu_seconds, args.seed, n_proj)
+    if rank == 0:
+        line = {
+            "metric": MIXER_METRIC, "value": tok * world / (ms * 1e-3), "unit": UNIT,
+            "n_gpus": world, "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+            "dtype": "bf16", "data": "synthetic",
+            "config": {"workload": w.name, "variant": args.variant, "B": w.B, "H": w.H, "N": w.N,
+                       "M": w.M, "D": w.D, "C": C, "projections": n_proj,
+                       "l2": "inputs larger than L2 (no flush)",
+                       "parallelism": f"replicas x{world}"},
+            "stage_ms": stage_ms, "roofline": roof, "layer_roofline": layer,
+            "cpu_baseline": cpu, "e2e": None, "clocks": clk, "gpu_launches": 7 * args.steps,
+        }
+        print(json.dumps(line), flush=True)
+    if world > 1:
+        import torch.distributed as dist
+        dist.destroy_process_group()
+    return 0
+
+
 def run_ours(args, w):
     from paper_2608_11519_gb300 import flarepp
 
@@ -481,6 +603,9 @@ def run_ours(args, w):
         return run_flare(args, w, flarepp, world, rank, dev, peaks, x, Y, ws, stream)
     if args.variant == "train":
         return run_train(args, w, flarepp, world, rank, dev, peaks, x, Y, ws, stream)
+    if args.variant in ("mixer", "mixer_shared"):
+        del x, Y
+        return run_mixer(args, w, flarepp, world, rank, dev, peaks, stream)
 
     ev_sets = [flarepp.StageEvents(stream) for _ in range(args.steps)]
     warm_ev = flarepp.StageEvents(stream)
@@ -612,11 +737,13 @@ def main():
     ap.add_argument("--impl", choices=("ours", "reference"), default="ours")
     ap.add_argument("--workload", default="mesh3d", choices=sorted(inputs.WORKLOADS))
     ap.add_argument("--seed", type=int, default=0)
-    ap.add_argument("--variant", choices=("flarepp", "shared", "flare", "train"),
+    ap.add_argument("--variant", choices=("flarepp", "shared", "flare", "train", "mixer",
+                                          "mixer_shared"),
                     default="flarepp",
                     help="flarepp: the routing chain (default); shared: the chain with Kt, Vt "
                          "tied to K, V; flare: FLARE with fixed learned queries; train: the "
-                         "chain's training forward and backward")
+                         "chain's training forward and backward; mixer(_shared): the whole "
+                         "FLARE++ mixer layer with four (two) projections")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--e2e-steps", type=int, default=5)
     ap.add_argument("--no-cpu-baseline", action="store_true")

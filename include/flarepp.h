@@ -224,6 +224,19 @@ FLAREPP_API flarepp_status flarepp_mixer_fwd(const flarepp_shape* shape, int n_p
                                              void* stream);
 
 /*
+ * flarepp_mixer_fwd that also records four caller-created CUDA events (cudaEvent_t) on
+ * `stream`: events[0] before the input projection, [1] after it, [2] after the routing chain,
+ * [3] after the output projection. n_events must be >= 4 and no event may be NULL (else
+ * FLAREPP_ERR_INVALID_ARGUMENT); on degenerate shapes no event is recorded.
+ */
+FLAREPP_API flarepp_status flarepp_mixer_fwd_profiled(const flarepp_shape* shape, int n_proj,
+                                                      const void* X, const void* W_in,
+                                                      const void* Wo, const void* seeds,
+                                                      float scale, void* O, void* workspace,
+                                                      size_t workspace_bytes, void* stream,
+                                                      void* const* events, int n_events);
+
+/*
  * Bytes of the state a training forward keeps for the backward (App. A.5): float32 Q and Z
  * [B, H, M, D] and the base-2 log-normalisers of the three calls,
  * L = log2 sum_j 2^(scale * log2(e) <a, b_j>), for calls 1 and 2 [B, H, M] and call 3

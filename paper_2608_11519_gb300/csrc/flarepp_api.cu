@@ -476,7 +476,8 @@ bool mixer_layout(const Plan& p, int n_proj, MixerLayout* L) {
 
 flarepp_status mixer_impl(const flarepp_shape* shape, int n_proj, const void* X, const void* W_in,
                           const void* Wo, const void* seeds, float scale, void* O,
-                          void* workspace, size_t workspace_bytes, void* stream) {
+                          void* workspace, size_t workspace_bytes, void* stream,
+                          void* const* events = nullptr) {
     Plan p;
     flarepp_status stt = make_plan(shape, &p);
     if (stt != FLAREPP_OK) return stt;
@@ -509,10 +510,15 @@ flarepp_status mixer_impl(const flarepp_shape* shape, int n_proj, const void* X,
     char* ws = (char*)workspace;
     int* status = (int*)(ws + p.off_status);
     if (cudaMemsetAsync(status, 0, sizeof(int32_t), st) != cudaSuccess) return FLAREPP_ERR_CUDA;
+    auto mark = [&](int i) {
+        return !events || cudaEventRecord((cudaEvent_t)events[i], st) == cudaSuccess;
+    };
     void* proj[4];
     for (int i = 0; i < 4; ++i) proj[i] = ws + L.off_proj[i < n_proj ? i : i - 2];
     // K, V, K~, V~ = X W_in^T, split into heads (eqs. flarepp_query_synthesis, flarepp_mixer)
-    if (tc_projection(p.B, p.N, p.H, p.D, n_proj, X, W_in, proj, status, st) != cudaSuccess)
+    if (!mark(0) ||
+        tc_projection(p.B, p.N, p.H, p.D, n_proj, X, W_in, proj, status, st) != cudaSuccess ||
+        !mark(1))
         return FLAREPP_ERR_CUDA;
     // the routing chain; the shared variant reads K, V as K~, V~ (App. C.2)
     void* Y = ws + L.off_y;
@@ -520,7 +526,9 @@ flarepp_status mixer_impl(const flarepp_shape* shape, int n_proj, const void* X,
                      p.total, stream, nullptr, nullptr, nullptr, 0, false);
     if (stt != FLAREPP_OK) return stt;
     // O = merge(Y) Wo^T
-    if (tc_output_projection(p.B, p.N, p.H, p.D, Y, Wo, O, status, st) != cudaSuccess)
+    if (!mark(2) ||
+        tc_output_projection(p.B, p.N, p.H, p.D, Y, Wo, O, status, st) != cudaSuccess ||
+        !mark(3))
         return FLAREPP_ERR_CUDA;
     return FLAREPP_OK;
 }
@@ -545,6 +553,18 @@ flarepp_status flarepp_mixer_fwd(const flarepp_shape* shape, int n_proj, const v
                                  void* O, void* workspace, size_t workspace_bytes, void* stream) {
     return flarepp::mixer_impl(shape, n_proj, X, W_in, Wo, seeds, scale, O, workspace,
                                workspace_bytes, stream);
+}
+
+flarepp_status flarepp_mixer_fwd_profiled(const flarepp_shape* shape, int n_proj, const void* X,
+                                          const void* W_in, const void* Wo, const void* seeds,
+                                          float scale, void* O, void* workspace,
+                                          size_t workspace_bytes, void* stream,
+                                          void* const* events, int n_events) {
+    if (!events || n_events < 4) return FLAREPP_ERR_INVALID_ARGUMENT;
+    for (int i = 0; i < 4; ++i)
+        if (!events[i]) return FLAREPP_ERR_INVALID_ARGUMENT;
+    return flarepp::mixer_impl(shape, n_proj, X, W_in, Wo, seeds, scale, O, workspace,
+                               workspace_bytes, stream, events);
 }
 
 size_t flarepp_route_saved_bytes(const flarepp_shape* shape) {

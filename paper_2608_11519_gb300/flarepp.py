@@ -24,7 +24,7 @@ _DTYPES = {torch.float32: F32, torch.bfloat16: BF16}
 EXPORTED = ("flarepp_route_workspace_bytes", "flarepp_route_fwd", "flarepp_route_fwd_debug",
             "flarepp_route_fwd_profiled", "flarepp_route_fwd_noalloc",
             "flarepp_flare_fwd", "flarepp_route_host_buffer_bytes", "flarepp_route_fwd_host",
-            "flarepp_mixer_workspace_bytes", "flarepp_mixer_fwd",
+            "flarepp_mixer_workspace_bytes", "flarepp_mixer_fwd", "flarepp_mixer_fwd_profiled",
             "flarepp_route_saved_bytes", "flarepp_route_fwd_train",
             "flarepp_route_bwd_workspace_bytes", "flarepp_route_bwd",
             "flarepp_route_device_status", "flarepp_status_string", "flarepp_version")
@@ -86,6 +86,10 @@ def load(path: str = None):
     lib.flarepp_mixer_fwd.restype = ctypes.c_int
     lib.flarepp_mixer_fwd.argtypes = [sp, ctypes.c_int, vp, vp, vp, vp, ctypes.c_float, vp, vp,
                                       sz, vp]
+    lib.flarepp_mixer_fwd_profiled.restype = ctypes.c_int
+    lib.flarepp_mixer_fwd_profiled.argtypes = [sp, ctypes.c_int, vp, vp, vp, vp, ctypes.c_float,
+                                               vp, vp, sz, vp, ctypes.POINTER(ctypes.c_void_p),
+                                               ctypes.c_int]
     lib.flarepp_route_saved_bytes.restype = sz
     lib.flarepp_route_saved_bytes.argtypes = [sp]
     lib.flarepp_route_fwd_train.restype = ctypes.c_int
@@ -314,7 +318,29 @@ def flare_fwd(Q, K, V, scale=None, Y=None, workspace=None, stream=None, Z_out=No
     return Y
 
 
-def mixer_fwd(X, W_in, Wo, seeds, scale=None, O=None, workspace=None, stream=None):
+MIXER_STAGES = ("projection", "chain", "output")
+
+
+class MixerEvents:
+    """Four timing events the library records around the mixer's stages
+    (flarepp_mixer_fwd_profiled)."""
+
+    def __init__(self, stream=None):
+        stream = stream or torch.cuda.current_stream()
+        self.events = [torch.cuda.Event(enable_timing=True) for _ in range(4)]
+        for e in self.events:  # create the underlying cudaEvent_t
+            e.record(stream)
+        self.handles = (ctypes.c_void_p * 4)(*[ctypes.c_void_p(int(e.cuda_event))
+                                               for e in self.events])
+
+    def stage_ms(self):
+        """Milliseconds of each stage of the last recorded call (synchronises on the events)."""
+        self.events[-1].synchronize()
+        return {s: self.events[i].elapsed_time(self.events[i + 1])
+                for i, s in enumerate(MIXER_STAGES)}
+
+
+def mixer_fwd(X, W_in, Wo, seeds, scale=None, O=None, workspace=None, stream=None, events=None):
     """The FLARE++ mixer layer (Fig. 1) on device tensors: X [B, N, C], W_in [P*C, C] (P = 4:
     K, V, K~, V~; P = 2: shared projection), Wo [C, C] (both out x in), seeds [H, M, D].
     Returns O [B, N, C]."""
@@ -340,10 +366,13 @@ def mixer_fwd(X, W_in, Wo, seeds, scale=None, O=None, workspace=None, stream=Non
     nbytes = int(lib.flarepp_mixer_workspace_bytes(ctypes.byref(shape), P))
     ws = (workspace if isinstance(workspace, Workspace) else Workspace()).get(nbytes, X.device)
     st = stream if stream is not None else torch.cuda.current_stream(X.device)
-    rc = lib.flarepp_mixer_fwd(ctypes.byref(shape), P, _ptr(X), _ptr(W_in), _ptr(Wo),
-                               _ptr(seeds), float(scale), _ptr(O),
-                               None if ws is None else ctypes.c_void_p(ws.data_ptr()), nbytes,
-                               ctypes.c_void_p(st.cuda_stream))
+    args = (ctypes.byref(shape), P, _ptr(X), _ptr(W_in), _ptr(Wo), _ptr(seeds), float(scale),
+            _ptr(O), None if ws is None else ctypes.c_void_p(ws.data_ptr()), nbytes,
+            ctypes.c_void_p(st.cuda_stream))
+    if events is None:
+        rc = lib.flarepp_mixer_fwd(*args)
+    else:
+        rc = lib.flarepp_mixer_fwd_profiled(*args, events.handles, 4)
     if rc != OK:
         raise FlareppError(rc, "flarepp_mixer_fwd")
     return O

@@ -119,6 +119,22 @@ def make_output_grad(w: Workload, seed: int = 0, device="cpu"):
     return torch.randn(w.B, w.H, w.N, w.D, generator=gen, device=device).to(w.torch_dtype)
 
 
+def make_mixer_inputs(w: Workload, seed: int = 0, device="cpu", n_proj: int = 4):
+    """Draw the mixer layer's inputs for workload ``w`` (C = H * D) in its dtype: X [B, N, C]
+    i.i.d. N(0, 1); W_in [n_proj * C, C] and Wo [C, C] i.i.d. N(0, 1 / C) (unit-variance
+    outputs); seeds [H, M, D] i.i.d. N(0, 1). Seed offset by 104729 from :func:`make_inputs`."""
+    gen = torch.Generator(device=device)
+    gen.manual_seed(int(seed) + 104729)
+    B, H, N, M, D = w.B, w.H, w.N, w.M, w.D
+    C = H * D
+    dt = w.torch_dtype
+    X = torch.randn(B, N, C, generator=gen, device=device).to(dt)
+    W_in = (torch.randn(n_proj * C, C, generator=gen, device=device) / math.sqrt(C)).to(dt)
+    Wo = (torch.randn(C, C, generator=gen, device=device) / math.sqrt(C)).to(dt)
+    seeds = torch.randn(H, M, D, generator=gen, device=device).to(dt)
+    return {"X": X, "W_in": W_in, "Wo": Wo, "seeds": seeds}
+
+
 def to_f64_numpy(inputs):
     """The exact values of each input as float64 numpy arrays (bf16 and f32 upcast exactly)."""
     return {k: v.detach().to("cpu", torch.float64).numpy() for k, v in inputs.items()}
