@@ -15,9 +15,9 @@
 // channels; persistent CTAs walk the tiles with the channel tile varying fastest, so the CTAs
 // that share a token tile run together and read it from L2.
 //
-// Roles (8 warps): warp 0 the TMA producer, warp 1 the MMA issuer (one elected lane; one
-// commit per slice frees its ring stage, one per tile hands the accumulator over), warps 4..7
-// the epilogue (TMEM lane = token row). Two TMEM accumulators of NT <= 256 columns let the
+// Roles (12 warps): warp 0 the TMA producer, warp 1 the MMA issuer (one elected lane; one
+// commit per slice frees its ring stage, one per tile hands the accumulator over), warps 4..11
+// two epilogue warpgroups (TMEM lane = token row; each takes half of the tile's channels). Two TMEM accumulators of NT <= 256 columns let the
 // epilogue of one tile overlap the products of the next. Every wait is bounded (2 s of
 // %globaltimer): on expiry the kernel records FLAREPP_ERR_TIMEOUT in the status word, every
 // role leaves its loops, the producer waits for its copies in flight, the MMA issuer for its
@@ -36,7 +36,8 @@ namespace {
 
 using namespace tc;
 
-constexpr int kThreads = 256;
+constexpr int kEpiGroups = 2;  // epilogue warpgroups; each takes half of a tile's channels
+constexpr int kThreads = (4 + 4 * kEpiGroups) * 32;
 constexpr int kFirstEpiWarp = 4;
 constexpr int kRows = 128;    // tokens per tile (TMEM lanes, MMA M)
 constexpr int kMaxNT = 256;   // output channels per tile, at most
@@ -137,7 +138,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         for (int b = 0; b < 2; ++b) {
             mbar_init(accfull0 + 8u * b, 1);
-            mbar_init(accempty0 + 8u * b, kRows);
+            mbar_init(accempty0 + 8u * b, kRows * kEpiGroups);
         }
         mbar_init(fin, 1);
         *abort_flag = 0;
@@ -236,9 +237,13 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
     } else if (warp >= kFirstEpiWarp) {
         // ------------------------------------------------------------ epilogue
+        // Warpgroup e takes channels [e * NT / 2, (e + 1) * NT / 2) of each tile, 64 columns
+        // per TMEM round (four loads, one wait).
         const int q = warp % 4;
+        const int e = (warp - kFirstEpiWarp) / 4;
         const int r = 32 * q + lane;
         const uint32_t lane_off = (uint32_t)(32 * q) << 16;
+        const int half = prm.NT / kEpiGroups;
         uint32_t j = 0;
         for (int64_t t = blockIdx.x; t < prm.n_tiles; t += gridDim.x, ++j) {
             const GTile T = gtile(prm, t);
@@ -248,32 +253,50 @@ __global__ void __launch_bounds__(kThreads, 1)
             const int64_t n = T.rt * kRows + r;
             const bool valid = n < prm.N;
             const uint32_t acc = tmem + lane_off + ab * kMaxNT;
-            for (int c16 = 0; c16 < prm.NT; c16 += 16) {
-                uint32_t v[16];
-                tmem_ld16(acc + c16, v);
+            // the tile's channels lie in one projection (NT divides C): its base pointer once
+            const int64_t c0 = T.ct * prm.NT + e * half;
+            const int64_t p = c0 / prm.C, cc0 = c0 % prm.C;
+            __nv_bfloat16* base = MODE != 0 ? prm.out[0]
+                                  : p == 0   ? prm.out[0]
+                                  : p == 1   ? prm.out[1]
+                                  : p == 2   ? prm.out[2]
+                                             : prm.out[3];
+            __nv_bfloat16* row = MODE == 0 ? base + (T.b * prm.H * prm.N + n) * D
+                                           : base + (T.b * prm.N + n) * prm.C + c0;
+            for (int c64 = 0; c64 < half; c64 += 64) {
+                const int w = half - c64 < 64 ? half - c64 : 64;  // 16, 32 or 64 columns
+                uint32_t v[64];
+                const uint32_t col = acc + e * half + c64;
+                tmem_ld16(col, v);
+                if (w > 16) tmem_ld16(col + 16, v + 16);
+                if (w > 32) {
+                    tmem_ld16(col + 32, v + 32);
+                    tmem_ld16(col + 48, v + 48);
+                }
+                // waits that name the loaded registers, so that no use moves above them
                 tmem_wait_ld16(v);
+                if (w > 16) tmem_wait_ld16(v + 16);
+                if (w > 32) {
+                    tmem_wait_ld16(v + 32);
+                    tmem_wait_ld16(v + 48);
+                }
                 if (!valid) continue;
 #pragma unroll
-                for (int g = 0; g < 2; ++g) {
-                    const int64_t c = T.ct * prm.NT + c16 + 8 * g;  // output channel
-                    uint4 w;
-                    w.x = pack_bf16(__uint_as_float(v[8 * g + 0]), __uint_as_float(v[8 * g + 1]));
-                    w.y = pack_bf16(__uint_as_float(v[8 * g + 2]), __uint_as_float(v[8 * g + 3]));
-                    w.z = pack_bf16(__uint_as_float(v[8 * g + 4]), __uint_as_float(v[8 * g + 5]));
-                    w.w = pack_bf16(__uint_as_float(v[8 * g + 6]), __uint_as_float(v[8 * g + 7]));
+                for (int g = 0; g < 8; ++g) {
+                    if (8 * g >= w) break;
+                    uint4 o;
+                    o.x = pack_bf16(__uint_as_float(v[8 * g + 0]), __uint_as_float(v[8 * g + 1]));
+                    o.y = pack_bf16(__uint_as_float(v[8 * g + 2]), __uint_as_float(v[8 * g + 3]));
+                    o.z = pack_bf16(__uint_as_float(v[8 * g + 4]), __uint_as_float(v[8 * g + 5]));
+                    o.w = pack_bf16(__uint_as_float(v[8 * g + 6]), __uint_as_float(v[8 * g + 7]));
                     __nv_bfloat16* dst;
                     if (MODE == 0) {
-                        const int64_t p = c / prm.C, cc = c % prm.C;
-                        const int64_t h = cc / D, d = cc % D;
-                        __nv_bfloat16* base = p == 0   ? prm.out[0]
-                                              : p == 1 ? prm.out[1]
-                                              : p == 2 ? prm.out[2]
-                                                       : prm.out[3];
-                        dst = base + ((T.b * prm.H + h) * prm.N + n) * D + d;
+                        const int64_t cc = cc0 + c64 + 8 * g;  // channel within the projection
+                        dst = row + (cc / D) * prm.N * D + (cc % D);
                     } else {
-                        dst = prm.out[0] + (T.b * prm.N + n) * prm.C + c;
+                        dst = row + c64 + 8 * g;
                     }
-                    *reinterpret_cast<uint4*>(dst) = w;
+                    *reinterpret_cast<uint4*>(dst) = o;
                 }
             }
             tc_fence_before();
