@@ -17,7 +17,8 @@
 //
 // Roles (12 warps): warp 0 the TMA producer, warp 1 the MMA issuer (one elected lane; one
 // commit per slice frees its ring stage, one per tile hands the accumulator over), warps 4..11
-// two epilogue warpgroups (TMEM lane = token row; each takes half of the tile's channels). Two TMEM accumulators of NT <= 256 columns let the
+// two epilogue warpgroups (TMEM lane = token row; each takes every other head of the tile and
+// writes it with one TMA store per head from a shared-memory staging block). Two TMEM accumulators of NT <= 256 columns let the
 // epilogue of one tile overlap the products of the next. Every wait is bounded (2 s of
 // %globaltimer): on expiry the kernel records FLAREPP_ERR_TIMEOUT in the status word, every
 // role leaves its loops, the producer waits for its copies in flight, the MMA issuer for its
@@ -49,11 +50,16 @@ struct GCfg {
     static constexpr int kASlice = kRows * D * 2;
     static constexpr int kBSlice = kMaxNT * D * 2;
     static constexpr int kStage = kASlice + kBSlice;
-    static constexpr int kStages = (192 * 1024) / kStage > 8 ? 8 : (192 * 1024) / kStage;
+    static constexpr int kStages = (160 * 1024) / kStage > 8 ? 8 : (160 * 1024) / kStage;
     static constexpr uint32_t kSwz = D == 16 ? kSw32 : (D == 32 ? kSw64 : kSw128);
     static constexpr uint32_t kSBO = 8 * D * 2;
-    static constexpr int kNumBars = 2 * kStages + 4 + 1;  // full, empty, accfull[2], accempty[2], fin
-    static constexpr int kNeed = 1024 + kStages * kStage + kNumBars * 8 + 16;
+    // per epilogue warpgroup: its heads of one tile, [head][128 rows][D] bf16, for TMA stores
+    static constexpr int kStaging = (kMaxNT / 2) * kRows * 2;
+    // full, empty, accfull[2], accempty[2], fin, then per epilogue warpgroup staging_free and
+    // staging_written
+    static constexpr int kNumBars = 2 * kStages + 4 + 1 + 2 * kEpiGroups;
+    static constexpr int kNeed =
+        1024 + kStages * kStage + kEpiGroups * kStaging + kNumBars * 8 + 16;
     static constexpr int kSmem = kNeed > 122880 ? kNeed : 122880;  // one CTA per SM
     static_assert(kSmem <= 232448, "shared memory budget");
 };
@@ -61,7 +67,7 @@ struct GCfg {
 struct GemmParams {
     int64_t B, N, H, C;
     int64_t n_out;      // output channels (P * C, or C)
-    int NT;             // output channels per tile (a multiple of 16, <= 256, divides C)
+    int NT;             // output channels per tile (whole heads, <= 256, divides C)
     uint32_t idesc;     // MMA instruction descriptor for M = 128, N = NT
     int64_t row_tiles;  // 128-token tiles per batch element
     int64_t col_tiles;  // n_out / NT
@@ -113,13 +119,16 @@ __device__ __forceinline__ uint32_t pack_bf16(float lo, float hi) {
 template <int D, int MODE>
 __global__ void __launch_bounds__(kThreads, 1)
     tc_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
+                   const __grid_constant__ CUtensorMap tmO0, const __grid_constant__ CUtensorMap tmO1,
+                   const __grid_constant__ CUtensorMap tmO2, const __grid_constant__ CUtensorMap tmO3,
                    const GemmParams prm) {
     using C = GCfg<D>;
     constexpr int kS = C::kStages;
     extern __shared__ uint8_t smem_raw[];
     uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                                ~static_cast<uintptr_t>(1023));
-    uint64_t* bars = reinterpret_cast<uint64_t*>(smem + kS * C::kStage);
+    uint8_t* staging = smem + kS * C::kStage;  // [kEpiGroups][kStaging]
+    uint64_t* bars = reinterpret_cast<uint64_t*>(staging + kEpiGroups * C::kStaging);
     uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + C::kNumBars);
     volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
     const uint32_t full0 = smem_u32(bars);
@@ -127,6 +136,8 @@ __global__ void __launch_bounds__(kThreads, 1)
     const uint32_t accfull0 = empty0 + 8u * kS;
     const uint32_t accempty0 = accfull0 + 16u;
     const uint32_t fin = accempty0 + 16u;
+    const uint32_t sfree0 = fin + 8u;                      // [kEpiGroups], count 1
+    const uint32_t swritten0 = sfree0 + 8u * kEpiGroups;   // [kEpiGroups], count 128
     const int warp = threadIdx.x >> 5;
     const int lane = threadIdx.x & 31;
     const int slices = (int)(prm.C / D);
@@ -141,6 +152,10 @@ __global__ void __launch_bounds__(kThreads, 1)
             mbar_init(accempty0 + 8u * b, kRows * kEpiGroups);
         }
         mbar_init(fin, 1);
+        for (int e = 0; e < kEpiGroups; ++e) {
+            mbar_init(sfree0 + 8u * e, 1);
+            mbar_init(swritten0 + 8u * e, kRows);
+        }
         *abort_flag = 0;
         fence_mbar_init();
         prefetch_tmap(&tmA);
@@ -237,71 +252,77 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
     } else if (warp >= kFirstEpiWarp) {
         // ------------------------------------------------------------ epilogue
-        // Warpgroup e takes channels [e * NT / 2, (e + 1) * NT / 2) of each tile, 64 columns
-        // per TMEM round (four loads, one wait).
+        // Warpgroup e takes the tile's heads e, e + 2, ...: each head's 128 x D block goes from
+        // TMEM through shared memory ([128 rows][D], one row per thread) to one TMA tensor
+        // store (rows beyond N are clipped by the store). Two mbarriers per warpgroup order the
+        // staging buffer (bounded waits): staging_free, which the leader arrives on once its
+        // previous stores have read the buffer, and staging_written, on which every thread
+        // arrives after its rows (and a proxy fence) and which the leader waits for before it
+        // issues the stores.
         const int q = warp % 4;
         const int e = (warp - kFirstEpiWarp) / 4;
         const int r = 32 * q + lane;
+        const bool leader = q == 0 && lane == 0;
         const uint32_t lane_off = (uint32_t)(32 * q) << 16;
-        const int half = prm.NT / kEpiGroups;
+        const int heads = prm.NT / D;
+        uint8_t* stg = staging + e * C::kStaging;
         uint32_t j = 0;
+        bool pending = false;
         for (int64_t t = blockIdx.x; t < prm.n_tiles; t += gridDim.x, ++j) {
             const GTile T = gtile(prm, t);
             const int ab = j & 1;
             if (!warp_wait(accfull0 + 8u * ab, (j >> 1) & 1, abort_flag, prm.status)) break;
             tc_fence_after();
-            const int64_t n = T.rt * kRows + r;
-            const bool valid = n < prm.N;
+            if (pending) {
+                if (leader) {
+                    bulk_wait_read();
+                    mbar_arrive(sfree0 + 8u * e);
+                }
+                if (!warp_wait(sfree0 + 8u * e, (j - 1) & 1, abort_flag, prm.status)) break;
+            }
             const uint32_t acc = tmem + lane_off + ab * kMaxNT;
-            // the tile's channels lie in one projection (NT divides C): its base pointer once
-            const int64_t c0 = T.ct * prm.NT + e * half;
-            const int64_t p = c0 / prm.C, cc0 = c0 % prm.C;
-            __nv_bfloat16* base = MODE != 0 ? prm.out[0]
-                                  : p == 0   ? prm.out[0]
-                                  : p == 1   ? prm.out[1]
-                                  : p == 2   ? prm.out[2]
-                                             : prm.out[3];
-            __nv_bfloat16* row = MODE == 0 ? base + (T.b * prm.H * prm.N + n) * D
-                                           : base + (T.b * prm.N + n) * prm.C + c0;
-            for (int c64 = 0; c64 < half; c64 += 64) {
-                const int w = half - c64 < 64 ? half - c64 : 64;  // 16, 32 or 64 columns
-                uint32_t v[64];
-                const uint32_t col = acc + e * half + c64;
-                tmem_ld16(col, v);
-                if (w > 16) tmem_ld16(col + 16, v + 16);
-                if (w > 32) {
-                    tmem_ld16(col + 32, v + 32);
-                    tmem_ld16(col + 48, v + 48);
-                }
-                // waits that name the loaded registers, so that no use moves above them
-                tmem_wait_ld16(v);
-                if (w > 16) tmem_wait_ld16(v + 16);
-                if (w > 32) {
-                    tmem_wait_ld16(v + 32);
-                    tmem_wait_ld16(v + 48);
-                }
-                if (!valid) continue;
+            int slot = 0;
+            for (int hh = e; hh < heads; hh += kEpiGroups, ++slot) {
+                uint32_t v[D];
 #pragma unroll
-                for (int g = 0; g < 8; ++g) {
-                    if (8 * g >= w) break;
+                for (int k = 0; k < D / 16; ++k) tmem_ld16(acc + hh * D + 16 * k, v + 16 * k);
+#pragma unroll
+                for (int k = 0; k < D / 16; ++k) tmem_wait_ld16(v + 16 * k);
+                uint4* dst = reinterpret_cast<uint4*>(stg + ((size_t)slot * kRows + r) * D * 2);
+#pragma unroll
+                for (int g = 0; g < D / 8; ++g) {
                     uint4 o;
                     o.x = pack_bf16(__uint_as_float(v[8 * g + 0]), __uint_as_float(v[8 * g + 1]));
                     o.y = pack_bf16(__uint_as_float(v[8 * g + 2]), __uint_as_float(v[8 * g + 3]));
                     o.z = pack_bf16(__uint_as_float(v[8 * g + 4]), __uint_as_float(v[8 * g + 5]));
                     o.w = pack_bf16(__uint_as_float(v[8 * g + 6]), __uint_as_float(v[8 * g + 7]));
-                    __nv_bfloat16* dst;
-                    if (MODE == 0) {
-                        const int64_t cc = cc0 + c64 + 8 * g;  // channel within the projection
-                        dst = row + (cc / D) * prm.N * D + (cc % D);
-                    } else {
-                        dst = row + c64 + 8 * g;
-                    }
-                    *reinterpret_cast<uint4*>(dst) = o;
+                    dst[g] = o;
                 }
             }
             tc_fence_before();
-            mbar_arrive(accempty0 + 8u * ab);
+            mbar_arrive(accempty0 + 8u * ab);  // the accumulator is read out
+            fence_proxy_async();
+            mbar_arrive(swritten0 + 8u * e);
+            if (q == 0 && !warp_wait(swritten0 + 8u * e, j & 1, abort_flag, prm.status)) break;
+            if (leader) {
+                slot = 0;
+                const int n0 = (int)(T.rt * kRows);
+                for (int hh = e; hh < heads; hh += kEpiGroups, ++slot) {
+                    const int64_t c = T.ct * prm.NT + (int64_t)hh * D;  // first channel
+                    const uint32_t src = smem_u32(stg + (size_t)slot * kRows * D * 2);
+                    if (MODE == 0) {
+                        const int64_t p = c / prm.C, h = (c % prm.C) / D;
+                        const CUtensorMap* m = p == 0 ? &tmO0 : p == 1 ? &tmO1 : p == 2 ? &tmO2 : &tmO3;
+                        tma_store_3d(m, src, 0, n0, (int)(T.b * prm.H + h));
+                    } else {
+                        tma_store_3d(&tmO0, src, (int)c, n0, (int)T.b);
+                    }
+                }
+                bulk_commit();
+            }
+            pending = true;
         }
+        if (leader) bulk_wait_all();
     }
     tc_fence_before();
     __syncthreads();
@@ -344,8 +365,8 @@ bool make_map(CUtensorMap* m, const void* base, int64_t D, int64_t inner, int64_
 }
 
 template <int D, int MODE>
-cudaError_t launch(const CUtensorMap& a, const CUtensorMap& b, const GemmParams& prm,
-                   cudaStream_t st) {
+cudaError_t launch(const CUtensorMap& a, const CUtensorMap& b, const CUtensorMap* o,
+                   const GemmParams& prm, cudaStream_t st) {
     using Cf = GCfg<D>;
     static cudaError_t attr = cudaFuncSetAttribute(
         tc_gemm_kernel<D, MODE>, cudaFuncAttributeMaxDynamicSharedMemorySize, Cf::kSmem);
@@ -355,15 +376,32 @@ cudaError_t launch(const CUtensorMap& a, const CUtensorMap& b, const GemmParams&
     cudaGetDevice(&dev);
     cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
     const int64_t grid = prm.n_tiles < sms ? prm.n_tiles : sms;
-    tc_gemm_kernel<D, MODE><<<(unsigned)grid, kThreads, Cf::kSmem, st>>>(a, b, prm);
+    tc_gemm_kernel<D, MODE><<<(unsigned)grid, kThreads, Cf::kSmem, st>>>(a, b, o[0], o[1], o[2],
+                                                                         o[3], prm);
     return cudaGetLastError();
 }
 
-// output channels per tile: the largest of 256, 128, 64, 32, 16 that divides C
-int tile_channels(int64_t C) {
-    for (int nt = kMaxNT; nt >= 16; nt /= 2)
-        if (C % nt == 0) return nt;
-    return 0;
+// output channels per tile: D times the largest power of two of heads that divides H and
+// keeps the tile within 256 channels
+int tile_channels(int64_t H, int64_t D) {
+    int heads = 1;
+    while (heads * 2 * D <= kMaxNT && H % (heads * 2) == 0) heads *= 2;
+    return (int)(heads * D);
+}
+
+// An unswizzled bf16 tensor of dims {inner, rows, z}, boxes of box_inner x 128 x 1 (the
+// epilogue's staged blocks).
+bool make_store_map(CUtensorMap* m, void* base, int64_t inner, int64_t rows, int64_t z,
+                    uint32_t box_inner) {
+    auto fn = encode_fn();
+    if (!fn) return false;
+    cuuint64_t dims[3] = {(cuuint64_t)inner, (cuuint64_t)rows, (cuuint64_t)z};
+    cuuint64_t strides[2] = {(cuuint64_t)(inner * 2), (cuuint64_t)(rows * inner * 2)};
+    cuuint32_t box[3] = {box_inner, (cuuint32_t)kRows, 1};
+    cuuint32_t estr[3] = {1, 1, 1};
+    return fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, base, dims, strides, box, estr,
+              CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE,
+              CU_TENSOR_MAP_L2_PROMOTION_NONE, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
 }  // namespace
@@ -377,22 +415,24 @@ cudaError_t tc_projection(int64_t B, int64_t N, int64_t H, int64_t D, int P, con
     prm.H = H;
     prm.C = C;
     prm.n_out = P * C;
-    prm.NT = tile_channels(C);
-    if (prm.NT == 0) return cudaErrorInvalidValue;
+    prm.NT = tile_channels(H, D);
     prm.idesc = idesc_bf16_f32(kRows, prm.NT, false, false);
     prm.row_tiles = (N + kRows - 1) / kRows;
     prm.col_tiles = prm.n_out / prm.NT;
     prm.n_tiles = B * prm.row_tiles * prm.col_tiles;
-    for (int p = 0; p < 4; ++p) prm.out[p] = (__nv_bfloat16*)outs[p < P ? p : 0];
+    for (int p = 0; p < 4; ++p) prm.out[p] = (__nv_bfloat16*)outs[p < P ? p : p - 2];
     prm.status = status;
-    CUtensorMap ma, mb;
+    CUtensorMap ma, mb, mo[4];
     if (!make_map(&ma, X, D, C, N, B, kRows) ||
         !make_map(&mb, W_in, D, C, prm.n_out, 1, (uint32_t)prm.NT))
         return cudaErrorInvalidValue;
+    for (int p = 0; p < 4; ++p)
+        if (!make_store_map(&mo[p], prm.out[p], D, N, B * H, (uint32_t)D))
+            return cudaErrorInvalidValue;
     switch (D) {
-        case 16: return launch<16, 0>(ma, mb, prm, st);
-        case 32: return launch<32, 0>(ma, mb, prm, st);
-        case 64: return launch<64, 0>(ma, mb, prm, st);
+        case 16: return launch<16, 0>(ma, mb, mo, prm, st);
+        case 32: return launch<32, 0>(ma, mb, mo, prm, st);
+        case 64: return launch<64, 0>(ma, mb, mo, prm, st);
         default: return cudaErrorInvalidValue;
     }
 }
@@ -406,22 +446,23 @@ cudaError_t tc_output_projection(int64_t B, int64_t N, int64_t H, int64_t D, con
     prm.H = H;
     prm.C = C;
     prm.n_out = C;
-    prm.NT = tile_channels(C);
-    if (prm.NT == 0) return cudaErrorInvalidValue;
+    prm.NT = tile_channels(H, D);
     prm.idesc = idesc_bf16_f32(kRows, prm.NT, false, false);
     prm.row_tiles = (N + kRows - 1) / kRows;
     prm.col_tiles = C / prm.NT;
     prm.n_tiles = B * prm.row_tiles * prm.col_tiles;
     prm.out[0] = prm.out[1] = prm.out[2] = prm.out[3] = (__nv_bfloat16*)O;
     prm.status = status;
-    CUtensorMap ma, mb;
+    CUtensorMap ma, mb, mo[4];
     if (!make_map(&ma, Y, D, D, N, B * H, kRows) ||
-        !make_map(&mb, Wo, D, C, C, 1, (uint32_t)prm.NT))
+        !make_map(&mb, Wo, D, C, C, 1, (uint32_t)prm.NT) ||
+        !make_store_map(&mo[0], O, C, N, B, (uint32_t)D))
         return cudaErrorInvalidValue;
+    mo[1] = mo[2] = mo[3] = mo[0];
     switch (D) {
-        case 16: return launch<16, 1>(ma, mb, prm, st);
-        case 32: return launch<32, 1>(ma, mb, prm, st);
-        case 64: return launch<64, 1>(ma, mb, prm, st);
+        case 16: return launch<16, 1>(ma, mb, mo, prm, st);
+        case 32: return launch<32, 1>(ma, mb, mo, prm, st);
+        case 64: return launch<64, 1>(ma, mb, mo, prm, st);
         default: return cudaErrorInvalidValue;
     }
 }
