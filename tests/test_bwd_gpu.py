@@ -202,3 +202,40 @@ def test_bwd_is_deterministic():
     b, _ = _gpu_grads(x, dY, w.scale)
     for u, v in zip(a, b):
         assert np.array_equal(u, v)
+
+
+@pytest.mark.parametrize("shape", [(1, 2, 700, 2048, 16, "bf16"), (1, 1, 500, 2048, 64, "bf16"),
+                                   (1, 1, 300, 1024, 32, "f32")],
+                         ids=["M2048_D16", "M2048_D64", "M1024_f32"])
+def test_bwd_largest_route_counts(shape):
+    """The largest supported M (2048) with the smallest and largest head widths."""
+    B, H, N, M, D, dt = shape
+    w = inputs.Workload("case", B, H, N, M, D, dt)
+    x = inputs.make_inputs(w, 4)
+    dY = inputs.make_output_grad(w, 4)
+    got, _ = _gpu_grads(x, dY, w.scale)
+    f = inputs.to_f64_numpy(x)
+    want = oracle.route_bwd(f["seeds"], f["Kt"], f["Vt"], f["K"], f["V"], w.scale, _np(dY))
+    _check_grads(got, want, TOL[dt])
+
+
+def test_bwd_guard_bands_untouched():
+    """The gradients are written inside their tensors only: each output is a view into a
+    larger buffer whose bands before and after keep their sentinel value."""
+    w = inputs.Workload("case", 2, 2, 777, 100, 32, "bf16")
+    x = {k: v.cuda() for k, v in inputs.make_inputs(w, 6).items()}
+    args = (x["seeds"], x["Kt"], x["Vt"], x["K"], x["V"])
+    Y, saved = flarepp.route_fwd_train(*args, w.scale)
+    dY = inputs.make_output_grad(w, 6).cuda()
+    band = 4096
+    grads, bufs = [], []
+    for t in args:
+        buf = torch.full((t.numel() + 2 * band,), 7.0, dtype=t.dtype, device="cuda")
+        bufs.append(buf)
+        grads.append(buf[band:band + t.numel()].view(t.shape))
+    flarepp.route_bwd(*args, Y, dY, saved, w.scale, grads=tuple(grads))
+    torch.cuda.synchronize()
+    for buf in bufs:
+        assert torch.all(buf[:band] == 7.0) and torch.all(buf[-band:] == 7.0)
+    for g in grads:
+        assert torch.isfinite(g.float()).all()

@@ -47,7 +47,8 @@ SHAPES = [
     (2, 4, 300, 40, 16, 4),
     (1, 2, 129, 20, 64, 4),
     (1, 8, 1000, 96, 32, 2),
-    (3, 3, 200, 30, 16, 2),   # C = 48: 16-channel tiles
+    (3, 3, 200, 30, 16, 2),   # C = 48: one head per tile
+    (1, 4, 600, 1024, 64, 4),  # D = 64 and a large route count
 ]
 
 
@@ -92,3 +93,15 @@ def test_mixer_degenerate_shapes():
     X, W_in, Wo, seeds = _case(2, 2, 0, 8, 16, 4, 1)  # N = 0: nothing to do
     O = flarepp.mixer_fwd(X.cuda(), W_in.cuda(), Wo.cuda(), seeds.cuda())
     assert O.numel() == 0
+
+
+def test_mixer_guard_bands_untouched():
+    """O is written inside its tensor only (the TMA stores clip rows beyond N)."""
+    X, W_in, Wo, seeds = _case(2, 4, 333, 48, 32, 4, 9)
+    band = 4096
+    buf = torch.full((X.numel() + 2 * band,), 5.0, dtype=X.dtype, device="cuda")
+    O = buf[band:band + X.numel()].view(X.shape)
+    flarepp.mixer_fwd(X.cuda(), W_in.cuda(), Wo.cuda(), seeds.cuda(), O=O)
+    torch.cuda.synchronize()
+    assert torch.all(buf[:band] == 5.0) and torch.all(buf[-band:] == 5.0)
+    assert torch.isfinite(O.float()).all()
