@@ -15,6 +15,9 @@ What it computes (FLARE++ paper):
   * ``mixer``          -- the FLARE++ token-mixing layer (Fig. 1; eqs. flarepp_query_synthesis
                           and flarepp_mixer): K, V, K~, V~ = X W^T split into heads, the routing
                           chain, then O = merge(Y) Wo^T; the projections are numpy matmuls
+  * ``mixer_bwd``      -- the mixer layer's gradients: dO through the output projection (a
+                          numpy matmul), the chain's backward (``route_bwd``), the projections'
+                          weight gradients and dX (numpy matmuls)
   * ``sdpa_bwd``       -- the backward of one SDPA from its saved output and log-normaliser
                           (App. A.5): P = exp(S - L), c = <dO, O>, dV = P^T dO,
                           dS = P o (dO V^T - c), dK = s dS^T Q, dQ = s dS K
@@ -153,6 +156,37 @@ class Oracle:
         merged = Y.transpose(0, 2, 1, 3).reshape(B, N, C)  # merge(Y): heads side by side
         return merged @ Wo.T
 
+    def mixer_bwd(self, X, W_in, Wo, seeds, scale, dO):
+        """Gradients of ``mixer`` for the output gradient dO [B, N, C]: returns
+        (dX [B, N, C], dW_in [P*C, C], dWo [C, C], dseeds [H, M, D]). With P = 2 the projections
+        of K~, V~ are those of K, V, so each block collects both gradients."""
+        X, W_in, Wo, seeds, dO = (self._f64(a) for a in (X, W_in, Wo, seeds, dO))
+        B, N, C = X.shape
+        H, M, D = seeds.shape
+        P = W_in.shape[0] // C
+        proj = X @ W_in.T
+
+        def heads(T):  # [B, N, C] -> [B, H, N, D]
+            return np.ascontiguousarray(T.reshape(B, N, H, D).transpose(0, 2, 1, 3))
+
+        def merge(T):  # [B, H, N, D] -> [B, N, C]
+            return T.transpose(0, 2, 1, 3).reshape(B, N, C)
+
+        K, V = heads(proj[..., :C]), heads(proj[..., C:2 * C])
+        Kt, Vt = (heads(proj[..., 2 * C:3 * C]), heads(proj[..., 3 * C:])) if P == 4 else (K, V)
+        _, _, Y = self.route(seeds, Kt, Vt, K, V, scale)
+        Ym = merge(Y)
+        # O = merge(Y) Wo^T
+        dWo = np.einsum("bno,bni->oi", dO, Ym)
+        dY = heads(dO @ Wo)
+        dseeds, dKt, dVt, dK, dV = self.route_bwd(seeds, Kt, Vt, K, V, scale, dY)
+        blocks = [dK, dV, dKt, dVt] if P == 4 else [dK + dKt, dV + dVt]
+        dproj = np.concatenate([merge(g) for g in blocks], axis=-1)  # [B, N, P*C]
+        # proj = X W_in^T
+        dW_in = np.einsum("bnr,bnc->rc", dproj, X)
+        dX = dproj @ W_in
+        return dX, dW_in, dWo, dseeds
+
     def sdpa_bwd(self, q, k, v, out, lse, dout, scale):
         """Backward of ``sdpa`` (App. A.5) from the forward's ``out`` and ``lse``.
 
@@ -246,6 +280,10 @@ def mixer(X, W_in, Wo, seeds, scale):
     return default().mixer(X, W_in, Wo, seeds, scale)
 
 
+def mixer_bwd(X, W_in, Wo, seeds, scale, dO):
+    return default().mixer_bwd(X, W_in, Wo, seeds, scale, dO)
+
+
 def sdpa_bwd(q, k, v, out, lse, dout, scale):
     return default().sdpa_bwd(q, k, v, out, lse, dout, scale)
 
@@ -268,4 +306,4 @@ def build() -> str:
 
 
 __all__ = ["Oracle", "default", "sdpa", "route", "flare", "encode_sharded", "mixer",
-           "sdpa_bwd", "route_bwd", "max_threads", "set_threads", "build"]
+           "mixer_bwd", "sdpa_bwd", "route_bwd", "max_threads", "set_threads", "build"]

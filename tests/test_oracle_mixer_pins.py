@@ -91,3 +91,59 @@ def test_shared_projection_layer():
     s = 0.4
     np.testing.assert_allclose(oracle.mixer(X, W2, Wo, seeds, s),
                                oracle.mixer(X, W4, Wo, seeds, s), atol=0)
+
+
+def _torch_mixer_grads(X, W_in, Wo, seeds, s, dO):
+    t = lambda a: torch.tensor(np.asarray(a, dtype=np.float64), requires_grad=True)
+    tX, tW, tWo, ts = t(X), t(W_in), t(Wo), t(seeds)
+    B, N, C = tX.shape
+    H, M, D = ts.shape
+    P = tW.shape[0] // C
+    proj = [F.linear(tX, tW[i * C:(i + 1) * C]) for i in range(P)]
+    split = lambda T: T.reshape(B, N, H, D).transpose(1, 2)
+    K, V = split(proj[0]), split(proj[1])
+    Kt, Vt = (split(proj[2]), split(proj[3])) if P == 4 else (K, V)
+    Qs = ts.unsqueeze(0).expand(B, H, M, D)
+    Q = F.scaled_dot_product_attention(Qs, Kt, Vt, scale=s)
+    Z = F.scaled_dot_product_attention(Q, K, V, scale=s)
+    Y = F.scaled_dot_product_attention(K, Q, Z, scale=s)
+    O = F.linear(Y.transpose(1, 2).reshape(B, N, C), tWo)
+    O.backward(torch.from_numpy(np.asarray(dO, dtype=np.float64)))
+    return tuple(a.grad.numpy() for a in (tX, tW, tWo, ts))
+
+
+def test_mixer_bwd_vs_torch_autograd():
+    rng = np.random.default_rng(31)
+    for (B, H, N, M, D, P) in [(2, 2, 30, 5, 4, 4), (1, 3, 25, 7, 4, 2), (2, 2, 17, 4, 8, 4)]:
+        X, W_in, Wo, seeds = _case(B, H, N, M, D, rng, P)
+        dO = rng.standard_normal(X.shape)
+        s = 1.0 / math.sqrt(D)
+        mine = oracle.mixer_bwd(X, W_in, Wo, seeds, s, dO)
+        ref = _torch_mixer_grads(X, W_in, Wo, seeds, s, dO)
+        for a, b in zip(mine, ref):
+            np.testing.assert_allclose(a, b, rtol=0, atol=1e-11 * max(1.0, np.abs(b).max()))
+
+
+def test_mixer_bwd_finite_differences():
+    rng = np.random.default_rng(32)
+    B, H, N, M, D, P = 1, 2, 6, 3, 2, 4
+    X, W_in, Wo, seeds = _case(B, H, N, M, D, rng, P)
+    dO = rng.standard_normal(X.shape)
+    s = 0.6
+    grads = oracle.mixer_bwd(X, W_in, Wo, seeds, s, dO)
+    ins = [X, W_in, Wo, seeds]
+    loss = lambda xs: float(np.sum(dO * oracle.mixer(*xs, s)))
+    h = 1e-5
+    for which in range(4):
+        fd = np.zeros_like(ins[which])
+        flat = ins[which].reshape(-1)
+        for i in range(flat.size):
+            keep = flat[i]
+            flat[i] = keep + h
+            lp = loss(ins)
+            flat[i] = keep - h
+            lm = loss(ins)
+            flat[i] = keep
+            fd.reshape(-1)[i] = (lp - lm) / (2 * h)
+        np.testing.assert_allclose(grads[which], fd, rtol=0,
+                                   atol=1e-7 * max(1.0, np.abs(fd).max()))
