@@ -237,6 +237,38 @@ FLAREPP_API flarepp_status flarepp_mixer_fwd_profiled(const flarepp_shape* shape
                                                       void* const* events, int n_events);
 
 /*
+ * Training the mixer layer. flarepp_mixer_fwd_train is flarepp_mixer_fwd that also fills
+ * `saved` (flarepp_mixer_saved_bytes(shape, n_proj) bytes of device memory, 16-byte aligned,
+ * disjoint from the workspace; layout private) with the chain's saved state and Y.
+ * flarepp_mixer_bwd then computes, for the output gradient dO [B, N, C]:
+ *   dX [B, N, C], dW_in [n_proj * C, C], dWo [C, C] (both out x in, like the weights) and
+ *   dseeds [H, M, D],
+ * all bf16, written (not accumulated): dO through the output projection (dWo = dO^T merge(Y),
+ * dY = split(dO Wo)), the chain's backward (App. A.5), then the projections' backward
+ * (dW_in = dP^T X, dX = dP W_in, the gradients of tied projections added for n_proj = 2).
+ * The projections are recomputed from X. workspace: flarepp_mixer_bwd_workspace_bytes(shape,
+ * n_proj) bytes, 256-byte aligned (its first 4 bytes are the device status word). Outputs
+ * must be 16-byte aligned and disjoint from each other and from the inputs. Degenerate
+ * shapes (N, M or B*H zero) write zeros to every non-empty gradient. Errors as for
+ * flarepp_mixer_fwd.
+ */
+FLAREPP_API size_t flarepp_mixer_saved_bytes(const flarepp_shape* shape, int n_proj);
+FLAREPP_API flarepp_status flarepp_mixer_fwd_train(const flarepp_shape* shape, int n_proj,
+                                                   const void* X, const void* W_in,
+                                                   const void* Wo, const void* seeds,
+                                                   float scale, void* O, void* saved,
+                                                   size_t saved_bytes, void* workspace,
+                                                   size_t workspace_bytes, void* stream);
+FLAREPP_API size_t flarepp_mixer_bwd_workspace_bytes(const flarepp_shape* shape, int n_proj);
+FLAREPP_API flarepp_status flarepp_mixer_bwd(const flarepp_shape* shape, int n_proj,
+                                             const void* X, const void* W_in, const void* Wo,
+                                             const void* seeds, float scale, const void* saved,
+                                             size_t saved_bytes, const void* dO, void* dX,
+                                             void* dW_in, void* dWo, void* dseeds,
+                                             void* workspace, size_t workspace_bytes,
+                                             void* stream);
+
+/*
  * Bytes of the state a training forward keeps for the backward (App. A.5): float32 Q and Z
  * [B, H, M, D] and the base-2 log-normalisers of the three calls,
  * L = log2 sum_j 2^(scale * log2(e) <a, b_j>), for calls 1 and 2 [B, H, M] and call 3

@@ -474,10 +474,23 @@ bool mixer_layout(const Plan& p, int n_proj, MixerLayout* L) {
     return true;
 }
 
+// State a training forward of the mixer keeps for its backward: the chain's saved state,
+// then Y [B][H][N][D] bf16.
+struct MixerSaved {
+    size_t off_y, total;
+};
+
+MixerSaved mixer_saved(const Plan& p) {
+    MixerSaved m;
+    m.off_y = align_up(saved_layout(p).total, kWsAlign);
+    m.total = align_up(m.off_y + (size_t)p.BH * (size_t)p.N * (size_t)p.D * 2, kWsAlign);
+    return m;
+}
+
 flarepp_status mixer_impl(const flarepp_shape* shape, int n_proj, const void* X, const void* W_in,
                           const void* Wo, const void* seeds, float scale, void* O,
                           void* workspace, size_t workspace_bytes, void* stream,
-                          void* const* events = nullptr) {
+                          void* const* events = nullptr, char* saved = nullptr) {
     Plan p;
     flarepp_status stt = make_plan(shape, &p);
     if (stt != FLAREPP_OK) return stt;
@@ -520,10 +533,11 @@ flarepp_status mixer_impl(const flarepp_shape* shape, int n_proj, const void* X,
         tc_projection(p.B, p.N, p.H, p.D, n_proj, X, W_in, proj, status, st) != cudaSuccess ||
         !mark(1))
         return FLAREPP_ERR_CUDA;
-    // the routing chain; the shared variant reads K, V as K~, V~ (App. C.2)
-    void* Y = ws + L.off_y;
+    // the routing chain; the shared variant reads K, V as K~, V~ (App. C.2). A training
+    // forward keeps Y and the chain's state in `saved`.
+    void* Y = saved ? saved + mixer_saved(p).off_y : ws + L.off_y;
     stt = route_impl(shape, seeds, proj[2], proj[3], proj[0], proj[1], scale, Y, workspace,
-                     p.total, stream, nullptr, nullptr, nullptr, 0, false);
+                     p.total, stream, nullptr, nullptr, nullptr, 0, false, saved);
     if (stt != FLAREPP_OK) return stt;
     // O = merge(Y) Wo^T
     if (!mark(2) ||
@@ -533,10 +547,178 @@ flarepp_status mixer_impl(const flarepp_shape* shape, int n_proj, const void* X,
     return FLAREPP_OK;
 }
 
+// Workspace of the mixer's backward: the chain's backward workspace first (its status word at
+// offset 0), then the recomputed projections, dY, the chain's gradients, the transposed
+// weights and the weight gradients' float32 partials.
+struct MixerBwdLayout {
+    size_t off_proj[4], off_dy, off_dproj[4], off_wot, off_wint, off_part, total;
+};
+
+MixerBwdLayout mixer_bwd_layout(const Plan& p, const BwdPlan& bp, int n_proj) {
+    MixerBwdLayout L;
+    const size_t tok = (size_t)p.BH * (size_t)p.N * (size_t)p.D * 2;
+    const int64_t C = p.H * p.D;
+    size_t off = align_up(bp.total, kWsAlign);
+    for (int i = 0; i < 4; ++i) {
+        L.off_proj[i] = off;
+        if (i < n_proj) off = align_up(off + tok, kWsAlign);
+    }
+    L.off_dy = off;
+    off = align_up(off + tok, kWsAlign);
+    for (int i = 0; i < 4; ++i) {
+        L.off_dproj[i] = off;
+        off = align_up(off + tok, kWsAlign);
+    }
+    L.off_wot = off;
+    off = align_up(off + (size_t)C * (size_t)C * 2, kWsAlign);
+    L.off_wint = off;
+    off = align_up(off + (size_t)C * 4 * (size_t)C * 2, kWsAlign);
+    L.off_part = off;
+    const size_t pa = wgrad_plan(p.B, p.N, C, C).part_bytes;
+    const size_t pb = wgrad_plan(p.B, p.N, 4 * C, C).part_bytes;
+    off = align_up(off + (pa > pb ? pa : pb), kWsAlign);
+    L.total = off;
+    return L;
+}
+
+flarepp_status mixer_bwd_impl(const flarepp_shape* shape, int n_proj, const void* X,
+                              const void* W_in, const void* Wo, const void* seeds, float scale,
+                              const void* saved, size_t saved_bytes, const void* dO, void* dX,
+                              void* dW_in, void* dWo, void* dseeds, void* workspace,
+                              size_t workspace_bytes, void* stream) {
+    Plan p;
+    flarepp_status stt = make_plan(shape, &p);
+    if (stt != FLAREPP_OK) return stt;
+    if (n_proj != 2 && n_proj != 4) return FLAREPP_ERR_INVALID_ARGUMENT;
+    if (p.dtype != FLAREPP_BF16) return FLAREPP_ERR_UNSUPPORTED;
+    if (!isfinite(scale)) return FLAREPP_ERR_INVALID_ARGUMENT;
+    cudaStream_t st = (cudaStream_t)stream;
+    const int64_t C = p.H * p.D;
+    const size_t x_bytes = (size_t)p.B * (size_t)p.N * (size_t)C * 2;
+    const size_t w_bytes = (size_t)n_proj * (size_t)C * (size_t)C * 2;
+    const size_t wo_bytes = (size_t)C * (size_t)C * 2;
+    const size_t seed_bytes = (size_t)p.H * (size_t)p.M * (size_t)p.D * 2;
+    // every pointer that a non-empty shape needs: present and aligned; outputs disjoint from
+    // the inputs
+    const void* ins[5] = {X, W_in, Wo, seeds, dO};
+    const size_t ib[5] = {x_bytes, w_bytes, wo_bytes, seed_bytes, x_bytes};
+    void* outs[4] = {dX, dW_in, dWo, dseeds};
+    const size_t ob[4] = {x_bytes, w_bytes, wo_bytes, seed_bytes};
+    for (int i = 0; i < 5; ++i)
+        if (ib[i] && (!ins[i] || !aligned16(ins[i]))) return FLAREPP_ERR_INVALID_ARGUMENT;
+    for (int i = 0; i < 4; ++i) {
+        if (ob[i] && (!outs[i] || !aligned16(outs[i]))) return FLAREPP_ERR_INVALID_ARGUMENT;
+        if (spans_overlap(ins, ib, 5, outs[i], ob[i])) return FLAREPP_ERR_INVALID_ARGUMENT;
+        for (int j = 0; j < i; ++j)
+            if (overlaps(outs[i], ob[i], outs[j], ob[j])) return FLAREPP_ERR_INVALID_ARGUMENT;
+    }
+    const bool work = p.BH && p.N && p.M;
+    if (!work) {  // every gradient that exists is zero
+        for (int i = 0; i < 4; ++i)
+            if (ob[i] && cudaMemsetAsync(outs[i], 0, ob[i], st) != cudaSuccess)
+                return FLAREPP_ERR_CUDA;
+        return FLAREPP_OK;
+    }
+    const MixerSaved ms = mixer_saved(p);
+    if (!saved || !aligned16(saved) || saved_bytes < ms.total) return FLAREPP_ERR_INVALID_ARGUMENT;
+    const BwdPlan bp = make_bwd_plan(p);
+    const MixerBwdLayout L = mixer_bwd_layout(p, bp, n_proj);
+    if (!workspace || ((uintptr_t)workspace % kWsAlign) != 0 || workspace_bytes < L.total)
+        return FLAREPP_ERR_WORKSPACE;
+    char* ws = (char*)workspace;
+    int* status = (int*)(ws + bp.off_status);
+    const char* sv = (const char*)saved;
+    const void* Y = sv + ms.off_y;
+    if (cudaMemsetAsync(status, 0, sizeof(int32_t), st) != cudaSuccess) return FLAREPP_ERR_CUDA;
+    void* proj[4];
+    for (int i = 0; i < 4; ++i) proj[i] = ws + L.off_proj[i < n_proj ? i : i - 2];
+    void* dY = ws + L.off_dy;
+    void* dproj[4];
+    for (int i = 0; i < 4; ++i) dproj[i] = ws + L.off_dproj[i];
+    void* WoT = ws + L.off_wot;
+    void* WinT = ws + L.off_wint;
+    float* part = (float*)(ws + L.off_part);
+    const int fold = 4 / n_proj;
+    cudaError_t e;
+    // the weights transposed (W_in repeated for tied projections: K~, V~ use W_K, W_V)
+    if ((e = transpose_bf16(Wo, C, C, 1, WoT, st)) != cudaSuccess ||
+        (e = transpose_bf16(W_in, n_proj * C, C, fold, WinT, st)) != cudaSuccess)
+        return FLAREPP_ERR_CUDA;
+    // the projections again (cheaper to recompute than to keep), and dY = split(dO Wo)
+    void* dys[4] = {dY, dY, dY, dY};
+    if (tc_projection(p.B, p.N, p.H, p.D, n_proj, X, W_in, proj, status, st) != cudaSuccess ||
+        tc_projection(p.B, p.N, p.H, p.D, 1, dO, WoT, dys, status, st) != cudaSuccess)
+        return FLAREPP_ERR_CUDA;
+    // dWo = dO^T merge(Y)
+    WgradSource sdo{0, 1, {dO, dO, dO, dO}};
+    WgradSource sy{1, 1, {Y, Y, Y, Y}};
+    if (tc_wgrad(p.B, p.N, p.H, p.D, sdo, sy, C, C, C, 1, part, dWo, status, st) != cudaSuccess)
+        return FLAREPP_ERR_CUDA;
+    // the chain's backward (App. A.5)
+    if (route_bwd(p, bp, seeds, proj[2], proj[3], proj[0], proj[1], scale, Y, dY, sv, dseeds,
+                  dproj[2], dproj[3], dproj[0], dproj[1], ws, st) != cudaSuccess)
+        return FLAREPP_ERR_CUDA;
+    // dW_in = dP^T X (tied projections fold their two gradients), dX = sum_p dP_p W_p
+    WgradSource sdp{1, 4, {dproj[0], dproj[1], dproj[2], dproj[3]}};
+    WgradSource sx{0, 1, {X, X, X, X}};
+    if (tc_wgrad(p.B, p.N, p.H, p.D, sdp, sx, 4 * C, C, n_proj * C, fold, part, dW_in, status,
+                 st) != cudaSuccess)
+        return FLAREPP_ERR_CUDA;
+    const void* dps[4] = {dproj[0], dproj[1], dproj[2], dproj[3]};
+    if (tc_heads_projection(p.B, p.N, p.H, p.D, 4, dps, WinT, dX, status, st) != cudaSuccess)
+        return FLAREPP_ERR_CUDA;
+    return FLAREPP_OK;
+}
+
 }  // namespace
 }  // namespace flarepp
 
 extern "C" {
+
+size_t flarepp_mixer_saved_bytes(const flarepp_shape* shape, int n_proj) {
+    flarepp::Plan p;
+    if (flarepp::make_plan(shape, &p) != FLAREPP_OK) return 0;
+    if ((n_proj != 2 && n_proj != 4) || p.dtype != FLAREPP_BF16) return 0;
+    if (p.BH == 0 || p.N == 0 || p.M == 0) return 0;
+    return flarepp::mixer_saved(p).total;
+}
+
+flarepp_status flarepp_mixer_fwd_train(const flarepp_shape* shape, int n_proj, const void* X,
+                                       const void* W_in, const void* Wo, const void* seeds,
+                                       float scale, void* O, void* saved, size_t saved_bytes,
+                                       void* workspace, size_t workspace_bytes, void* stream) {
+    flarepp::Plan p;
+    const flarepp_status stt = flarepp::make_plan(shape, &p);
+    if (stt != FLAREPP_OK) return stt;
+    if (p.dtype == FLAREPP_BF16 && p.BH && p.N && p.M) {
+        const size_t need = flarepp::mixer_saved(p).total;
+        if (!saved || !flarepp::aligned16(saved) || saved_bytes < need)
+            return FLAREPP_ERR_INVALID_ARGUMENT;
+        if (flarepp::overlaps(saved, need, workspace, workspace_bytes))
+            return FLAREPP_ERR_INVALID_ARGUMENT;
+    } else {
+        saved = nullptr;
+    }
+    return flarepp::mixer_impl(shape, n_proj, X, W_in, Wo, seeds, scale, O, workspace,
+                               workspace_bytes, stream, nullptr, (char*)saved);
+}
+
+size_t flarepp_mixer_bwd_workspace_bytes(const flarepp_shape* shape, int n_proj) {
+    flarepp::Plan p;
+    if (flarepp::make_plan(shape, &p) != FLAREPP_OK) return 0;
+    if ((n_proj != 2 && n_proj != 4) || p.dtype != FLAREPP_BF16) return 0;
+    if (p.BH == 0 || p.N == 0 || p.M == 0) return 0;
+    return flarepp::mixer_bwd_layout(p, flarepp::make_bwd_plan(p), n_proj).total;
+}
+
+flarepp_status flarepp_mixer_bwd(const flarepp_shape* shape, int n_proj, const void* X,
+                                 const void* W_in, const void* Wo, const void* seeds, float scale,
+                                 const void* saved, size_t saved_bytes, const void* dO, void* dX,
+                                 void* dW_in, void* dWo, void* dseeds, void* workspace,
+                                 size_t workspace_bytes, void* stream) {
+    return flarepp::mixer_bwd_impl(shape, n_proj, X, W_in, Wo, seeds, scale, saved, saved_bytes,
+                                   dO, dX, dW_in, dWo, dseeds, workspace, workspace_bytes, stream);
+}
 
 size_t flarepp_mixer_workspace_bytes(const flarepp_shape* shape, int n_proj) {
     flarepp::Plan p;

@@ -126,6 +126,36 @@ cudaError_t tc_projection(int64_t B, int64_t N, int64_t H, int64_t D, int P, con
 // merge(Y) times Wo [C][C] (out x in) into O [B][N][C], Y read head by head [B][H][N][D].
 cudaError_t tc_output_projection(int64_t B, int64_t N, int64_t H, int64_t D, const void* Y,
                                  const void* Wo, void* O, int* status, cudaStream_t st);
+// n_a head-layout tensors As[p] [B][H][N][D] side by side (channel p*C + h*D + d) times
+// W [C][n_a * C] (out x in) into O [B][N][C].
+cudaError_t tc_heads_projection(int64_t B, int64_t N, int64_t H, int64_t D, int n_a,
+                                const void* const* As, const void* W, void* O, int* status,
+                                cudaStream_t st);
+
+// ---- the mixer's weight gradients (tc_wgrad.cu), bf16
+// A channel source: `heads` = 1 for n tensors [B][H][N][D] side by side (channel p*C + h*D + d),
+// 0 for one matrix [B][N][C].
+struct WgradSource {
+    int heads;
+    int n;
+    const void* t[4];
+};
+struct WgradPlan {
+    int NT;
+    int64_t row_tiles, col_tiles, chunk_len, chunks_per_b, n_chunks;
+    size_t part_bytes;  // float32 partials [n_chunks][R][Cc]
+};
+WgradPlan wgrad_plan(int64_t B, int64_t N, int64_t R, int64_t Cc);
+// dW [R_out][Cc] (bf16) = sum over tokens of A(t, r) B(t, c) for r < R, c < Cc, the rows
+// r + k * R_out (k < fold) added into row r; `part` holds the plan's partials.
+cudaError_t tc_wgrad(int64_t B, int64_t N, int64_t H, int64_t D, const WgradSource& a,
+                     const WgradSource& b, int64_t R, int64_t Cc, int64_t R_out, int fold,
+                     float* part, void* dW, int* status, cudaStream_t st);
+// dst [Cc][rep * R] = the transpose of src [R][Cc] repeated rep times along its columns
+cudaError_t transpose_bf16(const void* src, int64_t R, int64_t Cc, int rep, void* dst,
+                           cudaStream_t st);
+// dst += src, elementwise over n bf16 values (float32 sum, rounded once)
+cudaError_t add_bf16(void* dst, const void* src, int64_t n, cudaStream_t st);
 
 // ---- tensor-core kernels (tc_kernels.cu), bf16 inputs
 // Encode call 1 (A = seeds) or call 2 (A = Q operand) into the chunk partials.

@@ -7,7 +7,9 @@
 //     projection), each split into H heads of width D and written to its [B][H][N][D] tensor,
 //     the layout the routing chain reads.
 //   output (MODE 1): A = merge(Y), read head by head straight from Y [B][H][N][D] (no merged
-//     copy is made), B = Wo [C][C]; O [B][N][C].
+//     copy is made), B = Wo [C][C]; O [B][N][C]. The same pass with up to four A tensors side
+//     by side (A channel p*C + h*D + d from tensor p) computes dX = sum_p dP_p W_p of the
+//     mixer's backward with B = W_in^T.
 //
 // The contraction over C runs in slices of D channels (one head), the unit that both A
 // layouts share; each slice is one TMA box of 128 tokens x D for A and NT channels x D for B,
@@ -66,6 +68,7 @@ struct GCfg {
 
 struct GemmParams {
     int64_t B, N, H, C;
+    int n_a;            // MODE 1: A tensors side by side (the contraction runs over n_a * C)
     int64_t n_out;      // output channels (P * C, or C)
     int NT;             // output channels per tile (whole heads, <= 256, divides C)
     uint32_t idesc;     // MMA instruction descriptor for M = 128, N = NT
@@ -118,7 +121,9 @@ __device__ __forceinline__ uint32_t pack_bf16(float lo, float hi) {
 
 template <int D, int MODE>
 __global__ void __launch_bounds__(kThreads, 1)
-    tc_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
+    tc_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmA1,
+                   const __grid_constant__ CUtensorMap tmA2, const __grid_constant__ CUtensorMap tmA3,
+                   const __grid_constant__ CUtensorMap tmB,
                    const __grid_constant__ CUtensorMap tmO0, const __grid_constant__ CUtensorMap tmO1,
                    const __grid_constant__ CUtensorMap tmO2, const __grid_constant__ CUtensorMap tmO3,
                    const GemmParams prm) {
@@ -140,7 +145,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     const uint32_t swritten0 = sfree0 + 8u * kEpiGroups;   // [kEpiGroups], count 128
     const int warp = threadIdx.x >> 5;
     const int lane = threadIdx.x & 31;
-    const int slices = (int)(prm.C / D);
+    const int slices = (int)(prm.C / D) * (MODE == 1 ? prm.n_a : 1);
 
     if (threadIdx.x == 0) {
         for (int st = 0; st < kS; ++st) {
@@ -159,6 +164,11 @@ __global__ void __launch_bounds__(kThreads, 1)
         *abort_flag = 0;
         fence_mbar_init();
         prefetch_tmap(&tmA);
+        if (MODE == 1 && prm.n_a > 1) {
+            prefetch_tmap(&tmA1);
+            prefetch_tmap(&tmA2);
+            prefetch_tmap(&tmA3);
+        }
         prefetch_tmap(&tmB);
     }
     if (warp == 1) {
@@ -187,12 +197,16 @@ __global__ void __launch_bounds__(kThreads, 1)
                 if (elect_one()) {
                     const uint32_t dst = smem_u32(smem + st * C::kStage);
                     mbar_expect_tx(full0 + 8u * st, bytes);
-                    if (MODE == 0)
+                    if (MODE == 0) {
                         tma_load_3d(dst, &tmA, h * D, (int)(T.rt * kRows), (int)T.b,
                                     full0 + 8u * st);
-                    else
-                        tma_load_3d(dst, &tmA, 0, (int)(T.rt * kRows), (int)(T.b * prm.H + h),
+                    } else {
+                        // slice h: head h % H of A tensor h / H
+                        const int p = h / (int)prm.H, hh = h % (int)prm.H;
+                        const CUtensorMap* ma = p == 0 ? &tmA : p == 1 ? &tmA1 : p == 2 ? &tmA2 : &tmA3;
+                        tma_load_3d(dst, ma, 0, (int)(T.rt * kRows), (int)(T.b * prm.H + hh),
                                     full0 + 8u * st);
+                    }
                     tma_load_3d(dst + C::kASlice, &tmB, h * D, (int)(T.ct * prm.NT), 0,
                                 full0 + 8u * st);
                 }
@@ -365,7 +379,7 @@ bool make_map(CUtensorMap* m, const void* base, int64_t D, int64_t inner, int64_
 }
 
 template <int D, int MODE>
-cudaError_t launch(const CUtensorMap& a, const CUtensorMap& b, const CUtensorMap* o,
+cudaError_t launch(const CUtensorMap* a, const CUtensorMap& b, const CUtensorMap* o,
                    const GemmParams& prm, cudaStream_t st) {
     using Cf = GCfg<D>;
     static cudaError_t attr = cudaFuncSetAttribute(
@@ -376,8 +390,8 @@ cudaError_t launch(const CUtensorMap& a, const CUtensorMap& b, const CUtensorMap
     cudaGetDevice(&dev);
     cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
     const int64_t grid = prm.n_tiles < sms ? prm.n_tiles : sms;
-    tc_gemm_kernel<D, MODE><<<(unsigned)grid, kThreads, Cf::kSmem, st>>>(a, b, o[0], o[1], o[2],
-                                                                         o[3], prm);
+    tc_gemm_kernel<D, MODE><<<(unsigned)grid, kThreads, Cf::kSmem, st>>>(
+        a[0], a[1], a[2], a[3], b, o[0], o[1], o[2], o[3], prm);
     return cudaGetLastError();
 }
 
@@ -422,10 +436,12 @@ cudaError_t tc_projection(int64_t B, int64_t N, int64_t H, int64_t D, int P, con
     prm.n_tiles = B * prm.row_tiles * prm.col_tiles;
     for (int p = 0; p < 4; ++p) prm.out[p] = (__nv_bfloat16*)outs[p < P ? p : p - 2];
     prm.status = status;
-    CUtensorMap ma, mb, mo[4];
-    if (!make_map(&ma, X, D, C, N, B, kRows) ||
+    CUtensorMap ma[4], mb, mo[4];
+    if (!make_map(&ma[0], X, D, C, N, B, kRows) ||
         !make_map(&mb, W_in, D, C, prm.n_out, 1, (uint32_t)prm.NT))
         return cudaErrorInvalidValue;
+    ma[1] = ma[2] = ma[3] = ma[0];
+    prm.n_a = 1;
     for (int p = 0; p < 4; ++p)
         if (!make_store_map(&mo[p], prm.out[p], D, N, B * H, (uint32_t)D))
             return cudaErrorInvalidValue;
@@ -439,12 +455,21 @@ cudaError_t tc_projection(int64_t B, int64_t N, int64_t H, int64_t D, int P, con
 
 cudaError_t tc_output_projection(int64_t B, int64_t N, int64_t H, int64_t D, const void* Y,
                                  const void* Wo, void* O, int* status, cudaStream_t st) {
+    const void* ys[1] = {Y};
+    return tc_heads_projection(B, N, H, D, 1, ys, Wo, O, status, st);
+}
+
+cudaError_t tc_heads_projection(int64_t B, int64_t N, int64_t H, int64_t D, int n_a,
+                                const void* const* As, const void* W, void* O, int* status,
+                                cudaStream_t st) {
     const int64_t C = H * D;
+    if (n_a < 1 || n_a > 4) return cudaErrorInvalidValue;
     GemmParams prm{};
     prm.B = B;
     prm.N = N;
     prm.H = H;
     prm.C = C;
+    prm.n_a = n_a;
     prm.n_out = C;
     prm.NT = tile_channels(H, D);
     prm.idesc = idesc_bf16_f32(kRows, prm.NT, false, false);
@@ -453,9 +478,11 @@ cudaError_t tc_output_projection(int64_t B, int64_t N, int64_t H, int64_t D, con
     prm.n_tiles = B * prm.row_tiles * prm.col_tiles;
     prm.out[0] = prm.out[1] = prm.out[2] = prm.out[3] = (__nv_bfloat16*)O;
     prm.status = status;
-    CUtensorMap ma, mb, mo[4];
-    if (!make_map(&ma, Y, D, D, N, B * H, kRows) ||
-        !make_map(&mb, Wo, D, C, C, 1, (uint32_t)prm.NT) ||
+    CUtensorMap ma[4], mb, mo[4];
+    for (int p = 0; p < 4; ++p)
+        if (!make_map(&ma[p], As[p < n_a ? p : 0], D, D, N, B * H, kRows))
+            return cudaErrorInvalidValue;
+    if (!make_map(&mb, W, D, n_a * C, C, 1, (uint32_t)prm.NT) ||
         !make_store_map(&mo[0], O, C, N, B, (uint32_t)D))
         return cudaErrorInvalidValue;
     mo[1] = mo[2] = mo[3] = mo[0];

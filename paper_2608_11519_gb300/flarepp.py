@@ -25,6 +25,8 @@ EXPORTED = ("flarepp_route_workspace_bytes", "flarepp_route_fwd", "flarepp_route
             "flarepp_route_fwd_profiled", "flarepp_route_fwd_noalloc",
             "flarepp_flare_fwd", "flarepp_route_host_buffer_bytes", "flarepp_route_fwd_host",
             "flarepp_mixer_workspace_bytes", "flarepp_mixer_fwd", "flarepp_mixer_fwd_profiled",
+            "flarepp_mixer_saved_bytes", "flarepp_mixer_fwd_train",
+            "flarepp_mixer_bwd_workspace_bytes", "flarepp_mixer_bwd",
             "flarepp_route_saved_bytes", "flarepp_route_fwd_train",
             "flarepp_route_bwd_workspace_bytes", "flarepp_route_bwd",
             "flarepp_route_device_status", "flarepp_status_string", "flarepp_version")
@@ -90,6 +92,16 @@ def load(path: str = None):
     lib.flarepp_mixer_fwd_profiled.argtypes = [sp, ctypes.c_int, vp, vp, vp, vp, ctypes.c_float,
                                                vp, vp, sz, vp, ctypes.POINTER(ctypes.c_void_p),
                                                ctypes.c_int]
+    lib.flarepp_mixer_saved_bytes.restype = sz
+    lib.flarepp_mixer_saved_bytes.argtypes = [sp, ctypes.c_int]
+    lib.flarepp_mixer_fwd_train.restype = ctypes.c_int
+    lib.flarepp_mixer_fwd_train.argtypes = [sp, ctypes.c_int, vp, vp, vp, vp, ctypes.c_float, vp,
+                                            vp, sz, vp, sz, vp]
+    lib.flarepp_mixer_bwd_workspace_bytes.restype = sz
+    lib.flarepp_mixer_bwd_workspace_bytes.argtypes = [sp, ctypes.c_int]
+    lib.flarepp_mixer_bwd.restype = ctypes.c_int
+    lib.flarepp_mixer_bwd.argtypes = [sp, ctypes.c_int, vp, vp, vp, vp, ctypes.c_float, vp, sz,
+                                      vp, vp, vp, vp, vp, vp, sz, vp]
     lib.flarepp_route_saved_bytes.restype = sz
     lib.flarepp_route_saved_bytes.argtypes = [sp]
     lib.flarepp_route_fwd_train.restype = ctypes.c_int
@@ -376,6 +388,73 @@ def mixer_fwd(X, W_in, Wo, seeds, scale=None, O=None, workspace=None, stream=Non
     if rc != OK:
         raise FlareppError(rc, "flarepp_mixer_fwd")
     return O
+
+
+def _mixer_shape(X, W_in, Wo, seeds):
+    for t in (X, W_in, Wo, seeds):
+        if not isinstance(t, torch.Tensor) or not t.is_contiguous():
+            raise ValueError("inputs must be contiguous torch tensors")
+        if t.dtype != torch.bfloat16:
+            raise TypeError("the mixer takes bfloat16 tensors")
+    if X.device.type != "cuda":
+        raise ValueError("the mixer takes device tensors")
+    B, N, C = X.shape
+    H, M, D = seeds.shape
+    if H * D != C or tuple(Wo.shape) != (C, C) or W_in.shape[1] != C or \
+            W_in.shape[0] not in (2 * C, 4 * C):
+        raise ValueError("expected X [B,N,C], W_in [P*C,C], Wo [C,C], seeds [H,M,D], C = H*D")
+    return make_shape(B, H, N, M, D, torch.bfloat16), W_in.shape[0] // C
+
+
+def mixer_fwd_train(X, W_in, Wo, seeds, scale=None, O=None, saved=None, workspace=None,
+                    stream=None):
+    """The mixer layer's forward that keeps its backward's state. Returns (O, saved)."""
+    lib = load()
+    shape, P = _mixer_shape(X, W_in, Wo, seeds)
+    if scale is None:
+        scale = 1.0 / math.sqrt(shape.D)
+    if O is None:
+        O = torch.empty_like(X)
+    sbytes = int(lib.flarepp_mixer_saved_bytes(ctypes.byref(shape), P))
+    if saved is None or saved.numel() < sbytes:
+        saved = torch.empty(max(sbytes, 1), dtype=torch.uint8, device=X.device)
+    nbytes = int(lib.flarepp_mixer_workspace_bytes(ctypes.byref(shape), P))
+    ws = (workspace if isinstance(workspace, Workspace) else Workspace()).get(nbytes, X.device)
+    st = stream if stream is not None else torch.cuda.current_stream(X.device)
+    rc = lib.flarepp_mixer_fwd_train(ctypes.byref(shape), P, _ptr(X), _ptr(W_in), _ptr(Wo),
+                                     _ptr(seeds), float(scale), _ptr(O), _ptr(saved), sbytes,
+                                     None if ws is None else ctypes.c_void_p(ws.data_ptr()),
+                                     nbytes, ctypes.c_void_p(st.cuda_stream))
+    if rc != OK:
+        raise FlareppError(rc, "flarepp_mixer_fwd_train")
+    return O, saved
+
+
+def mixer_bwd(X, W_in, Wo, seeds, saved, dO, scale=None, grads=None, workspace=None,
+              stream=None):
+    """The mixer layer's backward from :func:`mixer_fwd_train`'s ``saved``: returns
+    (dX, dW_in, dWo, dseeds) in bf16; ``grads`` may supply those four output tensors."""
+    lib = load()
+    shape, P = _mixer_shape(X, W_in, Wo, seeds)
+    if tuple(dO.shape) != tuple(X.shape) or dO.dtype != X.dtype or not dO.is_contiguous():
+        raise ValueError("dO must be a contiguous tensor of X's shape and dtype")
+    if scale is None:
+        scale = 1.0 / math.sqrt(shape.D)
+    if grads is None:
+        grads = (torch.empty_like(X), torch.empty_like(W_in), torch.empty_like(Wo),
+                 torch.empty_like(seeds))
+    nbytes = int(lib.flarepp_mixer_bwd_workspace_bytes(ctypes.byref(shape), P))
+    ws = (workspace if isinstance(workspace, Workspace) else Workspace()).get(nbytes, X.device)
+    st = stream if stream is not None else torch.cuda.current_stream(X.device)
+    rc = lib.flarepp_mixer_bwd(ctypes.byref(shape), P, _ptr(X), _ptr(W_in), _ptr(Wo),
+                               _ptr(seeds), float(scale), _ptr(saved),
+                               saved.numel() if saved is not None else 0, _ptr(dO),
+                               *(_ptr(g) for g in grads),
+                               None if ws is None else ctypes.c_void_p(ws.data_ptr()), nbytes,
+                               ctypes.c_void_p(st.cuda_stream))
+    if rc != OK:
+        raise FlareppError(rc, "flarepp_mixer_bwd")
+    return grads
 
 
 def route_fwd_train(seeds, Kt, Vt, K, V, scale=None, Y=None, saved=None, workspace=None,

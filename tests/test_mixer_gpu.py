@@ -105,3 +105,38 @@ def test_mixer_guard_bands_untouched():
     torch.cuda.synchronize()
     assert torch.all(buf[:band] == 5.0) and torch.all(buf[-band:] == 5.0)
     assert torch.isfinite(O.float()).all()
+
+
+BWD_SHAPES = [
+    # B, H, N, M, D, P
+    (1, 8, 2000, 128, 32, 4),
+    (2, 2, 500, 64, 32, 4),
+    (1, 4, 300, 40, 16, 2),
+    (2, 2, 257, 20, 64, 4),
+    (1, 1, 130, 16, 32, 2),   # C = D: one head
+]
+
+
+@pytest.mark.parametrize("shape", BWD_SHAPES, ids=[str(s) for s in BWD_SHAPES])
+def test_mixer_bwd_matches_oracle(shape):
+    """The layer's gradients (App. A.5 through the projections) against the oracle; each
+    tensor within 2e-2 of its own scale, as for the chain's backward."""
+    B, H, N, M, D, P = shape
+    X, W_in, Wo, seeds = _case(B, H, N, M, D, P, 13)
+    g = torch.Generator().manual_seed(14)
+    dO = torch.randn(X.shape, generator=g).to(torch.bfloat16)
+    s = 1.0 / math.sqrt(D)
+    dev = [t.cuda() for t in (X, W_in, Wo, seeds)]
+    O, saved = flarepp.mixer_fwd_train(*dev, s)
+    grads = flarepp.mixer_bwd(*dev, saved, dO.cuda(), s)
+    torch.cuda.synchronize()
+    O_plain = flarepp.mixer_fwd(*dev, s)
+    torch.cuda.synchronize()
+    assert torch.equal(O, O_plain)
+    want = oracle.mixer_bwd(_np(X), _np(W_in), _np(Wo), _np(seeds), s, _np(dO))
+    for name, got, ref in zip(("dX", "dW_in", "dWo", "dseeds"), grads, want):
+        got = _np(got)
+        assert got.shape == ref.shape, name
+        bound = 2e-2 * max(1.0, float(np.abs(ref).max()))
+        err = float(np.abs(got - ref).max())
+        assert err <= bound, f"{name}: {err} > {bound}"
