@@ -222,7 +222,15 @@ def run_reference(args, w):
         return 0
     import oracle
     n = int(min(w.N, args.ref_tokens))
-    if args.variant.startswith("mixer"):
+    if args.variant == "mixer_train":
+        # the layer's forward and backward on one batch element
+        m = inputs.to_f64_numpy(inputs.make_mixer_inputs(w.with_(B=1, N=n), args.seed, "cpu"))
+        dO = np.random.default_rng(args.seed).standard_normal(m["X"].shape)
+        step = lambda: oracle.mixer_bwd(m["X"], m["W_in"], m["Wo"], m["seeds"], w.scale, dO)
+        heads = w.H
+        sample = (f"one batch element, N={n} tokens, H={w.H} heads of the {w.name} shape "
+                  f"(M={w.M}, D={w.D}), float64 oracle (forward and backward), per step")
+    elif args.variant.startswith("mixer"):
         # the whole layer on one batch element: all H heads of n tokens
         m = inputs.to_f64_numpy(inputs.make_mixer_inputs(
             w.with_(B=1, N=n), args.seed, "cpu", 2 if args.variant == "mixer_shared" else 4))
@@ -245,7 +253,8 @@ def run_reference(args, w):
     dt = (time.perf_counter() - t0) / args.steps
     value = heads * n / dt
     metric = {"flare": FLARE_METRIC, "train": TRAIN_METRIC, "mixer": MIXER_METRIC,
-              "mixer_shared": MIXER_METRIC}.get(args.variant, METRIC)
+              "mixer_shared": MIXER_METRIC,
+              "mixer_train": MIXER_TRAIN_METRIC}.get(args.variant, METRIC)
     line = {"impl": "reference", "metric": metric, "value": value, "unit": UNIT,
             "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
             "ms_per_step": dt * 1e3, "higher_is_better": True, "scaling": "weak",
@@ -496,6 +505,90 @@ def mixer_cpu_sample(w, target_s, seed, n_proj):
                       f"D={w.D}), float64, {dt:.2f} s"}
 
 
+MIXER_TRAIN_METRIC = ("routed tokens·heads/sec for a training step of the FLARE++ mixer layer "
+                      "(forward with saved state + backward); % of roofline")
+
+
+def run_mixer_train(args, w, flarepp, world, rank, dev, peaks, stream):
+    """A training step of the mixer layer: flarepp_mixer_fwd_train then flarepp_mixer_bwd, each
+    bracketed by CUDA events, on device-resident inputs and output gradient."""
+    x = inputs.make_mixer_inputs(w, args.seed + rank, device=dev, n_proj=4)
+    dO = inputs.make_output_grad(w.with_(H=1, D=w.H * w.D), args.seed + rank,
+                                 device=dev).reshape(x["X"].shape)
+    O = torch.empty_like(x["X"])
+    ws_f, ws_b = flarepp.Workspace(), flarepp.Workspace()
+    grads = (torch.empty_like(x["X"]), torch.empty_like(x["W_in"]), torch.empty_like(x["Wo"]),
+             torch.empty_like(x["seeds"]))
+    saved = None
+
+    def step(ev=None):
+        nonlocal saved
+        if ev:
+            ev[0].record(stream)
+        _, saved = flarepp.mixer_fwd_train(x["X"], x["W_in"], x["Wo"], x["seeds"], w.scale, O=O,
+                                           saved=saved, workspace=ws_f, stream=stream)
+        if ev:
+            ev[1].record(stream)
+        flarepp.mixer_bwd(x["X"], x["W_in"], x["Wo"], x["seeds"], saved, dO, w.scale,
+                          grads=grads, workspace=ws_b, stream=stream)
+        if ev:
+            ev[2].record(stream)
+
+    for _ in range(args.warmup):
+        step()
+    torch.cuda.synchronize(dev)
+    evs = [[torch.cuda.Event(enable_timing=True) for _ in range(3)] for _ in range(args.steps)]
+    clocks = ClockSampler()
+    if rank == 0:
+        clocks.start()
+        time.sleep(0.3)
+    t0 = torch.cuda.Event(enable_timing=True)
+    t1 = torch.cuda.Event(enable_timing=True)
+    barrier(world)
+    torch.cuda.synchronize(dev)
+    t0.record(stream)
+    for i in range(args.steps):
+        step(evs[i])
+    t1.record(stream)
+    torch.cuda.synchronize(dev)
+    barrier(world)
+    clk = clocks.stop(dev.index) if rank == 0 else None
+    ms = max_over_ranks(t0.elapsed_time(t1), world) / args.steps
+    fwd_ms = sum(e[0].elapsed_time(e[1]) for e in evs) / args.steps
+    bwd_ms = sum(e[1].elapsed_time(e[2]) for e in evs) / args.steps
+    tok = w.B * w.H * w.N
+    BN, C = w.B * w.N, w.H * w.D
+    # backward algorithmic flops: the chain's 30 BNMHD, and per token 2 C^2 (dY) + 2 C^2 (dWo)
+    # + 2 C (4C) each for dW_in and dX (the projections' recompute is not counted)
+    flops = 30.0 * tok * w.M * w.D + BN * (4.0 * C * C + 16.0 * C * C)
+    tc_peak = peaks["bf16_tflops_sustained"]
+    roof = {"bound": "tensor", "achieved": flops / (bwd_ms * 1e-3) / 1e12, "peak": tc_peak,
+            "unit": "TFLOP/s", "peak_kind": "bf16_tflops_sustained (" + peaks["source"] + ")"}
+    roof["frac"] = roof["achieved"] / roof["peak"]
+    roof["kernel"] = "mixer backward (all launches)"
+    roof["ms_per_launch"] = bwd_ms
+    roof["algorithmic_flops_per_launch"] = flops
+    roof["traffic"] = None
+    if rank == 0:
+        line = {
+            "metric": MIXER_TRAIN_METRIC, "value": tok * world / (ms * 1e-3), "unit": UNIT,
+            "n_gpus": world, "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+            "dtype": "bf16", "data": "synthetic",
+            "config": {"workload": w.name, "variant": "mixer_train", "B": w.B, "H": w.H,
+                       "N": w.N, "M": w.M, "D": w.D, "C": C, "projections": 4,
+                       "l2": "inputs larger than L2 (no flush)",
+                       "parallelism": f"replicas x{world}"},
+            "stage_ms": {"forward_train": fwd_ms, "backward": bwd_ms}, "roofline": roof,
+            "cpu_baseline": None, "e2e": None, "clocks": clk, "gpu_launches": None,
+        }
+        print(json.dumps(line), flush=True)
+    if world > 1:
+        import torch.distributed as dist
+        dist.destroy_process_group()
+    return 0
+
+
 def run_mixer(args, w, flarepp, world, rank, dev, peaks, stream):
     """The FLARE++ mixer layer (Fig. 1) on device-resident inputs, each stage bracketed by the
     library's own events."""
@@ -606,6 +699,9 @@ def run_ours(args, w):
     if args.variant in ("mixer", "mixer_shared"):
         del x, Y
         return run_mixer(args, w, flarepp, world, rank, dev, peaks, stream)
+    if args.variant == "mixer_train":
+        del x, Y
+        return run_mixer_train(args, w, flarepp, world, rank, dev, peaks, stream)
 
     ev_sets = [flarepp.StageEvents(stream) for _ in range(args.steps)]
     warm_ev = flarepp.StageEvents(stream)
@@ -738,7 +834,7 @@ def main():
     ap.add_argument("--workload", default="mesh3d", choices=sorted(inputs.WORKLOADS))
     ap.add_argument("--seed", type=int, default=0)
     ap.add_argument("--variant", choices=("flarepp", "shared", "flare", "train", "mixer",
-                                          "mixer_shared"),
+                                          "mixer_shared", "mixer_train"),
                     default="flarepp",
                     help="flarepp: the routing chain (default); shared: the chain with Kt, Vt "
                          "tied to K, V; flare: FLARE with fixed learned queries; train: the "
