@@ -249,3 +249,37 @@ def test_mixer_entry_sizes_and_rejects(lib):
     p = list(ptr)
     p[5] = None
     assert call(S(), ptrs=p) == E.ERR_WORKSPACE
+
+
+def test_mixer_training_entries_reject(lib):
+    E = flarepp
+    s = S(B=1, H=8, N=4096, M=64, D=32)
+    sb = lambda sh, p: lib.flarepp_mixer_saved_bytes(ctypes.byref(sh), p)
+    wb = lambda sh, p: lib.flarepp_mixer_bwd_workspace_bytes(ctypes.byref(sh), p)
+    assert sb(s, 4) > 8 * 4096 * 32 * 2 and wb(s, 4) > wb(s, 2) > 0
+    assert sb(s, 3) == 0 and wb(S(dtype=flarepp.F32), 4) == 0 and wb(S(N=0), 4) == 0
+    v = lambda x: ctypes.c_void_p(x) if x else None
+    base = [FAKE + (i + 1) * (1 << 36) for i in range(11)]
+
+    def bwd(shape, n_proj=4, ptrs=None, scale=0.25, saved_bytes=None):
+        p = base if ptrs is None else ptrs
+        # X W_in Wo seeds | saved | dO | dX dW_in dWo dseeds | workspace
+        return lib.flarepp_mixer_bwd(
+            ctypes.byref(shape), n_proj, *(v(x) for x in p[:4]), ctypes.c_float(scale), v(p[4]),
+            sb(shape, n_proj) if saved_bytes is None else saved_bytes, v(p[5]),
+            *(v(x) for x in p[6:10]), v(p[10]), wb(shape, n_proj), None)
+
+    assert bwd(S(dtype=flarepp.F32)) == E.ERR_UNSUPPORTED
+    assert bwd(S(), n_proj=3) == E.ERR_INVALID_ARGUMENT
+    assert bwd(S(), scale=float("nan")) == E.ERR_INVALID_ARGUMENT
+    for i in (0, 1, 2, 3, 5, 6, 7, 8, 9):
+        p = list(base)
+        p[i] = None
+        assert bwd(S(), ptrs=p) == E.ERR_INVALID_ARGUMENT, i
+    p = list(base)
+    p[6] = base[0] + 32  # dX overlaps X
+    assert bwd(S(), ptrs=p) == E.ERR_INVALID_ARGUMENT
+    assert bwd(S(), saved_bytes=16) == E.ERR_INVALID_ARGUMENT
+    p = list(base)
+    p[10] = None
+    assert bwd(S(), ptrs=p) == E.ERR_WORKSPACE
