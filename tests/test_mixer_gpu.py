@@ -140,3 +140,26 @@ def test_mixer_bwd_matches_oracle(shape):
         bound = 2e-2 * max(1.0, float(np.abs(ref).max()))
         err = float(np.abs(got - ref).max())
         assert err <= bound, f"{name}: {err} > {bound}"
+
+
+def test_mixer_full_size_pde2d():
+    """The mixer layer and its backward at the pde2d workload's full size (B = 4, H = 8,
+    N = 16,384, M = 128, D = 32), inputs from the shared input recipe."""
+    from paper_2608_11519_gb300 import inputs
+    w = inputs.get("pde2d")
+    m = inputs.make_mixer_inputs(w, 2)
+    md = {k: v.cuda() for k, v in m.items()}
+    args = (md["X"], md["W_in"], md["Wo"], md["seeds"])
+    g = torch.Generator().manual_seed(3)
+    dO = torch.randn(md["X"].shape, generator=g).to(torch.bfloat16)
+    O, saved = flarepp.mixer_fwd_train(*args, w.scale)
+    grads = flarepp.mixer_bwd(*args, saved, dO.cuda(), w.scale)
+    torch.cuda.synchronize()
+    f = inputs.to_f64_numpy(m)
+    want_O = oracle.mixer(f["X"], f["W_in"], f["Wo"], f["seeds"], w.scale)
+    want = oracle.mixer_bwd(f["X"], f["W_in"], f["Wo"], f["seeds"], w.scale, _np(dO))
+    for name, got, ref in zip(("O", "dX", "dW_in", "dWo", "dseeds"), (O,) + tuple(grads),
+                              (want_O,) + tuple(want)):
+        bound = 2e-2 * max(1.0, float(np.abs(ref).max()))
+        err = float(np.abs(_np(got) - ref).max())
+        assert err <= bound, f"{name}: {err} > {bound}"
