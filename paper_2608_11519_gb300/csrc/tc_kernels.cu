@@ -24,9 +24,10 @@
 //                 swizzled K/V or Q/Z) from a non-blocking poll between its own waits
 //   warps 4..19   four softmax warpgroups; warpgroup s serves stream s and copies its A tile
 //                 from smem into TMEM (four warps per SMSP hide each other's latencies)
-// The softmax keeps a reference max that is recomputed exactly only on a stream's first
-// item or when an item's probabilities sum past 2^48 (values stay far inside the fp32 and
-// bf16 ranges); otherwise P = 2^(c S - m) with the old reference.
+// The softmax keeps a reference max, set on a stream's first item (the item's exact maximum
+// in the encode, its first score in the decode) and recomputed exactly only when an item's
+// probabilities sum past 2^48 (values stay far inside the fp32 and bf16 ranges); otherwise
+// P = 2^(c S - m) with the old reference.
 // Every wait is bounded (2 s of %globaltimer): on expiry the kernel records
 // FLAREPP_ERR_TIMEOUT in the status word, every role leaves its loops, the TMA issuer waits
 // for its copies in flight, and TMEM is freed.
@@ -259,16 +260,21 @@ __device__ __forceinline__ float exp_half(const uint32_t* sr, uint32_t* pr, int 
 }
 
 // P for a whole item tile of ITEM columns at TMEM column scol (S is read 32 columns at a
-// time); packed bf16 pairs go to pr[0 .. ITEM/2). Returns the row sum.
-template <int ITEM>
+// time); packed bf16 pairs go to pr[0 .. ITEM/2). Returns the row sum. With FIRST_REF and
+// `first` the reference m is first set to the row's own first score, c S[0]: any score of
+// the row is a valid reference (that score alone contributes 2^0 = 1 to the sum, so the
+// sum never underflows), and a reference far below the row's maximum shows up as a sum
+// past the fast-path limit, which sends the item to the exact-max path.
+template <int ITEM, bool FIRST_REF>
 __device__ __forceinline__ float exp_tile(uint32_t scol, uint32_t* pr, int nv, float c,
-                                          uint64_t c2, float m) {
+                                          uint64_t c2, float& m, bool first) {
     float sum = 0.f;
 #pragma unroll
     for (int h = 0; h < ITEM / 32; ++h) {
         uint32_t sr[32];
         tmem_ld32(scol + 32 * h, sr);
         tmem_wait_ld32(sr);
+        if (FIRST_REF && h == 0 && first) m = c * __uint_as_float(sr[0]);
         sum += exp_half(sr, pr + 16 * h, 32 * h, nv, c, c2, m);
     }
     return sum;
@@ -277,8 +283,11 @@ __device__ __forceinline__ float exp_tile(uint32_t scol, uint32_t* pr, int nv, f
 // One item of this warpgroup's stream for this thread's row: read S, update the online
 // softmax, write P back over S, signal the stream's MMA warp. S of item j being ready
 // means the PV of item j - B has completed, so the warpgroup leader frees that item's ring
-// stage. Returns false when the kernel is aborting.
-template <int D>
+// stage. Returns false when the kernel is aborting. FIRST_REF (the decode, whose units
+// are short) takes the first item's reference from its first score; otherwise (the
+// encode, whose units are long) the first item's reference is its exact maximum, which
+// measured faster there.
+template <int D, bool FIRST_REF>
 __device__ __forceinline__ bool softmax_step(SoftmaxStream& S, const Unit& U, uint32_t tmem,
                                              uint32_t lane_off, float c, uint64_t c2,
                                              uint32_t sready_s, uint32_t pready_s, uint32_t empty0,
@@ -301,9 +310,9 @@ __device__ __forceinline__ bool softmax_step(SoftmaxStream& S, const Unit& U, ui
     const uint32_t scol = tmem + lane_off + C::kColS + (S.s * C::B + b) * C::kItem;
     uint32_t pr[C::kItem / 2];
     float sum = 0.f;
-    bool slow = j == 0;
+    bool slow = !FIRST_REF && j == 0;
     if (!slow) {
-        sum = exp_tile<C::kItem>(scol, pr, nv, c, c2, S.m);
+        sum = exp_tile<C::kItem, FIRST_REF>(scol, pr, nv, c, c2, S.m, j == 0);
         slow = __any_sync(0xffffffffu, !(sum <= kFastLimit));
     }
     if (slow) {
@@ -339,7 +348,7 @@ __device__ __forceinline__ bool softmax_step(SoftmaxStream& S, const Unit& U, ui
                 tmem_st16(ocol + 16 * k, o);
             }
         }
-        sum = exp_tile<C::kItem>(scol, pr, nv, c, c2, S.m);
+        sum = exp_tile<C::kItem, false>(scol, pr, nv, c, c2, S.m, false);
     }
     S.l += sum;
     if (C::kItem == 64)
@@ -801,7 +810,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             }
             st.begin(U);
             while (alive && st.j < st.cnt)
-                alive = softmax_step<D>(st, U, tmem, lane_off, c, c2, sready_s,
+                alive = softmax_step<D, DEC>(st, U, tmem, lane_off, c, c2, sready_s,
                                         pready0 + 16u * st.s, empty0, wg_leader, it0, abort_flag,
                                         prm.status);
             if (alive)
