@@ -389,9 +389,87 @@ cudaError_t route_bwd_d(const Plan& p, const BwdPlan& bp, const T* seeds, const 
     return cudaGetLastError();
 }
 
+// ---------------------------------------------------------------- the merged T23 pass
+// T23C (tc_bwd.cu) multiplies V and dZ scaled by u = 2^(L3[n] - R) and w = 2^(R - L2[m])
+// for one shift R per (b, h). With R = min_m L2 both scales stay within 2^kMergeRange
+// whenever max_n L3 - R and max_m L2 - R do; a (b, h) outside that range (scores spread
+// over more than ~60 binary orders) is flagged and runs the unmerged T23 pass instead.
+constexpr float kMergeRange = 60.f;
+
+// part[bh][j] for j < kRangeParts: max of L3 over slice j of the tokens; part[bh][kRangeParts]
+// and [kRangeParts + 1]: min and max of L2 (from slice 0's block). One block per (bh, j).
+__global__ void __launch_bounds__(256) merge_range_kernel(const float* __restrict__ L2,
+                                                          const float* __restrict__ L3, int64_t M,
+                                                          int64_t N, float* __restrict__ part) {
+    __shared__ float red[3][8];
+    const int64_t bh = blockIdx.x / kRangeParts;
+    const int j = (int)(blockIdx.x % kRangeParts);
+    const int64_t per = (N + kRangeParts - 1) / kRangeParts;
+    const int64_t n0 = j * per, n1 = min(N, n0 + per);
+    float mx3 = -INFINITY, mn2 = INFINITY, mx2 = -INFINITY;
+    for (int64_t n = n0 + threadIdx.x; n < n1; n += blockDim.x) mx3 = fmaxf(mx3, L3[bh * N + n]);
+    if (j == 0)
+        for (int64_t m = threadIdx.x; m < M; m += blockDim.x) {
+            const float x = L2[bh * M + m];
+            mn2 = fminf(mn2, x);
+            mx2 = fmaxf(mx2, x);
+        }
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) {
+        mx3 = fmaxf(mx3, __shfl_xor_sync(0xffffffffu, mx3, off));
+        mn2 = fminf(mn2, __shfl_xor_sync(0xffffffffu, mn2, off));
+        mx2 = fmaxf(mx2, __shfl_xor_sync(0xffffffffu, mx2, off));
+    }
+    const int w = threadIdx.x >> 5;
+    if ((threadIdx.x & 31) == 0) {
+        red[0][w] = mx3;
+        red[1][w] = mn2;
+        red[2][w] = mx2;
+    }
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        for (int k = 1; k < (int)(blockDim.x >> 5); ++k) {
+            mx3 = fmaxf(mx3, red[0][k]);
+            mn2 = fminf(mn2, red[1][k]);
+            mx2 = fmaxf(mx2, red[2][k]);
+        }
+        float* o = part + bh * (kRangeParts + 2);
+        o[j] = mx3;
+        if (j == 0) {
+            o[kRangeParts] = mn2;
+            o[kRangeParts + 1] = mx2;
+        }
+    }
+}
+
+// R[bh] = min_m L2 and flags[bh] = 1 when the (b, h) runs the unmerged pass.
+__global__ void merge_flags_kernel(const float* __restrict__ part, int64_t BH,
+                                   float* __restrict__ Rb, int* __restrict__ flags) {
+    const int64_t bh = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+    if (bh >= BH) return;
+    const float* o = part + bh * (kRangeParts + 2);
+    float mx3 = -INFINITY;
+    for (int j = 0; j < kRangeParts; ++j) mx3 = fmaxf(mx3, o[j]);
+    const float R = o[kRangeParts], mx2 = o[kRangeParts + 1];
+    Rb[bh] = R;
+    flags[bh] = (mx3 - R <= kMergeRange && mx2 - R <= kMergeRange) ? 0 : 1;
+}
+
+// The merged pass's route operand w dZ: W[bh][m][:] = bf16(2^(R[bh] - L2[bh][m]) dZ[bh][m][:]).
+__global__ void merge_operand_kernel(const float* __restrict__ dz, const float* __restrict__ L2,
+                                     const float* __restrict__ Rb, int64_t M, int64_t D,
+                                     int64_t total, __nv_bfloat16* __restrict__ W) {
+    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < total;
+         i += (int64_t)gridDim.x * blockDim.x) {
+        const int64_t row = i / D;  // bh * M + m
+        W[i] = __float2bfloat16_rn(exp2f(Rb[row / M] - L2[row]) * dz[i]);
+    }
+}
+
 // The tensor-core path (bf16 inputs): c3, the bf16 operand copies of Q and Z, then
 // R3 -> reduce (dZ, the decoder's dQ, c2) -> T23 (dK, dV) and R2 -> reduce (dQ, c1) ->
-// T1 (dKt, dVt) and R1 -> reduce (dseeds).
+// T1 (dKt, dVt) and R1 -> reduce (dseeds). For D <= 32, T23 runs merged (T23C) for every
+// (b, h) whose statistics allow it and unmerged for the rest.
 template <int D>
 cudaError_t route_bwd_tc_d(const Plan& p, const BwdPlan& bp, const void* seeds, const void* Kt,
                            const void* Vt, const void* K, const void* V, float scale,
@@ -415,6 +493,10 @@ cudaError_t route_bwd_tc_d(const Plan& p, const BwdPlan& bp, const void* seeds, 
     T* zb = (T*)(ws + bp.off_zb);
     T* dzb = (T*)(ws + bp.off_dzb);
     T* dqb = (T*)(ws + bp.off_dqb);
+    T* wop = (T*)(ws + bp.off_w);
+    float* Rb = (float*)(ws + bp.off_rb);
+    int* flags = (int*)(ws + bp.off_flags);
+    float* rpart = (float*)(ws + bp.off_rpart);
     int* status = (int*)(ws + bp.off_status);
     const int64_t tok_rows = p.BH * p.N;
     const int64_t lat_rows = p.BH * p.M;
@@ -423,9 +505,16 @@ cudaError_t route_bwd_tc_d(const Plan& p, const BwdPlan& bp, const void* seeds, 
     const unsigned cvt_blocks = (unsigned)min((int64_t)1024, (lat + 255) / 256);
     cudaError_t e;
 
+    constexpr bool kMerged = D <= 32;
     launch_delta_tokens<D, T>((const T*)dY, (const T*)Y, tok_rows, c3, st);
     to_bf16_kernel<<<cvt_blocks, 256, 0, st>>>(Q32, qb, lat);
     to_bf16_kernel<<<cvt_blocks, 256, 0, st>>>(Z32, zb, lat);
+    if (kMerged) {
+        merge_range_kernel<<<(unsigned)(p.BH * kRangeParts), 256, 0, st>>>(L2, L3, p.M, p.N,
+                                                                           rpart);
+        merge_flags_kernel<<<(unsigned)((p.BH + 127) / 128), 128, 0, st>>>(rpart, p.BH, Rb,
+                                                                            flags);
+    }
     TcBwdOperands o{};
     // R3: route rows; S = Q K^T, dP = Z dY^T; column statistics L3, c3 -> dQ3, dZ partials
     o = TcBwdOperands{{qb, zb, zb}, {K, dY, dY}, nullptr, nullptr, L3, c3, pa, pb, nullptr,
@@ -436,6 +525,17 @@ cudaError_t route_bwd_tc_d(const Plan& p, const BwdPlan& bp, const void* seeds, 
                                                            nullptr, dzb);
     // T23: token rows; S = K Q^T, dP2 = V dZ^T, dP3 = dY Z^T -> dK, dV
     o = TcBwdOperands{{K, V, dY}, {qb, dzb, zb}, L3, c3, L2, c2, nullptr, nullptr, dK, dV};
+    if (kMerged) {
+        // T23C: S = K Q^T, T = dY Z^T + (u V) (w dZ)^T; the flagged (b, h) run T23 after it
+        merge_operand_kernel<<<cvt_blocks, 256, 0, st>>>(dz, L2, Rb, p.M, p.D, lat, wop);
+        TcBwdOperands om{{K, dY, V}, {qb, wop, zb}, L3, c3, L2, c2, nullptr, nullptr, dK, dV};
+        om.Rb = Rb;
+        om.flags = flags;
+        om.want = 0;
+        if ((e = tc_bwd_pass(p, bp, 5, om, scale, status, st)) != cudaSuccess) return e;
+        o.flags = flags;
+        o.want = 1;
+    }
     if ((e = tc_bwd_pass(p, bp, 3, o, scale, status, st)) != cudaSuccess) return e;
     // R2: route rows; S = Q K^T, dP = dZ V^T; row statistics L2, c2 -> dQ2 partials
     o = TcBwdOperands{{qb, dzb, dzb}, {K, V, V}, L2, c2, nullptr, nullptr, nullptr, pb, nullptr,

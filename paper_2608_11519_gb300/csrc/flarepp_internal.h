@@ -66,8 +66,12 @@ struct BwdPlan {
     size_t off_d3;              // c of call 3 [BH][N] f32 (+ 256 bytes of slack)
     size_t off_qb, off_zb;      // tensor-core path: bf16 MMA operands Q, Z [BH][M][D]
     size_t off_dzb, off_dqb;    // ... and dZ, dQ
+    size_t off_w;               // ... and the merged T23 pass's w dZ [BH][M][D] bf16
+    size_t off_rb, off_flags;   // its shift R [BH] f32 and fallback flags [BH] int32
+    size_t off_rpart;           // range partials [BH][kRangeParts + 2] f32
     size_t total;
 };
+constexpr int kRangeParts = 32;  // token slices of the merged pass's range reduction
 BwdPlan make_bwd_plan(const Plan& p);
 
 // ---- CUDA-core kernels (simt_kernels.cuh, instantiated in simt_f32.cu), float32 inputs
@@ -113,8 +117,12 @@ struct TcBwdOperands {
     float* pb;
     void* out0;
     void* out1;
+    const float* Rb = nullptr;  // T23C: the shift R of each (b, h)
+    const int* flags = nullptr;  // when set, only the (b, h) with flags[bh] == want run
+    int want = 0;
 };
-// pass: 0 = R3, 1 = R2, 2 = R1 (route rows), 3 = T23, 4 = T1 (token rows)
+// pass: 0 = R3, 1 = R2, 2 = R1 (route rows), 3 = T23, 4 = T1 (token rows), 5 = T23C (T23
+// with its two dP products merged; D = 16 and 32)
 cudaError_t tc_bwd_pass(const Plan& p, const BwdPlan& bp, int pass, const TcBwdOperands& o,
                         float scale, int* status, cudaStream_t st);
 

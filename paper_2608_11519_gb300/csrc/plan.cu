@@ -184,6 +184,14 @@ BwdPlan make_bwd_plan(const Plan& p) {
         off = align_up(off + op, kWsAlign);
         b.off_dqb = off;
         off = align_up(off + op, kWsAlign);
+        b.off_w = off;
+        off = align_up(off + op, kWsAlign);
+        b.off_rb = off;
+        off = align_up(off + (size_t)p.BH * 4, kWsAlign);
+        b.off_flags = off;
+        off = align_up(off + (size_t)p.BH * 4, kWsAlign);
+        b.off_rpart = off;
+        off = align_up(off + (size_t)p.BH * (kRangeParts + 2) * 4, kWsAlign);
     }
     b.total = off;
     return b;

@@ -51,25 +51,33 @@ constexpr int kRows = 128;  // TMEM lanes per stream, MMA M
 constexpr uint64_t kWaitLimitNs = 2000000000ull;
 constexpr uint32_t kTmemCols = 512;
 
-enum Pass : int { kR3 = 0, kR2 = 1, kR1 = 2, kT23 = 3, kT1 = 4 };
+enum Pass : int { kR3 = 0, kR2 = 1, kR1 = 2, kT23 = 3, kT1 = 4, kT23C = 5 };
 
 template <int D, int PASS>
 struct BCfg {
     static constexpr bool kRouteRows = PASS <= kR1;
-    static constexpr int kNA = PASS == kT23 ? 3 : 2;  // score products (A tiles, item tiles)
+    // T23C (calls 3 and 2 with their two dP products merged into one, see bwd_slice) keeps
+    // its A tiles in TMEM and multiplies them from there (`ts` products)
+    static constexpr bool kATmem = PASS == kT23C;
+    static constexpr int kNA = PASS == kT23 ? 3 : 2;  // score products (TMEM score tiles)
+    static constexpr int kNT = (PASS == kT23 || PASS == kT23C) ? 3 : 2;  // A and item tiles
     static constexpr int kNAcc = (PASS == kR2 || PASS == kR1) ? 1 : 2;
-    static constexpr bool kColStats = PASS == kR3 || PASS == kT23 || PASS == kT1;
-    static constexpr bool kRowStats = PASS == kR2 || PASS == kR1 || PASS == kT23;
-    // TMEM per stream: kNA score tiles of kItem columns, then kNAcc accumulators of D. The
-    // most streams (at most four) that fit in 512 columns, with the widest item of 64, 48 or
-    // 32 rows for that count: four streams make a 512-row group, so M = 512 fills every unit.
-    static constexpr uint32_t col_stream(int item) { return kNA * item + kNAcc * D; }
+    static constexpr bool kColStats = PASS == kR3 || PASS == kT23 || PASS == kT1 || kATmem;
+    static constexpr bool kRowStats = PASS == kR2 || PASS == kR1 || PASS == kT23 || kATmem;
+    // TMEM per stream: kNA score tiles of kItem columns, kNAcc accumulators of D, then (T23C)
+    // the kNT bf16 A tiles of D / 2 columns, padded to 32 columns. The most streams (at most four) that fit in 512
+    // columns, with the widest item of 64, 48 or 32 rows for that count: four streams make a
+    // 512-row group, so M = 512 fills every unit.
+    static constexpr uint32_t col_stream(int item) {
+        return kATmem ? (kNA * item + kNAcc * D + kNT * D / 2 + 31) / 32 * 32
+                      : kNA * item + kNAcc * D;
+    }
     static constexpr int fits(int ns, int item) { return ns * col_stream(item) <= kTmemCols; }
     static constexpr int pick_ns() {
         // T23 (three score products, 6 ss MMAs per item): two streams of 64-row items
         // measured faster than three of 32 (3.41 vs 3.60 ms at mesh3d); for R3 and T1 the
         // most streams win (two of 64 rows: 3.67 vs 2.12 ms; three of 48: 2.38 vs 2.17 ms)
-        if (PASS == kT23 && fits(2, 64)) return 2;
+        if ((PASS == kT23 || PASS == kT23C) && fits(2, 64)) return 2;
         for (int ns = 4; ns >= 1; --ns)
             if (fits(ns, 32)) return ns;
         return 0;
@@ -86,16 +94,16 @@ struct BCfg {
     static constexpr int kGroup = NS * kRows;  // rows per work unit
     static constexpr int kStages = kItem == 64 ? 6 : 10;
     static constexpr int kATile = kRows * D * 2;
-    static constexpr int kABytes = NS * kNA * kATile;  // one unit's A tiles
+    static constexpr int kABytes = NS * kNT * kATile;  // one unit's A tiles
     static constexpr int kItemTile = kItem * D * 2;
-    static constexpr int kStage = kNA * kItemTile;
+    static constexpr int kStage = kNT * kItemTile;
     // two shared-memory copies of a unit's A tiles when they fit beside the ring
     static constexpr int kABuf = 2 * kABytes + kStages * kStage <= 200 * 1024 ? 2 : 1;
     static constexpr uint32_t kSwz = D == 16 ? kSw32 : (D == 32 ? kSw64 : kSw128);
     static constexpr uint32_t kSBO = 8 * D * 2;
     // barriers: full[S], empty[S], afull[kABuf], afree[kABuf], then per stream sready,
-    //           pready, accdone, accfree, fin
-    static constexpr int kNumBars = 2 * kStages + 2 * kABuf + 5 * NS;
+    //           pready, accdone, accfree, fin, aready (T23C: the A tiles are in TMEM)
+    static constexpr int kNumBars = 2 * kStages + 2 * kABuf + 6 * NS;
     static constexpr int kStatBytes = kStages * 2 * kItem * 4;
     static constexpr int kData = kABuf * kABytes + kStages * kStage;
     static constexpr int kNeed = 1024 + kData + kStatBytes + kNumBars * 8 + 16;
@@ -104,6 +112,8 @@ struct BCfg {
     static_assert(kSmem <= 232448, "shared memory budget");
     static constexpr uint32_t kIdescS = idesc_bf16_f32(128, kItem, false, false);
     static constexpr uint32_t kIdescAcc = idesc_bf16_f32(128, D, false, true);
+    static constexpr uint32_t kColA = kNA * kItem + kNAcc * D;  // T23C: first A column
+    static_assert(!kATmem || D <= 32, "T23C serves D = 16 and 32");
 };
 
 struct BwdParams {
@@ -123,8 +133,17 @@ struct BwdParams {
     float* pb;
     __nv_bfloat16* out0;  // token-row passes: s * acc0 and acc1, [BH][N][D]
     __nv_bfloat16* out1;
+    const float* Rb;    // T23C: the shift R of each (b, h) [BH]
+    const int* flags;   // when not null: only the units of (b, h) with flags[bh] == want run
+    int want;
     int* status;
 };
+
+// Units of a (b, h) whose flag differs from the one this launch serves are skipped by every
+// role alike (no barrier, copy or product is issued for them).
+__device__ __forceinline__ bool unit_skipped(const BwdParams& p, int64_t bh) {
+    return p.flags != nullptr && p.flags[bh] != p.want;
+}
 
 struct BUnit {
     int64_t bh, g, chunk;
@@ -229,32 +248,57 @@ __device__ __forceinline__ bool warp_wait(uint32_t bar, uint32_t parity, volatil
     return __all_sync(0xffffffffu, got);
 }
 
-// One 16-column slice h of an item for this thread's row: reads the score tiles, writes
-// bf16 dS over score tile 0 and (when a second accumulator reads it) bf16 P over score
-// tile 1. Math on packed f32 pairs. The row statistics come as (-L, -L) and (-c, -c) pairs;
-// the column statistics sit negated in shared memory. When the item is short (FULL false),
-// columns at or beyond nv get P = dS = 0.
-template <int D, int PASS, bool FULL>
-__device__ __forceinline__ void bwd_slice(uint32_t t0, int h, int nv, uint64_t c2, uint64_t nLr2,
-                                          uint64_t ncr2, const float* nLc, const float* ncc) {
-    using C = BCfg<D, PASS>;
+// One 16-column slice h of an item for this thread's row (slice_load, slice_wait,
+// slice_math): reads the score tiles, writes bf16 dS over score tile 0 and (when a second
+// accumulator reads it) bf16 P over score tile 1. Math on packed f32 pairs. The row
+// statistics come as (-L, -L) and (-c, -c) pairs; the column statistics sit negated in
+// shared memory. When the item is short (FULL false), columns at or beyond nv get
+// P = dS = 0.
+//
+// T23C merges the two dP products of T23. With r = P2 / P3 = 2^(L3[n] - L2[m]) = u[n] w[m],
+// u[n] = 2^(L3[n] - R), w[m] = 2^(R - L2[m]) for a shift R per (b, h), score tile 1 holds
+//   T = dP3 + r dP2 = [dY | u V] [Z | w dZ]^T   (one product of depth 2D),
+// so that dS = P2 (dP2 - c2) + P3 (dP3 - c3) = P3 (T - c3 - u (w c2)), and E2 = P3 u =
+// 2^(c x - R) = P2 / w goes to tile 1: the second accumulator multiplies it by w dZ, giving
+// P2 dZ. One exponential per score. The column statistic is -(w c2); u2 holds (u, u).
+// (Where P3 underflows, P2 = P3 u w stays below 2^-66: R bounds u by 2^60 and w by 1.)
+template <int D, int PASS>
+struct SliceRegs {
     uint32_t sr[16], d1[16], d2[PASS == kT23 ? 16 : 1];
-    tmem_ld16(t0 + 16 * h, sr);
-    tmem_ld16(t0 + C::kItem + 16 * h, d1);
-    if (PASS == kT23) tmem_ld16(t0 + 2 * C::kItem + 16 * h, d2);
-    tmem_wait_ld16(sr);
-    tmem_wait_ld16(d1);
-    if (PASS == kT23) tmem_wait_ld16(d2);
+};
+template <int D, int PASS>
+__device__ __forceinline__ void slice_load(uint32_t t0, int h, SliceRegs<D, PASS>& g) {
+    using C = BCfg<D, PASS>;
+    tmem_ld16(t0 + 16 * h, g.sr);
+    tmem_ld16(t0 + C::kItem + 16 * h, g.d1);
+    if (PASS == kT23) tmem_ld16(t0 + 2 * C::kItem + 16 * h, g.d2);
+}
+template <int D, int PASS>
+__device__ __forceinline__ void slice_wait(SliceRegs<D, PASS>& g) {
+    tmem_wait_ld16(g.sr);
+    tmem_wait_ld16(g.d1);
+    if (PASS == kT23) tmem_wait_ld16(g.d2);
+}
+template <int D, int PASS, bool FULL>
+__device__ __forceinline__ void slice_math(uint32_t t0, int h, const SliceRegs<D, PASS>& g, int nv,
+                                           uint64_t c2, uint64_t nLr2, uint64_t ncr2,
+                                           const float* nLc, const float* ncc, uint64_t u2) {
+    using C = BCfg<D, PASS>;
     uint32_t ds[8], pp[8];
 #pragma unroll
     for (int k = 0; k < 8; ++k) {
         const int col = 16 * h + 2 * k;
-        const uint64_t x = ld_pair(sr, k);
-        const uint64_t dp = ld_pair(d1, k);
+        const uint64_t x = ld_pair(g.sr, k);
+        const uint64_t dp = ld_pair(g.d1, k);
         uint64_t p, d;
         if (PASS == kR2 || PASS == kR1) {
             p = ex2x2(fma2(x, c2, nLr2));
             d = mul2(p, add2(dp, ncr2));
+        } else if (PASS == kT23C) {
+            const uint64_t nwc = *reinterpret_cast<const uint64_t*>(nLc + col);
+            const uint64_t p3 = ex2x2(fma2(x, c2, nLr2));
+            p = mul2(p3, u2);  // E2 = P3 u
+            d = mul2(p3, fma2(u2, nwc, add2(dp, ncr2)));
         } else {
             const uint64_t nL = *reinterpret_cast<const uint64_t*>(nLc + col);
             const uint64_t nc = *reinterpret_cast<const uint64_t*>(ncc + col);
@@ -262,7 +306,7 @@ __device__ __forceinline__ void bwd_slice(uint32_t t0, int h, int nv, uint64_t c
             d = mul2(p, add2(dp, nc));
             if (PASS == kT23) {
                 const uint64_t p3 = ex2x2(fma2(x, c2, nLr2));
-                d = fma2(p3, add2(ld_pair(d2, k), ncr2), d);
+                d = fma2(p3, add2(ld_pair(g.d2, k), ncr2), d);
             }
         }
         if (!FULL) {
@@ -279,6 +323,22 @@ __device__ __forceinline__ void bwd_slice(uint32_t t0, int h, int nv, uint64_t c
     if (C::kNAcc == 2) tmem_st8(t0 + C::kItem + 8 * h, pp);
 }
 
+// One item for this thread's row, 16 columns at a time. (Issuing the next slice's loads
+// before the current slice's math measured slower in every pass.)
+template <int D, int PASS, bool FULL>
+__device__ __forceinline__ void bwd_item(uint32_t t0, int nv, uint64_t c2, uint64_t nLr2,
+                                         uint64_t ncr2, const float* nLc, const float* ncc,
+                                         uint64_t u2) {
+    using C = BCfg<D, PASS>;
+#pragma unroll
+    for (int h = 0; h < C::kItem / 16; ++h) {
+        SliceRegs<D, PASS> g;
+        slice_load<D, PASS>(t0, h, g);
+        slice_wait<D, PASS>(g);
+        slice_math<D, PASS, FULL>(t0, h, g, nv, c2, nLr2, ncr2, nLc, ncc, u2);
+    }
+}
+
 // ------------------------------------------------------------------ the kernel
 
 template <int D, int PASS>
@@ -292,8 +352,8 @@ __global__ void __launch_bounds__(BCfg<D, PASS>::kThreads, 1)
     extern __shared__ uint8_t smem_raw[];
     uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                                ~static_cast<uintptr_t>(1023));
-    uint8_t* abuf = smem;                          // kABuf x [NS][kNA] A tiles, swizzled
-    uint8_t* ring = smem + C::kABuf * C::kABytes;  // kStages x kNA item tiles, swizzled
+    uint8_t* abuf = smem;                          // kABuf x [NS][kNT] A tiles
+    uint8_t* ring = smem + C::kABuf * C::kABytes;  // kStages x kNT item tiles, swizzled
     float* stats = reinterpret_cast<float*>(ring + C::kStages * C::kStage);  // [S][2][kItem]
     uint64_t* bars = reinterpret_cast<uint64_t*>(stats + C::kStages * 2 * C::kItem);
     uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + C::kNumBars);
@@ -308,6 +368,7 @@ __global__ void __launch_bounds__(BCfg<D, PASS>::kThreads, 1)
     const uint32_t accdone0 = pready0 + 8u * NS;
     const uint32_t accfree0 = accdone0 + 8u * NS;
     const uint32_t fin0 = accfree0 + 8u * NS;
+    const uint32_t aready0 = fin0 + 8u * NS;
 
     const int warp = threadIdx.x >> 5;
     const int lane = threadIdx.x & 31;
@@ -319,7 +380,9 @@ __global__ void __launch_bounds__(BCfg<D, PASS>::kThreads, 1)
         }
         for (int b = 0; b < C::kABuf; ++b) {
             mbar_init(afull0 + 8u * b, 1);
-            mbar_init(afree0 + 8u * b, NS);
+            // released by each stream's MMA warp, or (A in TMEM) by every softmax thread
+            // once its rows are copied
+            mbar_init(afree0 + 8u * b, C::kATmem ? NS * kRows : NS);
         }
         for (int s = 0; s < NS; ++s) {
             mbar_init(sready0 + 8u * s, 1);
@@ -327,6 +390,7 @@ __global__ void __launch_bounds__(BCfg<D, PASS>::kThreads, 1)
             mbar_init(accdone0 + 8u * s, 1);
             mbar_init(accfree0 + 8u * s, kRows);
             mbar_init(fin0 + 8u * s, 1);
+            mbar_init(aready0 + 8u * s, kRows);
         }
         *abort_flag = 0;
         fence_mbar_init();
@@ -334,7 +398,7 @@ __global__ void __launch_bounds__(BCfg<D, PASS>::kThreads, 1)
         prefetch_tmap(&tmA1);
         prefetch_tmap(&tmI0);
         prefetch_tmap(&tmI1);
-        if (C::kNA == 3) {
+        if (C::kNT == 3) {
             prefetch_tmap(&tmA2);
             prefetch_tmap(&tmI2);
         }
@@ -352,24 +416,26 @@ __global__ void __launch_bounds__(BCfg<D, PASS>::kThreads, 1)
         // ------------------------------------------------------------ TMA producer
         uint32_t it = 0, ua = 0, a_issued = 0;
         bool ok = true;
-        for (int64_t u = blockIdx.x; u < prm.n_units && ok; u += gridDim.x, ++ua) {
+        for (int64_t u = blockIdx.x; u < prm.n_units && ok; u += gridDim.x) {
             const BUnit U = bwd_unit<D, PASS>(prm, u);
-            const int ab = ua % C::kABuf;
-            if (ua >= (uint32_t)C::kABuf &&
-                !warp_wait(afree0 + 8u * ab, ((ua / C::kABuf) - 1) & 1, abort_flag, prm.status)) {
+            if (unit_skipped(prm, U.bh)) continue;
+            const uint32_t uc = ua++;
+            const int ab = uc % C::kABuf;
+            if (uc >= (uint32_t)C::kABuf &&
+                !warp_wait(afree0 + 8u * ab, ((uc / C::kABuf) - 1) & 1, abort_flag, prm.status)) {
                 ok = false;
                 break;
             }
             if (elect_one()) {
-                mbar_expect_tx(afull0 + 8u * ab, U.n_act * C::kNA * C::kATile);
+                mbar_expect_tx(afull0 + 8u * ab, U.n_act * C::kNT * C::kATile);
                 const int za0 = (int)(prm.a0_per_head ? U.bh % prm.H : U.bh);
                 for (int s = 0; s < U.n_act; ++s) {
                     const int row = (int)(U.row0 + s * kRows);
-                    uint8_t* dst = abuf + ab * C::kABytes + s * C::kNA * C::kATile;
+                    uint8_t* dst = abuf + ab * C::kABytes + s * C::kNT * C::kATile;
                     tma_load_3d(smem_u32(dst), &tmA0, 0, row, za0, afull0 + 8u * ab);
                     tma_load_3d(smem_u32(dst + C::kATile), &tmA1, 0, row, (int)U.bh,
                                 afull0 + 8u * ab);
-                    if (C::kNA == 3)
+                    if (C::kNT == 3)
                         tma_load_3d(smem_u32(dst + 2 * C::kATile), &tmA2, 0, row, (int)U.bh,
                                     afull0 + 8u * ab);
                 }
@@ -377,6 +443,7 @@ __global__ void __launch_bounds__(BCfg<D, PASS>::kThreads, 1)
             __syncwarp();
             ++a_issued;
             const int zi0 = (int)(prm.i0_per_head ? U.bh % prm.H : U.bh);
+            const float R = C::kATmem ? prm.Rb[U.bh] : 0.f;
             for (int i = 0; i < U.n_items; ++i, ++it) {
                 const int st = it % C::kStages;
                 if (it >= (uint32_t)C::kStages &&
@@ -392,7 +459,7 @@ __global__ void __launch_bounds__(BCfg<D, PASS>::kThreads, 1)
                     tma_load_3d(dst, &tmI0, 0, (int)row, zi0, full0 + 8u * st);
                     tma_load_3d(dst + C::kItemTile, &tmI1, 0, (int)row, (int)U.bh,
                                 full0 + 8u * st);
-                    if (C::kNA == 3)
+                    if (C::kNT == 3)
                         tma_load_3d(dst + 2 * C::kItemTile, &tmI2, 0, (int)row, (int)U.bh,
                                     full0 + 8u * st);
                     // streams idle in this unit count as having released the stage
@@ -400,14 +467,19 @@ __global__ void __launch_bounds__(BCfg<D, PASS>::kThreads, 1)
                 }
                 __syncwarp();
                 if (C::kColStats) {
-                    // the item's column statistics, negated (P = 2^(c x + (-L)))
+                    // the item's column statistics, negated (P = 2^(c x + (-L))); T23C
+                    // stages -(w c2) with w = 2^(R - L2)
                     float* sl = stats + st * 2 * C::kItem;
                     const int64_t nvalid = U.item_end - row;
                     for (int k = lane; k < C::kItem; k += 32) {
                         const bool in = k < nvalid;
                         const int64_t idx = U.bh * (C::kRouteRows ? prm.N : prm.M) + row + k;
-                        sl[k] = in ? -prm.Lcol[idx] : 0.f;
-                        sl[C::kItem + k] = in ? -prm.ccol[idx] : 0.f;
+                        if (C::kATmem) {
+                            sl[k] = in ? -exp2f(R - prm.Lcol[idx]) * prm.ccol[idx] : 0.f;
+                        } else {
+                            sl[k] = in ? -prm.Lcol[idx] : 0.f;
+                            sl[C::kItem + k] = in ? -prm.ccol[idx] : 0.f;
+                        }
                     }
                     mbar_arrive(full0 + 8u * st);
                 }
@@ -436,7 +508,7 @@ __global__ void __launch_bounds__(BCfg<D, PASS>::kThreads, 1)
         // softmax frees ring stage j - 1 once S(j) is complete (the tensor pipe runs this
         // warp's products in order), and the last stage of a unit after acc_done.
         const int s = warp;
-        uint32_t it = 0, ua = 0, pj = 0, nu = 0;
+        uint32_t it = 0, ua = 0, pj = 0, nu = 0, ar = 0;
         bool ok = true;
         auto wait = [&](uint32_t bar, uint32_t parity) {
             return warp_wait(bar, parity, abort_flag, prm.status);
@@ -464,23 +536,38 @@ __global__ void __launch_bounds__(BCfg<D, PASS>::kThreads, 1)
                 }
             }
         };
-        for (int64_t u = blockIdx.x; u < prm.n_units && ok; u += gridDim.x, ++ua) {
+        for (int64_t u = blockIdx.x; u < prm.n_units && ok; u += gridDim.x) {
             const BUnit U = bwd_unit<D, PASS>(prm, u);
-            const int ab = ua % C::kABuf;
-            // the unit's A tiles (an idle stream waits too, so that its release of the A
-            // buffer counts for this unit's phase)
-            if (!wait(afull0 + 8u * ab, (ua / C::kABuf) & 1)) {
-                ok = false;
-                break;
-            }
-            if (s >= U.n_act) {
-                if (elect_one()) mbar_arrive(afree0 + 8u * ab);
-                __syncwarp();
-                it += U.n_items;
-                continue;
+            if (unit_skipped(prm, U.bh)) continue;
+            const uint32_t uc = ua++;
+            const int ab = uc % C::kABuf;
+            if (!C::kATmem) {
+                // the unit's A tiles (an idle stream waits too, so that its release of the
+                // A buffer counts for this unit's phase)
+                if (!wait(afull0 + 8u * ab, (uc / C::kABuf) & 1)) {
+                    ok = false;
+                    break;
+                }
+                if (s >= U.n_act) {
+                    if (elect_one()) mbar_arrive(afree0 + 8u * ab);
+                    __syncwarp();
+                    it += U.n_items;
+                    continue;
+                }
+            } else {
+                if (s >= U.n_act) {
+                    it += U.n_items;
+                    continue;
+                }
+                // the unit's A tiles, copied into TMEM by the softmax warpgroup
+                if (!wait(aready0 + 8u * s, ar & 1)) {
+                    ok = false;
+                    break;
+                }
+                ++ar;
             }
             tc_fence_after();
-            const uint32_t a_base = smem_u32(abuf + ab * C::kABytes + s * C::kNA * C::kATile);
+            const uint32_t a_base = smem_u32(abuf + ab * C::kABytes + s * C::kNT * C::kATile);
             int prev_st = 0;
             for (int i = 0; i <= U.n_items; ++i) {
                 const int st = it % C::kStages;
@@ -506,17 +593,46 @@ __global__ void __launch_bounds__(BCfg<D, PASS>::kThreads, 1)
                 if (i > 0) issue_acc(prev_st, i > 1);
                 if (i < U.n_items) {
                     const uint32_t i_base = smem_u32(ring + st * C::kStage);
-#pragma unroll
-                    for (int t = 0; t < C::kNA; ++t) {
+                    if (C::kATmem) {
+                        // S = K Q^T (item tile 0); T = dY Z^T (item tile 2) + (u V) (w dZ)^T
+                        // (item tile 1), with K, dY, u V in TMEM
+                        const uint32_t aK = t0 + C::kColA;
 #pragma unroll
                         for (int k = 0; k < D / 16; ++k) {
-                            const uint64_t ad =
-                                smem_desc(a_base + t * C::kATile + 32 * k, 16, C::kSBO, C::kSwz);
-                            const uint64_t bd =
-                                smem_desc(i_base + t * C::kItemTile + 32 * k, 16, C::kSBO, C::kSwz);
-                            if (elect_one())
-                                mma_ss(t0 + t * C::kItem, ad, bd, C::kIdescS, k > 0 ? 1u : 0u);
+                            const uint64_t bd = smem_desc(i_base + 32 * k, 16, C::kSBO, C::kSwz);
+                            if (elect_one()) mma_ts(t0, aK + 8 * k, bd, C::kIdescS, k > 0 ? 1u : 0u);
                             __syncwarp();
+                        }
+#pragma unroll
+                        for (int k = 0; k < D / 16; ++k) {
+                            const uint64_t bd = smem_desc(i_base + 2 * C::kItemTile + 32 * k, 16,
+                                                          C::kSBO, C::kSwz);
+                            if (elect_one())
+                                mma_ts(t0 + C::kItem, aK + D / 2 + 8 * k, bd, C::kIdescS,
+                                       k > 0 ? 1u : 0u);
+                            __syncwarp();
+                        }
+#pragma unroll
+                        for (int k = 0; k < D / 16; ++k) {
+                            const uint64_t bd = smem_desc(i_base + C::kItemTile + 32 * k, 16,
+                                                          C::kSBO, C::kSwz);
+                            if (elect_one())
+                                mma_ts(t0 + C::kItem, aK + D + 8 * k, bd, C::kIdescS, 1u);
+                            __syncwarp();
+                        }
+                    } else {
+#pragma unroll
+                        for (int t = 0; t < C::kNA; ++t) {
+#pragma unroll
+                            for (int k = 0; k < D / 16; ++k) {
+                                const uint64_t ad = smem_desc(a_base + t * C::kATile + 32 * k, 16,
+                                                              C::kSBO, C::kSwz);
+                                const uint64_t bd = smem_desc(i_base + t * C::kItemTile + 32 * k,
+                                                              16, C::kSBO, C::kSwz);
+                                if (elect_one())
+                                    mma_ss(t0 + t * C::kItem, ad, bd, C::kIdescS, k > 0 ? 1u : 0u);
+                                __syncwarp();
+                            }
                         }
                     }
                     if (elect_one()) mma_commit(sready0 + 8u * s);
@@ -526,7 +642,7 @@ __global__ void __launch_bounds__(BCfg<D, PASS>::kThreads, 1)
                 } else {
                     if (elect_one()) {
                         mma_commit(accdone0 + 8u * s);
-                        mma_commit(afree0 + 8u * ab);
+                        if (!C::kATmem) mma_commit(afree0 + 8u * ab);
                     }
                     __syncwarp();
                     ++nu;
@@ -548,10 +664,64 @@ __global__ void __launch_bounds__(BCfg<D, PASS>::kThreads, 1)
         const bool leader = q == 0 && lane == 0;
         const uint32_t t0 = tmem + ((uint32_t)(32 * q) << 16) + s * C::kColStream;
         const uint64_t c2 = pack_f32x2(prm.c, prm.c);
-        uint32_t it = 0, sj = 0, na = 0;
+        uint32_t it = 0, sj = 0, na = 0, ua = 0;
         bool ok = true;
+        // T23C: copy this stream's A rows of unit V (the ua-th unit of the CTA) from shared
+        // memory into TMEM: K, dY, and V scaled by u = 2^(L3 - R). Every thread then releases
+        // the shared-memory buffer; an idle stream only releases it.
+        auto copy_a = [&](const BUnit& V, uint32_t uv) -> bool {
+            const int ab = uv % C::kABuf;
+            if (!warp_wait(afull0 + 8u * ab, (uv / C::kABuf) & 1, abort_flag, prm.status))
+                return false;
+            if (s < V.n_act) {
+                const int64_t row = V.row0 + s * kRows + r;
+                const float uu =
+                    row < V.rows ? exp2f(prm.Lrow[V.bh * V.rows + row] - prm.Rb[V.bh]) : 0.f;
+                const uint8_t* src = abuf + ab * C::kABytes + s * C::kNT * C::kATile + r * D * 2;
+#pragma unroll
+                for (int t = 0; t < C::kNT; ++t) {
+                    uint32_t v[D / 2];
+                    const uint4* p4 = reinterpret_cast<const uint4*>(src + t * C::kATile);
+#pragma unroll
+                    for (int k = 0; k < D / 8; ++k) {
+                        const uint4 x = p4[k];
+                        v[4 * k] = x.x;
+                        v[4 * k + 1] = x.y;
+                        v[4 * k + 2] = x.z;
+                        v[4 * k + 3] = x.w;
+                    }
+                    if (t == 2) {
+#pragma unroll
+                        for (int k = 0; k < D / 2; ++k) {
+                            __nv_bfloat162 b = *reinterpret_cast<__nv_bfloat162*>(&v[k]);
+                            const float2 f = __bfloat1622float2(b);
+                            v[k] = pack_bf16(f.x * uu, f.y * uu);
+                        }
+                    }
+                    if (D == 16)
+                        tmem_st8(t0 + C::kColA + t * (D / 2), v);
+                    else
+                        tmem_st16(t0 + C::kColA + t * (D / 2), v);
+                }
+                tmem_wait_st();
+                tc_fence_before();
+                mbar_arrive(aready0 + 8u * s);
+            }
+            mbar_arrive(afree0 + 8u * ab);
+            return true;
+        };
+        bool copied = false;  // T23C: the current unit's A rows were copied ahead
         for (int64_t u = blockIdx.x; u < prm.n_units && ok; u += gridDim.x) {
             const BUnit U = bwd_unit<D, PASS>(prm, u);
+            if (unit_skipped(prm, U.bh)) continue;
+            const uint32_t uc = ua++;
+            if (C::kATmem) {
+                if (!copied && !copy_a(U, uc)) {
+                    ok = false;
+                    break;
+                }
+                copied = false;
+            }
             if (s >= U.n_act) {
                 it += U.n_items;
                 continue;
@@ -564,6 +734,9 @@ __global__ void __launch_bounds__(BCfg<D, PASS>::kThreads, 1)
                 cr = prm.crow[U.bh * U.rows + row];
             }
             const uint64_t nLr2 = pack_f32x2(-Lr, -Lr), ncr2 = pack_f32x2(-cr, -cr);
+            // T23C: u = 2^(L3 - R) of this row
+            const float uu = C::kATmem && valid ? exp2f(Lr - prm.Rb[U.bh]) : 0.f;
+            const uint64_t u2 = pack_f32x2(uu, uu);
             for (int i = 0; i < U.n_items; ++i, ++it) {
                 const int st = it % C::kStages;
                 if (!warp_wait(sready0 + 8u * s, sj & 1, abort_flag, prm.status)) {
@@ -583,20 +756,28 @@ __global__ void __launch_bounds__(BCfg<D, PASS>::kThreads, 1)
                     (int)min((int64_t)C::kItem, U.item_end - (U.item0 + (int64_t)i * C::kItem));
                 const float* nLc = stats + st * 2 * C::kItem;
                 const float* ncc = nLc + C::kItem;
-                if (nv == C::kItem) {
-#pragma unroll
-                    for (int h = 0; h < C::kItem / 16; ++h)
-                        bwd_slice<D, PASS, true>(t0, h, nv, c2, nLr2, ncr2, nLc, ncc);
-                } else {
-#pragma unroll
-                    for (int h = 0; h < C::kItem / 16; ++h)
-                        bwd_slice<D, PASS, false>(t0, h, nv, c2, nLr2, ncr2, nLc, ncc);
-                }
+                if (nv == C::kItem)
+                    bwd_item<D, PASS, true>(t0, nv, c2, nLr2, ncr2, nLc, ncc, u2);
+                else
+                    bwd_item<D, PASS, false>(t0, nv, c2, nLr2, ncr2, nLc, ncc, u2);
                 tmem_wait_st();
                 tc_fence_before();
                 mbar_arrive(pready0 + 8u * s);
             }
             if (!ok) break;
+            if (C::kATmem) {
+                // the score products of the unit's last item are complete (its S was seen),
+                // so the A rows of the CTA's next unit can go into TMEM now, ahead of this
+                // unit's epilogue
+                for (int64_t un = u + gridDim.x; un < prm.n_units; un += gridDim.x) {
+                    const BUnit V = bwd_unit<D, PASS>(prm, un);
+                    if (unit_skipped(prm, V.bh)) continue;
+                    if (!copy_a(V, ua)) ok = false;
+                    copied = ok;
+                    break;
+                }
+                if (!ok) break;
+            }
             // epilogue: the unit's accumulators
             if (!warp_wait(accdone0 + 8u * s, na & 1, abort_flag, prm.status)) {
                 ok = false;
@@ -681,18 +862,20 @@ PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
     return fn;
 }
 
-// A bf16 [z][rows][D] tensor, boxes of box_rows x D, swizzled to the row width.
+// A bf16 [z][rows][D] tensor, boxes of box_rows x D, swizzled to the row width (or plain
+// rows, for tiles that are copied into TMEM row by row).
 bool make_map(CUtensorMap* m, const void* base, int64_t D, int64_t rows, int64_t z,
-              uint32_t box_rows) {
+              uint32_t box_rows, bool swizzle = true) {
     auto fn = encode_fn();
     if (!fn) return false;
     cuuint64_t dims[3] = {(cuuint64_t)D, (cuuint64_t)rows, (cuuint64_t)z};
     cuuint64_t strides[2] = {(cuuint64_t)(D * 2), (cuuint64_t)(rows * D * 2)};
     cuuint32_t box[3] = {(cuuint32_t)D, box_rows, 1};
     cuuint32_t estr[3] = {1, 1, 1};
-    const CUtensorMapSwizzle sw = D == 16 ? CU_TENSOR_MAP_SWIZZLE_32B
-                                          : (D == 32 ? CU_TENSOR_MAP_SWIZZLE_64B
-                                                     : CU_TENSOR_MAP_SWIZZLE_128B);
+    const CUtensorMapSwizzle sw = !swizzle ? CU_TENSOR_MAP_SWIZZLE_NONE
+                                  : D == 16 ? CU_TENSOR_MAP_SWIZZLE_32B
+                                            : (D == 32 ? CU_TENSOR_MAP_SWIZZLE_64B
+                                                       : CU_TENSOR_MAP_SWIZZLE_128B);
     return fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(base), dims, strides, box,
               estr, CU_TENSOR_MAP_INTERLEAVE_NONE, sw, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
               CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
@@ -718,12 +901,12 @@ cudaError_t launch_pass(const void* const* srcs, const Plan& p, BwdParams prm, c
     const int64_t irows = Cf::kRouteRows ? p.N : p.M;
     CUtensorMap maps[6];
     for (int k = 0; k < 6; ++k) {
-        const bool used = (k % 3) < Cf::kNA;
+        const bool used = (k % 3) < Cf::kNT;
         const void* base = used ? srcs[k] : srcs[k - 2];
         const bool a_side = k < 3;
         const bool per_head = a_side ? (prm.a0_per_head && k == 0) : (prm.i0_per_head && k == 3);
         if (!make_map(&maps[k], base, p.D, a_side ? arows : irows, per_head ? p.H : p.BH,
-                      a_side ? (uint32_t)kRows : (uint32_t)Cf::kItem))
+                      a_side ? (uint32_t)kRows : (uint32_t)Cf::kItem, !(a_side && Cf::kATmem)))
             return cudaErrorInvalidValue;
     }
     int dev = 0, sms = kNumSMs;
@@ -738,11 +921,19 @@ cudaError_t launch_pass(const void* const* srcs, const Plan& p, BwdParams prm, c
 template <int PASS>
 cudaError_t launch_d(const void* const* srcs, const Plan& p, const BwdParams& prm,
                      cudaStream_t st) {
-    switch (p.D) {
-        case 16: return launch_pass<16, PASS>(srcs, p, prm, st);
-        case 32: return launch_pass<32, PASS>(srcs, p, prm, st);
-        case 64: return launch_pass<64, PASS>(srcs, p, prm, st);
-        default: return cudaErrorInvalidValue;
+    if constexpr (PASS == kT23C) {
+        switch (p.D) {
+            case 16: return launch_pass<16, kT23C>(srcs, p, prm, st);
+            case 32: return launch_pass<32, kT23C>(srcs, p, prm, st);
+            default: return cudaErrorInvalidValue;
+        }
+    } else {
+        switch (p.D) {
+            case 16: return launch_pass<16, PASS>(srcs, p, prm, st);
+            case 32: return launch_pass<32, PASS>(srcs, p, prm, st);
+            case 64: return launch_pass<64, PASS>(srcs, p, prm, st);
+            default: return cudaErrorInvalidValue;
+        }
     }
 }
 
@@ -770,6 +961,9 @@ cudaError_t tc_bwd_pass(const Plan& p, const BwdPlan& bp, int pass, const TcBwdO
     prm.pb = o.pb;
     prm.out0 = (__nv_bfloat16*)o.out0;
     prm.out1 = (__nv_bfloat16*)o.out1;
+    prm.Rb = o.Rb;
+    prm.flags = o.flags;
+    prm.want = o.want;
     prm.status = status;
     switch (pass) {
         case kR3: return launch_d<kR3>(srcs, p, prm, st);
@@ -777,6 +971,7 @@ cudaError_t tc_bwd_pass(const Plan& p, const BwdPlan& bp, int pass, const TcBwdO
         case kR1: return launch_d<kR1>(srcs, p, prm, st);
         case kT23: return launch_d<kT23>(srcs, p, prm, st);
         case kT1: return launch_d<kT1>(srcs, p, prm, st);
+        case kT23C: return launch_d<kT23C>(srcs, p, prm, st);
         default: return cudaErrorInvalidValue;
     }
 }

@@ -386,14 +386,19 @@ __device__ __forceinline__ bool finish_stream(SoftmaxStream& S, const Unit& U,
             }
         }
         const uint32_t ocol = tmem + lane_off + C::kColO + S.s * D;
-#pragma unroll
-        for (int kk = 0; kk < D / 16; ++kk) {
-            uint32_t t[16];
-            tmem_ld16(ocol + 16 * kk, t);
+        // every load of O in flight before one wait
+        uint32_t t[D];
+        if (D == 16) {
+            tmem_ld16(ocol, t);
             tmem_wait_ld16(t);
+        } else {
 #pragma unroll
-            for (int e = 0; e < 16; ++e) o[16 * kk + e] = __uint_as_float(t[e]);
+            for (int kk = 0; kk < D / 32; ++kk) tmem_ld32(ocol + 32 * kk, t + 32 * kk);
+#pragma unroll
+            for (int kk = 0; kk < D / 32; ++kk) tmem_wait_ld32(t + 32 * kk);
         }
+#pragma unroll
+        for (int d = 0; d < D; ++d) o[d] = __uint_as_float(t[d]);
     } else {
 #pragma unroll
         for (int d = 0; d < D; ++d) o[d] = 0.f;

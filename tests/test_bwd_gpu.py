@@ -239,3 +239,63 @@ def test_bwd_guard_bands_untouched():
         assert torch.all(buf[:band] == 7.0) and torch.all(buf[-band:] == 7.0)
     for g in grads:
         assert torch.isfinite(g.float()).all()
+
+
+def _stat_spread(f, scale):
+    """Per (b, h): max_n L3 - min_m L2 of the chain's calls 2 and 3 (base-2 log-normalisers
+    of the scores x = scale log2(e) <Q_m, K_n>, over tokens per route and over routes per
+    token), computed in float64 from the oracle's Q."""
+    c = scale / math.log(2)
+    out = []
+    B, H = f["K"].shape[:2]
+    for b in range(B):
+        for h in range(H):
+            x1 = c * f["seeds"][h] @ f["Kt"][b, h].T
+            a1 = np.exp2(x1 - x1.max(1, keepdims=True))
+            Q = (a1 / a1.sum(1, keepdims=True)) @ f["Vt"][b, h]
+            x2 = c * Q @ f["K"][b, h].T  # [M, N]
+            m2 = x2.max(1, keepdims=True)
+            L2 = m2[:, 0] + np.log2(np.exp2(x2 - m2).sum(1))
+            m3 = x2.max(0, keepdims=True)
+            L3 = m3[0] + np.log2(np.exp2(x2 - m3).sum(0))
+            out.append(max(L3.max() - L2.min(), L2.max() - L2.min()))
+    return out
+
+
+@pytest.mark.parametrize("D,fac,flagged", [(32, 8, False), (16, 8, False), (32, 16, True),
+                                           (16, 16, True)])
+def test_bwd_wide_score_ranges(D, fac, flagged):
+    """Sharp routes (seeds x 10) and, on heads 1 and 3, keys scaled by `fac` spread the
+    log-normalisers L2, L3 over tens of binary orders. The merged pass of calls 3 and 2
+    scales V and dZ by 2^(L3 - R) and 2^(R - L2); up to a spread of 60 it serves every head
+    (fac 8: spreads near 50), beyond it those heads run the unmerged pass while the others
+    stay merged (fac 16: spreads above 80 on heads 1 and 3). Both must match the oracle.
+
+    dK and dV (the outputs of those passes) are held to the bf16 tolerance where every head
+    runs merged; where heads 1 and 3 run unmerged, calls 2 and 3 are as sharp as call 1
+    and the unmerged pass itself reaches 2.5e-2 there, so those cases get 3e-2. The call-1
+    gradients (dseeds, dKt, dVt) get 7e-2: with routes this sharp, call 1's softmax is
+    nearly one-hot, dS1 = P1 (dP1 - c1) cancels, and the bf16 rounding of the dQ operand
+    shows through (errors up to 5.9e-2 of the gradient's scale, the same before and after
+    the merge, which does not touch call 1)."""
+    scale = 1.0 / math.sqrt(D)
+    w = inputs.Workload("case", 1, 4, 2000, 200, D, "bf16")
+    x = inputs.make_inputs(w, 5)
+    x["seeds"] = (x["seeds"].float() * 10).to(torch.bfloat16)
+    K = x["K"].float()
+    K[:, 1] *= fac
+    K[:, 3] *= fac
+    x["K"] = K.to(torch.bfloat16)
+    dY = inputs.make_output_grad(w, 5)
+    f = inputs.to_f64_numpy(x)
+    spread = _stat_spread(f, scale)
+    wide = [s > 60.0 for s in spread]
+    assert wide == [False, flagged, False, flagged], spread
+    assert max(spread) > 30.0, spread
+    got, _ = _gpu_grads(x, dY, scale)
+    want = oracle.route_bwd(f["seeds"], f["Kt"], f["Vt"], f["K"], f["V"], scale, _np(dY))
+    for name, g, r in zip(NAMES, got, want):
+        tol = (3e-2 if flagged else TOL["bf16"]) if name in ("dK", "dV") else 7e-2
+        bound = tol * max(1.0, float(np.abs(r).max()))
+        err = float(np.abs(g - r).max())
+        assert err <= bound and not math.isnan(err), f"{name}: {err} > {bound}"
