@@ -71,7 +71,7 @@ struct BwdPlan {
     size_t off_rpart;           // range partials [BH][kRangeParts + 2] f32
     size_t total;
 };
-constexpr int kRangeParts = 32;  // token slices of the merged pass's range reduction
+constexpr int kRangeParts = 128;  // token slices of the merged pass's range reduction
 BwdPlan make_bwd_plan(const Plan& p);
 
 // ---- CUDA-core kernels (simt_kernels.cuh, instantiated in simt_f32.cu), float32 inputs

@@ -144,6 +144,14 @@ struct BwdParams {
 __device__ __forceinline__ bool unit_skipped(const BwdParams& p, int64_t bh) {
     return p.flags != nullptr && p.flags[bh] != p.want;
 }
+// The unit before this CTA's first unit of the next (b, h): units are numbered (b, h)-major
+// with per_bh units each, and a CTA takes every gridDim.x-th one, so a skipped (b, h) is
+// stepped over whole.
+__device__ __forceinline__ int64_t skip_bh(int64_t bh, int64_t per_bh) {
+    const int64_t next = (bh + 1) * per_bh;
+    const int64_t g = gridDim.x;
+    return next + ((int64_t)blockIdx.x - next % g + g) % g - g;
+}
 
 struct BUnit {
     int64_t bh, g, chunk;
@@ -418,7 +426,10 @@ __global__ void __launch_bounds__(BCfg<D, PASS>::kThreads, 1)
         bool ok = true;
         for (int64_t u = blockIdx.x; u < prm.n_units && ok; u += gridDim.x) {
             const BUnit U = bwd_unit<D, PASS>(prm, u);
-            if (unit_skipped(prm, U.bh)) continue;
+            if (unit_skipped(prm, U.bh)) {
+                u = skip_bh(U.bh, C::kRouteRows ? prm.n_groups * prm.nchunk : prm.n_groups);
+                continue;
+            }
             const uint32_t uc = ua++;
             const int ab = uc % C::kABuf;
             if (uc >= (uint32_t)C::kABuf &&
@@ -538,7 +549,10 @@ __global__ void __launch_bounds__(BCfg<D, PASS>::kThreads, 1)
         };
         for (int64_t u = blockIdx.x; u < prm.n_units && ok; u += gridDim.x) {
             const BUnit U = bwd_unit<D, PASS>(prm, u);
-            if (unit_skipped(prm, U.bh)) continue;
+            if (unit_skipped(prm, U.bh)) {
+                u = skip_bh(U.bh, C::kRouteRows ? prm.n_groups * prm.nchunk : prm.n_groups);
+                continue;
+            }
             const uint32_t uc = ua++;
             const int ab = uc % C::kABuf;
             if (!C::kATmem) {
@@ -713,7 +727,10 @@ __global__ void __launch_bounds__(BCfg<D, PASS>::kThreads, 1)
         bool copied = false;  // T23C: the current unit's A rows were copied ahead
         for (int64_t u = blockIdx.x; u < prm.n_units && ok; u += gridDim.x) {
             const BUnit U = bwd_unit<D, PASS>(prm, u);
-            if (unit_skipped(prm, U.bh)) continue;
+            if (unit_skipped(prm, U.bh)) {
+                u = skip_bh(U.bh, C::kRouteRows ? prm.n_groups * prm.nchunk : prm.n_groups);
+                continue;
+            }
             const uint32_t uc = ua++;
             if (C::kATmem) {
                 if (!copied && !copy_a(U, uc)) {
@@ -771,7 +788,10 @@ __global__ void __launch_bounds__(BCfg<D, PASS>::kThreads, 1)
                 // unit's epilogue
                 for (int64_t un = u + gridDim.x; un < prm.n_units; un += gridDim.x) {
                     const BUnit V = bwd_unit<D, PASS>(prm, un);
-                    if (unit_skipped(prm, V.bh)) continue;
+                    if (unit_skipped(prm, V.bh)) {
+                        un = skip_bh(V.bh, prm.n_groups);
+                        continue;
+                    }
                     if (!copy_a(V, ua)) ok = false;
                     copied = ok;
                     break;
