@@ -239,14 +239,15 @@ FLAREPP_API flarepp_status flarepp_mixer_fwd_profiled(const flarepp_shape* shape
 /*
  * Training the mixer layer. flarepp_mixer_fwd_train is flarepp_mixer_fwd that also fills
  * `saved` (flarepp_mixer_saved_bytes(shape, n_proj) bytes of device memory, 16-byte aligned,
- * disjoint from the workspace; layout private) with the chain's saved state and Y.
+ * disjoint from the workspace; layout private) with the chain's saved state, Y and the
+ * n_proj projections (which the forward writes there instead of into its workspace).
  * flarepp_mixer_bwd then computes, for the output gradient dO [B, N, C]:
  *   dX [B, N, C], dW_in [n_proj * C, C], dWo [C, C] (both out x in, like the weights) and
  *   dseeds [H, M, D],
  * all bf16, written (not accumulated): dO through the output projection (dWo = dO^T merge(Y),
  * dY = split(dO Wo)), the chain's backward (App. A.5), then the projections' backward
  * (dW_in = dP^T X, dX = dP W_in, the gradients of tied projections added for n_proj = 2).
- * The projections are recomputed from X. workspace: flarepp_mixer_bwd_workspace_bytes(shape,
+ * The projections are read from `saved`. workspace: flarepp_mixer_bwd_workspace_bytes(shape,
  * n_proj) bytes, 256-byte aligned (its first 4 bytes are the device status word). Outputs
  * must be 16-byte aligned and disjoint from each other and from the inputs. Degenerate
  * shapes (N, M or B*H zero) write zeros to every non-empty gradient. Errors as for

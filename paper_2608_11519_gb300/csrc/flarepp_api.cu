@@ -475,15 +475,24 @@ bool mixer_layout(const Plan& p, int n_proj, MixerLayout* L) {
 }
 
 // State a training forward of the mixer keeps for its backward: the chain's saved state,
-// then Y [B][H][N][D] bf16.
+// then Y and the n_proj projections (K, V, K~, V~), each [B][H][N][D] bf16. The forward
+// writes the projections there directly, so keeping them costs memory only, and the
+// backward does not recompute them.
 struct MixerSaved {
-    size_t off_y, total;
+    size_t off_y, off_proj[4], total;
 };
 
-MixerSaved mixer_saved(const Plan& p) {
+MixerSaved mixer_saved(const Plan& p, int n_proj) {
+    const size_t tok = (size_t)p.BH * (size_t)p.N * (size_t)p.D * 2;
     MixerSaved m;
-    m.off_y = align_up(saved_layout(p).total, kWsAlign);
-    m.total = align_up(m.off_y + (size_t)p.BH * (size_t)p.N * (size_t)p.D * 2, kWsAlign);
+    size_t off = align_up(saved_layout(p).total, kWsAlign);
+    m.off_y = off;
+    off = align_up(off + tok, kWsAlign);
+    for (int i = 0; i < 4; ++i) {
+        m.off_proj[i] = off;
+        if (i < n_proj) off = align_up(off + tok, kWsAlign);
+    }
+    m.total = off;
     return m;
 }
 
@@ -526,8 +535,13 @@ flarepp_status mixer_impl(const flarepp_shape* shape, int n_proj, const void* X,
     auto mark = [&](int i) {
         return !events || cudaEventRecord((cudaEvent_t)events[i], st) == cudaSuccess;
     };
+    // the projections go to the workspace, or (training) into `saved` for the backward
+    const MixerSaved ms = mixer_saved(p, n_proj);
     void* proj[4];
-    for (int i = 0; i < 4; ++i) proj[i] = ws + L.off_proj[i < n_proj ? i : i - 2];
+    for (int i = 0; i < 4; ++i) {
+        const int k = i < n_proj ? i : i - 2;
+        proj[i] = saved ? saved + ms.off_proj[k] : ws + L.off_proj[k];
+    }
     // K, V, K~, V~ = X W_in^T, split into heads (eqs. flarepp_query_synthesis, flarepp_mixer)
     if (!mark(0) ||
         tc_projection(p.B, p.N, p.H, p.D, n_proj, X, W_in, proj, status, st) != cudaSuccess ||
@@ -535,7 +549,7 @@ flarepp_status mixer_impl(const flarepp_shape* shape, int n_proj, const void* X,
         return FLAREPP_ERR_CUDA;
     // the routing chain; the shared variant reads K, V as K~, V~ (App. C.2). A training
     // forward keeps Y and the chain's state in `saved`.
-    void* Y = saved ? saved + mixer_saved(p).off_y : ws + L.off_y;
+    void* Y = saved ? saved + ms.off_y : ws + L.off_y;
     stt = route_impl(shape, seeds, proj[2], proj[3], proj[0], proj[1], scale, Y, workspace,
                      p.total, stream, nullptr, nullptr, nullptr, 0, false, saved);
     if (stt != FLAREPP_OK) return stt;
@@ -548,21 +562,18 @@ flarepp_status mixer_impl(const flarepp_shape* shape, int n_proj, const void* X,
 }
 
 // Workspace of the mixer's backward: the chain's backward workspace first (its status word at
-// offset 0), then the recomputed projections, dY, the chain's gradients, the transposed
-// weights and the weight gradients' float32 partials.
+// offset 0), then dY, the chain's gradients, the transposed weights and the weight
+// gradients' float32 partials.
 struct MixerBwdLayout {
-    size_t off_proj[4], off_dy, off_dproj[4], off_wot, off_wint, off_part, total;
+    size_t off_dy, off_dproj[4], off_wot, off_wint, off_part, total;
 };
 
 MixerBwdLayout mixer_bwd_layout(const Plan& p, const BwdPlan& bp, int n_proj) {
     MixerBwdLayout L;
     const size_t tok = (size_t)p.BH * (size_t)p.N * (size_t)p.D * 2;
     const int64_t C = p.H * p.D;
+    (void)n_proj;
     size_t off = align_up(bp.total, kWsAlign);
-    for (int i = 0; i < 4; ++i) {
-        L.off_proj[i] = off;
-        if (i < n_proj) off = align_up(off + tok, kWsAlign);
-    }
     L.off_dy = off;
     off = align_up(off + tok, kWsAlign);
     for (int i = 0; i < 4; ++i) {
@@ -619,7 +630,7 @@ flarepp_status mixer_bwd_impl(const flarepp_shape* shape, int n_proj, const void
                 return FLAREPP_ERR_CUDA;
         return FLAREPP_OK;
     }
-    const MixerSaved ms = mixer_saved(p);
+    const MixerSaved ms = mixer_saved(p, n_proj);
     if (!saved || !aligned16(saved) || saved_bytes < ms.total) return FLAREPP_ERR_INVALID_ARGUMENT;
     const BwdPlan bp = make_bwd_plan(p);
     const MixerBwdLayout L = mixer_bwd_layout(p, bp, n_proj);
@@ -630,8 +641,8 @@ flarepp_status mixer_bwd_impl(const flarepp_shape* shape, int n_proj, const void
     const char* sv = (const char*)saved;
     const void* Y = sv + ms.off_y;
     if (cudaMemsetAsync(status, 0, sizeof(int32_t), st) != cudaSuccess) return FLAREPP_ERR_CUDA;
-    void* proj[4];
-    for (int i = 0; i < 4; ++i) proj[i] = ws + L.off_proj[i < n_proj ? i : i - 2];
+    const void* proj[4];
+    for (int i = 0; i < 4; ++i) proj[i] = sv + ms.off_proj[i < n_proj ? i : i - 2];
     void* dY = ws + L.off_dy;
     void* dproj[4];
     for (int i = 0; i < 4; ++i) dproj[i] = ws + L.off_dproj[i];
@@ -644,10 +655,9 @@ flarepp_status mixer_bwd_impl(const flarepp_shape* shape, int n_proj, const void
     if ((e = transpose_bf16(Wo, C, C, 1, WoT, st)) != cudaSuccess ||
         (e = transpose_bf16(W_in, n_proj * C, C, fold, WinT, st)) != cudaSuccess)
         return FLAREPP_ERR_CUDA;
-    // the projections again (cheaper to recompute than to keep), and dY = split(dO Wo)
+    // dY = split(dO Wo) (the projections K, V, K~, V~ come from the training forward)
     void* dys[4] = {dY, dY, dY, dY};
-    if (tc_projection(p.B, p.N, p.H, p.D, n_proj, X, W_in, proj, status, st) != cudaSuccess ||
-        tc_projection(p.B, p.N, p.H, p.D, 1, dO, WoT, dys, status, st) != cudaSuccess)
+    if (tc_projection(p.B, p.N, p.H, p.D, 1, dO, WoT, dys, status, st) != cudaSuccess)
         return FLAREPP_ERR_CUDA;
     // dWo = dO^T merge(Y)
     WgradSource sdo{0, 1, {dO, dO, dO, dO}};
@@ -680,7 +690,7 @@ size_t flarepp_mixer_saved_bytes(const flarepp_shape* shape, int n_proj) {
     if (flarepp::make_plan(shape, &p) != FLAREPP_OK) return 0;
     if ((n_proj != 2 && n_proj != 4) || p.dtype != FLAREPP_BF16) return 0;
     if (p.BH == 0 || p.N == 0 || p.M == 0) return 0;
-    return flarepp::mixer_saved(p).total;
+    return flarepp::mixer_saved(p, n_proj).total;
 }
 
 flarepp_status flarepp_mixer_fwd_train(const flarepp_shape* shape, int n_proj, const void* X,
@@ -691,7 +701,8 @@ flarepp_status flarepp_mixer_fwd_train(const flarepp_shape* shape, int n_proj, c
     const flarepp_status stt = flarepp::make_plan(shape, &p);
     if (stt != FLAREPP_OK) return stt;
     if (p.dtype == FLAREPP_BF16 && p.BH && p.N && p.M) {
-        const size_t need = flarepp::mixer_saved(p).total;
+        if (n_proj != 2 && n_proj != 4) return FLAREPP_ERR_INVALID_ARGUMENT;
+        const size_t need = flarepp::mixer_saved(p, n_proj).total;
         if (!saved || !flarepp::aligned16(saved) || saved_bytes < need)
             return FLAREPP_ERR_INVALID_ARGUMENT;
         if (flarepp::overlaps(saved, need, workspace, workspace_bytes))

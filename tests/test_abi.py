@@ -256,7 +256,10 @@ def test_mixer_training_entries_reject(lib):
     s = S(B=1, H=8, N=4096, M=64, D=32)
     sb = lambda sh, p: lib.flarepp_mixer_saved_bytes(ctypes.byref(sh), p)
     wb = lambda sh, p: lib.flarepp_mixer_bwd_workspace_bytes(ctypes.byref(sh), p)
-    assert sb(s, 4) > 8 * 4096 * 32 * 2 and wb(s, 4) > wb(s, 2) > 0
+    # the saved state holds Y and the projections (two more for n_proj = 4)
+    tok = 8 * 4096 * 32 * 2
+    assert sb(s, 4) - sb(s, 2) == 2 * tok and sb(s, 2) > 3 * tok
+    assert wb(s, 4) == wb(s, 2) > 0
     assert sb(s, 3) == 0 and wb(S(dtype=flarepp.F32), 4) == 0 and wb(S(N=0), 4) == 0
     v = lambda x: ctypes.c_void_p(x) if x else None
     base = [FAKE + (i + 1) * (1 << 36) for i in range(11)]
