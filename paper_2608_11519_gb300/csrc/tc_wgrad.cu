@@ -3,8 +3,12 @@
 // (dWo = dO^T merge(Y), dW_in = dP^T X, the backward of O = merge(Y) Wo^T and of
 // K, V, K~, V~ = X W_in^T in Fig. 1). Both operands are token-major in memory, so the
 // contraction runs over tokens with MN-major operand tiles: each tile is a set of D-wide
-// channel columns ("atoms"), one TMA box of 64 tokens x D channels each, swizzled to the
-// D-wide row like every other operand of the library. A channel source is either
+// channel columns ("atoms") of 64 tokens x D channels each, swizzled to the D-wide row like
+// every other operand of the library. A tile arrives as four-dimensional TMA boxes
+// {D channels, 64 tokens, atoms, 1} (the atom dimension steps over heads, or over the D-wide
+// column blocks of a plain matrix): one box per tile, or one per atom where a tile of a
+// HEADS source would cross from one tensor into the next. Few large boxes instead of one
+// per atom took dW_in from 1.20 to about 0.3 ms at mesh3d. A channel source is either
 //   HEADS: up to four tensors [B*H][N][D] side by side (channel r: tensor r / C, head
 //          (r % C) / D, column r % D), or
 //   PLAIN: one matrix [B][N][C] (channel r: column r).
@@ -56,6 +60,7 @@ struct WgParams {
     int64_t B, N, H, C;
     int64_t R, Cc;         // rows and columns of dW
     int a_heads, b_heads;  // source kinds: 1 = HEADS, 0 = PLAIN
+    int a_apb, b_apb;      // atoms per TMA box of each operand
     int NT;
     uint32_t idesc;
     int64_t chunk_len, chunks_per_b, n_chunks;
@@ -104,21 +109,23 @@ __device__ __forceinline__ bool warp_wait(uint32_t bar, uint32_t parity, volatil
 }
 
 // Load the atoms of channels [c0, c0 + width) of one source for tokens [n0, n0 + kTok) of
-// batch element b into consecutive atom slots at dst.
+// batch element b into consecutive atom slots at dst, in boxes of apb atoms (a box never
+// crosses from one tensor of a HEADS source into the next).
 template <int D>
 __device__ __forceinline__ void load_atoms(uint32_t dst, int heads_kind, const CUtensorMap* m0,
                                            const CUtensorMap* m1, const CUtensorMap* m2,
-                                           const CUtensorMap* m3, int64_t c0, int width,
-                                           int64_t C, int64_t H, int64_t b, int n0, uint32_t bar) {
+                                           const CUtensorMap* m3, int64_t c0, int width, int apb,
+                                           int64_t C, int64_t b, int n0, uint32_t bar) {
     using W = WCfg<D>;
-    for (int a = 0; a < width / D; ++a) {
-        const int64_t c = c0 + (int64_t)a * D;
+    for (int k = 0; k < width / (apb * D); ++k) {
+        const int64_t c = c0 + (int64_t)k * apb * D;
+        const uint32_t d = dst + k * apb * W::kAtom;
         if (heads_kind) {
-            const int64_t p = c / C, h = (c % C) / D;
+            const int64_t p = c / C;
             const CUtensorMap* m = p == 0 ? m0 : p == 1 ? m1 : p == 2 ? m2 : m3;
-            tma_load_3d(dst + a * W::kAtom, m, 0, n0, (int)(b * H + h), bar);
+            tma_load_4d(d, m, 0, n0, (int)((c % C) / D), (int)b, bar);
         } else {
-            tma_load_3d(dst + a * W::kAtom, m0, (int)c, n0, (int)b, bar);
+            tma_load_4d(d, m0, 0, n0, (int)(c / D), (int)b, bar);
         }
     }
 }
@@ -185,10 +192,10 @@ __global__ void __launch_bounds__(kThreads, 1)
                 if (elect_one()) {
                     const uint32_t dst = smem_u32(smem + st * W::kStage);
                     mbar_expect_tx(full0 + 8u * st, bytes);
-                    load_atoms<D>(dst, prm.a_heads, &tA0, &tA1, &tA2, &tA3, I.rt * kRowsW, kRowsW,
-                                  prm.C, prm.H, I.b, (int)n, full0 + 8u * st);
+                    load_atoms<D>(dst, prm.a_heads, &tA0, &tA1, &tA2, &tA3, I.rt * kRowsW,
+                                  kRowsW, prm.a_apb, prm.C, I.b, (int)n, full0 + 8u * st);
                     load_atoms<D>(dst + W::kAStage, prm.b_heads, &tB0, &tB1, &tB2, &tB3,
-                                  I.ct * prm.NT, prm.NT, prm.C, prm.H, I.b, (int)n,
+                                  I.ct * prm.NT, prm.NT, prm.b_apb, prm.C, I.b, (int)n,
                                   full0 + 8u * st);
                 }
                 __syncwarp();
@@ -333,30 +340,41 @@ PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
     return fn;
 }
 
-// bf16 {inner, rows, z}, boxes of D x kTok x 1, swizzled to the D-wide row
-bool make_map(CUtensorMap* m, const void* base, int64_t D, int64_t inner, int64_t rows,
-              int64_t z) {
+// bf16 {D channels, N tokens, atoms, B} with the given byte strides of dimensions 1..3;
+// boxes of D x kTok x `atoms` x 1, swizzled to the D-wide row. In shared memory a box is
+// atom-major: atom a is the kTok x D block at a * kTok * D * 2.
+bool make_map(CUtensorMap* m, const void* base, int64_t D, int64_t N, int64_t n_atoms,
+              int64_t B, int64_t s_tok, int64_t s_atom, int64_t s_b, int atoms) {
     auto fn = encode_fn();
     if (!fn) return false;
-    cuuint64_t dims[3] = {(cuuint64_t)inner, (cuuint64_t)rows, (cuuint64_t)z};
-    cuuint64_t strides[2] = {(cuuint64_t)(inner * 2), (cuuint64_t)(rows * inner * 2)};
-    cuuint32_t box[3] = {(cuuint32_t)D, (cuuint32_t)kTok, 1};
-    cuuint32_t estr[3] = {1, 1, 1};
+    cuuint64_t dims[4] = {(cuuint64_t)D, (cuuint64_t)N, (cuuint64_t)n_atoms, (cuuint64_t)B};
+    cuuint64_t strides[3] = {(cuuint64_t)s_tok, (cuuint64_t)s_atom, (cuuint64_t)s_b};
+    cuuint32_t box[4] = {(cuuint32_t)D, (cuuint32_t)kTok, (cuuint32_t)atoms, 1};
+    cuuint32_t estr[4] = {1, 1, 1, 1};
     const CUtensorMapSwizzle sw = D == 16 ? CU_TENSOR_MAP_SWIZZLE_32B
                                           : (D == 32 ? CU_TENSOR_MAP_SWIZZLE_64B
                                                      : CU_TENSOR_MAP_SWIZZLE_128B);
-    return fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(base), dims, strides, box,
+    return fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 4, const_cast<void*>(base), dims, strides, box,
               estr, CU_TENSOR_MAP_INTERLEAVE_NONE, sw, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
               CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
-// the maps of one source: HEADS (n tensors [B*H][N][D]) or PLAIN ([B][N][C])
+// Atoms per box for tiles of `width` channels: the whole tile, unless a tile of a HEADS
+// source could cross from one tensor into the next (C not a multiple of the width).
+int atoms_per_box(const WgradSource& s, int64_t C, int64_t D, int width) {
+    return (s.heads && C % width != 0) ? 1 : width / (int)D;
+}
+
+// the maps of one source, for boxes of `atoms` atoms: HEADS (n tensors [B*H][N][D], the
+// atoms are heads) or PLAIN ([B][N][C], the atoms are the D-wide column blocks)
 bool source_maps(CUtensorMap* m, const WgradSource& s, int64_t B, int64_t N, int64_t H,
-                 int64_t D) {
+                 int64_t D, int atoms) {
     for (int p = 0; p < 4; ++p) {
         const void* base = s.t[p < s.n ? p : 0];
-        const bool ok = s.heads ? make_map(&m[p], base, D, D, N, B * H)
-                                : make_map(&m[p], base, D, H * D, N, B);
+        const bool ok = s.heads ? make_map(&m[p], base, D, N, H, B, D * 2, N * D * 2,
+                                           H * N * D * 2, atoms)
+                                : make_map(&m[p], base, D, N, H, B, H * D * 2, D * 2,
+                                           N * H * D * 2, atoms);
         if (!ok) return false;
     }
     return true;
@@ -443,7 +461,9 @@ cudaError_t tc_wgrad(int64_t B, int64_t N, int64_t H, int64_t D, const WgradSour
     prm.part = part;
     prm.status = status;
     CUtensorMap ma[4], mb[4];
-    if (!source_maps(ma, a, B, N, H, D) || !source_maps(mb, b, B, N, H, D))
+    prm.a_apb = atoms_per_box(a, H * D, D, kRowsW);
+    prm.b_apb = atoms_per_box(b, H * D, D, w.NT);
+    if (!source_maps(ma, a, B, N, H, D, prm.a_apb) || !source_maps(mb, b, B, N, H, D, prm.b_apb))
         return cudaErrorInvalidValue;
     cudaError_t e;
     switch (D) {

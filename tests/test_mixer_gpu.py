@@ -114,6 +114,7 @@ BWD_SHAPES = [
     (1, 4, 300, 40, 16, 2),
     (2, 2, 257, 20, 64, 4),
     (1, 1, 130, 16, 32, 2),   # C = D: one head
+    (1, 6, 300, 32, 32, 4),   # C = 192: weight-gradient row tiles cross projections mid-tile
 ]
 
 
