@@ -302,7 +302,11 @@ __global__ void __launch_bounds__(kThreads, 1)
                 for (int k = 0; k < D / 16; ++k) tmem_ld16(acc + hh * D + 16 * k, v + 16 * k);
 #pragma unroll
                 for (int k = 0; k < D / 16; ++k) tmem_wait_ld16(v + 16 * k);
+                // the block is stored swizzled like the operands (16-byte chunk g of row r at
+                // g ^ (bits 7.. of the row's byte offset)), which the store map undoes: one
+                // thread per row then writes without shared-memory bank conflicts
                 uint4* dst = reinterpret_cast<uint4*>(stg + ((size_t)slot * kRows + r) * D * 2);
+                const int sw = ((r * D * 2) >> 7) & (D / 8 - 1);
 #pragma unroll
                 for (int g = 0; g < D / 8; ++g) {
                     uint4 o;
@@ -310,7 +314,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                     o.y = pack_bf16(__uint_as_float(v[8 * g + 2]), __uint_as_float(v[8 * g + 3]));
                     o.z = pack_bf16(__uint_as_float(v[8 * g + 4]), __uint_as_float(v[8 * g + 5]));
                     o.w = pack_bf16(__uint_as_float(v[8 * g + 6]), __uint_as_float(v[8 * g + 7]));
-                    dst[g] = o;
+                    dst[g ^ sw] = o;
                 }
             }
             tc_fence_before();
@@ -403,8 +407,8 @@ int tile_channels(int64_t H, int64_t D) {
     return (int)(heads * D);
 }
 
-// An unswizzled bf16 tensor of dims {inner, rows, z}, boxes of box_inner x 128 x 1 (the
-// epilogue's staged blocks).
+// A bf16 tensor of dims {inner, rows, z}, boxes of box_inner x 128 x 1 (the epilogue's
+// staged blocks), swizzled in shared memory to the box_inner-wide row.
 bool make_store_map(CUtensorMap* m, void* base, int64_t inner, int64_t rows, int64_t z,
                     uint32_t box_inner) {
     auto fn = encode_fn();
@@ -413,9 +417,12 @@ bool make_store_map(CUtensorMap* m, void* base, int64_t inner, int64_t rows, int
     cuuint64_t strides[2] = {(cuuint64_t)(inner * 2), (cuuint64_t)(rows * inner * 2)};
     cuuint32_t box[3] = {box_inner, (cuuint32_t)kRows, 1};
     cuuint32_t estr[3] = {1, 1, 1};
+    const CUtensorMapSwizzle sw = box_inner == 16 ? CU_TENSOR_MAP_SWIZZLE_32B
+                                  : (box_inner == 32 ? CU_TENSOR_MAP_SWIZZLE_64B
+                                                     : CU_TENSOR_MAP_SWIZZLE_128B);
     return fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, base, dims, strides, box, estr,
-              CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE,
-              CU_TENSOR_MAP_L2_PROMOTION_NONE, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+              CU_TENSOR_MAP_INTERLEAVE_NONE, sw, CU_TENSOR_MAP_L2_PROMOTION_NONE,
+              CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
 }  // namespace
