@@ -691,14 +691,17 @@ __global__ void __launch_bounds__(BCfg<D, PASS>::kThreads, 1)
                 const int64_t row = V.row0 + s * kRows + r;
                 const float uu =
                     row < V.rows ? exp2f(prm.Lrow[V.bh * V.rows + row] - prm.Rb[V.bh]) : 0.f;
+                // the tiles are swizzled to the D-wide row (16-byte chunk k of row r at
+                // k ^ (bits 7.. of the row's offset)): one-row-per-thread reads hit every bank
                 const uint8_t* src = abuf + ab * C::kABytes + s * C::kNT * C::kATile + r * D * 2;
+                const int sw = ((r * D * 2) >> 7) & (D / 8 - 1);
 #pragma unroll
                 for (int t = 0; t < C::kNT; ++t) {
                     uint32_t v[D / 2];
                     const uint4* p4 = reinterpret_cast<const uint4*>(src + t * C::kATile);
 #pragma unroll
                     for (int k = 0; k < D / 8; ++k) {
-                        const uint4 x = p4[k];
+                        const uint4 x = p4[k ^ sw];
                         v[4 * k] = x.x;
                         v[4 * k + 1] = x.y;
                         v[4 * k + 2] = x.z;
@@ -882,20 +885,18 @@ PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
     return fn;
 }
 
-// A bf16 [z][rows][D] tensor, boxes of box_rows x D, swizzled to the row width (or plain
-// rows, for tiles that are copied into TMEM row by row).
+// A bf16 [z][rows][D] tensor, boxes of box_rows x D, swizzled to the row width.
 bool make_map(CUtensorMap* m, const void* base, int64_t D, int64_t rows, int64_t z,
-              uint32_t box_rows, bool swizzle = true) {
+              uint32_t box_rows) {
     auto fn = encode_fn();
     if (!fn) return false;
     cuuint64_t dims[3] = {(cuuint64_t)D, (cuuint64_t)rows, (cuuint64_t)z};
     cuuint64_t strides[2] = {(cuuint64_t)(D * 2), (cuuint64_t)(rows * D * 2)};
     cuuint32_t box[3] = {(cuuint32_t)D, box_rows, 1};
     cuuint32_t estr[3] = {1, 1, 1};
-    const CUtensorMapSwizzle sw = !swizzle ? CU_TENSOR_MAP_SWIZZLE_NONE
-                                  : D == 16 ? CU_TENSOR_MAP_SWIZZLE_32B
-                                            : (D == 32 ? CU_TENSOR_MAP_SWIZZLE_64B
-                                                       : CU_TENSOR_MAP_SWIZZLE_128B);
+    const CUtensorMapSwizzle sw = D == 16 ? CU_TENSOR_MAP_SWIZZLE_32B
+                                          : (D == 32 ? CU_TENSOR_MAP_SWIZZLE_64B
+                                                     : CU_TENSOR_MAP_SWIZZLE_128B);
     return fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(base), dims, strides, box,
               estr, CU_TENSOR_MAP_INTERLEAVE_NONE, sw, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
               CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
@@ -926,7 +927,7 @@ cudaError_t launch_pass(const void* const* srcs, const Plan& p, BwdParams prm, c
         const bool a_side = k < 3;
         const bool per_head = a_side ? (prm.a0_per_head && k == 0) : (prm.i0_per_head && k == 3);
         if (!make_map(&maps[k], base, p.D, a_side ? arows : irows, per_head ? p.H : p.BH,
-                      a_side ? (uint32_t)kRows : (uint32_t)Cf::kItem, !(a_side && Cf::kATmem)))
+                      a_side ? (uint32_t)kRows : (uint32_t)Cf::kItem))
             return cudaErrorInvalidValue;
     }
     int dev = 0, sms = kNumSMs;
