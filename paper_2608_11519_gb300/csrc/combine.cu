@@ -28,9 +28,12 @@ __device__ __forceinline__ int slots_of_route(int64_t M, int64_t m, int64_t sub_
     return (int)(ns / na);
 }
 
-// One warp per (bh, m): merge the partial slots in ascending order (App. A.3):
+// One warp per (bh, m): merge the partial slots (App. A.3):
 //   g = max_r mx_r; w_r = 2^(mx_r - g); out = sum_r w_r acc_r / sum_r w_r l_r;
 //   the row's base-2 log-normaliser is g + log2(sum_r w_r l_r).
+// The lanes take the slots 32 at a time for the maximum and the weights (warp reductions);
+// the value sums then run over the slots with lanes as channels, each slot's weight taken
+// from its lane, so that the loads of consecutive slots are independent.
 template <int D>
 __global__ void combine_kernel(const float* __restrict__ pmax, const float* __restrict__ psum,
                                const float* __restrict__ pacc, int64_t rows, int64_t M,
@@ -45,26 +48,36 @@ __global__ void combine_kernel(const float* __restrict__ pmax, const float* __re
     const int64_t bh = row / M, m = row % M;
     const int used = slots_of_route(M, m, sub_per_chunk, group);
     const int64_t nslot = nchunk * sub_per_chunk;
+    const int64_t n = nchunk * used;  // the row's slots, s -> chunk s / used, part s % used
+    auto slot_row = [&](int64_t s) {
+        return (bh * nslot + (s / used) * sub_per_chunk + s % used) * M + m;
+    };
     float g = -INFINITY;
-    for (int64_t c = 0; c < nchunk; ++c)
-        for (int p = 0; p < used; ++p)
-            g = fmaxf(g, pmax[(bh * nslot + c * sub_per_chunk + p) * M + m]);
+    for (int64_t s = lane; s < n; s += 32) g = fmaxf(g, pmax[slot_row(s)]);
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) g = fmaxf(g, __shfl_xor_sync(0xffffffffu, g, off));
     float a = 0.f, u[PER];
 #pragma unroll
     for (int i = 0; i < PER; ++i) u[i] = 0.f;
     if (g != -INFINITY) {
-        for (int64_t c = 0; c < nchunk; ++c) {
-            for (int p = 0; p < used; ++p) {
-                const int64_t r = (bh * nslot + c * sub_per_chunk + p) * M + m;
-                const float w = fast_exp2(pmax[r] - g);
-                a = fmaf(w, psum[r], a);
+        for (int64_t s0 = 0; s0 < n; s0 += 32) {
+            const int64_t s = s0 + lane;
+            const float w = s < n ? fast_exp2(pmax[slot_row(s)] - g) : 0.f;
+            if (s < n) a = fmaf(w, psum[slot_row(s)], a);
+            const int cnt = (int)min((int64_t)32, n - s0);
+#pragma unroll 8
+            for (int j = 0; j < cnt; ++j) {
+                const float wj = __shfl_sync(0xffffffffu, w, j);
+                const int64_t r = slot_row(s0 + j);
 #pragma unroll
                 for (int i = 0; i < PER; ++i) {
                     const int d = lane + 32 * i;
-                    if (d < D) u[i] = fmaf(w, pacc[r * D + d], u[i]);
+                    if (d < D) u[i] = fmaf(wj, pacc[r * D + d], u[i]);
                 }
             }
         }
+#pragma unroll
+        for (int off = 16; off > 0; off >>= 1) a += __shfl_xor_sync(0xffffffffu, a, off);
     }
     const float inv = a > 0.f ? 1.f / a : 0.f;
     if (lse && lane == 0) lse[row] = a > 0.f ? g + log2f(a) : -INFINITY;
