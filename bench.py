@@ -275,6 +275,16 @@ def run_reference(args, w):
 FLARE_METRIC = "routed tokens·heads/sec for the 2-call FLARE layer (fixed queries); % of roofline"
 
 
+def chain_bwd_launches(w):
+    """Kernels of one chain backward: on the tensor-core path c3, two operand copies, R3 and
+    its reduce, T23 (with, for D <= 32, the range and flag kernels, the w dZ operand and the
+    merged pass before it), R2 and its reduce, T1, R1 and the seeds' reduce; on the
+    CUDA-core path c3 and three route passes, two token passes and three reduces."""
+    if w.dtype != "bf16":
+        return 9
+    return 11 + (4 if w.D <= 32 else 0)
+
+
 def flare_launches(w):
     """Kernels of one FLARE call: encode, merge and decode, plus the negation of the
     bf16 queries when the scale is negative."""
@@ -474,7 +484,8 @@ def run_train(args, w, flarepp, world, rank, dev, peaks, x, Y, ws, stream):
             "step_roofline": {"roofline_us": t_step * 1e6, "frac": t_step / (ms * 1e-3),
                               "flops": "42 BNMHD", "tensors": 15},
             "cpu_baseline": cpu, "e2e": None, "clocks": clk,
-            "gpu_launches": None,
+            "gpu_launches": (5 + (1 if w.dtype == "bf16" and w.scale < 0 else 0)
+                             + chain_bwd_launches(w)) * args.steps,
         }
         print(json.dumps(line), flush=True)
     if world > 1:
@@ -580,7 +591,11 @@ def run_mixer_train(args, w, flarepp, world, rank, dev, peaks, stream):
                        "l2": "inputs larger than L2 (no flush)",
                        "parallelism": f"replicas x{world}"},
             "stage_ms": {"forward_train": fwd_ms, "backward": bwd_ms}, "roofline": roof,
-            "cpu_baseline": None, "e2e": None, "clocks": clk, "gpu_launches": None,
+            "cpu_baseline": None, "e2e": None, "clocks": clk,
+            # forward: projection, the chain's five kernels, output projection; backward: two
+            # weight transposes, dY, dWo and its reduce, the chain's backward, dW_in and its
+            # reduce, dX
+            "gpu_launches": (7 + 8 + chain_bwd_launches(w)) * args.steps,
         }
         print(json.dumps(line), flush=True)
     if world > 1:
