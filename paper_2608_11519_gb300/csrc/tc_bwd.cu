@@ -3,10 +3,10 @@
 // Every SDPA(A, B, C) of the chain is differentiated from its saved log-normaliser L
 // (base 2) and c = <dO, O>:  P = 2^(x - L) with x = scale log2(e) <a, b>,
 // dS = P o (dP - c) with dP = <dO, C>, and the products dA = s dS B, dB = s dS^T A,
-// dC = P^T dO. Five passes cover the three calls. In every pass a score tile of 128 TMEM
-// lanes x kItem columns is produced by the tensor cores, turned into bf16 P and dS in place
-// by a softmax warpgroup, and consumed as the TMEM A operand of one or two accumulating
-// products whose B operand is the same streamed item:
+// dC = P^T dO. Five passes cover the three calls (T23 in one of two forms). In every pass a
+// score tile of 128 TMEM lanes x kItem columns is produced by the tensor cores, turned into
+// bf16 P and dS in place by a softmax warpgroup, and consumed as the TMEM A operand of one or
+// two accumulating products whose B operand is the same streamed item:
 //
 //   route-row passes (TMEM lanes are routes, items are tokens; per-chunk partial sums):
 //     R3  call 3, column statistics L3, c3 of the tokens:
@@ -20,15 +20,19 @@
 //         acc0 += dS Q (-> dK / s),  acc1 += P2 dZ (-> dV)
 //     T1  call 1, route statistics L1, c1:  S = Kt Qs^T, dP = Vt dQ^T;
 //         acc0 += dS Qs (-> dKt / s),  acc1 += P dQ (-> dVt)
-// Score products take both operands from shared memory (TMA, swizzled, K-major); the
-// accumulating products read P or dS from TMEM and the item, MN-major, from shared memory.
+//     T23C  T23 with its two dP products merged into one of depth 2D (see slice_math),
+//         one exponential per score and its A tiles in TMEM; it serves every (b, h) whose
+//         statistics allow it (D = 16, 32), T23 the others
+// Score products take both operands from shared memory (TMA, swizzled, K-major), except in
+// T23C (A from TMEM); the accumulating products read P or dS from TMEM and the item,
+// MN-major, from shared memory.
 //
 // Roles: one MMA warp per TMEM stream of 128 rows (a commit stalls only the warp that
 // issues it), one softmax warpgroup per stream (warps 4..), and a TMA producer warp that
 // also stages each item's column statistics in shared memory. A pass has as many streams as
-// its TMEM columns allow (at most four) and items of 64 rows when three streams fit with
-// them, else 32; the softmax works on 16-column slices in packed f32x2 arithmetic. A work
-// unit is (b*h, group of NS x 128 rows, chunk of items).
+// its TMEM columns allow (at most four), with the widest item (64, 48 or 32 rows) that fits
+// that count (T23 and T23C: two streams of 64 rows); the softmax works on 16-column slices
+// in packed f32x2 arithmetic. A work unit is (b*h, group of NS x 128 rows, chunk of items).
 // Every wait is bounded (2 s of %globaltimer): on expiry the kernel records
 // FLAREPP_ERR_TIMEOUT in the status word, every role leaves its loops, the producer waits
 // for its copies in flight, the MMA issuer for its products, and TMEM is freed.
