@@ -262,9 +262,7 @@ def run_reference(args, w):
             "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
             "ms_per_step": dt * 1e3, "higher_is_better": True, "scaling": "weak",
             "vs_baseline": None, "dtype": "f64", "data": "synthetic",
-            "config": {"workload": w.name, "variant": args.variant,
-                       "B": w.B, "H": w.H, "N": w.N, "M": w.M, "D": w.D,
-                       "input_dtype": w.dtype, "sample_tokens": n},
+            "config": arm_config(w, args.variant, world),
             "cpu_baseline": {"value": value, "unit": UNIT, "cores": oracle.max_threads(),
                              "kind": "oracle", "sample": sample},
             "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0,
@@ -276,6 +274,28 @@ def run_reference(args, w):
 # ------------------------------------------------------------------ our arm
 
 FLARE_METRIC = "routed tokens·heads/sec for the 2-call FLARE layer (fixed queries); % of roofline"
+
+
+def arm_config(w, variant, world):
+    """The `config` of a bench line; both arms of one variant print the same one."""
+    cfg = {"workload": w.name, "variant": variant, "B": w.B, "H": w.H, "N": w.N, "M": w.M,
+           "D": w.D}
+    tok = w.B * w.H * w.N
+    big = "inputs larger than L2 (no flush)"
+    if variant in ("flarepp", "shared"):
+        cfg["keys"] = f"clustered, {w.n_centres} centres" if w.n_centres else "iid"
+        cfg["l2"] = big if 5 * tok * w.D * w.elt_bytes > 2 * 129e6 else "inputs near L2 size"
+    elif variant == "flare":
+        cfg["queries"] = "the workload's seeds, as learned queries"
+        cfg["l2"] = big if 3 * tok * w.D * w.elt_bytes > 2 * 129e6 else "inputs near L2 size"
+    elif variant == "train":
+        cfg["l2"] = big
+    else:  # the mixer variants
+        cfg["C"] = w.H * w.D
+        cfg["projections"] = 2 if variant == "mixer_shared" else 4
+        cfg["l2"] = big
+    cfg["parallelism"] = f"replicas x{world}"
+    return cfg
 
 
 def chain_bwd_launches(w):
@@ -382,11 +402,7 @@ def run_flare(args, w, flarepp, world, rank, dev, peaks, x, Y, ws, stream):
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms,
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
             "dtype": "bf16" if w.dtype == "bf16" else "f32", "data": "synthetic",
-            "config": {"workload": w.name, "variant": "flare", "B": w.B, "H": w.H, "N": w.N,
-                       "M": w.M, "D": w.D, "queries": "the workload's seeds, as learned queries",
-                       "l2": "inputs larger than L2 (no flush)"
-                       if 3 * tok * w.D * w.elt_bytes > 2 * 129e6 else "inputs near L2 size",
-                       "parallelism": f"replicas x{world}"},
+            "config": arm_config(w, "flare", world),
             "roofline": roof, "cpu_baseline": cpu, "e2e": e2e, "clocks": clk,
             "gpu_launches": flare_launches(w) * args.steps,
         }
@@ -479,9 +495,7 @@ def run_train(args, w, flarepp, world, rank, dev, peaks, x, Y, ws, stream):
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms,
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
             "dtype": "bf16" if w.dtype == "bf16" else "f32", "data": "synthetic",
-            "config": {"workload": w.name, "variant": "train", "B": w.B, "H": w.H, "N": w.N,
-                       "M": w.M, "D": w.D, "l2": "inputs larger than L2 (no flush)",
-                       "parallelism": f"replicas x{world}"},
+            "config": arm_config(w, "train", world),
             "stage_ms": {"forward_train": fwd_ms, "backward": bwd_ms},
             "roofline": roof,
             "step_roofline": {"roofline_us": t_step * 1e6, "frac": t_step / (ms * 1e-3),
@@ -589,10 +603,7 @@ def run_mixer_train(args, w, flarepp, world, rank, dev, peaks, stream):
             "n_gpus": world, "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms,
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
             "dtype": "bf16", "data": "synthetic",
-            "config": {"workload": w.name, "variant": "mixer_train", "B": w.B, "H": w.H,
-                       "N": w.N, "M": w.M, "D": w.D, "C": C, "projections": 4,
-                       "l2": "inputs larger than L2 (no flush)",
-                       "parallelism": f"replicas x{world}"},
+            "config": arm_config(w, "mixer_train", world),
             "stage_ms": {"forward_train": fwd_ms, "backward": bwd_ms}, "roofline": roof,
             "cpu_baseline": None, "e2e": None, "clocks": clk,
             # forward: projection, the chain's five kernels, output projection; backward: two
@@ -681,10 +692,7 @@ def run_mixer(args, w, flarepp, world, rank, dev, peaks, stream):
             "n_gpus": world, "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms,
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
             "dtype": "bf16", "data": "synthetic",
-            "config": {"workload": w.name, "variant": args.variant, "B": w.B, "H": w.H, "N": w.N,
-                       "M": w.M, "D": w.D, "C": C, "projections": n_proj,
-                       "l2": "inputs larger than L2 (no flush)",
-                       "parallelism": f"replicas x{world}"},
+            "config": arm_config(w, args.variant, world),
             "stage_ms": stage_ms, "roofline": roof, "layer_roofline": layer,
             "cpu_baseline": cpu, "e2e": None, "clocks": clk, "gpu_launches": 7 * args.steps,
         }
@@ -826,12 +834,7 @@ def run_ours(args, w):
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms_per_step,
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
             "dtype": "bf16" if w.dtype == "bf16" else "f32", "data": "synthetic",
-            "config": {"workload": w.name, "variant": args.variant,
-                       "B": w.B, "H": w.H, "N": w.N, "M": w.M, "D": w.D,
-                       "keys": f"clustered, {w.n_centres} centres" if w.n_centres else "iid",
-                       "l2": "inputs larger than L2 (no flush)"
-                       if 5 * tok * w.D * w.elt_bytes > 2 * 129e6 else "inputs near L2 size",
-                       "parallelism": f"replicas x{world}"},
+            "config": arm_config(w, args.variant, world),
             "roofline": roof, "chain_roofline": chain, "stage_ms": stage_ms,
             "cpu_baseline": cpu, "e2e": e2e, "clocks": clk,
             "gpu_launches": 5 * args.steps,
