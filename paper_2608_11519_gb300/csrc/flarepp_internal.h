@@ -171,6 +171,7 @@ cudaError_t tc_encode(const Plan& p, int call, const void* k, const void* v, con
                       float scale, char* ws, cudaStream_t st);
 // Rows per tensor-core work unit (route group of the encode, token group of the decode).
 int64_t tc_group_rows(int64_t D);
+int64_t tc_encode_item_rows(int64_t D);  // tokens per item of the tensor-core encode
 // Decode call 3: Y = SDPA(K, Q, Z) from the Q and Z operand copies; also each token's
 // base-2 log-normaliser into `lse` [BH][N] when it is not null.
 cudaError_t tc_decode(const Plan& p, const void* K, float scale, void* Y, char* ws,

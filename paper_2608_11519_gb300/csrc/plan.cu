@@ -14,7 +14,6 @@ namespace {
 constexpr int64_t kMaxM = 2048;
 constexpr int64_t kMaxTokenHeads = int64_t(1) << 40;  // B*H*N limit (index headroom)
 constexpr int64_t kMaxTmaCoord = 2147483647 - 4096;  // TMA coordinates are signed 32-bit
-constexpr int64_t kTcItem = 64;               // tokens per tensor-core encode item
 
 bool mul_ok(int64_t a, int64_t b, int64_t* out) { return !__builtin_mul_overflow(a, b, out); }
 
@@ -58,9 +57,10 @@ flarepp_status make_plan(const flarepp_shape* s, Plan* p) {
     } else {
         // Tensor-core encode: a work unit is (bh, group of <= 512 routes, chunk of tokens) and
         // one persistent CTA per SM walks the units. Pick the chunk count that minimises
-        // waves x (64-token items per unit, scaled by the group's route tiles, + a fixed
-        // per-unit cost of about three items).
+        // waves x (items per unit, scaled by the group's route tiles, + a fixed per-unit
+        // cost of about three items); chunks are whole items.
         p->tc_group = tc_group_rows(s->D);
+        const int64_t kTcItem = tc_encode_item_rows(s->D);  // tokens per encode item
         p->n_groups = cdiv(s->M, p->tc_group);
         p->sub_per_chunk = 4;
         const int64_t ns = p->tc_group / 128;

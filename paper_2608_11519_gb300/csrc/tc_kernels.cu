@@ -56,11 +56,15 @@ constexpr float kLog2e = 1.4426950408889634f;
 // Sum of one item's probabilities above which the reference max is recomputed exactly.
 constexpr float kFastLimit = 281474976710656.0f;  // 2^48
 
-template <int D>
+template <int D, bool DEC>
 struct Cfg {
-    static constexpr int kItem = D == 64 ? 32 : 64;   // streamed rows per item
-    static constexpr int B = 1;                       // score buffers per stream
-    static constexpr int kABuf = D == 64 ? 1 : 2;     // TMEM copies of the A tiles
+    // Streamed rows per item. The encode's units are long (hundreds of items), so one TMEM
+    // copy of its A tiles costs nothing at unit boundaries, and the columns that frees widen
+    // its items to 80 rows: fewer per-item round trips per token. The decode's units are only
+    // M/64 items, so it keeps two copies (the next unit's A tiles go in ahead) and 64 rows.
+    static constexpr int kItem = D == 64 ? 32 : (DEC ? 64 : 80);
+    static constexpr int B = 1;                                   // score buffers per stream
+    static constexpr int kABuf = (D == 64 || !DEC) ? 1 : 2;     // TMEM copies of the A tiles
     static constexpr int kGroup = NS * kTileRows;     // resident rows per work unit
     static constexpr int kStages = D == 64 ? 8 : (kItem == 32 ? 16 : 8);  // multiple of 4
     static constexpr int kATile = kTileRows * D * 2;  // one 128-row operand tile
@@ -123,7 +127,7 @@ struct Unit {
 
 template <int D, bool DEC>
 __device__ __forceinline__ Unit get_unit(const TcParams& p, int64_t u) {
-    using C = Cfg<D>;
+    using C = Cfg<D, DEC>;
     Unit U;
     if (DEC) {
         U.tg = u % p.n_tok_groups;
@@ -207,12 +211,14 @@ struct SoftmaxStream {
     }
 };
 
-// Max over the valid columns [0, nv) of one 32-column half (columns base .. base + 31).
-__device__ __forceinline__ float half_max(const uint32_t* sr, int base, int nv) {
+// Max over the valid columns [0, nv) of one chunk of W = 32 or 16 columns (columns
+// base .. base + W - 1).
+template <int W>
+__device__ __forceinline__ float chunk_max(const uint32_t* sr, int base, int nv) {
     float a0 = -INFINITY, a1 = -INFINITY, a2 = -INFINITY, a3 = -INFINITY;
-    if (base + 32 <= nv) {
+    if (base + W <= nv) {
 #pragma unroll
-        for (int k = 0; k < 32; k += 8) {
+        for (int k = 0; k < W; k += 8) {
             a0 = max3f(a0, __uint_as_float(sr[k]), __uint_as_float(sr[k + 1]));
             a1 = max3f(a1, __uint_as_float(sr[k + 2]), __uint_as_float(sr[k + 3]));
             a2 = max3f(a2, __uint_as_float(sr[k + 4]), __uint_as_float(sr[k + 5]));
@@ -220,21 +226,23 @@ __device__ __forceinline__ float half_max(const uint32_t* sr, int base, int nv) 
         }
     } else {
 #pragma unroll
-        for (int k = 0; k < 32; ++k)
+        for (int k = 0; k < W; ++k)
             if (base + k < nv) a0 = fmaxf(a0, __uint_as_float(sr[k]));
     }
     return max3f(a0, a1, fmaxf(a2, a3));
 }
 
-// P = 2^(c S - m) for one 32-column half, packed bf16 pairs into pr[0..15]; returns the
-// half's row sum. Columns at or beyond nv are not part of the softmax: probability 0.
-__device__ __forceinline__ float exp_half(const uint32_t* sr, uint32_t* pr, int base, int nv,
-                                          float c, uint64_t c2, float m) {
-    if (base + 32 <= nv) {
+// P = 2^(c S - m) for one chunk of W = 32 or 16 columns, packed bf16 pairs into
+// pr[0 .. W/2); returns the chunk's row sum. Columns at or beyond nv are not part of the
+// softmax: probability 0.
+template <int W>
+__device__ __forceinline__ float exp_chunk(const uint32_t* sr, uint32_t* pr, int base, int nv,
+                                           float c, uint64_t c2, float m) {
+    if (base + W <= nv) {
         const uint64_t nm2 = pack_f32x2(-m, -m);
         uint64_t acc0 = 0, acc1 = 0;  // two packed (lo, hi) partial sums
 #pragma unroll
-        for (int k = 0; k < 16; k += 2) {
+        for (int k = 0; k < W / 2; k += 2) {
             pr[k] = exp2_pair(__uint_as_float(sr[2 * k]), __uint_as_float(sr[2 * k + 1]), c2,
                               nm2, acc0);
             pr[k + 1] = exp2_pair(__uint_as_float(sr[2 * k + 2]), __uint_as_float(sr[2 * k + 3]),
@@ -247,7 +255,7 @@ __device__ __forceinline__ float exp_half(const uint32_t* sr, uint32_t* pr, int 
     }
     float t0 = 0.f, t1 = 0.f;
 #pragma unroll
-    for (int k = 0; k < 16; ++k) {
+    for (int k = 0; k < W / 2; ++k) {
         const float p0 =
             base + 2 * k < nv ? ex2(fmaf(__uint_as_float(sr[2 * k]), c, -m)) : 0.f;
         const float p1 =
@@ -260,7 +268,8 @@ __device__ __forceinline__ float exp_half(const uint32_t* sr, uint32_t* pr, int 
 }
 
 // P for a whole item tile of ITEM columns at TMEM column scol (S is read 32 columns at a
-// time); packed bf16 pairs go to pr[0 .. ITEM/2). Returns the row sum. With FIRST_REF and
+// time, and a last 16 when ITEM is 80); packed bf16 pairs go to pr[0 .. ITEM/2). Returns the
+// row sum. With FIRST_REF and
 // `first` the reference m is first set to the row's own first score, c S[0]: any score of
 // the row is a valid reference (that score alone contributes 2^0 = 1 to the sum, so the
 // sum never underflows), and a reference far below the row's maximum shows up as a sum
@@ -275,7 +284,14 @@ __device__ __forceinline__ float exp_tile(uint32_t scol, uint32_t* pr, int nv, f
         tmem_ld32(scol + 32 * h, sr);
         tmem_wait_ld32(sr);
         if (FIRST_REF && h == 0 && first) m = c * __uint_as_float(sr[0]);
-        sum += exp_half(sr, pr + 16 * h, 32 * h, nv, c, c2, m);
+        sum += exp_chunk<32>(sr, pr + 16 * h, 32 * h, nv, c, c2, m);
+    }
+    if (ITEM % 32 == 16) {
+        constexpr int base = ITEM - 16;
+        uint32_t sr[16];
+        tmem_ld16(scol + base, sr);
+        tmem_wait_ld16(sr);
+        sum += exp_chunk<16>(sr, pr + base / 2, base, nv, c, c2, m);
     }
     return sum;
 }
@@ -283,17 +299,16 @@ __device__ __forceinline__ float exp_tile(uint32_t scol, uint32_t* pr, int nv, f
 // One item of this warpgroup's stream for this thread's row: read S, update the online
 // softmax, write P back over S, signal the stream's MMA warp. S of item j being ready
 // means the PV of item j - B has completed, so the warpgroup leader frees that item's ring
-// stage. Returns false when the kernel is aborting. FIRST_REF (the decode, whose units
-// are short) takes the first item's reference from its first score; otherwise (the
-// encode, whose units are long) the first item's reference is its exact maximum, which
-// measured faster there.
-template <int D, bool FIRST_REF>
+// stage. Returns false when the kernel is aborting. The decode (DEC), whose units are
+// short, takes the first item's reference from its first score; the encode, whose units
+// are long, takes the first item's exact maximum, which measured faster there.
+template <int D, bool DEC>
 __device__ __forceinline__ bool softmax_step(SoftmaxStream& S, const Unit& U, uint32_t tmem,
                                              uint32_t lane_off, float c, uint64_t c2,
                                              uint32_t sready_s, uint32_t pready_s, uint32_t empty0,
                                              bool wg_leader, uint32_t it0,
                                              volatile int* abort_flag, int* status) {
-    using C = Cfg<D>;
+    using C = Cfg<D, DEC>;
     const int j = S.j;
     const int b = j % C::B;
     const uint32_t par_j = (S.ph0 + (uint32_t)j) & 1u;
@@ -310,9 +325,9 @@ __device__ __forceinline__ bool softmax_step(SoftmaxStream& S, const Unit& U, ui
     const uint32_t scol = tmem + lane_off + C::kColS + (S.s * C::B + b) * C::kItem;
     uint32_t pr[C::kItem / 2];
     float sum = 0.f;
-    bool slow = !FIRST_REF && j == 0;
+    bool slow = !DEC && j == 0;
     if (!slow) {
-        sum = exp_tile<C::kItem, FIRST_REF>(scol, pr, nv, c, c2, S.m, j == 0);
+        sum = exp_tile<C::kItem, DEC>(scol, pr, nv, c, c2, S.m, j == 0);
         slow = __any_sync(0xffffffffu, !(sum <= kFastLimit));
     }
     if (slow) {
@@ -323,7 +338,13 @@ __device__ __forceinline__ bool softmax_step(SoftmaxStream& S, const Unit& U, ui
             uint32_t sr[32];
             tmem_ld32(scol + 32 * h, sr);
             tmem_wait_ld32(sr);
-            mx = fmaxf(mx, half_max(sr, 32 * h, nv));
+            mx = fmaxf(mx, chunk_max<32>(sr, 32 * h, nv));
+        }
+        if (C::kItem % 32 == 16) {
+            uint32_t sr[16];
+            tmem_ld16(scol + C::kItem - 16, sr);
+            tmem_wait_ld16(sr);
+            mx = fmaxf(mx, chunk_max<16>(sr, C::kItem - 16, nv));
         }
         const float cand = mx * c;
         bool need = false;
@@ -351,10 +372,14 @@ __device__ __forceinline__ bool softmax_step(SoftmaxStream& S, const Unit& U, ui
         sum = exp_tile<C::kItem, false>(scol, pr, nv, c, c2, S.m, false);
     }
     S.l += sum;
-    if (C::kItem == 64)
+    if (C::kItem == 80) {
         tmem_st32(scol, pr);
-    else
+        tmem_st8(scol + 32, pr + 32);
+    } else if (C::kItem == 64) {
+        tmem_st32(scol, pr);
+    } else {
         tmem_st16(scol, pr);
+    }
     tmem_wait_st();
     tc_fence_before();
     mbar_arrive(pready_s + 8u * b);
@@ -371,7 +396,7 @@ __device__ __forceinline__ bool finish_stream(SoftmaxStream& S, const Unit& U,
                                               uint32_t lane_off, int r, uint32_t sready_s,
                                               uint32_t empty0, bool wg_leader, uint32_t it0,
                                               volatile int* abort_flag) {
-    using C = Cfg<D>;
+    using C = Cfg<D, DEC>;
     const int a = S.s % U.n_a;
     const int par = S.s / U.n_a;
     float o[D];
@@ -437,10 +462,10 @@ __device__ __forceinline__ bool finish_stream(SoftmaxStream& S, const Unit& U,
 
 // PV of stream s: O_s (+)= P (score buffer pb) * C-tile of ring stage `st` (one elected
 // lane issues).
-template <int D>
+template <int D, bool DEC>
 __device__ __forceinline__ void issue_pv(uint32_t tmem, uint8_t* ring, int s, int pb, int st,
                                          int npv) {
-    using C = Cfg<D>;
+    using C = Cfg<D, DEC>;
     const uint32_t cb = smem_u32(ring + st * C::kStage + C::kItemTile);
 #pragma unroll
     for (int k = 0; k < C::kItem / 16; ++k) {
@@ -486,7 +511,7 @@ struct Producer {
     }
     // Issue what can be issued now (at most a few copies). Returns true if anything was.
     __device__ __forceinline__ bool poll(const TcParams& prm) {
-        using C = Cfg<D>;
+        using C = Cfg<D, DEC>;
         constexpr uint32_t kAhead = C::kABuf == 2 ? 1u : 0u;
         bool any = false;
         for (int n = 0; n < 4; ++n) {
@@ -538,7 +563,7 @@ struct Producer {
     }
     // After an abort: wait (bounded) until the newest copy of every buffer has landed.
     __device__ __forceinline__ void drain() {
-        using C = Cfg<D>;
+        using C = Cfg<D, DEC>;
         const uint64_t t0 = globaltimer_ns();
         for (int st = 0; st < C::kStages; ++st) {
             if ((uint32_t)st >= it) break;
@@ -563,7 +588,7 @@ template <int D, bool DEC>
 __global__ void __launch_bounds__(kThreads, 1)
     tc_chain_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
                     const __grid_constant__ CUtensorMap tmC, const TcParams prm) {
-    using C = Cfg<D>;
+    using C = Cfg<D, DEC>;
     extern __shared__ uint8_t smem_raw[];
     uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                                ~static_cast<uintptr_t>(1023));
@@ -682,7 +707,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                 if (!wait(pready0 + 16u * s + 8u * pb, pc & 1)) return false;
                 ++pc;
                 tc_fence_after();
-                issue_pv<D>(tmem, ring, s, jo % C::B, (jo & 1) ? stg1 : stg0, npv);
+                issue_pv<D, DEC>(tmem, ring, s, jo % C::B, (jo & 1) ? stg1 : stg0, npv);
                 ++npv;
                 return true;
             };
@@ -873,7 +898,7 @@ bool make_map(CUtensorMap* m, const void* base, int64_t D, int64_t rows, int64_t
 template <int D, bool DEC>
 cudaError_t launch(const CUtensorMap& a, const CUtensorMap& b, const CUtensorMap& c,
                    const TcParams& prm, cudaStream_t st) {
-    using Cf = Cfg<D>;
+    using Cf = Cfg<D, DEC>;
     static cudaError_t attr = cudaFuncSetAttribute(
         tc_chain_kernel<D, DEC>, cudaFuncAttributeMaxDynamicSharedMemorySize, Cf::kSmem);
     if (attr != cudaSuccess) return attr;
@@ -898,10 +923,13 @@ cudaError_t launch_d(int64_t D, const CUtensorMap& a, const CUtensorMap& b, cons
 
 }  // namespace
 
-// Streamed rows per item (the TMA box height of the ring tiles): Cfg<D>::kItem.
+// Streamed rows per item (the TMA box height of the ring tiles) of the encode or decode.
+template <bool DEC>
 uint32_t item_rows(int64_t D) {
-    return D == 16 ? Cfg<16>::kItem : (D == 32 ? Cfg<32>::kItem : Cfg<64>::kItem);
+    return D == 16 ? Cfg<16, DEC>::kItem : (D == 32 ? Cfg<32, DEC>::kItem : Cfg<64, DEC>::kItem);
 }
+
+int64_t tc_encode_item_rows(int64_t D) { return item_rows<false>(D); }
 
 int64_t tc_group_rows(int64_t D) {
     (void)D;
@@ -922,8 +950,8 @@ cudaError_t tc_encode(const Plan& p, int call, const void* k, const void* v, con
         a_z = p.BH;
     }
     if (!make_map(&ma, a_src, p.D, p.M, a_z, kTileRows, false) ||
-        !make_map(&mb, k, p.D, p.N, p.BH, item_rows(p.D), true) ||
-        !make_map(&mc, v, p.D, p.N, p.BH, item_rows(p.D), true))
+        !make_map(&mb, k, p.D, p.N, p.BH, item_rows<false>(p.D), true) ||
+        !make_map(&mc, v, p.D, p.N, p.BH, item_rows<false>(p.D), true))
         return cudaErrorInvalidValue;
     TcParams prm{};
     prm.BH = p.BH;
@@ -947,8 +975,8 @@ cudaError_t tc_decode(const Plan& p, const void* K, float scale, void* Y, char* 
                       cudaStream_t st, float* lse) {
     CUtensorMap ma, mb, mc;
     if (!make_map(&ma, K, p.D, p.N, p.BH, kTileRows, false) ||
-        !make_map(&mb, ws + p.off_qop, p.D, p.M, p.BH, item_rows(p.D), true) ||
-        !make_map(&mc, ws + p.off_zop, p.D, p.M, p.BH, item_rows(p.D), true))
+        !make_map(&mb, ws + p.off_qop, p.D, p.M, p.BH, item_rows<true>(p.D), true) ||
+        !make_map(&mc, ws + p.off_zop, p.D, p.M, p.BH, item_rows<true>(p.D), true))
         return cudaErrorInvalidValue;
     TcParams prm{};
     prm.BH = p.BH;
