@@ -31,10 +31,12 @@ __device__ __forceinline__ int slots_of_route(int64_t M, int64_t m, int64_t sub_
 // One warp per (bh, m): merge the partial slots (App. A.3):
 //   g = max_r mx_r; w_r = 2^(mx_r - g); out = sum_r w_r acc_r / sum_r w_r l_r;
 //   the row's base-2 log-normaliser is g + log2(sum_r w_r l_r).
-// The lanes take the slots 32 at a time for the maximum and the weights (warp reductions);
-// the value sums then run over the slots with lanes as channels, each slot's weight taken
-// from its lane, so that the loads of consecutive slots are independent.
-template <int D>
+// The slots are taken KB (4 or 32) at a time, and every load of a block is issued at once:
+// the lanes load one slot's maximum and sum each, and (lanes as channels) the values of all
+// KB slots. The blocks are merged online with a running maximum, so a row costs one round of
+// memory latency per KB slots (the merge is the same in every run: deterministic). KB = 4
+// serves rows of at most four slots with few instructions.
+template <int D, int KB>
 __global__ void combine_kernel(const float* __restrict__ pmax, const float* __restrict__ psum,
                                const float* __restrict__ pacc, int64_t rows, int64_t M,
                                int64_t nchunk, int64_t sub_per_chunk, int64_t group,
@@ -52,32 +54,46 @@ __global__ void combine_kernel(const float* __restrict__ pmax, const float* __re
     auto slot_row = [&](int64_t s) {
         return (bh * nslot + (s / used) * sub_per_chunk + s % used) * M + m;
     };
-    float g = -INFINITY;
-    for (int64_t s = lane; s < n; s += 32) g = fmaxf(g, pmax[slot_row(s)]);
-#pragma unroll
-    for (int off = 16; off > 0; off >>= 1) g = fmaxf(g, __shfl_xor_sync(0xffffffffu, g, off));
-    float a = 0.f, u[PER];
+    float g = -INFINITY, a = 0.f, u[PER];
 #pragma unroll
     for (int i = 0; i < PER; ++i) u[i] = 0.f;
-    if (g != -INFINITY) {
-        for (int64_t s0 = 0; s0 < n; s0 += 32) {
-            const int64_t s = s0 + lane;
-            const float w = s < n ? fast_exp2(pmax[slot_row(s)] - g) : 0.f;
-            if (s < n) a = fmaf(w, psum[slot_row(s)], a);
-            const int cnt = (int)min((int64_t)32, n - s0);
-#pragma unroll 8
-            for (int j = 0; j < cnt; ++j) {
-                const float wj = __shfl_sync(0xffffffffu, w, j);
-                const int64_t r = slot_row(s0 + j);
+    for (int64_t s0 = 0; s0 < n; s0 += KB) {
+        const int cnt = (int)min((int64_t)KB, n - s0);
+        const bool in = lane < cnt;
+        const int64_t rl = in ? slot_row(s0 + lane) : 0;
+        const float mx = in ? pmax[rl] : -INFINITY;
+        const float ps = in ? psum[rl] : 0.f;
+        float v[KB][PER];
 #pragma unroll
-                for (int i = 0; i < PER; ++i) {
-                    const int d = lane + 32 * i;
-                    if (d < D) u[i] = fmaf(wj, pacc[r * D + d], u[i]);
-                }
+        for (int j = 0; j < KB; ++j) {
+            const int64_t rj = j < cnt ? slot_row(s0 + j) : 0;
+#pragma unroll
+            for (int i = 0; i < PER; ++i) {
+                const int d = lane + 32 * i;
+                v[j][i] = (j < cnt && d < D) ? pacc[rj * D + d] : 0.f;
             }
         }
+        float gb = mx;
 #pragma unroll
-        for (int off = 16; off > 0; off >>= 1) a += __shfl_xor_sync(0xffffffffu, a, off);
+        for (int off = 16; off > 0; off >>= 1) gb = fmaxf(gb, __shfl_xor_sync(0xffffffffu, gb, off));
+        if (gb == -INFINITY) continue;  // every slot of the block is empty
+        const float gn = fmaxf(g, gb);
+        const float sc = fast_exp2(g - gn);  // 0 while g is -inf
+        a *= sc;
+#pragma unroll
+        for (int i = 0; i < PER; ++i) u[i] *= sc;
+        const float w = in ? fast_exp2(mx - gn) : 0.f;
+        float aw = w * ps;
+#pragma unroll
+        for (int off = 16; off > 0; off >>= 1) aw += __shfl_xor_sync(0xffffffffu, aw, off);
+        a += aw;
+#pragma unroll
+        for (int j = 0; j < KB; ++j) {
+            const float wj = __shfl_sync(0xffffffffu, w, j);
+#pragma unroll
+            for (int i = 0; i < PER; ++i) u[i] = fmaf(wj, v[j][i], u[i]);
+        }
+        g = gn;
     }
     const float inv = a > 0.f ? 1.f / a : 0.f;
     if (lse && lane == 0) lse[row] = a > 0.f ? g + log2f(a) : -INFINITY;
@@ -113,11 +129,17 @@ cudaError_t combine(const Plan& p, int call, char* ws, bool negate, cudaStream_t
     const float* psum = (const float*)(ws + p.off_psum);
     const float* pacc = (const float*)(ws + p.off_pacc);
     const float sign = negate ? -1.f : 1.f;
+    // slots per row at most: nchunk x sub_per_chunk
+    const bool few = p.nchunk * p.sub_per_chunk <= 4;
 #define FLAREPP_COMBINE(DD)                                                                    \
-    combine_kernel<DD><<<(unsigned)blocks, warps * 32, 0, st>>>(pmax, psum, pacc, rows, p.M,  \
-                                                                p.nchunk, p.sub_per_chunk,     \
-                                                                p.tc_group,                    \
-                                                                out32, outop, sign, lse);
+    if (few)                                                                                   \
+        combine_kernel<DD, 4><<<(unsigned)blocks, warps * 32, 0, st>>>(                        \
+            pmax, psum, pacc, rows, p.M, p.nchunk, p.sub_per_chunk, p.tc_group, out32, outop,  \
+            sign, lse);                                                                        \
+    else                                                                                       \
+        combine_kernel<DD, 32><<<(unsigned)blocks, warps * 32, 0, st>>>(                       \
+            pmax, psum, pacc, rows, p.M, p.nchunk, p.sub_per_chunk, p.tc_group, out32, outop,  \
+            sign, lse);
     switch (p.D) {
         case 16: FLAREPP_COMBINE(16) break;
         case 32: FLAREPP_COMBINE(32) break;
