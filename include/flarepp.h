@@ -173,6 +173,17 @@ FLAREPP_API flarepp_status flarepp_route_fwd_host(const flarepp_shape* shape, co
                                                   size_t device_buffer_bytes, void* stream);
 
 /*
+ * flarepp_flare_fwd (FLARE with the learned queries Q [H, M, D]) on HOST buffers Q, K, V, Y,
+ * with the same head groups and overlapped copies as flarepp_route_fwd_host (K and V are
+ * copied once). device_buffer: at least flarepp_route_host_buffer_bytes(shape) bytes,
+ * 256-byte aligned. Asynchronous and errors as flarepp_route_fwd_host.
+ */
+FLAREPP_API flarepp_status flarepp_flare_fwd_host(const flarepp_shape* shape, const void* Q,
+                                                  const void* K, const void* V, float scale,
+                                                  void* Y, void* device_buffer,
+                                                  size_t device_buffer_bytes, void* stream);
+
+/*
  * flarepp_route_fwd without a caller-provided workspace. The paper has no counterpart: this
  * entry point exists for callers that cannot allocate device memory when they call the
  * chain. Examples are a plugin whose host application owns all device memory, and a

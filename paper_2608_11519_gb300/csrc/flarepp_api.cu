@@ -125,7 +125,7 @@ flarepp_status route_impl(const flarepp_shape* shape, const void* seeds, const v
 // reads a per-(b, h) copy of Q as its keys.
 flarepp_status flare_impl(const flarepp_shape* shape, const void* Qh, const void* K, const void* V,
                           float scale, void* Y, void* workspace, size_t workspace_bytes,
-                          void* stream, float* Z_out) {
+                          void* stream, float* Z_out, bool reset_status = true) {
     Plan p;
     flarepp_status stt = make_plan(shape, &p);
     if (stt != FLAREPP_OK) return stt;
@@ -162,7 +162,7 @@ flarepp_status flare_impl(const flarepp_shape* shape, const void* Qh, const void
     char* ws = (char*)workspace;
     const bool tc = p.path == kPathTc;
     const bool neg = scale < 0.f;
-    if (cudaMemsetAsync(ws + p.off_status, 0, sizeof(int32_t), st) != cudaSuccess)
+    if (reset_status && cudaMemsetAsync(ws + p.off_status, 0, sizeof(int32_t), st) != cudaSuccess)
         return FLAREPP_ERR_CUDA;
     // the encode of call 1 with the learned queries, merged into Z
     if (tc && neg && negate_bf16(Qh, ws + p.off_seedneg, p.H * p.M * p.D, st) != cudaSuccess)
@@ -264,9 +264,12 @@ bool host_layout(const flarepp_shape* s, const Plan& p, const HostGroups& g, Hos
     return true;
 }
 
+// The chain (or, with `flare`, FLARE with the learned queries in seeds_h, K~ = K and V~ = V)
+// on host buffers.
 flarepp_status route_host_impl(const flarepp_shape* shape, const void* seeds_h, const void* Kt_h,
                                const void* Vt_h, const void* K_h, const void* V_h, float scale,
-                               void* Y_h, void* dbuf, size_t dbuf_bytes, void* stream) {
+                               void* Y_h, void* dbuf, size_t dbuf_bytes, void* stream,
+                               bool flare = false) {
     Plan p;
     flarepp_status stt = make_plan(shape, &p);
     if (stt != FLAREPP_OK) return stt;
@@ -353,9 +356,11 @@ flarepp_status route_host_impl(const flarepp_shape* shape, const void* seeds_h, 
         const size_t so = (size_t)(bh0 % p.H) * (size_t)p.M * (size_t)p.D * elt;
         ok = cudaStreamWaitEvent(st, e_in[k], 0) == cudaSuccess;
         if (!ok) break;
-        rc = route_impl(&gs, db + L.off_seeds + so, db + off_kt + o, db + off_vt + o,
-                        db + L.off_k + o, db + L.off_v + o, scale, db + L.off_y + o, db,
-                        L.ws_bytes, st, nullptr, nullptr, nullptr, 0, k == 0);
+        rc = flare ? flare_impl(&gs, db + L.off_seeds + so, db + L.off_k + o, db + L.off_v + o,
+                                scale, db + L.off_y + o, db, L.ws_bytes, st, nullptr, k == 0)
+                   : route_impl(&gs, db + L.off_seeds + so, db + off_kt + o, db + off_vt + o,
+                                db + L.off_k + o, db + L.off_v + o, scale, db + L.off_y + o, db,
+                                L.ws_bytes, st, nullptr, nullptr, nullptr, 0, k == 0);
         if (rc != FLAREPP_OK) break;
         ok = cudaEventRecord(e_done[k], st) == cudaSuccess &&
              cudaStreamWaitEvent(cout, e_done[k], 0) == cudaSuccess &&
@@ -856,6 +861,13 @@ size_t flarepp_route_host_buffer_bytes(const flarepp_shape* shape) {
     flarepp::HostLayout L;
     if (!flarepp::host_layout(shape, p, g, &L)) return 0;
     return L.total;
+}
+
+flarepp_status flarepp_flare_fwd_host(const flarepp_shape* shape, const void* Q, const void* K,
+                                      const void* V, float scale, void* Y, void* device_buffer,
+                                      size_t device_buffer_bytes, void* stream) {
+    return flarepp::route_host_impl(shape, Q, K, V, K, V, scale, Y, device_buffer,
+                                    device_buffer_bytes, stream, true);
 }
 
 flarepp_status flarepp_route_fwd_host(const flarepp_shape* shape, const void* seeds,

@@ -24,6 +24,7 @@ _DTYPES = {torch.float32: F32, torch.bfloat16: BF16}
 EXPORTED = ("flarepp_route_workspace_bytes", "flarepp_route_fwd", "flarepp_route_fwd_debug",
             "flarepp_route_fwd_profiled", "flarepp_route_fwd_noalloc",
             "flarepp_flare_fwd", "flarepp_route_host_buffer_bytes", "flarepp_route_fwd_host",
+            "flarepp_flare_fwd_host",
             "flarepp_mixer_workspace_bytes", "flarepp_mixer_fwd", "flarepp_mixer_fwd_profiled",
             "flarepp_mixer_saved_bytes", "flarepp_mixer_fwd_train",
             "flarepp_mixer_bwd_workspace_bytes", "flarepp_mixer_bwd",
@@ -83,6 +84,8 @@ def load(path: str = None):
     lib.flarepp_route_host_buffer_bytes.argtypes = [sp]
     lib.flarepp_route_fwd_host.restype = ctypes.c_int
     lib.flarepp_route_fwd_host.argtypes = [sp, vp, vp, vp, vp, vp, ctypes.c_float, vp, vp, sz, vp]
+    lib.flarepp_flare_fwd_host.restype = ctypes.c_int
+    lib.flarepp_flare_fwd_host.argtypes = [sp, vp, vp, vp, ctypes.c_float, vp, vp, sz, vp]
     lib.flarepp_mixer_workspace_bytes.restype = sz
     lib.flarepp_mixer_workspace_bytes.argtypes = [sp, ctypes.c_int]
     lib.flarepp_mixer_fwd.restype = ctypes.c_int
@@ -549,5 +552,37 @@ def route_fwd_host(seeds, Kt, Vt, K, V, scale=None, Y_host=None, device="cuda", 
                                     nbytes, ctypes.c_void_p(st.cuda_stream))
     if rc != 0:
         raise FlareppError(rc, "flarepp_route_fwd_host")
+    st.synchronize()
+    return Y_host
+
+
+def flare_fwd_host(Q, K, V, scale=None, Y_host=None, device="cuda", workspace=None, stream=None):
+    """FLARE with learned queries Q [H, M, D] on host tensors through
+    ``flarepp_flare_fwd_host``: copies in, FLARE, Y copied back into ``Y_host`` (allocated
+    pinned here if not given), overlapped by head groups. Returns Y_host once it is filled."""
+    lib = load()
+    shape = _shape_of(Q, K, V, K, V)
+    for t in (Q, K, V):
+        if t.is_cuda:
+            raise ValueError("flare_fwd_host takes host tensors")
+    if scale is None:
+        scale = 1.0 / math.sqrt(shape.D)
+    if Y_host is None:
+        Y_host = torch.empty(K.shape, dtype=K.dtype, pin_memory=True)
+    elif tuple(Y_host.shape) != tuple(K.shape) or Y_host.dtype != K.dtype or Y_host.is_cuda:
+        raise ValueError("Y_host must be a host tensor of K's shape and dtype")
+    dev = torch.device(device)
+    if dev.index is None:
+        dev = torch.device("cuda", torch.cuda.current_device())
+    nbytes = int(lib.flarepp_route_host_buffer_bytes(ctypes.byref(shape)))
+    ws = workspace if workspace is not None else Workspace()
+    buf = ws.get(nbytes, dev) if nbytes else None
+    st = stream if stream is not None else torch.cuda.current_stream(dev)
+    rc = lib.flarepp_flare_fwd_host(ctypes.byref(shape), _ptr(Q), _ptr(K), _ptr(V),
+                                    float(scale), _ptr(Y_host),
+                                    None if buf is None else ctypes.c_void_p(buf.data_ptr()),
+                                    nbytes, ctypes.c_void_p(st.cuda_stream))
+    if rc != 0:
+        raise FlareppError(rc, "flarepp_flare_fwd_host")
     st.synchronize()
     return Y_host

@@ -165,6 +165,23 @@ def test_host_entry_sizes_and_rejects_before_any_cuda_call(lib):
     assert host_call(S(), buf=FAKE + 7 * (1 << 36) + 128) == E.ERR_WORKSPACE  # not aligned
     assert host_call(S(N=0)) == E.OK  # empty Y: nothing to do
 
+    # FLARE on host buffers: the same checks through its own entry (Q, K, V, then Y)
+    def flare_host_call(shape, Y=FAKE + 6 * (1 << 36), buf=FAKE + 7 * (1 << 36), nbytes=None,
+                        scale=0.25):
+        ptrs = [ctypes.c_void_p(FAKE + (i + 1) * (1 << 36)) for i in range(3)]
+        nb = hb(shape) if nbytes is None else nbytes
+        return lib.flarepp_flare_fwd_host(ctypes.byref(shape), *ptrs, ctypes.c_float(scale),
+                                          ctypes.c_void_p(Y) if Y else None,
+                                          ctypes.c_void_p(buf) if buf else None, nb, None)
+
+    assert flare_host_call(S(D=48)) == E.ERR_UNSUPPORTED
+    assert flare_host_call(S(), scale=float("inf")) == E.ERR_INVALID_ARGUMENT
+    assert flare_host_call(S(), Y=0) == E.ERR_INVALID_ARGUMENT
+    assert flare_host_call(S(), Y=FAKE + 2 * (1 << 36) + 64) == E.ERR_INVALID_ARGUMENT  # Y on K
+    assert flare_host_call(S(), buf=0) == E.ERR_WORKSPACE
+    assert flare_host_call(S(), nbytes=1024) == E.ERR_WORKSPACE
+    assert flare_host_call(S(N=0)) == E.OK
+
 
 def test_backward_entry_sizes_and_rejects_before_any_cuda_call(lib):
     E = flarepp

@@ -268,6 +268,30 @@ def test_flare_fixed_queries(B, H, N, M, D, dtype, scale):
     _check("Y", _np(Y), Yo, TOL[dtype])
 
 
+@pytest.mark.parametrize("B,H,N,M,D,dtype,scale", [
+    (1, 8, 5000, 128, 32, "bf16", None),   # eight head groups
+    (2, 3, 1500, 40, 16, "bf16", -0.3),    # groups of whole batch elements, negative scale
+    (1, 4, 700, 20, 16, "f32", None),      # CUDA-core path
+])
+def test_flare_host_entry(B, H, N, M, D, dtype, scale):
+    """FLARE on host buffers (flarepp_flare_fwd_host, copies overlapped by head groups)
+    against the oracle; a group's plan may chunk its tokens differently from the whole
+    call's, so the comparison with the device entry is the oracle's tolerance, not bits. A
+    second call on the same device buffer gives the same bits and leaves the status clear."""
+    w = inputs.Workload("flare", B, H, N, M, D, dtype)
+    s = w.scale if scale is None else scale
+    x = inputs.make_inputs(w, seed=8)
+    f = inputs.to_f64_numpy(x)
+    _, Yo = oracle.flare(f["seeds"], f["K"], f["V"], s)
+    xh = {k: v.pin_memory() for k, v in x.items()}
+    ws = flarepp.Workspace()
+    Yh = flarepp.flare_fwd_host(xh["seeds"], xh["K"], xh["V"], s, workspace=ws).clone()
+    _check("Y host", _np(Yh), Yo, TOL[dtype])
+    Yh2 = flarepp.flare_fwd_host(xh["seeds"], xh["K"], xh["V"], s, workspace=ws)
+    assert torch.equal(Yh, Yh2)
+    assert flarepp.device_status((x["seeds"], x["K"], x["V"], x["K"], x["V"]), ws) == 0
+
+
 def test_shared_projection():
     """The shared-projection variant ties Kt, Vt to K, V (App. cost_model): the chain on
     aliased inputs, on device buffers and through the host entry (which copies K, V once)."""
