@@ -19,7 +19,8 @@
  *     Inputs and Y share one element type, chosen by flarepp_shape.dtype.
  *   - Pointers: device pointers (or managed memory), each 16-byte aligned. The caller owns
  *     every buffer; the library keeps no pointer after a call returns and allocates no
- *     device memory. Y must not overlap any input or the workspace.
+ *     device memory. Y must not overlap any input or the workspace, nor the workspace an
+ *     input (FLAREPP_ERR_INVALID_ARGUMENT).
  *   - Stream: all work is enqueued on `stream` (a cudaStream_t; NULL = legacy default
  *     stream) and the call returns without synchronising. The workspace must stay untouched
  *     until that work has finished.
@@ -219,7 +220,8 @@ FLAREPP_API flarepp_status flarepp_route_fwd_noalloc(const flarepp_shape* shape,
  *     uses K, V as K~, V~).
  *   X: [B, N, C]; W_in: [n_proj * C, C], out x in (row block 0 is W_K, then W_V, W_K~, W_V~);
  *     Wo: [C, C], out x in; seeds: [H, M, D]; O: [B, N, C]. Device pointers, 16-byte
- *     aligned; O must not overlap an input or the workspace. No biases.
+ *     aligned; neither O nor the workspace may overlap an input, nor O the workspace. No
+ *     biases.
  *   workspace: flarepp_mixer_workspace_bytes(shape, n_proj) bytes, 256-byte aligned; it holds
  *     the chain's workspace (its status word at offset 0, read by
  *     flarepp_route_device_status), the projections and Y.
@@ -260,7 +262,8 @@ FLAREPP_API flarepp_status flarepp_mixer_fwd_profiled(const flarepp_shape* shape
  * (dW_in = dP^T X, dX = dP W_in, the gradients of tied projections added for n_proj = 2).
  * The projections are read from `saved`. workspace: flarepp_mixer_bwd_workspace_bytes(shape,
  * n_proj) bytes, 256-byte aligned (its first 4 bytes are the device status word). Outputs
- * must be 16-byte aligned and disjoint from each other and from the inputs. Degenerate
+ * must be 16-byte aligned and disjoint from each other, from the inputs and from `saved`;
+ * the workspace must be disjoint from all of them. Degenerate
  * shapes (N, M or B*H zero) write zeros to every non-empty gradient. Errors as for
  * flarepp_mixer_fwd.
  */
@@ -317,7 +320,8 @@ FLAREPP_API size_t flarepp_route_bwd_workspace_bytes(const flarepp_shape* shape)
  *   dseeds [H, M, D], dKt, dVt, dK, dV [B, H, N, D]: outputs in the input dtype, written
  *     (not accumulated), 16-byte aligned, disjoint from each other and from every input.
  *   workspace: device memory, 256-byte aligned, flarepp_route_bwd_workspace_bytes(shape)
- *     bytes; its first 4 bytes are the device status word (flarepp_route_device_status).
+ *     bytes, disjoint from every input, `saved` and the outputs; its first 4 bytes are the
+ *     device status word (flarepp_route_device_status).
  * Degenerate shapes (N, M or B*H zero) write zeros to every non-empty output. Errors:
  * FLAREPP_ERR_INVALID_ARGUMENT (a missing, misaligned or overlapping pointer, too small a
  * saved buffer, non-finite scale), FLAREPP_ERR_UNSUPPORTED (as flarepp_route_fwd),

@@ -21,6 +21,13 @@ bool overlaps(const void* a, size_t na, const void* b, size_t nb) {
     return a0 < b0 + nb && b0 < a0 + na;
 }
 
+bool spans_overlap(const void* const* ptrs, const size_t* bytes, int n, const void* p,
+                   size_t nb) {
+    for (int i = 0; i < n; ++i)
+        if (overlaps(p, nb, ptrs[i], bytes[i])) return true;
+    return false;
+}
+
 flarepp_status route_impl(const flarepp_shape* shape, const void* seeds, const void* Kt,
                           const void* Vt, const void* K, const void* V, float scale, void* Y,
                           void* workspace, size_t workspace_bytes, void* stream, float* Q_out,
@@ -61,6 +68,15 @@ flarepp_status route_impl(const flarepp_shape* shape, const void* seeds, const v
         if (!workspace || ((uintptr_t)workspace % kWsAlign) != 0) return FLAREPP_ERR_WORKSPACE;
         if (workspace_bytes < p.total) return FLAREPP_ERR_WORKSPACE;
         if (overlaps(Y, tok_bytes, workspace, p.total)) return FLAREPP_ERR_INVALID_ARGUMENT;
+        // the kernels write the workspace while they read the inputs
+        const void* ins[5] = {seeds, Kt, Vt, K, V};
+        const size_t nb[5] = {seed_bytes, tok_bytes, tok_bytes, tok_bytes, tok_bytes};
+        if (spans_overlap(ins, nb, 5, workspace, p.total)) return FLAREPP_ERR_INVALID_ARGUMENT;
+        float* const qz[2] = {Q_out, Z_out};
+        for (float* q : qz)
+            if (q && qz_bytes &&
+                (overlaps(q, qz_bytes, workspace, p.total) || overlaps(q, qz_bytes, Y, tok_bytes)))
+                return FLAREPP_ERR_INVALID_ARGUMENT;
     }
 
     // degenerate shapes
@@ -149,6 +165,12 @@ flarepp_status flare_impl(const flarepp_shape* shape, const void* Qh, const void
         if (!workspace || ((uintptr_t)workspace % kWsAlign) != 0) return FLAREPP_ERR_WORKSPACE;
         if (workspace_bytes < p.total) return FLAREPP_ERR_WORKSPACE;
         if (overlaps(Y, tok_bytes, workspace, p.total)) return FLAREPP_ERR_INVALID_ARGUMENT;
+        const void* ins[3] = {Qh, K, V};
+        const size_t nb[3] = {q_bytes, tok_bytes, tok_bytes};
+        if (spans_overlap(ins, nb, 3, workspace, p.total)) return FLAREPP_ERR_INVALID_ARGUMENT;
+        if (Z_out && z_bytes &&
+            (overlaps(Z_out, z_bytes, workspace, p.total) || overlaps(Z_out, z_bytes, Y, tok_bytes)))
+            return FLAREPP_ERR_INVALID_ARGUMENT;
     }
     if (p.BH == 0) return FLAREPP_OK;
     if (p.N == 0) {  // every route has no keys: Z = 0 (App. A.3); Y is empty
@@ -302,7 +324,7 @@ flarepp_status route_host_impl(const flarepp_shape* shape, const void* seeds_h, 
     cudaStream_t cin = nullptr, cout = nullptr;
     cudaEvent_t ev[kMaxEvents] = {};
     int n_ev = 0;
-    if (g.n > 64) return FLAREPP_ERR_UNSUPPORTED;  // not reached: host_groups targets 4
+    if (g.n > 64) return FLAREPP_ERR_UNSUPPORTED;  // not reached: host_groups makes at most 8
     flarepp_status rc = FLAREPP_OK;
     auto cleanup = [&]() {
         for (int i = 0; i < n_ev; ++i) cudaEventDestroy(ev[i]);
@@ -378,13 +400,6 @@ flarepp_status route_host_impl(const flarepp_shape* shape, const void* seeds_h, 
 
 // ---------------------------------------------------------------- training forward, backward
 
-bool spans_overlap(const void* const* ptrs, const size_t* bytes, int n, const void* p,
-                   size_t nb) {
-    for (int i = 0; i < n; ++i)
-        if (overlaps(p, nb, ptrs[i], bytes[i])) return true;
-    return false;
-}
-
 flarepp_status route_fwd_train_impl(const flarepp_shape* shape, const void* seeds, const void* Kt,
                                     const void* Vt, const void* K, const void* V, float scale,
                                     void* Y, void* saved, size_t saved_bytes, void* workspace,
@@ -441,7 +456,7 @@ flarepp_status route_bwd_impl(const flarepp_shape* shape, const void* seeds, con
             for (int j = 0; j < i; ++j)
                 if (overlaps(outs[i], ob[i], outs[j], ob[j])) return FLAREPP_ERR_INVALID_ARGUMENT;
         }
-        if (overlaps(saved, sv.total, workspace, bp.total)) return FLAREPP_ERR_INVALID_ARGUMENT;
+        if (spans_overlap(ins, ib, 8, workspace, bp.total)) return FLAREPP_ERR_INVALID_ARGUMENT;
     }
     // degenerate shapes: every gradient that exists is zero
     if (!work) {
@@ -532,6 +547,11 @@ flarepp_status mixer_impl(const flarepp_shape* shape, int n_proj, const void* X,
     if (!workspace || ((uintptr_t)workspace % kWsAlign) != 0 || workspace_bytes < L.total)
         return FLAREPP_ERR_WORKSPACE;
     if (overlaps(O, x_bytes, workspace, L.total)) return FLAREPP_ERR_INVALID_ARGUMENT;
+    {
+        const void* ins[4] = {X, W_in, Wo, seeds};
+        const size_t nb[4] = {x_bytes, w_bytes, wo_bytes, seed_bytes};
+        if (spans_overlap(ins, nb, 4, workspace, L.total)) return FLAREPP_ERR_INVALID_ARGUMENT;
+    }
     if (p.M == 0)  // every decode row has no keys: Y = 0, so O = 0
         return cudaMemsetAsync(O, 0, x_bytes, st) == cudaSuccess ? FLAREPP_OK : FLAREPP_ERR_CUDA;
     char* ws = (char*)workspace;
@@ -641,6 +661,17 @@ flarepp_status mixer_bwd_impl(const flarepp_shape* shape, int n_proj, const void
     const MixerBwdLayout L = mixer_bwd_layout(p, bp, n_proj);
     if (!workspace || ((uintptr_t)workspace % kWsAlign) != 0 || workspace_bytes < L.total)
         return FLAREPP_ERR_WORKSPACE;
+    {
+        const void* all[9] = {X, W_in, Wo, seeds, dO, saved, dX, dW_in, dWo};
+        const size_t nb[9] = {x_bytes, w_bytes, wo_bytes, seed_bytes, x_bytes, ms.total,
+                              x_bytes, w_bytes, wo_bytes};
+        if (spans_overlap(all, nb, 9, workspace, L.total) ||
+            overlaps(dseeds, seed_bytes, workspace, L.total) ||
+            overlaps(dseeds, seed_bytes, saved, ms.total))
+            return FLAREPP_ERR_INVALID_ARGUMENT;
+        for (int i = 0; i < 4; ++i)
+            if (overlaps(outs[i], ob[i], saved, ms.total)) return FLAREPP_ERR_INVALID_ARGUMENT;
+    }
     char* ws = (char*)workspace;
     int* status = (int*)(ws + bp.off_status);
     const char* sv = (const char*)saved;

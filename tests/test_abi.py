@@ -107,6 +107,24 @@ def test_invalid_arguments_rejected_before_launch(lib):
     assert call(lib, S(), ws_bytes=16) == E.ERR_WORKSPACE
     assert call(lib, S(), ws=FAKE + 7 * (1 << 36) + 128) == E.ERR_WORKSPACE  # not 256-aligned
     assert call(lib, S(), ws=0) == E.ERR_WORKSPACE
+    # the kernels write the workspace while they read the inputs
+    assert call(lib, S(), ws=FAKE + 4 * (1 << 36)) == E.ERR_INVALID_ARGUMENT  # workspace on K
+    assert call(lib, S(), ws=FAKE + (1 << 36) - 256) == E.ERR_INVALID_ARGUMENT  # ends in seeds
+    # the debug entry's Q and Z copies may not land on the workspace or on Y
+    dbg = lambda q, z: lib.flarepp_route_fwd_debug(
+        ctypes.byref(S()), *(ctypes.c_void_p(FAKE + (i + 1) * (1 << 36)) for i in range(5)),
+        ctypes.c_float(0.25), ctypes.c_void_p(FAKE + 6 * (1 << 36)),
+        ctypes.c_void_p(FAKE + 7 * (1 << 36)), lib.flarepp_route_workspace_bytes(ctypes.byref(S())),
+        None, None if q is None else ctypes.c_void_p(q), None if z is None else ctypes.c_void_p(z))
+    assert dbg(FAKE + 7 * (1 << 36) + 256, None) == E.ERR_INVALID_ARGUMENT
+    assert dbg(None, FAKE + 6 * (1 << 36) + 64) == E.ERR_INVALID_ARGUMENT
+    # FLARE: the same rules through its own entry (Q, K, V, Y, workspace)
+    fl = lambda ws: lib.flarepp_flare_fwd(
+        ctypes.byref(S()), *(ctypes.c_void_p(FAKE + (i + 1) * (1 << 36)) for i in range(3)),
+        ctypes.c_float(0.25), ctypes.c_void_p(FAKE + 6 * (1 << 36)), ctypes.c_void_p(ws),
+        lib.flarepp_route_workspace_bytes(ctypes.byref(S())), None, None)
+    assert fl(FAKE + 3 * (1 << 36)) == E.ERR_INVALID_ARGUMENT  # workspace on V
+    assert fl(FAKE + 6 * (1 << 36)) == E.ERR_INVALID_ARGUMENT  # workspace on Y
     # profiled entry: events required
     assert lib.flarepp_route_fwd_profiled(ctypes.byref(S()), None, None, None, None, None,
                                           ctypes.c_float(0.25), None, None, 0, None, None,
@@ -225,6 +243,10 @@ def test_backward_entry_sizes_and_rejects_before_any_cuda_call(lib):
     p = list(base)
     p[13] = None
     assert bwd(S(), p) == E.ERR_WORKSPACE
+    for i in (5, 6, 7):  # the workspace on Y, dY or saved
+        p = list(base)
+        p[13] = base[i]
+        assert bwd(S(), p) == E.ERR_INVALID_ARGUMENT, i
     # the training forward checks its saved buffer
     v = lambda x: ctypes.c_void_p(x)
     fw = lambda saved, nbytes: lib.flarepp_route_fwd_train(
@@ -266,6 +288,10 @@ def test_mixer_entry_sizes_and_rejects(lib):
     p = list(ptr)
     p[5] = None
     assert call(S(), ptrs=p) == E.ERR_WORKSPACE
+    for i in range(4):  # the workspace on X, W_in, Wo or seeds
+        p = list(ptr)
+        p[5] = ptr[i]
+        assert call(S(), ptrs=p) == E.ERR_INVALID_ARGUMENT, i
 
 
 def test_mixer_training_entries_reject(lib):
@@ -303,3 +329,11 @@ def test_mixer_training_entries_reject(lib):
     p = list(base)
     p[10] = None
     assert bwd(S(), ptrs=p) == E.ERR_WORKSPACE
+    for i in (0, 4, 5, 6, 9):  # the workspace on X, saved, dO, dX or dseeds
+        p = list(base)
+        p[10] = base[i]
+        assert bwd(S(), ptrs=p) == E.ERR_INVALID_ARGUMENT, i
+    for i in (6, 9):  # dX or dseeds on saved
+        p = list(base)
+        p[i] = base[4] + 64
+        assert bwd(S(), ptrs=p) == E.ERR_INVALID_ARGUMENT, i
