@@ -169,6 +169,30 @@ def _shape_of(seeds, Kt, Vt, K, V) -> Shape:
     return make_shape(B, H, N, M, D, K.dtype)
 
 
+def _nbytes(t):
+    return 0 if t is None else t.numel() * t.element_size()
+
+
+def _check_out(t, like, name):
+    """A caller-supplied output: a contiguous tensor of ``like``'s shape and dtype (the kernels
+    write every element of it, so a smaller buffer would be written past its end)."""
+    if not isinstance(t, torch.Tensor) or tuple(t.shape) != tuple(like.shape) or \
+            t.dtype != like.dtype or not t.is_contiguous():
+        raise ValueError(f"{name} must be a contiguous {like.dtype} tensor of shape "
+                         f"{tuple(like.shape)}")
+    return t
+
+
+def _check_device(what, device, **tensors):
+    """Every tensor a device-side call touches sits on ``device``, a CUDA device: the library
+    takes raw pointers and cannot tell a host address, or another GPU's, from its own."""
+    if device.type != "cuda":
+        raise ValueError(f"{what} takes device tensors (the *_host entries take host tensors)")
+    for name, t in tensors.items():
+        if isinstance(t, torch.Tensor) and t.device != device:
+            raise ValueError(f"{what}: {name} is on {t.device}, expected {device}")
+
+
 class Workspace:
     """A reusable device workspace, grown on demand (one per stream at a time)."""
 
@@ -189,8 +213,10 @@ class Workspace:
 def _call(debug, seeds, Kt, Vt, K, V, scale, Y, workspace, stream, Q_out, Z_out, events=None):
     lib = load()
     shape = _shape_of(seeds, Kt, Vt, K, V)
-    if K.device.type != "cuda":
-        raise ValueError("route_fwd takes device tensors; use route_fwd_host for host tensors")
+    if Y is not None:
+        _check_out(Y, K, "Y")
+    _check_device("route_fwd", K.device, seeds=seeds, Kt=Kt, Vt=Vt, V=V, Y=Y, Q_out=Q_out,
+                  Z_out=Z_out, workspace=workspace)
     if scale is None:
         scale = 1.0 / math.sqrt(shape.D)
     if Y is None:
@@ -281,8 +307,9 @@ def route_fwd_noalloc(seeds, Kt, Vt, K, V, scale=None, Y=None, stream=None):
     Y is allocated here only when not given."""
     lib = load()
     shape = _shape_of(seeds, Kt, Vt, K, V)
-    if K.device.type != "cuda":
-        raise ValueError("route_fwd_noalloc takes device tensors")
+    if Y is not None:
+        _check_out(Y, K, "Y")
+    _check_device("route_fwd_noalloc", K.device, seeds=seeds, Kt=Kt, Vt=Vt, V=V, Y=Y)
     if scale is None:
         scale = 1.0 / math.sqrt(shape.D)
     if Y is None:
@@ -313,15 +340,16 @@ def flare_fwd(Q, K, V, scale=None, Y=None, workspace=None, stream=None, Z_out=No
     [B, H, N, D]. Returns Y; ``Z_out`` (float32 [B, H, M, D], device) receives Z if given."""
     lib = load()
     shape = _shape_of(Q, K, V, K, V)
-    if K.device.type != "cuda":
-        raise ValueError("flare_fwd takes device tensors")
+    if Y is not None:
+        _check_out(Y, K, "Y")
+    if Z_out is not None and (Z_out.dtype != torch.float32 or not Z_out.is_contiguous() or
+                              tuple(Z_out.shape) != (shape.B, shape.H, shape.M, shape.D)):
+        raise ValueError("Z_out must be a contiguous float32 [B, H, M, D] tensor")
+    _check_device("flare_fwd", K.device, Q=Q, V=V, Y=Y, Z_out=Z_out)
     if scale is None:
         scale = 1.0 / math.sqrt(shape.D)
     if Y is None:
         Y = torch.empty_like(K)
-    if Z_out is not None and (Z_out.dtype != torch.float32 or not Z_out.is_contiguous() or
-                              tuple(Z_out.shape) != (shape.B, shape.H, shape.M, shape.D)):
-        raise ValueError("Z_out must be a contiguous float32 [B, H, M, D] tensor")
     nbytes = int(lib.flarepp_route_workspace_bytes(ctypes.byref(shape)))
     ws = (workspace if isinstance(workspace, Workspace) else Workspace()).get(nbytes, K.device)
     st = stream if stream is not None else torch.cuda.current_stream(K.device)
@@ -360,22 +388,12 @@ def mixer_fwd(X, W_in, Wo, seeds, scale=None, O=None, workspace=None, stream=Non
     K, V, K~, V~; P = 2: shared projection), Wo [C, C] (both out x in), seeds [H, M, D].
     Returns O [B, N, C]."""
     lib = load()
-    for t in (X, W_in, Wo, seeds):
-        if not isinstance(t, torch.Tensor) or not t.is_contiguous():
-            raise ValueError("inputs must be contiguous torch tensors")
-        if t.dtype != torch.bfloat16:
-            raise TypeError("the mixer takes bfloat16 tensors")
-    if X.device.type != "cuda":
-        raise ValueError("mixer_fwd takes device tensors")
-    B, N, C = X.shape
-    H, M, D = seeds.shape
-    if H * D != C or tuple(Wo.shape) != (C, C) or W_in.shape[1] != C or \
-            W_in.shape[0] not in (2 * C, 4 * C):
-        raise ValueError("expected X [B,N,C], W_in [P*C,C], Wo [C,C], seeds [H,M,D], C = H*D")
-    P = W_in.shape[0] // C
-    shape = make_shape(B, H, N, M, D, torch.bfloat16)
+    shape, P = _mixer_shape(X, W_in, Wo, seeds)
+    if O is not None:
+        _check_out(O, X, "O")
+    _check_device("mixer_fwd", X.device, W_in=W_in, Wo=Wo, seeds=seeds, O=O)
     if scale is None:
-        scale = 1.0 / math.sqrt(D)
+        scale = 1.0 / math.sqrt(shape.D)
     if O is None:
         O = torch.empty_like(X)
     nbytes = int(lib.flarepp_mixer_workspace_bytes(ctypes.byref(shape), P))
@@ -399,8 +417,8 @@ def _mixer_shape(X, W_in, Wo, seeds):
             raise ValueError("inputs must be contiguous torch tensors")
         if t.dtype != torch.bfloat16:
             raise TypeError("the mixer takes bfloat16 tensors")
-    if X.device.type != "cuda":
-        raise ValueError("the mixer takes device tensors")
+    if X.dim() != 3 or W_in.dim() != 2 or Wo.dim() != 2 or seeds.dim() != 3:
+        raise ValueError("expected X [B,N,C], W_in [P*C,C], Wo [C,C], seeds [H,M,D], C = H*D")
     B, N, C = X.shape
     H, M, D = seeds.shape
     if H * D != C or tuple(Wo.shape) != (C, C) or W_in.shape[1] != C or \
@@ -414,12 +432,15 @@ def mixer_fwd_train(X, W_in, Wo, seeds, scale=None, O=None, saved=None, workspac
     """The mixer layer's forward that keeps its backward's state. Returns (O, saved)."""
     lib = load()
     shape, P = _mixer_shape(X, W_in, Wo, seeds)
+    if O is not None:
+        _check_out(O, X, "O")
+    _check_device("mixer_fwd_train", X.device, W_in=W_in, Wo=Wo, seeds=seeds, O=O, saved=saved)
     if scale is None:
         scale = 1.0 / math.sqrt(shape.D)
     if O is None:
         O = torch.empty_like(X)
     sbytes = int(lib.flarepp_mixer_saved_bytes(ctypes.byref(shape), P))
-    if saved is None or saved.numel() < sbytes:
+    if saved is None or _nbytes(saved) < sbytes:
         saved = torch.empty(max(sbytes, 1), dtype=torch.uint8, device=X.device)
     nbytes = int(lib.flarepp_mixer_workspace_bytes(ctypes.byref(shape), P))
     ws = (workspace if isinstance(workspace, Workspace) else Workspace()).get(nbytes, X.device)
@@ -441,6 +462,13 @@ def mixer_bwd(X, W_in, Wo, seeds, saved, dO, scale=None, grads=None, workspace=N
     shape, P = _mixer_shape(X, W_in, Wo, seeds)
     if tuple(dO.shape) != tuple(X.shape) or dO.dtype != X.dtype or not dO.is_contiguous():
         raise ValueError("dO must be a contiguous tensor of X's shape and dtype")
+    if grads is not None:
+        if len(grads) != 4:
+            raise ValueError("grads must hold four tensors: dX, dW_in, dWo, dseeds")
+        grads = tuple(_check_out(g, like, name) for g, like, name in
+                      zip(grads, (X, W_in, Wo, seeds), ("dX", "dW_in", "dWo", "dseeds")))
+    _check_device("mixer_bwd", X.device, W_in=W_in, Wo=Wo, seeds=seeds, saved=saved, dO=dO,
+                  **({} if grads is None else dict(zip(("dX", "dW_in", "dWo", "dseeds"), grads))))
     if scale is None:
         scale = 1.0 / math.sqrt(shape.D)
     if grads is None:
@@ -451,7 +479,7 @@ def mixer_bwd(X, W_in, Wo, seeds, saved, dO, scale=None, grads=None, workspace=N
     st = stream if stream is not None else torch.cuda.current_stream(X.device)
     rc = lib.flarepp_mixer_bwd(ctypes.byref(shape), P, _ptr(X), _ptr(W_in), _ptr(Wo),
                                _ptr(seeds), float(scale), _ptr(saved),
-                               saved.numel() if saved is not None else 0, _ptr(dO),
+                               _nbytes(saved), _ptr(dO),
                                *(_ptr(g) for g in grads),
                                None if ws is None else ctypes.c_void_p(ws.data_ptr()), nbytes,
                                ctypes.c_void_p(st.cuda_stream))
@@ -466,14 +494,15 @@ def route_fwd_train(seeds, Kt, Vt, K, V, scale=None, Y=None, saved=None, workspa
     Returns (Y, saved): ``saved`` is an opaque uint8 device tensor for :func:`route_bwd`."""
     lib = load()
     shape = _shape_of(seeds, Kt, Vt, K, V)
-    if K.device.type != "cuda":
-        raise ValueError("route_fwd_train takes device tensors")
+    if Y is not None:
+        _check_out(Y, K, "Y")
+    _check_device("route_fwd_train", K.device, seeds=seeds, Kt=Kt, Vt=Vt, V=V, Y=Y, saved=saved)
     if scale is None:
         scale = 1.0 / math.sqrt(shape.D)
     if Y is None:
         Y = torch.empty_like(K)
     sbytes = int(lib.flarepp_route_saved_bytes(ctypes.byref(shape)))
-    if saved is None or saved.numel() < sbytes:
+    if saved is None or _nbytes(saved) < sbytes:
         saved = torch.empty(max(sbytes, 1), dtype=torch.uint8, device=K.device)
     nbytes = int(lib.flarepp_route_workspace_bytes(ctypes.byref(shape)))
     ws = (workspace if isinstance(workspace, Workspace) else Workspace()).get(nbytes, K.device)
@@ -497,8 +526,14 @@ def route_bwd(seeds, Kt, Vt, K, V, Y, dY, saved, scale=None, grads=None, workspa
     for t in (Y, dY):
         if tuple(t.shape) != tuple(K.shape) or t.dtype != K.dtype or not t.is_contiguous():
             raise ValueError("Y and dY must be contiguous tensors of K's shape and dtype")
-    if K.device.type != "cuda":
-        raise ValueError("route_bwd takes device tensors")
+    names = ("dseeds", "dKt", "dVt", "dK", "dV")
+    if grads is not None:
+        if len(grads) != 5:
+            raise ValueError("grads must hold five tensors: dseeds, dKt, dVt, dK, dV")
+        grads = tuple(_check_out(g, like, name) for g, like, name in
+                      zip(grads, (seeds, Kt, Vt, K, V), names))
+    _check_device("route_bwd", K.device, seeds=seeds, Kt=Kt, Vt=Vt, V=V, Y=Y, dY=dY,
+                  saved=saved, **({} if grads is None else dict(zip(names, grads))))
     if scale is None:
         scale = 1.0 / math.sqrt(shape.D)
     if grads is None:
@@ -510,7 +545,7 @@ def route_bwd(seeds, Kt, Vt, K, V, Y, dY, saved, scale=None, grads=None, workspa
     st = stream if stream is not None else torch.cuda.current_stream(K.device)
     rc = lib.flarepp_route_bwd(ctypes.byref(shape), _ptr(seeds), _ptr(Kt), _ptr(Vt), _ptr(K),
                                _ptr(V), float(scale), _ptr(Y), _ptr(dY), _ptr(saved),
-                               saved.numel() if saved is not None else 0,
+                               _nbytes(saved),
                                *(_ptr(g) for g in grads),
                                None if ws is None else ctypes.c_void_p(ws.data_ptr()), nbytes,
                                ctypes.c_void_p(st.cuda_stream))

@@ -150,6 +150,36 @@ def test_python_binding_rejects_bad_tensors(lib):
         flarepp.route_fwd(s[:1], x, x, x, x)
     with pytest.raises(ValueError):
         flarepp.route_fwd(s, x.transpose(2, 3), x, x, x)
+    # caller-supplied outputs are checked before the device is looked at: a short Y would
+    # be written past its end
+    short = torch.zeros(1, 2, 4, 32, dtype=torch.bfloat16)
+    for f in (flarepp.route_fwd, flarepp.route_fwd_train, flarepp.route_fwd_noalloc):
+        with pytest.raises(ValueError, match="Y must"):
+            f(s, x, x, x, x, Y=short)
+    with pytest.raises(ValueError, match="Y must"):
+        flarepp.route_fwd(s, x, x, x, x, Y=x.float())
+    with pytest.raises(ValueError, match="Y must"):
+        flarepp.flare_fwd(s, x, x, Y=x.transpose(2, 3))
+    with pytest.raises(ValueError, match="grads must"):
+        flarepp.route_bwd(s, x, x, x, x, x, x, None, grads=(s, x, x, x))
+    with pytest.raises(ValueError, match="dV must"):
+        flarepp.route_bwd(s, x, x, x, x, x, x, None, grads=(s, x, x, x, short))
+    X = torch.zeros(1, 8, 64, dtype=torch.bfloat16)
+    W = torch.zeros(4 * 64, 64, dtype=torch.bfloat16)
+    Wo = torch.zeros(64, 64, dtype=torch.bfloat16)
+    sd = torch.zeros(2, 4, 32, dtype=torch.bfloat16)
+    with pytest.raises(ValueError, match="O must"):
+        flarepp.mixer_fwd(X, W, Wo, sd, O=X[:, :4])
+    with pytest.raises(ValueError, match="O must"):
+        flarepp.mixer_fwd_train(X, W, Wo, sd, O=X.float())
+    with pytest.raises(ValueError, match="dW_in must"):
+        flarepp.mixer_bwd(X, W, Wo, sd, None, X, grads=(X, W[:64], Wo, sd))
+    with pytest.raises(ValueError, match="expected X"):
+        flarepp.mixer_fwd(X[0], W, Wo, sd)
+    # well-formed host tensors still reach the device check
+    for f, a in ((flarepp.mixer_fwd, (X, W, Wo, sd)), (flarepp.route_fwd, (s, x, x, x, x))):
+        with pytest.raises(ValueError, match="takes device tensors"):
+            f(*a)
 
 
 def test_missing_library_fails_loudly(tmp_path):

@@ -319,3 +319,21 @@ def test_profiled_entry_records_stages():
     Y2 = flarepp.route_fwd(x["seeds"], x["Kt"], x["Vt"], x["K"], x["V"])
     torch.cuda.synchronize()
     assert torch.equal(Y, Y2)
+
+
+def test_binding_rejects_tensors_on_another_device():
+    """A host tensor among device tensors is refused before anything is launched: the
+    library takes raw pointers and would read host memory as device memory."""
+    w = inputs.get("tiny").with_(dtype="bf16")
+    x = inputs.make_inputs(w, seed=3, device="cuda")
+    for name in ("seeds", "Kt", "V"):
+        y = dict(x)
+        y[name] = y[name].cpu()
+        with pytest.raises(ValueError, match=name):
+            flarepp.route_fwd(y["seeds"], y["Kt"], y["Vt"], y["K"], y["V"])
+    with pytest.raises(ValueError, match="Y"):
+        flarepp.route_fwd(x["seeds"], x["Kt"], x["Vt"], x["K"], x["V"], Y=torch.empty_like(
+            x["K"], device="cpu"))
+    with pytest.raises(ValueError, match="saved"):
+        flarepp.route_bwd(x["seeds"], x["Kt"], x["Vt"], x["K"], x["V"], x["K"], x["V"],
+                          torch.empty(16, dtype=torch.uint8))
