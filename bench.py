@@ -91,8 +91,77 @@ def stage_work(w, stage):
     return flops, byts
 
 
+class NvmlSampler:
+    """SM clock, power and clock-event reasons read through NVML's C API (read-only queries)
+    by a thread that polls every 2 ms between start() and stop(), so that even a timed
+    region of a few tens of milliseconds gets many samples."""
+
+    # clock-event reason bits of nvml.h
+    REASONS = {0x4: "sw_power_cap", 0x8: "hw_slowdown", 0x20: "sw_thermal_slowdown",
+               0x40: "hw_thermal_slowdown", 0x80: "hw_power_brake_slowdown"}
+
+    def __init__(self, cuda_index):
+        import ctypes
+        import threading
+        self.ct = ctypes
+        self.nvml = ctypes.CDLL("libnvidia-ml.so.1")
+        if self.nvml.nvmlInit_v2() != 0:
+            raise OSError("nvmlInit failed")
+        self.dev = ctypes.c_void_p()
+        vis = os.environ.get("CUDA_VISIBLE_DEVICES", "").strip()
+        ent = vis.split(",")[cuda_index].strip() if vis else str(cuda_index)
+        if ent.isdigit():
+            rc = self.nvml.nvmlDeviceGetHandleByIndex_v2(ctypes.c_uint(int(ent)),
+                                                         ctypes.byref(self.dev))
+        else:
+            rc = self.nvml.nvmlDeviceGetHandleByUUID(ent.encode(), ctypes.byref(self.dev))
+        if rc != 0:
+            raise OSError(f"no NVML handle for CUDA device {cuda_index}")
+        self.get_reasons = getattr(self.nvml, "nvmlDeviceGetCurrentClocksEventReasons", None) \
+            or self.nvml.nvmlDeviceGetCurrentClocksThrottleReasons
+        self.smax = self._clock(self.nvml.nvmlDeviceGetMaxClockInfo)
+        self.samples = []
+        self.stop_flag = threading.Event()
+        self.thread = threading.Thread(target=self._poll, daemon=True)
+
+    def _clock(self, fn):
+        v = self.ct.c_uint()
+        return float(v.value) if fn(self.dev, 1, self.ct.byref(v)) == 0 else None  # 1: SM
+
+    def _poll(self):
+        ct = self.ct
+        mw, reasons = ct.c_uint(), ct.c_ulonglong()
+        while not self.stop_flag.is_set():
+            sm = self._clock(self.nvml.nvmlDeviceGetClockInfo)
+            pw = mw.value / 1000.0 if self.nvml.nvmlDeviceGetPowerUsage(
+                self.dev, ct.byref(mw)) == 0 else None
+            rs = reasons.value if self.get_reasons(self.dev, ct.byref(reasons)) == 0 else 0
+            if sm is not None:
+                self.samples.append((sm, pw, rs))
+            time.sleep(0.002)
+
+    def start(self):
+        self.thread.start()
+
+    def stop(self):
+        self.stop_flag.set()
+        self.thread.join(timeout=5)
+        self.nvml.nvmlShutdown()
+        if not self.samples:
+            return {"sm_mhz": None, "sm_max_mhz": self.smax, "reasons": ["no samples"]}
+        reasons = sorted({name for _, _, r in self.samples
+                          for bit, name in self.REASONS.items() if r & bit})
+        power = [p for _, p, _ in self.samples if p is not None]
+        return {"sm_mhz": statistics.median(s for s, _, _ in self.samples),
+                "sm_max_mhz": self.smax, "power_w_max": max(power) if power else None,
+                "power_w_median": statistics.median(power) if power else None,
+                "samples": len(self.samples), "source": "nvml, 2 ms polling",
+                "reasons": reasons}
+
+
 class ClockSampler:
-    """nvidia-smi sampling of SM clocks and throttle reasons during the timed region."""
+    """SM clocks and throttle reasons during the timed region: NVML polling where the driver's
+    NVML library loads, else nvidia-smi sampling every 200 ms."""
 
     FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
               "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
@@ -101,8 +170,15 @@ class ClockSampler:
     def __init__(self):
         self.proc = None
         self.path = None
+        self.nvml = None
 
-    def start(self):
+    def start(self, cuda_index=0):
+        try:
+            self.nvml = NvmlSampler(cuda_index)
+            self.nvml.start()
+            return
+        except (OSError, AttributeError, IndexError):
+            self.nvml = None
         try:
             fd, self.path = tempfile.mkstemp(suffix=".csv")
             os.close(fd)
@@ -110,10 +186,13 @@ class ClockSampler:
             self.proc = subprocess.Popen(
                 ["nvidia-smi", f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits",
                  "-lms", "200"], stdout=self.out, stderr=subprocess.DEVNULL)
+            time.sleep(0.3)  # let nvidia-smi start before the timed region
         except (OSError, FileNotFoundError):
             self.proc = None
 
     def stop(self, gpu_index):
+        if self.nvml is not None:
+            return self.nvml.stop()
         if self.proc is None:
             return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
         self.proc.terminate()
@@ -146,7 +225,7 @@ class ClockSampler:
         loaded = [s for s in sm if s > 0.5 * max(sm)] or sm
         return {"sm_mhz": statistics.median(loaded), "sm_max_mhz": max(smax),
                 "power_w_max": max(power) if power else None, "samples": len(sm),
-                "reasons": sorted(reasons)}
+                "source": "nvidia-smi, 200 ms sampling", "reasons": sorted(reasons)}
 
 
 def dist_setup(n_gpus):
@@ -323,8 +402,7 @@ def run_flare(args, w, flarepp, world, rank, dev, peaks, x, Y, ws, stream):
     torch.cuda.synchronize(dev)
     clocks = ClockSampler()
     if rank == 0:
-        clocks.start()
-        time.sleep(0.3)
+        clocks.start(dev.index)
     t0 = torch.cuda.Event(enable_timing=True)
     t1 = torch.cuda.Event(enable_timing=True)
     barrier(world)
@@ -440,8 +518,7 @@ def run_train(args, w, flarepp, world, rank, dev, peaks, x, Y, ws, stream):
     evs = [[torch.cuda.Event(enable_timing=True) for _ in range(3)] for _ in range(args.steps)]
     clocks = ClockSampler()
     if rank == 0:
-        clocks.start()
-        time.sleep(0.3)
+        clocks.start(dev.index)
     t0 = torch.cuda.Event(enable_timing=True)
     t1 = torch.cuda.Event(enable_timing=True)
     barrier(world)
@@ -563,8 +640,7 @@ def run_mixer_train(args, w, flarepp, world, rank, dev, peaks, stream):
     evs = [[torch.cuda.Event(enable_timing=True) for _ in range(3)] for _ in range(args.steps)]
     clocks = ClockSampler()
     if rank == 0:
-        clocks.start()
-        time.sleep(0.3)
+        clocks.start(dev.index)
     t0 = torch.cuda.Event(enable_timing=True)
     t1 = torch.cuda.Event(enable_timing=True)
     barrier(world)
@@ -628,8 +704,7 @@ def run_mixer(args, w, flarepp, world, rank, dev, peaks, stream):
     evs = [flarepp.MixerEvents(stream) for _ in range(args.steps)]
     clocks = ClockSampler()
     if rank == 0:
-        clocks.start()
-        time.sleep(0.3)
+        clocks.start(dev.index)
     t0 = torch.cuda.Event(enable_timing=True)
     t1 = torch.cuda.Event(enable_timing=True)
     barrier(world)
@@ -732,8 +807,7 @@ def run_ours(args, w):
 
     clocks = ClockSampler()
     if rank == 0:
-        clocks.start()
-        time.sleep(0.3)
+        clocks.start(dev.index)
     t_start = torch.cuda.Event(enable_timing=True)
     t_end = torch.cuda.Event(enable_timing=True)
     barrier(world)
@@ -844,7 +918,7 @@ def run_ours(args, w):
 def main():
     ap = argparse.ArgumentParser(description=__doc__)
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=20)
+    ap.add_argument("--steps", type=int, default=200)
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", choices=("ours", "reference"), default="ours")
     ap.add_argument("--workload", default="mesh3d", choices=sorted(inputs.WORKLOADS))
