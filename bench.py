@@ -297,36 +297,49 @@ def cpu_oracle_sample(w, target_s, seed=0, variant="flarepp"):
 
 # ------------------------------------------------------------------ reference arm
 
+def reference_step(args, w, n):
+    """One step of the reference arm on an n-token sample of the workload: returns the call,
+    the heads it routes and a description of the sample."""
+    import oracle
+    if args.variant == "mixer_train":
+        # the layer's forward and backward on one batch element
+        m = inputs.to_f64_numpy(inputs.make_mixer_inputs(w.with_(B=1, N=n), args.seed, "cpu"))
+        dO = np.random.default_rng(args.seed).standard_normal(m["X"].shape)
+        return (lambda: oracle.mixer_bwd(m["X"], m["W_in"], m["Wo"], m["seeds"], w.scale, dO),
+                w.H, f"one batch element, N={n} tokens, H={w.H} heads of the {w.name} shape "
+                     f"(M={w.M}, D={w.D}), float64 oracle (forward and backward), per step")
+    if args.variant.startswith("mixer"):
+        # the whole layer on one batch element: all H heads of n tokens
+        m = inputs.to_f64_numpy(inputs.make_mixer_inputs(
+            w.with_(B=1, N=n), args.seed, "cpu", 2 if args.variant == "mixer_shared" else 4))
+        return (lambda: oracle.mixer(m["X"], m["W_in"], m["Wo"], m["seeds"], w.scale),
+                w.H, f"one batch element, N={n} tokens, H={w.H} heads of the {w.name} shape "
+                     f"(M={w.M}, D={w.D}), float64 oracle on the host cores, per step")
+    f = inputs.to_f64_numpy(inputs.make_inputs(w.with_(B=1, H=1, N=n), args.seed))
+    return (lambda: oracle_call(f, w, args.variant), 1,
+            f"one head, N={n} tokens of the {w.name} shape (M={w.M}, D={w.D}), float64 "
+            f"oracle on the host cores, per step")
+
+
 def run_reference(args, w):
     world = int(os.environ.get("WORLD_SIZE", "1"))
     rank = int(os.environ.get("RANK", "0"))
     if rank != 0:
         return 0
     import oracle
-    n = int(min(w.N, args.ref_tokens))
-    if args.variant == "mixer_train":
-        # the layer's forward and backward on one batch element
-        m = inputs.to_f64_numpy(inputs.make_mixer_inputs(w.with_(B=1, N=n), args.seed, "cpu"))
-        dO = np.random.default_rng(args.seed).standard_normal(m["X"].shape)
-        step = lambda: oracle.mixer_bwd(m["X"], m["W_in"], m["Wo"], m["seeds"], w.scale, dO)
-        heads = w.H
-        sample = (f"one batch element, N={n} tokens, H={w.H} heads of the {w.name} shape "
-                  f"(M={w.M}, D={w.D}), float64 oracle (forward and backward), per step")
-    elif args.variant.startswith("mixer"):
-        # the whole layer on one batch element: all H heads of n tokens
-        m = inputs.to_f64_numpy(inputs.make_mixer_inputs(
-            w.with_(B=1, N=n), args.seed, "cpu", 2 if args.variant == "mixer_shared" else 4))
-        step = lambda: oracle.mixer(m["X"], m["W_in"], m["Wo"], m["seeds"], w.scale)
-        heads = w.H
-        sample = (f"one batch element, N={n} tokens, H={w.H} heads of the {w.name} shape "
-                  f"(M={w.M}, D={w.D}), float64 oracle on the host cores, per step")
-    else:
-        x = inputs.make_inputs(w.with_(B=1, H=1, N=n), args.seed)
-        f = inputs.to_f64_numpy(x)
-        step = lambda: oracle_call(f, w, args.variant)
-        heads = 1
-        sample = (f"one head, N={n} tokens of the {w.name} shape (M={w.M}, D={w.D}), float64 "
-                  f"oracle on the host cores, per step")
+    # the sample: at most --ref-tokens tokens, fewer when the warm-up and timed steps would
+    # take more than about --ref-seconds (a probe on 1024 tokens gives the time per token),
+    # but no fewer than 1024 tokens, so that the tokens still outnumber the routes
+    cap = int(min(w.N, args.ref_tokens))
+    n0 = min(cap, 1024)
+    probe_step = reference_step(args, w, n0)[0]
+    t0 = time.perf_counter()
+    probe_step()
+    per_token = (time.perf_counter() - t0) / n0
+    del probe_step
+    calls = max(1, args.steps + args.warmup)
+    n = int(min(cap, max(n0, args.ref_seconds / (calls * per_token))))
+    step, heads, sample = reference_step(args, w, n)
     for _ in range(args.warmup):
         step()
     t0 = time.perf_counter()
@@ -935,7 +948,10 @@ def main():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-seconds", type=float, default=12.0)
     ap.add_argument("--ref-tokens", type=int, default=16384,
-                    help="token sample per reference step (one head)")
+                    help="largest token sample per reference step")
+    ap.add_argument("--ref-seconds", type=float, default=60.0,
+                    help="about how long the reference arm's warm-up and timed steps take; "
+                         "the token sample shrinks to fit")
     args = ap.parse_args()
     w = inputs.get(args.workload)
     if args.warmup < 3 and args.impl == "ours":
