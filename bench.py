@@ -100,11 +100,11 @@ class NvmlSampler:
     REASONS = {0x4: "sw_power_cap", 0x8: "hw_slowdown", 0x20: "sw_thermal_slowdown",
                0x40: "hw_thermal_slowdown", 0x80: "hw_power_brake_slowdown"}
 
-    def __init__(self, cuda_index):
+    def __init__(self, cuda_index, lib=None):
         import ctypes
         import threading
         self.ct = ctypes
-        self.nvml = ctypes.CDLL("libnvidia-ml.so.1")
+        self.nvml = lib if lib is not None else ctypes.CDLL("libnvidia-ml.so.1")
         if self.nvml.nvmlInit_v2() != 0:
             raise OSError("nvmlInit failed")
         self.dev = ctypes.c_void_p()
