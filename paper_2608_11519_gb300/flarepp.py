@@ -206,7 +206,8 @@ class Workspace:
         if self.buf is None or self.buf.numel() < nbytes or self.buf.device != device:
             self.buf = torch.empty(nbytes + 256, dtype=torch.uint8, device=device)
         # the library wants 256-byte alignment; torch allocations are at least that aligned
-        assert self.buf.data_ptr() % 256 == 0
+        if self.buf.data_ptr() % 256 != 0:
+            raise RuntimeError("workspace allocation is not 256-byte aligned")
         return self.buf
 
 
