@@ -944,7 +944,7 @@ def main():
                          "chain's training forward and backward; mixer(_shared): the whole "
                          "FLARE++ mixer layer with four (two) projections")
     ap.add_argument("--no-e2e", action="store_true")
-    ap.add_argument("--e2e-steps", type=int, default=5)
+    ap.add_argument("--e2e-steps", type=int, default=10)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-seconds", type=float, default=12.0)
     ap.add_argument("--ref-tokens", type=int, default=16384,
