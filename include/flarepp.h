@@ -57,7 +57,7 @@ typedef enum {
 typedef enum {
     FLAREPP_OK = 0,
     FLAREPP_ERR_INVALID_ARGUMENT = 1, /* null/misaligned pointer, negative size, NaN/inf scale,
-                                         overlapping Y, bad dtype */
+                                         overlapping buffers, bad dtype */
     FLAREPP_ERR_UNSUPPORTED = 2,      /* a valid shape outside the supported set (D, M limits) */
     FLAREPP_ERR_WORKSPACE = 3,        /* workspace missing, misaligned or too small */
     FLAREPP_ERR_CUDA = 4,             /* a CUDA call or kernel launch failed */
