@@ -1,4 +1,5 @@
-"""Write tests/golden/route_small.json: a small routing-chain case and the oracle's answer.
+"""Write tests/golden/route_small.json (a small routing-chain case and the oracle's answer)
+and tests/golden/route_bwd_small.json (the oracle's gradients of that case for a stored dY).
 
 The inputs are drawn here with numpy (seed 2608) and stored in full; the expected Q, Z
 and Y come only from the float64 oracle (Sec. 3.2, eqs. flarepp_dynamic_query and
@@ -36,7 +37,25 @@ def main():
                    dict(seeds=seeds, Kt=Kt, Vt=Vt, K=K, V=V).items()},
         "expected": {"Q": Q.tolist(), "Z": Z.tolist(), "Y": Y.tolist()},
     }
-    out = os.path.join(os.path.dirname(os.path.abspath(__file__)), "route_small.json")
+    here = os.path.dirname(os.path.abspath(__file__))
+    out = os.path.join(here, "route_small.json")
+    with open(out, "w") as f:
+        json.dump(doc, f, indent=None, separators=(",", ":"))
+        f.write("\n")
+    print(out)
+
+    # the backward of the same case for an output gradient dY (drawn after the inputs, so
+    # the forward case above does not change)
+    dY = r(B, H, N, D)
+    grads = oracle.route_bwd(seeds, Kt, Vt, K, V, s, dY)
+    doc = {
+        "what": "gradients of the routing chain of route_small.json (same inputs and scale) for "
+                "the output gradient dY (App. A.5); expected values from the float64 oracle",
+        "dY": dY.tolist(),
+        "expected": {k: g.tolist() for k, g in
+                     zip(("dseeds", "dKt", "dVt", "dK", "dV"), grads)},
+    }
+    out = os.path.join(here, "route_bwd_small.json")
     with open(out, "w") as f:
         json.dump(doc, f, indent=None, separators=(",", ":"))
         f.write("\n")

@@ -187,3 +187,23 @@ def test_bwd_pins_reject_planted_mistakes(plant, tmp_path):
         except AssertionError:
             failed.append(pin.__name__)
     assert failed, f"plant {plant} passed every backward pin"
+
+
+def test_golden_bwd_fixture_regression():
+    """The oracle's backward still reproduces the stored small case
+    (tests/golden/route_bwd_small.json, on the inputs of route_small.json), whose values the
+    pins above were green for when it was written."""
+    import json
+    import os
+    here = os.path.join(os.path.dirname(__file__), "golden")
+    with open(os.path.join(here, "route_small.json")) as f:
+        fwd = json.load(f)
+    with open(os.path.join(here, "route_bwd_small.json")) as f:
+        bwd = json.load(f)
+    x = {k: np.array(v) for k, v in fwd["inputs"].items()}
+    got = oracle_pkg.route_bwd(x["seeds"], x["Kt"], x["Vt"], x["K"], x["V"], fwd["scale"],
+                               np.array(bwd["dY"]))
+    for name, g in zip(("dseeds", "dKt", "dVt", "dK", "dV"), got):
+        want = np.array(bwd["expected"][name])
+        assert g.shape == want.shape
+        np.testing.assert_allclose(g, want, rtol=0, atol=1e-13, err_msg=name)
