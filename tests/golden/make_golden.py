@@ -24,7 +24,8 @@ def main():
     rng = np.random.default_rng(2608)
     B, H, N, M, D = 1, 2, 40, 6, 16
     s = 1.0 / math.sqrt(D)
-    # values rounded to multiples of 2^-8 so that they are exact in float32 and bf16
+    # values rounded to multiples of 2^-8 so that they are exact in float32 (not in bf16,
+    # whose 8 significant bits do not hold 2^-8 steps above 1): the GPU cases run in float32
     r = lambda *sh: np.round(rng.standard_normal(sh) * 256.0) / 256.0
     seeds, Kt, Vt, K, V = r(H, M, D), r(B, H, N, D) * 2.0, r(B, H, N, D), r(B, H, N, D) * 2.0, r(B, H, N, D)
     Q, Z, Y = oracle.route(seeds, Kt, Vt, K, V, s)

@@ -299,3 +299,20 @@ def test_bwd_wide_score_ranges(D, fac, flagged):
         bound = tol * max(1.0, float(np.abs(r).max()))
         err = float(np.abs(g - r).max())
         assert err <= bound and not math.isnan(err), f"{name}: {err} > {bound}"
+
+
+def test_golden_bwd_fixture_f32():
+    """The float32 backward on the stored case (tests/golden/route_small.json inputs,
+    route_bwd_small.json's dY and oracle gradients)."""
+    import json
+    import os
+    here = os.path.join(os.path.dirname(__file__), "golden")
+    with open(os.path.join(here, "route_small.json")) as fh:
+        fwd = json.load(fh)
+    with open(os.path.join(here, "route_bwd_small.json")) as fh:
+        bwd = json.load(fh)
+    x = {k: torch.tensor(v, dtype=torch.float32) for k, v in fwd["inputs"].items()}
+    dY = torch.tensor(bwd["dY"], dtype=torch.float32)
+    got, _ = _gpu_grads(x, dY, fwd["scale"])
+    want = [np.array(bwd["expected"][n]) for n in NAMES]
+    _check_grads(got, want, TOL["f32"], " (stored case)")
