@@ -60,18 +60,18 @@ def kernel_source_hash():
     return h.hexdigest()[:16]
 
 
-def recorded_traffic(workload, stage):
+def recorded_traffic(workload, stage, how=False):
     """DRAM bytes per launch from the committed ncu summary, if it was taken on the current
-    kernel sources (else None)."""
+    kernel sources (else None); with ``how``, also the record's note on how it was taken."""
     p = os.path.join(ROOT, "profiles", "traffic.json")
-    if not os.path.exists(p):
-        return None
-    with open(p) as f:
-        d = json.load(f)
-    e = d.get(workload, {}).get(stage)
-    if not e or e.get("source_hash") != kernel_source_hash():
-        return None
-    return e.get("dram_bytes_per_launch")
+    e = None
+    if os.path.exists(p):
+        with open(p) as f:
+            e = json.load(f).get(workload, {}).get(stage)
+        if e and e.get("source_hash") != kernel_source_hash():
+            e = None
+    value = e.get("dram_bytes_per_launch") if e else None
+    return (value, e.get("how") if e else None) if how else value
 
 
 def stage_work(w, stage):
@@ -859,7 +859,9 @@ def run_ours(args, w):
     roof["ms_per_launch"] = stage_ms[dominant]
     roof["algorithmic_flops_per_launch"] = flops
     roof["algorithmic_bytes_per_launch"] = byts
-    roof["traffic"] = recorded_traffic(w.name, dominant)
+    roof["traffic"], how = recorded_traffic(w.name, dominant, how=True)
+    if how:
+        roof["traffic_source"] = how
 
     # whole-chain roofline: max(12 BNMHD / tensor peak, 5 BHND elt / HBM); the shared
     # projection streams 3 token tensors (K, V, Y) instead of 5

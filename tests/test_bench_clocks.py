@@ -116,3 +116,17 @@ def test_nvidia_smi_csv_parsing(tmp_path):
     assert r["samples"] == 2 and r["sm_max_mhz"] == 2070.0
     assert r["sm_mhz"] == pytest.approx(2062.5)
     assert r["reasons"] == ["sw_power_cap"]  # GPU 1's hw_slowdown is not ours
+
+
+def test_recorded_traffic_only_for_the_captured_sources(monkeypatch):
+    """The roofline's DRAM traffic comes from the committed ncu record only while the kernel
+    sources hash to the value it was taken at; otherwise the bench line reports null."""
+    import json
+    with open(os.path.join(ROOT, "profiles", "traffic.json")) as f:
+        rec = json.load(f)["mesh3d"]["decode"]
+    monkeypatch.setattr(bench, "kernel_source_hash", lambda: rec["source_hash"])
+    value, how = bench.recorded_traffic("mesh3d", "decode", how=True)
+    assert value == rec["dram_bytes_per_launch"] and "ncu" in how
+    monkeypatch.setattr(bench, "kernel_source_hash", lambda: "0" * 16)
+    assert bench.recorded_traffic("mesh3d", "decode", how=True) == (None, None)
+    assert bench.recorded_traffic("no-such-workload", "decode") is None
