@@ -1,6 +1,7 @@
-"""bench.py's clock record on the host: the NVML sampler against a fake NVML library (read-only
-queries: clocks, power, clock-event reasons), and the nvidia-smi fallback's CSV parsing. No GPU
-and no driver library are touched."""
+"""bench.py's clock and traffic records on the host: the NVML sampler against a fake NVML
+library (read-only queries: clocks, power, clock-event reasons), the nvidia-smi fallback's CSV
+parsing, and the committed ncu traffic record's tie to the kernel sources. No GPU and no driver
+library are touched."""
 import os
 import sys
 import time
