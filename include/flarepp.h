@@ -197,6 +197,8 @@ FLAREPP_API flarepp_status flarepp_flare_fwd_host(const flarepp_shape* shape, co
  *   - First call per device: it looks up the array's device address (cudaGetSymbolAddress
  *     with that device current) and caches it. Make that first call before any stream
  *     capture.
+ *   - Device: the call uses the array of the current device, so `stream` must belong to the
+ *     current device; a stream of another device returns FLAREPP_ERR_INVALID_ARGUMENT.
  *   - Sharing: every call on a device shares the one array, and the array keeps the last
  *     call's contents. Each call clears the status word and writes all the scratch it
  *     reads. Calls whose work overlaps on the GPU (other streams, other host threads) race

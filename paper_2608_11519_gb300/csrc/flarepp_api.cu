@@ -6,9 +6,35 @@
 #include <stdint.h>
 #include <string.h>
 
+#include <mutex>
+#include <utility>
+#include <vector>
+
 #include "flarepp_internal.h"
 
 namespace flarepp {
+
+cudaError_t ensure_smem_limit(const void* func, int bytes) {
+    constexpr int kMaxDevices = 64;
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return e;
+    if (dev < 0 || dev >= kMaxDevices) return cudaErrorInvalidDevice;
+    static std::mutex mu;
+    static std::vector<std::pair<const void*, uint64_t>> done;  // kernel, devices set
+    std::lock_guard<std::mutex> lock(mu);
+    for (auto& d : done)
+        if (d.first == func) {
+            if (d.second >> dev & 1u) return cudaSuccess;
+            e = cudaFuncSetAttribute(func, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
+            if (e == cudaSuccess) d.second |= uint64_t(1) << dev;
+            return e;
+        }
+    e = cudaFuncSetAttribute(func, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
+    if (e == cudaSuccess) done.emplace_back(func, uint64_t(1) << dev);
+    return e;
+}
+
 namespace {
 
 constexpr int kStageEvents = 6;

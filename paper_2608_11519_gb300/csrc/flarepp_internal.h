@@ -40,6 +40,11 @@ struct Plan {
     size_t total;
 };
 
+// Raise the dynamic shared-memory limit of kernel `func` to `bytes` on the current device,
+// once per (kernel, device): the attribute is per device, so a process that launches on
+// several GPUs sets it on each (flarepp_api.cu).
+cudaError_t ensure_smem_limit(const void* func, int bytes);
+
 // Fill `p` for `s` (plan.cu); returns FLAREPP_OK or the validation error for the shape itself.
 flarepp_status make_plan(const flarepp_shape* s, Plan* p);
 

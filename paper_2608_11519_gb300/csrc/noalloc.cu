@@ -53,6 +53,15 @@ extern "C" flarepp_status flarepp_route_fwd_noalloc(const flarepp_shape* shape, 
     // An invalid shape needs no workspace; flarepp_route_fwd then reports why it is invalid.
     const size_t need = flarepp_route_workspace_bytes(shape);
     if (need > flarepp::kNoAllocScratchBytes) return FLAREPP_ERR_WORKSPACE;
+    // The scratch address is the current device's; a stream of another device would run
+    // the kernels there against this device's array.
+    if (need > 0) {
+        int cur = 0, sdev = 0;
+        if (cudaGetDevice(&cur) != cudaSuccess ||
+            cudaStreamGetDevice((cudaStream_t)stream, &sdev) != cudaSuccess)
+            return FLAREPP_ERR_CUDA;
+        if (sdev != cur) return FLAREPP_ERR_INVALID_ARGUMENT;
+    }
     void* scratch = nullptr;
     if (need > 0 && flarepp::scratch_address(&scratch) != cudaSuccess) return FLAREPP_ERR_CUDA;
     return flarepp_route_fwd(shape, seeds, Kt, Vt, K, V, scale, Y, scratch,

@@ -909,8 +909,7 @@ bool make_map(CUtensorMap* m, const void* base, int64_t D, int64_t rows, int64_t
 template <int D, int PASS>
 cudaError_t launch_pass(const void* const* srcs, const Plan& p, BwdParams prm, cudaStream_t st) {
     using Cf = BCfg<D, PASS>;
-    static cudaError_t attr = cudaFuncSetAttribute(
-        tc_bwd_kernel<D, PASS>, cudaFuncAttributeMaxDynamicSharedMemorySize, Cf::kSmem);
+    const cudaError_t attr = ensure_smem_limit((const void*)tc_bwd_kernel<D, PASS>, Cf::kSmem);
     if (attr != cudaSuccess) return attr;
     if (Cf::kRouteRows) {
         prm.n_groups = (prm.M + Cf::kGroup - 1) / Cf::kGroup;

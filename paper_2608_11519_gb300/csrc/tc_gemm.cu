@@ -386,8 +386,7 @@ template <int D, int MODE>
 cudaError_t launch(const CUtensorMap* a, const CUtensorMap& b, const CUtensorMap* o,
                    const GemmParams& prm, cudaStream_t st) {
     using Cf = GCfg<D>;
-    static cudaError_t attr = cudaFuncSetAttribute(
-        tc_gemm_kernel<D, MODE>, cudaFuncAttributeMaxDynamicSharedMemorySize, Cf::kSmem);
+    const cudaError_t attr = ensure_smem_limit((const void*)tc_gemm_kernel<D, MODE>, Cf::kSmem);
     if (attr != cudaSuccess) return attr;
     if (prm.n_tiles == 0) return cudaSuccess;
     int dev = 0, sms = kNumSMs;

@@ -899,8 +899,7 @@ template <int D, bool DEC>
 cudaError_t launch(const CUtensorMap& a, const CUtensorMap& b, const CUtensorMap& c,
                    const TcParams& prm, cudaStream_t st) {
     using Cf = Cfg<D, DEC>;
-    static cudaError_t attr = cudaFuncSetAttribute(
-        tc_chain_kernel<D, DEC>, cudaFuncAttributeMaxDynamicSharedMemorySize, Cf::kSmem);
+    const cudaError_t attr = ensure_smem_limit((const void*)tc_chain_kernel<D, DEC>, Cf::kSmem);
     if (attr != cudaSuccess) return attr;
     int dev = 0, sms = kNumSMs;
     cudaGetDevice(&dev);

@@ -384,8 +384,7 @@ template <int D>
 cudaError_t launch(const CUtensorMap* ma, const CUtensorMap* mb, const WgParams& prm,
                    cudaStream_t st) {
     using Wc = WCfg<D>;
-    static cudaError_t attr = cudaFuncSetAttribute(
-        tc_wgrad_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize, Wc::kSmem);
+    const cudaError_t attr = ensure_smem_limit((const void*)tc_wgrad_kernel<D>, Wc::kSmem);
     if (attr != cudaSuccess) return attr;
     if (prm.n_items == 0) return cudaSuccess;
     int dev = 0, sms = kNumSMs;

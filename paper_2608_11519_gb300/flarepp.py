@@ -10,6 +10,8 @@ call raises.
     Y = flarepp.route_fwd_host(seeds, Kt, Vt, K, V)         # host tensors in, host Y out
 """
 import ctypes
+import functools
+import inspect
 import math
 import os
 
@@ -193,6 +195,30 @@ def _check_device(what, device, **tensors):
             raise ValueError(f"{what}: {name} is on {t.device}, expected {device}")
 
 
+def _on_device(arg):
+    """Run the wrapped entry with the CUDA device of argument ``arg`` current. The library
+    works on the current device (the no-allocation entry looks its scratch array up there,
+    and launches go to the current device's context), so a call on tensors of another GPU
+    must make that GPU current first. ``arg`` names a device tensor, or the ``device``
+    argument of a host entry."""
+    def wrap(fn):
+        sig = inspect.signature(fn)
+
+        @functools.wraps(fn)
+        def call(*a, **kw):
+            v = sig.bind_partial(*a, **kw).arguments.get(arg)
+            if v is None and arg in sig.parameters:
+                v = sig.parameters[arg].default
+            dev = v.device if isinstance(v, torch.Tensor) else (
+                torch.device(v) if isinstance(v, (str, torch.device)) else None)
+            if dev is None or dev.type != "cuda" or dev.index is None:
+                return fn(*a, **kw)
+            with torch.cuda.device(dev):
+                return fn(*a, **kw)
+        return call
+    return wrap
+
+
 class Workspace:
     """A reusable device workspace, grown on demand (one per stream at a time)."""
 
@@ -259,17 +285,20 @@ def device_status(shape_or_tensors, workspace, stream=None) -> int:
     shape = (shape_or_tensors if isinstance(shape_or_tensors, Shape)
              else _shape_of(*shape_or_tensors))
     buf = workspace.buf if isinstance(workspace, Workspace) else workspace
-    if stream is None:
-        stream = torch.cuda.current_stream()
-    out = ctypes.c_int32(-1)
-    rc = load().flarepp_route_device_status(ctypes.byref(shape), _ptr(buf),
-                                            ctypes.c_void_p(stream.cuda_stream),
-                                            ctypes.byref(out))
+    dev = buf.device if isinstance(buf, torch.Tensor) and buf.is_cuda else None
+    with torch.cuda.device(dev):
+        if stream is None:
+            stream = torch.cuda.current_stream()
+        out = ctypes.c_int32(-1)
+        rc = load().flarepp_route_device_status(ctypes.byref(shape), _ptr(buf),
+                                                ctypes.c_void_p(stream.cuda_stream),
+                                                ctypes.byref(out))
     if rc != OK:
         raise FlareppError(rc, "flarepp_route_device_status")
     return int(out.value)
 
 
+@_on_device("K")
 def route_fwd(seeds, Kt, Vt, K, V, scale=None, Y=None, workspace=None, stream=None):
     """Y = routing chain (Sec. 3.2) on device tensors; returns Y [B,H,N,D] (enqueued on
     ``stream``, default torch's current stream)."""
@@ -293,6 +322,7 @@ class StageEvents:
                 for i, name in enumerate(STAGES)}
 
 
+@_on_device("K")
 def route_fwd_profiled(seeds, Kt, Vt, K, V, events: StageEvents, scale=None, Y=None,
                        workspace=None, stream=None):
     """``route_fwd`` that records ``events`` around each stage on the launching stream."""
@@ -300,6 +330,7 @@ def route_fwd_profiled(seeds, Kt, Vt, K, V, events: StageEvents, scale=None, Y=N
                  events.handles)
 
 
+@_on_device("K")
 def route_fwd_noalloc(seeds, Kt, Vt, K, V, scale=None, Y=None, stream=None):
     """``route_fwd`` through flarepp_route_fwd_noalloc: for callers that cannot allocate
     device memory at call time, the library uses its own fixed 64 MiB scratch array instead
@@ -325,6 +356,7 @@ def route_fwd_noalloc(seeds, Kt, Vt, K, V, scale=None, Y=None, stream=None):
     return Y
 
 
+@_on_device("K")
 def route_fwd_debug(seeds, Kt, Vt, K, V, scale=None, Y=None, workspace=None, stream=None):
     """Like ``route_fwd``, also returning the float32 intermediates Q and Z [B,H,M,D]."""
     B, H, N, D = K.shape
@@ -335,6 +367,7 @@ def route_fwd_debug(seeds, Kt, Vt, K, V, scale=None, Y=None, workspace=None, str
     return Y, Q, Z
 
 
+@_on_device("K")
 def flare_fwd(Q, K, V, scale=None, Y=None, workspace=None, stream=None, Z_out=None):
     """FLARE with learned queries (Sec. 3, eq. prelim_flare_sdpa) on device tensors:
     Z = SDPA(Q_h, K, V), Y = SDPA(K, Q_h, Z). Q [H, M, D] is shared by the batch; K, V
@@ -384,6 +417,7 @@ class MixerEvents:
                 for i, s in enumerate(MIXER_STAGES)}
 
 
+@_on_device("X")
 def mixer_fwd(X, W_in, Wo, seeds, scale=None, O=None, workspace=None, stream=None, events=None):
     """The FLARE++ mixer layer (Fig. 1) on device tensors: X [B, N, C], W_in [P*C, C] (P = 4:
     K, V, K~, V~; P = 2: shared projection), Wo [C, C] (both out x in), seeds [H, M, D].
@@ -428,6 +462,7 @@ def _mixer_shape(X, W_in, Wo, seeds):
     return make_shape(B, H, N, M, D, torch.bfloat16), W_in.shape[0] // C
 
 
+@_on_device("X")
 def mixer_fwd_train(X, W_in, Wo, seeds, scale=None, O=None, saved=None, workspace=None,
                     stream=None):
     """The mixer layer's forward that keeps its backward's state. Returns (O, saved)."""
@@ -455,6 +490,7 @@ def mixer_fwd_train(X, W_in, Wo, seeds, scale=None, O=None, saved=None, workspac
     return O, saved
 
 
+@_on_device("X")
 def mixer_bwd(X, W_in, Wo, seeds, saved, dO, scale=None, grads=None, workspace=None,
               stream=None):
     """The mixer layer's backward from :func:`mixer_fwd_train`'s ``saved``: returns
@@ -489,6 +525,7 @@ def mixer_bwd(X, W_in, Wo, seeds, saved, dO, scale=None, grads=None, workspace=N
     return grads
 
 
+@_on_device("K")
 def route_fwd_train(seeds, Kt, Vt, K, V, scale=None, Y=None, saved=None, workspace=None,
                     stream=None):
     """The chain's forward that also keeps the state its backward needs (App. A.5).
@@ -517,6 +554,7 @@ def route_fwd_train(seeds, Kt, Vt, K, V, scale=None, Y=None, saved=None, workspa
     return Y, saved
 
 
+@_on_device("K")
 def route_bwd(seeds, Kt, Vt, K, V, Y, dY, saved, scale=None, grads=None, workspace=None,
               stream=None):
     """Backward of the chain (App. A.5) from :func:`route_fwd_train`'s ``Y`` and ``saved``.
@@ -555,6 +593,7 @@ def route_bwd(seeds, Kt, Vt, K, V, Y, dY, saved, scale=None, grads=None, workspa
     return grads
 
 
+@_on_device("device")
 def route_fwd_host(seeds, Kt, Vt, K, V, scale=None, Y_host=None, device="cuda", workspace=None,
                    stream=None, dev_bufs=None):
     """End-to-end call on host tensors through ``flarepp_route_fwd_host``: the library copies
@@ -592,6 +631,7 @@ def route_fwd_host(seeds, Kt, Vt, K, V, scale=None, Y_host=None, device="cuda", 
     return Y_host
 
 
+@_on_device("device")
 def flare_fwd_host(Q, K, V, scale=None, Y_host=None, device="cuda", workspace=None, stream=None):
     """FLARE with learned queries Q [H, M, D] on host tensors through
     ``flarepp_flare_fwd_host``: copies in, FLARE, Y copied back into ``Y_host`` (allocated

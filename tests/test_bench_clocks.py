@@ -131,3 +131,17 @@ def test_recorded_traffic_only_for_the_captured_sources(monkeypatch):
     monkeypatch.setattr(bench, "kernel_source_hash", lambda: "0" * 16)
     assert bench.recorded_traffic("mesh3d", "decode", how=True) == (None, None)
     assert bench.recorded_traffic("no-such-workload", "decode") is None
+
+
+def test_tensor_peak_follows_timed_region():
+    """A kernel timed over a short region is compared with the burst GEMM peak; only a
+    seconds-long timed region, which runs into the power cap as the sustained GEMM loop
+    does, takes the sustained peak."""
+    peaks = {"bf16_tflops": 1913.9, "bf16_tflops_sustained": 1717.3, "source": "measured"}
+    v, kind = bench.tc_peak_for(peaks, 0.054)
+    assert v == 1913.9 and kind == "bf16_tflops (measured)"
+    v, kind = bench.tc_peak_for(peaks, bench.SUSTAINED_REGION_S - 1e-3)
+    assert v == 1913.9
+    v, kind = bench.tc_peak_for(peaks, bench.SUSTAINED_REGION_S)
+    assert v == 1717.3 and kind == "bf16_tflops_sustained (measured)"
+    assert bench.tc_peak_for(peaks, 10.0, bf16=False) == (None, None)

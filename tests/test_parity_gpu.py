@@ -114,11 +114,18 @@ def test_longseq_full_size():
 
 
 def test_mesh3d_full_size_sampled():
-    _slice_check(inputs.get("mesh3d"), [(0, 5)], sample_tokens=2048)
+    """The largest workload at full size: Q and Z of three heads in full, Y on 4096 sampled
+    tokens of each (plus the first and last)."""
+    _slice_check(inputs.get("mesh3d"), [(0, 0), (0, 5), (0, 7)], sample_tokens=4096)
 
 
-@pytest.mark.parametrize("M,D", [(16, 16), (64, 32), (128, 64), (256, 16)])
+SWEEP = [(m, d) for m in (16, 32, 64, 128, 256, 512, 1024, 2048) for d in (16, 32, 64)]
+
+
+@pytest.mark.parametrize("M,D", SWEEP)
 def test_sweep_full_size(M, D):
+    """Every point of the M x D sweep at its full size (N = 262,144): one (b, h) slice of Q,
+    Z and Y in full against the oracle, the hull bound on every output."""
     _slice_check(inputs.get(f"sweep_M{M}_D{D}"), [(0, 3)])
 
 
