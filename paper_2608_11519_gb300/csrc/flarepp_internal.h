@@ -174,6 +174,10 @@ cudaError_t add_bf16(void* dst, const void* src, int64_t n, cudaStream_t st);
 // Encode call 1 (A = seeds) or call 2 (A = Q operand) into the chunk partials.
 cudaError_t tc_encode(const Plan& p, int call, const void* k, const void* v, const void* seeds,
                       float scale, char* ws, cudaStream_t st);
+// Test hook of the bounded waits: until reset (kernel = 0), the launches of one tensor-core
+// chain kernel (1, 2: the encode of call 1 or 2; 3: the decode) wait at most wait_ns at each
+// barrier, and CTA 0's producer never loads ring item `ring_item` (so that a wait runs out).
+void set_tc_test_fault(int kernel, int64_t ring_item, uint64_t wait_ns);
 // Rows per tensor-core work unit (route group of the encode, token group of the decode).
 int64_t tc_group_rows(int64_t D);
 int64_t tc_encode_item_rows(int64_t D);  // tokens per item of the tensor-core encode

@@ -95,6 +95,9 @@ flarepp_status make_plan(const flarepp_shape* s, Plan* p) {
         }
         p->chunk_len = cdiv(cdiv(s->N, best_n), kTcItem) * kTcItem;
         p->nchunk = cdiv(s->N, p->chunk_len);
+        // the kernels count their work units in 32 bits
+        if (per_chunk * p->nchunk > INT32_MAX || bh * cdiv(s->N, p->tc_group) > INT32_MAX)
+            return FLAREPP_ERR_UNSUPPORTED;
     }
 
     const size_t rows =

@@ -45,9 +45,15 @@ namespace {
 
 using namespace tc;
 
-constexpr int kWarps = 20;
+constexpr int kWarps = 24;
 constexpr int kThreads = kWarps * 32;
-constexpr int kFirstSoftmaxWarp = 4;
+constexpr int kProducerWarp = 4;      // warpgroup 1: the TMA producer and three idle warps
+constexpr int kFirstSoftmaxWarp = 8;
+// Registers per thread after the split (launch: 80 x 768 threads): warpgroups 0 (MMA) and 1
+// (producer) lower to 40, the four softmax warpgroups raise to 96.
+constexpr uint32_t kRegsControl = 40;
+constexpr uint32_t kRegsSoftmax = 96;
+static_assert(kRegsControl * 256 + kRegsSoftmax * 512 <= 80 * 768, "register split");
 constexpr int NS = 4;           // TMEM streams
 constexpr int kTileRows = 128;  // TMEM lanes, MMA M
 constexpr uint64_t kWaitLimitNs = 2000000000ull;
@@ -460,128 +466,6 @@ __device__ __forceinline__ bool finish_stream(SoftmaxStream& S, const Unit& U,
     return true;
 }
 
-// PV of stream s: O_s (+)= P (score buffer pb) * C-tile of ring stage `st` (one elected
-// lane issues).
-template <int D, bool DEC>
-__device__ __forceinline__ void issue_pv(uint32_t tmem, uint8_t* ring, int s, int pb, int st,
-                                         int npv) {
-    using C = Cfg<D, DEC>;
-    const uint32_t cb = smem_u32(ring + st * C::kStage + C::kItemTile);
-#pragma unroll
-    for (int k = 0; k < C::kItem / 16; ++k) {
-        const uint64_t bd = smem_desc(cb + k * 16 * D * 2, C::kItemTile, C::kSBO, C::kSwz);
-        if (elect_one())
-            mma_ts(tmem + C::kColO + s * D, tmem + C::kColS + (s * C::B + pb) * C::kItem + 8 * k,
-                   bd, C::kIdescPV, (npv > 0 || k > 0) ? 1u : 0u);
-        __syncwarp();
-    }
-}
-
-// The TMA side of MMA warp 0: issues A tiles and ring items whenever their buffers are
-// free, without ever blocking (called from the warp's own wait loops). Warp-uniform. With
-// two TMEM copies of the A tiles the A tiles run one unit ahead of the ring items, so that
-// the softmax can copy the next unit's A tiles into TMEM while it works on the current one.
-template <int D, bool DEC>
-struct Producer {
-    const CUtensorMap* tmA;
-    const CUtensorMap* tmB;
-    const CUtensorMap* tmC;
-    uint8_t* abuf;
-    uint8_t* ring;
-    uint32_t full0, empty0, asfull0, asempty0;
-    int64_t u;      // unit whose ring items are being issued
-    uint32_t ui;    // its ordinal among this CTA's units
-    int i;          // its next item
-    uint32_t it;    // ring items issued
-    int64_t u_a;    // next unit whose A tiles are to be issued
-    uint32_t ua;    // units whose A tiles were issued
-    Unit U;
-
-    __device__ __forceinline__ void start(const TcParams& prm) {
-        u = blockIdx.x;
-        ui = 0;
-        i = 0;
-        it = 0;
-        u_a = blockIdx.x;
-        ua = 0;
-        if (u < prm.n_units) U = get_unit<D, DEC>(prm, u);
-    }
-    __device__ __forceinline__ bool done(const TcParams& prm) const {
-        return u >= prm.n_units && u_a >= prm.n_units;
-    }
-    // Issue what can be issued now (at most a few copies). Returns true if anything was.
-    __device__ __forceinline__ bool poll(const TcParams& prm) {
-        using C = Cfg<D, DEC>;
-        constexpr uint32_t kAhead = C::kABuf == 2 ? 1u : 0u;
-        bool any = false;
-        for (int n = 0; n < 4; ++n) {
-            if (u_a < prm.n_units && ua <= ui + kAhead) {
-                const int ab = ua & 1;
-                if (__all_sync(0xffffffffu,
-                               mbar_test_wait(asempty0 + 8u * ab, ((ua >> 1) & 1) ^ 1))) {
-                    const Unit UA = get_unit<D, DEC>(prm, u_a);
-                    if (elect_one()) {
-                        mbar_expect_tx(asfull0 + 8u * ab, UA.n_a * C::kATile);
-                        for (int a = 0; a < UA.n_a; ++a)
-                            tma_load_3d(smem_u32(abuf + ab * C::kABytes + a * C::kATile), tmA, 0,
-                                        UA.rowA0 + a * kTileRows, UA.zA, asfull0 + 8u * ab);
-                    }
-                    __syncwarp();
-                    ++ua;
-                    u_a += gridDim.x;
-                    any = true;
-                    continue;
-                }
-            }
-            if (u >= prm.n_units) return any;
-            if (i < U.n_items) {
-                const int st = it % C::kStages;
-                if (!__all_sync(0xffffffffu,
-                                mbar_test_wait(empty0 + 8u * st, ((it / C::kStages) & 1) ^ 1)))
-                    return any;
-                if (elect_one()) {
-                    mbar_expect_tx(full0 + 8u * st, C::kStage);
-                    const int row = (int)(U.item0 + (int64_t)i * C::kItem);
-                    const uint32_t dst = smem_u32(ring + st * C::kStage);
-                    tma_load_3d(dst, tmB, 0, row, U.zB, full0 + 8u * st);
-                    tma_load_3d(dst + C::kItemTile, tmC, 0, row, U.zB, full0 + 8u * st);
-                    // streams that do not consume this item count as having released it
-                    for (int x = U.n_a; x < NS; ++x) mbar_arrive(empty0 + 8u * st);
-                }
-                __syncwarp();
-                ++it;
-                ++i;
-                any = true;
-                continue;
-            }
-            u += gridDim.x;
-            ++ui;
-            i = 0;
-            if (u < prm.n_units) U = get_unit<D, DEC>(prm, u);
-        }
-        return any;
-    }
-    // After an abort: wait (bounded) until the newest copy of every buffer has landed.
-    __device__ __forceinline__ void drain() {
-        using C = Cfg<D, DEC>;
-        const uint64_t t0 = globaltimer_ns();
-        for (int st = 0; st < C::kStages; ++st) {
-            if ((uint32_t)st >= it) break;
-            const uint32_t x = it - 1 - ((it - 1 - st) % C::kStages);
-            while (!mbar_try_wait(full0 + 8u * st, (x / C::kStages) & 1) &&
-                   globaltimer_ns() - t0 < kWaitLimitNs) {
-            }
-        }
-        for (int b = 0; b < 2; ++b) {
-            if ((uint32_t)b >= ua) break;
-            const uint32_t y = ua - 1 - ((ua - 1 - b) % 2);
-            while (!mbar_try_wait(asfull0 + 8u * b, (y >> 1) & 1) &&
-                   globaltimer_ns() - t0 < kWaitLimitNs) {
-            }
-        }
-    }
-};
-
 // ------------------------------------------------------------------ the kernel
 
 template <int D, bool DEC>
@@ -643,140 +527,164 @@ __global__ void __launch_bounds__(kThreads, 1)
     tc_fence_after();
     const uint32_t tmem = *tmem_slot;
 
-    if (warp < kFirstSoftmaxWarp) {
+    if (warp < kProducerWarp) {
         // ------------------------------------------------------------ MMA warps
         // Warp s drives stream s. For each of its items: the PV of its previous item (P
         // from TMEM, V or Z from the ring), the S of this item (A from TMEM, K or Q from the
-        // ring) and one commit, which the softmax waits on. It observes the full barrier of
-        // every ring item in order, so each parity test names one phase. Warp 0 also keeps
-        // the TMA producer going whenever it would otherwise wait.
+        // ring) and one commit, which the softmax waits on, all from one elected lane with
+        // descriptors derived from two precomputed ones. It observes the full barrier of every
+        // ring item in order, so each parity test names one phase.
+        regs_lower<kRegsControl>();
         const int s = warp;
-        Producer<D, DEC> prod;
-        prod.tmA = &tmA;
-        prod.tmB = &tmB;
-        prod.tmC = &tmC;
-        prod.abuf = abuf;
-        prod.ring = ring;
-        prod.full0 = full0;
-        prod.empty0 = empty0;
-        prod.asfull0 = asfull0;
-        prod.asempty0 = asempty0;
-        if (s == 0) prod.start(prm);
-        // wait for a barrier phase; warp 0 feeds the producer meanwhile
-        auto wait = [&](uint32_t bar, uint32_t parity) -> bool {
-            if (s != 0) return warp_wait(bar, parity, abort_flag, prm.status);
-            uint64_t t0 = 0;
-            for (uint32_t n = 0;; ++n) {
-                if (__all_sync(0xffffffffu, mbar_test_wait(bar, parity))) return true;
-                if (prod.poll(prm)) {
-                    t0 = 0;
-                    continue;
-                }
-                if ((n & 63u) == 0) {
-                    if (__any_sync(0xffffffffu, *abort_flag != 0)) return false;
-                    const uint64_t now = globaltimer_ns();
-                    if (t0 == 0) t0 = now;
-                    if (now - t0 > kWaitLimitNs) {
-                        if (lane == 0) {
-                            *abort_flag = 1;
-                            atomicExch(prm.status, (int)FLAREPP_ERR_TIMEOUT);
-                        }
-                        __syncwarp();
-                        return false;
-                    }
-                }
-            }
-        };
-        uint32_t it = 0, ua = 0, pc0 = 0, pc1 = 0;  // p_ready phases consumed per buffer
+        const uint32_t ring_u = smem_u32(ring);
+        const uint64_t dS0 = smem_desc(ring_u, 16, C::kSBO, C::kSwz);
+        const uint64_t dV0 = smem_desc(ring_u + C::kItemTile, C::kItemTile, C::kSBO, C::kSwz);
+        const uint32_t d_s = tmem + C::kColS + s * C::kItem;  // B = 1: one score buffer
+        const uint32_t d_o = tmem + C::kColO + s * D;
+        const uint32_t sready_s = sready0 + 16u * s;
+        const uint32_t pready_s = pready0 + 16u * s;
+        uint32_t it = 0, ua = 0, pc = 0;  // ring items seen, units, p_ready phases consumed
         bool ok = true;
         for (int64_t u = blockIdx.x; u < prm.n_units && ok; u += gridDim.x, ++ua) {
             const Unit U = get_unit<D, DEC>(prm, u);
             const int tb = ua % C::kABuf;
-            if (!wait(aready0 + 8u * tb, (ua / C::kABuf) & 1)) break;
+            if (!warp_wait(aready0 + 8u * tb, (ua / C::kABuf) & 1, abort_flag, prm.status)) break;
             tc_fence_after();
             const int a = s % U.n_a;
             const int par = s / U.n_a;
             const uint32_t a_tmem = tmem + C::kColA + (tb * NS + a) * (D / 2);
-            const uint32_t sready_s = sready0 + 16u * s;
-            int j = 0, npv = 0;
-            int stg0 = 0, stg1 = 0;  // ring stages of this stream's items j with j % 2 == 0, 1
-            // PV of item jo = j - B (P in buffer jo % B), after its P is written
-            auto pv_of = [&](int jo) -> bool {
-                const int pb = jo % C::B;
-                uint32_t& pc = pb == 0 ? pc0 : pc1;
-                if (!wait(pready0 + 16u * s + 8u * pb, pc & 1)) return false;
-                ++pc;
-                tc_fence_after();
-                issue_pv<D, DEC>(tmem, ring, s, jo % C::B, (jo & 1) ? stg1 : stg0, npv);
-                ++npv;
-                return true;
-            };
+            int j = 0;
+            uint32_t st_prev = 0;  // ring stage of the stream's previous item
             for (int i = 0; i < U.n_items; ++i, ++it) {
-                const int st = it % C::kStages;
-                const bool mine = (i % U.n_par) == par;
-                // the item's full barrier first (the softmax is still busy with item j - B, so
-                // this wait is off the P -> PV -> S round trip), then the PV of item j - B,
-                // which frees the score buffer for S(j). Item i lands once item i - kStages
-                // is released; with kStages >= 2 B NS that item's PV was issued in an
-                // earlier iteration, so this wait cannot close a cycle.
-                if (!wait(full0 + 8u * st, (it / C::kStages) & 1)) {
+                const uint32_t st = it % C::kStages;
+                // the item's full barrier first (the softmax is still busy with item j - 1, so
+                // this wait is off the P -> PV -> S round trip), then the P of item j - 1.
+                // Item i lands once item i - kStages is released; with kStages >= 2 NS that
+                // item's PV was issued in an earlier iteration, so this wait closes no cycle.
+                if (!warp_wait(full0 + 8u * st, (it / C::kStages) & 1, abort_flag, prm.status)) {
                     ok = false;
                     break;
                 }
-                if (!mine) continue;
-                if (j >= C::B && !pv_of(j - C::B)) {
-                    ok = false;
-                    break;
+                if ((i % U.n_par) != par) continue;
+                if (j > 0) {
+                    if (!warp_wait(pready_s, pc & 1, abort_flag, prm.status)) {
+                        ok = false;
+                        break;
+                    }
+                    ++pc;
                 }
                 tc_fence_after();
-                const int b = j % C::B;
-                const uint32_t bb = smem_u32(ring + st * C::kStage);
+                if (elect_one()) {
+                    if (j > 0) {
+                        const uint64_t dv = dV0 + ((st_prev * C::kStage) >> 4);
 #pragma unroll
-                for (int k = 0; k < D / 16; ++k) {
-                    const uint64_t bd = smem_desc(bb + 32 * k, 16, C::kSBO, C::kSwz);
-                    if (elect_one())
-                        mma_ts(tmem + C::kColS + (s * C::B + b) * C::kItem, a_tmem + 8 * k, bd,
-                               C::kIdescS, k > 0 ? 1u : 0u);
-                    __syncwarp();
+                        for (int k = 0; k < C::kItem / 16; ++k)
+                            mma_ts(d_o, d_s + 8 * k, dv + (uint64_t)(2 * D * k), C::kIdescPV,
+                                   (j > 1 || k > 0) ? 1u : 0u);
+                    }
+                    const uint64_t ds = dS0 + ((st * C::kStage) >> 4);
+#pragma unroll
+                    for (int k = 0; k < D / 16; ++k)
+                        mma_ts(d_s, a_tmem + 8 * k, ds + (uint64_t)(2 * k), C::kIdescS,
+                               k > 0 ? 1u : 0u);
+                    mma_commit(sready_s);
                 }
-                if (elect_one()) mma_commit(sready_s + 8u * b);
                 __syncwarp();
-                if (j & 1)
-                    stg1 = st;
-                else
-                    stg0 = st;
+                st_prev = st;
                 ++j;
             }
             if (!ok) break;
-            // the PV of the unit's last item, then o_done: O is final for the softmax
-            if (j > 0) {
-                if (!pv_of(j - C::B)) break;
-                if (elect_one()) mma_commit(sready_s + 8u);
-                __syncwarp();
-            }
+            // the PV of the unit's last item, then o_done: O is final for the softmax; and
             // this stream's MMAs no longer read the unit's TMEM A buffer
-            if (elect_one()) mma_commit(afree0 + 8u * tb);
+            if (j > 0 && !warp_wait(pready_s, pc & 1, abort_flag, prm.status)) break;
+            if (j > 0) ++pc;
+            tc_fence_after();
+            if (elect_one()) {
+                if (j > 0) {
+                    const uint64_t dv = dV0 + ((st_prev * C::kStage) >> 4);
+#pragma unroll
+                    for (int k = 0; k < C::kItem / 16; ++k)
+                        mma_ts(d_o, d_s + 8 * k, dv + (uint64_t)(2 * D * k), C::kIdescPV,
+                               (j > 1 || k > 0) ? 1u : 0u);
+                    mma_commit(sready_s + 8u);
+                }
+                mma_commit(afree0 + 8u * tb);
+            }
             __syncwarp();
         }
-        if (s == 0) {
-            // issue whatever the other streams still need (normally nothing is left)
-            uint64_t t0 = globaltimer_ns();
-            while (!*abort_flag && !prod.done(prm)) {
-                if (prod.poll(prm)) {
-                    t0 = globaltimer_ns();
-                } else if (globaltimer_ns() - t0 > kWaitLimitNs) {
-                    if (lane == 0) {
-                        *abort_flag = 1;
-                        atomicExch(prm.status, (int)FLAREPP_ERR_TIMEOUT);
+    } else if (warp < kFirstSoftmaxWarp) {
+        // ------------------------------------------------------------ TMA producer
+        // Order: A(0) [, A(1) with two TMEM copies], items(0), A(next), items(1), ... A group
+        // of unit k goes into shared buffer k % 2 once the softmax has copied the group before
+        // it in that buffer into TMEM. Every wait blocks (try_wait), so the warp takes no issue
+        // slots while it waits.
+        regs_lower<kRegsControl>();
+        if (warp == kProducerWarp) {
+            constexpr uint32_t kAhead = C::kABuf == 2 ? 1u : 0u;
+            const int64_t G = gridDim.x;
+            uint32_t it = 0, na = 0;  // ring items and A groups issued
+            bool ok = true;
+            auto issue_a = [&](uint32_t k, int64_t u) -> bool {
+                const int ab = k & 1;
+                if (!warp_wait(asempty0 + 8u * ab, ((k >> 1) & 1) ^ 1, abort_flag, prm.status))
+                    return false;
+                const Unit UA = get_unit<D, DEC>(prm, u);
+                if (elect_one()) {
+                    mbar_expect_tx(asfull0 + 8u * ab, UA.n_a * C::kATile);
+                    for (int a = 0; a < UA.n_a; ++a)
+                        tma_load_3d(smem_u32(abuf + ab * C::kABytes + a * C::kATile), &tmA, 0,
+                                    UA.rowA0 + a * kTileRows, UA.zA, asfull0 + 8u * ab);
+                }
+                __syncwarp();
+                ++na;
+                return true;
+            };
+            for (uint32_t k = 0; k <= kAhead && ok; ++k)
+                if (blockIdx.x + k * G < prm.n_units) ok = issue_a(k, blockIdx.x + k * G);
+            uint32_t k = 0;
+            for (int64_t u = blockIdx.x; u < prm.n_units && ok; u += G, ++k) {
+                const Unit U = get_unit<D, DEC>(prm, u);
+                for (int i = 0; i < U.n_items; ++i, ++it) {
+                    const int st = it % C::kStages;
+                    if (!warp_wait(empty0 + 8u * st, ((it / C::kStages) & 1) ^ 1, abort_flag,
+                                   prm.status)) {
+                        ok = false;
+                        break;
+                    }
+                    if (elect_one()) {
+                        mbar_expect_tx(full0 + 8u * st, C::kStage);
+                        const int row = (int)(U.item0 + (int64_t)i * C::kItem);
+                        const uint32_t dst = smem_u32(ring + st * C::kStage);
+                        tma_load_3d(dst, &tmB, 0, row, U.zB, full0 + 8u * st);
+                        tma_load_3d(dst + C::kItemTile, &tmC, 0, row, U.zB, full0 + 8u * st);
+                        // streams that do not take this item count as having released it
+                        for (int x = U.n_a; x < NS; ++x) mbar_arrive(empty0 + 8u * st);
                     }
                     __syncwarp();
-                    break;
+                }
+                const int64_t un = u + (1 + kAhead) * G;
+                if (ok && un < prm.n_units) ok = issue_a(k + 1 + kAhead, un);
+            }
+            if (!ok) {
+                // after an abort: wait (bounded) until the newest copy into every buffer landed
+                const uint64_t t0 = globaltimer_ns();
+                for (uint32_t st = 0; st < (uint32_t)C::kStages && st < it; ++st) {
+                    const uint32_t x = it - 1 - ((it - 1 - st) % C::kStages);
+                    while (!mbar_try_wait(full0 + 8u * st, (x / C::kStages) & 1) &&
+                           globaltimer_ns() - t0 < kWaitLimitNs) {
+                    }
+                }
+                for (uint32_t b = 0; b < 2 && b < na; ++b) {
+                    const uint32_t y = na - 1 - ((na - 1 - b) % 2);
+                    while (!mbar_try_wait(asfull0 + 8u * b, (y >> 1) & 1) &&
+                           globaltimer_ns() - t0 < kWaitLimitNs) {
+                    }
                 }
             }
-            if (*abort_flag) prod.drain();
         }
     } else {
         // ------------------------------------------------------------ softmax warpgroups
+        regs_raise<kRegsSoftmax>();
         const int wg = (warp - kFirstSoftmaxWarp) >> 2;
         const int q = warp & 3;
         const int r = q * 32 + lane;
