@@ -415,10 +415,23 @@ def chain_bwd_launches(w):
     return 11 + (4 if w.D <= 32 else 0)
 
 
+def chain_fwd_launches(w):
+    """Kernels of one chain forward: on the tensor-core path each encode and the decode is a
+    fast kernel followed by its safe kernel (which returns at once unless the fast one
+    overflowed), plus two merges and, for a negative scale, the negation of the seeds: 8
+    (9); on the CUDA-core path encode, merge, encode, merge, decode: 5."""
+    if w.dtype != "bf16":
+        return 5
+    return 8 + (1 if w.scale < 0 else 0)
+
+
 def flare_launches(w):
-    """Kernels of one FLARE call: encode, merge and decode, plus the negation of the
-    bf16 queries when the scale is negative."""
-    return 3 + (1 if w.dtype == "bf16" and w.scale < 0 else 0)
+    """Kernels of one FLARE call: encode, merge and decode (the encode and decode as a fast
+    and a safe kernel on the tensor-core path), plus the negation of the bf16 queries when
+    the scale is negative."""
+    if w.dtype != "bf16":
+        return 3
+    return 5 + (1 if w.scale < 0 else 0)
 
 
 def run_flare(args, w, flarepp, world, rank, dev, peaks, x, Y, ws, stream):
@@ -601,8 +614,7 @@ def run_train(args, w, flarepp, world, rank, dev, peaks, x, Y, ws, stream):
             "step_roofline": {"roofline_us": t_step * 1e6, "frac": t_step / (ms * 1e-3),
                               "flops": "42 BNMHD", "tensors": 15},
             "cpu_baseline": cpu, "e2e": None, "clocks": clk,
-            "gpu_launches": (5 + (1 if w.dtype == "bf16" and w.scale < 0 else 0)
-                             + chain_bwd_launches(w)) * args.steps,
+            "gpu_launches": (chain_fwd_launches(w) + chain_bwd_launches(w)) * args.steps,
         }
         print(json.dumps(line), flush=True)
     if world > 1:
@@ -705,10 +717,11 @@ def run_mixer_train(args, w, flarepp, world, rank, dev, peaks, stream):
             "config": arm_config(w, "mixer_train", world),
             "stage_ms": {"forward_train": fwd_ms, "backward": bwd_ms}, "roofline": roof,
             "cpu_baseline": None, "e2e": None, "clocks": clk,
-            # forward: projection, the chain's five kernels, output projection; backward: two
+            # forward: projection, the chain's kernels, output projection; backward: two
             # weight transposes, dY, dWo and its reduce, the chain's backward, dW_in and its
             # reduce, dX
-            "gpu_launches": (7 + 8 + chain_bwd_launches(w)) * args.steps,
+            "gpu_launches": (2 + chain_fwd_launches(w) + 8 + chain_bwd_launches(w))
+                            * args.steps,
         }
         print(json.dumps(line), flush=True)
     if world > 1:
@@ -792,7 +805,8 @@ def run_mixer(args, w, flarepp, world, rank, dev, peaks, stream):
             "dtype": "bf16", "data": "synthetic",
             "config": arm_config(w, args.variant, world),
             "stage_ms": stage_ms, "roofline": roof, "layer_roofline": layer,
-            "cpu_baseline": cpu, "e2e": None, "clocks": clk, "gpu_launches": 7 * args.steps,
+            "cpu_baseline": cpu, "e2e": None, "clocks": clk,
+            "gpu_launches": (2 + chain_fwd_launches(w)) * args.steps,
         }
         print(json.dumps(line), flush=True)
     if world > 1:
@@ -942,7 +956,7 @@ def run_ours(args, w):
             "config": arm_config(w, args.variant, world),
             "roofline": roof, "chain_roofline": chain, "stage_ms": stage_ms,
             "cpu_baseline": cpu, "e2e": e2e, "clocks": clk,
-            "gpu_launches": 5 * args.steps,
+            "gpu_launches": chain_fwd_launches(w) * args.steps,
         }
         print(json.dumps(line), flush=True)
     if world > 1:

@@ -130,6 +130,8 @@ flarepp_status route_impl(const flarepp_shape* shape, const void* seeds, const v
     };
     if (reset_status && cudaMemsetAsync(ws + p.off_status, 0, sizeof(int32_t), st) != cudaSuccess)
         return FLAREPP_ERR_CUDA;
+    if (tc && cudaMemsetAsync(ws + p.off_overflow, 0, 3 * sizeof(int32_t), st) != cudaSuccess)
+        return FLAREPP_ERR_CUDA;
     if (tc && neg &&
         negate_bf16(seeds, ws + p.off_seedneg, p.H * p.M * p.D, st) != cudaSuccess)
         return FLAREPP_ERR_CUDA;
@@ -211,6 +213,8 @@ flarepp_status flare_impl(const flarepp_shape* shape, const void* Qh, const void
     const bool tc = p.path == kPathTc;
     const bool neg = scale < 0.f;
     if (reset_status && cudaMemsetAsync(ws + p.off_status, 0, sizeof(int32_t), st) != cudaSuccess)
+        return FLAREPP_ERR_CUDA;
+    if (tc && cudaMemsetAsync(ws + p.off_overflow, 0, 3 * sizeof(int32_t), st) != cudaSuccess)
         return FLAREPP_ERR_CUDA;
     // the encode of call 1 with the learned queries, merged into Z
     if (tc && neg && negate_bf16(Qh, ws + p.off_seedneg, p.H * p.M * p.D, st) != cudaSuccess)

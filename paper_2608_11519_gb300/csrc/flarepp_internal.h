@@ -33,6 +33,7 @@ struct Plan {
     int64_t sub_per_chunk;     // partial slots per chunk (1 CUDA-core, 4 tensor-core)
     // workspace layout (byte offsets from the workspace base, each 256-byte aligned)
     size_t off_status;                    // int32 device status word (FLAREPP_OK or _TIMEOUT)
+    size_t off_overflow;                  // int32 x 3: the tensor-core kernels' overflow words
     size_t off_pmax, off_psum, off_pacc;  // partials [BH][nchunk*sub][M] f32 x2, (...)[D] f32
     size_t off_q32, off_z32;              // Q, Z float32 [BH][M][D]
     size_t off_qop, off_zop;              // bf16 MMA operand copies of Q, Z [BH][M][D]

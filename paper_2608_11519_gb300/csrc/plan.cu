@@ -104,7 +104,10 @@ flarepp_status make_plan(const flarepp_shape* s, Plan* p) {
         (size_t)bh * (size_t)p->nchunk * (size_t)p->sub_per_chunk * (size_t)s->M;
     size_t off = 0;
     p->off_status = off;
-    off = align_up(off + sizeof(int32_t), kWsAlign);
+    // the overflow words of encode calls 1 and 2 and of the decode (tensor-core path) share
+    // the status word's 256-byte block
+    p->off_overflow = off + 16;
+    off = align_up(off + 16 + 3 * sizeof(int32_t), kWsAlign);
     p->off_pmax = off;
     off = align_up(off + rows * sizeof(float), kWsAlign);
     p->off_psum = off;

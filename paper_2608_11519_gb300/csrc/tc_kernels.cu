@@ -115,6 +115,7 @@ struct TcParams {
     float* lse;  // decode: each token's base-2 log-normaliser, or null
     int64_t n_units;
     int* status;
+    int* overflow;  // raised by the fast kernel; the safe kernel runs only when it is set
 };
 
 // route tiles of encode group g, rounded up to 1, 2 or 4 (a divisor of the stream count)
@@ -208,6 +209,7 @@ struct SoftmaxStream {
     float m, l;     // reference max (base 2, scaled) and running sum
     uint32_t ph0;   // s_ready phases completed in earlier units (one per item)
     uint32_t od;    // o_done phases completed in earlier units (one per unit with items)
+    bool over;      // fast kernel: some item's sum passed kFastLimit
     __device__ __forceinline__ void begin(const Unit& U) {
         const int par = s / U.n_a;
         cnt = U.n_items > par ? (U.n_items - par + U.n_par - 1) / U.n_par : 0;
@@ -280,7 +282,11 @@ __device__ __forceinline__ float exp_chunk(const uint32_t* sr, uint32_t* pr, int
 // the row is a valid reference (that score alone contributes 2^0 = 1 to the sum, so the
 // sum never underflows), and a reference far below the row's maximum shows up as a sum
 // past the fast-path limit, which sends the item to the exact-max path.
-template <int ITEM, bool FIRST_REF>
+//
+// STORE (the fast kernel): each chunk's P goes back to TMEM as soon as it is packed (it covers
+// only columns already read), so S is gone by the end. Otherwise P stays in pr for the
+// caller, and S stays intact until the caller writes it.
+template <int ITEM, bool FIRST_REF, bool STORE>
 __device__ __forceinline__ float exp_tile(uint32_t scol, uint32_t* pr, int nv, float c,
                                           uint64_t c2, float& m, bool first) {
     float sum = 0.f;
@@ -291,13 +297,15 @@ __device__ __forceinline__ float exp_tile(uint32_t scol, uint32_t* pr, int nv, f
         tmem_wait_ld32(sr);
         if (FIRST_REF && h == 0 && first) m = c * __uint_as_float(sr[0]);
         sum += exp_chunk<32>(sr, pr + 16 * h, 32 * h, nv, c, c2, m);
+        if constexpr (STORE) tmem_st16(scol + 16 * h, pr + 16 * h);
     }
-    if (ITEM % 32 == 16) {
+    if constexpr (ITEM % 32 == 16) {
         constexpr int base = ITEM - 16;
         uint32_t sr[16];
         tmem_ld16(scol + base, sr);
         tmem_wait_ld16(sr);
         sum += exp_chunk<16>(sr, pr + base / 2, base, nv, c, c2, m);
+        if constexpr (STORE) tmem_st8(scol + base / 2, pr + base / 2);
     }
     return sum;
 }
@@ -305,15 +313,23 @@ __device__ __forceinline__ float exp_tile(uint32_t scol, uint32_t* pr, int nv, f
 // One item of this warpgroup's stream for this thread's row: read S, update the online
 // softmax, write P back over S, signal the stream's MMA warp. S of item j being ready
 // means the PV of item j - B has completed, so the warpgroup leader frees that item's ring
-// stage. Returns false when the kernel is aborting. The decode (DEC), whose units are
-// short, takes the first item's reference from its first score; the encode, whose units
-// are long, takes the first item's exact maximum, which measured faster there.
-template <int D, bool DEC>
+// stage. Returns false when the kernel is aborting.
+//   fast kernel (!SAFE): the reference is kept from the items before (a unit's first item
+//     takes its first score) and P is stored chunk by chunk, so S is gone by the end of the
+//     item. A sum past kFastLimit (a score far above the reference) cannot be repaired
+//     here: the thread notes it, the kernel raises the launch's overflow word when it ends,
+//     and the safe kernel that follows on the stream recomputes the whole launch.
+//   safe kernel: P is stored once the item's sum is known; a sum past kFastLimit sends the
+//     item to the exact-max path, which reads S again (the decode, whose units are short,
+//     takes the first item's reference from its first score; the encode, whose units are
+//     long, takes the first item's exact maximum).
+template <int D, bool DEC, bool SAFE>
 __device__ __forceinline__ bool softmax_step(SoftmaxStream& S, const Unit& U, uint32_t tmem,
                                              uint32_t lane_off, float c, uint64_t c2,
                                              uint32_t sready_s, uint32_t pready_s, uint32_t empty0,
                                              bool wg_leader, uint32_t it0,
-                                             volatile int* abort_flag, int* status) {
+                                             volatile int* abort_flag, int* status,
+                                             volatile int* overflow) {
     using C = Cfg<D, DEC>;
     const int j = S.j;
     const int b = j % C::B;
@@ -331,9 +347,19 @@ __device__ __forceinline__ bool softmax_step(SoftmaxStream& S, const Unit& U, ui
     const uint32_t scol = tmem + lane_off + C::kColS + (S.s * C::B + b) * C::kItem;
     uint32_t pr[C::kItem / 2];
     float sum = 0.f;
+    if constexpr (!SAFE) {
+        sum = exp_tile<C::kItem, true, true>(scol, pr, nv, c, c2, S.m, j == 0);
+        tmem_wait_st();
+        tc_fence_before();
+        mbar_arrive(pready_s + 8u * b);
+        S.over |= !(sum <= kFastLimit);  // checked once, when the kernel ends
+        S.l += sum;
+        ++S.j;
+        return true;
+    }
     bool slow = !DEC && j == 0;
     if (!slow) {
-        sum = exp_tile<C::kItem, DEC>(scol, pr, nv, c, c2, S.m, j == 0);
+        sum = exp_tile<C::kItem, DEC, false>(scol, pr, nv, c, c2, S.m, j == 0);
         slow = __any_sync(0xffffffffu, !(sum <= kFastLimit));
     }
     if (slow) {
@@ -375,13 +401,13 @@ __device__ __forceinline__ bool softmax_step(SoftmaxStream& S, const Unit& U, ui
                 tmem_st16(ocol + 16 * k, o);
             }
         }
-        sum = exp_tile<C::kItem, false>(scol, pr, nv, c, c2, S.m, false);
+        sum = exp_tile<C::kItem, false, false>(scol, pr, nv, c, c2, S.m, false);
     }
     S.l += sum;
-    if (C::kItem == 80) {
+    if constexpr (C::kItem == 80) {
         tmem_st32(scol, pr);
         tmem_st8(scol + 32, pr + 32);
-    } else if (C::kItem == 64) {
+    } else if constexpr (C::kItem == 64) {
         tmem_st32(scol, pr);
     } else {
         tmem_st16(scol, pr);
@@ -468,11 +494,18 @@ __device__ __forceinline__ bool finish_stream(SoftmaxStream& S, const Unit& U,
 
 // ------------------------------------------------------------------ the kernel
 
-template <int D, bool DEC>
+template <int D, bool DEC, bool SAFE>
 __global__ void __launch_bounds__(kThreads, 1)
     tc_chain_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
                     const __grid_constant__ CUtensorMap tmC, const TcParams prm) {
     using C = Cfg<D, DEC>;
+    if constexpr (SAFE) {
+        // the safe kernel recomputes the launch only when the fast one overflowed
+        __shared__ int run;
+        if (threadIdx.x == 0) run = *reinterpret_cast<volatile int*>(prm.overflow);
+        __syncthreads();
+        if (!run) return;
+    }
     extern __shared__ uint8_t smem_raw[];
     uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                                ~static_cast<uintptr_t>(1023));
@@ -696,6 +729,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         st.s = wg;
         st.ph0 = 0;
         st.od = 0;
+        st.over = false;
         const uint32_t sready_s = sready0 + 16u * wg;
         bool alive = true;
         uint32_t ua = 0, it0 = 0;
@@ -748,14 +782,15 @@ __global__ void __launch_bounds__(kThreads, 1)
             }
             st.begin(U);
             while (alive && st.j < st.cnt)
-                alive = softmax_step<D, DEC>(st, U, tmem, lane_off, c, c2, sready_s,
-                                        pready0 + 16u * st.s, empty0, wg_leader, it0, abort_flag,
-                                        prm.status);
+                alive = softmax_step<D, DEC, SAFE>(st, U, tmem, lane_off, c, c2, sready_s,
+                                                   pready0 + 16u * st.s, empty0, wg_leader, it0,
+                                                   abort_flag, prm.status, prm.overflow);
             if (alive)
                 alive = finish_stream<D, DEC>(st, U, prm, tmem, lane_off, r, sready_s, empty0,
                                               wg_leader, it0, abort_flag);
             it0 += U.n_items;
         }
+        if (!SAFE && __any_sync(0xffffffffu, st.over) && lane == 0) *prm.overflow = 1;
     }
 
     tc_fence_before();
@@ -803,17 +838,22 @@ bool make_map(CUtensorMap* m, const void* base, int64_t D, int64_t rows, int64_t
               CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
+// The fast kernel, then the safe one on the same stream (it returns at once unless the
+// fast kernel raised the overflow word, which the plan keeps zeroed before each call).
 template <int D, bool DEC>
 cudaError_t launch(const CUtensorMap& a, const CUtensorMap& b, const CUtensorMap& c,
                    const TcParams& prm, cudaStream_t st) {
     using Cf = Cfg<D, DEC>;
-    const cudaError_t attr = ensure_smem_limit((const void*)tc_chain_kernel<D, DEC>, Cf::kSmem);
-    if (attr != cudaSuccess) return attr;
+    cudaError_t e = ensure_smem_limit((const void*)tc_chain_kernel<D, DEC, false>, Cf::kSmem);
+    if (e == cudaSuccess)
+        e = ensure_smem_limit((const void*)tc_chain_kernel<D, DEC, true>, Cf::kSmem);
+    if (e != cudaSuccess) return e;
     int dev = 0, sms = kNumSMs;
     cudaGetDevice(&dev);
     cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
     const int64_t grid = prm.n_units < sms ? prm.n_units : sms;
-    tc_chain_kernel<D, DEC><<<(unsigned)grid, kThreads, Cf::kSmem, st>>>(a, b, c, prm);
+    tc_chain_kernel<D, DEC, false><<<(unsigned)grid, kThreads, Cf::kSmem, st>>>(a, b, c, prm);
+    tc_chain_kernel<D, DEC, true><<<(unsigned)grid, kThreads, Cf::kSmem, st>>>(a, b, c, prm);
     return cudaGetLastError();
 }
 
@@ -875,6 +915,7 @@ cudaError_t tc_encode(const Plan& p, int call, const void* k, const void* v, con
     prm.pacc = (float*)(ws + p.off_pacc);
     prm.n_units = p.BH * p.n_groups * p.nchunk;
     prm.status = (int*)(ws + p.off_status);
+    prm.overflow = (int*)(ws + p.off_overflow) + (call - 1);
     return launch_d<false>(p.D, ma, mb, mc, prm, st);
 }
 
@@ -897,6 +938,7 @@ cudaError_t tc_decode(const Plan& p, const void* K, float scale, void* Y, char* 
     prm.lse = lse;
     prm.n_units = p.BH * prm.n_tok_groups;
     prm.status = (int*)(ws + p.off_status);
+    prm.overflow = (int*)(ws + p.off_overflow) + 2;
     return launch_d<true>(p.D, ma, mb, mc, prm, st);
 }
 

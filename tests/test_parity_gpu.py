@@ -275,6 +275,33 @@ def test_flare_fixed_queries(B, H, N, M, D, dtype, scale):
     _check("Y", _np(Y), Yo, TOL[dtype])
 
 
+@pytest.mark.parametrize("D,M", [(16, 300), (32, 520), (64, 130)])
+def test_bf16_logits_far_above_reference(D, M):
+    """Scores far above a row's running reference. The bf16 kernels take each unit's first
+    score as the reference and overwrite S with P as they go; a row whose later scores
+    exceed the reference by tens of base-2 units is recomputed exactly. With scale 3, the
+    base-2 logits have a spread of about 25 per standard deviation, so nearly every encode
+    and decode row takes that path at least once. FLARE's queries are exact bf16 inputs, so
+    the softmaxes (nearly one-hot) are compared without the chain's amplification of
+    operand rounding."""
+    w = inputs.Workload("flare", 1, 3, 2000, M, D, "bf16")
+    s = 3.0
+    x = inputs.make_inputs(w, seed=9)
+    f = inputs.to_f64_numpy(x)
+    Zo, Yo = oracle.flare(f["seeds"], f["K"], f["V"], s)
+    xd = {k: v.cuda() for k, v in x.items()}
+    Z = torch.empty((1, 3, M, D), dtype=torch.float32, device="cuda")
+    Y = flarepp.flare_fwd(xd["seeds"], xd["K"], xd["V"], s, Z_out=Z)
+    torch.cuda.synchronize()
+    _check("Z", _np(Z), Zo, TOL["bf16"])
+    # The decode's rows are nearly one-hot here, so the bf16 rounding of its P (relative
+    # 2^-9 per probability) no longer averages out over many routes: between two close
+    # routes it moves Y by up to 2^-8 |Z_a - Z_b| (|Z| <= max|V| ~ 4: 0.031), and the bf16
+    # operand copy of Z adds 2^-9 |Z| (0.008). An exact-path mistake (a wrong reference,
+    # a sum counted twice) moves Y by O(1).
+    _check("Y", _np(Y), Yo, 4e-2)
+
+
 @pytest.mark.parametrize("B,H,N,M,D,dtype,scale", [
     (1, 8, 5000, 128, 32, "bf16", None),   # eight head groups
     (2, 3, 1500, 40, 16, "bf16", -0.3),    # groups of whole batch elements, negative scale
