@@ -347,6 +347,21 @@ FLAREPP_API flarepp_status flarepp_route_device_status(const flarepp_shape* shap
                                                        const void* workspace, void* stream,
                                                        int32_t* status_out);
 
+/*
+ * Test hook of the bounded waits; the paper has no counterpart. It lets a test make a wait
+ * inside a tensor-core kernel run out without faulting or hanging the GPU.
+ *   kernel: which launch of later calls it applies to: 1 or 2, the encode of call 1 or 2;
+ *     3, the decode; 0 turns the hook off (the default).
+ *   ring_item: the index, in the order it is loaded, of an item of CTA 0's ring of K/V (or
+ *     Q/Z) tiles that the kernel's load warp then never loads, so that the waits for it run
+ *     out (-1: none).
+ *   wait_ns: the bound of every wait of that launch (0: the default of 2 s).
+ * Process-wide state, for tests only: it applies to every later call from any thread until it
+ * is turned off. A launch whose wait ran out stops early and records FLAREPP_ERR_TIMEOUT in
+ * the device status word (flarepp_route_device_status); its outputs are invalid.
+ */
+FLAREPP_API void flarepp_test_wait_fault(int kernel, int64_t ring_item, uint64_t wait_ns);
+
 /* Static description of a status code (never NULL). */
 FLAREPP_API const char* flarepp_status_string(flarepp_status status);
 

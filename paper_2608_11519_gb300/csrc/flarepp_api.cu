@@ -953,4 +953,8 @@ const char* flarepp_status_string(flarepp_status status) {
 
 const char* flarepp_version(void) { return "0.1.0"; }
 
+void flarepp_test_wait_fault(int kernel, int64_t ring_item, uint64_t wait_ns) {
+    flarepp::set_tc_test_fault(kernel, ring_item, wait_ns);
+}
+
 }  // extern "C"

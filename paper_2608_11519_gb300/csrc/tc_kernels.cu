@@ -56,7 +56,7 @@ constexpr uint32_t kRegsSoftmax = 96;
 static_assert(kRegsControl * 256 + kRegsSoftmax * 512 <= 80 * 768, "register split");
 constexpr int NS = 4;           // TMEM streams
 constexpr int kTileRows = 128;  // TMEM lanes, MMA M
-constexpr uint64_t kWaitLimitNs = 2000000000ull;
+constexpr uint64_t kDefaultWaitNs = 2000000000ull;
 constexpr uint32_t kTmemCols = 512;
 constexpr float kLog2e = 1.4426950408889634f;
 // Sum of one item's probabilities above which the reference max is recomputed exactly.
@@ -116,6 +116,8 @@ struct TcParams {
     int64_t n_units;
     int* status;
     int* overflow;  // raised by the fast kernel; the safe kernel runs only when it is set
+    uint64_t wait_ns;     // bound of every wait (kDefaultWaitNs unless the test hook is set)
+    int64_t withhold_it;  // test hook: ring item of CTA 0 the producer never loads (-1: none)
 };
 
 // route tiles of encode group g, rounded up to 1, 2 or 4 (a divisor of the stream count)
@@ -178,14 +180,14 @@ __device__ __forceinline__ uint32_t pack_bf16(float lo, float hi) {
 
 // Bounded wait on an mbarrier phase. Returns false when the kernel is aborting.
 __device__ __forceinline__ bool wait_bar(uint32_t bar, uint32_t parity, volatile int* abort_flag,
-                                         int* status) {
+                                         int* status, uint64_t limit) {
     if (mbar_try_wait(bar, parity)) return true;
     const uint64_t t0 = globaltimer_ns();
     for (uint32_t i = 1;; ++i) {
         if (mbar_try_wait(bar, parity)) return true;
         if ((i & 63u) == 0) {
             if (*abort_flag) return false;
-            if (globaltimer_ns() - t0 > kWaitLimitNs) {
+            if (globaltimer_ns() - t0 > limit) {
                 *abort_flag = 1;
                 atomicExch(status, (int)FLAREPP_ERR_TIMEOUT);
                 return false;
@@ -195,8 +197,8 @@ __device__ __forceinline__ bool wait_bar(uint32_t bar, uint32_t parity, volatile
 }
 // The same wait taken by a whole warp: true only if every lane saw the phase complete.
 __device__ __forceinline__ bool warp_wait(uint32_t bar, uint32_t parity, volatile int* abort_flag,
-                                          int* status) {
-    const bool got = wait_bar(bar, parity, abort_flag, status);
+                                          int* status, uint64_t limit) {
+    const bool got = wait_bar(bar, parity, abort_flag, status, limit);
     return __all_sync(0xffffffffu, got);
 }
 
@@ -329,12 +331,12 @@ __device__ __forceinline__ bool softmax_step(SoftmaxStream& S, const Unit& U, ui
                                              uint32_t sready_s, uint32_t pready_s, uint32_t empty0,
                                              bool wg_leader, uint32_t it0,
                                              volatile int* abort_flag, int* status,
-                                             volatile int* overflow) {
+                                             uint64_t limit, volatile int* overflow) {
     using C = Cfg<D, DEC>;
     const int j = S.j;
     const int b = j % C::B;
     const uint32_t par_j = (S.ph0 + (uint32_t)j) & 1u;
-    if (!warp_wait(sready_s + 8u * b, par_j, abort_flag, status)) return false;
+    if (!warp_wait(sready_s + 8u * b, par_j, abort_flag, status, limit)) return false;
     tc_fence_after();
     const int par = S.s / U.n_a;
     if (wg_leader && j >= C::B) {
@@ -433,7 +435,7 @@ __device__ __forceinline__ bool finish_stream(SoftmaxStream& S, const Unit& U,
     const int par = S.s / U.n_a;
     float o[D];
     if (S.cnt > 0) {
-        if (!warp_wait(sready_s + 8u, S.od & 1u, abort_flag, prm.status)) return false;
+        if (!warp_wait(sready_s + 8u, S.od & 1u, abort_flag, prm.status, prm.wait_ns)) return false;
         ++S.od;
         tc_fence_after();
         if (wg_leader) {
@@ -581,7 +583,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         for (int64_t u = blockIdx.x; u < prm.n_units && ok; u += gridDim.x, ++ua) {
             const Unit U = get_unit<D, DEC>(prm, u);
             const int tb = ua % C::kABuf;
-            if (!warp_wait(aready0 + 8u * tb, (ua / C::kABuf) & 1, abort_flag, prm.status)) break;
+            if (!warp_wait(aready0 + 8u * tb, (ua / C::kABuf) & 1, abort_flag, prm.status, prm.wait_ns)) break;
             tc_fence_after();
             const int a = s % U.n_a;
             const int par = s / U.n_a;
@@ -594,13 +596,13 @@ __global__ void __launch_bounds__(kThreads, 1)
                 // this wait is off the P -> PV -> S round trip), then the P of item j - 1.
                 // Item i lands once item i - kStages is released; with kStages >= 2 NS that
                 // item's PV was issued in an earlier iteration, so this wait closes no cycle.
-                if (!warp_wait(full0 + 8u * st, (it / C::kStages) & 1, abort_flag, prm.status)) {
+                if (!warp_wait(full0 + 8u * st, (it / C::kStages) & 1, abort_flag, prm.status, prm.wait_ns)) {
                     ok = false;
                     break;
                 }
                 if ((i % U.n_par) != par) continue;
                 if (j > 0) {
-                    if (!warp_wait(pready_s, pc & 1, abort_flag, prm.status)) {
+                    if (!warp_wait(pready_s, pc & 1, abort_flag, prm.status, prm.wait_ns)) {
                         ok = false;
                         break;
                     }
@@ -629,7 +631,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             if (!ok) break;
             // the PV of the unit's last item, then o_done: O is final for the softmax; and
             // this stream's MMAs no longer read the unit's TMEM A buffer
-            if (j > 0 && !warp_wait(pready_s, pc & 1, abort_flag, prm.status)) break;
+            if (j > 0 && !warp_wait(pready_s, pc & 1, abort_flag, prm.status, prm.wait_ns)) break;
             if (j > 0) ++pc;
             tc_fence_after();
             if (elect_one()) {
@@ -656,10 +658,12 @@ __global__ void __launch_bounds__(kThreads, 1)
             constexpr uint32_t kAhead = C::kABuf == 2 ? 1u : 0u;
             const int64_t G = gridDim.x;
             uint32_t it = 0, na = 0;  // ring items and A groups issued
+            int64_t withheld = -1;
             bool ok = true;
             auto issue_a = [&](uint32_t k, int64_t u) -> bool {
                 const int ab = k & 1;
-                if (!warp_wait(asempty0 + 8u * ab, ((k >> 1) & 1) ^ 1, abort_flag, prm.status))
+                if (!warp_wait(asempty0 + 8u * ab, ((k >> 1) & 1) ^ 1, abort_flag, prm.status,
+                               prm.wait_ns))
                     return false;
                 const Unit UA = get_unit<D, DEC>(prm, u);
                 if (elect_one()) {
@@ -680,9 +684,13 @@ __global__ void __launch_bounds__(kThreads, 1)
                 for (int i = 0; i < U.n_items; ++i, ++it) {
                     const int st = it % C::kStages;
                     if (!warp_wait(empty0 + 8u * st, ((it / C::kStages) & 1) ^ 1, abort_flag,
-                                   prm.status)) {
+                                   prm.status, prm.wait_ns)) {
                         ok = false;
                         break;
+                    }
+                    if (blockIdx.x == 0 && (int64_t)it == prm.withhold_it) {
+                        withheld = it;  // never loaded: the waits of its consumers run out
+                        continue;
                     }
                     if (elect_one()) {
                         mbar_expect_tx(full0 + 8u * st, C::kStage);
@@ -703,14 +711,15 @@ __global__ void __launch_bounds__(kThreads, 1)
                 const uint64_t t0 = globaltimer_ns();
                 for (uint32_t st = 0; st < (uint32_t)C::kStages && st < it; ++st) {
                     const uint32_t x = it - 1 - ((it - 1 - st) % C::kStages);
-                    while (!mbar_try_wait(full0 + 8u * st, (x / C::kStages) & 1) &&
-                           globaltimer_ns() - t0 < kWaitLimitNs) {
+                    while ((int64_t)x != withheld &&
+                           !mbar_try_wait(full0 + 8u * st, (x / C::kStages) & 1) &&
+                           globaltimer_ns() - t0 < prm.wait_ns) {
                     }
                 }
                 for (uint32_t b = 0; b < 2 && b < na; ++b) {
                     const uint32_t y = na - 1 - ((na - 1 - b) % 2);
                     while (!mbar_try_wait(asfull0 + 8u * b, (y >> 1) & 1) &&
-                           globaltimer_ns() - t0 < kWaitLimitNs) {
+                           globaltimer_ns() - t0 < prm.wait_ns) {
                     }
                 }
             }
@@ -740,9 +749,9 @@ __global__ void __launch_bounds__(kThreads, 1)
             const int n_a = get_unit<D, DEC>(prm, u_c).n_a;
             const int ab = ua_c & 1;
             const int tb = ua_c % C::kABuf;
-            if (!warp_wait(asfull0 + 8u * ab, (ua_c >> 1) & 1, abort_flag, prm.status))
+            if (!warp_wait(asfull0 + 8u * ab, (ua_c >> 1) & 1, abort_flag, prm.status, prm.wait_ns))
                 return false;
-            if (!warp_wait(afree0 + 8u * tb, ((ua_c / C::kABuf) & 1) ^ 1, abort_flag, prm.status))
+            if (!warp_wait(afree0 + 8u * tb, ((ua_c / C::kABuf) & 1) ^ 1, abort_flag, prm.status, prm.wait_ns))
                 return false;
             tc_fence_after();
             if (st.s < n_a) {
@@ -784,7 +793,8 @@ __global__ void __launch_bounds__(kThreads, 1)
             while (alive && st.j < st.cnt)
                 alive = softmax_step<D, DEC, SAFE>(st, U, tmem, lane_off, c, c2, sready_s,
                                                    pready0 + 16u * st.s, empty0, wg_leader, it0,
-                                                   abort_flag, prm.status, prm.overflow);
+                                                   abort_flag, prm.status, prm.wait_ns,
+                                                   prm.overflow);
             if (alive)
                 alive = finish_stream<D, DEC>(st, U, prm, tmem, lane_off, r, sready_s, empty0,
                                               wg_leader, it0, abort_flag);
@@ -803,6 +813,27 @@ __global__ void __launch_bounds__(kThreads, 1)
 }
 
 // ------------------------------------------------------------------ host side
+
+// The test hook's setting (set_tc_test_fault): the launch it applies to (0: none; 1, 2: the
+// encode of call 1 or 2; 3: the decode), the ring item withheld in CTA 0 and the wait bound
+// of that launch.
+struct TestFault {
+    int kernel = 0;
+    int64_t ring_item = -1;
+    uint64_t wait_ns = kDefaultWaitNs;
+};
+std::mutex g_fault_mu;
+TestFault g_fault;
+
+void apply_fault(int kernel, TcParams& prm) {
+    std::lock_guard<std::mutex> lock(g_fault_mu);
+    prm.wait_ns = kDefaultWaitNs;
+    prm.withhold_it = -1;
+    if (g_fault.kernel != 0 && g_fault.kernel == kernel) {
+        prm.wait_ns = g_fault.wait_ns;
+        prm.withhold_it = g_fault.ring_item;
+    }
+}
 
 PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
     static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
@@ -878,6 +909,13 @@ uint32_t item_rows(int64_t D) {
 
 int64_t tc_encode_item_rows(int64_t D) { return item_rows<false>(D); }
 
+void set_tc_test_fault(int kernel, int64_t ring_item, uint64_t wait_ns) {
+    std::lock_guard<std::mutex> lock(g_fault_mu);
+    g_fault.kernel = kernel;
+    g_fault.ring_item = ring_item;
+    g_fault.wait_ns = wait_ns > 0 ? wait_ns : kDefaultWaitNs;
+}
+
 int64_t tc_group_rows(int64_t D) {
     (void)D;
     return NS * kTileRows;
@@ -916,6 +954,7 @@ cudaError_t tc_encode(const Plan& p, int call, const void* k, const void* v, con
     prm.n_units = p.BH * p.n_groups * p.nchunk;
     prm.status = (int*)(ws + p.off_status);
     prm.overflow = (int*)(ws + p.off_overflow) + (call - 1);
+    apply_fault(call, prm);
     return launch_d<false>(p.D, ma, mb, mc, prm, st);
 }
 
@@ -939,6 +978,7 @@ cudaError_t tc_decode(const Plan& p, const void* K, float scale, void* Y, char* 
     prm.n_units = p.BH * prm.n_tok_groups;
     prm.status = (int*)(ws + p.off_status);
     prm.overflow = (int*)(ws + p.off_overflow) + 2;
+    apply_fault(3, prm);
     return launch_d<true>(p.D, ma, mb, mc, prm, st);
 }
 

@@ -78,6 +78,8 @@ def load(path: str = None):
     lib.flarepp_route_fwd_profiled.restype = ctypes.c_int
     lib.flarepp_route_fwd_profiled.argtypes = [sp, vp, vp, vp, vp, vp, ctypes.c_float, vp, vp, sz,
                                                vp, ctypes.POINTER(ctypes.c_void_p), ctypes.c_int]
+    lib.flarepp_test_wait_fault.restype = None
+    lib.flarepp_test_wait_fault.argtypes = [ctypes.c_int, ctypes.c_int64, ctypes.c_uint64]
     lib.flarepp_route_fwd_noalloc.restype = ctypes.c_int
     lib.flarepp_route_fwd_noalloc.argtypes = [sp, vp, vp, vp, vp, vp, ctypes.c_float, vp, vp]
     lib.flarepp_flare_fwd.restype = ctypes.c_int
