@@ -351,7 +351,10 @@ FLAREPP_API flarepp_status flarepp_route_device_status(const flarepp_shape* shap
  * Test hook of the bounded waits; the paper has no counterpart. It lets a test make a wait
  * inside a tensor-core kernel run out without faulting or hanging the GPU.
  *   kernel: which launch of later calls it applies to: 1 or 2, the encode of call 1 or 2;
- *     3, the decode; 0 turns the hook off (the default).
+ *     3, the decode; 4 + p, pass p of flarepp_route_bwd's tensor-core passes (0: the route
+ *     pass of call 3, 1: of call 2, 2: of call 1, 3: the token pass of calls 2 and 3, 4: of
+ *     call 1, 5: the merged token pass of calls 2 and 3); 0 turns the hook off (the
+ *     default).
  *   ring_item: the index, in the order it is loaded, of an item of CTA 0's ring of K/V (or
  *     Q/Z) tiles that the kernel's load warp then never loads, so that the waits for it run
  *     out (-1: none).

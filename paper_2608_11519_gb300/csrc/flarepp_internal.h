@@ -179,6 +179,10 @@ cudaError_t tc_encode(const Plan& p, int call, const void* k, const void* v, con
 // chain kernel (1, 2: the encode of call 1 or 2; 3: the decode) wait at most wait_ns at each
 // barrier, and CTA 0's producer never loads ring item `ring_item` (so that a wait runs out).
 void set_tc_test_fault(int kernel, int64_t ring_item, uint64_t wait_ns);
+// The wait bound and withheld ring item of a launch of tensor-core kernel `kernel` (1, 2:
+// encode; 3: decode; 4 + p: backward pass p): the hook's setting for that kernel, else 2 s and
+// none.
+void test_fault_for(int kernel, uint64_t* wait_ns, int64_t* ring_item);
 // Rows per tensor-core work unit (route group of the encode, token group of the decode).
 int64_t tc_group_rows(int64_t D);
 int64_t tc_encode_item_rows(int64_t D);  // tokens per item of the tensor-core encode

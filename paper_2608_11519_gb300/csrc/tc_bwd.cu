@@ -52,7 +52,7 @@ using namespace tc;
 
 constexpr int kFirstSoftmaxWarp = 4;
 constexpr int kRows = 128;  // TMEM lanes per stream, MMA M
-constexpr uint64_t kWaitLimitNs = 2000000000ull;
+
 constexpr uint32_t kTmemCols = 512;
 
 enum Pass : int { kR3 = 0, kR2 = 1, kR1 = 2, kT23 = 3, kT1 = 4, kT23C = 5 };
@@ -141,6 +141,8 @@ struct BwdParams {
     const int* flags;   // when not null: only the units of (b, h) with flags[bh] == want run
     int want;
     int* status;
+    uint64_t wait_ns;     // bound of every wait (2 s unless the test hook is set)
+    int64_t withhold_it;  // test hook: ring item of CTA 0 the producer never loads (-1: none)
 };
 
 // Units of a (b, h) whose flag differs from the one this launch serves are skipped by every
@@ -239,14 +241,14 @@ __device__ __forceinline__ uint64_t ld_pair(const uint32_t* r, int k) {
 
 // Bounded wait on an mbarrier phase. Returns false when the kernel is aborting.
 __device__ __forceinline__ bool wait_bar(uint32_t bar, uint32_t parity, volatile int* abort_flag,
-                                         int* status) {
+                                         int* status, uint64_t limit) {
     if (mbar_try_wait(bar, parity)) return true;
     const uint64_t t0 = globaltimer_ns();
     for (uint32_t i = 1;; ++i) {
         if (mbar_try_wait(bar, parity)) return true;
         if ((i & 63u) == 0) {
             if (*abort_flag) return false;
-            if (globaltimer_ns() - t0 > kWaitLimitNs) {
+            if (globaltimer_ns() - t0 > limit) {
                 *abort_flag = 1;
                 atomicExch(status, (int)FLAREPP_ERR_TIMEOUT);
                 return false;
@@ -255,8 +257,8 @@ __device__ __forceinline__ bool wait_bar(uint32_t bar, uint32_t parity, volatile
     }
 }
 __device__ __forceinline__ bool warp_wait(uint32_t bar, uint32_t parity, volatile int* abort_flag,
-                                          int* status) {
-    const bool got = wait_bar(bar, parity, abort_flag, status);
+                                          int* status, uint64_t limit) {
+    const bool got = wait_bar(bar, parity, abort_flag, status, limit);
     return __all_sync(0xffffffffu, got);
 }
 
@@ -427,6 +429,7 @@ __global__ void __launch_bounds__(BCfg<D, PASS>::kThreads, 1)
     if (warp == C::kProdWarp) {
         // ------------------------------------------------------------ TMA producer
         uint32_t it = 0, ua = 0, a_issued = 0;
+        int64_t withheld = -1;
         bool ok = true;
         for (int64_t u = blockIdx.x; u < prm.n_units && ok; u += gridDim.x) {
             const BUnit U = bwd_unit<D, PASS>(prm, u);
@@ -437,7 +440,7 @@ __global__ void __launch_bounds__(BCfg<D, PASS>::kThreads, 1)
             const uint32_t uc = ua++;
             const int ab = uc % C::kABuf;
             if (uc >= (uint32_t)C::kABuf &&
-                !warp_wait(afree0 + 8u * ab, ((uc / C::kABuf) - 1) & 1, abort_flag, prm.status)) {
+                !warp_wait(afree0 + 8u * ab, ((uc / C::kABuf) - 1) & 1, abort_flag, prm.status, prm.wait_ns)) {
                 ok = false;
                 break;
             }
@@ -463,9 +466,13 @@ __global__ void __launch_bounds__(BCfg<D, PASS>::kThreads, 1)
                 const int st = it % C::kStages;
                 if (it >= (uint32_t)C::kStages &&
                     !warp_wait(empty0 + 8u * st, ((it / C::kStages) - 1) & 1, abort_flag,
-                               prm.status)) {
+                               prm.status, prm.wait_ns)) {
                     ok = false;
                     break;
+                }
+                if (blockIdx.x == 0 && (int64_t)it == prm.withhold_it) {
+                    withheld = it;  // never loaded: the waits of its consumers run out
+                    continue;
                 }
                 const int64_t row = U.item0 + (int64_t)i * C::kItem;
                 if (elect_one()) {
@@ -505,14 +512,15 @@ __global__ void __launch_bounds__(BCfg<D, PASS>::kThreads, 1)
             const uint64_t t0 = globaltimer_ns();
             for (int st = 0; st < C::kStages && (uint32_t)st < it; ++st) {
                 const uint32_t x = it - 1 - ((it - 1 - st) % C::kStages);
-                while (!mbar_try_wait(full0 + 8u * st, (x / C::kStages) & 1) &&
-                       globaltimer_ns() - t0 < kWaitLimitNs) {
+                while ((int64_t)x != withheld &&
+                       !mbar_try_wait(full0 + 8u * st, (x / C::kStages) & 1) &&
+                       globaltimer_ns() - t0 < prm.wait_ns) {
                 }
             }
             for (int b = 0; b < C::kABuf && (uint32_t)b < a_issued; ++b) {
                 const uint32_t x = a_issued - 1 - ((a_issued - 1 - b) % C::kABuf);
                 while (!mbar_try_wait(afull0 + 8u * b, (x / C::kABuf) & 1) &&
-                       globaltimer_ns() - t0 < kWaitLimitNs) {
+                       globaltimer_ns() - t0 < prm.wait_ns) {
                 }
             }
         }
@@ -526,7 +534,7 @@ __global__ void __launch_bounds__(BCfg<D, PASS>::kThreads, 1)
         uint32_t it = 0, ua = 0, pj = 0, nu = 0, ar = 0;
         bool ok = true;
         auto wait = [&](uint32_t bar, uint32_t parity) {
-            return warp_wait(bar, parity, abort_flag, prm.status);
+            return warp_wait(bar, parity, abort_flag, prm.status, prm.wait_ns);
         };
         const uint32_t t0 = tmem + s * C::kColStream;
         const uint32_t acc = t0 + C::kNA * C::kItem;
@@ -672,7 +680,7 @@ __global__ void __launch_bounds__(BCfg<D, PASS>::kThreads, 1)
         __syncwarp();
         const uint64_t tw = globaltimer_ns();
         while (!__all_sync(0xffffffffu, mbar_try_wait(fin0 + 8u * s, 0)) &&
-               globaltimer_ns() - tw < kWaitLimitNs) {
+               globaltimer_ns() - tw < prm.wait_ns) {
         }
     } else if (warp >= kFirstSoftmaxWarp && warp < kFirstSoftmaxWarp + 4 * NS) {
         // ------------------------------------------------------------ softmax warpgroups
@@ -689,7 +697,7 @@ __global__ void __launch_bounds__(BCfg<D, PASS>::kThreads, 1)
         // the shared-memory buffer; an idle stream only releases it.
         auto copy_a = [&](const BUnit& V, uint32_t uv) -> bool {
             const int ab = uv % C::kABuf;
-            if (!warp_wait(afull0 + 8u * ab, (uv / C::kABuf) & 1, abort_flag, prm.status))
+            if (!warp_wait(afull0 + 8u * ab, (uv / C::kABuf) & 1, abort_flag, prm.status, prm.wait_ns))
                 return false;
             if (s < V.n_act) {
                 const int64_t row = V.row0 + s * kRows + r;
@@ -763,7 +771,7 @@ __global__ void __launch_bounds__(BCfg<D, PASS>::kThreads, 1)
             const uint64_t u2 = pack_f32x2(uu, uu);
             for (int i = 0; i < U.n_items; ++i, ++it) {
                 const int st = it % C::kStages;
-                if (!warp_wait(sready0 + 8u * s, sj & 1, abort_flag, prm.status)) {
+                if (!warp_wait(sready0 + 8u * s, sj & 1, abort_flag, prm.status, prm.wait_ns)) {
                     ok = false;
                     break;
                 }
@@ -771,7 +779,7 @@ __global__ void __launch_bounds__(BCfg<D, PASS>::kThreads, 1)
                 // S of item i complete: every product of item i - 1 is, so its stage is free
                 if (i > 0 && leader) mbar_arrive(empty0 + 8u * ((it - 1) % C::kStages));
                 if (C::kColStats &&
-                    !warp_wait(full0 + 8u * st, (it / C::kStages) & 1, abort_flag, prm.status)) {
+                    !warp_wait(full0 + 8u * st, (it / C::kStages) & 1, abort_flag, prm.status, prm.wait_ns)) {
                     ok = false;
                     break;
                 }
@@ -806,7 +814,7 @@ __global__ void __launch_bounds__(BCfg<D, PASS>::kThreads, 1)
                 if (!ok) break;
             }
             // epilogue: the unit's accumulators
-            if (!warp_wait(accdone0 + 8u * s, na & 1, abort_flag, prm.status)) {
+            if (!warp_wait(accdone0 + 8u * s, na & 1, abort_flag, prm.status, prm.wait_ns)) {
                 ok = false;
                 break;
             }
@@ -989,6 +997,7 @@ cudaError_t tc_bwd_pass(const Plan& p, const BwdPlan& bp, int pass, const TcBwdO
     prm.flags = o.flags;
     prm.want = o.want;
     prm.status = status;
+    test_fault_for(4 + pass, &prm.wait_ns, &prm.withhold_it);
     switch (pass) {
         case kR3: return launch_d<kR3>(srcs, p, prm, st);
         case kR2: return launch_d<kR2>(srcs, p, prm, st);

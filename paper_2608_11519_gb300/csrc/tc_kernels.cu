@@ -909,6 +909,16 @@ uint32_t item_rows(int64_t D) {
 
 int64_t tc_encode_item_rows(int64_t D) { return item_rows<false>(D); }
 
+void test_fault_for(int kernel, uint64_t* wait_ns, int64_t* ring_item) {
+    std::lock_guard<std::mutex> lock(g_fault_mu);
+    *wait_ns = kDefaultWaitNs;
+    *ring_item = -1;
+    if (g_fault.kernel != 0 && g_fault.kernel == kernel) {
+        *wait_ns = g_fault.wait_ns;
+        *ring_item = g_fault.ring_item;
+    }
+}
+
 void set_tc_test_fault(int kernel, int64_t ring_item, uint64_t wait_ns) {
     std::lock_guard<std::mutex> lock(g_fault_mu);
     g_fault.kernel = kernel;
