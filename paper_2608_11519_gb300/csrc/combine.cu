@@ -4,6 +4,7 @@
 #include <math.h>
 
 #include "flarepp_internal.h"
+#include "tc_ptx.cuh"
 
 namespace flarepp {
 namespace {
@@ -44,6 +45,8 @@ __global__ void combine_kernel(const float* __restrict__ pmax, const float* __re
                                __nv_bfloat16* __restrict__ outop, float op_sign,
                                float* __restrict__ lse) {
     constexpr int PER = (D + 31) / 32;
+    tc::pdl_trigger();
+    tc::pdl_wait();  // the partials and the outputs belong to the kernels around this one
     const int lane = threadIdx.x & 31;
     const int64_t row = (int64_t)blockIdx.x * (blockDim.x / 32) + threadIdx.x / 32;
     if (row >= rows) return;
@@ -132,22 +135,16 @@ cudaError_t combine(const Plan& p, int call, char* ws, bool negate, cudaStream_t
     // slots per row at most: nchunk x sub_per_chunk
     const bool few = p.nchunk * p.sub_per_chunk <= 4;
 #define FLAREPP_COMBINE(DD)                                                                    \
-    if (few)                                                                                   \
-        combine_kernel<DD, 4><<<(unsigned)blocks, warps * 32, 0, st>>>(                        \
-            pmax, psum, pacc, rows, p.M, p.nchunk, p.sub_per_chunk, p.tc_group, out32, outop,  \
-            sign, lse);                                                                        \
-    else                                                                                       \
-        combine_kernel<DD, 32><<<(unsigned)blocks, warps * 32, 0, st>>>(                       \
-            pmax, psum, pacc, rows, p.M, p.nchunk, p.sub_per_chunk, p.tc_group, out32, outop,  \
-            sign, lse);
+    return launch_pdl(few ? combine_kernel<DD, 4> : combine_kernel<DD, 32>,                   \
+                      dim3((unsigned)blocks), dim3(warps * 32), 0, st, pmax, psum, pacc, rows, \
+                      p.M, p.nchunk, p.sub_per_chunk, p.tc_group, out32, outop, sign, lse);
     switch (p.D) {
-        case 16: FLAREPP_COMBINE(16) break;
-        case 32: FLAREPP_COMBINE(32) break;
-        case 64: FLAREPP_COMBINE(64) break;
-        default: return cudaErrorInvalidValue;
+        case 16: FLAREPP_COMBINE(16)
+        case 32: FLAREPP_COMBINE(32)
+        case 64: FLAREPP_COMBINE(64)
     }
 #undef FLAREPP_COMBINE
-    return cudaGetLastError();
+    return cudaErrorInvalidValue;
 }
 
 cudaError_t negate_bf16(const void* src, void* dst, int64_t n, cudaStream_t st) {

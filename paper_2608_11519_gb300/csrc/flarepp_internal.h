@@ -41,6 +41,25 @@ struct Plan {
     size_t total;
 };
 
+// Launch `kernel` on `st` with programmatic stream serialization: its blocks may start while
+// the kernel before it on the stream finishes, and wait for it at their pdl_wait (the kernels
+// of the chain call it before touching memory that the previous kernel writes or reads).
+template <typename... Params, typename... Args>
+cudaError_t launch_pdl(void (*kernel)(Params...), dim3 grid, dim3 block, size_t smem,
+                       cudaStream_t st, Args... args) {
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = grid;
+    cfg.blockDim = block;
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = st;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, kernel, args...);
+}
+
 // Raise the dynamic shared-memory limit of kernel `func` to `bytes` on the current device,
 // once per (kernel, device): the attribute is per device, so a process that launches on
 // several GPUs sets it on each (flarepp_api.cu).

@@ -501,9 +501,11 @@ __global__ void __launch_bounds__(kThreads, 1)
     tc_chain_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
                     const __grid_constant__ CUtensorMap tmC, const TcParams prm) {
     using C = Cfg<D, DEC>;
+    pdl_trigger();
     if constexpr (SAFE) {
         // the safe kernel recomputes the launch only when the fast one overflowed
         __shared__ int run;
+        pdl_wait();
         if (threadIdx.x == 0) run = *reinterpret_cast<volatile int*>(prm.overflow);
         __syncthreads();
         if (!run) return;
@@ -561,6 +563,8 @@ __global__ void __launch_bounds__(kThreads, 1)
     __syncthreads();
     tc_fence_after();
     const uint32_t tmem = *tmem_slot;
+    // every global access below may depend on the kernel before this one
+    pdl_wait();
 
     if (warp < kProducerWarp) {
         // ------------------------------------------------------------ MMA warps
@@ -883,9 +887,12 @@ cudaError_t launch(const CUtensorMap& a, const CUtensorMap& b, const CUtensorMap
     cudaGetDevice(&dev);
     cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
     const int64_t grid = prm.n_units < sms ? prm.n_units : sms;
-    tc_chain_kernel<D, DEC, false><<<(unsigned)grid, kThreads, Cf::kSmem, st>>>(a, b, c, prm);
-    tc_chain_kernel<D, DEC, true><<<(unsigned)grid, kThreads, Cf::kSmem, st>>>(a, b, c, prm);
-    return cudaGetLastError();
+    e = launch_pdl(tc_chain_kernel<D, DEC, false>, dim3((unsigned)grid), dim3(kThreads),
+                   Cf::kSmem, st, a, b, c, prm);
+    if (e == cudaSuccess)
+        e = launch_pdl(tc_chain_kernel<D, DEC, true>, dim3((unsigned)grid), dim3(kThreads),
+                       Cf::kSmem, st, a, b, c, prm);
+    return e;
 }
 
 template <bool DEC>
