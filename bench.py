@@ -369,7 +369,7 @@ def run_reference(args, w):
             "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
             "ms_per_step": dt * 1e3, "higher_is_better": True, "scaling": "weak",
             "vs_baseline": None, "dtype": "f64", "data": "synthetic",
-            "config": arm_config(w, args.variant, world),
+            "config": arm_config(w, args.variant, world, args.l2),
             "cpu_baseline": {"value": value, "unit": UNIT, "cores": oracle.max_threads(),
                              "kind": "oracle", "sample": sample},
             "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0,
@@ -383,7 +383,33 @@ def run_reference(args, w):
 FLARE_METRIC = "routed tokens·heads/sec for the 2-call FLARE layer (fixed queries); % of roofline"
 
 
-def arm_config(w, variant, world):
+L2_BYTES = 129e6
+FLUSH_BYTES = 256 << 20  # twice the L2
+
+
+def chain_inputs_fit_l2(w, variant):
+    """Whether the chain's streamed tensors (K~, V~, K, V and Y; K, V and Y when shared) stay
+    within twice the L2, so that a warm L2 could hold a large share of them across steps."""
+    n = 3 if variant == "shared" else 5
+    return n * w.B * w.H * w.N * w.D * w.elt_bytes <= 2 * L2_BYTES
+
+
+def l2_mode(mode, w, variant):
+    """'flush' or 'warm' for the chain variants: `auto` flushes exactly when the streamed
+    tensors are near the L2's size, where leftover lines would flatter a step."""
+    if mode == "auto":
+        return "flush" if chain_inputs_fit_l2(w, variant) else "warm"
+    return mode
+
+
+def l2_flush_buffer(mode, w, variant, dev):
+    """A buffer larger than the L2 that each timed step overwrites first, or None."""
+    if l2_mode(mode, w, variant) != "flush":
+        return None
+    return torch.empty(FLUSH_BYTES, dtype=torch.uint8, device=dev)
+
+
+def arm_config(w, variant, world, l2="auto"):
     """The `config` of a bench line; both arms of one variant print the same one."""
     cfg = {"workload": w.name, "variant": variant, "B": w.B, "H": w.H, "N": w.N, "M": w.M,
            "D": w.D}
@@ -391,7 +417,12 @@ def arm_config(w, variant, world):
     big = "inputs larger than L2 (no flush)"
     if variant in ("flarepp", "shared"):
         cfg["keys"] = f"clustered, {w.n_centres} centres" if w.n_centres else "iid"
-        cfg["l2"] = big if 5 * tok * w.D * w.elt_bytes > 2 * 129e6 else "inputs near L2 size"
+        if l2_mode(l2, w, variant) == "flush":
+            cfg["l2"] = "flushed before each step (256 MiB written between the step's events)"
+        elif chain_inputs_fit_l2(w, variant):
+            cfg["l2"] = "warm: no flush, inputs near L2 size"
+        else:
+            cfg["l2"] = big
     elif variant == "flare":
         cfg["queries"] = "the workload's seeds, as learned queries"
         cfg["l2"] = big if 3 * tok * w.D * w.elt_bytes > 2 * 129e6 else "inputs near L2 size"
@@ -845,22 +876,35 @@ def run_ours(args, w):
         flarepp.route_fwd(*args_, scale=w.scale, Y=Y, workspace=ws, stream=stream)
     torch.cuda.synchronize(dev)
 
-    # the timed region: whole calls of the public entry, no events inside a step
+    # the timed region: whole calls of the public entry, no events inside a step; with the L2
+    # flushed, each step is bracketed by its own events and the flush runs between them
+    flush = l2_flush_buffer(args.l2, w, args.variant, dev)
     clocks = ClockSampler()
     if rank == 0:
         clocks.start(dev.index)
-    t_start = torch.cuda.Event(enable_timing=True)
-    t_end = torch.cuda.Event(enable_timing=True)
     barrier(world)
     torch.cuda.synchronize(dev)
-    t_start.record(stream)
-    for i in range(args.steps):
-        flarepp.route_fwd(*args_, scale=w.scale, Y=Y, workspace=ws, stream=stream)
-    t_end.record(stream)
-    torch.cuda.synchronize(dev)
+    if flush is None:
+        t_start = torch.cuda.Event(enable_timing=True)
+        t_end = torch.cuda.Event(enable_timing=True)
+        t_start.record(stream)
+        for i in range(args.steps):
+            flarepp.route_fwd(*args_, scale=w.scale, Y=Y, workspace=ws, stream=stream)
+        t_end.record(stream)
+        torch.cuda.synchronize(dev)
+        total_ms = t_start.elapsed_time(t_end)
+    else:
+        evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+               for _ in range(args.steps)]
+        for i in range(args.steps):
+            flush.fill_(i & 0x7F)
+            evs[i][0].record(stream)
+            flarepp.route_fwd(*args_, scale=w.scale, Y=Y, workspace=ws, stream=stream)
+            evs[i][1].record(stream)
+        torch.cuda.synchronize(dev)
+        total_ms = sum(a.elapsed_time(b) for a, b in evs)
     barrier(world)
     clk = clocks.stop(dev.index) if rank == 0 else None
-    total_ms = t_start.elapsed_time(t_end)
     total_ms = max_over_ranks(total_ms, world)
     ms_per_step = total_ms / args.steps
 
@@ -869,6 +913,8 @@ def run_ours(args, w):
     n_prof = max(1, min(args.steps, 20))
     ev_sets = [flarepp.StageEvents(stream) for _ in range(n_prof)]
     for i in range(n_prof):
+        if flush is not None:
+            flush.fill_(i & 0x7F)
         flarepp.route_fwd_profiled(*args_, ev_sets[i], scale=w.scale, Y=Y, workspace=ws)
     torch.cuda.synchronize(dev)
     stage_ms = {s: 0.0 for s in flarepp.STAGES}
@@ -958,7 +1004,7 @@ def run_ours(args, w):
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms_per_step,
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
             "dtype": "bf16" if w.dtype == "bf16" else "f32", "data": "synthetic",
-            "config": arm_config(w, args.variant, world),
+            "config": arm_config(w, args.variant, world, args.l2),
             "roofline": roof, "chain_roofline": chain, "stage_ms": stage_ms,
             "cpu_baseline": cpu, "e2e": e2e, "clocks": clk,
             "gpu_launches": chain_fwd_launches(w) * args.steps,
@@ -985,6 +1031,9 @@ def main():
                          "tied to K, V; flare: FLARE with fixed learned queries; train: the "
                          "chain's training forward and backward; mixer(_shared): the whole "
                          "FLARE++ mixer layer with four (two) projections")
+    ap.add_argument("--l2", choices=("auto", "flush", "warm"), default="auto",
+                    help="chain variants: flush the L2 before each timed step, or not; auto "
+                         "flushes when the streamed tensors are near the L2's size")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--e2e-steps", type=int, default=10)
     ap.add_argument("--no-cpu-baseline", action="store_true")

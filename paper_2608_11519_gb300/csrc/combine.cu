@@ -15,99 +15,99 @@ __device__ __forceinline__ float fast_exp2(float x) {
     return y;
 }
 
-// Partial slots a route's chunks use: 1 on the CUDA-core path. On the tensor-core path a
-// work unit covers a group of `group` routes in tiles of 128; a unit with n_a route tiles
-// (rounded to 1, 2 or 4) splits each chunk over (group / 128) / n_a token-parity streams.
-__device__ __forceinline__ int slots_of_route(int64_t M, int64_t m, int64_t sub_per_chunk,
-                                              int64_t group) {
-    if (sub_per_chunk == 1) return 1;
-    const int64_t ns = group / 128;
-    const int64_t g = m / group;
-    const int64_t rem = M - g * group;
-    const int64_t tiles = rem >= group ? ns : (rem + 127) / 128;
-    const int64_t na = tiles <= 1 ? 1 : (tiles <= 2 ? 2 : 4);
-    return (int)(ns / na);
+// log2 of the partial slots a route's chunks use: 1 slot on the CUDA-core path. On the
+// tensor-core path a work unit covers a group of 2^group_log2 routes in tiles of 128; a unit
+// with n_a route tiles (rounded to 1, 2 or 4) splits each chunk over (group / 128) / n_a
+// token-parity streams.
+__device__ __forceinline__ int slots_log2(int M, int m, int sub_per_chunk, int group_log2) {
+    if (sub_per_chunk == 1) return 0;
+    const int ns_log2 = group_log2 - 7;
+    const int g0 = (m >> group_log2) << group_log2;
+    const int rem = M - g0;
+    const int tiles = rem >= (1 << group_log2) ? (1 << ns_log2) : (rem + 127) >> 7;
+    const int na_log2 = tiles <= 1 ? 0 : (tiles <= 2 ? 1 : 2);
+    return ns_log2 - na_log2;
 }
 
-// One warp per (bh, m): merge the partial slots (App. A.3):
+// Merge of the partial slots of one row (App. A.3):
 //   g = max_r mx_r; w_r = 2^(mx_r - g); out = sum_r w_r acc_r / sum_r w_r l_r;
 //   the row's base-2 log-normaliser is g + log2(sum_r w_r l_r).
-// The slots are taken KB (4 or 32) at a time, and every load of a block is issued at once:
-// the lanes load one slot's maximum and sum each, and (lanes as channels) the values of all
-// KB slots. The blocks are merged online with a running maximum, so a row costs one round of
-// memory latency per KB slots (the merge is the same in every run: deterministic). KB = 4
-// serves rows of at most four slots with few instructions.
+// T = D / 4 threads per row, each with four channels (one 16-byte load per slot); a block of
+// 256 threads covers 256 / T rows of one (b, h), which blockIdx.y + gridDim.y * blockIdx.z
+// names. The slots are taken KB at a time, all loads of a block issued together, and merged
+// online in slot order (chunk by chunk, parts in order): the same merge in every run.
 template <int D, int KB>
-__global__ void combine_kernel(const float* __restrict__ pmax, const float* __restrict__ psum,
-                               const float* __restrict__ pacc, int64_t rows, int64_t M,
-                               int64_t nchunk, int64_t sub_per_chunk, int64_t group,
-                               float* __restrict__ out32,
-                               __nv_bfloat16* __restrict__ outop, float op_sign,
-                               float* __restrict__ lse) {
-    constexpr int PER = (D + 31) / 32;
+__global__ void __launch_bounds__(256)
+    combine_kernel(const float* __restrict__ pmax, const float* __restrict__ psum,
+                   const float* __restrict__ pacc, int64_t BH, int M, int nchunk,
+                   int sub_per_chunk, int group_log2, float* __restrict__ out32,
+                   __nv_bfloat16* __restrict__ outop, float op_sign, float* __restrict__ lse) {
+    constexpr int T = D / 4;
+    constexpr int kRowsPerBlock = 256 / T;
     tc::pdl_trigger();
     tc::pdl_wait();  // the partials and the outputs belong to the kernels around this one
-    const int lane = threadIdx.x & 31;
-    const int64_t row = (int64_t)blockIdx.x * (blockDim.x / 32) + threadIdx.x / 32;
-    if (row >= rows) return;
-    const int64_t bh = row / M, m = row % M;
-    const int used = slots_of_route(M, m, sub_per_chunk, group);
-    const int64_t nslot = nchunk * sub_per_chunk;
-    const int64_t n = nchunk * used;  // the row's slots, s -> chunk s / used, part s % used
-    auto slot_row = [&](int64_t s) {
-        return (bh * nslot + (s / used) * sub_per_chunk + s % used) * M + m;
-    };
-    float g = -INFINITY, a = 0.f, u[PER];
-#pragma unroll
-    for (int i = 0; i < PER; ++i) u[i] = 0.f;
-    for (int64_t s0 = 0; s0 < n; s0 += KB) {
-        const int cnt = (int)min((int64_t)KB, n - s0);
-        const bool in = lane < cnt;
-        const int64_t rl = in ? slot_row(s0 + lane) : 0;
-        const float mx = in ? pmax[rl] : -INFINITY;
-        const float ps = in ? psum[rl] : 0.f;
-        float v[KB][PER];
+    const int64_t bh = (int64_t)blockIdx.z * gridDim.y + blockIdx.y;
+    const int m = blockIdx.x * kRowsPerBlock + (int)(threadIdx.x / T);
+    const int q = (int)(threadIdx.x % T);
+    if (bh >= BH || m >= M) return;
+    const int ul = slots_log2(M, m, sub_per_chunk, group_log2);
+    const int n = nchunk << ul;  // slot s: chunk s >> ul, part s & (2^ul - 1)
+    const int64_t row = bh * M + m;
+    // partial row of slot s: (bh * nchunk * sub + (s >> ul) * sub + (s & mask)) * M + m
+    const int64_t base = bh * (int64_t)nchunk * sub_per_chunk * M + m;
+    const int mask = (1 << ul) - 1;
+    float g = -INFINITY, a = 0.f;
+    float4 u = make_float4(0.f, 0.f, 0.f, 0.f);
+    for (int s0 = 0; s0 < n; s0 += KB) {
+        float mx[KB], ps[KB];
+        float4 v[KB];
 #pragma unroll
         for (int j = 0; j < KB; ++j) {
-            const int64_t rj = j < cnt ? slot_row(s0 + j) : 0;
-#pragma unroll
-            for (int i = 0; i < PER; ++i) {
-                const int d = lane + 32 * i;
-                v[j][i] = (j < cnt && d < D) ? pacc[rj * D + d] : 0.f;
+            const int s = s0 + j;
+            mx[j] = -INFINITY;
+            ps[j] = 0.f;
+            v[j] = make_float4(0.f, 0.f, 0.f, 0.f);
+            if (s < n) {
+                const int64_t r =
+                    base + ((int64_t)(s >> ul) * sub_per_chunk + (s & mask)) * (int64_t)M;
+                mx[j] = __ldg(pmax + r);
+                ps[j] = __ldg(psum + r);
+                v[j] = __ldg(reinterpret_cast<const float4*>(pacc + r * D) + q);
             }
         }
-        float gb = mx;
+        float gb = mx[0];
 #pragma unroll
-        for (int off = 16; off > 0; off >>= 1) gb = fmaxf(gb, __shfl_xor_sync(0xffffffffu, gb, off));
+        for (int j = 1; j < KB; ++j) gb = fmaxf(gb, mx[j]);
         if (gb == -INFINITY) continue;  // every slot of the block is empty
         const float gn = fmaxf(g, gb);
         const float sc = fast_exp2(g - gn);  // 0 while g is -inf
         a *= sc;
-#pragma unroll
-        for (int i = 0; i < PER; ++i) u[i] *= sc;
-        const float w = in ? fast_exp2(mx - gn) : 0.f;
-        float aw = w * ps;
-#pragma unroll
-        for (int off = 16; off > 0; off >>= 1) aw += __shfl_xor_sync(0xffffffffu, aw, off);
-        a += aw;
+        u.x *= sc;
+        u.y *= sc;
+        u.z *= sc;
+        u.w *= sc;
 #pragma unroll
         for (int j = 0; j < KB; ++j) {
-            const float wj = __shfl_sync(0xffffffffu, w, j);
-#pragma unroll
-            for (int i = 0; i < PER; ++i) u[i] = fmaf(wj, v[j][i], u[i]);
+            const float w = fast_exp2(mx[j] - gn);  // 0 for an empty slot
+            a = fmaf(w, ps[j], a);
+            u.x = fmaf(w, v[j].x, u.x);
+            u.y = fmaf(w, v[j].y, u.y);
+            u.z = fmaf(w, v[j].z, u.z);
+            u.w = fmaf(w, v[j].w, u.w);
         }
         g = gn;
     }
     const float inv = a > 0.f ? 1.f / a : 0.f;
-    if (lse && lane == 0) lse[row] = a > 0.f ? g + log2f(a) : -INFINITY;
-#pragma unroll
-    for (int i = 0; i < PER; ++i) {
-        const int d = lane + 32 * i;
-        if (d < D) {
-            const float val = u[i] * inv;
-            out32[row * D + d] = val;
-            if (outop) outop[row * D + d] = __float2bfloat16_rn(op_sign * val);
-        }
+    if (lse && q == 0) lse[row] = a > 0.f ? g + log2f(a) : -INFINITY;
+    const float4 o = make_float4(u.x * inv, u.y * inv, u.z * inv, u.w * inv);
+    reinterpret_cast<float4*>(out32 + row * D)[q] = o;
+    if (outop) {
+        const __nv_bfloat162 lo = __floats2bfloat162_rn(op_sign * o.x, op_sign * o.y);
+        const __nv_bfloat162 hi = __floats2bfloat162_rn(op_sign * o.z, op_sign * o.w);
+        uint2 pk;
+        pk.x = *reinterpret_cast<const uint32_t*>(&lo);
+        pk.y = *reinterpret_cast<const uint32_t*>(&hi);
+        reinterpret_cast<uint2*>(outop + row * D)[q] = pk;
     }
 }
 
@@ -122,9 +122,6 @@ __global__ void negate_bf16_kernel(const __nv_bfloat16* __restrict__ src,
 
 cudaError_t combine(const Plan& p, int call, char* ws, bool negate, cudaStream_t st,
                     float* lse) {
-    const int64_t rows = p.BH * p.M;
-    const int warps = 8;
-    const int64_t blocks = (rows + warps - 1) / warps;
     float* out32 = (float*)(ws + (call == 1 ? p.off_q32 : p.off_z32));
     __nv_bfloat16* outop = nullptr;
     if (p.path == kPathTc) outop = (__nv_bfloat16*)(ws + (call == 1 ? p.off_qop : p.off_zop));
@@ -132,12 +129,27 @@ cudaError_t combine(const Plan& p, int call, char* ws, bool negate, cudaStream_t
     const float* psum = (const float*)(ws + p.off_psum);
     const float* pacc = (const float*)(ws + p.off_pacc);
     const float sign = negate ? -1.f : 1.f;
+    // the group of routes a tensor-core unit covers is a power of two (tile rows x streams)
+    int group_log2 = 0;
+    if (p.sub_per_chunk > 1) {
+        while ((int64_t(1) << group_log2) < p.tc_group) ++group_log2;
+        if ((int64_t(1) << group_log2) != p.tc_group || group_log2 < 7) return cudaErrorInvalidValue;
+    }
+    if (p.nchunk * p.sub_per_chunk > INT32_MAX || p.M > INT32_MAX) return cudaErrorInvalidValue;
+    // (b, h) over gridDim.y x gridDim.z (each at most 65535)
+    const int64_t gy = p.BH < 65535 ? p.BH : 65535;
+    const int64_t gz = (p.BH + gy - 1) / gy;
+    if (gz > 65535) return cudaErrorInvalidValue;
     // slots per row at most: nchunk x sub_per_chunk
     const bool few = p.nchunk * p.sub_per_chunk <= 4;
-#define FLAREPP_COMBINE(DD)                                                                    \
-    return launch_pdl(few ? combine_kernel<DD, 4> : combine_kernel<DD, 32>,                   \
-                      dim3((unsigned)blocks), dim3(warps * 32), 0, st, pmax, psum, pacc, rows, \
-                      p.M, p.nchunk, p.sub_per_chunk, p.tc_group, out32, outop, sign, lse);
+#define FLAREPP_COMBINE(DD)                                                                  \
+    {                                                                                        \
+        const int64_t gx = (p.M + (256 / (DD / 4)) - 1) / (256 / (DD / 4));                 \
+        return launch_pdl(few ? combine_kernel<DD, 4> : combine_kernel<DD, 8>,               \
+                          dim3((unsigned)gx, (unsigned)gy, (unsigned)gz), dim3(256), 0, st,  \
+                          pmax, psum, pacc, p.BH, (int)p.M, (int)p.nchunk,                   \
+                          (int)p.sub_per_chunk, group_log2, out32, outop, sign, lse);        \
+    }
     switch (p.D) {
         case 16: FLAREPP_COMBINE(16)
         case 32: FLAREPP_COMBINE(32)

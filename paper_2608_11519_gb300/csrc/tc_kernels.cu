@@ -4,33 +4,38 @@
 // (Sec. 3.2, eqs. flarepp_dynamic_query and flarepp_mixer):
 //
 //   encode (calls 1, 2): TMEM lanes are routes. A group of NS route tiles (128 routes
-//     each; the A operand: seeds or Q) meets a stream of 64-token items (K and V tiles)
-//     from one chunk of the sequence. Each route row keeps an online softmax over tokens,
-//     and the CTA writes per-chunk partials (reference max, sum, unnormalised value sum)
+//     each; the A operand: seeds or Q) meets a stream of items of kItem tokens (K and V
+//     tiles) from one chunk of the sequence. Each route row keeps an online softmax over
+//     tokens, and the CTA writes per-chunk partials (reference, sum, unnormalised value sum)
 //     for the log-sum-exp merge of App. A.3.
 //   decode (call 3): TMEM lanes are tokens. A group of NS token tiles (K, 128 tokens each)
-//     meets a stream of 64-route items (Q and Z tiles). Each token row keeps an online
-//     softmax over routes and writes its normalised row of Y.
+//     meets a stream of items of kItem routes (Q and Z tiles). Each token row keeps an
+//     online softmax over routes and writes its normalised row of Y.
 //
 // Work is cut into four TMEM "streams". Stream s owns one score buffer of 128 x kItem fp32
-// (kItem = 64 tokens or routes, 32 for D = 64; S is rewritten in place as bf16 P, the A
-// operand of the PV product) and a 128 x D fp32 accumulator O, and reads one resident A
-// tile kept in TMEM, so that S = A * B^T is a TMEM x SMEM product. With two TMEM copies of
-// the A tiles (D <= 32) the softmax copies the next unit's tiles while it works on the
-// current unit, so a unit boundary does not drain the pipeline. Roles (20 warps):
-//   warps 0..3    one MMA warp per stream: for item j, the PV of item j-B and the S of
-//                 item j, then one commit (a commit stalls only the warp that issues it);
-//                 warp 0 also issues the TMA loads (A tiles, unswizzled; the item ring,
-//                 swizzled K/V or Q/Z) from a non-blocking poll between its own waits
-//   warps 4..19   four softmax warpgroups; warpgroup s serves stream s and copies its A tile
+// (S is rewritten in place as bf16 P, the A operand of the PV product) and a 128 x D fp32
+// accumulator O, and reads one resident A tile kept in TMEM, so that S = A * B^T is a
+// TMEM x SMEM product. With two TMEM copies of the A tiles (the decode, D <= 32) the softmax
+// copies the next unit's tiles while it works on the current unit, so a unit boundary does
+// not drain the pipeline. Roles (24 warps, a register split gives warpgroups 0 and 1 40
+// registers per thread and the four softmax warpgroups 96):
+//   warps 0..3    one MMA warp per stream: for item j, the PV of item j-1 and the S of
+//                 item j, then one commit, all issued from one elected lane (a commit
+//                 stalls only the warp that issues it)
+//   warp 4        the TMA producer (A tiles, unswizzled; the item ring, swizzled K/V or
+//                 Q/Z), with blocking waits; warps 5..7 only take part in the split
+//   warps 8..23   four softmax warpgroups; warpgroup s serves stream s and copies its A tile
 //                 from smem into TMEM (four warps per SMSP hide each other's latencies)
-// The softmax keeps a reference max, set on a stream's first item (the item's exact maximum
-// in the encode, its first score in the decode) and recomputed exactly only when an item's
-// probabilities sum past 2^48 (values stay far inside the fp32 and bf16 ranges); otherwise
-// P = 2^(c S - m) with the old reference.
-// Every wait is bounded (2 s of %globaltimer): on expiry the kernel records
-// FLAREPP_ERR_TIMEOUT in the status word, every role leaves its loops, the TMA issuer waits
-// for its copies in flight, and TMEM is freed.
+// Each launch is a pair of kernels on the stream. The fast kernel keeps, per row, the first
+// score of the unit as its reference m (any score of the row is a valid reference: it alone
+// adds 2^0 to the sum) and computes P = 2^(c S - m) with no maximum pass, storing P chunk by
+// chunk. An item whose probabilities sum past 2^48 (a score far above the reference) cannot
+// be repaired there: the kernel raises the launch's overflow word when it ends, and the safe
+// kernel after it, which otherwise returns at once, recomputes the launch with the exact
+// maximum wherever the sum passes that limit.
+// Every wait is bounded (2 s of %globaltimer, or the test hook's limit): on expiry the
+// kernel records FLAREPP_ERR_TIMEOUT in the status word, every role leaves its loops, the
+// producer waits for its copies in flight, and TMEM is freed.
 #include <cuda.h>
 #include <cudaTypedefs.h>
 #include <cuda_bf16.h>

@@ -145,3 +145,20 @@ def test_tensor_peak_follows_timed_region():
     v, kind = bench.tc_peak_for(peaks, bench.SUSTAINED_REGION_S)
     assert v == 1717.3 and kind == "bf16_tflops_sustained (measured)"
     assert bench.tc_peak_for(peaks, 10.0, bf16=False) == (None, None)
+
+
+def test_l2_flush_choice_follows_input_size():
+    """The chain is timed with the L2 flushed before each step exactly when its streamed
+    tensors come near the L2's size (pde2d: 168 MB), and warm where they exceed it twice
+    over (longseq, mesh3d); either can be forced, and the line's config says which ran."""
+    from paper_2608_11519_gb300 import inputs
+    pde, lng, mesh = inputs.get("pde2d"), inputs.get("longseq"), inputs.get("mesh3d")
+    assert bench.l2_mode("auto", pde, "flarepp") == "flush"
+    assert bench.l2_mode("auto", lng, "flarepp") == "warm"
+    assert bench.l2_mode("auto", mesh, "flarepp") == "warm"
+    assert bench.l2_mode("warm", pde, "flarepp") == "warm"
+    assert bench.l2_mode("flush", mesh, "flarepp") == "flush"
+    assert bench.FLUSH_BYTES > bench.L2_BYTES
+    assert bench.arm_config(pde, "flarepp", 1)["l2"].startswith("flushed")
+    assert bench.arm_config(pde, "flarepp", 1, "warm")["l2"].startswith("warm")
+    assert bench.arm_config(mesh, "flarepp", 1)["l2"] == "inputs larger than L2 (no flush)"
