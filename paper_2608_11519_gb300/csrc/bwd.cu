@@ -90,6 +90,17 @@ __global__ void to_bf16_kernel(const float* __restrict__ src, __nv_bfloat16* __r
         dst[i] = __float2bfloat16_rn(src[i]);
 }
 
+// hi = bf16(src), lo = bf16(src - hi): the operand pair the training forward gave Q
+__global__ void to_bf16_hilo_kernel(const float* __restrict__ src, __nv_bfloat16* __restrict__ hi,
+                                    __nv_bfloat16* __restrict__ lo, int64_t n) {
+    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n;
+         i += (int64_t)gridDim.x * blockDim.x) {
+        const __nv_bfloat16 h = __float2bfloat16_rn(src[i]);
+        hi[i] = h;
+        lo[i] = __float2bfloat16_rn(src[i] - __bfloat162float(h));
+    }
+}
+
 // Route pass of call MODE (3, 2 or 1) over one chunk of tokens; thread = route m.
 //   MODE 3: a = Q, keys b = K, w = dY, g = Z, column statistics L3[n], c3[n];
 //           pa += P w (dZ), pb += dS k (dQ / s)
@@ -182,7 +193,9 @@ __global__ void __launch_bounds__(128) route_pass_kernel(
 //   MODE 3: dZ = sum pa, dQ = s sum pb, c2 = <dZ, Z>
 //   MODE 2: dQ += s sum pb, c1 = <dQ, Q>
 //   MODE 1: dseeds[h, m] = s sum_b sum_chunks pb (rows = H * M)
-// `op`, when not null, receives a bf16 copy of dZ (MODE 3) or dQ (MODE 2).
+// `op`, when not null, receives a bf16 copy of dZ (MODE 3) or dQ (MODE 2). In MODE 2 c1 is
+// then taken from that copy: the passes of call 1 form dP = dQ K~^T from the bf16 dQ, and
+// dS = P (dP - c1) cancels for a nearly one-hot P only when c1 = <dQ, Q> uses the same dQ.
 template <int D, typename T, int MODE>
 __global__ void bwd_reduce_kernel(const float* __restrict__ pa, const float* __restrict__ pb,
                                   int64_t rows, int64_t B, int64_t H, int64_t M, int64_t nchunk,
@@ -240,8 +253,13 @@ __global__ void bwd_reduce_kernel(const float* __restrict__ pa, const float* __r
             } else {
                 const float v = dq[row * D + d] + scale * sb[i];
                 dq[row * D + d] = v;
-                dot = fmaf(v, O[row * D + d], dot);
-                if (op) op[row * D + d] = __float2bfloat16_rn(v);
+                float vc = v;
+                if (op) {
+                    const __nv_bfloat16 vb = __float2bfloat16_rn(v);
+                    op[row * D + d] = vb;
+                    vc = __bfloat162float(vb);
+                }
+                dot = fmaf(vc, O[row * D + d], dot);
             }
         }
     }
@@ -507,7 +525,12 @@ cudaError_t route_bwd_tc_d(const Plan& p, const BwdPlan& bp, const void* seeds, 
 
     constexpr bool kMerged = D <= 32;
     launch_delta_tokens<D, T>((const T*)dY, (const T*)Y, tok_rows, c3, st);
-    to_bf16_kernel<<<cvt_blocks, 256, 0, st>>>(Q32, qb, lat);
+    // Q as the training forward gave it to calls 2 and 3: a hi/lo pair for D <= 32
+    T* qlo = kMerged ? (T*)(ws + bp.off_qlo) : nullptr;
+    if (qlo)
+        to_bf16_hilo_kernel<<<cvt_blocks, 256, 0, st>>>(Q32, qb, qlo, lat);
+    else
+        to_bf16_kernel<<<cvt_blocks, 256, 0, st>>>(Q32, qb, lat);
     to_bf16_kernel<<<cvt_blocks, 256, 0, st>>>(Z32, zb, lat);
     if (kMerged) {
         merge_range_kernel<<<(unsigned)(p.BH * kRangeParts), 256, 0, st>>>(L2, L3, p.M, p.N,
@@ -519,12 +542,14 @@ cudaError_t route_bwd_tc_d(const Plan& p, const BwdPlan& bp, const void* seeds, 
     // R3: route rows; S = Q K^T, dP = Z dY^T; column statistics L3, c3 -> dQ3, dZ partials
     o = TcBwdOperands{{qb, zb, zb}, {K, dY, dY}, nullptr, nullptr, L3, c3, pa, pb, nullptr,
                       nullptr};
+    o.lo = qlo;
     if ((e = tc_bwd_pass(p, bp, 0, o, scale, status, st)) != cudaSuccess) return e;
     bwd_reduce_kernel<D, T, 3><<<red_blocks, 256, 0, st>>>(pa, pb, lat_rows, p.B, p.H, p.M,
                                                            bp.nchunk, scale, Z32, dz, dq, c2,
                                                            nullptr, dzb);
     // T23: token rows; S = K Q^T, dP2 = V dZ^T, dP3 = dY Z^T -> dK, dV
     o = TcBwdOperands{{K, V, dY}, {qb, dzb, zb}, L3, c3, L2, c2, nullptr, nullptr, dK, dV};
+    o.lo = qlo;
     if (kMerged) {
         // T23C: S = K Q^T, T = dY Z^T + (u V) (w dZ)^T; the flagged (b, h) run T23 after it
         merge_operand_kernel<<<cvt_blocks, 256, 0, st>>>(dz, L2, Rb, p.M, p.D, lat, wop);
@@ -532,6 +557,7 @@ cudaError_t route_bwd_tc_d(const Plan& p, const BwdPlan& bp, const void* seeds, 
         om.Rb = Rb;
         om.flags = flags;
         om.want = 0;
+        om.lo = qlo;
         if ((e = tc_bwd_pass(p, bp, 5, om, scale, status, st)) != cudaSuccess) return e;
         o.flags = flags;
         o.want = 1;
@@ -540,6 +566,7 @@ cudaError_t route_bwd_tc_d(const Plan& p, const BwdPlan& bp, const void* seeds, 
     // R2: route rows; S = Q K^T, dP = dZ V^T; row statistics L2, c2 -> dQ2 partials
     o = TcBwdOperands{{qb, dzb, dzb}, {K, V, V}, L2, c2, nullptr, nullptr, nullptr, pb, nullptr,
                       nullptr};
+    o.lo = qlo;
     if ((e = tc_bwd_pass(p, bp, 1, o, scale, status, st)) != cudaSuccess) return e;
     bwd_reduce_kernel<D, T, 2><<<red_blocks, 256, 0, st>>>(nullptr, pb, lat_rows, p.B, p.H, p.M,
                                                            bp.nchunk, scale, Q32, nullptr, dq, c1,

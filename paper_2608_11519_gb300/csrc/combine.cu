@@ -41,7 +41,8 @@ __global__ void __launch_bounds__(256)
     combine_kernel(const float* __restrict__ pmax, const float* __restrict__ psum,
                    const float* __restrict__ pacc, int64_t BH, int M, int nchunk,
                    int sub_per_chunk, int group_log2, float* __restrict__ out32,
-                   __nv_bfloat16* __restrict__ outop, float op_sign, float* __restrict__ lse) {
+                   __nv_bfloat16* __restrict__ outop, __nv_bfloat16* __restrict__ outlo,
+                   float op_sign, float* __restrict__ lse) {
     constexpr int T = D / 4;
     constexpr int kRowsPerBlock = 256 / T;
     tc::pdl_trigger();
@@ -102,12 +103,24 @@ __global__ void __launch_bounds__(256)
     const float4 o = make_float4(u.x * inv, u.y * inv, u.z * inv, u.w * inv);
     reinterpret_cast<float4*>(out32 + row * D)[q] = o;
     if (outop) {
-        const __nv_bfloat162 lo = __floats2bfloat162_rn(op_sign * o.x, op_sign * o.y);
-        const __nv_bfloat162 hi = __floats2bfloat162_rn(op_sign * o.z, op_sign * o.w);
+        const __nv_bfloat162 h01 = __floats2bfloat162_rn(op_sign * o.x, op_sign * o.y);
+        const __nv_bfloat162 h23 = __floats2bfloat162_rn(op_sign * o.z, op_sign * o.w);
         uint2 pk;
-        pk.x = *reinterpret_cast<const uint32_t*>(&lo);
-        pk.y = *reinterpret_cast<const uint32_t*>(&hi);
+        pk.x = *reinterpret_cast<const uint32_t*>(&h01);
+        pk.y = *reinterpret_cast<const uint32_t*>(&h23);
         reinterpret_cast<uint2*>(outop + row * D)[q] = pk;
+        if (outlo) {
+            // what bf16 rounding left out: op_sign * o - hi, rounded to bf16 again
+            const float2 h0 = __bfloat1622float2(h01), h1 = __bfloat1622float2(h23);
+            const __nv_bfloat162 l0 =
+                __floats2bfloat162_rn(op_sign * o.x - h0.x, op_sign * o.y - h0.y);
+            const __nv_bfloat162 l1 =
+                __floats2bfloat162_rn(op_sign * o.z - h1.x, op_sign * o.w - h1.y);
+            uint2 pl;
+            pl.x = *reinterpret_cast<const uint32_t*>(&l0);
+            pl.y = *reinterpret_cast<const uint32_t*>(&l1);
+            reinterpret_cast<uint2*>(outlo + row * D)[q] = pl;
+        }
     }
 }
 
@@ -121,10 +134,12 @@ __global__ void negate_bf16_kernel(const __nv_bfloat16* __restrict__ src,
 }  // namespace
 
 cudaError_t combine(const Plan& p, int call, char* ws, bool negate, cudaStream_t st,
-                    float* lse) {
+                    float* lse, bool lo) {
     float* out32 = (float*)(ws + (call == 1 ? p.off_q32 : p.off_z32));
     __nv_bfloat16* outop = nullptr;
     if (p.path == kPathTc) outop = (__nv_bfloat16*)(ws + (call == 1 ? p.off_qop : p.off_zop));
+    __nv_bfloat16* outlo = nullptr;
+    if (lo && call == 1 && p.path == kPathTc) outlo = (__nv_bfloat16*)(ws + p.off_qlo);
     const float* pmax = (const float*)(ws + p.off_pmax);
     const float* psum = (const float*)(ws + p.off_psum);
     const float* pacc = (const float*)(ws + p.off_pacc);
@@ -148,7 +163,7 @@ cudaError_t combine(const Plan& p, int call, char* ws, bool negate, cudaStream_t
         return launch_pdl(few ? combine_kernel<DD, 4> : combine_kernel<DD, 8>,               \
                           dim3((unsigned)gx, (unsigned)gy, (unsigned)gz), dim3(256), 0, st,  \
                           pmax, psum, pacc, p.BH, (int)p.M, (int)p.nchunk,                   \
-                          (int)p.sub_per_chunk, group_log2, out32, outop, sign, lse);        \
+                          (int)p.sub_per_chunk, group_log2, out32, outop, outlo, sign, lse); \
     }
     switch (p.D) {
         case 16: FLAREPP_COMBINE(16)

@@ -124,8 +124,12 @@ flarepp_status route_impl(const flarepp_shape* shape, const void* seeds, const v
     auto mark = [&](int i) {
         return !events || cudaEventRecord((cudaEvent_t)events[i], st) == cudaSuccess;
     };
+    // The training forward (D <= 32) gives the scores of calls 2 and 3 Q as a hi/lo pair of
+    // bf16 operands, so that the function its backward differentiates sees Q to about 2^-17
+    // (with bf16 Q alone, sharp softmaxes move the gradient by several percent).
+    const bool lo = tc && saved && p.D <= 32;
     auto encode = [&](int call, const void* k, const void* v) {
-        return tc ? tc_encode(p, call, k, v, seeds, scale, ws, st)
+        return tc ? tc_encode(p, call, k, v, seeds, scale, ws, st, lo)
                   : simt_encode_f32(p, call, k, v, seeds, scale, ws, st);
     };
     if (reset_status && cudaMemsetAsync(ws + p.off_status, 0, sizeof(int32_t), st) != cudaSuccess)
@@ -142,11 +146,12 @@ flarepp_status route_impl(const flarepp_shape* shape, const void* seeds, const v
     float* l1 = saved ? (float*)(saved + sv.off_l1) : nullptr;
     float* l2 = saved ? (float*)(saved + sv.off_l2) : nullptr;
     float* l3 = saved ? (float*)(saved + sv.off_l3) : nullptr;
-    if (combine(p, 1, ws, neg, st, l1) != cudaSuccess || !mark(2)) return FLAREPP_ERR_CUDA;
+    if (combine(p, 1, ws, neg, st, l1, lo) != cudaSuccess || !mark(2)) return FLAREPP_ERR_CUDA;
     if (encode(2, K, V) != cudaSuccess || !mark(3)) return FLAREPP_ERR_CUDA;
     if (combine(p, 2, ws, false, st, l2) != cudaSuccess || !mark(4)) return FLAREPP_ERR_CUDA;
     cudaError_t e;
-    e = tc ? tc_decode(p, K, scale, Y, ws, st, l3) : simt_decode_f32(p, K, scale, Y, ws, st, l3);
+    e = tc ? tc_decode(p, K, scale, Y, ws, st, l3, lo)
+           : simt_decode_f32(p, K, scale, Y, ws, st, l3);
     if (e != cudaSuccess || !mark(5)) return FLAREPP_ERR_CUDA;
     if (saved) {
         Q_out = (float*)(saved + sv.off_q);

@@ -37,6 +37,7 @@ struct Plan {
     size_t off_pmax, off_psum, off_pacc;  // partials [BH][nchunk*sub][M] f32 x2, (...)[D] f32
     size_t off_q32, off_z32;              // Q, Z float32 [BH][M][D]
     size_t off_qop, off_zop;              // bf16 MMA operand copies of Q, Z [BH][M][D]
+    size_t off_qlo;                       // bf16 lo part of Q's operand, Q - qop [BH][M][D]
     size_t off_seedneg;                   // bf16 -seeds [H][M][D] (used when scale < 0)
     size_t total;
 };
@@ -91,6 +92,7 @@ struct BwdPlan {
     size_t off_d3;              // c of call 3 [BH][N] f32 (+ 256 bytes of slack)
     size_t off_qb, off_zb;      // tensor-core path: bf16 MMA operands Q, Z [BH][M][D]
     size_t off_dzb, off_dqb;    // ... and dZ, dQ
+    size_t off_qlo;             // ... and Q's lo part, Q - bf16(Q) (D <= 32)
     size_t off_w;               // ... and the merged T23 pass's w dZ [BH][M][D] bf16
     size_t off_rb, off_flags;   // its shift R [BH] f32 and fallback flags [BH] int32
     size_t off_rpart;           // range partials [BH][kRangeParts + 2] f32
@@ -122,8 +124,10 @@ cudaError_t route_bwd(const Plan& p, const BwdPlan& bp, const void* seeds, const
 // the bf16 MMA operand copy when the tensor-core path consumes it (negated when
 // `negate`, which together with negated seeds turns a negative scale into |scale|).
 // The base-2 log-normaliser of each merged row goes to `lse` [BH][M] when it is not null.
+// With `lo` (call 1, tensor-core path) the merge also writes bf16(Q' - bf16(Q')), Q' the
+// possibly negated Q, to the workspace's lo operand.
 cudaError_t combine(const Plan& p, int call, char* ws, bool negate, cudaStream_t st,
-                    float* lse = nullptr);
+                    float* lse = nullptr, bool lo = false);
 // dst = -src elementwise (bf16; exact)
 cudaError_t negate_bf16(const void* src, void* dst, int64_t n, cudaStream_t st);
 
@@ -145,6 +149,9 @@ struct TcBwdOperands {
     const float* Rb = nullptr;  // T23C: the shift R of each (b, h)
     const int* flags = nullptr;  // when set, only the (b, h) with flags[bh] == want run
     int want = 0;
+    // Q's bf16 lo operand (Q - bf16(Q)) for the hi/lo score products of R3, R2, T23 and T23C
+    // at D <= 32, or null (plain bf16 Q)
+    const void* lo = nullptr;
 };
 // pass: 0 = R3, 1 = R2, 2 = R1 (route rows), 3 = T23, 4 = T1 (token rows), 5 = T23C (T23
 // with its two dP products merged; D = 16 and 32)
@@ -191,9 +198,10 @@ cudaError_t transpose_bf16(const void* src, int64_t R, int64_t Cc, int rep, void
 cudaError_t add_bf16(void* dst, const void* src, int64_t n, cudaStream_t st);
 
 // ---- tensor-core kernels (tc_kernels.cu), bf16 inputs
-// Encode call 1 (A = seeds) or call 2 (A = Q operand) into the chunk partials.
+// Encode call 1 (A = seeds) or call 2 (A = Q operand) into the chunk partials. With `lo`
+// (call 2, D <= 32) the scores take Q as its hi and lo bf16 operands.
 cudaError_t tc_encode(const Plan& p, int call, const void* k, const void* v, const void* seeds,
-                      float scale, char* ws, cudaStream_t st);
+                      float scale, char* ws, cudaStream_t st, bool lo = false);
 // Test hook of the bounded waits: until reset (kernel = 0), the launches of one tensor-core
 // chain kernel (1, 2: the encode of call 1 or 2; 3: the decode) wait at most wait_ns at each
 // barrier, and CTA 0's producer never loads ring item `ring_item` (so that a wait runs out).
@@ -206,8 +214,9 @@ void test_fault_for(int kernel, uint64_t* wait_ns, int64_t* ring_item);
 int64_t tc_group_rows(int64_t D);
 int64_t tc_encode_item_rows(int64_t D);  // tokens per item of the tensor-core encode
 // Decode call 3: Y = SDPA(K, Q, Z) from the Q and Z operand copies; also each token's
-// base-2 log-normaliser into `lse` [BH][N] when it is not null.
+// base-2 log-normaliser into `lse` [BH][N] when it is not null. With `lo` (D <= 32) the
+// scores take Q as its hi and lo bf16 operands.
 cudaError_t tc_decode(const Plan& p, const void* K, float scale, void* Y, char* ws,
-                      cudaStream_t st, float* lse = nullptr);
+                      cudaStream_t st, float* lse = nullptr, bool lo = false);
 
 }  // namespace flarepp

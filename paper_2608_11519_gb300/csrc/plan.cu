@@ -125,6 +125,8 @@ flarepp_status make_plan(const flarepp_shape* s, Plan* p) {
         off = align_up(off + op, kWsAlign);
         p->off_zop = off;
         off = align_up(off + op, kWsAlign);
+        p->off_qlo = off;
+        off = align_up(off + op, kWsAlign);
         p->off_seedneg = off;
         off = align_up(off + (size_t)s->H * (size_t)s->M * (size_t)s->D * 2, kWsAlign);
     }
@@ -203,6 +205,8 @@ BwdPlan make_bwd_plan(const Plan& p) {
         b.off_dzb = off;
         off = align_up(off + op, kWsAlign);
         b.off_dqb = off;
+        off = align_up(off + op, kWsAlign);
+        b.off_qlo = off;
         off = align_up(off + op, kWsAlign);
         b.off_w = off;
         off = align_up(off + op, kWsAlign);

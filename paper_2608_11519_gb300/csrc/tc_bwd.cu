@@ -57,8 +57,13 @@ constexpr uint32_t kTmemCols = 512;
 
 enum Pass : int { kR3 = 0, kR2 = 1, kR1 = 2, kT23 = 3, kT1 = 4, kT23C = 5 };
 
-template <int D, int PASS>
+// LO (D <= 32; the backward of the training forward, whose calls 2 and 3 take Q as a hi/lo
+// pair of bf16 operands): the score products S = Q K^T (R3, R2) and S = K Q^T (T23, T23C) add
+// the product with Q's lo tile, kept as one more A tile (R3, R2) or item tile (T23, T23C)
+// after the others. Nothing else changes: the TMEM layout, items and statistics are LO's too.
+template <int D, int PASS, bool LO = false>
 struct BCfg {
+    static_assert(!LO || D <= 32, "the hi/lo form of Q serves D = 16 and 32");
     static constexpr bool kRouteRows = PASS <= kR1;
     // T23C (calls 3 and 2 with their two dP products merged into one, see bwd_slice) keeps
     // its A tiles in TMEM and multiplies them from there (`ts` products)
@@ -66,6 +71,10 @@ struct BCfg {
     static constexpr int kNA = PASS == kT23 ? 3 : 2;  // score products (TMEM score tiles)
     static constexpr int kNT = (PASS == kT23 || PASS == kT23C) ? 3 : 2;  // A and item tiles
     static constexpr int kNAcc = (PASS == kR2 || PASS == kR1) ? 1 : 2;
+    static constexpr bool kLoA = LO && (PASS == kR3 || PASS == kR2);   // Q is A operand 0
+    static constexpr bool kLoI = LO && (PASS == kT23 || PASS == kT23C);  // Q is item operand 0
+    static constexpr int kNTA = kNT + (kLoA ? 1 : 0);  // A tiles per stream in shared memory
+    static constexpr int kNTI = kNT + (kLoI ? 1 : 0);  // item tiles per ring stage
     static constexpr bool kColStats = PASS == kR3 || PASS == kT23 || PASS == kT1 || kATmem;
     static constexpr bool kRowStats = PASS == kR2 || PASS == kR1 || PASS == kT23 || kATmem;
     // TMEM per stream: kNA score tiles of kItem columns, kNAcc accumulators of D, then (T23C)
@@ -98,9 +107,9 @@ struct BCfg {
     static constexpr int kGroup = NS * kRows;  // rows per work unit
     static constexpr int kStages = kItem == 64 ? 6 : 10;
     static constexpr int kATile = kRows * D * 2;
-    static constexpr int kABytes = NS * kNT * kATile;  // one unit's A tiles
+    static constexpr int kABytes = NS * kNTA * kATile;  // one unit's A tiles
     static constexpr int kItemTile = kItem * D * 2;
-    static constexpr int kStage = kNT * kItemTile;
+    static constexpr int kStage = kNTI * kItemTile;
     // two shared-memory copies of a unit's A tiles when they fit beside the ring
     static constexpr int kABuf = 2 * kABytes + kStages * kStage <= 200 * 1024 ? 2 : 1;
     static constexpr uint32_t kSwz = D == 16 ? kSw32 : (D == 32 ? kSw64 : kSw128);
@@ -355,19 +364,19 @@ __device__ __forceinline__ void bwd_item(uint32_t t0, int nv, uint64_t c2, uint6
 
 // ------------------------------------------------------------------ the kernel
 
-template <int D, int PASS>
+template <int D, int PASS, bool LO>
 __global__ void __launch_bounds__(BCfg<D, PASS>::kThreads, 1)
     tc_bwd_kernel(const __grid_constant__ CUtensorMap tmA0, const __grid_constant__ CUtensorMap tmA1,
                   const __grid_constant__ CUtensorMap tmA2, const __grid_constant__ CUtensorMap tmI0,
                   const __grid_constant__ CUtensorMap tmI1, const __grid_constant__ CUtensorMap tmI2,
-                  const BwdParams prm) {
-    using C = BCfg<D, PASS>;
+                  const __grid_constant__ CUtensorMap tmLo, const BwdParams prm) {
+    using C = BCfg<D, PASS, LO>;
     constexpr int NS = C::NS;
     extern __shared__ uint8_t smem_raw[];
     uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                                ~static_cast<uintptr_t>(1023));
-    uint8_t* abuf = smem;                          // kABuf x [NS][kNT] A tiles
-    uint8_t* ring = smem + C::kABuf * C::kABytes;  // kStages x kNT item tiles, swizzled
+    uint8_t* abuf = smem;                          // kABuf x [NS][kNTA] A tiles
+    uint8_t* ring = smem + C::kABuf * C::kABytes;  // kStages x kNTI item tiles, swizzled
     float* stats = reinterpret_cast<float*>(ring + C::kStages * C::kStage);  // [S][2][kItem]
     uint64_t* bars = reinterpret_cast<uint64_t*>(stats + C::kStages * 2 * C::kItem);
     uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + C::kNumBars);
@@ -416,6 +425,7 @@ __global__ void __launch_bounds__(BCfg<D, PASS>::kThreads, 1)
             prefetch_tmap(&tmA2);
             prefetch_tmap(&tmI2);
         }
+        if (LO) prefetch_tmap(&tmLo);
     }
     if (warp == 0) {
         tmem_alloc(smem_u32(tmem_slot), kTmemCols);
@@ -445,16 +455,19 @@ __global__ void __launch_bounds__(BCfg<D, PASS>::kThreads, 1)
                 break;
             }
             if (elect_one()) {
-                mbar_expect_tx(afull0 + 8u * ab, U.n_act * C::kNT * C::kATile);
+                mbar_expect_tx(afull0 + 8u * ab, U.n_act * C::kNTA * C::kATile);
                 const int za0 = (int)(prm.a0_per_head ? U.bh % prm.H : U.bh);
                 for (int s = 0; s < U.n_act; ++s) {
                     const int row = (int)(U.row0 + s * kRows);
-                    uint8_t* dst = abuf + ab * C::kABytes + s * C::kNT * C::kATile;
+                    uint8_t* dst = abuf + ab * C::kABytes + s * C::kNTA * C::kATile;
                     tma_load_3d(smem_u32(dst), &tmA0, 0, row, za0, afull0 + 8u * ab);
                     tma_load_3d(smem_u32(dst + C::kATile), &tmA1, 0, row, (int)U.bh,
                                 afull0 + 8u * ab);
                     if (C::kNT == 3)
                         tma_load_3d(smem_u32(dst + 2 * C::kATile), &tmA2, 0, row, (int)U.bh,
+                                    afull0 + 8u * ab);
+                    if (C::kLoA)
+                        tma_load_3d(smem_u32(dst + C::kNT * C::kATile), &tmLo, 0, row, (int)U.bh,
                                     afull0 + 8u * ab);
                 }
             }
@@ -483,6 +496,9 @@ __global__ void __launch_bounds__(BCfg<D, PASS>::kThreads, 1)
                                 full0 + 8u * st);
                     if (C::kNT == 3)
                         tma_load_3d(dst + 2 * C::kItemTile, &tmI2, 0, (int)row, (int)U.bh,
+                                    full0 + 8u * st);
+                    if (C::kLoI)
+                        tma_load_3d(dst + C::kNT * C::kItemTile, &tmLo, 0, (int)row, (int)U.bh,
                                     full0 + 8u * st);
                     // streams idle in this unit count as having released the stage
                     for (int x = U.n_act; x < NS; ++x) mbar_arrive(empty0 + 8u * st);
@@ -593,7 +609,7 @@ __global__ void __launch_bounds__(BCfg<D, PASS>::kThreads, 1)
                 ++ar;
             }
             tc_fence_after();
-            const uint32_t a_base = smem_u32(abuf + ab * C::kABytes + s * C::kNT * C::kATile);
+            const uint32_t a_base = smem_u32(abuf + ab * C::kABytes + s * C::kNTA * C::kATile);
             int prev_st = 0;
             for (int i = 0; i <= U.n_items; ++i) {
                 const int st = it % C::kStages;
@@ -629,6 +645,16 @@ __global__ void __launch_bounds__(BCfg<D, PASS>::kThreads, 1)
                             if (elect_one()) mma_ts(t0, aK + 8 * k, bd, C::kIdescS, k > 0 ? 1u : 0u);
                             __syncwarp();
                         }
+                        if (C::kLoI) {
+                            // S += K lo(Q)^T (the item's last tile)
+#pragma unroll
+                            for (int k = 0; k < D / 16; ++k) {
+                                const uint64_t bd = smem_desc(
+                                    i_base + C::kNT * C::kItemTile + 32 * k, 16, C::kSBO, C::kSwz);
+                                if (elect_one()) mma_ts(t0, aK + 8 * k, bd, C::kIdescS, 1u);
+                                __syncwarp();
+                            }
+                        }
 #pragma unroll
                         for (int k = 0; k < D / 16; ++k) {
                             const uint64_t bd = smem_desc(i_base + 2 * C::kItemTile + 32 * k, 16,
@@ -658,6 +684,21 @@ __global__ void __launch_bounds__(BCfg<D, PASS>::kThreads, 1)
                                 if (elect_one())
                                     mma_ss(t0 + t * C::kItem, ad, bd, C::kIdescS, k > 0 ? 1u : 0u);
                                 __syncwarp();
+                            }
+                            if (t == 0 && (C::kLoA || C::kLoI)) {
+                                // S += lo(Q) K^T (the A tiles' last) or K lo(Q)^T (the item's)
+                                const uint32_t a_lo = a_base + (C::kLoA ? C::kNT * C::kATile : 0);
+                                const uint32_t i_lo =
+                                    i_base + (C::kLoI ? C::kNT * C::kItemTile : 0);
+#pragma unroll
+                                for (int k = 0; k < D / 16; ++k) {
+                                    const uint64_t ad =
+                                        smem_desc(a_lo + 32 * k, 16, C::kSBO, C::kSwz);
+                                    const uint64_t bd =
+                                        smem_desc(i_lo + 32 * k, 16, C::kSBO, C::kSwz);
+                                    if (elect_one()) mma_ss(t0, ad, bd, C::kIdescS, 1u);
+                                    __syncwarp();
+                                }
                             }
                         }
                     }
@@ -705,7 +746,7 @@ __global__ void __launch_bounds__(BCfg<D, PASS>::kThreads, 1)
                     row < V.rows ? exp2f(prm.Lrow[V.bh * V.rows + row] - prm.Rb[V.bh]) : 0.f;
                 // the tiles are swizzled to the D-wide row (16-byte chunk k of row r at
                 // k ^ (bits 7.. of the row's offset)): one-row-per-thread reads hit every bank
-                const uint8_t* src = abuf + ab * C::kABytes + s * C::kNT * C::kATile + r * D * 2;
+                const uint8_t* src = abuf + ab * C::kABytes + s * C::kNTA * C::kATile + r * D * 2;
                 const int sw = ((r * D * 2) >> 7) & (D / 8 - 1);
 #pragma unroll
                 for (int t = 0; t < C::kNT; ++t) {
@@ -914,10 +955,10 @@ bool make_map(CUtensorMap* m, const void* base, int64_t D, int64_t rows, int64_t
               CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
-template <int D, int PASS>
+template <int D, int PASS, bool LO>
 cudaError_t launch_pass(const void* const* srcs, const Plan& p, BwdParams prm, cudaStream_t st) {
-    using Cf = BCfg<D, PASS>;
-    const cudaError_t attr = ensure_smem_limit((const void*)tc_bwd_kernel<D, PASS>, Cf::kSmem);
+    using Cf = BCfg<D, PASS, LO>;
+    const cudaError_t attr = ensure_smem_limit((const void*)tc_bwd_kernel<D, PASS, LO>, Cf::kSmem);
     if (attr != cudaSuccess) return attr;
     if (Cf::kRouteRows) {
         prm.n_groups = (prm.M + Cf::kGroup - 1) / Cf::kGroup;
@@ -941,29 +982,46 @@ cudaError_t launch_pass(const void* const* srcs, const Plan& p, BwdParams prm, c
                       a_side ? (uint32_t)kRows : (uint32_t)Cf::kItem))
             return cudaErrorInvalidValue;
     }
+    // Q's lo tiles (LO): an A operand of the route-row passes, an item of the token-row ones
+    CUtensorMap mlo = maps[0];
+    if (LO && !make_map(&mlo, srcs[6], p.D, Cf::kLoA ? arows : irows, p.BH,
+                        Cf::kLoA ? (uint32_t)kRows : (uint32_t)Cf::kItem))
+        return cudaErrorInvalidValue;
     int dev = 0, sms = kNumSMs;
     cudaGetDevice(&dev);
     cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
     const int64_t grid = prm.n_units < sms ? prm.n_units : sms;
-    tc_bwd_kernel<D, PASS><<<(unsigned)grid, Cf::kThreads, Cf::kSmem, st>>>(
-        maps[0], maps[1], maps[2], maps[3], maps[4], maps[5], prm);
+    tc_bwd_kernel<D, PASS, LO><<<(unsigned)grid, Cf::kThreads, Cf::kSmem, st>>>(
+        maps[0], maps[1], maps[2], maps[3], maps[4], maps[5], mlo, prm);
     return cudaGetLastError();
 }
 
+// `lo` (srcs[6] holds Q's lo operand): the hi/lo score products, for the passes whose scores
+// take Q (R3, R2, T23, T23C) at D <= 32.
 template <int PASS>
 cudaError_t launch_d(const void* const* srcs, const Plan& p, const BwdParams& prm,
-                     cudaStream_t st) {
+                     cudaStream_t st, bool lo) {
+    constexpr bool kHasQ = PASS == kR3 || PASS == kR2 || PASS == kT23 || PASS == kT23C;
+    if constexpr (kHasQ) {
+        if (lo) {
+            switch (p.D) {
+                case 16: return launch_pass<16, PASS, true>(srcs, p, prm, st);
+                case 32: return launch_pass<32, PASS, true>(srcs, p, prm, st);
+                default: return cudaErrorInvalidValue;
+            }
+        }
+    }
     if constexpr (PASS == kT23C) {
         switch (p.D) {
-            case 16: return launch_pass<16, kT23C>(srcs, p, prm, st);
-            case 32: return launch_pass<32, kT23C>(srcs, p, prm, st);
+            case 16: return launch_pass<16, kT23C, false>(srcs, p, prm, st);
+            case 32: return launch_pass<32, kT23C, false>(srcs, p, prm, st);
             default: return cudaErrorInvalidValue;
         }
     } else {
         switch (p.D) {
-            case 16: return launch_pass<16, PASS>(srcs, p, prm, st);
-            case 32: return launch_pass<32, PASS>(srcs, p, prm, st);
-            case 64: return launch_pass<64, PASS>(srcs, p, prm, st);
+            case 16: return launch_pass<16, PASS, false>(srcs, p, prm, st);
+            case 32: return launch_pass<32, PASS, false>(srcs, p, prm, st);
+            case 64: return launch_pass<64, PASS, false>(srcs, p, prm, st);
             default: return cudaErrorInvalidValue;
         }
     }
@@ -973,7 +1031,8 @@ cudaError_t launch_d(const void* const* srcs, const Plan& p, const BwdParams& pr
 
 cudaError_t tc_bwd_pass(const Plan& p, const BwdPlan& bp, int pass, const TcBwdOperands& o,
                         float scale, int* status, cudaStream_t st) {
-    const void* srcs[6] = {o.a[0], o.a[1], o.a[2], o.i[0], o.i[1], o.i[2]};
+    const void* srcs[7] = {o.a[0], o.a[1], o.a[2], o.i[0], o.i[1], o.i[2], o.lo};
+    const bool lo = o.lo != nullptr && p.D <= 32;
     BwdParams prm{};
     prm.BH = p.BH;
     prm.H = p.H;
@@ -999,12 +1058,12 @@ cudaError_t tc_bwd_pass(const Plan& p, const BwdPlan& bp, int pass, const TcBwdO
     prm.status = status;
     test_fault_for(4 + pass, &prm.wait_ns, &prm.withhold_it);
     switch (pass) {
-        case kR3: return launch_d<kR3>(srcs, p, prm, st);
-        case kR2: return launch_d<kR2>(srcs, p, prm, st);
-        case kR1: return launch_d<kR1>(srcs, p, prm, st);
-        case kT23: return launch_d<kT23>(srcs, p, prm, st);
-        case kT1: return launch_d<kT1>(srcs, p, prm, st);
-        case kT23C: return launch_d<kT23C>(srcs, p, prm, st);
+        case kR3: return launch_d<kR3>(srcs, p, prm, st, lo);
+        case kR2: return launch_d<kR2>(srcs, p, prm, st, lo);
+        case kR1: return launch_d<kR1>(srcs, p, prm, st, false);
+        case kT23: return launch_d<kT23>(srcs, p, prm, st, lo);
+        case kT1: return launch_d<kT1>(srcs, p, prm, st, false);
+        case kT23C: return launch_d<kT23C>(srcs, p, prm, st, lo);
         default: return cudaErrorInvalidValue;
     }
 }

@@ -67,21 +67,31 @@ constexpr float kLog2e = 1.4426950408889634f;
 // Sum of one item's probabilities above which the reference max is recomputed exactly.
 constexpr float kFastLimit = 281474976710656.0f;  // 2^48
 
-template <int D, bool DEC>
+// LO (the training forward, D <= 32): Q enters the scores of calls 2 and 3 as a pair of bf16
+// operands, hi = bf16(Q) and lo = bf16(Q - hi), and each score product is the sum of the two
+// products (S = (hi + lo) B^T in the encode of call 2, S = A (hi + lo)^T in the decode), so the
+// scores see Q to about 2^-17 instead of bf16's 2^-9. The encode keeps both A tiles in TMEM;
+// the decode's items carry Q's lo tile as a third tile.
+template <int D, bool DEC, bool LO = false>
 struct Cfg {
+    static_assert(!LO || D <= 32, "the hi/lo form of Q serves D = 16 and 32");
+    static constexpr bool kLoA = LO && !DEC;  // encode of call 2: A = Q as hi and lo tiles
+    static constexpr bool kLoB = LO && DEC;   // decode: every item also carries Q's lo tile
+    static constexpr int kANum = kLoA ? 2 : 1;  // A tiles per stream
     // Streamed rows per item. The encode's units are long (hundreds of items), so one TMEM
     // copy of its A tiles costs nothing at unit boundaries, and the columns that frees widen
-    // its items to 80 rows: fewer per-item round trips per token. The decode's units are only
-    // M/64 items, so it keeps two copies (the next unit's A tiles go in ahead) and 64 rows.
-    static constexpr int kItem = D == 64 ? 32 : (DEC ? 64 : 80);
+    // its items to 80 rows: fewer per-item round trips per token (with the lo tile too, the
+    // columns allow 64). The decode's units are only M/64 items, so it keeps two copies (the
+    // next unit's A tiles go in ahead) and 64 rows.
+    static constexpr int kItem = D == 64 ? 32 : ((DEC || LO) ? 64 : 80);
     static constexpr int B = 1;                                   // score buffers per stream
     static constexpr int kABuf = (D == 64 || !DEC) ? 1 : 2;     // TMEM copies of the A tiles
     static constexpr int kGroup = NS * kTileRows;     // resident rows per work unit
     static constexpr int kStages = D == 64 ? 8 : (kItem == 32 ? 16 : 8);  // multiple of 4
     static constexpr int kATile = kTileRows * D * 2;  // one 128-row operand tile
-    static constexpr int kABytes = NS * kATile;
+    static constexpr int kABytes = NS * kANum * kATile;
     static constexpr int kItemTile = kItem * D * 2;
-    static constexpr int kStage = 2 * kItemTile;
+    static constexpr int kStage = (kLoB ? 3 : 2) * kItemTile;
     static constexpr uint32_t kSwz = D == 16 ? kSw32 : (D == 32 ? kSw64 : kSw128);
     static constexpr uint32_t kSBO = 8 * D * 2;  // bytes between 8-row groups
     // barriers: full[S], empty[S], asmem_full[2], asmem_empty[2], a_ready[2], a_free[2],
@@ -100,8 +110,8 @@ struct Cfg {
     // TMEM columns
     static constexpr uint32_t kColS = 0;                  // NS x B x kItem
     static constexpr uint32_t kColO = NS * B * kItem;     // NS x D
-    static constexpr uint32_t kColA = kColO + NS * D;     // kABuf x NS tiles x D/2
-    static_assert(kColA + kABuf * NS * (D / 2) <= kTmemCols, "TMEM budget");
+    static constexpr uint32_t kColA = kColO + NS * D;     // kABuf x NS x kANum tiles x D/2
+    static_assert(kColA + kABuf * NS * kANum * (D / 2) <= kTmemCols, "TMEM budget");
     static_assert(kSmem <= 232448, "shared memory budget");
     static_assert(kStages >= 2 * B * NS, "ring depth: the full wait precedes the PV");
     static_assert(B == 1, "the s_ready / o_done protocol has one score buffer per stream");
@@ -139,9 +149,9 @@ struct Unit {
     int64_t item0, item_end;
 };
 
-template <int D, bool DEC>
+template <int D, bool DEC, bool LO>
 __device__ __forceinline__ Unit get_unit(const TcParams& p, int64_t u) {
-    using C = Cfg<D, DEC>;
+    using C = Cfg<D, DEC, LO>;
     Unit U;
     if (DEC) {
         U.tg = u % p.n_tok_groups;
@@ -330,14 +340,14 @@ __device__ __forceinline__ float exp_tile(uint32_t scol, uint32_t* pr, int nv, f
 //     item to the exact-max path, which reads S again (the decode, whose units are short,
 //     takes the first item's reference from its first score; the encode, whose units are
 //     long, takes the first item's exact maximum).
-template <int D, bool DEC, bool SAFE>
+template <int D, bool DEC, bool SAFE, bool LO>
 __device__ __forceinline__ bool softmax_step(SoftmaxStream& S, const Unit& U, uint32_t tmem,
                                              uint32_t lane_off, float c, uint64_t c2,
                                              uint32_t sready_s, uint32_t pready_s, uint32_t empty0,
                                              bool wg_leader, uint32_t it0,
                                              volatile int* abort_flag, int* status,
                                              uint64_t limit, volatile int* overflow) {
-    using C = Cfg<D, DEC>;
+    using C = Cfg<D, DEC, LO>;
     const int j = S.j;
     const int b = j % C::B;
     const uint32_t par_j = (S.ph0 + (uint32_t)j) & 1u;
@@ -429,13 +439,13 @@ __device__ __forceinline__ bool softmax_step(SoftmaxStream& S, const Unit& U, ui
 // After the stream's last item: wait for o_done (all of the unit's PVs are complete), free
 // the ring stage of the last item, read O and write the unit's result for
 // this row (the chunk partial in the encode, the normalised output row of Y in the decode).
-template <int D, bool DEC>
+template <int D, bool DEC, bool LO>
 __device__ __forceinline__ bool finish_stream(SoftmaxStream& S, const Unit& U,
                                               const TcParams& prm, uint32_t tmem,
                                               uint32_t lane_off, int r, uint32_t sready_s,
                                               uint32_t empty0, bool wg_leader, uint32_t it0,
                                               volatile int* abort_flag) {
-    using C = Cfg<D, DEC>;
+    using C = Cfg<D, DEC, LO>;
     const int a = S.s % U.n_a;
     const int par = S.s / U.n_a;
     float o[D];
@@ -501,11 +511,12 @@ __device__ __forceinline__ bool finish_stream(SoftmaxStream& S, const Unit& U,
 
 // ------------------------------------------------------------------ the kernel
 
-template <int D, bool DEC, bool SAFE>
+template <int D, bool DEC, bool SAFE, bool LO>
 __global__ void __launch_bounds__(kThreads, 1)
     tc_chain_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
-                    const __grid_constant__ CUtensorMap tmC, const TcParams prm) {
-    using C = Cfg<D, DEC>;
+                    const __grid_constant__ CUtensorMap tmC, const __grid_constant__ CUtensorMap tmL,
+                    const TcParams prm) {
+    using C = Cfg<D, DEC, LO>;
     pdl_trigger();
     if constexpr (SAFE) {
         // the safe kernel recomputes the launch only when the fast one overflowed
@@ -518,8 +529,8 @@ __global__ void __launch_bounds__(kThreads, 1)
     extern __shared__ uint8_t smem_raw[];
     uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                                ~static_cast<uintptr_t>(1023));
-    uint8_t* abuf = smem;                   // 2 x NS unswizzled A tiles
-    uint8_t* ring = smem + 2 * C::kABytes;  // kStages x (B tile, C tile), swizzled
+    uint8_t* abuf = smem;                   // 2 x NS x kANum unswizzled A tiles
+    uint8_t* ring = smem + 2 * C::kABytes;  // kStages x (B tile, C tile[, lo tile]), swizzled
     uint64_t* bars = reinterpret_cast<uint64_t*>(ring + C::kStages * C::kStage);
     uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + C::kNumBars);
     volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
@@ -559,6 +570,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         prefetch_tmap(&tmA);
         prefetch_tmap(&tmB);
         prefetch_tmap(&tmC);
+        if constexpr (LO) prefetch_tmap(&tmL);
     }
     if (warp == 1) {
         tmem_alloc(smem_u32(tmem_slot), kTmemCols);
@@ -590,13 +602,13 @@ __global__ void __launch_bounds__(kThreads, 1)
         uint32_t it = 0, ua = 0, pc = 0;  // ring items seen, units, p_ready phases consumed
         bool ok = true;
         for (int64_t u = blockIdx.x; u < prm.n_units && ok; u += gridDim.x, ++ua) {
-            const Unit U = get_unit<D, DEC>(prm, u);
+            const Unit U = get_unit<D, DEC, LO>(prm, u);
             const int tb = ua % C::kABuf;
             if (!warp_wait(aready0 + 8u * tb, (ua / C::kABuf) & 1, abort_flag, prm.status, prm.wait_ns)) break;
             tc_fence_after();
             const int a = s % U.n_a;
             const int par = s / U.n_a;
-            const uint32_t a_tmem = tmem + C::kColA + (tb * NS + a) * (D / 2);
+            const uint32_t a_tmem = tmem + C::kColA + (tb * NS + a) * C::kANum * (D / 2);
             int j = 0;
             uint32_t st_prev = 0;  // ring stage of the stream's previous item
             for (int i = 0; i < U.n_items; ++i, ++it) {
@@ -631,6 +643,20 @@ __global__ void __launch_bounds__(kThreads, 1)
                     for (int k = 0; k < D / 16; ++k)
                         mma_ts(d_s, a_tmem + 8 * k, ds + (uint64_t)(2 * k), C::kIdescS,
                                k > 0 ? 1u : 0u);
+                    if constexpr (C::kLoA) {
+                        // S += lo(Q) K^T: the lo tile follows the hi tile in TMEM
+#pragma unroll
+                        for (int k = 0; k < D / 16; ++k)
+                            mma_ts(d_s, a_tmem + D / 2 + 8 * k, ds + (uint64_t)(2 * k), C::kIdescS,
+                                   1u);
+                    }
+                    if constexpr (C::kLoB) {
+                        // S += K lo(Q)^T: the item's third tile
+                        const uint64_t dl = ds + (uint64_t)((2 * C::kItemTile) >> 4);
+#pragma unroll
+                        for (int k = 0; k < D / 16; ++k)
+                            mma_ts(d_s, a_tmem + 8 * k, dl + (uint64_t)(2 * k), C::kIdescS, 1u);
+                    }
                     mma_commit(sready_s);
                 }
                 __syncwarp();
@@ -674,12 +700,17 @@ __global__ void __launch_bounds__(kThreads, 1)
                 if (!warp_wait(asempty0 + 8u * ab, ((k >> 1) & 1) ^ 1, abort_flag, prm.status,
                                prm.wait_ns))
                     return false;
-                const Unit UA = get_unit<D, DEC>(prm, u);
+                const Unit UA = get_unit<D, DEC, LO>(prm, u);
                 if (elect_one()) {
-                    mbar_expect_tx(asfull0 + 8u * ab, UA.n_a * C::kATile);
-                    for (int a = 0; a < UA.n_a; ++a)
-                        tma_load_3d(smem_u32(abuf + ab * C::kABytes + a * C::kATile), &tmA, 0,
-                                    UA.rowA0 + a * kTileRows, UA.zA, asfull0 + 8u * ab);
+                    mbar_expect_tx(asfull0 + 8u * ab, UA.n_a * C::kANum * C::kATile);
+                    for (int a = 0; a < UA.n_a; ++a) {
+                        uint8_t* dst = abuf + ab * C::kABytes + a * C::kANum * C::kATile;
+                        tma_load_3d(smem_u32(dst), &tmA, 0, UA.rowA0 + a * kTileRows, UA.zA,
+                                    asfull0 + 8u * ab);
+                        if constexpr (C::kLoA)
+                            tma_load_3d(smem_u32(dst + C::kATile), &tmL, 0,
+                                        UA.rowA0 + a * kTileRows, UA.zA, asfull0 + 8u * ab);
+                    }
                 }
                 __syncwarp();
                 ++na;
@@ -689,7 +720,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                 if (blockIdx.x + k * G < prm.n_units) ok = issue_a(k, blockIdx.x + k * G);
             uint32_t k = 0;
             for (int64_t u = blockIdx.x; u < prm.n_units && ok; u += G, ++k) {
-                const Unit U = get_unit<D, DEC>(prm, u);
+                const Unit U = get_unit<D, DEC, LO>(prm, u);
                 for (int i = 0; i < U.n_items; ++i, ++it) {
                     const int st = it % C::kStages;
                     if (!warp_wait(empty0 + 8u * st, ((it / C::kStages) & 1) ^ 1, abort_flag,
@@ -707,6 +738,9 @@ __global__ void __launch_bounds__(kThreads, 1)
                         const uint32_t dst = smem_u32(ring + st * C::kStage);
                         tma_load_3d(dst, &tmB, 0, row, U.zB, full0 + 8u * st);
                         tma_load_3d(dst + C::kItemTile, &tmC, 0, row, U.zB, full0 + 8u * st);
+                        if constexpr (C::kLoB)
+                            tma_load_3d(dst + 2 * C::kItemTile, &tmL, 0, row, U.zB,
+                                        full0 + 8u * st);
                         // streams that do not take this item count as having released it
                         for (int x = U.n_a; x < NS; ++x) mbar_arrive(empty0 + 8u * st);
                     }
@@ -755,7 +789,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         // Copy this warpgroup's A tile of unit ua (one row per thread) from smem into TMEM
         // copy ua % kABuf, once the MMAs of the unit that last used that copy are complete.
         auto copy_a = [&](uint32_t ua_c, int64_t u_c) -> bool {
-            const int n_a = get_unit<D, DEC>(prm, u_c).n_a;
+            const int n_a = get_unit<D, DEC, LO>(prm, u_c).n_a;
             const int ab = ua_c & 1;
             const int tb = ua_c % C::kABuf;
             if (!warp_wait(asfull0 + 8u * ab, (ua_c >> 1) & 1, abort_flag, prm.status, prm.wait_ns))
@@ -764,23 +798,27 @@ __global__ void __launch_bounds__(kThreads, 1)
                 return false;
             tc_fence_after();
             if (st.s < n_a) {
-                const uint4* src = reinterpret_cast<const uint4*>(abuf + ab * C::kABytes +
-                                                                  st.s * C::kATile + r * D * 2);
-                uint32_t v[D / 2];
 #pragma unroll
-                for (int k = 0; k < D / 8; ++k) {
-                    const uint4 x = src[k];
-                    v[4 * k] = x.x;
-                    v[4 * k + 1] = x.y;
-                    v[4 * k + 2] = x.z;
-                    v[4 * k + 3] = x.w;
-                }
-                const uint32_t acol = tmem + lane_off + C::kColA + (tb * NS + st.s) * (D / 2);
-                if (D == 16) {
-                    tmem_st8(acol, v);
-                } else {
+                for (int h = 0; h < C::kANum; ++h) {  // the hi tile, then (LO) the lo tile
+                    const uint4* src = reinterpret_cast<const uint4*>(
+                        abuf + ab * C::kABytes + (st.s * C::kANum + h) * C::kATile + r * D * 2);
+                    uint32_t v[D / 2];
 #pragma unroll
-                    for (int k = 0; k < D / 32; ++k) tmem_st16(acol + 16 * k, v + 16 * k);
+                    for (int k = 0; k < D / 8; ++k) {
+                        const uint4 x = src[k];
+                        v[4 * k] = x.x;
+                        v[4 * k + 1] = x.y;
+                        v[4 * k + 2] = x.z;
+                        v[4 * k + 3] = x.w;
+                    }
+                    const uint32_t acol = tmem + lane_off + C::kColA +
+                                          ((tb * NS + st.s) * C::kANum + h) * (D / 2);
+                    if (D == 16) {
+                        tmem_st8(acol, v);
+                    } else {
+#pragma unroll
+                        for (int k = 0; k < D / 32; ++k) tmem_st16(acol + 16 * k, v + 16 * k);
+                    }
                 }
             }
             tmem_wait_st();
@@ -790,7 +828,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             return true;
         };
         for (int64_t u = blockIdx.x; u < prm.n_units && alive; u += gridDim.x, ++ua) {
-            const Unit U = get_unit<D, DEC>(prm, u);
+            const Unit U = get_unit<D, DEC, LO>(prm, u);
             // this unit's A tiles (copied one unit ahead when TMEM holds two copies)
             if (kAhead) {
                 if (ua == 0 && !copy_a(0, u)) break;
@@ -800,12 +838,12 @@ __global__ void __launch_bounds__(kThreads, 1)
             }
             st.begin(U);
             while (alive && st.j < st.cnt)
-                alive = softmax_step<D, DEC, SAFE>(st, U, tmem, lane_off, c, c2, sready_s,
+                alive = softmax_step<D, DEC, SAFE, LO>(st, U, tmem, lane_off, c, c2, sready_s,
                                                    pready0 + 16u * st.s, empty0, wg_leader, it0,
                                                    abort_flag, prm.status, prm.wait_ns,
                                                    prm.overflow);
             if (alive)
-                alive = finish_stream<D, DEC>(st, U, prm, tmem, lane_off, r, sready_s, empty0,
+                alive = finish_stream<D, DEC, LO>(st, U, prm, tmem, lane_off, r, sready_s, empty0,
                                               wg_leader, it0, abort_flag);
             it0 += U.n_items;
         }
@@ -880,33 +918,42 @@ bool make_map(CUtensorMap* m, const void* base, int64_t D, int64_t rows, int64_t
 
 // The fast kernel, then the safe one on the same stream (it returns at once unless the
 // fast kernel raised the overflow word, which the plan keeps zeroed before each call).
-template <int D, bool DEC>
+template <int D, bool DEC, bool LO>
 cudaError_t launch(const CUtensorMap& a, const CUtensorMap& b, const CUtensorMap& c,
-                   const TcParams& prm, cudaStream_t st) {
-    using Cf = Cfg<D, DEC>;
-    cudaError_t e = ensure_smem_limit((const void*)tc_chain_kernel<D, DEC, false>, Cf::kSmem);
+                   const CUtensorMap& l, const TcParams& prm, cudaStream_t st) {
+    using Cf = Cfg<D, DEC, LO>;
+    cudaError_t e = ensure_smem_limit((const void*)tc_chain_kernel<D, DEC, false, LO>, Cf::kSmem);
     if (e == cudaSuccess)
-        e = ensure_smem_limit((const void*)tc_chain_kernel<D, DEC, true>, Cf::kSmem);
+        e = ensure_smem_limit((const void*)tc_chain_kernel<D, DEC, true, LO>, Cf::kSmem);
     if (e != cudaSuccess) return e;
     int dev = 0, sms = kNumSMs;
     cudaGetDevice(&dev);
     cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
     const int64_t grid = prm.n_units < sms ? prm.n_units : sms;
-    e = launch_pdl(tc_chain_kernel<D, DEC, false>, dim3((unsigned)grid), dim3(kThreads),
-                   Cf::kSmem, st, a, b, c, prm);
+    e = launch_pdl(tc_chain_kernel<D, DEC, false, LO>, dim3((unsigned)grid), dim3(kThreads),
+                   Cf::kSmem, st, a, b, c, l, prm);
     if (e == cudaSuccess)
-        e = launch_pdl(tc_chain_kernel<D, DEC, true>, dim3((unsigned)grid), dim3(kThreads),
-                       Cf::kSmem, st, a, b, c, prm);
+        e = launch_pdl(tc_chain_kernel<D, DEC, true, LO>, dim3((unsigned)grid), dim3(kThreads),
+                       Cf::kSmem, st, a, b, c, l, prm);
     return e;
 }
 
+// `l` (the map of Q's lo tiles) is read only by the LO kernels (D <= 32).
 template <bool DEC>
-cudaError_t launch_d(int64_t D, const CUtensorMap& a, const CUtensorMap& b, const CUtensorMap& c,
-                     const TcParams& prm, cudaStream_t st) {
+cudaError_t launch_d(int64_t D, bool lo, const CUtensorMap& a, const CUtensorMap& b,
+                     const CUtensorMap& c, const CUtensorMap& l, const TcParams& prm,
+                     cudaStream_t st) {
+    if (lo) {
+        switch (D) {
+            case 16: return launch<16, DEC, true>(a, b, c, l, prm, st);
+            case 32: return launch<32, DEC, true>(a, b, c, l, prm, st);
+        }
+        return cudaErrorInvalidValue;
+    }
     switch (D) {
-        case 16: return launch<16, DEC>(a, b, c, prm, st);
-        case 32: return launch<32, DEC>(a, b, c, prm, st);
-        case 64: return launch<64, DEC>(a, b, c, prm, st);
+        case 16: return launch<16, DEC, false>(a, b, c, l, prm, st);
+        case 32: return launch<32, DEC, false>(a, b, c, l, prm, st);
+        case 64: return launch<64, DEC, false>(a, b, c, l, prm, st);
     }
     return cudaErrorInvalidValue;
 }
@@ -915,7 +962,8 @@ cudaError_t launch_d(int64_t D, const CUtensorMap& a, const CUtensorMap& b, cons
 
 // Streamed rows per item (the TMA box height of the ring tiles) of the encode or decode.
 template <bool DEC>
-uint32_t item_rows(int64_t D) {
+uint32_t item_rows(int64_t D, bool lo = false) {
+    if (lo) return D == 16 ? Cfg<16, DEC, true>::kItem : Cfg<32, DEC, true>::kItem;
     return D == 16 ? Cfg<16, DEC>::kItem : (D == 32 ? Cfg<32, DEC>::kItem : Cfg<64, DEC>::kItem);
 }
 
@@ -944,9 +992,10 @@ int64_t tc_group_rows(int64_t D) {
 }
 
 cudaError_t tc_encode(const Plan& p, int call, const void* k, const void* v, const void* seeds,
-                      float scale, char* ws, cudaStream_t st) {
-    CUtensorMap ma, mb, mc;
+                      float scale, char* ws, cudaStream_t st, bool lo) {
+    CUtensorMap ma, mb, mc, ml;
     const bool neg = scale < 0.f;
+    lo = lo && call == 2 && p.D <= 32;  // call 1's A operand (the seeds) is exact in bf16
     const void* a_src;
     int64_t a_z;
     if (call == 1) {
@@ -957,8 +1006,11 @@ cudaError_t tc_encode(const Plan& p, int call, const void* k, const void* v, con
         a_z = p.BH;
     }
     if (!make_map(&ma, a_src, p.D, p.M, a_z, kTileRows, false) ||
-        !make_map(&mb, k, p.D, p.N, p.BH, item_rows<false>(p.D), true) ||
-        !make_map(&mc, v, p.D, p.N, p.BH, item_rows<false>(p.D), true))
+        !make_map(&mb, k, p.D, p.N, p.BH, item_rows<false>(p.D, lo), true) ||
+        !make_map(&mc, v, p.D, p.N, p.BH, item_rows<false>(p.D, lo), true))
+        return cudaErrorInvalidValue;
+    ml = ma;
+    if (lo && !make_map(&ml, ws + p.off_qlo, p.D, p.M, a_z, kTileRows, false))
         return cudaErrorInvalidValue;
     TcParams prm{};
     prm.BH = p.BH;
@@ -977,15 +1029,19 @@ cudaError_t tc_encode(const Plan& p, int call, const void* k, const void* v, con
     prm.status = (int*)(ws + p.off_status);
     prm.overflow = (int*)(ws + p.off_overflow) + (call - 1);
     apply_fault(call, prm);
-    return launch_d<false>(p.D, ma, mb, mc, prm, st);
+    return launch_d<false>(p.D, lo, ma, mb, mc, ml, prm, st);
 }
 
 cudaError_t tc_decode(const Plan& p, const void* K, float scale, void* Y, char* ws,
-                      cudaStream_t st, float* lse) {
-    CUtensorMap ma, mb, mc;
+                      cudaStream_t st, float* lse, bool lo) {
+    CUtensorMap ma, mb, mc, ml;
+    lo = lo && p.D <= 32;
     if (!make_map(&ma, K, p.D, p.N, p.BH, kTileRows, false) ||
-        !make_map(&mb, ws + p.off_qop, p.D, p.M, p.BH, item_rows<true>(p.D), true) ||
-        !make_map(&mc, ws + p.off_zop, p.D, p.M, p.BH, item_rows<true>(p.D), true))
+        !make_map(&mb, ws + p.off_qop, p.D, p.M, p.BH, item_rows<true>(p.D, lo), true) ||
+        !make_map(&mc, ws + p.off_zop, p.D, p.M, p.BH, item_rows<true>(p.D, lo), true))
+        return cudaErrorInvalidValue;
+    ml = ma;
+    if (lo && !make_map(&ml, ws + p.off_qlo, p.D, p.M, p.BH, item_rows<true>(p.D, lo), true))
         return cudaErrorInvalidValue;
     TcParams prm{};
     prm.BH = p.BH;
@@ -1001,7 +1057,7 @@ cudaError_t tc_decode(const Plan& p, const void* K, float scale, void* Y, char* 
     prm.status = (int*)(ws + p.off_status);
     prm.overflow = (int*)(ws + p.off_overflow) + 2;
     apply_fault(3, prm);
-    return launch_d<true>(p.D, ma, mb, mc, prm, st);
+    return launch_d<true>(p.D, lo, ma, mb, mc, ml, prm, st);
 }
 
 }  // namespace flarepp

@@ -133,7 +133,13 @@ def test_mixer_bwd_matches_oracle(shape):
     torch.cuda.synchronize()
     O_plain = flarepp.mixer_fwd(*dev, s)
     torch.cuda.synchronize()
-    assert torch.equal(O, O_plain)
+    if D > 32:
+        assert torch.equal(O, O_plain)
+    else:
+        # the training forward's calls 2 and 3 take Q as a hi/lo operand pair: O differs from
+        # the plain forward's by bf16 rounding only
+        a, b = O.float(), O_plain.float()
+        assert float((a - b).abs().max()) <= 2e-2 * max(1.0, float(b.abs().max()))
     want = oracle.mixer_bwd(_np(X), _np(W_in), _np(Wo), _np(seeds), s, _np(dO))
     for name, got, ref in zip(("dX", "dW_in", "dWo", "dseeds"), grads, want):
         got = _np(got)
