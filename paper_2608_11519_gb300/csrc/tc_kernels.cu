@@ -149,13 +149,17 @@ struct Unit {
     int64_t item0, item_end;
 };
 
+// The plan keeps unit counts, and so every quotient below, within 32 bits; 32-bit divisions by
+// runtime values cost a few instructions where 64-bit ones cost about seventy.
 template <int D, bool DEC, bool LO>
-__device__ __forceinline__ Unit get_unit(const TcParams& p, int64_t u) {
+__device__ __forceinline__ Unit get_unit(const TcParams& p, int64_t u64) {
     using C = Cfg<D, DEC, LO>;
+    const uint32_t u = (uint32_t)u64;
     Unit U;
     if (DEC) {
-        U.tg = u % p.n_tok_groups;
-        U.bh = u / p.n_tok_groups;
+        const uint32_t ntg = (uint32_t)p.n_tok_groups;
+        U.tg = u % ntg;
+        U.bh = u / ntg;
         U.chunk = 0;
         U.g = 0;
         U.zA = (int)U.bh;
@@ -165,12 +169,13 @@ __device__ __forceinline__ Unit get_unit(const TcParams& p, int64_t u) {
         U.item0 = 0;
         U.item_end = p.M;
     } else {
-        U.chunk = u % p.nchunk;
-        const int64_t t = u / p.nchunk;
-        U.g = t % p.n_groups;
-        U.bh = t / p.n_groups;
+        const uint32_t nchunk = (uint32_t)p.nchunk, ngroups = (uint32_t)p.n_groups;
+        U.chunk = u % nchunk;
+        const uint32_t t = u / nchunk;
+        U.g = t % ngroups;
+        U.bh = t / ngroups;
         U.tg = 0;
-        U.zA = (int)(p.a_per_head ? U.bh % p.H : U.bh);
+        U.zA = (int)(p.a_per_head ? (uint32_t)U.bh % (uint32_t)p.H : (uint32_t)U.bh);
         U.rowA0 = (int)(U.g * C::kGroup);
         U.n_a = na_of_group(p.M, U.g);
         U.n_par = NS / U.n_a;
@@ -222,13 +227,14 @@ __device__ __forceinline__ bool warp_wait(uint32_t bar, uint32_t parity, volatil
 // Online-softmax state of one TMEM stream, held by every thread of its warpgroup for its row.
 struct SoftmaxStream {
     int s;          // stream index
+    int par;        // token parity of the stream's items in this unit (s / n_a)
     int cnt, j;     // items of the stream in this unit, items done
     float m, l;     // reference max (base 2, scaled) and running sum
     uint32_t ph0;   // s_ready phases completed in earlier units (one per item)
     uint32_t od;    // o_done phases completed in earlier units (one per unit with items)
     bool over;      // fast kernel: some item's sum passed kFastLimit
     __device__ __forceinline__ void begin(const Unit& U) {
-        const int par = s / U.n_a;
+        par = s / U.n_a;
         cnt = U.n_items > par ? (U.n_items - par + U.n_par - 1) / U.n_par : 0;
         j = 0;
         m = -INFINITY;
@@ -353,7 +359,7 @@ __device__ __forceinline__ bool softmax_step(SoftmaxStream& S, const Unit& U, ui
     const uint32_t par_j = (S.ph0 + (uint32_t)j) & 1u;
     if (!warp_wait(sready_s + 8u * b, par_j, abort_flag, status, limit)) return false;
     tc_fence_after();
-    const int par = S.s / U.n_a;
+    const int par = S.par;
     if (wg_leader && j >= C::B) {
         const int i_old = par + (j - C::B) * U.n_par;
         mbar_arrive(empty0 + 8u * ((it0 + i_old) % C::kStages));
@@ -447,7 +453,7 @@ __device__ __forceinline__ bool finish_stream(SoftmaxStream& S, const Unit& U,
                                               volatile int* abort_flag) {
     using C = Cfg<D, DEC, LO>;
     const int a = S.s % U.n_a;
-    const int par = S.s / U.n_a;
+    const int par = S.par;
     float o[D];
     if (S.cnt > 0) {
         if (!warp_wait(sready_s + 8u, S.od & 1u, abort_flag, prm.status, prm.wait_ns)) return false;
@@ -621,7 +627,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                     ok = false;
                     break;
                 }
-                if ((i % U.n_par) != par) continue;
+                if ((i & (U.n_par - 1)) != par) continue;
                 if (j > 0) {
                     if (!warp_wait(pready_s, pc & 1, abort_flag, prm.status, prm.wait_ns)) {
                         ok = false;
