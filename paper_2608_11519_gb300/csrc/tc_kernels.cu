@@ -78,14 +78,20 @@ struct Cfg {
     static constexpr bool kLoA = LO && !DEC;  // encode of call 2: A = Q as hi and lo tiles
     static constexpr bool kLoB = LO && DEC;   // decode: every item also carries Q's lo tile
     static constexpr int kANum = kLoA ? 2 : 1;  // A tiles per stream
-    // Streamed rows per item. The encode's units are long (hundreds of items), so one TMEM
-    // copy of its A tiles costs nothing at unit boundaries, and the columns that frees widen
-    // its items to 80 rows: fewer per-item round trips per token (with the lo tile too, the
-    // columns allow 64). The decode's units are only M/64 items, so it keeps two copies (the
-    // next unit's A tiles go in ahead) and 64 rows.
+    // Where the A tiles live. The encode's units are long (hundreds of items): its A tiles are
+    // copied into TMEM once per unit (`ts` score products), and the single copy leaves the
+    // columns that widen its items to 80 rows (64 with the lo tile too): fewer per-item round
+    // trips per token. The decode's units are only M/64 items, so per-unit costs show: its A
+    // tiles stay in shared memory where the TMA puts them (swizzled like the ring tiles; `ss`
+    // score products), double-buffered so the next unit's tiles land during this one, and
+    // nothing copies them. Where TMEM has the room (D <= 32) the decode also keeps two O
+    // accumulators per stream, one per unit parity, so a unit's epilogue can wait until the
+    // next unit's first item is under way.
     static constexpr int kItem = D == 64 ? 32 : ((DEC || LO) ? 64 : 80);
-    static constexpr int B = 1;                                   // score buffers per stream
-    static constexpr int kABuf = (D == 64 || !DEC) ? 1 : 2;     // TMEM copies of the A tiles
+    static constexpr int B = 1;                               // score buffers per stream
+    static constexpr bool kASmem = DEC;                       // A read by the MMA from smem
+    static constexpr int kABuf = DEC ? 0 : 1;                 // TMEM copies of the A tiles
+    static constexpr int kOBuf = (DEC && D <= 32) ? 2 : 1;    // O accumulators per stream
     static constexpr int kGroup = NS * kTileRows;     // resident rows per work unit
     static constexpr int kStages = D == 64 ? 8 : (kItem == 32 ? 16 : 8);  // multiple of 4
     static constexpr int kATile = kTileRows * D * 2;  // one 128-row operand tile
@@ -96,10 +102,16 @@ struct Cfg {
     static constexpr uint32_t kSBO = 8 * D * 2;  // bytes between 8-row groups
     // barriers: full[S], empty[S], asmem_full[2], asmem_empty[2], a_ready[2], a_free[2],
     //           sync[NS][2] = {s_ready, o_done} per stream (S of an item complete; every PV
-    //           of the stream's unit complete), p_ready[NS][2] (slot 0 used). A barrier that
-    //           a warp waits on by parity never runs two phases ahead of that warp: s_ready
-    //           of the next item needs this item's P (p_ready counts every warp of the
-    //           warpgroup), o_done of the next unit needs that unit's P.
+    //           of the stream's unit complete), p_ready[NS][2] (slot 0 used). The encode's A
+    //           tiles go asmem_full -> softmax copy into TMEM -> asmem_empty and a_ready, and
+    //           a_free (one commit per MMA warp after a unit's last MMA) frees the TMEM copy. In
+    //           the decode the MMAs wait on asmem_full themselves, and a_free counts one arrive
+    //           per softmax warpgroup once it has seen the unit's last S. With two O
+    //           accumulators a decode unit's last PV goes out with the next unit's first S, so
+    //           o_done is committed only for a CTA's last unit. A barrier that a warp waits on
+    //           by parity never runs two phases ahead of that warp: s_ready of the next item
+    //           needs this item's P (p_ready counts every warp of the warpgroup), o_done of the
+    //           next unit needs that unit's P.
     static constexpr int kNumBars = 2 * kStages + 8 + 4 * NS;
     static constexpr int kData = 2 * kABytes + kStages * kStage;
     static constexpr int kNeed = 1024 + kData + kNumBars * 8 + 16;
@@ -109,12 +121,13 @@ struct Cfg {
     static constexpr uint32_t kIdescPV = idesc_bf16_f32(128, D, false, true);
     // TMEM columns
     static constexpr uint32_t kColS = 0;                  // NS x B x kItem
-    static constexpr uint32_t kColO = NS * B * kItem;     // NS x D
-    static constexpr uint32_t kColA = kColO + NS * D;     // kABuf x NS x kANum tiles x D/2
+    static constexpr uint32_t kColO = NS * B * kItem;         // kOBuf x NS x D
+    static constexpr uint32_t kColA = kColO + kOBuf * NS * D;  // kABuf x NS x kANum tiles x D/2
     static_assert(kColA + kABuf * NS * kANum * (D / 2) <= kTmemCols, "TMEM budget");
     static_assert(kSmem <= 232448, "shared memory budget");
     static_assert(kStages >= 2 * B * NS, "ring depth: the full wait precedes the PV");
     static_assert(B == 1, "the s_ready / o_done protocol has one score buffer per stream");
+    static_assert(kABuf <= 1 && (kABuf == 1) != kASmem, "A: one TMEM copy or shared memory");
 };
 
 struct TcParams {
@@ -229,6 +242,8 @@ struct SoftmaxStream {
     int s;          // stream index
     int par;        // token parity of the stream's items in this unit (s / n_a)
     int cnt, j;     // items of the stream in this unit, items done
+    int ob;         // O accumulator of this unit (0, or the unit's parity with two)
+    int ab;         // shared-memory A buffer of this unit (the unit's parity)
     float m, l;     // reference max (base 2, scaled) and running sum
     uint32_t ph0;   // s_ready phases completed in earlier units (one per item)
     uint32_t od;    // o_done phases completed in earlier units (one per unit with items)
@@ -350,7 +365,7 @@ template <int D, bool DEC, bool SAFE, bool LO>
 __device__ __forceinline__ bool softmax_step(SoftmaxStream& S, const Unit& U, uint32_t tmem,
                                              uint32_t lane_off, float c, uint64_t c2,
                                              uint32_t sready_s, uint32_t pready_s, uint32_t empty0,
-                                             bool wg_leader, uint32_t it0,
+                                             uint32_t afree0, bool wg_leader, uint32_t it0,
                                              volatile int* abort_flag, int* status,
                                              uint64_t limit, volatile int* overflow) {
     using C = Cfg<D, DEC, LO>;
@@ -364,6 +379,8 @@ __device__ __forceinline__ bool softmax_step(SoftmaxStream& S, const Unit& U, ui
         const int i_old = par + (j - C::B) * U.n_par;
         mbar_arrive(empty0 + 8u * ((it0 + i_old) % C::kStages));
     }
+    // decode: the unit's last S is complete, so its MMAs no longer read the A buffer
+    if (C::kASmem && wg_leader && j == S.cnt - 1) mbar_arrive(afree0 + 8u * S.ab);
     const int item = par + j * U.n_par;
     const int64_t start = U.item0 + (int64_t)item * C::kItem;
     const int nv = (int)min((int64_t)C::kItem, U.item_end - start);
@@ -412,7 +429,7 @@ __device__ __forceinline__ bool softmax_step(SoftmaxStream& S, const Unit& U, ui
         }
         if (__any_sync(0xffffffffu, need)) {
             // (the PV of item j - 1 is complete: S of item j followed it in the tensor pipe)
-            const uint32_t ocol = tmem + lane_off + C::kColO + S.s * D;
+            const uint32_t ocol = tmem + lane_off + C::kColO + (S.ob * NS + S.s) * D;
             const float f = need ? alpha : 1.f;
 #pragma unroll
             for (int k = 0; k < D / 16; ++k) {
@@ -442,30 +459,45 @@ __device__ __forceinline__ bool softmax_step(SoftmaxStream& S, const Unit& U, ui
     return true;
 }
 
-// After the stream's last item: wait for o_done (all of the unit's PVs are complete), free
-// the ring stage of the last item, read O and write the unit's result for
-// this row (the chunk partial in the encode, the normalised output row of Y in the decode).
+// The end of one unit of the stream, for this row: the unit's online-softmax state (m, l),
+// its item count, the ring item its items start from, its O accumulator and (decode) its A
+// buffer. Wait until all of the unit's PVs are complete, free the ring stage of the last item
+// (and, if the stream had no items, the unit's shared-memory A buffer), read O and write the
+// unit's result (the chunk partial in the encode, the normalised output row of Y in the
+// decode).
+// `deferred`: the decode with two O accumulators runs this one unit late, after the next
+// unit's first item, whose s_ready was committed after the unit's last PV (the MMA warp
+// issues the two together); otherwise the wait is on o_done.
+struct UnitEnd {
+    float m, l;
+    int cnt, ob, ab;
+    uint32_t it0;
+};
+
 template <int D, bool DEC, bool LO>
-__device__ __forceinline__ bool finish_stream(SoftmaxStream& S, const Unit& U,
+__device__ __forceinline__ bool finish_stream(SoftmaxStream& S, const UnitEnd& E, const Unit& U,
                                               const TcParams& prm, uint32_t tmem,
                                               uint32_t lane_off, int r, uint32_t sready_s,
-                                              uint32_t empty0, bool wg_leader, uint32_t it0,
-                                              volatile int* abort_flag) {
+                                              uint32_t empty0, uint32_t afree0, bool wg_leader,
+                                              bool deferred, volatile int* abort_flag) {
     using C = Cfg<D, DEC, LO>;
     const int a = S.s % U.n_a;
-    const int par = S.par;
+    const int par = S.s / U.n_a;
     float o[D];
-    if (S.cnt > 0) {
-        if (!warp_wait(sready_s + 8u, S.od & 1u, abort_flag, prm.status, prm.wait_ns)) return false;
-        ++S.od;
-        tc_fence_after();
+    if (E.cnt > 0) {
+        if (!deferred) {
+            if (!warp_wait(sready_s + 8u, S.od & 1u, abort_flag, prm.status, prm.wait_ns))
+                return false;
+            ++S.od;
+            tc_fence_after();
+        }
         if (wg_leader) {
-            for (int jj = S.cnt - C::B < 0 ? 0 : S.cnt - C::B; jj < S.cnt; ++jj) {
+            for (int jj = E.cnt - C::B < 0 ? 0 : E.cnt - C::B; jj < E.cnt; ++jj) {
                 const int i_old = par + jj * U.n_par;
-                mbar_arrive(empty0 + 8u * ((it0 + i_old) % C::kStages));
+                mbar_arrive(empty0 + 8u * ((E.it0 + i_old) % C::kStages));
             }
         }
-        const uint32_t ocol = tmem + lane_off + C::kColO + S.s * D;
+        const uint32_t ocol = tmem + lane_off + C::kColO + (E.ob * NS + S.s) * D;
         // every load of O in flight before one wait
         uint32_t t[D];
         if (D == 16) {
@@ -480,14 +512,16 @@ __device__ __forceinline__ bool finish_stream(SoftmaxStream& S, const Unit& U,
 #pragma unroll
         for (int d = 0; d < D; ++d) o[d] = __uint_as_float(t[d]);
     } else {
+        // (no MMA of this stream read the unit's A tile)
+        if constexpr (C::kASmem)
+            if (wg_leader) mbar_arrive(afree0 + 8u * E.ab);
 #pragma unroll
         for (int d = 0; d < D; ++d) o[d] = 0.f;
     }
-    S.ph0 += (uint32_t)S.cnt;
     if (DEC) {
         const int64_t tok = U.tg * C::kGroup + a * kTileRows + r;
         if (tok < prm.N) {
-            const float inv = 1.f / S.l;
+            const float inv = 1.f / E.l;
             uint4* dst = reinterpret_cast<uint4*>(prm.Y + (U.bh * prm.N + tok) * D);
 #pragma unroll
             for (int kk = 0; kk < D / 8; ++kk) {
@@ -498,14 +532,14 @@ __device__ __forceinline__ bool finish_stream(SoftmaxStream& S, const Unit& U,
                 v.w = pack_bf16(o[8 * kk + 6] * inv, o[8 * kk + 7] * inv);
                 dst[kk] = v;
             }
-            if (prm.lse) prm.lse[U.bh * prm.N + tok] = S.m + log2f(S.l);
+            if (prm.lse) prm.lse[U.bh * prm.N + tok] = E.m + log2f(E.l);
         }
     } else {
         const int64_t route = U.g * C::kGroup + a * kTileRows + r;
         if (route < prm.M) {
             const int64_t idx = (U.bh * (prm.nchunk * 4) + U.chunk * 4 + par) * prm.M + route;
-            prm.pmax[idx] = S.cnt > 0 ? S.m : -INFINITY;
-            prm.psum[idx] = S.l;
+            prm.pmax[idx] = E.cnt > 0 ? E.m : -INFINITY;
+            prm.psum[idx] = E.l;
             float4* dst = reinterpret_cast<float4*>(prm.pacc + idx * D);
 #pragma unroll
             for (int kk = 0; kk < D / 4; ++kk)
@@ -592,31 +626,44 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (warp < kProducerWarp) {
         // ------------------------------------------------------------ MMA warps
         // Warp s drives stream s. For each of its items: the PV of its previous item (P
-        // from TMEM, V or Z from the ring), the S of this item (A from TMEM, K or Q from the
-        // ring) and one commit, which the softmax waits on, all from one elected lane with
-        // descriptors derived from two precomputed ones. It observes the full barrier of every
-        // ring item in order, so each parity test names one phase.
+        // from TMEM, V or Z from the ring), the S of this item (A from TMEM in the encode, from
+        // shared memory in the decode; K or Q from the ring) and one commit, which the softmax
+        // waits on, all from one elected lane with descriptors derived from precomputed ones.
+        // It observes the full barrier of every ring item in order, so each parity test names
+        // one phase.
         regs_lower<kRegsControl>();
         const int s = warp;
         const uint32_t ring_u = smem_u32(ring);
         const uint64_t dS0 = smem_desc(ring_u, 16, C::kSBO, C::kSwz);
         const uint64_t dV0 = smem_desc(ring_u + C::kItemTile, C::kItemTile, C::kSBO, C::kSwz);
+        const uint64_t dA0 = smem_desc(smem_u32(abuf), 16, C::kSBO, C::kSwz);
         const uint32_t d_s = tmem + C::kColS + s * C::kItem;  // B = 1: one score buffer
-        const uint32_t d_o = tmem + C::kColO + s * D;
         const uint32_t sready_s = sready0 + 16u * s;
         const uint32_t pready_s = pready0 + 16u * s;
         uint32_t it = 0, ua = 0, pc = 0;  // ring items seen, units, p_ready phases consumed
+        // The PV owed for the stream's previous item (its ring stage, the O accumulator it adds
+        // into, whether it adds or starts it) goes out with the next S under one commit. In the
+        // decode with two O accumulators it crosses unit boundaries too: a unit then ends with
+        // no commit of its own, and s_ready of the next unit's first item also says that the
+        // unit's O is final and its A tile no longer read.
+        bool pv_owed = false;
+        uint32_t pv_st = 0, pv_o = 0, pv_acc = 0;
         bool ok = true;
         for (int64_t u = blockIdx.x; u < prm.n_units && ok; u += gridDim.x, ++ua) {
             const Unit U = get_unit<D, DEC, LO>(prm, u);
-            const int tb = ua % C::kABuf;
-            if (!warp_wait(aready0 + 8u * tb, (ua / C::kABuf) & 1, abort_flag, prm.status, prm.wait_ns)) break;
-            tc_fence_after();
             const int a = s % U.n_a;
             const int par = s / U.n_a;
-            const uint32_t a_tmem = tmem + C::kColA + (tb * NS + a) * C::kANum * (D / 2);
+            // the unit's A tile: shared-memory buffer ua % 2 as the TMA wrote it (decode), or
+            // the TMEM copy the softmax made of it (encode)
+            const int ab = ua & 1;
+            if (!warp_wait(C::kASmem ? asfull0 + 8u * ab : aready0, C::kASmem ? (ua >> 1) & 1 : ua & 1,
+                           abort_flag, prm.status, prm.wait_ns))
+                break;
+            tc_fence_after();
+            const uint64_t dA = dA0 + ((uint64_t)(ab * C::kABytes + a * C::kATile) >> 4);
+            const uint32_t a_tmem = tmem + C::kColA + a * C::kANum * (D / 2);
+            const uint32_t d_o = tmem + C::kColO + ((C::kOBuf == 2 ? ab : 0) * NS + s) * D;
             int j = 0;
-            uint32_t st_prev = 0;  // ring stage of the stream's previous item
             for (int i = 0; i < U.n_items; ++i, ++it) {
                 const uint32_t st = it % C::kStages;
                 // the item's full barrier first (the softmax is still busy with item j - 1, so
@@ -628,7 +675,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                     break;
                 }
                 if ((i & (U.n_par - 1)) != par) continue;
-                if (j > 0) {
+                if (pv_owed) {
                     if (!warp_wait(pready_s, pc & 1, abort_flag, prm.status, prm.wait_ns)) {
                         ok = false;
                         break;
@@ -637,18 +684,23 @@ __global__ void __launch_bounds__(kThreads, 1)
                 }
                 tc_fence_after();
                 if (elect_one()) {
-                    if (j > 0) {
-                        const uint64_t dv = dV0 + ((st_prev * C::kStage) >> 4);
+                    if (pv_owed) {
+                        const uint64_t dv = dV0 + ((pv_st * C::kStage) >> 4);
 #pragma unroll
                         for (int k = 0; k < C::kItem / 16; ++k)
-                            mma_ts(d_o, d_s + 8 * k, dv + (uint64_t)(2 * D * k), C::kIdescPV,
-                                   (j > 1 || k > 0) ? 1u : 0u);
+                            mma_ts(pv_o, d_s + 8 * k, dv + (uint64_t)(2 * D * k), C::kIdescPV,
+                                   (pv_acc || k > 0) ? 1u : 0u);
                     }
                     const uint64_t ds = dS0 + ((st * C::kStage) >> 4);
 #pragma unroll
-                    for (int k = 0; k < D / 16; ++k)
-                        mma_ts(d_s, a_tmem + 8 * k, ds + (uint64_t)(2 * k), C::kIdescS,
-                               k > 0 ? 1u : 0u);
+                    for (int k = 0; k < D / 16; ++k) {
+                        if constexpr (C::kASmem)
+                            mma_ss(d_s, dA + (uint64_t)(2 * k), ds + (uint64_t)(2 * k), C::kIdescS,
+                                   k > 0 ? 1u : 0u);
+                        else
+                            mma_ts(d_s, a_tmem + 8 * k, ds + (uint64_t)(2 * k), C::kIdescS,
+                                   k > 0 ? 1u : 0u);
+                    }
                     if constexpr (C::kLoA) {
                         // S += lo(Q) K^T: the lo tile follows the hi tile in TMEM
 #pragma unroll
@@ -661,50 +713,57 @@ __global__ void __launch_bounds__(kThreads, 1)
                         const uint64_t dl = ds + (uint64_t)((2 * C::kItemTile) >> 4);
 #pragma unroll
                         for (int k = 0; k < D / 16; ++k)
-                            mma_ts(d_s, a_tmem + 8 * k, dl + (uint64_t)(2 * k), C::kIdescS, 1u);
+                            mma_ss(d_s, dA + (uint64_t)(2 * k), dl + (uint64_t)(2 * k), C::kIdescS,
+                                   1u);
                     }
                     mma_commit(sready_s);
                 }
                 __syncwarp();
-                st_prev = st;
+                pv_owed = true;
+                pv_st = st;
+                pv_o = d_o;
+                pv_acc = j > 0 ? 1u : 0u;
                 ++j;
             }
             if (!ok) break;
+            // decode with two O accumulators: the last PV goes out with the next unit's first S
+            if (C::kOBuf == 2 && u + gridDim.x < prm.n_units) continue;
             // the PV of the unit's last item, then o_done: O is final for the softmax; and
-            // this stream's MMAs no longer read the unit's TMEM A buffer
-            if (j > 0 && !warp_wait(pready_s, pc & 1, abort_flag, prm.status, prm.wait_ns)) break;
-            if (j > 0) ++pc;
+            // (encode) a_free: this stream's MMAs no longer read the unit's TMEM A copy
+            if (pv_owed && !warp_wait(pready_s, pc & 1, abort_flag, prm.status, prm.wait_ns)) break;
+            if (pv_owed) ++pc;
             tc_fence_after();
             if (elect_one()) {
-                if (j > 0) {
-                    const uint64_t dv = dV0 + ((st_prev * C::kStage) >> 4);
+                if (pv_owed) {
+                    const uint64_t dv = dV0 + ((pv_st * C::kStage) >> 4);
 #pragma unroll
                     for (int k = 0; k < C::kItem / 16; ++k)
-                        mma_ts(d_o, d_s + 8 * k, dv + (uint64_t)(2 * D * k), C::kIdescPV,
-                               (j > 1 || k > 0) ? 1u : 0u);
+                        mma_ts(pv_o, d_s + 8 * k, dv + (uint64_t)(2 * D * k), C::kIdescPV,
+                               (pv_acc || k > 0) ? 1u : 0u);
                     mma_commit(sready_s + 8u);
                 }
-                mma_commit(afree0 + 8u * tb);
+                if constexpr (!C::kASmem) mma_commit(afree0);
             }
             __syncwarp();
+            pv_owed = false;
         }
     } else if (warp < kFirstSoftmaxWarp) {
         // ------------------------------------------------------------ TMA producer
-        // Order: A(0) [, A(1) with two TMEM copies], items(0), A(next), items(1), ... A group
-        // of unit k goes into shared buffer k % 2 once the softmax has copied the group before
-        // it in that buffer into TMEM. Every wait blocks (try_wait), so the warp takes no issue
-        // slots while it waits.
+        // Order: A(0), items(0), A(1), items(1), ... The A group of unit k goes into shared
+        // buffer k % 2 once the group before it in that buffer is no longer needed: copied into
+        // TMEM by the softmax (encode), or read by the last S product of its unit, which each
+        // softmax warpgroup reports when it sees that S (decode). Every wait blocks
+        // (try_wait), so the warp takes no issue slots while it waits.
         regs_lower<kRegsControl>();
         if (warp == kProducerWarp) {
-            constexpr uint32_t kAhead = C::kABuf == 2 ? 1u : 0u;
             const int64_t G = gridDim.x;
             uint32_t it = 0, na = 0;  // ring items and A groups issued
             int64_t withheld = -1;
             bool ok = true;
             auto issue_a = [&](uint32_t k, int64_t u) -> bool {
                 const int ab = k & 1;
-                if (!warp_wait(asempty0 + 8u * ab, ((k >> 1) & 1) ^ 1, abort_flag, prm.status,
-                               prm.wait_ns))
+                if (!warp_wait((C::kASmem ? afree0 : asempty0) + 8u * ab, ((k >> 1) & 1) ^ 1,
+                               abort_flag, prm.status, prm.wait_ns))
                     return false;
                 const Unit UA = get_unit<D, DEC, LO>(prm, u);
                 if (elect_one()) {
@@ -722,8 +781,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                 ++na;
                 return true;
             };
-            for (uint32_t k = 0; k <= kAhead && ok; ++k)
-                if (blockIdx.x + k * G < prm.n_units) ok = issue_a(k, blockIdx.x + k * G);
+            if (blockIdx.x < prm.n_units) ok = issue_a(0, blockIdx.x);
             uint32_t k = 0;
             for (int64_t u = blockIdx.x; u < prm.n_units && ok; u += G, ++k) {
                 const Unit U = get_unit<D, DEC, LO>(prm, u);
@@ -752,8 +810,8 @@ __global__ void __launch_bounds__(kThreads, 1)
                     }
                     __syncwarp();
                 }
-                const int64_t un = u + (1 + kAhead) * G;
-                if (ok && un < prm.n_units) ok = issue_a(k + 1 + kAhead, un);
+                const int64_t un = u + G;
+                if (ok && un < prm.n_units) ok = issue_a(k + 1, un);
             }
             if (!ok) {
                 // after an abort: wait (bounded) until the newest copy into every buffer landed
@@ -791,16 +849,13 @@ __global__ void __launch_bounds__(kThreads, 1)
         const uint32_t sready_s = sready0 + 16u * wg;
         bool alive = true;
         uint32_t ua = 0, it0 = 0;
-        constexpr bool kAhead = C::kABuf == 2;
-        // Copy this warpgroup's A tile of unit ua (one row per thread) from smem into TMEM
-        // copy ua % kABuf, once the MMAs of the unit that last used that copy are complete.
-        auto copy_a = [&](uint32_t ua_c, int64_t u_c) -> bool {
-            const int n_a = get_unit<D, DEC, LO>(prm, u_c).n_a;
+        // Encode: copy this warpgroup's A tile of unit ua (one row per thread) from smem into
+        // the TMEM copy, once the MMAs of the unit before are complete.
+        auto copy_a = [&](uint32_t ua_c, int n_a) -> bool {
             const int ab = ua_c & 1;
-            const int tb = ua_c % C::kABuf;
             if (!warp_wait(asfull0 + 8u * ab, (ua_c >> 1) & 1, abort_flag, prm.status, prm.wait_ns))
                 return false;
-            if (!warp_wait(afree0 + 8u * tb, ((ua_c / C::kABuf) & 1) ^ 1, abort_flag, prm.status, prm.wait_ns))
+            if (!warp_wait(afree0, (ua_c & 1) ^ 1, abort_flag, prm.status, prm.wait_ns))
                 return false;
             tc_fence_after();
             if (st.s < n_a) {
@@ -817,8 +872,8 @@ __global__ void __launch_bounds__(kThreads, 1)
                         v[4 * k + 2] = x.z;
                         v[4 * k + 3] = x.w;
                     }
-                    const uint32_t acol = tmem + lane_off + C::kColA +
-                                          ((tb * NS + st.s) * C::kANum + h) * (D / 2);
+                    const uint32_t acol =
+                        tmem + lane_off + C::kColA + (st.s * C::kANum + h) * (D / 2);
                     if (D == 16) {
                         tmem_st8(acol, v);
                     } else {
@@ -829,28 +884,48 @@ __global__ void __launch_bounds__(kThreads, 1)
             }
             tmem_wait_st();
             tc_fence_before();
-            mbar_arrive(aready0 + 8u * tb);
+            mbar_arrive(aready0);
             mbar_arrive(asempty0 + 8u * ab);
             return true;
         };
+        // With two O accumulators (decode) the end of a unit (reading O, the stores) runs after
+        // the next unit's first item, whose s_ready also covers the unit's last PV, so it
+        // overlaps that item's round trip to the MMA warp. Every decode unit gives every stream
+        // all of its items (at least one), so that first item always exists.
+        bool owed = false;
+        UnitEnd prev{};
         for (int64_t u = blockIdx.x; u < prm.n_units && alive; u += gridDim.x, ++ua) {
             const Unit U = get_unit<D, DEC, LO>(prm, u);
-            // this unit's A tiles (copied one unit ahead when TMEM holds two copies)
-            if (kAhead) {
-                if (ua == 0 && !copy_a(0, u)) break;
-                if (u + gridDim.x < prm.n_units && !copy_a(ua + 1, u + gridDim.x)) break;
-            } else if (!copy_a(ua, u)) {
-                break;
-            }
+            if constexpr (!C::kASmem)
+                if (!copy_a(ua, U.n_a)) break;
             st.begin(U);
-            while (alive && st.j < st.cnt)
+            st.ob = C::kOBuf == 2 ? (int)(ua & 1) : 0;
+            st.ab = (int)(ua & 1);
+            while (alive && st.j < st.cnt) {
                 alive = softmax_step<D, DEC, SAFE, LO>(st, U, tmem, lane_off, c, c2, sready_s,
-                                                   pready0 + 16u * st.s, empty0, wg_leader, it0,
+                                                   pready0 + 16u * st.s, empty0, afree0, wg_leader,
+                                                   it0,
                                                    abort_flag, prm.status, prm.wait_ns,
                                                    prm.overflow);
-            if (alive)
-                alive = finish_stream<D, DEC, LO>(st, U, prm, tmem, lane_off, r, sready_s, empty0,
-                                              wg_leader, it0, abort_flag);
+                if (owed && alive) {
+                    alive = finish_stream<D, DEC, LO>(st, prev,
+                                                      get_unit<D, DEC, LO>(prm, u - gridDim.x),
+                                                      prm, tmem, lane_off, r, sready_s, empty0,
+                                                      afree0, wg_leader, true, abort_flag);
+                    owed = false;
+                }
+            }
+            if (alive) {
+                const UnitEnd e{st.m, st.l, st.cnt, st.ob, st.ab, it0};
+                if (C::kOBuf == 2 && u + gridDim.x < prm.n_units) {
+                    prev = e;
+                    owed = true;
+                } else {
+                    alive = finish_stream<D, DEC, LO>(st, e, U, prm, tmem, lane_off, r, sready_s,
+                                                      empty0, afree0, wg_leader, false, abort_flag);
+                }
+            }
+            st.ph0 += (uint32_t)st.cnt;
             it0 += U.n_items;
         }
         if (!SAFE && __any_sync(0xffffffffu, st.over) && lane == 0) *prm.overflow = 1;
@@ -904,7 +979,7 @@ PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
 
 // 3D bf16 map over [z, rows, D] (D innermost) with a box of box_rows x D. `swizzled` picks
 // the swizzle matching one D-wide row (MMA operand tiles); otherwise rows are stored plain
-// (A tiles, which the softmax threads copy into TMEM row by row).
+// (the encode's A tiles, which the softmax threads copy into TMEM row by row).
 bool make_map(CUtensorMap* m, const void* base, int64_t D, int64_t rows, int64_t z,
               uint32_t box_rows, bool swizzled) {
     auto fn = encode_fn();
@@ -1042,7 +1117,8 @@ cudaError_t tc_decode(const Plan& p, const void* K, float scale, void* Y, char* 
                       cudaStream_t st, float* lse, bool lo) {
     CUtensorMap ma, mb, mc, ml;
     lo = lo && p.D <= 32;
-    if (!make_map(&ma, K, p.D, p.N, p.BH, kTileRows, false) ||
+    // the decode's MMAs read the token tiles from shared memory: swizzled like the ring tiles
+    if (!make_map(&ma, K, p.D, p.N, p.BH, kTileRows, true) ||
         !make_map(&mb, ws + p.off_qop, p.D, p.M, p.BH, item_rows<true>(p.D, lo), true) ||
         !make_map(&mc, ws + p.off_zop, p.D, p.M, p.BH, item_rows<true>(p.D, lo), true))
         return cudaErrorInvalidValue;
