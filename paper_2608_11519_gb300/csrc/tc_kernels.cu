@@ -86,8 +86,9 @@ struct Cfg {
     // score products), double-buffered so the next unit's tiles land during this one, and
     // nothing copies them. Where TMEM has the room (D <= 32) the decode also keeps two O
     // accumulators per stream, one per unit parity, so a unit's epilogue can wait until the
-    // next unit's first item is under way.
-    static constexpr int kItem = D == 64 ? 32 : ((DEC || LO) ? 64 : 80);
+    // next unit's first item is under way; at D = 64 the columns instead widen its items from
+    // 32 to 48 routes (S 4 x 48 + O 4 x 64 columns).
+    static constexpr int kItem = D == 64 ? (DEC ? 48 : 32) : ((DEC || LO) ? 64 : 80);
     static constexpr int B = 1;                               // score buffers per stream
     static constexpr bool kASmem = DEC;                       // A read by the MMA from smem
     static constexpr int kABuf = DEC ? 0 : 1;                 // TMEM copies of the A tiles
@@ -447,6 +448,9 @@ __device__ __forceinline__ bool softmax_step(SoftmaxStream& S, const Unit& U, ui
     if constexpr (C::kItem == 80) {
         tmem_st32(scol, pr);
         tmem_st8(scol + 32, pr + 32);
+    } else if constexpr (C::kItem == 48) {
+        tmem_st16(scol, pr);
+        tmem_st8(scol + 16, pr + 16);
     } else if constexpr (C::kItem == 64) {
         tmem_st32(scol, pr);
     } else {
