@@ -78,20 +78,23 @@ struct Cfg {
     static constexpr bool kLoA = LO && !DEC;  // encode of call 2: A = Q as hi and lo tiles
     static constexpr bool kLoB = LO && DEC;   // decode: every item also carries Q's lo tile
     static constexpr int kANum = kLoA ? 2 : 1;  // A tiles per stream
-    // Where the A tiles live. The encode's units are long (hundreds of items): its A tiles are
-    // copied into TMEM once per unit (`ts` score products), and the single copy leaves the
-    // columns that widen its items to 80 rows (64 with the lo tile too): fewer per-item round
-    // trips per token. The decode's units are only M/64 items, so per-unit costs show: its A
-    // tiles stay in shared memory where the TMA puts them (swizzled like the ring tiles; `ss`
-    // score products), double-buffered so the next unit's tiles land during this one, and
+    // Where the A tiles live. The encode's units are long (hundreds of items): at D <= 32 its A
+    // tiles are copied into TMEM once per unit (`ts` score products), and the single copy leaves
+    // the columns that widen its items to 80 rows (64 with the lo tile too): fewer per-item
+    // round trips per token. The decode's units are only M/64 items, so per-unit costs show:
+    // its A tiles stay in shared memory where the TMA puts them (swizzled like the ring tiles;
+    // `ss` score products), double-buffered so the next unit's tiles land during this one, and
     // nothing copies them. Where TMEM has the room (D <= 32) the decode also keeps two O
     // accumulators per stream, one per unit parity, so a unit's epilogue can wait until the
     // next unit's first item is under way; at D = 64 the columns instead widen its items from
-    // 32 to 48 routes (S 4 x 48 + O 4 x 64 columns).
-    static constexpr int kItem = D == 64 ? (DEC ? 48 : 32) : ((DEC || LO) ? 64 : 80);
+    // 32 to 48 routes (S 4 x 48 + O 4 x 64 columns). The encode at D = 64 also reads its A
+    // tiles from shared memory (one buffer: its units are long), and the columns a TMEM copy
+    // would take widen its items from 32 to 64 tokens (S 4 x 64 + O 4 x 64).
+    static constexpr bool kASmem = DEC || D == 64;            // A read by the MMA from smem
+    static constexpr int kItem = D == 64 ? (DEC ? 48 : 64) : ((DEC || LO) ? 64 : 80);
     static constexpr int B = 1;                               // score buffers per stream
-    static constexpr bool kASmem = DEC;                       // A read by the MMA from smem
-    static constexpr int kABuf = DEC ? 0 : 1;                 // TMEM copies of the A tiles
+    static constexpr int kABuf = kASmem ? 0 : 1;              // TMEM copies of the A tiles
+    static constexpr int kABufS = (kASmem && !DEC) ? 1 : 2;   // shared-memory A buffers
     static constexpr int kOBuf = (DEC && D <= 32) ? 2 : 1;    // O accumulators per stream
     static constexpr int kGroup = NS * kTileRows;     // resident rows per work unit
     static constexpr int kStages = D == 64 ? 8 : (kItem == 32 ? 16 : 8);  // multiple of 4
@@ -114,7 +117,7 @@ struct Cfg {
     //           needs this item's P (p_ready counts every warp of the warpgroup), o_done of the
     //           next unit needs that unit's P.
     static constexpr int kNumBars = 2 * kStages + 8 + 4 * NS;
-    static constexpr int kData = 2 * kABytes + kStages * kStage;
+    static constexpr int kData = kABufS * kABytes + kStages * kStage;
     static constexpr int kNeed = 1024 + kData + kNumBars * 8 + 16;
     // at least 120 KB so that one CTA owns an SM and its 512 TMEM columns
     static constexpr int kSmem = kNeed > 122880 ? kNeed : 122880;
@@ -244,7 +247,7 @@ struct SoftmaxStream {
     int par;        // token parity of the stream's items in this unit (s / n_a)
     int cnt, j;     // items of the stream in this unit, items done
     int ob;         // O accumulator of this unit (0, or the unit's parity with two)
-    int ab;         // shared-memory A buffer of this unit (the unit's parity)
+    int ab;         // shared-memory A buffer of this unit
     float m, l;     // reference max (base 2, scaled) and running sum
     uint32_t ph0;   // s_ready phases completed in earlier units (one per item)
     uint32_t od;    // o_done phases completed in earlier units (one per unit with items)
@@ -573,8 +576,8 @@ __global__ void __launch_bounds__(kThreads, 1)
     extern __shared__ uint8_t smem_raw[];
     uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                                ~static_cast<uintptr_t>(1023));
-    uint8_t* abuf = smem;                   // 2 x NS x kANum unswizzled A tiles
-    uint8_t* ring = smem + 2 * C::kABytes;  // kStages x (B tile, C tile[, lo tile]), swizzled
+    uint8_t* abuf = smem;                         // kABufS x NS x kANum A tiles
+    uint8_t* ring = smem + C::kABufS * C::kABytes;  // kStages x (B tile, C tile[, lo tile]), swizzled
     uint64_t* bars = reinterpret_cast<uint64_t*>(ring + C::kStages * C::kStage);
     uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + C::kNumBars);
     volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
@@ -657,11 +660,12 @@ __global__ void __launch_bounds__(kThreads, 1)
             const Unit U = get_unit<D, DEC, LO>(prm, u);
             const int a = s % U.n_a;
             const int par = s / U.n_a;
-            // the unit's A tile: shared-memory buffer ua % 2 as the TMA wrote it (decode), or
-            // the TMEM copy the softmax made of it (encode)
-            const int ab = ua & 1;
-            if (!warp_wait(C::kASmem ? asfull0 + 8u * ab : aready0, C::kASmem ? (ua >> 1) & 1 : ua & 1,
-                           abort_flag, prm.status, prm.wait_ns))
+            // the unit's A tile: shared-memory buffer ua % kABufS as the TMA wrote it (decode,
+            // and the encode at D = 64), or the TMEM copy the softmax made of it
+            const int ab = ua % C::kABufS;
+            if (!warp_wait(C::kASmem ? asfull0 + 8u * ab : aready0,
+                           C::kASmem ? (ua / C::kABufS) & 1 : ua & 1, abort_flag, prm.status,
+                           prm.wait_ns))
                 break;
             tc_fence_after();
             const uint64_t dA = dA0 + ((uint64_t)(ab * C::kABytes + a * C::kATile) >> 4);
@@ -754,10 +758,10 @@ __global__ void __launch_bounds__(kThreads, 1)
     } else if (warp < kFirstSoftmaxWarp) {
         // ------------------------------------------------------------ TMA producer
         // Order: A(0), items(0), A(1), items(1), ... The A group of unit k goes into shared
-        // buffer k % 2 once the group before it in that buffer is no longer needed: copied into
-        // TMEM by the softmax (encode), or read by the last S product of its unit, which each
-        // softmax warpgroup reports when it sees that S (decode). Every wait blocks
-        // (try_wait), so the warp takes no issue slots while it waits.
+        // buffer k % kABufS once the group before it in that buffer is no longer needed: copied
+        // into TMEM by the softmax, or (A read from shared memory) read by the last S product of
+        // its unit, which each softmax warpgroup reports when it sees that S. Every wait
+        // blocks (try_wait), so the warp takes no issue slots while it waits.
         regs_lower<kRegsControl>();
         if (warp == kProducerWarp) {
             const int64_t G = gridDim.x;
@@ -765,9 +769,9 @@ __global__ void __launch_bounds__(kThreads, 1)
             int64_t withheld = -1;
             bool ok = true;
             auto issue_a = [&](uint32_t k, int64_t u) -> bool {
-                const int ab = k & 1;
-                if (!warp_wait((C::kASmem ? afree0 : asempty0) + 8u * ab, ((k >> 1) & 1) ^ 1,
-                               abort_flag, prm.status, prm.wait_ns))
+                const int ab = k % C::kABufS;
+                if (!warp_wait((C::kASmem ? afree0 : asempty0) + 8u * ab,
+                               ((k / C::kABufS) & 1) ^ 1, abort_flag, prm.status, prm.wait_ns))
                     return false;
                 const Unit UA = get_unit<D, DEC, LO>(prm, u);
                 if (elect_one()) {
@@ -827,9 +831,9 @@ __global__ void __launch_bounds__(kThreads, 1)
                            globaltimer_ns() - t0 < prm.wait_ns) {
                     }
                 }
-                for (uint32_t b = 0; b < 2 && b < na; ++b) {
-                    const uint32_t y = na - 1 - ((na - 1 - b) % 2);
-                    while (!mbar_try_wait(asfull0 + 8u * b, (y >> 1) & 1) &&
+                for (uint32_t b = 0; b < (uint32_t)C::kABufS && b < na; ++b) {
+                    const uint32_t y = na - 1 - ((na - 1 - b) % C::kABufS);
+                    while (!mbar_try_wait(asfull0 + 8u * b, (y / C::kABufS) & 1) &&
                            globaltimer_ns() - t0 < prm.wait_ns) {
                     }
                 }
@@ -904,7 +908,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                 if (!copy_a(ua, U.n_a)) break;
             st.begin(U);
             st.ob = C::kOBuf == 2 ? (int)(ua & 1) : 0;
-            st.ab = (int)(ua & 1);
+            st.ab = (int)(ua % C::kABufS);
             while (alive && st.j < st.cnt) {
                 alive = softmax_step<D, DEC, SAFE, LO>(st, U, tmem, lane_off, c, c2, sready_s,
                                                    pready0 + 16u * st.s, empty0, afree0, wg_leader,
@@ -1045,6 +1049,13 @@ cudaError_t launch_d(int64_t D, bool lo, const CUtensorMap& a, const CUtensorMap
 
 }  // namespace
 
+// Whether the MMAs of the encode or decode read the A tiles from shared memory (then the A
+// tensor map is swizzled like the ring tiles) rather than from a TMEM copy.
+template <bool DEC>
+bool a_in_smem(int64_t D) {
+    return D == 16 ? Cfg<16, DEC>::kASmem : (D == 32 ? Cfg<32, DEC>::kASmem : Cfg<64, DEC>::kASmem);
+}
+
 // Streamed rows per item (the TMA box height of the ring tiles) of the encode or decode.
 template <bool DEC>
 uint32_t item_rows(int64_t D, bool lo = false) {
@@ -1090,7 +1101,8 @@ cudaError_t tc_encode(const Plan& p, int call, const void* k, const void* v, con
         a_src = ws + p.off_qop;
         a_z = p.BH;
     }
-    if (!make_map(&ma, a_src, p.D, p.M, a_z, kTileRows, false) ||
+    // at D = 64 the encode's MMAs read the A tiles from shared memory: swizzled like the ring
+    if (!make_map(&ma, a_src, p.D, p.M, a_z, kTileRows, a_in_smem<false>(p.D)) ||
         !make_map(&mb, k, p.D, p.N, p.BH, item_rows<false>(p.D, lo), true) ||
         !make_map(&mc, v, p.D, p.N, p.BH, item_rows<false>(p.D, lo), true))
         return cudaErrorInvalidValue;
@@ -1122,7 +1134,7 @@ cudaError_t tc_decode(const Plan& p, const void* K, float scale, void* Y, char* 
     CUtensorMap ma, mb, mc, ml;
     lo = lo && p.D <= 32;
     // the decode's MMAs read the token tiles from shared memory: swizzled like the ring tiles
-    if (!make_map(&ma, K, p.D, p.N, p.BH, kTileRows, true) ||
+    if (!make_map(&ma, K, p.D, p.N, p.BH, kTileRows, a_in_smem<true>(p.D)) ||
         !make_map(&mb, ws + p.off_qop, p.D, p.M, p.BH, item_rows<true>(p.D, lo), true) ||
         !make_map(&mc, ws + p.off_zop, p.D, p.M, p.BH, item_rows<true>(p.D, lo), true))
         return cudaErrorInvalidValue;
