@@ -14,18 +14,18 @@
 //
 // Work is cut into four TMEM "streams". Stream s owns one score buffer of 128 x kItem fp32
 // (S is rewritten in place as bf16 P, the A operand of the PV product) and a 128 x D fp32
-// accumulator O, and reads one resident A tile kept in TMEM, so that S = A * B^T is a
-// TMEM x SMEM product. With two TMEM copies of the A tiles (the decode, D <= 32) the softmax
-// copies the next unit's tiles while it works on the current unit, so a unit boundary does
-// not drain the pipeline. Roles (24 warps, a register split gives warpgroups 0 and 1 40
-// registers per thread and the four softmax warpgroups 96):
+// accumulator O (two in the decode at D <= 32, one per unit parity), and reads one resident A
+// tile in shared memory, so that S = A * B^T is a SMEM x SMEM product and all TMEM columns go
+// to S and O. The decode double-buffers its A tiles, so the next unit's tiles land while the
+// current unit runs. Roles (24 warps, a register split gives warpgroups 0 and 1 40 registers
+// per thread and the four softmax warpgroups 96):
 //   warps 0..3    one MMA warp per stream: for item j, the PV of item j-1 and the S of
 //                 item j, then one commit, all issued from one elected lane (a commit
 //                 stalls only the warp that issues it)
-//   warp 4        the TMA producer (A tiles, unswizzled; the item ring, swizzled K/V or
-//                 Q/Z), with blocking waits; warps 5..7 only take part in the split
-//   warps 8..23   four softmax warpgroups; warpgroup s serves stream s and copies its A tile
-//                 from smem into TMEM (four warps per SMSP hide each other's latencies)
+//   warp 4        the TMA producer (A tiles and the item ring, K/V or Q/Z, all swizzled to
+//                 one D-wide row), with blocking waits; warps 5..7 only take part in the split
+//   warps 8..23   four softmax warpgroups; warpgroup s serves stream s (four warps per SMSP
+//                 hide each other's latencies)
 // Each launch is a pair of kernels on the stream. The fast kernel keeps, per row, the first
 // score of the unit as its reference m (any score of the row is a valid reference: it alone
 // adds 2^0 to the sum) and computes P = 2^(c S - m) with no maximum pass, storing P chunk by
@@ -78,45 +78,38 @@ struct Cfg {
     static constexpr bool kLoA = LO && !DEC;  // encode of call 2: A = Q as hi and lo tiles
     static constexpr bool kLoB = LO && DEC;   // decode: every item also carries Q's lo tile
     static constexpr int kANum = kLoA ? 2 : 1;  // A tiles per stream
-    // Where the A tiles live. The encode's units are long (hundreds of items): at D <= 32 its A
-    // tiles are copied into TMEM once per unit (`ts` score products), and the single copy leaves
-    // the columns that widen its items to 80 rows (64 with the lo tile too): fewer per-item
-    // round trips per token. The decode's units are only M/64 items, so per-unit costs show:
-    // its A tiles stay in shared memory where the TMA puts them (swizzled like the ring tiles;
-    // `ss` score products), double-buffered so the next unit's tiles land during this one, and
-    // nothing copies them. Where TMEM has the room (D <= 32) the decode also keeps two O
-    // accumulators per stream, one per unit parity, so a unit's epilogue can wait until the
-    // next unit's first item is under way; at D = 64 the columns instead widen its items from
-    // 32 to 48 routes (S 4 x 48 + O 4 x 64 columns). The encode at D = 64 also reads its A
-    // tiles from shared memory (one buffer: its units are long), and the columns a TMEM copy
-    // would take widen its items from 32 to 64 tokens (S 4 x 64 + O 4 x 64).
-    static constexpr bool kASmem = DEC || D == 64;            // A read by the MMA from smem
-    static constexpr int kItem = D == 64 ? (DEC ? 48 : 64) : ((DEC || LO) ? 64 : 80);
-    static constexpr int B = 1;                               // score buffers per stream
-    static constexpr int kABuf = kASmem ? 0 : 1;              // TMEM copies of the A tiles
-    static constexpr int kABufS = (kASmem && !DEC) ? 1 : 2;   // shared-memory A buffers
+    // The A tiles (the route tiles in the encode, the token tiles in the decode) stay in shared
+    // memory where the TMA puts them, swizzled like the ring tiles, and the MMAs read them there
+    // (`ss` score products); nothing copies them into TMEM, so all 512 columns go to the score
+    // tiles and accumulators. The encode's units are long (hundreds of items): one A buffer,
+    // and items of 96 tokens (64 at D = 64: S 4 x 64 + O 4 x 64 columns), so the per-item round
+    // trip is paid once per 96 tokens. The decode's units are only M/64 items, so per-unit costs
+    // show: its A tiles are double-buffered so the next unit's land during this one, and where
+    // TMEM has the room (D <= 32) it keeps two O accumulators per stream, one per unit parity,
+    // so that a unit's epilogue can wait until the next unit's first item is under way; at
+    // D = 64 the columns instead widen its items to 48 routes (S 4 x 48 + O 4 x 64).
+    static constexpr int kItem = D == 64 ? (DEC ? 48 : 64) : (DEC ? 64 : 96);
+    static constexpr int B = 1;                         // score buffers per stream
+    static constexpr int kABufS = DEC ? 2 : 1;          // shared-memory A buffers
     static constexpr int kOBuf = (DEC && D <= 32) ? 2 : 1;    // O accumulators per stream
     static constexpr int kGroup = NS * kTileRows;     // resident rows per work unit
-    static constexpr int kStages = D == 64 ? 8 : (kItem == 32 ? 16 : 8);  // multiple of 4
+    static constexpr int kStages = 8;                 // ring items (>= 2 B NS)
     static constexpr int kATile = kTileRows * D * 2;  // one 128-row operand tile
     static constexpr int kABytes = NS * kANum * kATile;
     static constexpr int kItemTile = kItem * D * 2;
     static constexpr int kStage = (kLoB ? 3 : 2) * kItemTile;
     static constexpr uint32_t kSwz = D == 16 ? kSw32 : (D == 32 ? kSw64 : kSw128);
     static constexpr uint32_t kSBO = 8 * D * 2;  // bytes between 8-row groups
-    // barriers: full[S], empty[S], asmem_full[2], asmem_empty[2], a_ready[2], a_free[2],
-    //           sync[NS][2] = {s_ready, o_done} per stream (S of an item complete; every PV
-    //           of the stream's unit complete), p_ready[NS][2] (slot 0 used). The encode's A
-    //           tiles go asmem_full -> softmax copy into TMEM -> asmem_empty and a_ready, and
-    //           a_free (one commit per MMA warp after a unit's last MMA) frees the TMEM copy. In
-    //           the decode the MMAs wait on asmem_full themselves, and a_free counts one arrive
-    //           per softmax warpgroup once it has seen the unit's last S. With two O
-    //           accumulators a decode unit's last PV goes out with the next unit's first S, so
+    // barriers: full[S], empty[S], a_full[2] (a unit's A tiles landed), a_free[2] (one arrive
+    //           per softmax warpgroup once it has seen the unit's last S: the buffer may be
+    //           refilled), sync[NS][2] = {s_ready, o_done} per stream (S of an item complete;
+    //           every PV of the stream's unit complete), p_ready[NS][2] (slot 0 used). With two
+    //           O accumulators a decode unit's last PV goes out with the next unit's first S, so
     //           o_done is committed only for a CTA's last unit. A barrier that a warp waits on
     //           by parity never runs two phases ahead of that warp: s_ready of the next item
     //           needs this item's P (p_ready counts every warp of the warpgroup), o_done of the
-    //           next unit needs that unit's P.
-    static constexpr int kNumBars = 2 * kStages + 8 + 4 * NS;
+    //           next unit needs that unit's P, a_full of unit k + 2 needs a_free of unit k.
+    static constexpr int kNumBars = 2 * kStages + 4 + 4 * NS;
     static constexpr int kData = kABufS * kABytes + kStages * kStage;
     static constexpr int kNeed = 1024 + kData + kNumBars * 8 + 16;
     // at least 120 KB so that one CTA owns an SM and its 512 TMEM columns
@@ -124,14 +117,12 @@ struct Cfg {
     static constexpr uint32_t kIdescS = idesc_bf16_f32(128, kItem, false, false);
     static constexpr uint32_t kIdescPV = idesc_bf16_f32(128, D, false, true);
     // TMEM columns
-    static constexpr uint32_t kColS = 0;                  // NS x B x kItem
-    static constexpr uint32_t kColO = NS * B * kItem;         // kOBuf x NS x D
-    static constexpr uint32_t kColA = kColO + kOBuf * NS * D;  // kABuf x NS x kANum tiles x D/2
-    static_assert(kColA + kABuf * NS * kANum * (D / 2) <= kTmemCols, "TMEM budget");
+    static constexpr uint32_t kColS = 0;               // NS x B x kItem
+    static constexpr uint32_t kColO = NS * B * kItem;  // kOBuf x NS x D
+    static_assert(kColO + kOBuf * NS * D <= kTmemCols, "TMEM budget");
     static_assert(kSmem <= 232448, "shared memory budget");
     static_assert(kStages >= 2 * B * NS, "ring depth: the full wait precedes the PV");
     static_assert(B == 1, "the s_ready / o_done protocol has one score buffer per stream");
-    static_assert(kABuf <= 1 && (kABuf == 1) != kASmem, "A: one TMEM copy or shared memory");
 };
 
 struct TcParams {
@@ -383,8 +374,8 @@ __device__ __forceinline__ bool softmax_step(SoftmaxStream& S, const Unit& U, ui
         const int i_old = par + (j - C::B) * U.n_par;
         mbar_arrive(empty0 + 8u * ((it0 + i_old) % C::kStages));
     }
-    // decode: the unit's last S is complete, so its MMAs no longer read the A buffer
-    if (C::kASmem && wg_leader && j == S.cnt - 1) mbar_arrive(afree0 + 8u * S.ab);
+    // the unit's last S is complete, so its MMAs no longer read the A buffer
+    if (wg_leader && j == S.cnt - 1) mbar_arrive(afree0 + 8u * S.ab);
     const int item = par + j * U.n_par;
     const int64_t start = U.item0 + (int64_t)item * C::kItem;
     const int nv = (int)min((int64_t)C::kItem, U.item_end - start);
@@ -454,6 +445,9 @@ __device__ __forceinline__ bool softmax_step(SoftmaxStream& S, const Unit& U, ui
     } else if constexpr (C::kItem == 48) {
         tmem_st16(scol, pr);
         tmem_st8(scol + 16, pr + 16);
+    } else if constexpr (C::kItem == 96) {
+        tmem_st32(scol, pr);
+        tmem_st16(scol + 32, pr + 32);
     } else if constexpr (C::kItem == 64) {
         tmem_st32(scol, pr);
     } else {
@@ -520,8 +514,7 @@ __device__ __forceinline__ bool finish_stream(SoftmaxStream& S, const UnitEnd& E
         for (int d = 0; d < D; ++d) o[d] = __uint_as_float(t[d]);
     } else {
         // (no MMA of this stream read the unit's A tile)
-        if constexpr (C::kASmem)
-            if (wg_leader) mbar_arrive(afree0 + 8u * E.ab);
+        if (wg_leader) mbar_arrive(afree0 + 8u * E.ab);
 #pragma unroll
         for (int d = 0; d < D; ++d) o[d] = 0.f;
     }
@@ -584,13 +577,10 @@ __global__ void __launch_bounds__(kThreads, 1)
 
     const uint32_t full0 = smem_u32(bars);
     const uint32_t empty0 = full0 + 8u * C::kStages;
-    const uint32_t asfull0 = full0 + 8u * (2 * C::kStages);
-    const uint32_t asempty0 = asfull0 + 16u;
-    const uint32_t aready0 = asfull0 + 32u;
-    const uint32_t afree0 = asfull0 + 48u;
-    const uint32_t sready0 = asfull0 + 64u;       // [NS][2]
+    const uint32_t afull0 = full0 + 8u * (2 * C::kStages);
+    const uint32_t afree0 = afull0 + 16u;
+    const uint32_t sready0 = afull0 + 32u;        // [NS][2]
     const uint32_t pready0 = sready0 + 16u * NS;  // [NS][2]
-    constexpr uint32_t kSoftmaxThreads = (kWarps - kFirstSoftmaxWarp) * 32;
 
     const int warp = threadIdx.x >> 5;
     const int lane = threadIdx.x & 31;
@@ -601,9 +591,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             mbar_init(empty0 + 8u * st, NS);
         }
         for (int b = 0; b < 2; ++b) {
-            mbar_init(asfull0 + 8u * b, 1);
-            mbar_init(asempty0 + 8u * b, kSoftmaxThreads);
-            mbar_init(aready0 + 8u * b, kSoftmaxThreads);
+            mbar_init(afull0 + 8u * b, 1);
             mbar_init(afree0 + 8u * b, NS);
         }
         for (int s = 0; s < NS; ++s) {
@@ -660,16 +648,12 @@ __global__ void __launch_bounds__(kThreads, 1)
             const Unit U = get_unit<D, DEC, LO>(prm, u);
             const int a = s % U.n_a;
             const int par = s / U.n_a;
-            // the unit's A tile: shared-memory buffer ua % kABufS as the TMA wrote it (decode,
-            // and the encode at D = 64), or the TMEM copy the softmax made of it
+            // the unit's A tile: shared-memory buffer ua % kABufS as the TMA wrote it
             const int ab = ua % C::kABufS;
-            if (!warp_wait(C::kASmem ? asfull0 + 8u * ab : aready0,
-                           C::kASmem ? (ua / C::kABufS) & 1 : ua & 1, abort_flag, prm.status,
+            if (!warp_wait(afull0 + 8u * ab, (ua / C::kABufS) & 1, abort_flag, prm.status,
                            prm.wait_ns))
                 break;
-            tc_fence_after();
-            const uint64_t dA = dA0 + ((uint64_t)(ab * C::kABytes + a * C::kATile) >> 4);
-            const uint32_t a_tmem = tmem + C::kColA + a * C::kANum * (D / 2);
+            const uint64_t dA = dA0 + ((uint64_t)(ab * C::kABytes + a * C::kANum * C::kATile) >> 4);
             const uint32_t d_o = tmem + C::kColO + ((C::kOBuf == 2 ? ab : 0) * NS + s) * D;
             int j = 0;
             for (int i = 0; i < U.n_items; ++i, ++it) {
@@ -701,19 +685,15 @@ __global__ void __launch_bounds__(kThreads, 1)
                     }
                     const uint64_t ds = dS0 + ((st * C::kStage) >> 4);
 #pragma unroll
-                    for (int k = 0; k < D / 16; ++k) {
-                        if constexpr (C::kASmem)
-                            mma_ss(d_s, dA + (uint64_t)(2 * k), ds + (uint64_t)(2 * k), C::kIdescS,
-                                   k > 0 ? 1u : 0u);
-                        else
-                            mma_ts(d_s, a_tmem + 8 * k, ds + (uint64_t)(2 * k), C::kIdescS,
-                                   k > 0 ? 1u : 0u);
-                    }
+                    for (int k = 0; k < D / 16; ++k)
+                        mma_ss(d_s, dA + (uint64_t)(2 * k), ds + (uint64_t)(2 * k), C::kIdescS,
+                               k > 0 ? 1u : 0u);
                     if constexpr (C::kLoA) {
-                        // S += lo(Q) K^T: the lo tile follows the hi tile in TMEM
+                        // S += lo(Q) K^T: the lo tile follows the hi tile
+                        const uint64_t dAl = dA + (uint64_t)(C::kATile >> 4);
 #pragma unroll
                         for (int k = 0; k < D / 16; ++k)
-                            mma_ts(d_s, a_tmem + D / 2 + 8 * k, ds + (uint64_t)(2 * k), C::kIdescS,
+                            mma_ss(d_s, dAl + (uint64_t)(2 * k), ds + (uint64_t)(2 * k), C::kIdescS,
                                    1u);
                     }
                     if constexpr (C::kLoB) {
@@ -736,8 +716,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             if (!ok) break;
             // decode with two O accumulators: the last PV goes out with the next unit's first S
             if (C::kOBuf == 2 && u + gridDim.x < prm.n_units) continue;
-            // the PV of the unit's last item, then o_done: O is final for the softmax; and
-            // (encode) a_free: this stream's MMAs no longer read the unit's TMEM A copy
+            // the PV of the unit's last item, then o_done: O is final for the softmax
             if (pv_owed && !warp_wait(pready_s, pc & 1, abort_flag, prm.status, prm.wait_ns)) break;
             if (pv_owed) ++pc;
             tc_fence_after();
@@ -750,7 +729,6 @@ __global__ void __launch_bounds__(kThreads, 1)
                                (pv_acc || k > 0) ? 1u : 0u);
                     mma_commit(sready_s + 8u);
                 }
-                if constexpr (!C::kASmem) mma_commit(afree0);
             }
             __syncwarp();
             pv_owed = false;
@@ -758,10 +736,9 @@ __global__ void __launch_bounds__(kThreads, 1)
     } else if (warp < kFirstSoftmaxWarp) {
         // ------------------------------------------------------------ TMA producer
         // Order: A(0), items(0), A(1), items(1), ... The A group of unit k goes into shared
-        // buffer k % kABufS once the group before it in that buffer is no longer needed: copied
-        // into TMEM by the softmax, or (A read from shared memory) read by the last S product of
-        // its unit, which each softmax warpgroup reports when it sees that S. Every wait
-        // blocks (try_wait), so the warp takes no issue slots while it waits.
+        // buffer k % kABufS once the group before it in that buffer has been read by the last S
+        // product of its unit, which each softmax warpgroup reports when it sees that S. Every
+        // wait blocks (try_wait), so the warp takes no issue slots while it waits.
         regs_lower<kRegsControl>();
         if (warp == kProducerWarp) {
             const int64_t G = gridDim.x;
@@ -770,19 +747,19 @@ __global__ void __launch_bounds__(kThreads, 1)
             bool ok = true;
             auto issue_a = [&](uint32_t k, int64_t u) -> bool {
                 const int ab = k % C::kABufS;
-                if (!warp_wait((C::kASmem ? afree0 : asempty0) + 8u * ab,
+                if (!warp_wait(afree0 + 8u * ab,
                                ((k / C::kABufS) & 1) ^ 1, abort_flag, prm.status, prm.wait_ns))
                     return false;
                 const Unit UA = get_unit<D, DEC, LO>(prm, u);
                 if (elect_one()) {
-                    mbar_expect_tx(asfull0 + 8u * ab, UA.n_a * C::kANum * C::kATile);
+                    mbar_expect_tx(afull0 + 8u * ab, UA.n_a * C::kANum * C::kATile);
                     for (int a = 0; a < UA.n_a; ++a) {
                         uint8_t* dst = abuf + ab * C::kABytes + a * C::kANum * C::kATile;
                         tma_load_3d(smem_u32(dst), &tmA, 0, UA.rowA0 + a * kTileRows, UA.zA,
-                                    asfull0 + 8u * ab);
+                                    afull0 + 8u * ab);
                         if constexpr (C::kLoA)
                             tma_load_3d(smem_u32(dst + C::kATile), &tmL, 0,
-                                        UA.rowA0 + a * kTileRows, UA.zA, asfull0 + 8u * ab);
+                                        UA.rowA0 + a * kTileRows, UA.zA, afull0 + 8u * ab);
                     }
                 }
                 __syncwarp();
@@ -833,7 +810,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                 }
                 for (uint32_t b = 0; b < (uint32_t)C::kABufS && b < na; ++b) {
                     const uint32_t y = na - 1 - ((na - 1 - b) % C::kABufS);
-                    while (!mbar_try_wait(asfull0 + 8u * b, (y / C::kABufS) & 1) &&
+                    while (!mbar_try_wait(afull0 + 8u * b, (y / C::kABufS) & 1) &&
                            globaltimer_ns() - t0 < prm.wait_ns) {
                     }
                 }
@@ -857,45 +834,6 @@ __global__ void __launch_bounds__(kThreads, 1)
         const uint32_t sready_s = sready0 + 16u * wg;
         bool alive = true;
         uint32_t ua = 0, it0 = 0;
-        // Encode: copy this warpgroup's A tile of unit ua (one row per thread) from smem into
-        // the TMEM copy, once the MMAs of the unit before are complete.
-        auto copy_a = [&](uint32_t ua_c, int n_a) -> bool {
-            const int ab = ua_c & 1;
-            if (!warp_wait(asfull0 + 8u * ab, (ua_c >> 1) & 1, abort_flag, prm.status, prm.wait_ns))
-                return false;
-            if (!warp_wait(afree0, (ua_c & 1) ^ 1, abort_flag, prm.status, prm.wait_ns))
-                return false;
-            tc_fence_after();
-            if (st.s < n_a) {
-#pragma unroll
-                for (int h = 0; h < C::kANum; ++h) {  // the hi tile, then (LO) the lo tile
-                    const uint4* src = reinterpret_cast<const uint4*>(
-                        abuf + ab * C::kABytes + (st.s * C::kANum + h) * C::kATile + r * D * 2);
-                    uint32_t v[D / 2];
-#pragma unroll
-                    for (int k = 0; k < D / 8; ++k) {
-                        const uint4 x = src[k];
-                        v[4 * k] = x.x;
-                        v[4 * k + 1] = x.y;
-                        v[4 * k + 2] = x.z;
-                        v[4 * k + 3] = x.w;
-                    }
-                    const uint32_t acol =
-                        tmem + lane_off + C::kColA + (st.s * C::kANum + h) * (D / 2);
-                    if (D == 16) {
-                        tmem_st8(acol, v);
-                    } else {
-#pragma unroll
-                        for (int k = 0; k < D / 32; ++k) tmem_st16(acol + 16 * k, v + 16 * k);
-                    }
-                }
-            }
-            tmem_wait_st();
-            tc_fence_before();
-            mbar_arrive(aready0);
-            mbar_arrive(asempty0 + 8u * ab);
-            return true;
-        };
         // With two O accumulators (decode) the end of a unit (reading O, the stores) runs after
         // the next unit's first item, whose s_ready also covers the unit's last PV, so it
         // overlaps that item's round trip to the MMA warp. Every decode unit gives every stream
@@ -904,8 +842,6 @@ __global__ void __launch_bounds__(kThreads, 1)
         UnitEnd prev{};
         for (int64_t u = blockIdx.x; u < prm.n_units && alive; u += gridDim.x, ++ua) {
             const Unit U = get_unit<D, DEC, LO>(prm, u);
-            if constexpr (!C::kASmem)
-                if (!copy_a(ua, U.n_a)) break;
             st.begin(U);
             st.ob = C::kOBuf == 2 ? (int)(ua & 1) : 0;
             st.ab = (int)(ua % C::kABufS);
@@ -985,21 +921,19 @@ PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
     return fn;
 }
 
-// 3D bf16 map over [z, rows, D] (D innermost) with a box of box_rows x D. `swizzled` picks
-// the swizzle matching one D-wide row (MMA operand tiles); otherwise rows are stored plain
-// (the encode's A tiles, which the softmax threads copy into TMEM row by row).
+// 3D bf16 map over [z, rows, D] (D innermost) with a box of box_rows x D, swizzled to match
+// one D-wide row (the layout the MMA descriptors of every operand tile assume).
 bool make_map(CUtensorMap* m, const void* base, int64_t D, int64_t rows, int64_t z,
-              uint32_t box_rows, bool swizzled) {
+              uint32_t box_rows) {
     auto fn = encode_fn();
     if (!fn) return false;
     cuuint64_t dims[3] = {(cuuint64_t)D, (cuuint64_t)rows, (cuuint64_t)z};
     cuuint64_t strides[2] = {(cuuint64_t)(D * 2), (cuuint64_t)(rows * D * 2)};
     cuuint32_t box[3] = {(cuuint32_t)D, box_rows, 1};
     cuuint32_t estr[3] = {1, 1, 1};
-    CUtensorMapSwizzle sw = CU_TENSOR_MAP_SWIZZLE_NONE;
-    if (swizzled)
-        sw = D == 16 ? CU_TENSOR_MAP_SWIZZLE_32B
-                     : (D == 32 ? CU_TENSOR_MAP_SWIZZLE_64B : CU_TENSOR_MAP_SWIZZLE_128B);
+    const CUtensorMapSwizzle sw =
+        D == 16 ? CU_TENSOR_MAP_SWIZZLE_32B
+                : (D == 32 ? CU_TENSOR_MAP_SWIZZLE_64B : CU_TENSOR_MAP_SWIZZLE_128B);
     return fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(base), dims, strides, box,
               estr, CU_TENSOR_MAP_INTERLEAVE_NONE, sw, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
               CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
@@ -1049,13 +983,6 @@ cudaError_t launch_d(int64_t D, bool lo, const CUtensorMap& a, const CUtensorMap
 
 }  // namespace
 
-// Whether the MMAs of the encode or decode read the A tiles from shared memory (then the A
-// tensor map is swizzled like the ring tiles) rather than from a TMEM copy.
-template <bool DEC>
-bool a_in_smem(int64_t D) {
-    return D == 16 ? Cfg<16, DEC>::kASmem : (D == 32 ? Cfg<32, DEC>::kASmem : Cfg<64, DEC>::kASmem);
-}
-
 // Streamed rows per item (the TMA box height of the ring tiles) of the encode or decode.
 template <bool DEC>
 uint32_t item_rows(int64_t D, bool lo = false) {
@@ -1101,13 +1028,12 @@ cudaError_t tc_encode(const Plan& p, int call, const void* k, const void* v, con
         a_src = ws + p.off_qop;
         a_z = p.BH;
     }
-    // at D = 64 the encode's MMAs read the A tiles from shared memory: swizzled like the ring
-    if (!make_map(&ma, a_src, p.D, p.M, a_z, kTileRows, a_in_smem<false>(p.D)) ||
-        !make_map(&mb, k, p.D, p.N, p.BH, item_rows<false>(p.D, lo), true) ||
-        !make_map(&mc, v, p.D, p.N, p.BH, item_rows<false>(p.D, lo), true))
+    if (!make_map(&ma, a_src, p.D, p.M, a_z, kTileRows) ||
+        !make_map(&mb, k, p.D, p.N, p.BH, item_rows<false>(p.D, lo)) ||
+        !make_map(&mc, v, p.D, p.N, p.BH, item_rows<false>(p.D, lo)))
         return cudaErrorInvalidValue;
     ml = ma;
-    if (lo && !make_map(&ml, ws + p.off_qlo, p.D, p.M, a_z, kTileRows, false))
+    if (lo && !make_map(&ml, ws + p.off_qlo, p.D, p.M, a_z, kTileRows))
         return cudaErrorInvalidValue;
     TcParams prm{};
     prm.BH = p.BH;
@@ -1133,13 +1059,12 @@ cudaError_t tc_decode(const Plan& p, const void* K, float scale, void* Y, char* 
                       cudaStream_t st, float* lse, bool lo) {
     CUtensorMap ma, mb, mc, ml;
     lo = lo && p.D <= 32;
-    // the decode's MMAs read the token tiles from shared memory: swizzled like the ring tiles
-    if (!make_map(&ma, K, p.D, p.N, p.BH, kTileRows, a_in_smem<true>(p.D)) ||
-        !make_map(&mb, ws + p.off_qop, p.D, p.M, p.BH, item_rows<true>(p.D, lo), true) ||
-        !make_map(&mc, ws + p.off_zop, p.D, p.M, p.BH, item_rows<true>(p.D, lo), true))
+    if (!make_map(&ma, K, p.D, p.N, p.BH, kTileRows) ||
+        !make_map(&mb, ws + p.off_qop, p.D, p.M, p.BH, item_rows<true>(p.D, lo)) ||
+        !make_map(&mc, ws + p.off_zop, p.D, p.M, p.BH, item_rows<true>(p.D, lo)))
         return cudaErrorInvalidValue;
     ml = ma;
-    if (lo && !make_map(&ml, ws + p.off_qlo, p.D, p.M, p.BH, item_rows<true>(p.D, lo), true))
+    if (lo && !make_map(&ml, ws + p.off_qlo, p.D, p.M, p.BH, item_rows<true>(p.D, lo)))
         return cudaErrorInvalidValue;
     TcParams prm{};
     prm.BH = p.BH;

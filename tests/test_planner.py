@@ -19,7 +19,7 @@ HARNESS = r"""
 
 // tokens per encode item and routes per group, as the tensor-core encode defines them
 namespace flarepp {
-int64_t tc_encode_item_rows(int64_t D) { return D == 64 ? 32 : 80; }
+int64_t tc_encode_item_rows(int64_t D) { return D == 64 ? 64 : 96; }
 int64_t tc_group_rows(int64_t D) { (void)D; return 512; }
 }  // namespace flarepp
 
@@ -64,7 +64,7 @@ int main() {
     };
     for (int64_t B : {1, 2, 4, 16, 64})
         for (int64_t H : {1, 3, 8, 16})
-            for (int64_t N : {1, 79, 80, 81, 5000, 16384, 100000, 1 << 20, (1 << 20) + 17})
+            for (int64_t N : {1, 63, 64, 65, 95, 96, 97, 5000, 16384, 100000, 1 << 20, (1 << 20) + 17})
                 for (int64_t M : {1, 128, 300, 512, 513, 2048})
                     for (int64_t D : {16, 32, 64}) check(B, H, N, M, D);
     for (int i = 0; i < 1500; ++i)
