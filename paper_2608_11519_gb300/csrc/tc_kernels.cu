@@ -93,13 +93,19 @@ struct Cfg {
     static constexpr int kABufS = DEC ? 2 : 1;          // shared-memory A buffers
     static constexpr int kOBuf = (DEC && D <= 32) ? 2 : 1;    // O accumulators per stream
     static constexpr int kGroup = NS * kTileRows;     // resident rows per work unit
-    static constexpr int kStages = 8;                 // ring items (>= 2 B NS)
     static constexpr int kATile = kTileRows * D * 2;  // one 128-row operand tile
     static constexpr int kABytes = NS * kANum * kATile;
     static constexpr int kItemTile = kItem * D * 2;
     static constexpr int kStage = (kLoB ? 3 : 2) * kItemTile;
     static constexpr uint32_t kSwz = D == 16 ? kSw32 : (D == 32 ? kSw64 : kSw128);
     static constexpr uint32_t kSBO = 8 * D * 2;  // bytes between 8-row groups
+    // Ring items. A stream that takes every n_par-th item (an encode unit with fewer than four
+    // route tiles gives each stream one token parity) looks ahead only kStages / n_par of its
+    // own items, and the copy of its next item cannot start before the stream frees the stage
+    // kStages items back; so the encode takes as many stages as shared memory holds, up to 16.
+    // The decode's streams take every item, and 8 stages cover the copy latency.
+    static constexpr int kStagesFit = (232448 - 2048 - kABufS * kABytes) / kStage;
+    static constexpr int kStages = DEC ? 8 : (kStagesFit < 16 ? kStagesFit : 16);
     // barriers: full[S], empty[S], a_full[2] (a unit's A tiles landed), a_free[2] (one arrive
     //           per softmax warpgroup once it has seen the unit's last S: the buffer may be
     //           refilled), sync[NS][2] = {s_ready, o_done} per stream (S of an item complete;
