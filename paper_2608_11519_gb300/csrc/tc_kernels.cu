@@ -90,7 +90,9 @@ struct Cfg {
     // D = 64 the columns instead widen its items to 48 routes (S 4 x 48 + O 4 x 64).
     static constexpr int kItem = D == 64 ? (DEC ? 48 : 64) : (DEC ? 64 : 96);
     static constexpr int B = 1;                         // score buffers per stream
-    static constexpr int kABufS = DEC ? 2 : 1;          // shared-memory A buffers
+    // shared-memory A buffers (four for the decode at small M measured no faster than two)
+    static constexpr int kABufS = DEC ? 2 : 1;
+    static constexpr int kAAhead = kABufS > 1 ? kABufS - 1 : 1;  // units the A copies run ahead
     static constexpr int kOBuf = (DEC && D <= 32) ? 2 : 1;    // O accumulators per stream
     static constexpr int kGroup = NS * kTileRows;     // resident rows per work unit
     static constexpr int kATile = kTileRows * D * 2;  // one 128-row operand tile
@@ -106,16 +108,17 @@ struct Cfg {
     // The decode's streams take every item, and 8 stages cover the copy latency.
     static constexpr int kStagesFit = (232448 - 2048 - kABufS * kABytes) / kStage;
     static constexpr int kStages = DEC ? 8 : (kStagesFit < 16 ? kStagesFit : 16);
-    // barriers: full[S], empty[S], a_full[2] (a unit's A tiles landed), a_free[2] (one arrive
-    //           per softmax warpgroup once it has seen the unit's last S: the buffer may be
-    //           refilled), sync[NS][2] = {s_ready, o_done} per stream (S of an item complete;
-    //           every PV of the stream's unit complete), p_ready[NS][2] (slot 0 used). With two
-    //           O accumulators a decode unit's last PV goes out with the next unit's first S, so
-    //           o_done is committed only for a CTA's last unit. A barrier that a warp waits on
-    //           by parity never runs two phases ahead of that warp: s_ready of the next item
-    //           needs this item's P (p_ready counts every warp of the warpgroup), o_done of the
-    //           next unit needs that unit's P, a_full of unit k + 2 needs a_free of unit k.
-    static constexpr int kNumBars = 2 * kStages + 4 + 4 * NS;
+    // barriers: full[S], empty[S], a_full[kABufS] (a unit's A tiles landed), a_free[kABufS]
+    //           (one arrive per softmax warpgroup once it has seen the unit's last S: the
+    //           buffer may be refilled), sync[NS][2] = {s_ready, o_done} per stream (S of an
+    //           item complete; every PV of the stream's unit complete), p_ready[NS][2] (slot 0
+    //           used). With two O accumulators a decode unit's last PV goes out with the next
+    //           unit's first S, so o_done is committed only for a CTA's last unit. A barrier that
+    //           a warp waits on by parity never runs two phases ahead of that warp: s_ready of
+    //           the next item needs this item's P (p_ready counts every warp of the warpgroup),
+    //           o_done of the next unit needs that unit's P, a_full of unit k + kABufS needs
+    //           a_free of unit k.
+    static constexpr int kNumBars = 2 * kStages + 2 * kABufS + 4 * NS;
     static constexpr int kData = kABufS * kABytes + kStages * kStage;
     static constexpr int kNeed = 1024 + kData + kNumBars * 8 + 16;
     // at least 120 KB so that one CTA owns an SM and its 512 TMEM columns
@@ -584,8 +587,8 @@ __global__ void __launch_bounds__(kThreads, 1)
     const uint32_t full0 = smem_u32(bars);
     const uint32_t empty0 = full0 + 8u * C::kStages;
     const uint32_t afull0 = full0 + 8u * (2 * C::kStages);
-    const uint32_t afree0 = afull0 + 16u;
-    const uint32_t sready0 = afull0 + 32u;        // [NS][2]
+    const uint32_t afree0 = afull0 + 8u * C::kABufS;
+    const uint32_t sready0 = afree0 + 8u * C::kABufS;  // [NS][2]
     const uint32_t pready0 = sready0 + 16u * NS;  // [NS][2]
 
     const int warp = threadIdx.x >> 5;
@@ -596,7 +599,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             mbar_init(full0 + 8u * st, 1);
             mbar_init(empty0 + 8u * st, NS);
         }
-        for (int b = 0; b < 2; ++b) {
+        for (int b = 0; b < C::kABufS; ++b) {
             mbar_init(afull0 + 8u * b, 1);
             mbar_init(afree0 + 8u * b, NS);
         }
@@ -660,7 +663,9 @@ __global__ void __launch_bounds__(kThreads, 1)
                            prm.wait_ns))
                 break;
             const uint64_t dA = dA0 + ((uint64_t)(ab * C::kABytes + a * C::kANum * C::kATile) >> 4);
-            const uint32_t d_o = tmem + C::kColO + ((C::kOBuf == 2 ? ab : 0) * NS + s) * D;
+            // O accumulator of this unit: the unit's parity with two, else the only one (the A
+            // buffer index above runs to kABufS - 1 and must not pick it)
+            const uint32_t d_o = tmem + C::kColO + ((C::kOBuf == 2 ? (int)(ua & 1) : 0) * NS + s) * D;
             int j = 0;
             for (int i = 0; i < U.n_items; ++i, ++it) {
                 const uint32_t st = it % C::kStages;
@@ -741,10 +746,11 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
     } else if (warp < kFirstSoftmaxWarp) {
         // ------------------------------------------------------------ TMA producer
-        // Order: A(0), items(0), A(1), items(1), ... The A group of unit k goes into shared
-        // buffer k % kABufS once the group before it in that buffer has been read by the last S
-        // product of its unit, which each softmax warpgroup reports when it sees that S. Every
-        // wait blocks (try_wait), so the warp takes no issue slots while it waits.
+        // Order: A(0) .. A(kAAhead - 1), items(0), A(kAAhead), items(1), A(kAAhead + 1), ...
+        // The A group of unit k goes into shared buffer k % kABufS once the group before it in
+        // that buffer has been read by the last S product of its unit, which each softmax
+        // warpgroup reports when it sees that S. Every wait blocks (try_wait), so the warp takes
+        // no issue slots while it waits.
         regs_lower<kRegsControl>();
         if (warp == kProducerWarp) {
             const int64_t G = gridDim.x;
@@ -772,7 +778,8 @@ __global__ void __launch_bounds__(kThreads, 1)
                 ++na;
                 return true;
             };
-            if (blockIdx.x < prm.n_units) ok = issue_a(0, blockIdx.x);
+            for (uint32_t k = 0; k < (uint32_t)C::kAAhead && ok; ++k)
+                if (blockIdx.x + k * G < prm.n_units) ok = issue_a(k, blockIdx.x + k * G);
             uint32_t k = 0;
             for (int64_t u = blockIdx.x; u < prm.n_units && ok; u += G, ++k) {
                 const Unit U = get_unit<D, DEC, LO>(prm, u);
@@ -801,8 +808,8 @@ __global__ void __launch_bounds__(kThreads, 1)
                     }
                     __syncwarp();
                 }
-                const int64_t un = u + G;
-                if (ok && un < prm.n_units) ok = issue_a(k + 1, un);
+                const int64_t un = u + C::kAAhead * G;
+                if (ok && un < prm.n_units) ok = issue_a(k + C::kAAhead, un);
             }
             if (!ok) {
                 // after an abort: wait (bounded) until the newest copy into every buffer landed
