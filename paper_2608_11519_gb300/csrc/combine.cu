@@ -32,11 +32,39 @@ __device__ __forceinline__ int slots_log2(int M, int m, int sub_per_chunk, int g
 // Merge of the partial slots of one row (App. A.3):
 //   g = max_r mx_r; w_r = 2^(mx_r - g); out = sum_r w_r acc_r / sum_r w_r l_r;
 //   the row's base-2 log-normaliser is g + log2(sum_r w_r l_r).
-// T = D / 4 threads per row, each with four channels (one 16-byte load per slot); a block of
-// 256 threads covers 256 / T rows of one (b, h), which blockIdx.y + gridDim.y * blockIdx.z
-// names. The slots are taken KB at a time, all loads of a block issued together, and merged
-// online in slot order (chunk by chunk, parts in order): the same merge in every run.
-template <int D, int KB>
+// T = D / 4 channel groups per row (four channels each, one 16-byte load per slot), each taken
+// by P adjacent lanes; a block of 256 threads covers 256 / (T P) rows of one (b, h), which
+// blockIdx.y + gridDim.y * blockIdx.z names. The slots are taken KB at a time (all loads of a
+// batch issued together): lane p of a group merges batches p, p + P, p + 2P, ... online, and
+// the P partial merges are then combined by a butterfly over the group's lanes, whose result
+// lane 0 writes. The order is fixed, so every run gives the same bits. P > 1 serves rows with
+// many slots (many chunks of a group with one route tile, each in four token-parity parts),
+// which one lane would take one batch after another.
+template <int P>
+__device__ __forceinline__ void merge_lanes(float& g, float& a, float4& u) {
+    const unsigned lane = threadIdx.x & 31u;
+    const unsigned mask = ((1u << P) - 1u) << (lane & ~(unsigned)(P - 1));
+#pragma unroll
+    for (int off = 1; off < P; off <<= 1) {
+        const float g2 = __shfl_xor_sync(mask, g, off);
+        const float a2 = __shfl_xor_sync(mask, a, off);
+        const float x2 = __shfl_xor_sync(mask, u.x, off);
+        const float y2 = __shfl_xor_sync(mask, u.y, off);
+        const float z2 = __shfl_xor_sync(mask, u.z, off);
+        const float w2 = __shfl_xor_sync(mask, u.w, off);
+        const float gn = fmaxf(g, g2);
+        if (gn == -INFINITY) continue;  // both halves empty so far
+        const float s1 = fast_exp2(g - gn), s2 = fast_exp2(g2 - gn);  // 0 for an empty half
+        a = a * s1 + a2 * s2;
+        u.x = u.x * s1 + x2 * s2;
+        u.y = u.y * s1 + y2 * s2;
+        u.z = u.z * s1 + z2 * s2;
+        u.w = u.w * s1 + w2 * s2;
+        g = gn;
+    }
+}
+
+template <int D, int KB, int P>
 __global__ void __launch_bounds__(256)
     combine_kernel(const float* __restrict__ pmax, const float* __restrict__ psum,
                    const float* __restrict__ pacc, int64_t BH, int M, int nchunk,
@@ -44,12 +72,15 @@ __global__ void __launch_bounds__(256)
                    __nv_bfloat16* __restrict__ outop, __nv_bfloat16* __restrict__ outlo,
                    float op_sign, float* __restrict__ lse) {
     constexpr int T = D / 4;
-    constexpr int kRowsPerBlock = 256 / T;
+    constexpr int kRowsPerBlock = 256 / (T * P);
+    static_assert(P == 1 || P == 2 || P == 4 || P == 8, "lanes per channel group");
     tc::pdl_trigger();
     tc::pdl_wait();  // the partials and the outputs belong to the kernels around this one
     const int64_t bh = (int64_t)blockIdx.z * gridDim.y + blockIdx.y;
-    const int m = blockIdx.x * kRowsPerBlock + (int)(threadIdx.x / T);
-    const int q = (int)(threadIdx.x % T);
+    const int m = blockIdx.x * kRowsPerBlock + (int)(threadIdx.x / (T * P));
+    const int q = (int)((threadIdx.x / P) % T);
+    const int lp = (int)(threadIdx.x % P);
+    // (all P lanes of a channel group share m, so they leave or stay together)
     if (bh >= BH || m >= M) return;
     const int ul = slots_log2(M, m, sub_per_chunk, group_log2);
     const int n = nchunk << ul;  // slot s: chunk s >> ul, part s & (2^ul - 1)
@@ -59,7 +90,7 @@ __global__ void __launch_bounds__(256)
     const int mask = (1 << ul) - 1;
     float g = -INFINITY, a = 0.f;
     float4 u = make_float4(0.f, 0.f, 0.f, 0.f);
-    for (int s0 = 0; s0 < n; s0 += KB) {
+    for (int s0 = lp * KB; s0 < n; s0 += KB * P) {
         float mx[KB], ps[KB];
         float4 v[KB];
 #pragma unroll
@@ -97,6 +128,10 @@ __global__ void __launch_bounds__(256)
             u.w = fmaf(w, v[j].w, u.w);
         }
         g = gn;
+    }
+    if constexpr (P > 1) {
+        merge_lanes<P>(g, a, u);
+        if (lp != 0) return;
     }
     const float inv = a > 0.f ? 1.f / a : 0.f;
     if (lse && q == 0) lse[row] = a > 0.f ? g + log2f(a) : -INFINITY;
@@ -155,15 +190,31 @@ cudaError_t combine(const Plan& p, int call, char* ws, bool negate, cudaStream_t
     const int64_t gy = p.BH < 65535 ? p.BH : 65535;
     const int64_t gz = (p.BH + gy - 1) / gy;
     if (gz > 65535) return cudaErrorInvalidValue;
-    // slots per row at most: nchunk x sub_per_chunk
-    const bool few = p.nchunk * p.sub_per_chunk <= 4;
-#define FLAREPP_COMBINE(DD)                                                                  \
-    {                                                                                        \
-        const int64_t gx = (p.M + (256 / (DD / 4)) - 1) / (256 / (DD / 4));                 \
-        return launch_pdl(few ? combine_kernel<DD, 4> : combine_kernel<DD, 8>,               \
-                          dim3((unsigned)gx, (unsigned)gy, (unsigned)gz), dim3(256), 0, st,  \
-                          pmax, psum, pacc, p.BH, (int)p.M, (int)p.nchunk,                   \
-                          (int)p.sub_per_chunk, group_log2, out32, outop, outlo, sign, lse); \
+    // slots per row at most: nchunk, times the token-parity parts of the last (partial) route
+    // group's rows on the tensor-core path. Up to 32 slots (four batches), one lane per channel
+    // group takes them; beyond that (many chunks of a one-tile group), four lanes share a row's
+    // batches.
+    int64_t n_slots = p.nchunk;
+    if (p.sub_per_chunk > 1) {
+        const int64_t group = int64_t(1) << group_log2, rem = p.M % group;
+        const int64_t tiles = rem == 0 ? group / 128 : (rem + 127) / 128;
+        const int64_t na = tiles <= 1 ? 1 : (tiles <= 2 ? 2 : 4);
+        n_slots = p.nchunk * ((group / 128) / na);
+    }
+#define FLAREPP_COMBINE_P(DD, KB, PP)                                                         \
+    {                                                                                         \
+        constexpr int64_t rows = 256 / ((DD / 4) * PP);                                       \
+        const int64_t gx = (p.M + rows - 1) / rows;                                           \
+        return launch_pdl(combine_kernel<DD, KB, PP>,                                         \
+                          dim3((unsigned)gx, (unsigned)gy, (unsigned)gz), dim3(256), 0, st,   \
+                          pmax, psum, pacc, p.BH, (int)p.M, (int)p.nchunk,                    \
+                          (int)p.sub_per_chunk, group_log2, out32, outop, outlo, sign, lse);  \
+    }
+#define FLAREPP_COMBINE(DD)                                   \
+    {                                                         \
+        if (n_slots <= 4) FLAREPP_COMBINE_P(DD, 4, 1)         \
+        if (n_slots <= 32) FLAREPP_COMBINE_P(DD, 8, 1)        \
+        FLAREPP_COMBINE_P(DD, 8, 4)                           \
     }
     switch (p.D) {
         case 16: FLAREPP_COMBINE(16)
@@ -171,6 +222,7 @@ cudaError_t combine(const Plan& p, int call, char* ws, bool negate, cudaStream_t
         case 64: FLAREPP_COMBINE(64)
     }
 #undef FLAREPP_COMBINE
+#undef FLAREPP_COMBINE_P
     return cudaErrorInvalidValue;
 }
 
