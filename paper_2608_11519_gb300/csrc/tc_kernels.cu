@@ -82,13 +82,13 @@ struct Cfg {
     // memory where the TMA puts them, swizzled like the ring tiles, and the MMAs read them there
     // (`ss` score products); nothing copies them into TMEM, so all 512 columns go to the score
     // tiles and accumulators. The encode's units are long (hundreds of items): one A buffer,
-    // and items of 96 tokens (64 at D = 64: S 4 x 64 + O 4 x 64 columns), so the per-item round
-    // trip is paid once per 96 tokens. The decode's units are only M/64 items, so per-unit costs
+    // and items of 96 tokens (112 at D = 16; 64 at D = 64: S 4 x 64 + O 4 x 64 columns), so the
+    // per-item round trip is paid once per 96 tokens. The decode's units are only M/64 items, so per-unit costs
     // show: its A tiles are double-buffered so the next unit's land during this one, and where
     // TMEM has the room (D <= 32) it keeps two O accumulators per stream, one per unit parity,
     // so that a unit's epilogue can wait until the next unit's first item is under way; at
     // D = 64 the columns instead widen its items to 48 routes (S 4 x 48 + O 4 x 64).
-    static constexpr int kItem = D == 64 ? (DEC ? 48 : 64) : (DEC ? 64 : 96);
+    static constexpr int kItem = D == 64 ? (DEC ? 48 : 64) : (DEC ? 64 : (D == 16 ? 112 : 96));
     static constexpr int B = 1;                         // score buffers per stream
     // shared-memory A buffers (four for the decode at small M measured no faster than two)
     static constexpr int kABufS = DEC ? 2 : 1;
@@ -457,6 +457,10 @@ __device__ __forceinline__ bool softmax_step(SoftmaxStream& S, const Unit& U, ui
     } else if constexpr (C::kItem == 96) {
         tmem_st32(scol, pr);
         tmem_st16(scol + 32, pr + 32);
+    } else if constexpr (C::kItem == 112) {
+        tmem_st32(scol, pr);
+        tmem_st16(scol + 32, pr + 32);
+        tmem_st8(scol + 48, pr + 48);
     } else if constexpr (C::kItem == 64) {
         tmem_st32(scol, pr);
     } else {

@@ -19,7 +19,7 @@ HARNESS = r"""
 
 // tokens per encode item and routes per group, as the tensor-core encode defines them
 namespace flarepp {
-int64_t tc_encode_item_rows(int64_t D) { return D == 64 ? 64 : 96; }
+int64_t tc_encode_item_rows(int64_t D) { return D == 64 ? 64 : (D == 16 ? 112 : 96); }
 int64_t tc_group_rows(int64_t D) { (void)D; return 512; }
 }  // namespace flarepp
 
