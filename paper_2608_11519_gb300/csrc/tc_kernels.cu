@@ -318,7 +318,8 @@ __device__ __forceinline__ float exp_chunk(const uint32_t* sr, uint32_t* pr, int
 }
 
 // P for a whole item tile of ITEM columns at TMEM column scol (S is read 32 columns at a
-// time, and a last 16 when ITEM is 80); packed bf16 pairs go to pr[0 .. ITEM/2). Returns the
+// time, and a last 16 when ITEM is an odd multiple of 16); packed bf16 pairs go to
+// pr[0 .. ITEM/2). Returns the
 // row sum. With FIRST_REF and
 // `first` the reference m is first set to the row's own first score, c S[0]: any score of
 // the row is a valid reference (that score alone contributes 2^0 = 1 to the sum, so the
@@ -350,6 +351,19 @@ __device__ __forceinline__ float exp_tile(uint32_t scol, uint32_t* pr, int nv, f
         if constexpr (STORE) tmem_st8(scol + base / 2, pr + base / 2);
     }
     return sum;
+}
+
+// P of a whole item (ITEM / 2 packed words) to TMEM column scol, 32, 16 and 8 words at a time.
+template <int ITEM>
+__device__ __forceinline__ void store_p(uint32_t scol, uint32_t* pr) {
+    constexpr int W = ITEM / 2;
+    static_assert(W % 8 == 0, "P comes in multiples of 8 words");
+#pragma unroll
+    for (int w = 0; w + 32 <= W; w += 32) tmem_st32(scol + w, pr + w);
+    constexpr int w16 = W / 32 * 32;
+    if constexpr (W - w16 >= 16) tmem_st16(scol + w16, pr + w16);
+    constexpr int w8 = w16 + (W - w16 >= 16 ? 16 : 0);
+    if constexpr (W - w8 >= 8) tmem_st8(scol + w8, pr + w8);
 }
 
 // One item of this warpgroup's stream for this thread's row: read S, update the online
@@ -448,24 +462,7 @@ __device__ __forceinline__ bool softmax_step(SoftmaxStream& S, const Unit& U, ui
         sum = exp_tile<C::kItem, false, false>(scol, pr, nv, c, c2, S.m, false);
     }
     S.l += sum;
-    if constexpr (C::kItem == 80) {
-        tmem_st32(scol, pr);
-        tmem_st8(scol + 32, pr + 32);
-    } else if constexpr (C::kItem == 48) {
-        tmem_st16(scol, pr);
-        tmem_st8(scol + 16, pr + 16);
-    } else if constexpr (C::kItem == 96) {
-        tmem_st32(scol, pr);
-        tmem_st16(scol + 32, pr + 32);
-    } else if constexpr (C::kItem == 112) {
-        tmem_st32(scol, pr);
-        tmem_st16(scol + 32, pr + 32);
-        tmem_st8(scol + 48, pr + 48);
-    } else if constexpr (C::kItem == 64) {
-        tmem_st32(scol, pr);
-    } else {
-        tmem_st16(scol, pr);
-    }
+    store_p<C::kItem>(scol, pr);
     tmem_wait_st();
     tc_fence_before();
     mbar_arrive(pready_s + 8u * b);
@@ -864,10 +861,9 @@ __global__ void __launch_bounds__(kThreads, 1)
             st.ab = (int)(ua % C::kABufS);
             while (alive && st.j < st.cnt) {
                 alive = softmax_step<D, DEC, SAFE, LO>(st, U, tmem, lane_off, c, c2, sready_s,
-                                                   pready0 + 16u * st.s, empty0, afree0, wg_leader,
-                                                   it0,
-                                                   abort_flag, prm.status, prm.wait_ns,
-                                                   prm.overflow);
+                                                   pready0 + 16u * st.s, empty0, afree0,
+                                                   wg_leader, it0, abort_flag, prm.status,
+                                                   prm.wait_ns, prm.overflow);
                 if (owed && alive) {
                     alive = finish_stream<D, DEC, LO>(st, prev,
                                                       get_unit<D, DEC, LO>(prm, u - gridDim.x),
