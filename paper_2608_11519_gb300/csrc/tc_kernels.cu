@@ -70,8 +70,9 @@ constexpr float kFastLimit = 281474976710656.0f;  // 2^48
 // LO (the training forward, D <= 32): Q enters the scores of calls 2 and 3 as a pair of bf16
 // operands, hi = bf16(Q) and lo = bf16(Q - hi), and each score product is the sum of the two
 // products (S = (hi + lo) B^T in the encode of call 2, S = A (hi + lo)^T in the decode), so the
-// scores see Q to about 2^-17 instead of bf16's 2^-9. The encode keeps both A tiles in TMEM;
-// the decode's items carry Q's lo tile as a third tile.
+// scores see Q to about 2^-17 instead of bf16's 2^-9. The encode keeps both A tiles in its
+// shared-memory A buffer (the lo tile after the hi tile); the decode's items carry Q's lo tile
+// as a third tile.
 template <int D, bool DEC, bool LO = false>
 struct Cfg {
     static_assert(!LO || D <= 32, "the hi/lo form of Q serves D = 16 and 32");
@@ -82,12 +83,13 @@ struct Cfg {
     // memory where the TMA puts them, swizzled like the ring tiles, and the MMAs read them there
     // (`ss` score products); nothing copies them into TMEM, so all 512 columns go to the score
     // tiles and accumulators. The encode's units are long (hundreds of items): one A buffer,
-    // and items of 96 tokens (112 at D = 16; 64 at D = 64: S 4 x 64 + O 4 x 64 columns), so the
-    // per-item round trip is paid once per 96 tokens. The decode's units are only M/64 items, so per-unit costs
-    // show: its A tiles are double-buffered so the next unit's land during this one, and where
-    // TMEM has the room (D <= 32) it keeps two O accumulators per stream, one per unit parity,
-    // so that a unit's epilogue can wait until the next unit's first item is under way; at
-    // D = 64 the columns instead widen its items to 48 routes (S 4 x 48 + O 4 x 64).
+    // and items of 96 tokens (112 at D = 16; 64 at D = 64: S 4 x 64 + O 4 x 64 columns), so
+    // the per-item round trip is paid once per 96 tokens. The decode's units are only M/64
+    // items, so per-unit costs show: its A tiles are double-buffered so the next unit's land
+    // during this one, and where TMEM has the room (D <= 32) it keeps two O accumulators per
+    // stream, one per unit parity, so that a unit's epilogue can wait until the next unit's
+    // first item is under way; at D = 64 the columns instead widen its items to 48 routes
+    // (S 4 x 48 + O 4 x 64).
     static constexpr int kItem = D == 64 ? (DEC ? 48 : 64) : (DEC ? 64 : (D == 16 ? 112 : 96));
     static constexpr int B = 1;                         // score buffers per stream
     // shared-memory A buffers (four for the decode at small M measured no faster than two)
@@ -250,7 +252,7 @@ struct SoftmaxStream {
     int ab;         // shared-memory A buffer of this unit
     float m, l;     // reference max (base 2, scaled) and running sum
     uint32_t ph0;   // s_ready phases completed in earlier units (one per item)
-    uint32_t od;    // o_done phases completed in earlier units (one per unit with items)
+    uint32_t od;    // o_done phases consumed (one per unit whose end waits on it)
     bool over;      // fast kernel: some item's sum passed kFastLimit
     __device__ __forceinline__ void begin(const Unit& U) {
         par = s / U.n_a;
@@ -369,7 +371,8 @@ __device__ __forceinline__ void store_p(uint32_t scol, uint32_t* pr) {
 // One item of this warpgroup's stream for this thread's row: read S, update the online
 // softmax, write P back over S, signal the stream's MMA warp. S of item j being ready
 // means the PV of item j - B has completed, so the warpgroup leader frees that item's ring
-// stage. Returns false when the kernel is aborting.
+// stage; the S of the unit's last item was the last product to read the unit's A tiles, so
+// the leader then also frees the A buffer. Returns false when the kernel is aborting.
 //   fast kernel (!SAFE): the reference is kept from the items before (a unit's first item
 //     takes its first score) and P is stored chunk by chunk, so S is gone by the end of the
 //     item. A sum past kFastLimit (a score far above the reference) cannot be repaired
@@ -580,7 +583,8 @@ __global__ void __launch_bounds__(kThreads, 1)
     uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                                ~static_cast<uintptr_t>(1023));
     uint8_t* abuf = smem;                         // kABufS x NS x kANum A tiles
-    uint8_t* ring = smem + C::kABufS * C::kABytes;  // kStages x (B tile, C tile[, lo tile]), swizzled
+    // kStages x (B tile, C tile[, lo tile]), swizzled like the A tiles
+    uint8_t* ring = smem + C::kABufS * C::kABytes;
     uint64_t* bars = reinterpret_cast<uint64_t*>(ring + C::kStages * C::kStage);
     uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + C::kNumBars);
     volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
@@ -666,7 +670,8 @@ __global__ void __launch_bounds__(kThreads, 1)
             const uint64_t dA = dA0 + ((uint64_t)(ab * C::kABytes + a * C::kANum * C::kATile) >> 4);
             // O accumulator of this unit: the unit's parity with two, else the only one (the A
             // buffer index above runs to kABufS - 1 and must not pick it)
-            const uint32_t d_o = tmem + C::kColO + ((C::kOBuf == 2 ? (int)(ua & 1) : 0) * NS + s) * D;
+            const int ob = C::kOBuf == 2 ? (int)(ua & 1) : 0;
+            const uint32_t d_o = tmem + C::kColO + (ob * NS + s) * D;
             int j = 0;
             for (int i = 0; i < U.n_items; ++i, ++it) {
                 const uint32_t st = it % C::kStages;
