@@ -191,8 +191,12 @@ def test_constant_values_give_constant_output():
     assert float((Y.float() - x["V"].float()).abs().max()) <= 2e-2
 
 
-def test_deterministic_bitwise():
-    w = inputs.get("pde2d").with_(B=2, N=9000)
+@pytest.mark.parametrize("shape", [
+    dict(B=2, N=9000),                  # pde2d's routes: one route tile, four token parities
+    dict(B=1, H=8, N=65536, M=16),      # 19 chunks x 4 parities: the merge splits slots over lanes
+])
+def test_deterministic_bitwise(shape):
+    w = inputs.get("pde2d").with_(**shape)
     x = inputs.make_inputs(w, seed=4, device="cuda")
     a = flarepp.route_fwd(x["seeds"], x["Kt"], x["Vt"], x["K"], x["V"])
     b = flarepp.route_fwd(x["seeds"], x["Kt"], x["Vt"], x["K"], x["V"])
