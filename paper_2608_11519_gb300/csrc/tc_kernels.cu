@@ -400,8 +400,17 @@ __device__ __forceinline__ bool softmax_step(SoftmaxStream& S, const Unit& U, ui
         const int i_old = par + (j - C::B) * U.n_par;
         mbar_arrive(empty0 + 8u * ((it0 + i_old) % C::kStages));
     }
-    // the unit's last S is complete, so its MMAs no longer read the A buffer
-    if (wg_leader && j == S.cnt - 1) mbar_arrive(afree0 + 8u * S.ab);
+    // the unit's last S is complete, so its MMAs no longer read the A buffer. Stream 0 (which
+    // always has items) also arrives for the streams with no item in the unit (short encode
+    // chunks split by token parity), which do not arrive themselves: arriving at once, such a
+    // stream could arrive for the next unit as well before a slower stream arrived for this
+    // one, completing this unit's phase of a_free while that stream's last S still reads.
+    if (wg_leader && j == S.cnt - 1) {
+        uint32_t n = 1;
+        if constexpr (!DEC)
+            if (S.s == 0 && U.n_items < U.n_par) n += U.n_a * (U.n_par - U.n_items);
+        mbar_arrive_n(afree0 + 8u * S.ab, n);
+    }
     const int item = par + j * U.n_par;
     const int64_t start = U.item0 + (int64_t)item * C::kItem;
     const int nv = (int)min((int64_t)C::kItem, U.item_end - start);
@@ -526,8 +535,6 @@ __device__ __forceinline__ bool finish_stream(SoftmaxStream& S, const UnitEnd& E
 #pragma unroll
         for (int d = 0; d < D; ++d) o[d] = __uint_as_float(t[d]);
     } else {
-        // (no MMA of this stream read the unit's A tile)
-        if (wg_leader) mbar_arrive(afree0 + 8u * E.ab);
 #pragma unroll
         for (int d = 0; d < D; ++d) o[d] = 0.f;
     }
